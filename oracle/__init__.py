@@ -1,0 +1,280 @@
+"""InertiaKV oracle -- plain, slow, fp64 CPU restatement of the decode-step eviction loop.
+
+TEST INFRASTRUCTURE ONLY.  Only the test suite, ``__graft_entry__.smoke()`` and
+the CPU-baseline / reference legs of ``bench.py`` may import this package.  The
+CUDA library never imports, links or calls it, and it shares no code with it.
+
+What it computes, in the paper's order and notation (arxiv 2609.03515):
+
+* Sec. 3, problem statement: a decode-side budget ``B`` per sequence; eviction
+  is irreversible; whenever the cache exceeds ``B`` the tokens with the lowest
+  utility ``m_t(i)`` are evicted.
+* Eq. 1: per-step score ``s_t(i) = (1/H) sum_h a_t^(h)(i)``, where ``a_t^(h)`` is
+  the last query's softmax attention of head ``h`` over the cached tokens.
+* Eq. 4 + Appendix "Layer scoring": the EMA state is updated after every
+  eligible layer, ``m_{t,l} = alpha m_{t,l-1} + (1-alpha) s_{t,l}``, with
+  ``m_{t,0} = m_{t-1,K}``.
+* Appendix "Momentum initialization": ``m_0 = 0``; no EMA during prefill.
+* Eq. 6 (Lazy refresh): refresh steps ``R_r = {t >= 1 : (t-1) mod r = 0}``;
+  off-refresh the state is carried unchanged and no attention score is taken.
+* Score-Free box (Sec. 3.2): score at step 1 only, then freeze; eviction
+  continues with the frozen ranking.
+* Appendix "New token insertion during non-refresh steps": the new token's
+  state is the mean of the existing tokens' state; it may be evicted at once.
+* Appendix "Eviction on non-refresh steps": the stale state still drives
+  eviction, so the budget always holds.
+
+Readings taken where the paper is silent (each also stated where it is used):
+
+* R1 (granularity): one state row per sequence, shared by every layer and KV
+  head (``GRAN_SEQ``, Eq. 1 with ``m_t in R^{L_t}``).  ``GRAN_KVHEAD`` keeps one
+  row per (sequence, KV head) whose score is the mean over that head's query
+  group (Appendix "Per-step scoring", GQA sentence); its kept set applies to
+  that KV head in every layer.
+* R2 (eviction time): eviction happens once per step, after all layers, with
+  the step's final state ``m_{t,K}``; the same kept set applies to every layer.
+* R3 (new token on refresh steps): state 0 (as ``m_0 = 0``), then scored in
+  the same step.  The mean rule applies on non-refresh steps only.
+* R4 (ties): among equal utilities the lower cache slot is kept; ``-0.0``
+  equals ``+0.0``; NaN ranks below every number.
+* R5 (order): survivors keep their relative order (stable compaction); the
+  appended token is last before eviction.
+* R6 (self-attention): the appended token is part of its own step's softmax.
+* R7 (scale): softmax scale ``1/sqrt(d)``; keys are used as stored.
+* R8 (eligible layers): all layers unless a layer mask says otherwise.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from typing import List, Optional, Sequence
+
+import numpy as np
+
+GRAN_SEQ = 0
+GRAN_KVHEAD = 1
+
+
+# --------------------------------------------------------------------------
+# Attention and the per-step score (Eq. 1)
+# --------------------------------------------------------------------------
+def softmax(z: np.ndarray) -> np.ndarray:
+    """Row softmax with the usual max shift (Vaswani et al., as cited for Eq. 1)."""
+    z = np.asarray(z, dtype=np.float64)
+    zmax = np.max(z, axis=-1, keepdims=True)
+    e = np.exp(z - zmax)
+    return e / np.sum(e, axis=-1, keepdims=True)
+
+
+def last_query_attention(q: np.ndarray, K: Sequence[np.ndarray], V: Sequence[np.ndarray]):
+    """Attention of one layer's last query over its cached tokens (Eq. 1's ``a_t^(h)``).
+
+    q: [H, d] (the new token's query per head); K[g], V[g]: [L, d] per KV head.
+    Query head h reads KV head ``h // (H / H_kv)`` (grouped-query attention).
+    Returns (a [H, L] softmax probabilities, out [H, d] attention output).
+    """
+    q = np.asarray(q, dtype=np.float64)
+    H, d = q.shape
+    n_kv = len(K)
+    group = H // n_kv
+    L = K[0].shape[0]
+    a = np.empty((H, L))
+    out = np.empty((H, d))
+    for h in range(H):
+        g = h // group
+        z = (np.asarray(K[g], np.float64) @ q[h]) / np.sqrt(d)
+        a[h] = softmax(z)
+        out[h] = a[h] @ np.asarray(V[g], np.float64)
+    return a, out
+
+
+def pooled_score(a: np.ndarray, granularity: int, kv_heads: int) -> np.ndarray:
+    """Eq. 1: mean of the heads' probabilities per cached token.
+
+    GRAN_SEQ -> [1, L], mean over all H heads.
+    GRAN_KVHEAD -> [H_kv, L], mean over each KV head's query group (reading R1).
+    """
+    H, L = a.shape
+    if granularity == GRAN_SEQ:
+        return a.mean(axis=0, keepdims=True)
+    return a.reshape(kv_heads, H // kv_heads, L).mean(axis=1)
+
+
+# --------------------------------------------------------------------------
+# Aggregation (Eq. 4, Appendix "Layer scoring")
+# --------------------------------------------------------------------------
+def ema_update(m: np.ndarray, s: np.ndarray, alpha: float) -> np.ndarray:
+    """Eq. 4: m <- alpha m + (1 - alpha) s."""
+    return alpha * m + (1.0 - alpha) * s
+
+
+def layer_sequential_ema(m_prev: np.ndarray, layer_scores: Sequence[np.ndarray], alpha: float) -> np.ndarray:
+    """Appendix "Layer scoring": m_{t,0} = m_{t-1,K}; m_{t,l} = alpha m_{t,l-1} + (1-alpha) s_{t,l}."""
+    m = np.array(m_prev, dtype=np.float64, copy=True)
+    for s in layer_scores:
+        m = ema_update(m, s, alpha)
+    return m
+
+
+# --------------------------------------------------------------------------
+# Schedule (Eq. 6, Score-Free box)
+# --------------------------------------------------------------------------
+def is_refresh(t: int, refresh_period: int, score_free: bool) -> bool:
+    """Eq. 6: t in R_r iff (t-1) mod r == 0 (t is 1-based).  Score-Free: t == 1 only."""
+    if score_free:
+        return t == 1
+    return (t - 1) % refresh_period == 0
+
+
+def new_token_state(m_row: np.ndarray, refresh: bool, refresh_init: str = "zero") -> float:
+    """Utility given to the appended token.
+
+    Non-refresh step: mean of the existing L_t - 1 tokens' state (Appendix "New
+    token insertion", also the Score-Free box).  Refresh step: 0 (reading R3).
+    """
+    if refresh and refresh_init == "zero":
+        return 0.0
+    if m_row.size == 0:
+        return 0.0
+    return float(np.mean(m_row))
+
+
+# --------------------------------------------------------------------------
+# Budgeted selection (Sec. 3: evict the lowest m while the cache exceeds B)
+# --------------------------------------------------------------------------
+def select_keep(m_row: np.ndarray, budget: int) -> np.ndarray:
+    """Kept slots, ascending: the ``budget`` highest utilities (ties: lower slot, R4).
+
+    A full sort by (NaN last, m descending, slot ascending); no partial selection.
+    """
+    m_row = np.asarray(m_row, dtype=np.float64)
+    L = m_row.shape[0]
+    if L <= budget:
+        return np.arange(L)
+    nan = np.isnan(m_row)
+    key = np.where(nan, -np.inf, m_row)
+    order = np.lexsort((np.arange(L), -key, nan))
+    return np.sort(order[:budget])
+
+
+# --------------------------------------------------------------------------
+# Cache state and one decode step
+# --------------------------------------------------------------------------
+@dataclass
+class Params:
+    alpha: float = 0.8                 # Sec. 3.1 default 0.8
+    refresh_period: int = 1            # r of Eq. 6; 1 = full refresh
+    score_free: bool = False
+    granularity: int = GRAN_SEQ
+    layer_mask: Optional[List[bool]] = None   # eligible layers (R8)
+    refresh_init: str = "zero"         # R3
+
+
+@dataclass
+class SeqState:
+    """One sequence's cache: K[l][g], V[l][g] are [L, d]; m, pos are [R, L]."""
+
+    K: List[List[np.ndarray]]
+    V: List[List[np.ndarray]]
+    m: np.ndarray
+    pos: np.ndarray
+    budget: int
+    next_pos: int
+    granularity: int = GRAN_SEQ
+
+    @property
+    def length(self) -> int:
+        return self.m.shape[1]
+
+    @property
+    def layers(self) -> int:
+        return len(self.K)
+
+    @property
+    def kv_heads(self) -> int:
+        return len(self.K[0])
+
+    def row_of(self, g: int) -> int:
+        return 0 if self.granularity == GRAN_SEQ else g
+
+
+def prefill_state(K: Sequence[Sequence[np.ndarray]], V: Sequence[Sequence[np.ndarray]], budget: int,
+                  granularity: int = GRAN_SEQ) -> SeqState:
+    """State after prefill: full cache, m_0 = 0 (Appendix "Momentum initialization")."""
+    layers, kv = len(K), len(K[0])
+    L0 = K[0][0].shape[0]
+    R = 1 if granularity == GRAN_SEQ else kv
+    return SeqState(
+        K=[[np.array(K[l][g], np.float64) for g in range(kv)] for l in range(layers)],
+        V=[[np.array(V[l][g], np.float64) for g in range(kv)] for l in range(layers)],
+        m=np.zeros((R, L0)), pos=np.tile(np.arange(L0, dtype=np.int64), (R, 1)),
+        budget=budget, next_pos=L0, granularity=granularity)
+
+
+def append_token(st: SeqState, k_new: np.ndarray, v_new: np.ndarray, refresh: bool, p: Params) -> None:
+    """Append the new token's K/V rows ([layers][kv_heads][d]) at the end of the cache."""
+    R = st.m.shape[0]
+    init = np.array([new_token_state(st.m[r], refresh, p.refresh_init) for r in range(R)])
+    for l in range(st.layers):
+        for g in range(st.kv_heads):
+            st.K[l][g] = np.vstack([st.K[l][g], np.asarray(k_new[l][g], np.float64)[None]])
+            st.V[l][g] = np.vstack([st.V[l][g], np.asarray(v_new[l][g], np.float64)[None]])
+    st.m = np.concatenate([st.m, init[:, None]], axis=1)
+    st.pos = np.concatenate([st.pos, np.full((R, 1), st.next_pos, np.int64)], axis=1)
+    st.next_pos += 1
+
+
+def attend_and_score(st: SeqState, q_t: np.ndarray, refresh: bool, p: Params) -> np.ndarray:
+    """All layers' attention outputs [layers][H][d]; on refresh steps, the
+    layer-sequential EMA of Eq. 1 scores over the eligible layers (Appendix "Layer scoring")."""
+    outs = []
+    for l in range(st.layers):
+        if st.granularity == GRAN_SEQ:
+            a, o = last_query_attention(q_t[l], st.K[l], st.V[l])
+        else:
+            # each KV head holds its own kept set; query group of head g reads it
+            H = q_t[l].shape[0]
+            group = H // st.kv_heads
+            a_parts, o_parts = [], []
+            for g in range(st.kv_heads):
+                ag, og = last_query_attention(q_t[l][g * group:(g + 1) * group], [st.K[l][g]], [st.V[l][g]])
+                a_parts.append(ag)
+                o_parts.append(og)
+            a, o = np.vstack(a_parts), np.vstack(o_parts)
+        outs.append(o)
+        eligible = p.layer_mask is None or p.layer_mask[l]
+        if refresh and eligible:
+            s = pooled_score(a, st.granularity, st.kv_heads)
+            st.m = ema_update(st.m, s, p.alpha)
+    return np.stack(outs)
+
+
+def evict(st: SeqState, keep_override: Optional[Sequence[np.ndarray]] = None) -> List[np.ndarray]:
+    """Evict down to the budget (Sec. 3), stable compaction (R5).  Returns kept slots per row."""
+    R = st.m.shape[0]
+    keeps = []
+    for r in range(R):
+        keep = select_keep(st.m[r], st.budget) if keep_override is None else np.asarray(keep_override[r])
+        keeps.append(np.asarray(keep, np.int64))
+    if st.length <= st.budget and keep_override is None:
+        return keeps
+    new_m = np.stack([st.m[r][keeps[r]] for r in range(R)])
+    new_pos = np.stack([st.pos[r][keeps[r]] for r in range(R)])
+    for l in range(st.layers):
+        for g in range(st.kv_heads):
+            kr = keeps[st.row_of(g)]
+            st.K[l][g] = st.K[l][g][kr]
+            st.V[l][g] = st.V[l][g][kr]
+    st.m, st.pos = new_m, new_pos
+    return keeps
+
+
+def decode_step(st: SeqState, t: int, q_t: np.ndarray, k_new: np.ndarray, v_new: np.ndarray, p: Params) -> np.ndarray:
+    """One decode step t (1-based) for one sequence; returns the attention outputs [layers][H][d].
+
+    q_t: [layers][H][d]; k_new, v_new: [layers][H_kv][d].
+    """
+    refresh = is_refresh(t, p.refresh_period, p.score_free)
+    append_token(st, k_new, v_new, refresh, p)
+    out = attend_and_score(st, q_t, refresh, p)
+    evict(st)
+    return out

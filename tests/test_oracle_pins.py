@@ -1,0 +1,429 @@
+"""Pins the CPU oracle to what the paper and the mathematics fix (no GPU needed).
+
+Each test checks the oracle against something other than itself: a closed form
+the paper states, a textbook routine, brute force on tiny inputs, or an
+invariant of the method.  A plausible slip in the oracle (dropped term, wrong
+sign, wrong index, transposed operand, wrong layer order, wrong schedule)
+fails at least one of them.
+"""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _load(name):
+    with open(os.path.join(GOLD, name)) as f:
+        return json.load(f)
+
+
+def _num(x):
+    return float(x) if not isinstance(x, str) else float(x.replace("inf", "inf"))
+
+
+def _rand_state(rng, layers=3, kv=2, L0=40, d=8, budget=12, gran=O.GRAN_SEQ, heavy=True):
+    K = [[rng.standard_normal((L0, d)) for _ in range(kv)] for _ in range(layers)]
+    V = [[rng.standard_normal((L0, d)) for _ in range(kv)] for _ in range(layers)]
+    if heavy:  # a few strongly attended tokens so rankings are not pure noise
+        for l in range(layers):
+            for g in range(kv):
+                K[l][g][::7] *= 3.0
+    return O.prefill_state(K, V, budget, gran)
+
+
+def _rand_inputs(rng, T, layers=3, H=4, kv=2, d=8):
+    q = rng.standard_normal((T, layers, H, d))
+    kn = rng.standard_normal((T, layers, kv, d))
+    vn = rng.standard_normal((T, layers, kv, d))
+    return q, kn, vn
+
+
+def _clone(st):
+    return O.SeqState(K=[[k.copy() for k in row] for row in st.K], V=[[v.copy() for v in row] for row in st.V],
+                      m=st.m.copy(), pos=st.pos.copy(), budget=st.budget, next_pos=st.next_pos,
+                      granularity=st.granularity)
+
+
+# ---------------------------------------------------------------- attention
+def test_softmax_rows_sum_to_one():
+    rng = np.random.default_rng(0)
+    z = rng.standard_normal((50, 300)) * 30
+    a = O.softmax(z)
+    assert np.all(a >= 0)
+    assert np.max(np.abs(a.sum(-1) - 1.0)) < 1e-12
+
+
+def test_attention_golden_two_tokens():
+    g = _load("attention_two_tokens.json")
+    a, out = O.last_query_attention(np.array(g["q"]), [np.array(k) for k in g["K"]], [np.array(v) for v in g["V"]])
+    assert np.allclose(a, g["a"], atol=1e-15, rtol=0)
+    assert np.allclose(out, g["out"], atol=1e-14, rtol=0)
+
+
+def test_attention_matches_library_sdpa_gqa():
+    """GQA last-query attention equals torch's fp64 scaled_dot_product_attention
+    with the KV heads repeated over their query groups (textbook special case)."""
+    rng = np.random.default_rng(1)
+    H, kv, L, d = 8, 2, 37, 16
+    q = rng.standard_normal((H, d))
+    K = [rng.standard_normal((L, d)) for _ in range(kv)]
+    V = [rng.standard_normal((L, d)) for _ in range(kv)]
+    _, out = O.last_query_attention(q, K, V)
+    Kt = torch.tensor(np.stack(K)).repeat_interleave(H // kv, 0)[None]
+    Vt = torch.tensor(np.stack(V)).repeat_interleave(H // kv, 0)[None]
+    ref = torch.nn.functional.scaled_dot_product_attention(torch.tensor(q)[None, :, None], Kt, Vt)[0, :, 0]
+    assert np.max(np.abs(out - ref.numpy())) < 1e-12
+
+
+def test_attention_bruteforce_loops():
+    rng = np.random.default_rng(2)
+    H, kv, L, d = 4, 2, 5, 3
+    q = rng.standard_normal((H, d))
+    K = [rng.standard_normal((L, d)) for _ in range(kv)]
+    V = [rng.standard_normal((L, d)) for _ in range(kv)]
+    a, out = O.last_query_attention(q, K, V)
+    for h in range(H):
+        g = h // 2
+        z = [sum(q[h][e] * K[g][i][e] for e in range(d)) / math.sqrt(d) for i in range(L)]
+        den = sum(math.exp(x) for x in z)
+        for i in range(L):
+            assert abs(a[h][i] - math.exp(z[i]) / den) < 1e-14
+        for e in range(d):
+            assert abs(out[h][e] - sum(math.exp(z[i]) / den * V[g][i][e] for i in range(L))) < 1e-13
+
+
+def test_pooled_score_granularities_bruteforce():
+    rng = np.random.default_rng(3)
+    a = rng.random((6, 9))
+    s_seq = O.pooled_score(a, O.GRAN_SEQ, 3)
+    s_kv = O.pooled_score(a, O.GRAN_KVHEAD, 3)
+    assert s_seq.shape == (1, 9) and s_kv.shape == (3, 9)
+    for i in range(9):
+        assert abs(s_seq[0, i] - sum(a[h, i] for h in range(6)) / 6) < 1e-15
+        for g in range(3):
+            assert abs(s_kv[g, i] - (a[2 * g, i] + a[2 * g + 1, i]) / 2) < 1e-15
+
+
+# ---------------------------------------------------------------- EMA
+def test_layer_weights_golden():
+    """Appendix 'Layer scoring': prior weight alpha^K, layer l weight (1-alpha) alpha^(K-l)."""
+    for c in _load("layer_weights.json")["cases"]:
+        K, alpha = c["K"], c["alpha"]
+        # one-hot probes recover each weight from the recurrence
+        prior = O.layer_sequential_ema(np.array([1.0]), [np.array([0.0])] * K, alpha)[0]
+        assert abs(prior - c["prior"]) < 1e-12
+        for l in range(K):
+            s = [np.array([1.0 if j == l else 0.0]) for j in range(K)]
+            w = O.layer_sequential_ema(np.array([0.0]), s, alpha)[0]
+            assert abs(w - c["layer"][l]) < 1e-12
+        assert abs(c["prior"] + sum(c["layer"]) - 1.0) < 1e-12
+
+
+def test_layer_sequential_matches_closed_form_weights():
+    rng = np.random.default_rng(4)
+    K, alpha = 7, 0.73
+    m0 = rng.random(11)
+    S = [rng.random(11) for _ in range(K)]
+    got = O.layer_sequential_ema(m0, S, alpha)
+    want = alpha ** K * m0 + sum((1 - alpha) * alpha ** (K - 1 - l) * S[l] for l in range(K))
+    assert np.max(np.abs(got - want)) < 1e-14
+
+
+def test_momentum_dominance_golden():
+    g = _load("momentum_dominance.json")
+    rng = np.random.default_rng(5)
+    s = rng.random(64)
+    delta = rng.standard_normal(64)
+    delta *= g["rel_perturbation"] * np.linalg.norm(s) / np.linalg.norm(delta)
+    m = rng.random(64)
+    rel = np.linalg.norm(O.ema_update(m, s + delta, g["alpha"]) - O.ema_update(m, s, g["alpha"])) / np.linalg.norm(s)
+    assert abs(rel - g["expected_rel_change"]) < 1e-12
+    assert round(100 * rel) == g["paper_rounded_percent"]
+
+
+def test_prop1a_expectation_closed_form():
+    """Prop. 1(a) proof: E[mu_T] = (1 - alpha^T) s_bar from mu_0 = 0."""
+    rng = np.random.default_rng(6)
+    alpha, T, n = 0.8, 12, 400000
+    s = rng.random((T, n))  # iid U[0,1], mean 1/2
+    mu = np.zeros(n)
+    for t in range(T):
+        mu = O.ema_update(mu, s[t], alpha)
+    want = (1 - alpha ** T) * 0.5
+    se = np.std(mu) / np.sqrt(n)
+    assert abs(mu.mean() - want) < 5 * se
+
+
+def test_prop1b_variance_bound_monte_carlo():
+    """Prop. 1(b): Var[mu_T(i) - mu_T(j)] <= 2(1-alpha)/(1+alpha) sigma^2, and for iid
+    scores the finite-T value is that bound times (1 - alpha^(2T))."""
+    rng = np.random.default_rng(7)
+    for alpha in (0.5, 0.8, 0.95):
+        T, n = 60, 200000
+        sigma2 = 1.0 / 12.0
+        mi = np.zeros(n)
+        mj = np.zeros(n)
+        for _ in range(T):
+            mi = O.ema_update(mi, rng.random(n) + 0.1, alpha)
+            mj = O.ema_update(mj, rng.random(n), alpha)
+        var = np.var(mi - mj)
+        bound = 2 * (1 - alpha) / (1 + alpha) * sigma2
+        exact = bound * (1 - alpha ** (2 * T))
+        assert abs(var - exact) / exact < 0.02
+        assert var <= bound * 1.02
+
+
+def test_ema_constant_stream_through_decode_loop():
+    """Uniform attention (all-zero keys) gives a constant score s = 1/L at every layer and
+    step; with B = L0 the prefill tokens survive and end at m = (1 - alpha^(K T)) / L
+    (geometric series, Prop. 1 proof with mu_0 = 0)."""
+    layers, kv, H, d, L0, T, alpha = 3, 2, 4, 8, 20, 5, 0.7
+    K = [[np.zeros((L0, d)) for _ in range(kv)] for _ in range(layers)]
+    V = [[np.ones((L0, d)) for _ in range(kv)] for _ in range(layers)]
+    st = O.prefill_state(K, V, budget=L0)
+    p = O.Params(alpha=alpha)
+    rng = np.random.default_rng(8)
+    for t in range(1, T + 1):
+        q = rng.standard_normal((layers, H, d))
+        out = O.decode_step(st, t, q, np.zeros((layers, kv, d)), np.ones((layers, kv, d)), p)
+        assert np.allclose(out, 1.0, atol=1e-14)
+        assert st.length == L0
+    assert np.array_equal(st.pos[0], np.arange(L0))
+    want = (1 - alpha ** (layers * T)) / (L0 + 1)
+    assert np.max(np.abs(st.m[0] - want)) < 1e-15
+
+
+def _spike_layers(layers, kv, H, d, L0, spikes, z_spike):
+    """Keys zero except one token per layer (spikes[l]) aligned with the query,
+    giving that token logit z_spike and every other token logit 0."""
+    K = [[np.zeros((L0, d)) for _ in range(kv)] for _ in range(layers)]
+    for l in range(layers):
+        for g in range(kv):
+            K[l][g][spikes[l], 0] = z_spike * math.sqrt(d)
+    V = [[np.zeros((L0, d)) for _ in range(kv)] for _ in range(layers)]
+    q = np.zeros((layers, H, d))
+    q[:, :, 0] = 1.0
+    return K, V, q
+
+
+def test_layer_order_through_decode_step():
+    """One refresh step where each layer spikes on a different token: the resulting
+    state must carry the paper's layer weights in layer order."""
+    layers, kv, H, d, L0, alpha, zs = 4, 2, 4, 4, 10, 0.6, 2.0
+    spikes = [1, 4, 6, 8]
+    K, V, q = _spike_layers(layers, kv, H, d, L0, spikes, zs)
+    st = O.prefill_state(K, V, budget=L0 + 1)
+    O.decode_step(st, 1, q, np.zeros((layers, kv, d)), np.zeros((layers, kv, d)), O.Params(alpha=alpha))
+    L = L0 + 1
+    den = math.exp(zs) + L - 1
+    for i in range(L):
+        want = 0.0
+        for l in range(layers):
+            s = math.exp(zs) / den if i == spikes[l] else 1.0 / den
+            want += (1 - alpha) * alpha ** (layers - 1 - l) * s
+        assert abs(st.m[0, i] - want) < 1e-15
+
+
+def test_alpha_zero_keeps_only_last_eligible_layer():
+    """Sec. 5.1: alpha = 0 retains only the last processed layer."""
+    layers, kv, H, d, L0, zs = 3, 1, 2, 4, 8, 1.5
+    spikes = [0, 3, 5]
+    K, V, q = _spike_layers(layers, kv, H, d, L0, spikes, zs)
+    for mask, last in (([True, True, True], 2), ([True, True, False], 1)):
+        st = O.prefill_state(K, V, budget=L0 + 1)
+        O.decode_step(st, 1, q, np.zeros((layers, kv, d)), np.zeros((layers, kv, d)),
+                      O.Params(alpha=0.0, layer_mask=mask))
+        den = math.exp(zs) + L0
+        want = np.full(L0 + 1, 1.0 / den)
+        want[spikes[last]] = math.exp(zs) / den
+        assert np.max(np.abs(st.m[0] - want)) < 1e-15
+
+
+# ---------------------------------------------------------------- schedule
+def test_refresh_sets():
+    assert [t for t in range(1, 14) if O.is_refresh(t, 4, False)] == [1, 5, 9, 13]
+    assert [t for t in range(1, 6) if O.is_refresh(t, 1, False)] == [1, 2, 3, 4, 5]
+    assert [t for t in range(1, 9) if O.is_refresh(t, 3, True)] == [1]
+
+
+def _run(st, q, kn, vn, p, T0=1):
+    outs = []
+    for i in range(q.shape[0]):
+        outs.append(O.decode_step(st, T0 + i, q[i], kn[i], vn[i], p))
+    return outs
+
+
+@pytest.mark.parametrize("gran", [O.GRAN_SEQ, O.GRAN_KVHEAD])
+def test_lazy_r1_equals_full_refresh(gran):
+    rng = np.random.default_rng(9)
+    st = _rand_state(rng, gran=gran)
+    q, kn, vn = _rand_inputs(rng, 10)
+    a, b = _clone(st), _clone(st)
+    oa = _run(a, q, kn, vn, O.Params(alpha=0.8, refresh_period=1, granularity=gran))
+    ob = _run(b, q, kn, vn, O.Params(alpha=0.8, granularity=gran))
+    assert all(np.array_equal(x, y) for x, y in zip(oa, ob))
+    assert np.array_equal(a.m, b.m) and np.array_equal(a.pos, b.pos)
+
+
+def test_lazy_off_refresh_state_carried_and_mean_init():
+    """Eq. 6: off-refresh m_t = m_{t-1} (survivors bit-unchanged); the new token gets the
+    mean of the existing L_t - 1 tokens (Appendix 'New token insertion')."""
+    rng = np.random.default_rng(10)
+    st = _rand_state(rng)
+    q, kn, vn = _rand_inputs(rng, 9)
+    p = O.Params(alpha=0.8, refresh_period=3)
+    for i in range(9):
+        t = i + 1
+        before = dict(zip(st.pos[0].tolist(), st.m[0].tolist()))
+        mean_before = float(np.mean(st.m[0]))
+        new_pos = st.next_pos
+        O.decode_step(st, t, q[i], kn[i], vn[i], p)
+        if not O.is_refresh(t, 3, False):
+            for pos, m in zip(st.pos[0].tolist(), st.m[0].tolist()):
+                if pos == new_pos:
+                    assert m == mean_before
+                else:
+                    assert m == before[pos]
+        assert st.length == min(st.budget, st.length)
+
+
+def test_score_free_equals_lazy_with_long_period():
+    rng = np.random.default_rng(11)
+    st = _rand_state(rng)
+    q, kn, vn = _rand_inputs(rng, 8)
+    a, b, c = _clone(st), _clone(st), _clone(st)
+    oa = _run(a, q, kn, vn, O.Params(alpha=0.9, score_free=True))
+    ob = _run(b, q, kn, vn, O.Params(alpha=0.9, refresh_period=100))
+    assert all(np.array_equal(x, y) for x, y in zip(oa, ob))
+    assert np.array_equal(a.m, b.m) and np.array_equal(a.pos, b.pos)
+    # step 1 of Score-Free equals step 1 of full refresh
+    O.decode_step(c, 1, q[0], kn[0], vn[0], O.Params(alpha=0.9))
+    d = _clone(st)
+    O.decode_step(d, 1, q[0], kn[0], vn[0], O.Params(alpha=0.9, score_free=True))
+    assert np.array_equal(c.m, d.m) and np.array_equal(c.pos, d.pos)
+
+
+def test_score_free_freezes_prefill_ranking():
+    rng = np.random.default_rng(12)
+    st = _rand_state(rng, L0=60, budget=20)
+    q, kn, vn = _rand_inputs(rng, 10)
+    p = O.Params(alpha=0.9, score_free=True)
+    O.decode_step(st, 1, q[0], kn[0], vn[0], p)
+    frozen = {pos: m for pos, m in zip(st.pos[0].tolist(), st.m[0].tolist()) if pos < 60}
+    for i in range(1, 10):
+        O.decode_step(st, i + 1, q[i], kn[i], vn[i], p)
+        for pos, m in zip(st.pos[0].tolist(), st.m[0].tolist()):
+            if pos < 60:
+                assert m == frozen[pos]
+
+
+# ---------------------------------------------------------------- selection / eviction
+def _valid_by_definition(m, keep, B):
+    """Brute-force check of Sec. 3's rule with the tie reading: every kept token ranks
+    above every evicted one under (NaN lowest, m descending, slot ascending)."""
+    def rank_key(i):
+        x = m[i]
+        return (0 if math.isnan(x) else 1, -math.inf if math.isnan(x) else x, -i)
+    ks = set(keep)
+    if len(ks) != min(B, len(m)):
+        return False
+    return all(rank_key(i) > rank_key(j) for i in ks for j in range(len(m)) if j not in ks)
+
+
+def test_selection_golden():
+    for c in _load("selection_cases.json")["cases"]:
+        m = np.array([float(x) for x in c["m"]])
+        keep = O.select_keep(m, c["B"])
+        assert keep.tolist() == c["keep"], c
+
+
+def test_selection_bruteforce_subsets():
+    rng = np.random.default_rng(13)
+    pool = [0.0, -0.0, 0.25, 0.5, 1.0, -1.0, np.inf, -np.inf, np.nan, 1e-300]
+    for trial in range(300):
+        L = int(rng.integers(1, 8))
+        m = np.array([pool[int(i)] for i in rng.integers(0, len(pool), L)])
+        for B in range(0, L + 2):
+            keep = O.select_keep(m, B).tolist()
+            valid = [list(S) for S in itertools.combinations(range(L), min(B, L))
+                     if _valid_by_definition(m, list(S), B)]
+            assert valid == [keep], (m, B, keep, valid)
+
+
+def test_selection_positive_scale_invariance():
+    """Corollary 2: uniform positive scaling is invisible to the ranking."""
+    rng = np.random.default_rng(14)
+    for _ in range(50):
+        m = rng.random(200) ** 3
+        B = int(rng.integers(1, 200))
+        for c in (3.7, 1e-6, 2.0 ** 40):
+            assert np.array_equal(O.select_keep(m, B), O.select_keep(c * m, B))
+
+
+@pytest.mark.parametrize("r,sf", [(1, False), (4, False), (1, True)])
+def test_budget_always_holds_and_compaction_is_stable(r, sf):
+    """Appendix 'Eviction on non-refresh steps': |cache| <= B on every step; kept rows are
+    the previous rows at the kept slots, in ascending slot order (stable)."""
+    rng = np.random.default_rng(15)
+    st = _rand_state(rng, L0=50, budget=17)
+    q, kn, vn = _rand_inputs(rng, 12)
+    p = O.Params(alpha=0.85, refresh_period=r, score_free=sf)
+    for i in range(12):
+        t = i + 1
+        refresh = O.is_refresh(t, r, sf)
+        O.append_token(st, kn[i], vn[i], refresh, p)
+        O.attend_and_score(st, q[i], refresh, p)
+        snap = _clone(st)
+        keeps = O.evict(st)
+        assert st.length == min(snap.length, st.budget)
+        k = keeps[0]
+        assert np.all(np.diff(k) > 0)
+        assert _valid_by_definition(snap.m[0].tolist(), k.tolist(), st.budget)
+        assert np.array_equal(st.pos[0], snap.pos[0][k])
+        assert np.array_equal(st.m[0], snap.m[0][k])
+        for l in range(st.layers):
+            for g in range(st.kv_heads):
+                assert np.array_equal(st.K[l][g], snap.K[l][g][k])
+                assert np.array_equal(st.V[l][g], snap.V[l][g][k])
+
+
+def test_kvhead_rows_select_independently():
+    rng = np.random.default_rng(16)
+    st = _rand_state(rng, gran=O.GRAN_KVHEAD, L0=30, budget=9)
+    q, kn, vn = _rand_inputs(rng, 3)
+    p = O.Params(alpha=0.8, granularity=O.GRAN_KVHEAD)
+    O.append_token(st, kn[0], vn[0], True, p)
+    O.attend_and_score(st, q[0], True, p)
+    snap = _clone(st)
+    O.evict(st)
+    for g in range(st.kv_heads):
+        k = O.select_keep(snap.m[g], 9)
+        assert np.array_equal(st.pos[g], snap.pos[g][k])
+        for l in range(st.layers):
+            assert np.array_equal(st.K[l][g], snap.K[l][g][k])
+    assert not np.array_equal(st.pos[0], st.pos[1])
+
+
+def test_new_token_can_be_evicted_same_step():
+    """Appendix: the new token may be evicted on the step it arrives (non-refresh, mean init
+    below every survivor when the existing state is uniform except one low token)."""
+    K = [[np.zeros((4, 2))]]
+    V = [[np.zeros((4, 2))]]
+    st = O.prefill_state(K, V, budget=4)
+    st.m[0] = np.array([1.0, 1.0, 1.0, 0.2])   # mean 0.8 < 1.0 but > 0.2
+    O.append_token(st, np.zeros((1, 1, 2)), np.zeros((1, 1, 2)), False, O.Params())
+    assert st.m[0, -1] == pytest.approx(0.8)
+    O.evict(st)
+    assert st.pos[0].tolist() == [0, 1, 2, 4]
+    st.m[0] = np.array([1.0, 1.0, 1.0, 1.0])
+    O.append_token(st, np.zeros((1, 1, 2)), np.zeros((1, 1, 2)), False, O.Params())
+    O.evict(st)  # mean 1.0 ties every survivor; the new token holds the highest slot
+    assert st.pos[0].tolist() == [0, 1, 2, 4]
