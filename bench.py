@@ -1,0 +1,468 @@
+#!/usr/bin/env python3
+"""Decode-step throughput of the InertiaKV eviction path on GB300.
+
+Default workload: Llama-3.1-8B-shaped single-stream decode (32 layers, 32 query
+heads, 8 KV heads, head_dim 128, bf16 K/V/q, fp32 utilities), prefilled
+context 32768, budget 10% (3277 tokens), full-refresh EMA with alpha = 0.9.
+Synthetic inputs from the seeded generator (heavy tokens, sinks, drifting
+queries).  A step = one ikv_step call: append, attention of all layers,
+Eq. 1 score + layer-sequential EMA (refresh steps), budgeted selection, stable
+compaction.  Warm-up steps start at decode step 1 (which evicts ~90% of the
+prefill); timed steps are the steady state that follows.
+
+One JSON line on stdout (rank 0).  N > 1 (torchrun): every rank runs its own
+replica on its own GPU (independent sequences, weak scaling); value = tokens
+of all ranks / max time.
+  --impl reference : times the CPU oracle on the host cores instead.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+os.environ.setdefault("OPENBLAS_NUM_THREADS", "1")
+os.environ.setdefault("MKL_NUM_THREADS", "1")
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode tokens/s at 10% KV budget (full/Lazy4/Score-Free); % of HBM peak"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", type=int, default=1)
+    ap.add_argument("--no-modes", action="store_true", help="skip the Lazy4 / Score-Free lines")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline")
+    ap.add_argument("--compact", default="stable", choices=["stable", "holefill"])
+    ap.add_argument("--cpu-steps", type=int, default=0, help="oracle steps in the CPU sample (0 = auto)")
+    return ap.parse_args()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle sample (reference arm and cpu_baseline)
+# ---------------------------------------------------------------------------
+class OracleSample:
+    """The CPU oracle stepping one sequence of the workload at its steady-state size.
+
+    Sample: a cache of B tokens (the workload's decode budget) drawn from the
+    seeded generator, then oracle decode steps from t = 2 on (append, attention
+    of every layer, Eq. 1 score + layer-sequential EMA on refresh steps,
+    eviction back to B).  Built once; each step() is timed on its own."""
+
+    def __init__(self, w, max_steps: int):
+        import numpy as np
+
+        import gen
+        import oracle as O
+
+        self.O, self.w = O, w
+        u = w.u_table()
+        B = w.budgets()[0]
+        K, V = [], []
+        for l in range(w.layers):
+            k, v = w.kv_block(0, l, 0, B, u)
+            K.append([k[g].astype(np.float64) for g in range(w.kv_heads)])
+            V.append([v[g].astype(np.float64) for g in range(w.kv_heads)])
+        self.st = O.prefill_state(K, V, B)
+        self.st.m[0] = np.linspace(1e-4, 2e-4, B)
+        self.p = O.Params(alpha=w.alpha, refresh_period=w.refresh_period, score_free=w.score_free)
+        self.t = 2
+        qs = w.queries(2, 2 + max_steps, u)
+        self.q64 = gen.bf16_to_f32(qs).astype(np.float64) if w.dtype == gen.BF16 else qs.astype(np.float64)
+        self.u = u
+        self.B = B
+
+    def step(self) -> float:
+        i = self.t - 2
+        kn, vn = self.w.new_tokens(self.t, self.u)
+        t0 = time.perf_counter()
+        self.O.decode_step(self.st, self.t, self.q64[i][:, 0], kn[:, 0], vn[:, 0], self.p)
+        dt = time.perf_counter() - t0
+        self.t += 1
+        return dt
+
+    def describe(self, n: int) -> str:
+        w = self.w
+        return (f"{n} oracle decode steps of one sequence with a {self.B}-token cache (the decode budget), "
+                f"{w.layers} layers x {w.q_heads} q heads / {w.kv_heads} kv heads x d {w.head_dim}, "
+                f"fp64 numpy, 1 BLAS thread; tokens/s = steps / summed step time")
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import gen
+
+    w = gen.config(args.config)
+    s = OracleSample(w, args.warmup + args.steps)
+    for _ in range(args.warmup):
+        s.step()
+    sec = sum(s.step() for _ in range(args.steps))
+    value = w.batch * args.steps / sec
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * sec / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": w.name, "prefill": w.prefill[0], "budget": w.budgets()[0],
+                                            "alpha": w.alpha, "refresh_period": w.refresh_period},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                             "sample": s.describe(args.steps)},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    def __init__(self, index: int):
+        self.f = tempfile.NamedTemporaryFile(mode="w+", suffix=".csv", delete=False)
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", f"--id={index}", f"--query-gpu={q}", "--format=csv,noheader,nounits",
+                                       "-lms", "100"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.p.terminate()
+        self.p.wait()
+        self.f.flush()
+        self.f.seek(0)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.f.read().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        os.unlink(self.f.name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def setup(w, device, compact_mode):
+    import numpy as np
+    import torch
+
+    import gen
+    from paper_2609_03515_gb300 import DecodeCache, ikv
+
+    c = DecodeCache(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.cap,
+                    dtype=ikv.IKV_BF16 if w.dtype == gen.BF16 else ikv.IKV_F32, page_size=w.page_size,
+                    device=device, page_perm_seed=1)
+    return c
+
+
+def reset(c, w, u_dev):
+    import torch
+
+    import gen
+
+    c.set_prefill(w.prefill, w.budgets())
+    sp = w.spec()
+    L0 = torch.tensor(w.prefill, dtype=torch.int32, device=c.k.device)
+    rc = gen.cuda_lib().ikvgen_fill_paged_cuda(ctypes.byref(sp), u_dev.data_ptr(), c.k.data_ptr(), c.v.data_ptr(),
+                                               c.block_table.data_ptr(), L0.data_ptr(), c.num_pages, c.page_size,
+                                               c.max_pages, max(w.prefill), w.dtype,
+                                               torch.cuda.current_stream().cuda_stream)
+    assert rc == 0
+    torch.cuda.synchronize()
+
+
+def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_detail: bool, dist):
+    """Warm-up then K timed steps of one schedule; returns a dict of measurements."""
+    import torch
+
+    from paper_2609_03515_gb300 import ikv
+
+    reset(c, w, u_dev)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode)
+    budgets = w.budgets()
+    lens = list(w.prefill)
+    out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=c.torch_dtype, device=c.k.device)
+    stream = torch.cuda.current_stream()
+
+    def step(t, timing=None):
+        nonlocal lens
+        if timing is not None:
+            p.timing = ctypes.pointer(timing)
+        else:
+            p.timing = None
+        ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws,
+                     ws.numel(), stream)
+        lens = [min(L + 1, B) if L + 1 > B else L + 1 for L, B in zip(lens, budgets)]
+
+    W, K = args.warmup, args.steps
+    for t in range(1, W + 1):
+        step(t)
+    torch.cuda.synchronize()
+    evs = []
+    timings = []
+    if want_detail:
+        for _ in range(K):
+            e = [torch.cuda.Event(enable_timing=True) for _ in range(7)]
+            evs.append(e)
+            tm = ikv.ikv_timing(*[x.cuda_event for x in e])
+            timings.append(tm)
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(torch.cuda.current_device()) if want_detail else None
+    launches0 = ikv.ikv_launch_count()
+    start.record(stream)
+    for i in range(K):
+        step(W + 1 + i, timings[i] if want_detail else None)
+    stop.record(stream)
+    torch.cuda.synchronize()
+    launches = ikv.ikv_launch_count() - launches0
+    ms = start.elapsed_time(stop)
+    if dist:
+        tt = torch.tensor([ms], device=c.k.device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    res = {"ms": ms, "launches": launches, "lens": lens}
+    if want_detail:
+        res["clocks"] = clocks.stop()
+        names = ["append", "attend", "combine", "score_ema", "select", "compact"]
+        per = {n: [] for n in names}
+        for e in evs:
+            for j, n in enumerate(names):
+                per[n].append(e[j].elapsed_time(e[j + 1]))
+        res["kernel_ms"] = {n: sum(v) / len(v) for n, v in per.items()}
+    return res
+
+
+def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist):
+    """Same steps through the C ABI, inputs from pinned host memory and the output read back every step."""
+    import torch
+
+    from paper_2609_03515_gb300 import ikv
+
+    reset(c, w, u_dev)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode)
+    budgets = w.budgets()
+    lens = list(w.prefill)
+    dev = c.k.device
+    q_d = torch.empty(qs_h.shape[1:], dtype=qs_h.dtype, device=dev)
+    kn_d = torch.empty(kn_h.shape[1:], dtype=kn_h.dtype, device=dev)
+    vn_d = torch.empty_like(kn_d)
+    out_d = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=c.torch_dtype, device=dev)
+    out_h = torch.empty(out_d.shape, dtype=out_d.dtype, pin_memory=True)
+    stream = torch.cuda.current_stream()
+
+    def step(t):
+        nonlocal lens
+        q_d.copy_(qs_h[t - 1], non_blocking=True)
+        kn_d.copy_(kn_h[t - 1], non_blocking=True)
+        vn_d.copy_(vn_h[t - 1], non_blocking=True)
+        ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, q_d, kn_d, vn_d, out_d, ws, ws.numel(), stream)
+        out_h.copy_(out_d, non_blocking=True)
+        lens = [min(L + 1, B) if L + 1 > B else L + 1 for L, B in zip(lens, budgets)]
+
+    W, K = args.warmup, args.steps
+    for t in range(1, W + 1):
+        step(t)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for i in range(K):
+        step(W + 1 + i)
+    stop.record(stream)
+    torch.cuda.synchronize()
+    ms = start.elapsed_time(stop)
+    if dist:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    h2d = (q_d.numel() + kn_d.numel() + vn_d.numel()) * q_d.element_size()
+    d2h = out_d.numel() * out_d.element_size()
+    return ms, h2d, d2h
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as tdist
+
+        torch.cuda.set_device(local)
+        tdist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        dist = tdist
+    else:
+        torch.cuda.set_device(0)
+
+    import gen
+    import __graft_entry__
+
+    if rank == 0 or world == 1:
+        __graft_entry__.build()
+    if dist:
+        dist.barrier()
+    from paper_2609_03515_gb300 import ikv
+
+    w = gen.config(args.config)
+    # each rank decodes its own independent sequences (distinct seed per rank)
+    w = w.with_(seed=w.seed + 1000 * rank)
+    total_steps = args.warmup + args.steps
+    if total_steps > w.steps:
+        w = w.with_(steps=total_steps)
+    compact_mode = ikv.IKV_COMPACT_STABLE if args.compact == "stable" else ikv.IKV_COMPACT_HOLEFILL
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        n = args.cpu_steps or 8
+        smp = OracleSample(w, n + 1)
+        smp.step()  # first step outside the sample (allocator warm-up)
+        sec = sum(smp.step() for _ in range(n))
+        cpu = {"value": n / sec, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": smp.describe(n)}
+        del smp
+
+    dev = torch.device("cuda", torch.cuda.current_device())
+    u = w.u_table()
+    u_dev = torch.from_numpy(u).to(dev)
+    c = setup(w, dev, compact_mode)
+    ws = c.step_workspace()
+    T = total_steps
+    qs_h = w.queries(1, T + 1, u)
+    tdt = c.torch_dtype
+    if w.dtype == gen.BF16:
+        qs_t = torch.from_numpy(qs_h.view(np.int16)).view(torch.bfloat16)
+    else:
+        qs_t = torch.from_numpy(qs_h)
+    qs_dev = qs_t.to(dev)
+    kn_dev = torch.empty((T, w.layers, w.batch, w.kv_heads, w.head_dim), dtype=tdt, device=dev)
+    vn_dev = torch.empty_like(kn_dev)
+    sp = w.spec()
+    L0 = torch.tensor(w.prefill, dtype=torch.int32, device=dev)
+    rc = gen.cuda_lib().ikvgen_fill_tokens_cuda(ctypes.byref(sp), u_dev.data_ptr(), L0.data_ptr(), 1, T + 1, w.dtype,
+                                                kn_dev.data_ptr(), vn_dev.data_ptr(),
+                                                torch.cuda.current_stream().cuda_stream)
+    assert rc == 0
+    torch.cuda.synchronize()
+
+    full = run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, True, dist)
+    modes = {}
+    if not args.no_modes:
+        for name, ww in (("lazy4", w.with_(refresh_period=4)), ("score_free", w.with_(score_free=True))):
+            r = run_mode(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, False, dist)
+            modes[name] = r
+    qs_pin = qs_t.pin_memory()
+    kn_pin = kn_dev.cpu().pin_memory()
+    vn_pin = vn_dev.cpu().pin_memory()
+    e2e_ms, h2d, d2h = run_e2e(args, w, c, u_dev, ws, compact_mode, qs_pin, kn_pin, vn_pin, dist)
+
+    K = args.steps
+    tokens = w.batch * K * world
+    value = tokens / (full["ms"] / 1e3)
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return
+
+    peak, peak_kind = load_peaks()
+    # attention kernel roofline: algorithmic bytes of one launch at the steady-state length
+    L = [min(x + 1, B + 1) for x, B in zip(w.prefill, w.budgets())]  # length seen by the timed steps
+    esz = 2 if w.dtype == gen.BF16 else 4
+    kv_bytes = sum(L) * w.layers * w.kv_heads * w.head_dim * 2 * esz
+    q_bytes = w.layers * w.batch * w.q_heads * w.head_dim * esz
+    att_ms = full["kernel_ms"]["attend"]
+    achieved = (kv_bytes + q_bytes) / (att_ms / 1e3) / 1e9
+    traffic = None
+    prof = os.path.join(ROOT, "profiles", "attend_traffic.json")
+    if os.path.exists(prof):
+        try:
+            with open(prof) as f:
+                d = json.load(f)
+            if d.get("kernel_rev") == "attend_v1" and d.get("workload") == w.name:
+                traffic = d.get("bytes_per_launch")
+        except (OSError, ValueError):
+            traffic = None
+    line = {
+        "metric": METRIC,
+        "value": value,
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": args.warmup,
+        "ms_per_step": full["ms"] / K,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16" if w.dtype == gen.BF16 else "f32",
+        "data": "synthetic",
+        "config": {"workload": w.name, "batch_per_gpu": w.batch, "layers": w.layers, "q_heads": w.q_heads,
+                   "kv_heads": w.kv_heads, "head_dim": w.head_dim, "prefill": w.prefill[0] if w.batch == 1 else w.prefill,
+                   "budget": w.budgets(), "alpha": w.alpha, "refresh": "full", "compaction": args.compact,
+                   "timed_steps": f"decode steps {args.warmup + 1}..{args.warmup + K} (steady state; step 1 in warm-up)",
+                   "l2": "inputs exceed L2 (K/V working set %.0f MB > 129 MB), no flush" % (kv_bytes / 1e6),
+                   "parallelism": f"replicas x{world}"},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                     "traffic": traffic, "kernel": "attend_split_kernel", "peak_kind": peak_kind,
+                     "bytes_per_launch": kv_bytes + q_bytes, "ms_per_launch": att_ms},
+        "kernel_ms_per_step": full["kernel_ms"],
+        "cpu_baseline": cpu,
+        "e2e": {"value": w.batch * K * world / (e2e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": full["launches"],
+        "clocks": full["clocks"],
+        "modes": {"full": value, **{k: w.batch * K * world / (v["ms"] / 1e3) for k, v in modes.items()}},
+    }
+    if modes:
+        line["speedup_vs_full"] = {k: (w.batch * K * world / (v["ms"] / 1e3)) / value for k, v in modes.items()}
+    print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,219 @@
+/*
+ * ikv.h -- C ABI of the InertiaKV decode-step eviction path on GB300 (sm_103a).
+ *
+ * InertiaKV (arxiv 2609.03515) keeps, per sequence, a running utility m over
+ * the cached tokens.  Every decode step appends the new token, runs grouped-
+ * query decode attention, and (on refresh steps) folds each eligible layer's
+ * head-averaged last-query attention probabilities into m with an EMA, layer
+ * after layer.  Whenever the cache exceeds its budget B the lowest-utility
+ * tokens are evicted for good and the surviving K/V rows are compacted.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Every function returns ikv_status; IKV_OK == 0.  On error nothing is
+ *    launched and ikv_last_error() returns a message (thread-local).
+ *  - Tensor pointers are DEVICE pointers owned by the caller and borrowed for
+ *    the duration of the call.  The library allocates and frees nothing;
+ *    scratch memory comes from the caller's workspace (ws, ws_bytes), sized
+ *    by the matching *_workspace_size function.  The workspace needs no
+ *    initialisation and carries nothing between calls.
+ *  - Work is enqueued asynchronously on the caller's stream; arguments are
+ *    checked on the host before anything is launched.  Errors raised by a
+ *    kernel after launch surface as IKV_ERR_CUDA on a later call.
+ *  - dtype of K/V/q/out: IKV_F32 or IKV_BF16.  Utilities, scores and all
+ *    accumulation are fp32.  head_dim must be 64 or 128 and
+ *    q_heads / kv_heads (the GQA group size G) one of 1, 2, 4, 7, 8.
+ *  - Alignment: K/V pools, q, out, k_new, v_new must be 16-byte aligned.
+ *
+ * Paged K/V layout
+ * ----------------
+ *  k, v: [layers][num_pages][kv_heads][page_size][head_dim] (dtype).
+ *  Sequence b owns logical pages 0..max_pages-1 mapped through
+ *  block_table[b][p] to physical pages; its cache slot j lives in logical page
+ *  j / page_size at offset j % page_size.  cap = max_pages * page_size is the
+ *  slot capacity of a row.  Slots 0..len[b]-1 are valid.
+ *
+ * Utility rows
+ * ------------
+ *  Granularity IKV_GRAN_SEQ (default): one utility row per sequence (rows =
+ *  batch), Eq. 1 averages all q_heads, and the kept set applies to every
+ *  layer and KV head.  IKV_GRAN_KVHEAD: one row per (sequence, KV head)
+ *  (rows = batch * kv_heads, row index b * kv_heads + g), the score averages
+ *  that KV head's query group, and the kept set applies to that KV head in
+ *  every layer.  ema, pos and keep arrays are [rows][cap].
+ */
+#ifndef IKV_H
+#define IKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    IKV_OK = 0,
+    IKV_ERR_ARG = 1,         /* null pointer, out-of-range scalar */
+    IKV_ERR_SHAPE = 2,       /* inconsistent or unsupported sizes */
+    IKV_ERR_ALIGN = 3,       /* pointer not 16-byte aligned */
+    IKV_ERR_WORKSPACE = 4,   /* workspace missing or too small */
+    IKV_ERR_UNSUPPORTED = 5, /* valid request this build does not implement */
+    IKV_ERR_CUDA = 6         /* a CUDA runtime call failed (incl. earlier async errors) */
+} ikv_status;
+
+enum { IKV_F32 = 0, IKV_BF16 = 1 };
+enum { IKV_GRAN_SEQ = 0, IKV_GRAN_KVHEAD = 1 };
+enum { IKV_COMPACT_STABLE = 0, IKV_COMPACT_HOLEFILL = 1 };
+enum { IKV_INIT_ZERO = 0, IKV_INIT_MEAN = 1 };
+
+typedef struct {
+    int32_t batch, layers, q_heads, kv_heads, head_dim;
+    int32_t dtype;        /* IKV_F32 | IKV_BF16 */
+    int32_t granularity;  /* IKV_GRAN_SEQ | IKV_GRAN_KVHEAD */
+} ikv_shape;
+
+typedef struct {
+    void *k, *v;                 /* paged pools, see above (device) */
+    const int32_t *block_table;  /* [batch][max_pages] physical page ids (device) */
+    int32_t num_pages;           /* physical pages per layer in the pools */
+    int32_t page_size;           /* slots per page, >= 1 */
+    int32_t max_pages;           /* logical pages per sequence; cap = max_pages * page_size */
+    int32_t *len;                /* [batch] valid slots per sequence (device) */
+    int32_t *pos;                /* [rows][cap] original token position per slot (device) */
+    int32_t *next_pos;           /* [batch] position given to the next appended token (device) */
+    int32_t max_len;             /* HOST-side upper bound on every len[b]; sizes launch grids */
+} ikv_cache;
+
+/* Optional per-kernel CUDA events recorded on the call's stream by ikv_step
+ * (caller-created with cudaEventCreate; NULL members are skipped):
+ * begin (before the append), append_end, attend_end (after the attention
+ * kernel), combine_end (after the split combine), score_end (after the score
+ * + EMA kernels), select_end, end (after compaction). */
+typedef struct {
+    cudaEvent_t begin, append_end, attend_end, combine_end, score_end, select_end, end;
+} ikv_timing;
+
+typedef struct {
+    float alpha;                    /* EMA coefficient of Eq. 4, in [0, 1] */
+    int32_t refresh_period;         /* r of Eq. 6 (>= 1; 1 = full refresh) */
+    int32_t score_free;             /* 1: score at step 1 only, then freeze (Sec. 3.2) */
+    const int32_t *budget;          /* [batch] decode budget B per sequence (device) */
+    const uint8_t *layer_eligible;  /* HOST [layers] 0/1, NULL = all layers eligible */
+    int32_t compact_mode;           /* IKV_COMPACT_STABLE (order-preserving) | IKV_COMPACT_HOLEFILL */
+    int32_t refresh_init;           /* utility of a token appended on a refresh step:
+                                       IKV_INIT_ZERO (m_0 = 0 rule) | IKV_INIT_MEAN */
+    const ikv_timing *timing;       /* nullable */
+} ikv_params;
+
+/* Message for the last error on this thread ("" if none). */
+const char *ikv_last_error(void);
+
+/* Number of kernels this library has launched in this process. */
+int64_t ikv_launch_count(void);
+
+/* ---------------------------------------------------------------------------
+ * ikv_decode_attend_score -- one layer of decode attention plus its score.
+ *
+ * Eq. 1 and Appendix "Per-step scoring" (last query's attention weights,
+ * mean-pooled over heads; GQA heads share their KV head).  For every sequence
+ * b and query head h of layer `layer`:
+ *     out[b][h] = softmax(q[b][h] . K_g^T / sqrt(d)) V_g  over slots 0..len[b]-1
+ * with g = h / G.  If score != NULL it also writes, for i < len[b],
+ *     score[r][i] = mean over the row's heads of softmax probability of slot i
+ * (all q_heads for IKV_GRAN_SEQ, the KV head's group for IKV_GRAN_KVHEAD).
+ * If ema != NULL the EMA of Eq. 4 is applied in place for i < len[b]:
+ *     ema[r][i] = alpha * ema[r][i] + (1 - alpha) * score_i
+ * which is one layer of the Appendix's layer-sequential update.
+ *
+ *  q, out: [batch][q_heads][head_dim] (dtype).  score, ema: [rows][cap] fp32.
+ *  ws: at least ikv_attend_workspace_size() bytes.
+ * ------------------------------------------------------------------------- */
+ikv_status ikv_attend_workspace_size(const ikv_shape *shape, const ikv_cache *cache, size_t *bytes);
+ikv_status ikv_decode_attend_score(const ikv_shape *shape, const ikv_cache *cache, int32_t layer,
+                                   const void *q, void *out, float *score, float *ema, float alpha,
+                                   void *ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * ikv_ema_update -- Eq. 4 on a score array, in place.
+ *     ema[r][i] = alpha * ema[r][i] + (1 - alpha) * score[r][i],  i < len[r / rows_per_seq]
+ *  rows_per_seq: 1 for IKV_GRAN_SEQ, kv_heads for IKV_GRAN_KVHEAD.
+ * ------------------------------------------------------------------------- */
+ikv_status ikv_ema_update(int32_t rows, int32_t cap, float *ema, const float *score, const int32_t *len,
+                          int32_t rows_per_seq, float alpha, cudaStream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * ikv_select_budget -- which tokens survive (Sec. 3: evict the lowest m_t(i)
+ * whenever the cache exceeds B).
+ *
+ * For row r with L = len[r / rows_per_seq] and B = budget[r / rows_per_seq]:
+ * if L <= B every slot is kept (keep[r][j] = j, keep_len[r] = L); otherwise
+ * keep[r][0..B) lists, in ascending slot order, the B slots with the largest
+ * util[r][i] (i < L).  Ties keep the lower slot; -0.0 equals +0.0; NaN ranks
+ * below every number.  Bit-exact: the result depends only on the fp32 values.
+ *  util: [rows][cap] fp32; keep: [rows][cap] int32; keep_len: [rows] int32.
+ * ------------------------------------------------------------------------- */
+ikv_status ikv_select_budget(int32_t rows, int32_t cap, const float *util, const int32_t *len,
+                             int32_t rows_per_seq, const int32_t *budget, int32_t *keep, int32_t *keep_len,
+                             cudaStream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * ikv_compact_kv -- in-place gather compaction after eviction ("cache
+ * remapping" of the Appendix "Hook-level profiling" paragraph).
+ *
+ * For every sequence b, layer and KV head g (utility row r of (b, g)):
+ * slot j of the compacted row holds what slot keep[r][j] held, j < keep_len[r].
+ * The same gather is applied to pos and, if ema != NULL, to ema.  Afterwards
+ * len[b] = keep_len[r].  IKV_COMPACT_STABLE preserves the survivors' order
+ * (moves only the shifted suffix); IKV_COMPACT_HOLEFILL moves survivors that
+ * sit at slots >= keep_len into the evicted slots below keep_len, keeping the
+ * same set but not its order (fewer moved rows).
+ *  keep/keep_len as produced by ikv_select_budget.  ws: at least
+ *  ikv_compact_workspace_size() bytes (0 for the stable mode).
+ * ------------------------------------------------------------------------- */
+ikv_status ikv_compact_workspace_size(const ikv_shape *shape, const ikv_cache *cache, int32_t mode, size_t *bytes);
+ikv_status ikv_compact_kv(const ikv_shape *shape, ikv_cache *cache, const int32_t *keep, const int32_t *keep_len,
+                          float *ema, int32_t mode, void *ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * ikv_append_token -- add the new token of every sequence at slot len[b].
+ *
+ * Writes k_new/v_new ([layers][batch][kv_heads][head_dim]) into slot len[b]
+ * of every layer, sets pos[r][len[b]] = next_pos[b], and gives the token the
+ * utility 0 (init_mean == 0) or the mean utility of the existing len[b]
+ * tokens of its row (init_mean == 1, Appendix "New token insertion during
+ * non-refresh steps").  Then len[b] += 1 and next_pos[b] += 1.
+ * Fails with IKV_ERR_SHAPE (host) if max_len + 1 > cap.
+ * ------------------------------------------------------------------------- */
+ikv_status ikv_append_token(const ikv_shape *shape, ikv_cache *cache, const void *k_new, const void *v_new,
+                            float *ema, int32_t init_mean, void *ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * ikv_step -- one whole decode step t (1-based) of InertiaKV / -Lazy /
+ * Score-Free for every sequence of the batch:
+ *   1. refresh = score_free ? (t == 1) : ((t - 1) % refresh_period == 0)   (Eq. 6)
+ *   2. append the new token (utility: refresh_init on refresh steps, the mean
+ *      of the existing utilities otherwise; Appendix "New token insertion")
+ *   3. attention of every layer over all len[b] slots (the new token included)
+ *   4. refresh steps only: for each eligible layer in ascending order,
+ *      ema = alpha * ema + (1 - alpha) * s_layer  (Eq. 1, Eq. 4, Appendix
+ *      "Layer scoring"); off-refresh steps leave ema untouched (Eq. 6)
+ *   5. if len[b] > budget[b]: keep the budget[b] highest utilities and compact
+ *      (Appendix "Eviction on non-refresh steps": also on off-refresh steps)
+ *  q: [layers][batch][q_heads][head_dim]; k_new, v_new: [layers][batch][kv_heads][head_dim];
+ *  out: [layers][batch][q_heads][head_dim] (all dtype).  ema: [rows][cap] fp32.
+ *  cache->max_len bounds len[] BEFORE the append; the step needs max_len + 1 <= cap.
+ *  After the step the caller should lower max_len to max(budget) if it tracks it.
+ * ------------------------------------------------------------------------- */
+ikv_status ikv_step_workspace_size(const ikv_shape *shape, const ikv_cache *cache, size_t *bytes);
+ikv_status ikv_step(const ikv_shape *shape, const ikv_params *params, ikv_cache *cache, float *ema, int32_t t,
+                    const void *q, const void *k_new, const void *v_new, void *out, void *ws, size_t ws_bytes,
+                    cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* IKV_H */

@@ -1,0 +1,125 @@
+"""InertiaKV decode-step eviction path on GB300 (sm_103a): Python side.
+
+``ikv`` binds the C ABI of ``libikv.so`` (include/ikv.h).  ``DecodeCache``
+allocates the device tensors a caller hands to that ABI -- paged K/V pools,
+block table, lengths, positions, utilities, budgets and workspace -- using
+PyTorch purely as the device allocator.  All arithmetic of the path runs in
+the CUDA library.
+"""
+from __future__ import annotations
+
+from typing import Optional, Sequence
+
+import torch
+
+from . import ikv
+
+__all__ = ["ikv", "DecodeCache"]
+
+
+class DecodeCache:
+    """Device buffers of one batch of decode sequences.
+
+    k, v:        [layers][num_pages][kv_heads][page_size][head_dim] (bf16 or fp32)
+    block_table: [batch][max_pages] int32 physical page of each logical page
+    len:         [batch] int32;  next_pos: [batch] int32
+    pos, ema:    [rows][cap] int32 / fp32, rows = batch (per-sequence state) or batch * kv_heads
+    budget:      [batch] int32
+    """
+
+    def __init__(self, batch: int, layers: int, q_heads: int, kv_heads: int, head_dim: int, cap_tokens: int,
+                 dtype: int = ikv.IKV_BF16, page_size: int = 64, granularity: int = ikv.IKV_GRAN_SEQ,
+                 device: str = "cuda", page_perm_seed: Optional[int] = None):
+        self.batch, self.layers, self.q_heads, self.kv_heads, self.head_dim = batch, layers, q_heads, kv_heads, head_dim
+        self.dtype, self.granularity, self.page_size = dtype, granularity, page_size
+        self.max_pages = (cap_tokens + page_size - 1) // page_size
+        self.cap = self.max_pages * page_size
+        self.num_pages = batch * self.max_pages
+        tdt = torch.bfloat16 if dtype == ikv.IKV_BF16 else torch.float32
+        self.torch_dtype = tdt
+        shp = (layers, self.num_pages, kv_heads, page_size, head_dim)
+        self.k = torch.zeros(shp, dtype=tdt, device=device)
+        self.v = torch.zeros(shp, dtype=tdt, device=device)
+        pages = torch.arange(self.num_pages, dtype=torch.int32)
+        if page_perm_seed is not None:
+            g = torch.Generator().manual_seed(page_perm_seed)
+            pages = pages[torch.randperm(self.num_pages, generator=g)]
+        self.block_table = pages.view(batch, self.max_pages).to(device)
+        self.rows = batch if granularity == ikv.IKV_GRAN_SEQ else batch * kv_heads
+        self.len = torch.zeros(batch, dtype=torch.int32, device=device)
+        self.next_pos = torch.zeros(batch, dtype=torch.int32, device=device)
+        self.pos = torch.zeros((self.rows, self.cap), dtype=torch.int32, device=device)
+        self.ema = torch.zeros((self.rows, self.cap), dtype=torch.float32, device=device)
+        self.budget = torch.zeros(batch, dtype=torch.int32, device=device)
+        self.max_len = 0
+
+    # ---- ABI structs ------------------------------------------------------
+    def shape(self) -> ikv.ikv_shape:
+        return ikv.ikv_shape(self.batch, self.layers, self.q_heads, self.kv_heads, self.head_dim, self.dtype,
+                             self.granularity)
+
+    def cache(self, max_len: Optional[int] = None) -> ikv.ikv_cache:
+        ml = self.max_len if max_len is None else max_len
+        return ikv.ikv_cache(self.k.data_ptr(), self.v.data_ptr(), self.block_table.data_ptr(), self.num_pages,
+                             self.page_size, self.max_pages, self.len.data_ptr(), self.pos.data_ptr(),
+                             self.next_pos.data_ptr(), ml)
+
+    @property
+    def rows_per_seq(self) -> int:
+        return 1 if self.granularity == ikv.IKV_GRAN_SEQ else self.kv_heads
+
+    # ---- host-side helpers (setup / inspection) ----------------------------
+    def set_prefill(self, lengths: Sequence[int], budgets: Sequence[int]) -> None:
+        """Mark slots [0, L0_b) as holding positions 0..L0_b-1 with utility 0 (m_0 = 0)."""
+        dev = self.len.device
+        self.len.copy_(torch.tensor(list(lengths), dtype=torch.int32, device=dev))
+        self.next_pos.copy_(self.len)
+        self.budget.copy_(torch.tensor(list(budgets), dtype=torch.int32, device=dev))
+        ar = torch.arange(self.cap, dtype=torch.int32, device=dev)
+        self.pos.copy_(ar.expand(self.rows, self.cap))
+        self.ema.zero_()
+        self.max_len = max(lengths)
+
+    def slot_rows(self, b: int, layer: int, g: int, n: int) -> torch.Tensor:
+        """K/V rows [n][head_dim] of slots 0..n-1 of (b, layer, g), gathered through the block table."""
+        slots = torch.arange(n, device=self.k.device)
+        pages = self.block_table[b, (slots // self.page_size).long()].long()
+        return pages, slots % self.page_size
+
+    def gather(self, pool: torch.Tensor, b: int, layer: int, g: int, n: int) -> torch.Tensor:
+        pages, off = self.slot_rows(b, layer, g, n)
+        return pool[layer, pages, g, off]
+
+    def scatter(self, pool: torch.Tensor, b: int, layer: int, g: int, rows: torch.Tensor, start: int = 0) -> None:
+        n = rows.shape[0]
+        slots = torch.arange(start, start + n, device=pool.device)
+        pages = self.block_table[b, (slots // self.page_size).long()].long()
+        pool[layer, pages, g, slots % self.page_size] = rows.to(pool.dtype)
+
+    def step_workspace(self) -> torch.Tensor:
+        n = ikv.ikv_step_workspace_size(self.shape(), self.cache(self.cap - 1))
+        return torch.empty(n, dtype=torch.uint8, device=self.k.device)
+
+    def params(self, alpha: float, refresh_period: int = 1, score_free: bool = False,
+               compact_mode: int = ikv.IKV_COMPACT_STABLE, refresh_init: int = ikv.IKV_INIT_ZERO,
+               layer_eligible: Optional[Sequence[int]] = None) -> ikv.ikv_params:
+        p = ikv.ikv_params()
+        p.alpha = alpha
+        p.refresh_period = refresh_period
+        p.score_free = 1 if score_free else 0
+        p.budget = self.budget.data_ptr()
+        if layer_eligible is not None:
+            self._elig = (ctypes_u8 * self.layers)(*[1 if x else 0 for x in layer_eligible])
+            p.layer_eligible = ctypes_addr(self._elig)
+        p.compact_mode = compact_mode
+        p.refresh_init = refresh_init
+        return p
+
+
+import ctypes as _ct  # noqa: E402
+
+ctypes_u8 = _ct.c_uint8
+
+
+def ctypes_addr(x) -> int:
+    return _ct.addressof(x)

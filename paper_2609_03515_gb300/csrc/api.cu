@@ -1,0 +1,461 @@
+// C ABI of the InertiaKV decode-step path: argument checks, workspace layout
+// and the launch sequence of one decode step.  No allocation happens here.
+#include <atomic>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+#include "ikv_internal.cuh"
+
+namespace ikv {
+
+static std::atomic<int64_t> g_launches{0};
+void note_launch(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+ikv_status fail(ikv_status s, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+    return s;
+}
+
+ikv_status cuda_fail(cudaError_t e, const char *what) {
+    return fail(IKV_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define IKV_TRY_CUDA(expr, what)                         \
+    do {                                                 \
+        cudaError_t _e = (expr);                         \
+        if (_e != cudaSuccess) return cuda_fail(_e, what); \
+    } while (0)
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int sm_count() {
+    static int cached[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+    if (cached[dev] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+        cached[dev] = n;
+    }
+    return cached[dev];
+}
+
+ikv_status check_shape(const ikv_shape *s) {
+    if (!s) return fail(IKV_ERR_ARG, "shape is NULL");
+    if (s->batch <= 0 || s->layers <= 0 || s->q_heads <= 0 || s->kv_heads <= 0)
+        return fail(IKV_ERR_SHAPE, "batch/layers/heads must be positive");
+    if (s->layers > kMaxLayers) return fail(IKV_ERR_SHAPE, "layers > %d", kMaxLayers);
+    if (s->q_heads % s->kv_heads) return fail(IKV_ERR_SHAPE, "q_heads %% kv_heads != 0");
+    const int G = s->q_heads / s->kv_heads;
+    if (!(G == 1 || G == 2 || G == 4 || G == 7 || G == 8))
+        return fail(IKV_ERR_UNSUPPORTED, "GQA group %d not supported (1, 2, 4, 7, 8)", G);
+    if (s->head_dim != 64 && s->head_dim != 128) return fail(IKV_ERR_UNSUPPORTED, "head_dim must be 64 or 128");
+    if (s->dtype != IKV_F32 && s->dtype != IKV_BF16) return fail(IKV_ERR_ARG, "dtype must be IKV_F32 or IKV_BF16");
+    if (s->granularity != IKV_GRAN_SEQ && s->granularity != IKV_GRAN_KVHEAD)
+        return fail(IKV_ERR_ARG, "granularity must be IKV_GRAN_SEQ or IKV_GRAN_KVHEAD");
+    return IKV_OK;
+}
+
+int elem_bytes(const ikv_shape *s) { return s->dtype == IKV_BF16 ? 2 : 4; }
+int rows_per_seq(const ikv_shape *s) { return s->granularity == IKV_GRAN_SEQ ? 1 : s->kv_heads; }
+
+ikv_status check_cache(const ikv_shape *s, const ikv_cache *c, bool need_pos) {
+    if (!c) return fail(IKV_ERR_ARG, "cache is NULL");
+    if (!c->k || !c->v || !c->block_table || !c->len) return fail(IKV_ERR_ARG, "cache k/v/block_table/len is NULL");
+    if (need_pos && (!c->pos || !c->next_pos)) return fail(IKV_ERR_ARG, "cache pos/next_pos is NULL");
+    if (!aligned16(c->k) || !aligned16(c->v)) return fail(IKV_ERR_ALIGN, "K/V pools must be 16-byte aligned");
+    if (c->page_size <= 0 || c->max_pages <= 0 || c->num_pages <= 0)
+        return fail(IKV_ERR_SHAPE, "page_size/max_pages/num_pages must be positive");
+    const int64_t cap = (int64_t)c->page_size * c->max_pages;
+    if (cap > (int64_t)(1 << 30)) return fail(IKV_ERR_SHAPE, "cap too large");
+    if (c->max_len < 0 || c->max_len > cap) return fail(IKV_ERR_SHAPE, "max_len %d outside [0, cap=%lld]", c->max_len, (long long)cap);
+    (void)s;
+    return IKV_OK;
+}
+
+int32_t cap_of(const ikv_cache *c) { return c->page_size * c->max_pages; }
+
+PagedView view_of(const ikv_shape *s, const ikv_cache *c) {
+    PagedView v;
+    v.block_table = c->block_table;
+    v.num_pages = c->num_pages;
+    v.page_size = c->page_size;
+    v.max_pages = c->max_pages;
+    v.kv_heads = s->kv_heads;
+    v.head_dim = s->head_dim;
+    return v;
+}
+
+// ---- workspace layout ------------------------------------------------------
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+struct AttendWs {
+    size_t part_ml, part_o, lse2, logits, end;
+};
+
+AttendWs attend_ws(const ikv_shape *s, int32_t cap, int n_layers, bool logits) {
+    AttendWs w;
+    size_t off = 0;
+    const size_t bhl = (size_t)s->batch * n_layers * s->q_heads;
+    w.part_ml = off;
+    off = align256(off + bhl * kMaxSplits * 2 * sizeof(float));
+    w.part_o = off;
+    off = align256(off + bhl * kMaxSplits * s->head_dim * sizeof(float));
+    w.lse2 = off;
+    off = align256(off + bhl * sizeof(float));
+    w.logits = off;
+    if (logits) off = align256(off + bhl * (size_t)cap * sizeof(float));
+    w.end = off;
+    return w;
+}
+
+struct StepWs {
+    AttendWs at;
+    size_t keep, keep_len, done, moves, n_moves, end;
+};
+
+StepWs step_ws(const ikv_shape *s, int32_t cap) {
+    StepWs w;
+    w.at = attend_ws(s, cap, s->layers, true);
+    size_t off = w.at.end;
+    const size_t R = (size_t)s->batch * rows_per_seq(s);
+    w.keep = off;
+    off = align256(off + R * cap * sizeof(int32_t));
+    w.keep_len = off;
+    off = align256(off + R * sizeof(int32_t));
+    w.done = off;
+    off = align256(off + (size_t)s->batch * sizeof(int32_t));
+    w.moves = off;
+    off = align256(off + R * cap * 2 * sizeof(int32_t));
+    w.n_moves = off;
+    off = align256(off + R * sizeof(int32_t));
+    w.end = off;
+    return w;
+}
+
+template <typename T>
+T *at(void *ws, size_t off) {
+    return reinterpret_cast<T *>(reinterpret_cast<unsigned char *>(ws) + off);
+}
+
+// split-K partition for lengths up to max_len
+void choose_splits(const ikv_shape *s, int n_layers, int32_t max_len, int32_t *split_tokens, int32_t *n_splits) {
+    const int64_t units = (int64_t)s->batch * n_layers * s->kv_heads;
+    const int64_t want = (int64_t)sm_count() * 4;
+    int64_t splits = (want + units - 1) / units;
+    const int64_t by_len = (max_len + kMinSplitTokens - 1) / kMinSplitTokens;
+    if (splits > by_len) splits = by_len;
+    if (splits > kMaxSplits) splits = kMaxSplits;
+    if (splits < 1) splits = 1;
+    int64_t st = (max_len + splits - 1) / splits;
+    st = (st + kTileTokens - 1) / kTileTokens * kTileTokens;
+    if (st < kTileTokens) st = kTileTokens;
+    *split_tokens = (int32_t)st;
+    int64_t ns = (max_len + st - 1) / st;
+    if (ns < 1) ns = 1;
+    *n_splits = (int32_t)ns;
+}
+
+// attention (+ combine) over layers [layer0, layer0 + n_layers)
+ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, int32_t n_layers, int32_t max_len,
+                      const void *q, void *out, void *ws, const AttendWs &w, bool logits, int32_t *split_out,
+                      int32_t *nsplit_out, cudaStream_t st, const ikv_timing *tm = nullptr) {
+    AttendArgs a{};
+    a.k = c->k;
+    a.v = c->v;
+    a.pv = view_of(s, c);
+    a.len = c->len;
+    a.q = q;
+    a.batch = s->batch;
+    a.q_heads = s->q_heads;
+    a.layer0 = layer0;
+    a.n_layers = n_layers;
+    choose_splits(s, n_layers, max_len, &a.split_tokens, &a.n_splits);
+    a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)s->head_dim));
+    a.logits = logits ? at<float>(ws, w.logits) : nullptr;
+    a.cap = cap_of(c);
+    a.part_ml = at<float>(ws, w.part_ml);
+    a.part_o = at<float>(ws, w.part_o);
+    if (max_len > 0) IKV_TRY_CUDA(launch_attend(a, s->dtype, s->head_dim, s->q_heads / s->kv_heads, st), "attend launch");
+    if (tm && tm->attend_end) IKV_TRY_CUDA(cudaEventRecord(tm->attend_end, st), "cudaEventRecord");
+    CombineArgs cb{};
+    cb.len = c->len;
+    cb.batch = s->batch;
+    cb.q_heads = s->q_heads;
+    cb.n_layers = n_layers;
+    cb.split_tokens = a.split_tokens;
+    cb.n_splits = a.n_splits;
+    cb.head_dim = s->head_dim;
+    cb.part_ml = a.part_ml;
+    cb.part_o = a.part_o;
+    cb.out = out;
+    cb.lse2 = at<float>(ws, w.lse2);
+    IKV_TRY_CUDA(launch_combine(cb, s->dtype, st), "combine launch");
+    if (split_out) *split_out = a.split_tokens;
+    if (nsplit_out) *nsplit_out = a.n_splits;
+    return IKV_OK;
+}
+
+ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, const int32_t *elig, int n_elig,
+                     int32_t max_len, void *ws, const AttendWs &w, float alpha, float *ema, float *score,
+                     cudaStream_t st) {
+    for (int k0 = 0; k0 < n_elig; k0 += kMaxLayersPerScorePass) {
+        ScoreArgs sa{};
+        sa.len = c->len;
+        sa.batch = s->batch;
+        sa.q_heads = s->q_heads;
+        sa.kv_heads = s->kv_heads;
+        sa.rows_per_seq = rows_per_seq(s);
+        sa.n_layers = n_layers;
+        sa.cap = cap_of(c);
+        sa.logits = at<float>(ws, w.logits);
+        sa.lse2 = at<float>(ws, w.lse2);
+        sa.n_elig = n_elig - k0 < kMaxLayersPerScorePass ? n_elig - k0 : kMaxLayersPerScorePass;
+        for (int k = 0; k < sa.n_elig; ++k) sa.elig[k] = elig[k0 + k];
+        sa.alpha = alpha;
+        sa.ema = ema;
+        sa.score = score;
+        IKV_TRY_CUDA(launch_score_ema(sa, max_len, st), "score launch");
+    }
+    return IKV_OK;
+}
+
+ikv_status record(cudaEvent_t e, cudaStream_t st) {
+    if (e) IKV_TRY_CUDA(cudaEventRecord(e, st), "cudaEventRecord");
+    return IKV_OK;
+}
+
+}  // namespace
+}  // namespace ikv
+
+using namespace ikv;
+
+extern "C" {
+
+const char *ikv_last_error(void) { return g_err; }
+
+int64_t ikv_launch_count(void) { return g_launches.load(); }
+
+ikv_status ikv_attend_workspace_size(const ikv_shape *shape, const ikv_cache *cache, size_t *bytes) {
+    g_err[0] = 0;
+    ikv_status e = check_shape(shape);
+    if (e) return e;
+    if ((e = check_cache(shape, cache, false))) return e;
+    if (!bytes) return fail(IKV_ERR_ARG, "bytes is NULL");
+    *bytes = attend_ws(shape, cap_of(cache), 1, true).end;
+    return IKV_OK;
+}
+
+ikv_status ikv_decode_attend_score(const ikv_shape *shape, const ikv_cache *cache, int32_t layer, const void *q,
+                                   void *out, float *score, float *ema, float alpha, void *ws, size_t ws_bytes,
+                                   cudaStream_t stream) {
+    g_err[0] = 0;
+    ikv_status e = check_shape(shape);
+    if (e) return e;
+    if ((e = check_cache(shape, cache, false))) return e;
+    if (layer < 0 || layer >= shape->layers) return fail(IKV_ERR_ARG, "layer %d out of range", layer);
+    if (!q || !out) return fail(IKV_ERR_ARG, "q/out is NULL");
+    if (!aligned16(q) || !aligned16(out)) return fail(IKV_ERR_ALIGN, "q/out must be 16-byte aligned");
+    if (ema && !(alpha >= 0.f && alpha <= 1.f)) return fail(IKV_ERR_ARG, "alpha must be in [0, 1]");
+    const bool want_score = score || ema;
+    const AttendWs w = attend_ws(shape, cap_of(cache), 1, want_score);
+    if (!ws || ws_bytes < w.end) return fail(IKV_ERR_WORKSPACE, "workspace needs %zu bytes", w.end);
+    if ((e = run_attend(shape, cache, layer, 1, cache->max_len, q, out, ws, w, want_score, nullptr, nullptr, stream)))
+        return e;
+    if (want_score) {
+        const int32_t elig0 = 0;
+        if ((e = run_score(shape, cache, 1, &elig0, 1, cache->max_len, ws, w, ema ? alpha : 0.f, ema, score, stream)))
+            return e;
+    }
+    return IKV_OK;
+}
+
+ikv_status ikv_ema_update(int32_t rows, int32_t cap, float *ema, const float *score, const int32_t *len,
+                          int32_t rows_per_seq_, float alpha, cudaStream_t stream) {
+    g_err[0] = 0;
+    if (rows < 0 || cap < 0 || rows_per_seq_ <= 0) return fail(IKV_ERR_SHAPE, "rows/cap/rows_per_seq out of range");
+    if (rows > 0 && (!ema || !score || !len)) return fail(IKV_ERR_ARG, "ema/score/len is NULL");
+    if (!(alpha >= 0.f && alpha <= 1.f)) return fail(IKV_ERR_ARG, "alpha must be in [0, 1]");
+    IKV_TRY_CUDA(launch_ema_update(rows, cap, ema, score, len, rows_per_seq_, alpha, cap, stream), "ema launch");
+    return IKV_OK;
+}
+
+ikv_status ikv_select_budget(int32_t rows, int32_t cap, const float *util, const int32_t *len, int32_t rows_per_seq_,
+                             const int32_t *budget, int32_t *keep, int32_t *keep_len, cudaStream_t stream) {
+    g_err[0] = 0;
+    if (rows < 0 || cap < 0 || rows_per_seq_ <= 0) return fail(IKV_ERR_SHAPE, "rows/cap/rows_per_seq out of range");
+    if (rows > 0 && (!util || !len || !budget || !keep || !keep_len))
+        return fail(IKV_ERR_ARG, "util/len/budget/keep/keep_len is NULL");
+    IKV_TRY_CUDA(launch_select(rows, cap, util, len, rows_per_seq_, budget, keep, keep_len, stream), "select launch");
+    return IKV_OK;
+}
+
+ikv_status ikv_compact_workspace_size(const ikv_shape *shape, const ikv_cache *cache, int32_t mode, size_t *bytes) {
+    g_err[0] = 0;
+    ikv_status e = check_shape(shape);
+    if (e) return e;
+    if ((e = check_cache(shape, cache, false))) return e;
+    if (!bytes) return fail(IKV_ERR_ARG, "bytes is NULL");
+    if (mode == IKV_COMPACT_STABLE) {
+        *bytes = 0;
+        return IKV_OK;
+    }
+    if (mode != IKV_COMPACT_HOLEFILL) return fail(IKV_ERR_ARG, "unknown compact mode %d", mode);
+    const size_t R = (size_t)shape->batch * rows_per_seq(shape);
+    *bytes = align256(R * cap_of(cache) * 2 * sizeof(int32_t)) + align256(R * sizeof(int32_t));
+    return IKV_OK;
+}
+
+static ikv_status compact_impl(const ikv_shape *shape, ikv_cache *cache, const int32_t *keep, const int32_t *keep_len,
+                               float *ema, int32_t mode, int32_t *moves, int32_t *n_moves, cudaStream_t stream) {
+    CompactArgs a{};
+    a.k = cache->k;
+    a.v = cache->v;
+    a.pv = view_of(shape, cache);
+    a.batch = shape->batch;
+    a.layers = shape->layers;
+    a.rows_per_seq = rows_per_seq(shape);
+    a.cap = cap_of(cache);
+    a.elem_bytes = elem_bytes(shape);
+    a.len = cache->len;
+    a.pos = cache->pos;
+    a.ema = ema;
+    a.keep = keep;
+    a.keep_len = keep_len;
+    a.moves = moves;
+    a.n_moves = n_moves;
+    IKV_TRY_CUDA(launch_compact(a, mode, stream), "compact launch");
+    return IKV_OK;
+}
+
+ikv_status ikv_compact_kv(const ikv_shape *shape, ikv_cache *cache, const int32_t *keep, const int32_t *keep_len,
+                          float *ema, int32_t mode, void *ws, size_t ws_bytes, cudaStream_t stream) {
+    g_err[0] = 0;
+    ikv_status e = check_shape(shape);
+    if (e) return e;
+    if ((e = check_cache(shape, cache, true))) return e;
+    if (!keep || !keep_len) return fail(IKV_ERR_ARG, "keep/keep_len is NULL");
+    size_t need = 0;
+    if ((e = ikv_compact_workspace_size(shape, cache, mode, &need))) return e;
+    int32_t *moves = nullptr, *n_moves = nullptr;
+    if (mode == IKV_COMPACT_HOLEFILL) {
+        if (!ws || ws_bytes < need) return fail(IKV_ERR_WORKSPACE, "workspace needs %zu bytes", need);
+        const size_t R = (size_t)shape->batch * rows_per_seq(shape);
+        moves = at<int32_t>(ws, 0);
+        n_moves = at<int32_t>(ws, align256(R * cap_of(cache) * 2 * sizeof(int32_t)));
+    }
+    return compact_impl(shape, cache, keep, keep_len, ema, mode, moves, n_moves, stream);
+}
+
+static ikv_status append_impl(const ikv_shape *shape, ikv_cache *cache, const void *k_new, const void *v_new,
+                              float *ema, int32_t init_mean, int32_t *done, cudaStream_t stream) {
+    AppendArgs a{};
+    a.k = cache->k;
+    a.v = cache->v;
+    a.pv = view_of(shape, cache);
+    a.batch = shape->batch;
+    a.layers = shape->layers;
+    a.rows_per_seq = rows_per_seq(shape);
+    a.cap = cap_of(cache);
+    a.elem_bytes = elem_bytes(shape);
+    a.k_new = k_new;
+    a.v_new = v_new;
+    a.len = cache->len;
+    a.pos = cache->pos;
+    a.next_pos = cache->next_pos;
+    a.ema = ema;
+    a.init_mean = ema ? init_mean : 0;
+    a.done = done;
+    IKV_TRY_CUDA(cudaMemsetAsync(done, 0, sizeof(int32_t) * shape->batch, stream), "cudaMemsetAsync");
+    IKV_TRY_CUDA(launch_append(a, stream), "append launch");
+    return IKV_OK;
+}
+
+ikv_status ikv_append_token(const ikv_shape *shape, ikv_cache *cache, const void *k_new, const void *v_new,
+                            float *ema, int32_t init_mean, void *ws, size_t ws_bytes, cudaStream_t stream) {
+    g_err[0] = 0;
+    ikv_status e = check_shape(shape);
+    if (e) return e;
+    if ((e = check_cache(shape, cache, true))) return e;
+    if (!k_new || !v_new) return fail(IKV_ERR_ARG, "k_new/v_new is NULL");
+    if (!aligned16(k_new) || !aligned16(v_new)) return fail(IKV_ERR_ALIGN, "k_new/v_new must be 16-byte aligned");
+    if (cache->max_len + 1 > cap_of(cache)) return fail(IKV_ERR_SHAPE, "no free slot: max_len + 1 > cap");
+    const size_t need = align256((size_t)shape->batch * sizeof(int32_t));
+    if (!ws || ws_bytes < need) return fail(IKV_ERR_WORKSPACE, "workspace needs %zu bytes", need);
+    return append_impl(shape, cache, k_new, v_new, ema, init_mean, at<int32_t>(ws, 0), stream);
+}
+
+ikv_status ikv_step_workspace_size(const ikv_shape *shape, const ikv_cache *cache, size_t *bytes) {
+    g_err[0] = 0;
+    ikv_status e = check_shape(shape);
+    if (e) return e;
+    if ((e = check_cache(shape, cache, false))) return e;
+    if (!bytes) return fail(IKV_ERR_ARG, "bytes is NULL");
+    *bytes = step_ws(shape, cap_of(cache)).end;
+    return IKV_OK;
+}
+
+ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, int32_t t,
+                    const void *q, const void *k_new, const void *v_new, void *out, void *ws, size_t ws_bytes,
+                    cudaStream_t stream) {
+    g_err[0] = 0;
+    ikv_status e = check_shape(shape);
+    if (e) return e;
+    if ((e = check_cache(shape, cache, true))) return e;
+    if (!p) return fail(IKV_ERR_ARG, "params is NULL");
+    if (!ema || !q || !k_new || !v_new || !out || !p->budget) return fail(IKV_ERR_ARG, "ema/q/k_new/v_new/out/budget is NULL");
+    if (!aligned16(q) || !aligned16(out) || !aligned16(k_new) || !aligned16(v_new))
+        return fail(IKV_ERR_ALIGN, "q/out/k_new/v_new must be 16-byte aligned");
+    if (t < 1) return fail(IKV_ERR_ARG, "t is 1-based (got %d)", t);
+    if (!(p->alpha >= 0.f && p->alpha <= 1.f)) return fail(IKV_ERR_ARG, "alpha must be in [0, 1]");
+    if (p->refresh_period < 1) return fail(IKV_ERR_ARG, "refresh_period must be >= 1");
+    if (p->compact_mode != IKV_COMPACT_STABLE && p->compact_mode != IKV_COMPACT_HOLEFILL)
+        return fail(IKV_ERR_ARG, "unknown compact mode %d", p->compact_mode);
+    if (p->refresh_init != IKV_INIT_ZERO && p->refresh_init != IKV_INIT_MEAN)
+        return fail(IKV_ERR_ARG, "unknown refresh_init %d", p->refresh_init);
+    const int32_t cap = cap_of(cache);
+    if (cache->max_len + 1 > cap) return fail(IKV_ERR_SHAPE, "no free slot: max_len + 1 > cap");
+    const StepWs w = step_ws(shape, cap);
+    if (!ws || ws_bytes < w.end) return fail(IKV_ERR_WORKSPACE, "workspace needs %zu bytes", w.end);
+
+    const bool refresh = p->score_free ? (t == 1) : ((t - 1) % p->refresh_period == 0);
+    int32_t elig[kMaxLayers];
+    int n_elig = 0;
+    for (int l = 0; l < shape->layers; ++l)
+        if (!p->layer_eligible || p->layer_eligible[l]) elig[n_elig++] = l;
+    const bool scoring = refresh && n_elig > 0;
+    const int32_t L1 = cache->max_len + 1;
+    const ikv_timing *tm = p->timing;
+
+    if (tm && (e = record(tm->begin, stream))) return e;
+    const int32_t init_mean = refresh ? (p->refresh_init == IKV_INIT_MEAN) : 1;
+    if ((e = append_impl(shape, cache, k_new, v_new, ema, init_mean, at<int32_t>(ws, w.done), stream))) return e;
+    if (tm && (e = record(tm->append_end, stream))) return e;
+    if ((e = run_attend(shape, cache, 0, shape->layers, L1, q, out, ws, w.at, scoring, nullptr, nullptr, stream, tm)))
+        return e;
+    if (tm && (e = record(tm->combine_end, stream))) return e;
+    if (scoring && (e = run_score(shape, cache, shape->layers, elig, n_elig, L1, ws, w.at, p->alpha, ema, nullptr, stream)))
+        return e;
+    if (tm && (e = record(tm->score_end, stream))) return e;
+    const int32_t R = shape->batch * rows_per_seq(shape);
+    IKV_TRY_CUDA(launch_select(R, cap, ema, cache->len, rows_per_seq(shape), p->budget, at<int32_t>(ws, w.keep),
+                               at<int32_t>(ws, w.keep_len), stream),
+                 "select launch");
+    if (tm && (e = record(tm->select_end, stream))) return e;
+    if ((e = compact_impl(shape, cache, at<int32_t>(ws, w.keep), at<int32_t>(ws, w.keep_len), ema, p->compact_mode,
+                          at<int32_t>(ws, w.moves), at<int32_t>(ws, w.n_moves), stream)))
+        return e;
+    if (tm && (e = record(tm->end, stream))) return e;
+    return IKV_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,309 @@
+// In-place gather compaction of the paged K/V after eviction, and the append
+// of each step's new token.
+//
+// Stable mode: slot j <- slot keep[j] for j < n, keep ascending, so keep[j] >= j
+// and once keep[j] != j every later slot moves too: only the suffix from the
+// first moved slot j* is touched.  One CTA per (sequence, layer, kv head) walks
+// that suffix in ascending 32-row tiles through a 4-stage cp.async ring.  A
+// tile's sources are >= its first destination, and every earlier tile's
+// destinations lie below that, so reading ahead of the writes is safe; within
+// a tile all reads land (wait + barrier) before any write.  Extra CTAs per row
+// move the utility and position arrays the same way and set len = n.
+//
+// Hole-fill mode: survivors at slots >= n move into the evicted slots below n
+// (k-th hole <- k-th such survivor).  Sources and destinations are disjoint,
+// so every move is independent; the move list is built per row first.
+#include "ikv_internal.cuh"
+
+namespace ikv {
+namespace {
+
+constexpr int kCompThreads = 256;
+constexpr int kCompRows = 32;
+constexpr int kCompStages = 4;
+
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem) {
+    const uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+__device__ __forceinline__ int block_min_int(int v, int *scratch) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(0xffffffffu, v, o));
+    if ((threadIdx.x & 31) == 0) scratch[threadIdx.x >> 5] = v;
+    __syncthreads();
+    int r = scratch[0];
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) r = min(r, scratch[w]);
+    __syncthreads();
+    return r;
+}
+
+__device__ __forceinline__ float block_sum(float v, float *scratch) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if ((threadIdx.x & 31) == 0) scratch[threadIdx.x >> 5] = v;
+    __syncthreads();
+    float r = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) r += scratch[w];
+    __syncthreads();
+    return r;
+}
+
+__global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const CompactArgs a) {
+    extern __shared__ __align__(16) unsigned char cbuf[];
+    __shared__ int scratch[32];
+    const int tid = threadIdx.x;
+    const int b = blockIdx.y, x = blockIdx.x;
+    const int kvh = a.pv.kv_heads;
+    const int nkv = a.layers * kvh;
+    if (x < nkv) {
+        const int l = x / kvh, g = x % kvh;
+        const int r = b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g);
+        const int n = a.keep_len[r];
+        const int32_t *kp = a.keep + (int64_t)r * a.cap;
+        int first = n;
+        for (int j = tid; j < n; j += kCompThreads)
+            if (kp[j] != j) first = min(first, j);
+        const int jstar = block_min_int(first, scratch);
+        if (jstar >= n) return;
+        const int rowB = a.pv.head_dim * a.elem_bytes;
+        const int CPR = rowB >> 4;
+        const int stageB = 2 * kCompRows * rowB;
+        const int n_tiles = (n - jstar + kCompRows - 1) / kCompRows;
+        unsigned char *kb = reinterpret_cast<unsigned char *>(a.k);
+        unsigned char *vb = reinterpret_cast<unsigned char *>(a.v);
+        auto issue = [&](int tile) {
+            unsigned char *st = cbuf + (tile % kCompStages) * stageB;
+            for (int idx = tid; idx < kCompRows * CPR; idx += kCompThreads) {
+                const int jj = idx / CPR, c = idx % CPR;
+                const int j = jstar + tile * kCompRows + jj;
+                if (j < n) {
+                    const int64_t src = a.pv.row(b, l, g, kp[j]);
+                    cp_async16(st + jj * rowB + c * 16, kb + src * rowB + c * 16);
+                    cp_async16(st + (kCompRows + jj) * rowB + c * 16, vb + src * rowB + c * 16);
+                }
+            }
+        };
+#pragma unroll
+        for (int i = 0; i < kCompStages - 1; ++i) {
+            if (i < n_tiles) issue(i);
+            cp_async_commit();
+        }
+        for (int tile = 0; tile < n_tiles; ++tile) {
+            __syncthreads();  // the stage about to be refilled was written out last iteration
+            if (tile + kCompStages - 1 < n_tiles) issue(tile + kCompStages - 1);
+            cp_async_commit();
+            cp_async_wait<kCompStages - 1>();
+            __syncthreads();  // every read of this tile has landed before any write
+            const unsigned char *st = cbuf + (tile % kCompStages) * stageB;
+            for (int idx = tid; idx < kCompRows * CPR; idx += kCompThreads) {
+                const int jj = idx / CPR, c = idx % CPR;
+                const int j = jstar + tile * kCompRows + jj;
+                if (j < n) {
+                    const int64_t dst = a.pv.row(b, l, g, j);
+                    *reinterpret_cast<uint4 *>(kb + dst * rowB + c * 16) =
+                        *reinterpret_cast<const uint4 *>(st + jj * rowB + c * 16);
+                    *reinterpret_cast<uint4 *>(vb + dst * rowB + c * 16) =
+                        *reinterpret_cast<const uint4 *>(st + (kCompRows + jj) * rowB + c * 16);
+                }
+            }
+        }
+        cp_async_wait<0>();
+        return;
+    }
+    // utility / position rows
+    const int rr = x - nkv;
+    const int r = b * a.rows_per_seq + rr;
+    const int n = a.keep_len[r];
+    const int32_t *kp = a.keep + (int64_t)r * a.cap;
+    int32_t *pos = a.pos + (int64_t)r * a.cap;
+    float *ema = a.ema ? a.ema + (int64_t)r * a.cap : nullptr;
+    constexpr int PER = 16;
+    for (int base = 0; base < n; base += kCompThreads * PER) {
+        int32_t pv[PER];
+        float ev[PER];
+        int src[PER];
+#pragma unroll
+        for (int u = 0; u < PER; ++u) {
+            const int j = base + u * kCompThreads + tid;
+            src[u] = j < n ? kp[j] : j;
+            if (j < n && src[u] != j) {
+                pv[u] = pos[src[u]];
+                ev[u] = ema ? ema[src[u]] : 0.f;
+            }
+        }
+        __syncthreads();
+#pragma unroll
+        for (int u = 0; u < PER; ++u) {
+            const int j = base + u * kCompThreads + tid;
+            if (j < n && src[u] != j) {
+                pos[j] = pv[u];
+                if (ema) ema[j] = ev[u];
+            }
+        }
+        __syncthreads();
+    }
+    if (rr == 0 && tid == 0) a.len[b] = n;
+}
+
+// Hole-fill move list of one row: for every evicted slot h < n (the k-th such),
+// move the k-th survivor found at a slot >= n into it.
+__global__ void holefill_plan_kernel(const CompactArgs a) {
+    const int r = blockIdx.x;
+    const int n = a.keep_len[r];
+    const int32_t *kp = a.keep + (int64_t)r * a.cap;
+    // survivors below n: lower_bound(kp, n)
+    int lo = 0, hi = n;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (kp[mid] < n) lo = mid + 1; else hi = mid;
+    }
+    const int below = lo;
+    const int n_tail = n - below;
+    int32_t *mv = a.moves + (int64_t)r * a.cap * 2;
+    for (int h = threadIdx.x; h < n; h += blockDim.x) {
+        int l2 = 0, h2 = below;  // entries < h among kp[0..below)
+        while (l2 < h2) {
+            const int mid = (l2 + h2) >> 1;
+            if (kp[mid] < h) l2 = mid + 1; else h2 = mid;
+        }
+        const bool kept = l2 < below && kp[l2] == h;
+        if (!kept) {
+            const int hole = h - l2;
+            mv[2 * hole] = kp[below + hole];
+            mv[2 * hole + 1] = h;
+        }
+    }
+    if (threadIdx.x == 0) a.n_moves[r] = n_tail;
+}
+
+__global__ void __launch_bounds__(kCompThreads) holefill_move_kernel(const CompactArgs a) {
+    const int tid = threadIdx.x;
+    const int b = blockIdx.y, x = blockIdx.x;
+    const int kvh = a.pv.kv_heads;
+    const int nkv = a.layers * kvh;
+    if (x < nkv) {
+        const int l = x / kvh, g = x % kvh;
+        const int r = b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g);
+        const int nm = a.n_moves[r];
+        const int32_t *mv = a.moves + (int64_t)r * a.cap * 2;
+        const int rowB = a.pv.head_dim * a.elem_bytes;
+        const int CPR = rowB >> 4;
+        unsigned char *kb = reinterpret_cast<unsigned char *>(a.k);
+        unsigned char *vb = reinterpret_cast<unsigned char *>(a.v);
+        for (int idx = tid; idx < nm * CPR; idx += kCompThreads) {
+            const int m = idx / CPR, c = idx % CPR;
+            const int64_t src = a.pv.row(b, l, g, mv[2 * m]);
+            const int64_t dst = a.pv.row(b, l, g, mv[2 * m + 1]);
+            *reinterpret_cast<uint4 *>(kb + dst * rowB + c * 16) = *reinterpret_cast<const uint4 *>(kb + src * rowB + c * 16);
+            *reinterpret_cast<uint4 *>(vb + dst * rowB + c * 16) = *reinterpret_cast<const uint4 *>(vb + src * rowB + c * 16);
+        }
+        return;
+    }
+    const int rr = x - nkv;
+    const int r = b * a.rows_per_seq + rr;
+    const int nm = a.n_moves[r];
+    const int32_t *mv = a.moves + (int64_t)r * a.cap * 2;
+    int32_t *pos = a.pos + (int64_t)r * a.cap;
+    float *ema = a.ema ? a.ema + (int64_t)r * a.cap : nullptr;
+    for (int m = tid; m < nm; m += kCompThreads) {
+        const int s = mv[2 * m], d = mv[2 * m + 1];
+        pos[d] = pos[s];
+        if (ema) ema[d] = ema[s];
+    }
+    if (rr == 0 && tid == 0) a.len[b] = a.keep_len[r];
+}
+
+// New token of every sequence into slot len[b] of every layer and kv head.
+// CTAs (x, b) copy 8 rows each; CTA 0 also sets the row utilities / positions;
+// the last CTA of sequence b to arrive advances len[b] and next_pos[b] (every
+// CTA reads len[b] before it arrives, so nobody sees the new value early).
+constexpr int kAppendRows = 8;
+
+__global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a) {
+    __shared__ float scratch[32];
+    const int tid = threadIdx.x;
+    const int b = blockIdx.y;
+    const int L = a.len[b];
+    const int kvh = a.pv.kv_heads;
+    const int nkv = a.layers * kvh;
+    const int rowB = a.pv.head_dim * a.elem_bytes;
+    const int CPR = rowB >> 4;
+    if (L < a.cap) {
+        unsigned char *kb = reinterpret_cast<unsigned char *>(a.k);
+        unsigned char *vb = reinterpret_cast<unsigned char *>(a.v);
+        const unsigned char *kn = reinterpret_cast<const unsigned char *>(a.k_new);
+        const unsigned char *vn = reinterpret_cast<const unsigned char *>(a.v_new);
+        for (int idx = tid; idx < kAppendRows * CPR; idx += kCompThreads) {
+            const int x = blockIdx.x * kAppendRows + idx / CPR, c = idx % CPR;
+            if (x < nkv) {
+                const int l = x / kvh, g = x % kvh;
+                const int64_t src = (((int64_t)l * a.batch + b) * kvh + g) * rowB + c * 16;
+                const int64_t dst = a.pv.row(b, l, g, L) * rowB + c * 16;
+                *reinterpret_cast<uint4 *>(kb + dst) = *reinterpret_cast<const uint4 *>(kn + src);
+                *reinterpret_cast<uint4 *>(vb + dst) = *reinterpret_cast<const uint4 *>(vn + src);
+            }
+        }
+        if (blockIdx.x == 0) {
+            const int np = a.next_pos[b];
+            for (int rr = 0; rr < a.rows_per_seq; ++rr) {
+                const int64_t r = (int64_t)b * a.rows_per_seq + rr;
+                float init = 0.f;
+                if (a.init_mean && L > 0) {
+                    float s = 0.f;
+                    for (int i = tid; i < L; i += kCompThreads) s += a.ema[r * a.cap + i];
+                    init = block_sum(s, scratch) / (float)L;
+                }
+                if (tid == 0) {
+                    if (a.ema) a.ema[r * a.cap + L] = init;
+                    a.pos[r * a.cap + L] = np;
+                }
+            }
+        }
+    }
+    __syncthreads();
+    if (tid == 0) {
+        __threadfence();
+        const int prev = atomicAdd(&a.done[b], 1);
+        if (prev == (int)gridDim.x - 1) {
+            __threadfence();
+            if (L < a.cap) {
+                a.len[b] = L + 1;
+                a.next_pos[b] = a.next_pos[b] + 1;
+            }
+            a.done[b] = 0;
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_compact(const CompactArgs &a, int mode, cudaStream_t st) {
+    dim3 grid(a.layers * a.pv.kv_heads + a.rows_per_seq, a.batch);
+    if (mode == IKV_COMPACT_STABLE) {
+        const int smem = kCompStages * 2 * kCompRows * a.pv.head_dim * a.elem_bytes;
+        cudaError_t e = cudaFuncSetAttribute(compact_stable_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess) return e;
+        compact_stable_kernel<<<grid, kCompThreads, smem, st>>>(a);
+        note_launch();
+        return cudaGetLastError();
+    }
+    holefill_plan_kernel<<<a.batch * a.rows_per_seq, 256, 0, st>>>(a);
+    note_launch();
+    holefill_move_kernel<<<grid, kCompThreads, 0, st>>>(a);
+    note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_append(const AppendArgs &a, cudaStream_t st) {
+    const int nkv = a.layers * a.pv.kv_heads;
+    dim3 grid((nkv + kAppendRows - 1) / kAppendRows, a.batch);
+    append_kernel<<<grid, kCompThreads, 0, st>>>(a);
+    note_launch();
+    return cudaGetLastError();
+}
+
+}  // namespace ikv

@@ -1,0 +1,100 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "ikv.h"
+
+namespace ikv {
+
+constexpr int kTileTokens = 64;    // K/V rows staged per attention tile
+constexpr int kAttendThreads = 128;
+constexpr int kMaxSplits = 64;     // split-K partitions per (seq, layer, kv head)
+constexpr int kMinSplitTokens = 256;
+constexpr int kMaxLayersPerScorePass = 32;
+constexpr int kMaxLayers = 512;
+
+// Launch-count bookkeeping (host).
+void note_launch(int n = 1);
+
+// Where a (sequence, slot) row of layer l / kv head g lives in the paged pool.
+struct PagedView {
+    const int32_t *block_table;
+    int32_t num_pages, page_size, max_pages, kv_heads, head_dim;
+    __device__ __forceinline__ int64_t row(int32_t b, int32_t l, int32_t g, int32_t slot) const {
+        const int32_t page = block_table[(int64_t)b * max_pages + slot / page_size];
+        return (((int64_t)l * num_pages + page) * kv_heads + g) * page_size + slot % page_size;
+    }
+};
+
+struct AttendArgs {
+    const void *k, *v;          // pools
+    PagedView pv;
+    const int32_t *len;         // [batch]
+    const void *q;              // q for layer layer0: element (li, b, h, e) at q + ((li*batch + b)*H + h)*D + e
+    int32_t batch, q_heads, layer0, n_layers;
+    int32_t split_tokens, n_splits;
+    float scale_log2;           // log2(e) / sqrt(d)
+    float *logits;              // [batch][n_layers][H][cap] log2-domain logits, or null
+    int32_t cap;
+    float *part_ml;             // [batch][n_layers][H][n_splits][2]  (running max, sum) in log2 domain
+    float *part_o;              // [batch][n_layers][H][n_splits][D]  unnormalised partial output
+};
+
+struct CombineArgs {
+    const int32_t *len;
+    int32_t batch, q_heads, n_layers, split_tokens, n_splits, head_dim;
+    const float *part_ml, *part_o;
+    void *out;                  // [n_layers][batch][H][D] (dtype)
+    float *lse2;                // [batch][n_layers][H] log2-sum-exp, or null
+};
+
+struct ScoreArgs {
+    const int32_t *len;         // [batch]
+    int32_t batch, q_heads, kv_heads, rows_per_seq, n_layers, cap;
+    const float *logits;        // [batch][n_layers][H][cap]
+    const float *lse2;          // [batch][n_layers][H]
+    int32_t n_elig;             // eligible local layers, in ascending order
+    const int32_t *elig_dev;    // unused placeholder
+    float alpha;
+    float *ema;                 // [rows][cap] or null
+    float *score;               // [rows][cap] or null (only meaningful with one layer)
+    int32_t elig[kMaxLayersPerScorePass];
+};
+
+// launchers (return cudaError_t of the launch)
+cudaError_t launch_attend(const AttendArgs &a, int dtype, int head_dim, int group, cudaStream_t st);
+cudaError_t launch_combine(const CombineArgs &a, int dtype, cudaStream_t st);
+cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, cudaStream_t st);
+cudaError_t launch_ema_update(int32_t rows, int32_t cap, float *ema, const float *score, const int32_t *len,
+                              int32_t rows_per_seq, float alpha, int32_t max_len, cudaStream_t st);
+cudaError_t launch_select(int32_t rows, int32_t cap, const float *util, const int32_t *len, int32_t rows_per_seq,
+                          const int32_t *budget, int32_t *keep, int32_t *keep_len, cudaStream_t st);
+
+struct CompactArgs {
+    void *k, *v;
+    PagedView pv;
+    int32_t batch, layers, rows_per_seq, cap, elem_bytes;
+    int32_t *len, *pos;
+    float *ema;
+    const int32_t *keep, *keep_len;
+    int32_t *moves;             // hole-fill: [rows][cap][2] (src, dst), null for stable
+    int32_t *n_moves;           // hole-fill: [rows]
+};
+cudaError_t launch_compact(const CompactArgs &a, int mode, cudaStream_t st);
+
+struct AppendArgs {
+    void *k, *v;
+    PagedView pv;
+    int32_t batch, layers, rows_per_seq, cap, elem_bytes;
+    const void *k_new, *v_new;  // [layers][batch][kv_heads][D]
+    int32_t *len, *pos, *next_pos;
+    float *ema;
+    int32_t init_mean;
+    int32_t *done;              // [batch] arrival counters, zero on entry; reset by the last CTA
+};
+cudaError_t launch_append(const AppendArgs &a, cudaStream_t st);
+
+}  // namespace ikv

@@ -1,0 +1,190 @@
+// Budgeted selection: keep the B highest utilities of a row (Sec. 3: evict the
+// lowest m whenever the cache exceeds B).
+//
+// One 1024-thread CTA per utility row.  Utilities map to order-preserving
+// 32-bit keys (sign-flipped IEEE bits; -0.0 folded onto +0.0; NaN -> 0, the
+// lowest key).  General case: an MSB-first radix select with 8-bit digits
+// (four passes, warp-aggregated shared-memory histograms) finds the exact B-th
+// largest key theta and how many theta-valued slots survive; one more pass
+// writes the kept slots in ascending order (two block scans per 1024-slot
+// chunk), keeping the lowest slots among keys equal to theta.  Steady-state
+// case L == B + 1: a single pass finds the one slot to evict (lowest key, and
+// among equal keys the highest slot).  The result depends only on the fp32
+// values, so it is bit-exact against any correct sort.
+#include "ikv_internal.cuh"
+
+namespace ikv {
+namespace {
+
+constexpr int kSelThreads = 1024;
+
+__device__ __forceinline__ uint32_t ord_key(float f) {
+    uint32_t u = __float_as_uint(f);
+    if ((u & 0x7FFFFFFFu) > 0x7F800000u) return 0u;  // NaN: lowest
+    if ((u & 0x7FFFFFFFu) == 0u) u = 0u;              // -0.0 == +0.0
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// exclusive scan of one value per thread across the block; returns (exclusive, total)
+__device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t *warp_tot, uint32_t &total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    uint32_t x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) warp_tot[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+        uint32_t t = warp_tot[lane];
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_up_sync(0xffffffffu, t, o);
+            if (lane >= o) t += y;
+        }
+        warp_tot[lane] = t;  // inclusive over warps
+    }
+    __syncthreads();
+    const uint32_t before = warp == 0 ? 0u : warp_tot[warp - 1];
+    total = warp_tot[31];
+    __syncthreads();
+    return before + x - v;
+}
+
+__global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const float *__restrict__ util,
+                                                              const int32_t *__restrict__ len, int32_t rps,
+                                                              const int32_t *__restrict__ budget, int32_t *keep,
+                                                              int32_t *keep_len) {
+    __shared__ uint32_t hist[256];
+    __shared__ uint32_t warp_tot[32];
+    __shared__ unsigned long long s_min[32];
+    __shared__ uint32_t s_digit, s_above;
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int r = blockIdx.x;
+    const int L = len[r / rps];
+    int B = budget[r / rps];
+    if (B < 0) B = 0;
+    const float *u = util + (int64_t)r * cap;
+    int32_t *kp = keep + (int64_t)r * cap;
+
+    if (L <= B) {
+        for (int j = tid; j < L; j += kSelThreads) kp[j] = j;
+        if (tid == 0) keep_len[r] = L;
+        return;
+    }
+    if (B == 0) {
+        if (tid == 0) keep_len[r] = 0;
+        return;
+    }
+
+    if (L == B + 1) {
+        // evict exactly one: minimum of (key, ~slot)
+        unsigned long long best = ~0ull;
+        for (int i = tid; i < L; i += kSelThreads) {
+            const unsigned long long v = ((unsigned long long)ord_key(u[i]) << 32) | (uint32_t)(~(uint32_t)i);
+            best = v < best ? v : best;
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const unsigned long long y = __shfl_xor_sync(0xffffffffu, best, o);
+            best = y < best ? y : best;
+        }
+        if (lane == 0) s_min[warp] = best;
+        __syncthreads();
+        if (warp == 0) {
+            best = s_min[lane];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                const unsigned long long y = __shfl_xor_sync(0xffffffffu, best, o);
+                best = y < best ? y : best;
+            }
+            if (lane == 0) s_min[0] = best;
+        }
+        __syncthreads();
+        const int ev = (int)(~(uint32_t)(s_min[0] & 0xFFFFFFFFull));
+        for (int j = tid; j < B; j += kSelThreads) kp[j] = j < ev ? j : j + 1;
+        if (tid == 0) keep_len[r] = B;
+        return;
+    }
+
+    uint32_t prefix = 0u, mask = 0u, k = (uint32_t)B;
+    for (int pass = 0; pass < 4; ++pass) {
+        const int shift = 24 - 8 * pass;
+        for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0u;
+        __syncthreads();
+        for (int base = 0; base < L; base += kSelThreads) {
+            const int i = base + tid;
+            uint32_t digit = 0xFFFFu;
+            if (i < L) {
+                const uint32_t key = ord_key(u[i]);
+                if ((key & mask) == prefix) digit = (key >> shift) & 0xFFu;
+            }
+            const uint32_t peers = __match_any_sync(0xffffffffu, digit);
+            if (digit != 0xFFFFu && lane == __ffs(peers) - 1) atomicAdd(&hist[digit], (uint32_t)__popc(peers));
+        }
+        __syncthreads();
+        // inclusive counts from the top digit down: thread t < 256 holds digit 255 - t
+        uint32_t v = 0u, x = 0u;
+        if (tid < 256) {
+            v = hist[255 - tid];
+            x = v;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+                if (lane >= o) x += y;
+            }
+            if (lane == 31) warp_tot[warp] = x;
+        }
+        __syncthreads();
+        if (tid < 256) {
+            uint32_t before = 0u;
+            for (int w = 0; w < warp; ++w) before += warp_tot[w];
+            const uint32_t incl = before + x;
+            const uint32_t above = incl - v;
+            if (above < k && incl >= k) {  // exactly one digit satisfies this
+                s_digit = 255u - (uint32_t)tid;
+                s_above = above;
+            }
+        }
+        __syncthreads();
+        const uint32_t dsel = s_digit;
+        k -= s_above;
+        prefix |= dsel << shift;
+        mask |= 0xFFu << shift;
+        __syncthreads();
+    }
+    const uint32_t theta = prefix;
+    const uint32_t need_eq = k;  // theta-valued slots that survive (lowest slots first)
+
+    uint32_t run_eq = 0u, run_keep = 0u;
+    for (int base = 0; base < L; base += kSelThreads) {
+        const int i = base + tid;
+        uint32_t key = 0u;
+        bool in = i < L;
+        if (in) key = ord_key(u[i]);
+        const uint32_t gt = (in && key > theta) ? 1u : 0u;
+        const uint32_t eq = (in && key == theta) ? 1u : 0u;
+        uint32_t eq_tot, kp_tot;
+        const uint32_t eq_rank = block_excl_scan(eq, warp_tot, eq_tot);
+        const uint32_t kf = (gt || (eq && run_eq + eq_rank < need_eq)) ? 1u : 0u;
+        const uint32_t at = block_excl_scan(kf, warp_tot, kp_tot);
+        if (kf) kp[run_keep + at] = i;
+        run_eq += eq_tot;
+        run_keep += kp_tot;
+    }
+    if (tid == 0) keep_len[r] = B;
+}
+
+}  // namespace
+
+cudaError_t launch_select(int32_t rows, int32_t cap, const float *util, const int32_t *len, int32_t rows_per_seq,
+                          const int32_t *budget, int32_t *keep, int32_t *keep_len, cudaStream_t st) {
+    if (rows <= 0) return cudaSuccess;
+    select_kernel<<<rows, kSelThreads, 0, st>>>(cap, util, len, rows_per_seq, budget, keep, keep_len);
+    note_launch();
+    return cudaGetLastError();
+}
+
+}  // namespace ikv

@@ -1,0 +1,184 @@
+"""Shared test plumbing: build a device cache from a workload, mirror it in the
+oracle, and step both in lock-step.
+
+Inputs come only from ``gen`` (host draws uploaded, or the device generator
+whose bits are tested equal to the host's).  Expected values come only from
+``oracle``.  After each step the oracle adopts the GPU's kept set when that set
+is valid under the boundary rule (every token above theta + gap kept, every
+token below theta - gap evicted), so legal near-tie choices cannot make the
+trajectories diverge.
+"""
+from __future__ import annotations
+
+import ctypes
+from dataclasses import dataclass, field
+from typing import List, Optional
+
+import numpy as np
+import torch
+
+import gen
+import oracle as O
+from paper_2609_03515_gb300 import DecodeCache, ikv
+
+GAP = 1e-4          # retained-set boundary rule
+TOL_M = 1e-3        # utilities, fp32 vs fp64
+TOL_OUT_BF16 = 2e-2
+TOL_OUT_F32 = 1e-4
+
+
+def torch_dtype(w: gen.Workload):
+    return torch.bfloat16 if w.dtype == gen.BF16 else torch.float32
+
+
+def make_cache(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, page_perm_seed: Optional[int] = 7,
+               extra_cap: int = 0) -> DecodeCache:
+    c = DecodeCache(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.cap + extra_cap,
+                    dtype=ikv.IKV_BF16 if w.dtype == gen.BF16 else ikv.IKV_F32, page_size=w.page_size,
+                    granularity=gran, page_perm_seed=page_perm_seed)
+    c.set_prefill(w.prefill, w.budgets())
+    return c
+
+
+def fill_host(c: DecodeCache, w: gen.Workload, u: np.ndarray):
+    """Upload host-generated prefill K/V; returns them as [b][l] -> (K[g], V[g]) float64 lists."""
+    kv = []
+    for b in range(w.batch):
+        per_l = []
+        for l in range(w.layers):
+            k, v = w.kv_block(b, l, 0, w.prefill[b], u)
+            for g in range(w.kv_heads):
+                c.scatter(c.k, b, l, g, torch.from_numpy(k[g]).cuda())
+                c.scatter(c.v, b, l, g, torch.from_numpy(v[g]).cuda())
+            per_l.append((k.astype(np.float64), v.astype(np.float64)))
+        kv.append(per_l)
+    return kv
+
+
+def fill_device(c: DecodeCache, w: gen.Workload, u_dev: torch.Tensor) -> None:
+    sp = w.spec()
+    L0 = torch.tensor(w.prefill, dtype=torch.int32, device="cuda")
+    st = torch.cuda.current_stream().cuda_stream
+    rc = gen.cuda_lib().ikvgen_fill_paged_cuda(ctypes.byref(sp), u_dev.data_ptr(), c.k.data_ptr(), c.v.data_ptr(),
+                                               c.block_table.data_ptr(), L0.data_ptr(), c.num_pages, c.page_size,
+                                               c.max_pages, max(w.prefill), w.dtype, st)
+    assert rc == 0, rc
+
+
+def oracle_states(w: gen.Workload, kv, gran: int) -> List[O.SeqState]:
+    sts = []
+    for b in range(w.batch):
+        K = [[kv[b][l][0][g] for g in range(w.kv_heads)] for l in range(w.layers)]
+        V = [[kv[b][l][1][g] for g in range(w.kv_heads)] for l in range(w.layers)]
+        sts.append(O.prefill_state(K, V, w.budgets()[b], O.GRAN_SEQ if gran == ikv.IKV_GRAN_SEQ else O.GRAN_KVHEAD))
+    return sts
+
+
+def as_f64(x: np.ndarray, w: gen.Workload) -> np.ndarray:
+    if w.dtype == gen.BF16:
+        return gen.bf16_to_f32(x).astype(np.float64)
+    return x.astype(np.float64)
+
+
+def to_device(x: np.ndarray, w: gen.Workload) -> torch.Tensor:
+    """Host array (bf16 bits or fp32) -> device tensor of the workload dtype."""
+    if w.dtype == gen.BF16:
+        if x.dtype != np.uint16:
+            x = gen.f32_to_bf16_bits(x)
+        return torch.from_numpy(x.view(np.int16)).cuda().view(torch.bfloat16)
+    return torch.from_numpy(np.ascontiguousarray(x, np.float32)).cuda()
+
+
+def boundary_ok(m_o: np.ndarray, kept_mask: np.ndarray, budget: int, gap: float = GAP):
+    """Retained-set rule against the oracle's utilities m_o (one row)."""
+    L = m_o.shape[0]
+    if L <= budget:
+        return bool(kept_mask.all()), 0.0
+    theta = np.sort(m_o)[::-1][budget - 1]
+    must_keep = m_o > theta + gap
+    must_drop = m_o < theta - gap
+    ok = bool(np.all(kept_mask[must_keep]) and not np.any(kept_mask[must_drop]) and kept_mask.sum() == budget)
+    return ok, float(theta)
+
+
+@dataclass
+class StepReport:
+    t: int
+    out_err: float = 0.0
+    m_err: float = 0.0
+    kv_err: float = 0.0
+    set_ok: bool = True
+    strict_set_equal: bool = True
+    refresh: bool = True
+
+
+def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: int = ikv.IKV_COMPACT_STABLE,
+                 steps: Optional[int] = None, kv_check_layers=(0, -1), page_perm_seed: Optional[int] = 7,
+                 refresh_init: int = ikv.IKV_INIT_ZERO, layer_eligible=None) -> List[StepReport]:
+    T = w.steps if steps is None else steps
+    u = w.u_table()
+    c = make_cache(w, gran, page_perm_seed)
+    kv = fill_host(c, w, u)
+    sts = oracle_states(w, kv, gran)
+    op = O.Params(alpha=w.alpha, refresh_period=w.refresh_period, score_free=w.score_free,
+                  granularity=O.GRAN_SEQ if gran == ikv.IKV_GRAN_SEQ else O.GRAN_KVHEAD,
+                  layer_mask=None if layer_eligible is None else [bool(x) for x in layer_eligible],
+                  refresh_init="zero" if refresh_init == ikv.IKV_INIT_ZERO else "mean")
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, refresh_init, layer_eligible)
+    ws = c.step_workspace()
+    qs = w.queries(1, T + 1, u)
+    budgets = w.budgets()
+    lens = list(w.prefill)
+    out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
+    tol_out = TOL_OUT_BF16 if w.dtype == gen.BF16 else TOL_OUT_F32
+    reports = []
+    R = c.rows_per_seq
+    for t in range(1, T + 1):
+        kn, vn = w.new_tokens(t, u)
+        ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, to_device(qs[t - 1], w), to_device(kn, w),
+                     to_device(vn, w), out, ws, ws.numel())
+        lens = [min(L + 1, B) if L + 1 > B else L + 1 for L, B in zip(lens, budgets)]
+        torch.cuda.synchronize()
+        out_h = out.float().cpu().numpy()
+        ema_h = c.ema.cpu().numpy()
+        pos_h = c.pos.cpu().numpy()
+        len_h = c.len.cpu().numpy()
+        refresh = O.is_refresh(t, w.refresh_period, w.score_free)
+        rep = StepReport(t=t, refresh=refresh)
+        q64 = as_f64(qs[t - 1], w)
+        for b, st in enumerate(sts):
+            O.append_token(st, kn[:, b], vn[:, b], refresh, op)
+            o_out = O.attend_and_score(st, q64[:, b], refresh, op)
+            rep.out_err = max(rep.out_err, float(np.max(np.abs(out_h[:, b] - o_out))))
+            assert len_h[b] == min(st.length, budgets[b]), (t, b, len_h[b], st.length)
+            keeps = []
+            for rr in range(R):
+                r = b * R + rr
+                n = int(len_h[b])
+                gpos = pos_h[r, :n]
+                gm = ema_h[r, :n]
+                slot_of = {int(pp): i for i, pp in enumerate(st.pos[rr])}
+                assert len(set(gpos.tolist())) == n
+                oslots = np.array([slot_of[int(pp)] for pp in gpos])
+                kept_mask = np.zeros(st.length, bool)
+                kept_mask[oslots] = True
+                ok, _ = boundary_ok(st.m[rr], kept_mask, budgets[b])
+                rep.set_ok &= ok
+                own = set(O.select_keep(st.m[rr], budgets[b]).tolist())
+                rep.strict_set_equal &= own == set(oslots.tolist())
+                rep.m_err = max(rep.m_err, float(np.max(np.abs(gm - st.m[rr][oslots]))))
+                keeps.append(np.sort(oslots))
+            O.evict(st, keep_override=keeps)
+            # compacted K/V rows equal the oracle's rows at the same positions
+            for l in kv_check_layers:
+                for g in range(w.kv_heads):
+                    rr = 0 if R == 1 else g
+                    n = int(len_h[b])
+                    gk = c.gather(c.k, b, l % w.layers, g, n).float().cpu().numpy()
+                    gv = c.gather(c.v, b, l % w.layers, g, n).float().cpu().numpy()
+                    order = np.argsort(np.argsort(pos_h[b * R + rr, :n]))  # gpu slot -> rank by position
+                    ok_rows = st.K[l][g][order]
+                    ov_rows = st.V[l][g][order]
+                    rep.kv_err = max(rep.kv_err, float(np.max(np.abs(gk - ok_rows))), float(np.max(np.abs(gv - ov_rows))))
+        reports.append(rep)
+    return reports

@@ -1,0 +1,124 @@
+"""C-ABI checks that need no GPU: the library loads, exports every entry point
+declared in include/*.h, and rejects bad arguments on the host before any launch."""
+import ctypes
+import glob
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_03515_gb300 import build as B
+
+    B.build()
+    from paper_2609_03515_gb300 import ikv
+
+    return ikv
+
+
+def declared_symbols():
+    names = set()
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        src = open(h).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        for m in re.finditer(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\*?\s*(ikv_[a-z0-9_]+)\s*\(", src, re.M):
+            names.add(m.group(1))
+    return sorted(names)
+
+
+def test_header_declares_the_entry_points():
+    names = declared_symbols()
+    for must in ("ikv_decode_attend_score", "ikv_ema_update", "ikv_select_budget", "ikv_compact_kv", "ikv_step"):
+        assert must in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    so = ctypes.CDLL(lib.LIB_PATH)
+    missing = [n for n in declared_symbols() if not hasattr(so, n)]
+    assert not missing, missing
+
+
+def _shape(lib, **kw):
+    d = dict(batch=1, layers=2, q_heads=4, kv_heads=2, head_dim=64, dtype=lib.IKV_F32, granularity=lib.IKV_GRAN_SEQ)
+    d.update(kw)
+    return lib.ikv_shape(**d)
+
+
+def _cache(lib, **kw):
+    d = dict(k=16, v=16, block_table=16, num_pages=4, page_size=64, max_pages=4, len=16, pos=16, next_pos=16,
+             max_len=100)
+    d.update(kw)
+    return lib.ikv_cache(**d)
+
+
+def test_argument_checks_fail_before_launch(lib):
+    n = lib.SZ(0)
+    bad = [
+        (_shape(lib, head_dim=96), _cache(lib), lib.IKV_ERR_UNSUPPORTED),
+        (_shape(lib, q_heads=6, kv_heads=2), _cache(lib), lib.IKV_ERR_UNSUPPORTED),   # group 3
+        (_shape(lib, q_heads=5, kv_heads=2), _cache(lib), lib.IKV_ERR_SHAPE),
+        (_shape(lib, dtype=7), _cache(lib), lib.IKV_ERR_ARG),
+        (_shape(lib), _cache(lib, k=0), lib.IKV_ERR_ARG),
+        (_shape(lib), _cache(lib, k=8), lib.IKV_ERR_ALIGN),
+        (_shape(lib), _cache(lib, max_len=10_000), lib.IKV_ERR_SHAPE),
+        (_shape(lib), _cache(lib, page_size=0), lib.IKV_ERR_SHAPE),
+    ]
+    for shp, cch, want in bad:
+        st = lib.raw_status("ikv_step_workspace_size", ctypes.byref(shp), ctypes.byref(cch), ctypes.byref(n))
+        assert st == want, (st, want, lib.ikv_last_error())
+        assert lib.ikv_last_error() != ""
+    st = lib.raw_status("ikv_step_workspace_size", ctypes.byref(_shape(lib)), ctypes.byref(_cache(lib)),
+                        ctypes.byref(n))
+    assert st == lib.IKV_OK and n.value > 0
+
+
+def test_step_rejects_bad_schedule_and_workspace(lib):
+    shp, cch = _shape(lib), _cache(lib)
+    p = lib.ikv_params()
+    p.alpha, p.refresh_period, p.budget = 0.9, 1, 16
+    args = lambda t, ws, wsb: (ctypes.byref(shp), ctypes.byref(p), ctypes.byref(cch), 16, t, 16, 16, 16, 16, ws, wsb,
+                               None)
+    assert lib.raw_status("ikv_step", *args(0, 16, 1 << 40)) == lib.IKV_ERR_ARG          # t is 1-based
+    assert lib.raw_status("ikv_step", *args(1, 0, 0)) == lib.IKV_ERR_WORKSPACE
+    assert lib.raw_status("ikv_step", *args(1, 16, 10)) == lib.IKV_ERR_WORKSPACE
+    p.refresh_period = 0
+    assert lib.raw_status("ikv_step", *args(1, 16, 1 << 40)) == lib.IKV_ERR_ARG
+    p.refresh_period, p.alpha = 1, 1.5
+    assert lib.raw_status("ikv_step", *args(1, 16, 1 << 40)) == lib.IKV_ERR_ARG
+    p.alpha, p.compact_mode = 0.9, 9
+    assert lib.raw_status("ikv_step", *args(1, 16, 1 << 40)) == lib.IKV_ERR_ARG
+    p.compact_mode = 0
+    full = _cache(lib, max_len=256)  # no free slot for the append
+    assert lib.raw_status("ikv_step", ctypes.byref(shp), ctypes.byref(p), ctypes.byref(full), 16, 1, 16, 16, 16, 16,
+                          16, 1 << 40, None) == lib.IKV_ERR_SHAPE
+
+
+def test_other_entry_points_reject_nulls(lib):
+    assert lib.raw_status("ikv_select_budget", 2, 8, None, 16, 1, 16, 16, 16, None) == lib.IKV_ERR_ARG
+    assert lib.raw_status("ikv_select_budget", -1, 8, 16, 16, 1, 16, 16, 16, None) == lib.IKV_ERR_SHAPE
+    assert lib.raw_status("ikv_ema_update", 2, 8, 16, None, 16, 1, ctypes.c_float(0.5), None) == lib.IKV_ERR_ARG
+    assert lib.raw_status("ikv_ema_update", 2, 8, 16, 16, 16, 1, ctypes.c_float(-0.5), None) == lib.IKV_ERR_ARG
+    shp, cch = _shape(lib), _cache(lib)
+    assert lib.raw_status("ikv_compact_kv", ctypes.byref(shp), ctypes.byref(cch), None, 16, None, 0, None, 0,
+                          None) == lib.IKV_ERR_ARG
+    assert lib.raw_status("ikv_compact_kv", ctypes.byref(shp), ctypes.byref(cch), 16, 16, None, 1, None, 0,
+                          None) == lib.IKV_ERR_WORKSPACE
+    assert lib.raw_status("ikv_decode_attend_score", ctypes.byref(shp), ctypes.byref(cch), 5, 16, 16, None, None,
+                          ctypes.c_float(0.9), 16, 1 << 40, None) == lib.IKV_ERR_ARG   # layer out of range
+    assert lib.raw_status("ikv_decode_attend_score", ctypes.byref(shp), ctypes.byref(cch), 0, 8, 16, None, None,
+                          ctypes.c_float(0.9), 16, 1 << 40, None) == lib.IKV_ERR_ALIGN
+    assert lib.raw_status("ikv_append_token", ctypes.byref(shp), ctypes.byref(cch), 16, 16, None, 0, None, 0,
+                          None) == lib.IKV_ERR_WORKSPACE
+
+
+def test_product_package_does_not_reference_the_oracle():
+    """The CUDA path and its binding never import or link the CPU oracle."""
+    pkg = os.path.join(ROOT, "paper_2609_03515_gb300")
+    for path in glob.glob(os.path.join(pkg, "**", "*.*"), recursive=True):
+        if path.endswith((".py", ".cu", ".cuh", ".h")):
+            src = open(path).read()
+            assert "oracle" not in src.replace("oracle-free", ""), path

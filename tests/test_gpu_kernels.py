@@ -1,0 +1,286 @@
+"""Per-entry-point parity of the CUDA library against the CPU oracle (GPU only).
+
+Inputs: seeded draws from ``gen``.  Expected values: ``oracle`` only.
+Sizes span several 64-token tiles, several split-K partitions and ragged tails.
+"""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+import gen
+import oracle as O
+from harness import as_f64, fill_device, make_cache, to_device
+from paper_2609_03515_gb300 import DecodeCache, ikv
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+
+    __graft_entry__.build()
+
+
+# ------------------------------------------------------------------ generator
+def test_device_generator_matches_host_bits():
+    w = gen.Workload("t", 3, 2, 8, 2, 128, [100, 257, 64], 4, dtype=gen.BF16, seed=11, page_size=32)
+    u = w.u_table()
+    c = make_cache(w, page_perm_seed=3)
+    fill_device(c, w, torch.from_numpy(u).cuda())
+    torch.cuda.synchronize()
+    for b in range(w.batch):
+        for l in range(w.layers):
+            k, v = w.kv_block(b, l, 0, w.prefill[b], u)
+            for g in range(w.kv_heads):
+                gk = c.gather(c.k, b, l, g, w.prefill[b]).float().cpu().numpy()
+                gv = c.gather(c.v, b, l, g, w.prefill[b]).float().cpu().numpy()
+                assert np.array_equal(gk, k[g]) and np.array_equal(gv, v[g])
+    # appended tokens and raw normals
+    L0 = torch.tensor(w.prefill, dtype=torch.int32, device="cuda")
+    kk = torch.empty((2, w.layers, w.batch, w.kv_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+    vv = torch.empty_like(kk)
+    sp = w.spec()
+    assert gen.cuda_lib().ikvgen_fill_tokens_cuda(ctypes.byref(sp), torch.from_numpy(u).cuda().data_ptr(),
+                                                  L0.data_ptr(), 3, 5, w.dtype, kk.data_ptr(), vv.data_ptr(),
+                                                  torch.cuda.current_stream().cuda_stream) == 0
+    torch.cuda.synchronize()
+    for i, t in enumerate((3, 4)):
+        K, V = w.new_tokens(t, u)
+        assert np.array_equal(kk[i].float().cpu().numpy(), K) and np.array_equal(vv[i].float().cpu().numpy(), V)
+    n = 1 << 20
+    dn = torch.empty(n, dtype=torch.float32, device="cuda")
+    gen.cuda_lib().ikvgen_normals_cuda(5, 1, n, dn.data_ptr(), torch.cuda.current_stream().cuda_stream)
+    hn = np.empty(n, np.float32)
+    gen.host_lib().ikvgen_normals(5, 1, n, hn.ctypes.data)
+    assert np.array_equal(dn.cpu().numpy(), hn)
+
+
+# ------------------------------------------------------------------ attention + score
+ATT_CASES = [
+    # dtype, d, H, Hkv, lengths, gran
+    (gen.F32, 64, 4, 2, [512, 37, 1], ikv.IKV_GRAN_SEQ),
+    (gen.BF16, 128, 32, 8, [700, 64, 1500], ikv.IKV_GRAN_SEQ),
+    (gen.BF16, 128, 28, 4, [333, 1025], ikv.IKV_GRAN_SEQ),
+    (gen.BF16, 128, 28, 4, [333, 1025], ikv.IKV_GRAN_KVHEAD),
+    (gen.BF16, 64, 8, 8, [129, 3000], ikv.IKV_GRAN_SEQ),
+    (gen.F32, 128, 16, 2, [65, 2100], ikv.IKV_GRAN_KVHEAD),
+    (gen.BF16, 128, 16, 16, [5000], ikv.IKV_GRAN_SEQ),
+]
+
+
+@pytest.mark.parametrize("dt,d,H,Hkv,lens,gran", ATT_CASES)
+def test_decode_attend_score_matches_oracle(dt, d, H, Hkv, lens, gran):
+    w = gen.Workload("a", len(lens), 3, H, Hkv, d, lens, 1, dtype=dt, seed=21, page_size=64)
+    u = w.u_table()
+    c = make_cache(w, gran, page_perm_seed=5)
+    fill_device(c, w, torch.from_numpy(u).cuda())
+    layer = 2
+    q_h = w.queries(1, 2, u)[0, layer]                     # [batch][H][d]
+    q = to_device(q_h, w)
+    out = torch.empty((w.batch, H, d), dtype=q.dtype, device="cuda")
+    score = torch.full((c.rows, c.cap), -7.0, device="cuda")
+    rng = np.random.default_rng(3)
+    ema0 = torch.from_numpy(rng.random((c.rows, c.cap)).astype(np.float32)).cuda()
+    ema = ema0.clone()
+    cch = c.cache(max(lens))
+    ws = torch.empty(ikv.ikv_attend_workspace_size(c.shape(), cch), dtype=torch.uint8, device="cuda")
+    alpha = 0.85
+    ikv.ikv_decode_attend_score(c.shape(), cch, layer, q, out, score, ema, alpha, ws, ws.numel())
+    torch.cuda.synchronize()
+    q64 = as_f64(q_h, w)
+    tol_out = 2e-2 if dt == gen.BF16 else 1e-4
+    R = c.rows_per_seq
+    for b, L in enumerate(lens):
+        k, v = w.kv_block(b, layer, 0, L, u)
+        K = [k[g].astype(np.float64) for g in range(Hkv)]
+        V = [v[g].astype(np.float64) for g in range(Hkv)]
+        a, o = O.last_query_attention(q64[b], K, V)
+        assert np.max(np.abs(out[b].float().cpu().numpy() - o)) < tol_out
+        s = O.pooled_score(a, O.GRAN_SEQ if gran == ikv.IKV_GRAN_SEQ else O.GRAN_KVHEAD, Hkv)
+        for rr in range(R):
+            r = b * R + rr
+            gs = score[r, :L].cpu().numpy()
+            assert np.max(np.abs(gs - s[rr])) < 2e-5
+            want = O.ema_update(ema0[r, :L].double().cpu().numpy(), s[rr], alpha)
+            assert np.max(np.abs(ema[r, :L].cpu().numpy() - want)) < 2e-5
+            assert torch.all(score[r, L:] == -7.0)       # nothing written past len
+            assert torch.equal(ema[r, L:], ema0[r, L:])
+
+
+def test_decode_attend_without_score_leaves_state():
+    w = gen.Workload("a", 2, 1, 32, 8, 128, [900, 50], 1, dtype=gen.BF16, seed=2)
+    u = w.u_table()
+    c = make_cache(w)
+    fill_device(c, w, torch.from_numpy(u).cuda())
+    q_h = w.queries(1, 2, u)[0, 0]
+    out = torch.empty((2, 32, 128), dtype=torch.bfloat16, device="cuda")
+    cch = c.cache(900)
+    ws = torch.empty(ikv.ikv_attend_workspace_size(c.shape(), cch), dtype=torch.uint8, device="cuda")
+    ikv.ikv_decode_attend_score(c.shape(), cch, 0, to_device(q_h, w), out, None, None, 0.9, ws, ws.numel())
+    torch.cuda.synchronize()
+    for b, L in enumerate(w.prefill):
+        k, v = w.kv_block(b, 0, 0, L, u)
+        _, o = O.last_query_attention(as_f64(q_h, w)[b], [x.astype(np.float64) for x in k],
+                                      [x.astype(np.float64) for x in v])
+        assert np.max(np.abs(out[b].float().cpu().numpy() - o)) < 2e-2
+
+
+def test_ema_update_matches_eq4():
+    rng = np.random.default_rng(4)
+    rows, cap = 5, 1000
+    m0 = rng.random((rows, cap)).astype(np.float32)
+    s = rng.random((rows, cap)).astype(np.float32)
+    lens = np.array([1000, 3, 0, 999, 500], np.int32)
+    ema = torch.from_numpy(m0).cuda()
+    ikv.ikv_ema_update(rows, cap, ema, torch.from_numpy(s).cuda(), torch.from_numpy(lens).cuda(), 1, 0.7)
+    torch.cuda.synchronize()
+    got = ema.cpu().numpy()
+    for r in range(rows):
+        L = lens[r]
+        assert np.max(np.abs(got[r, :L] - O.ema_update(m0[r, :L].astype(np.float64), s[r, :L], 0.7)), initial=0) < 1e-6
+        assert np.array_equal(got[r, L:], m0[r, L:])
+
+
+# ------------------------------------------------------------------ selection
+def _select_gpu(util: np.ndarray, lens, budgets, rps=1):
+    rows, cap = util.shape
+    keep = torch.full((rows, cap), -1, dtype=torch.int32, device="cuda")
+    keep_len = torch.full((rows,), -1, dtype=torch.int32, device="cuda")
+    ikv.ikv_select_budget(rows, cap, torch.from_numpy(util).cuda(), torch.tensor(lens, dtype=torch.int32).cuda(), rps,
+                          torch.tensor(budgets, dtype=torch.int32).cuda(), keep, keep_len)
+    torch.cuda.synchronize()
+    return keep.cpu().numpy(), keep_len.cpu().numpy()
+
+
+def _check_select(util, lens, budgets, rps=1):
+    keep, keep_len = _select_gpu(util, lens, budgets, rps)
+    for r in range(util.shape[0]):
+        L, B = lens[r // rps], budgets[r // rps]
+        want = O.select_keep(util[r, :L].astype(np.float64), B)
+        assert keep_len[r] == len(want), (r, keep_len[r], len(want))
+        assert np.array_equal(keep[r, :len(want)], want), r
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_select_bit_exact_random(seed):
+    rng = np.random.default_rng(seed)
+    cap = 70000
+    lens = [32769, 3278, 65537, 1, 7, 2049, 5000, 6555]
+    budgets = [3277, 3277, 6554, 1, 0, 2048, 5000, 6554]
+    util = (rng.random((len(lens), cap)) ** 4).astype(np.float32)
+    _check_select(util, lens, budgets)
+
+
+def test_select_ties_and_special_values():
+    rng = np.random.default_rng(9)
+    cap = 5000
+    pool = np.array([0.0, -0.0, 0.25, 0.5, 1.0, -1.0, np.inf, -np.inf, np.nan, 1e-30, 1e-38], np.float32)
+    rows = 12
+    util = pool[rng.integers(0, len(pool), (rows, cap))]
+    lens = [cap, cap, 4000, 1000, 11, 12, 2, 4097, 4096, 3000, 5, cap]
+    budgets = [2500, 1, 3999, 999, 3, 12, 1, 4096, 4096, 2999, 0, cap - 1]
+    _check_select(util, lens, budgets)
+    # all equal: the lowest slots survive
+    _check_select(np.full((2, 3000), 0.125, np.float32), [3000, 2999], [100, 2998])
+
+
+def test_select_scale_invariance_on_gpu():
+    """Corollary 2: uniform positive scaling does not change the kept set."""
+    rng = np.random.default_rng(10)
+    util = (rng.random((3, 4000)) ** 3).astype(np.float32)
+    lens, budgets = [4000, 3000, 2000], [400, 2999, 7]
+    k1, _ = _select_gpu(util, lens, budgets)
+    k2, _ = _select_gpu((util * np.float32(4.0)).astype(np.float32), lens, budgets)   # exact power-of-two scale
+    assert np.array_equal(k1, k2)
+
+
+def test_select_kvhead_rows_share_length():
+    rng = np.random.default_rng(11)
+    util = rng.random((6, 800)).astype(np.float32)
+    _check_select(util, [800, 500], [300, 10], rps=3)
+
+
+# ------------------------------------------------------------------ compaction and append
+@pytest.mark.parametrize("mode", [ikv.IKV_COMPACT_STABLE, ikv.IKV_COMPACT_HOLEFILL])
+@pytest.mark.parametrize("gran", [ikv.IKV_GRAN_SEQ, ikv.IKV_GRAN_KVHEAD])
+def test_compact_matches_oracle_eviction(mode, gran):
+    w = gen.Workload("c", 3, 2, 8, 2, 128, [1000, 3278, 70], 1, dtype=gen.BF16, seed=31, page_size=16)
+    u = w.u_table()
+    c = make_cache(w, gran, page_perm_seed=9)
+    fill_device(c, w, torch.from_numpy(u).cuda())
+    rng = np.random.default_rng(12)
+    util = rng.random((c.rows, c.cap)).astype(np.float32)
+    if True:  # one sequence in steady state: a single eviction
+        util[c.rows_per_seq:2 * c.rows_per_seq, :3278] = rng.random((c.rows_per_seq, 3278))
+    c.ema.copy_(torch.from_numpy(util).cuda())
+    budgets = [100, 3277, 70]
+    c.budget.copy_(torch.tensor(budgets, dtype=torch.int32).cuda())
+    keep = torch.empty((c.rows, c.cap), dtype=torch.int32, device="cuda")
+    keep_len = torch.empty((c.rows,), dtype=torch.int32, device="cuda")
+    ikv.ikv_select_budget(c.rows, c.cap, c.ema, c.len, c.rows_per_seq, c.budget, keep, keep_len)
+    cch = c.cache(3278)
+    nws = ikv.ikv_compact_workspace_size(c.shape(), cch, mode)
+    ws = torch.empty(max(nws, 1), dtype=torch.uint8, device="cuda")
+    ikv.ikv_compact_kv(c.shape(), cch, keep, keep_len, c.ema, mode, ws, nws)
+    torch.cuda.synchronize()
+    R = c.rows_per_seq
+    pos = c.pos.cpu().numpy()
+    ema = c.ema.cpu().numpy()
+    assert c.len.cpu().tolist() == [min(L, B) for L, B in zip(w.prefill, budgets)]
+    for b in range(w.batch):
+        L = w.prefill[b]
+        K = [[None] * w.kv_heads for _ in range(w.layers)]
+        V = [[None] * w.kv_heads for _ in range(w.layers)]
+        for l in range(w.layers):
+            k, v = w.kv_block(b, l, 0, L, u)
+            for g in range(w.kv_heads):
+                K[l][g], V[l][g] = k[g].astype(np.float64), v[g].astype(np.float64)
+        st = O.prefill_state(K, V, budgets[b], O.GRAN_SEQ if gran == ikv.IKV_GRAN_SEQ else O.GRAN_KVHEAD)
+        st.m = util[b * R:(b + 1) * R, :L].astype(np.float64)
+        O.evict(st)
+        n = st.length
+        for rr in range(R):
+            gp = pos[b * R + rr, :n]
+            if mode == ikv.IKV_COMPACT_STABLE:
+                assert np.array_equal(gp, st.pos[rr])
+                assert np.array_equal(ema[b * R + rr, :n], st.m[rr].astype(np.float32))
+            else:
+                assert set(gp.tolist()) == set(st.pos[rr].tolist())
+                order = np.argsort(gp)
+                assert np.array_equal(ema[b * R + rr, :n][order], st.m[rr].astype(np.float32))
+        for l in range(w.layers):
+            for g in range(w.kv_heads):
+                rr = 0 if R == 1 else g
+                gp = pos[b * R + rr, :n]
+                rank = np.argsort(np.argsort(gp))
+                gk = c.gather(c.k, b, l, g, n).float().cpu().numpy()
+                gv = c.gather(c.v, b, l, g, n).float().cpu().numpy()
+                assert np.array_equal(gk, st.K[l][g][rank]) and np.array_equal(gv, st.V[l][g][rank])
+
+
+@pytest.mark.parametrize("init_mean", [0, 1])
+def test_append_token(init_mean):
+    w = gen.Workload("p", 2, 3, 8, 2, 64, [130, 5], 1, dtype=gen.F32, seed=41, page_size=64)
+    u = w.u_table()
+    c = make_cache(w, ikv.IKV_GRAN_KVHEAD)
+    fill_device(c, w, torch.from_numpy(u).cuda())
+    rng = np.random.default_rng(13)
+    m0 = rng.random((c.rows, c.cap)).astype(np.float32)
+    c.ema.copy_(torch.from_numpy(m0).cuda())
+    kn, vn = w.new_tokens(1, u)
+    ws = torch.empty(4096, dtype=torch.uint8, device="cuda")
+    ikv.ikv_append_token(c.shape(), c.cache(130), to_device(kn, w), to_device(vn, w), c.ema, init_mean, ws, 4096)
+    torch.cuda.synchronize()
+    assert c.len.cpu().tolist() == [131, 6] and c.next_pos.cpu().tolist() == [131, 6]
+    for b, L in enumerate(w.prefill):
+        for g in range(w.kv_heads):
+            r = b * w.kv_heads + g
+            want = O.new_token_state(m0[r, :L].astype(np.float64), refresh=not init_mean, refresh_init="zero")
+            assert abs(float(c.ema[r, L]) - want) < 1e-6
+            assert int(c.pos[r, L]) == L
+            for l in range(w.layers):
+                assert np.array_equal(c.gather(c.k, b, l, g, L + 1)[L].cpu().numpy(), kn[l, b, g])
+                assert np.array_equal(c.gather(c.v, b, l, g, L + 1)[L].cpu().numpy(), vn[l, b, g])

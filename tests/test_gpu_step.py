@@ -1,0 +1,92 @@
+"""Whole decode steps (ikv_step) in lock-step with the oracle (GPU only).
+
+Each case runs several decode steps, with eviction on every step, and checks
+per step: attention outputs (bf16: 2e-2, fp32: 1e-4 absolute), utilities of
+the kept tokens (1e-3 absolute, fp32 vs fp64), the retained set under the
+boundary rule (gap 1e-4 around the oracle's B-th utility), and the compacted
+K/V rows bit for bit.
+"""
+import numpy as np
+import pytest
+import torch
+
+import gen
+from harness import run_lockstep
+from paper_2609_03515_gb300 import ikv
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+
+    __graft_entry__.build()
+
+
+def _assert(reps, tol_out, strict_fraction=0.0):
+    for r in reps:
+        assert r.set_ok, r
+        assert r.out_err < tol_out, r
+        assert r.m_err < 1e-3, r
+        assert r.kv_err == 0.0, r
+    if strict_fraction:
+        assert np.mean([r.strict_set_equal for r in reps]) >= strict_fraction
+
+
+def small_llama(**kw):
+    base = dict(name="llama-small", batch=3, layers=3, q_heads=32, kv_heads=8, head_dim=128,
+                prefill=[300, 777, 1200], steps=10, dtype=gen.BF16, alpha=0.9, seed=5, page_size=64)
+    base.update(kw)
+    return gen.Workload(**base)
+
+
+def test_config0_full_trajectory():
+    """The tiny fp32 workload end to end: 16 steps, full refresh, alpha 0.9, B = 51."""
+    w = gen.config(0)
+    reps = run_lockstep(w)
+    _assert(reps, 1e-4, strict_fraction=1.0)
+
+
+def test_small_llama_full_refresh():
+    _assert(run_lockstep(small_llama()), 2e-2)
+
+
+def test_small_llama_lazy_refresh():
+    _assert(run_lockstep(small_llama(refresh_period=3, steps=9)), 2e-2)
+
+
+def test_small_llama_score_free():
+    _assert(run_lockstep(small_llama(score_free=True, steps=8)), 2e-2)
+
+
+def test_small_llama_kvhead_rows():
+    _assert(run_lockstep(small_llama(steps=6), gran=ikv.IKV_GRAN_KVHEAD), 2e-2)
+
+
+def test_holefill_keeps_the_same_sets():
+    _assert(run_lockstep(small_llama(steps=6), compact_mode=ikv.IKV_COMPACT_HOLEFILL), 2e-2)
+
+
+def test_sparse_layer_mask_and_mean_init_on_refresh():
+    w = small_llama(steps=5, layers=4)
+    _assert(run_lockstep(w, layer_eligible=[1, 0, 1, 0], refresh_init=ikv.IKV_INIT_MEAN), 2e-2)
+
+
+def test_qwen_group7():
+    w = gen.Workload("qwen-small", 2, 2, 28, 4, 128, [2000, 513], 6, dtype=gen.BF16, seed=6, alpha=0.5)
+    _assert(run_lockstep(w), 2e-2)
+
+
+def test_budget_edges():
+    # no eviction ever (B >= L0 + steps), and a budget of one token
+    w = small_llama(batch=2, prefill=[100, 200], steps=4, budget_frac=1.0, layers=2)
+    _assert(run_lockstep(w, steps=4), 2e-2)
+    w1 = small_llama(batch=1, prefill=[90], steps=4, budget_frac=0.011, layers=2)
+    assert w1.budgets() == [1]
+    _assert(run_lockstep(w1), 2e-2)
+
+
+def test_alpha_zero_and_one():
+    _assert(run_lockstep(small_llama(alpha=0.0, steps=3, layers=2)), 2e-2)
+    _assert(run_lockstep(small_llama(alpha=1.0, steps=3, layers=2)), 2e-2)
