@@ -50,6 +50,28 @@ def parse():
     return ap.parse_args()
 
 
+def max_over_ranks(ms: float, dist, device=None) -> float:
+    """Slowest rank's time: the job's time for weak-scaled replicas (all ranks start
+    after the same barrier)."""
+    if dist is None:
+        return ms
+    import torch
+
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(tokens_per_rank: int, world: int, ms_max: float) -> float:
+    """Whole-job tokens/s: every rank decodes its own sequences."""
+    return tokens_per_rank * world / (ms_max / 1e3)
+
+
+def rank_seed(base_seed: int, rank: int) -> int:
+    """Each rank decodes different sequences."""
+    return base_seed + 1000 * rank
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -250,11 +272,7 @@ def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_d
     stop.record(stream)
     torch.cuda.synchronize()
     launches = ikv.ikv_launch_count() - launches0
-    ms = start.elapsed_time(stop)
-    if dist:
-        tt = torch.tensor([ms], device=c.k.device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(start.elapsed_time(stop), dist, c.k.device)
     res = {"ms": ms, "launches": launches, "lens": lens}
     if want_detail:
         res["clocks"] = clocks.stop()
@@ -306,11 +324,7 @@ def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist):
         step(W + 1 + i)
     stop.record(stream)
     torch.cuda.synchronize()
-    ms = start.elapsed_time(stop)
-    if dist:
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(start.elapsed_time(stop), dist, dev)
     h2d = (q_d.numel() + kn_d.numel() + vn_d.numel()) * q_d.element_size()
     d2h = out_d.numel() * out_d.element_size()
     return ms, h2d, d2h
@@ -344,7 +358,7 @@ def run_ours(args):
 
     w = gen.config(args.config)
     # each rank decodes its own independent sequences (distinct seed per rank)
-    w = w.with_(seed=w.seed + 1000 * rank)
+    w = w.with_(seed=rank_seed(w.seed, rank))
     total_steps = args.warmup + args.steps
     if total_steps > w.steps:
         w = w.with_(steps=total_steps)
@@ -394,8 +408,7 @@ def run_ours(args):
     e2e_ms, h2d, d2h = run_e2e(args, w, c, u_dev, ws, compact_mode, qs_pin, kn_pin, vn_pin, dist)
 
     K = args.steps
-    tokens = w.batch * K * world
-    value = tokens / (full["ms"] / 1e3)
+    value = job_throughput(w.batch * K, world, full["ms"])
     if rank != 0:
         if dist:
             dist.destroy_process_group()

@@ -8,6 +8,14 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 
+def pytest_sessionstart(session):
+    # the CUDA library and the generator are compiled in place (nvcc cross-compiles
+    # without a GPU); test modules import the binding at collection time
+    import __graft_entry__
+
+    __graft_entry__.build()
+
+
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300, sm_103a) and the built CUDA libraries")
 

@@ -12,9 +12,9 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 @pytest.fixture(scope="module")
 def lib():
-    from paper_2609_03515_gb300 import build as B
+    import __graft_entry__
 
-    B.build()
+    __graft_entry__.build()
     from paper_2609_03515_gb300 import ikv
 
     return ikv
