@@ -257,6 +257,8 @@ def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_d
     if want_detail:
         for _ in range(K):
             e = [torch.cuda.Event(enable_timing=True) for _ in range(7)]
+            for x in e:
+                x.record(stream)  # torch creates the CUDA event on first record; the library re-records it
             evs.append(e)
             tm = ikv.ikv_timing(*[x.cuda_event for x in e])
             timings.append(tm)
