@@ -72,6 +72,25 @@ def rank_seed(base_seed: int, rank: int) -> int:
     return base_seed + 1000 * rank
 
 
+ATTEND_KERNEL_REV = "attend_v1"
+
+
+def profiled_traffic(workload: str):
+    """DRAM bytes per launch of the attention kernel from the committed ncu summary,
+    or None when that summary was taken on another kernel revision or workload."""
+    import re
+
+    path = os.path.join(ROOT, "profiles", f"attend_split_kernel__{workload}.md")
+    if not os.path.exists(path):
+        return None
+    txt = open(path).read()
+    rev = re.search(r"^kernel_rev:\s*(\S+)", txt, re.M)
+    tb = re.search(r"^traffic_bytes_per_launch:\s*(\d+)", txt, re.M)
+    if not rev or not tb or rev.group(1) != ATTEND_KERNEL_REV:
+        return None
+    return int(tb.group(1))
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -424,16 +443,7 @@ def run_ours(args):
     q_bytes = w.layers * w.batch * w.q_heads * w.head_dim * esz
     att_ms = full["kernel_ms"]["attend"]
     achieved = (kv_bytes + q_bytes) / (att_ms / 1e3) / 1e9
-    traffic = None
-    prof = os.path.join(ROOT, "profiles", "attend_traffic.json")
-    if os.path.exists(prof):
-        try:
-            with open(prof) as f:
-                d = json.load(f)
-            if d.get("kernel_rev") == "attend_v1" and d.get("workload") == w.name:
-                traffic = d.get("bytes_per_launch")
-        except (OSError, ValueError):
-            traffic = None
+    traffic = profiled_traffic(w.name)
     line = {
         "metric": METRIC,
         "value": value,
