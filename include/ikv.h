@@ -137,6 +137,30 @@ ikv_status ikv_decode_attend_score(const ikv_shape *shape, const ikv_cache *cach
                                    void *ws, size_t ws_bytes, cudaStream_t stream);
 
 /* ---------------------------------------------------------------------------
+ * ikv_decode_attend_score_static -- ikv_decode_attend_score without a
+ * caller workspace.  The paper has no counterpart: this is for callers that
+ * cannot allocate device memory (a runtime that hands out all device memory
+ * up front and forbids later cudaMalloc, an operator hook inside a framework
+ * that owns the allocator, a loop that cannot afford cudaMalloc's implicit
+ * synchronisation).  It allocates nothing; its scratch is a fixed device
+ * array inside the library of ikv_static_scratch_bytes() bytes (16 MiB),
+ * held by every GPU that loads the library until the process exits.
+ *  - Arguments and results are those of ikv_decode_attend_score.
+ *  - Shapes whose scratch (ikv_attend_workspace_size) exceeds the array are
+ *    rejected with IKV_ERR_WORKSPACE and a message; nothing is launched.
+ *  - The first call on a device looks up the array's device address (with
+ *    that device current); make that first call before any stream capture.
+ *  - All calls share the one array, which keeps the last call's contents
+ *    (nothing in it needs clearing).  Calls whose GPU work overlaps -- other
+ *    streams or other host threads on the same device -- race on it; the
+ *    caller must serialise them.
+ * ------------------------------------------------------------------------- */
+size_t ikv_static_scratch_bytes(void);
+ikv_status ikv_decode_attend_score_static(const ikv_shape *shape, const ikv_cache *cache, int32_t layer,
+                                          const void *q, void *out, float *score, float *ema, float alpha,
+                                          cudaStream_t stream);
+
+/* ---------------------------------------------------------------------------
  * ikv_ema_update -- Eq. 4 on a score array, in place.
  *     ema[r][i] = alpha * ema[r][i] + (1 - alpha) * score[r][i],  i < len[r / rows_per_seq]
  *  rows_per_seq: 1 for IKV_GRAN_SEQ, kv_heads for IKV_GRAN_KVHEAD.

@@ -235,6 +235,15 @@ ikv_status record(cudaEvent_t e, cudaStream_t st) {
 }
 
 }  // namespace
+
+ikv_status report(ikv_status s, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+    return s;
+}
+
 }  // namespace ikv
 
 using namespace ikv;

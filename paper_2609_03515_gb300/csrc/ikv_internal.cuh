@@ -19,6 +19,9 @@ constexpr int kMaxLayers = 512;
 // Launch-count bookkeeping (host).
 void note_launch(int n = 1);
 
+// Set the thread's ikv_last_error() message and return `s` (host).
+ikv_status report(ikv_status s, const char *fmt, ...);
+
 // Where a (sequence, slot) row of layer l / kv head g lives in the paged pool.
 struct PagedView {
     const int32_t *block_table;

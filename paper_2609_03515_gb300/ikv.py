@@ -63,6 +63,8 @@ def _load():
         "ikv_launch_count": ([], ctypes.c_int64),
         "ikv_attend_workspace_size": ([SP, CP, ctypes.POINTER(SZ)], I32),
         "ikv_decode_attend_score": ([SP, CP, I32, P, P, P, P, F32, P, SZ, P], I32),
+        "ikv_static_scratch_bytes": ([], SZ),
+        "ikv_decode_attend_score_static": ([SP, CP, I32, P, P, P, P, F32, P], I32),
         "ikv_ema_update": ([I32, I32, P, P, P, I32, F32, P], I32),
         "ikv_select_budget": ([I32, I32, P, P, I32, P, P, P, P], I32),
         "ikv_compact_workspace_size": ([SP, CP, I32, ctypes.POINTER(SZ)], I32),
@@ -120,6 +122,16 @@ def ikv_attend_workspace_size(shape: ikv_shape, cache: ikv_cache) -> int:
 def ikv_decode_attend_score(shape, cache, layer, q, out, score, ema, alpha, ws, ws_bytes, stream=None) -> None:
     _check(_lib.ikv_decode_attend_score(ctypes.byref(shape), ctypes.byref(cache), layer, _p(q), _p(out), _p(score),
                                         _p(ema), alpha, _p(ws), ws_bytes, _stream(stream)), "ikv_decode_attend_score")
+
+
+def ikv_static_scratch_bytes() -> int:
+    return int(_lib.ikv_static_scratch_bytes())
+
+
+def ikv_decode_attend_score_static(shape, cache, layer, q, out, score, ema, alpha, stream=None) -> None:
+    _check(_lib.ikv_decode_attend_score_static(ctypes.byref(shape), ctypes.byref(cache), layer, _p(q), _p(out),
+                                               _p(score), _p(ema), alpha, _stream(stream)),
+           "ikv_decode_attend_score_static")
 
 
 def ikv_ema_update(rows, cap, ema, score, length, rows_per_seq, alpha, stream=None) -> None:
