@@ -24,6 +24,11 @@
  *    accumulation are fp32.  head_dim must be 64 or 128 and
  *    q_heads / kv_heads (the GQA group size G) one of 1, 2, 4, 7, 8.
  *  - Alignment: K/V pools, q, out, k_new, v_new must be 16-byte aligned.
+ *  - bf16 pools with head_dim 128 and page_size 8..128 dividing 128 (or a
+ *    multiple of 128) take the tensor-core attention path, which reads whole
+ *    128-slot tiles: slots at or past len[b] inside a sequence's last tile
+ *    must hold finite values (any finite values; zero-initialised pools and
+ *    evicted rows qualify), and every block_table entry must name a valid page.
  *
  * Paged K/V layout
  * ----------------
@@ -113,6 +118,12 @@ const char *ikv_last_error(void);
 
 /* Number of kernels this library has launched in this process. */
 int64_t ikv_launch_count(void);
+
+/* Device-side error word of the current device, then cleared (synchronises
+ * the device).  0 = no error.  Bit 0: a bounded wait inside the tensor-core
+ * attention kernel ran out (the kernel abandoned its work and returned);
+ * bit 1: a split longer than the kernel's TMEM budget reached the device. */
+ikv_status ikv_device_status(uint32_t *flags);
 
 /* ---------------------------------------------------------------------------
  * ikv_decode_attend_score -- one layer of decode attention plus its score.

@@ -147,18 +147,23 @@ T *at(void *ws, size_t off) {
     return reinterpret_cast<T *>(reinterpret_cast<unsigned char *>(ws) + off);
 }
 
-// split-K partition for lengths up to max_len
-void choose_splits(const ikv_shape *s, int n_layers, int32_t max_len, int32_t *split_tokens, int32_t *n_splits) {
+// split-K partition for lengths up to max_len: enough CTAs to fill the GPU
+// (ctas_per_sm x SMs), splits a multiple of `granule` tokens and at most
+// `max_split` tokens long, at most kMaxSplits per (sequence, layer, kv head)
+void choose_splits(const ikv_shape *s, int n_layers, int32_t max_len, int granule, int max_split,
+                   int32_t *split_tokens, int32_t *n_splits) {
     const int64_t units = (int64_t)s->batch * n_layers * s->kv_heads;
     const int64_t want = (int64_t)sm_count() * 4;
     int64_t splits = (want + units - 1) / units;
     const int64_t by_len = (max_len + kMinSplitTokens - 1) / kMinSplitTokens;
     if (splits > by_len) splits = by_len;
+    const int64_t need = (max_len + max_split - 1) / max_split;
+    if (splits < need) splits = need;
     if (splits > kMaxSplits) splits = kMaxSplits;
     if (splits < 1) splits = 1;
     int64_t st = (max_len + splits - 1) / splits;
-    st = (st + kTileTokens - 1) / kTileTokens * kTileTokens;
-    if (st < kTileTokens) st = kTileTokens;
+    st = (st + granule - 1) / granule * granule;
+    if (st < granule) st = granule;
     *split_tokens = (int32_t)st;
     int64_t ns = (max_len + st - 1) / st;
     if (ns < 1) ns = 1;
@@ -179,13 +184,25 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
     a.q_heads = s->q_heads;
     a.layer0 = layer0;
     a.n_layers = n_layers;
-    choose_splits(s, n_layers, max_len, &a.split_tokens, &a.n_splits);
+    const int group = s->q_heads / s->kv_heads;
+    const uint64_t pool_rows = (uint64_t)(layer0 + n_layers) * c->num_pages * s->kv_heads * c->page_size;
+    const bool tc = tc_supported(s->dtype, s->head_dim, group, c->page_size) &&
+                    (int64_t)max_len <= (int64_t)kMaxSplits * tc_max_split_tokens() && pool_rows < (1ull << 31);
+    if (tc)
+        choose_splits(s, n_layers, max_len, 128, tc_max_split_tokens(), &a.split_tokens, &a.n_splits);
+    else
+        choose_splits(s, n_layers, max_len, kTileTokens, 1 << 30, &a.split_tokens, &a.n_splits);
     a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)s->head_dim));
     a.logits = logits ? at<float>(ws, w.logits) : nullptr;
     a.cap = cap_of(c);
     a.part_ml = at<float>(ws, w.part_ml);
     a.part_o = at<float>(ws, w.part_o);
-    if (max_len > 0) IKV_TRY_CUDA(launch_attend(a, s->dtype, s->head_dim, s->q_heads / s->kv_heads, st), "attend launch");
+    if (max_len > 0) {
+        if (tc)
+            IKV_TRY_CUDA(launch_attend_tc(a, group, st), "tensor-core attend launch");
+        else
+            IKV_TRY_CUDA(launch_attend(a, s->dtype, s->head_dim, group, st), "attend launch");
+    }
     if (tm && tm->attend_end) IKV_TRY_CUDA(cudaEventRecord(tm->attend_end, st), "cudaEventRecord");
     CombineArgs cb{};
     cb.len = c->len;

@@ -1,0 +1,517 @@
+// Tensor-core split-K decode attention with logits, bf16, head_dim 128 (sm_103a).
+//
+// Same contract as attend_split_kernel (one CTA per split, kv head, sequence x
+// layer; writes log2-domain logits and per-split (max, sum, O) partials), built
+// from Blackwell pieces:
+//   * TMA (cp.async.bulk.tensor.2d, 128-byte swizzle) streams 128-token K and V
+//     tiles out of the paged pool (one box per page segment and 64-column half)
+//     into a 3-stage ring guarded by mbarriers;
+//   * tcgen05.mma (kind::f16, bf16 in, fp32 accumulate in TMEM) computes
+//       S_i[128 tokens x 16] = K_i[128 x 128] . Q^T[128 x 16]   (Q: G heads, zero-padded to 16)
+//       O[128 dims x 16]    += V_i^T[128 x 128] . P_i^T[128 x 16]
+//     with K-major operands for QK and an MN-major (transposed) V for PV;
+//   * the softmax runs as two sweeps over the S tiles kept in TMEM: the split
+//     maximum per head, then exp2, logits write-out, row sums and the bf16 P
+//     operand (double-buffered in shared memory) that feeds the PV MMA.
+// Warp roles (192 threads): warps 0-3 own TMEM lanes 0-127 (softmax, epilogue),
+// warp 4 issues TMA loads, warp 5 issues MMAs.  Every mbarrier wait is bounded;
+// on timeout the CTA records an error code, stops issuing work, waits for its
+// in-flight copies, frees its TMEM and returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "ikv_internal.cuh"
+
+namespace ikv {
+
+__device__ unsigned int g_tc_error = 0;
+
+namespace {
+
+constexpr int kTile = 128;
+constexpr int kD = 128;
+constexpr int kNst = 3;
+constexpr int kStage = kTile * kD * 2;          // 32 KB: one K or V tile
+constexpr int kHalf = kStage / 2;               // one 64-column half (16 KB)
+constexpr int kN = 16;                          // padded head count (MMA N)
+constexpr int kOpBytes = kN * kD * 2;           // 4 KB: Q or one P operand
+constexpr int kTmemCols = 256;
+constexpr int kOcol = kTmemCols - kN;           // O accumulator columns [240, 256)
+constexpr int kMaxTiles = kOcol / kN;           // 15 S tiles
+constexpr int kThreads = 192;
+constexpr uint64_t kWaitNs = 1000000000ull;   // 1 s: orders of magnitude above any legitimate wait
+
+constexpr int kOffQ = kNst * kStage;
+constexpr int kOffP = kOffQ + kOpBytes;
+constexpr int kOffRed = kOffP + 2 * kOpBytes;
+constexpr int kOffBar = kOffRed + 4 * kN * 4;
+// barriers: full[kNst], empty[kNst], s_full, p_full[2], p_empty[2], o_full
+constexpr int kNumBar = 2 * kNst + 6;
+constexpr int kOffMisc = kOffBar + kNumBar * 8;
+constexpr int kSmemBytes = kOffMisc + 16 + 1024;   // + slack for 1024-byte alignment
+
+enum : unsigned { kErrTimeout = 1u };
+
+struct TcArgs {
+    const int32_t *len;
+    const int32_t *block_table;
+    int32_t num_pages, page_size, max_pages, kv_heads, rows_per_box;
+    const __nv_bfloat16 *q;     // q + ((li*batch + b)*H + h)*128
+    int32_t batch, q_heads, layer0, n_layers, split_tokens, n_splits, cap;
+    float scale_log2;
+    float *logits;              // may be null
+    float *part_ml, *part_o;
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+// Bounded wait on an mbarrier phase (non-blocking polls, at most kWaitNs of wall
+// time).  Returns false -- raising the CTA's abort flag and the global error
+// word -- if the phase does not complete in time, or returns false at once if
+// another role of the CTA has already aborted.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort) {
+    if (mbar_test(bar, parity)) return true;
+    const uint64_t start = global_ns();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_test(bar, parity)) return true;
+        if (i > 64) __nanosleep(32);
+        if ((i & 63u) == 0) {
+            if (*abort) return false;
+            if (global_ns() - start > kWaitNs) break;
+        }
+    }
+    *abort = 1;
+    atomicOr(&g_tc_error, kErrTimeout);
+    return false;
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+// smem matrix descriptor, 128-byte swizzle (sm_100 family, version 1)
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    uint64_t d = (uint64_t)((saddr >> 4) & 0x3FFFu);
+    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)2 << 61;
+    return d;
+}
+// instruction descriptor kind::f16: bf16 x bf16 -> f32, A K-major or MN-major, B K-major
+__host__ __device__ constexpr uint32_t idesc_bf16(bool a_mn_major, int M, int N) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn_major ? 1u : 0u) << 15) | ((uint32_t)(N >> 3) << 17) |
+           ((uint32_t)(M >> 4) << 24);
+}
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\ttcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+            d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(acc)
+        : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void fence_after_sync() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_before_sync() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+__device__ __forceinline__ void softmax_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+template <int NC>
+__device__ __forceinline__ void tmem_ld(uint32_t taddr, float *v);
+template <>
+__device__ __forceinline__ void tmem_ld<4>(uint32_t taddr, float *v) {
+    uint32_t r[4];
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 4; ++i) v[i] = __uint_as_float(r[i]);
+}
+template <>
+__device__ __forceinline__ void tmem_ld<8>(uint32_t taddr, float *v) {
+    uint32_t r[8];
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                 : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// byte offset of element (row, col) inside a [rows][64] bf16 block stored with
+// the 128-byte swizzle (128-byte rows, 16-byte chunks permuted by row % 8)
+__device__ __forceinline__ uint32_t sw128(uint32_t row, uint32_t col) {
+    return row * 128u + ((((col >> 3) ^ row) & 7u) << 4) + ((col & 7u) << 1);
+}
+
+template <int G>
+__global__ void __launch_bounds__(kThreads, 2)
+    attend_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, const TcArgs a) {
+    constexpr int NC = G <= 4 ? 4 : 8;  // TMEM columns read per S tile
+    extern __shared__ unsigned char smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    unsigned char *sm = smem_raw + (base - raw);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int s = blockIdx.x, g = blockIdx.y;
+    const int b = blockIdx.z % a.batch, li = blockIdx.z / a.batch;
+    const int l = a.layer0 + li;
+    const int L = a.len[b];
+    const int t0 = s * a.split_tokens;
+    if (t0 >= L) return;
+    const int t1 = min(t0 + a.split_tokens, L);
+    const int n = (t1 - t0 + kTile - 1) / kTile;
+    if (n > kMaxTiles) {  // the host sizes splits to fit TMEM; refuse rather than overrun
+        if (threadIdx.x == 0) atomicOr(&g_tc_error, 2u);
+        return;
+    }
+    const int H = a.q_heads;
+
+    const uint32_t sQ = base + kOffQ, sP = base + kOffP;
+    float *red = reinterpret_cast<float *>(sm + kOffRed);
+    const uint32_t bar0 = base + kOffBar;
+    auto full = [&](int i) { return bar0 + 8u * i; };
+    auto empty = [&](int i) { return bar0 + 8u * (kNst + i); };
+    const uint32_t s_full = bar0 + 8u * (2 * kNst);
+    auto p_full = [&](int i) { return bar0 + 8u * (2 * kNst + 1 + i); };
+    auto p_empty = [&](int i) { return bar0 + 8u * (2 * kNst + 3 + i); };
+    const uint32_t o_full = bar0 + 8u * (2 * kNst + 5);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(sm + kOffMisc);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + kOffMisc + 4);
+
+    if (tid == 0) {
+        for (int i = 0; i < kNst; ++i) {
+            mbar_init(full(i), 1);
+            mbar_init(empty(i), 1);
+        }
+        mbar_init(s_full, 1);
+        mbar_init(p_full(0), 128);
+        mbar_init(p_full(1), 128);
+        mbar_init(p_empty(0), 1);
+        mbar_init(p_empty(1), 1);
+        mbar_init(o_full, 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    // Q operand [16 heads][128 dims], heads >= G zero; both P buffers zeroed (rows >= G stay zero)
+    {
+        const __nv_bfloat16 *qg = a.q + (((int64_t)li * a.batch + b) * H + (int64_t)g * G) * kD;
+        for (int i = tid; i < kN * kD; i += kThreads) {
+            const int h = i / kD, c = i % kD;
+            const __nv_bfloat16 v = h < G ? qg[h * kD + c] : __float2bfloat16_rn(0.f);
+            *reinterpret_cast<__nv_bfloat16 *>(sm + kOffQ + (c >> 6) * (kN * 128) + sw128(h, c & 63)) = v;
+        }
+        for (int i = tid; i < 2 * kOpBytes / 16; i += kThreads)
+            reinterpret_cast<uint4 *>(sm + kOffP)[i] = make_uint4(0, 0, 0, 0);
+    }
+    fence_async_smem();
+    fence_before_sync();
+    __syncthreads();
+    fence_after_sync();
+    const uint32_t tmem = *tmem_slot;
+    const uint32_t tS = tmem, tO = tmem + kOcol;
+
+    if (warp == 4) {
+        // ---------------- TMA producer
+        if (lane == 0) {
+            const int boxes = kTile / a.rows_per_box;
+            int issued = 0;
+            for (int j = 0; j < 2 * n; ++j) {
+                const int st = j % kNst;
+                if (j >= kNst && !mbar_wait(empty(st), ((j / kNst) - 1) & 1, abort_flag)) break;
+                mbar_expect_tx(full(st), kStage);
+                const int tile = j < n ? j : j - n;
+                const CUtensorMap *tm = j < n ? &tmK : &tmV;
+                const uint32_t dst = base + st * kStage;
+                for (int bx = 0; bx < boxes; ++bx) {
+                    const int tok = t0 + tile * kTile + bx * a.rows_per_box;
+                    int lp = tok / a.page_size;
+                    if (lp >= a.max_pages) lp = a.max_pages - 1;
+                    const int page = a.block_table[(int64_t)b * a.max_pages + lp];
+                    const int row = ((l * a.num_pages + page) * a.kv_heads + g) * a.page_size + tok % a.page_size;
+                    tma_load_2d(dst + bx * a.rows_per_box * 128, tm, 0, row, full(st));
+                    tma_load_2d(dst + kHalf + bx * a.rows_per_box * 128, tm, 64, row, full(st));
+                }
+                issued = j + 1;
+            }
+            // drain: the last phase issued on each stage must have landed before the CTA exits
+            for (int j = issued - 1; j >= 0 && j >= issued - kNst; --j) (void)mbar_wait(full(j % kNst), (j / kNst) & 1, abort_flag);
+        }
+        __syncwarp();
+    } else if (warp == 5) {
+        // ---------------- MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t id_qk = idesc_bf16(false, 128, kN);
+            constexpr uint32_t id_pv = idesc_bf16(true, 128, kN);
+            bool ok = true;
+            for (int i = 0; i < n && ok; ++i) {
+                const int st = i % kNst;
+                if (!(ok = mbar_wait(full(st), (i / kNst) & 1, abort_flag))) break;
+                fence_after_sync();
+                const uint32_t ka = base + st * kStage;
+#pragma unroll
+                for (int kk = 0; kk < kD / 16; ++kk) {
+                    const uint64_t da = sdesc(ka + (kk >> 2) * kHalf + (kk & 3) * 32, 16, 1024);
+                    const uint64_t db = sdesc(sQ + (kk >> 2) * (kN * 128) + (kk & 3) * 32, 16, 1024);
+                    mma_bf16(tS + kN * i, da, db, id_qk, kk > 0 ? 1u : 0u);
+                }
+                mma_commit(empty(st));
+            }
+            mma_commit(s_full);
+            for (int i = 0; i < n && ok; ++i) {
+                const int j = n + i, st = j % kNst;
+                if (!(ok = mbar_wait(full(st), (j / kNst) & 1, abort_flag))) break;
+                if (!(ok = mbar_wait(p_full(i & 1), (i >> 1) & 1, abort_flag))) break;
+                fence_after_sync();
+                const uint32_t va = base + st * kStage;
+                const uint32_t pb = sP + (i & 1) * kOpBytes;
+#pragma unroll
+                for (int kk = 0; kk < kTile / 16; ++kk) {
+                    // A = V^T (MN-major): 64-dim atoms 16 KB apart (LBO), 8-token groups 1 KB apart (SBO)
+                    const uint64_t da = sdesc(va + kk * 2048, kHalf, 1024);
+                    const uint64_t db = sdesc(pb + (kk >> 2) * (kN * 128) + (kk & 3) * 32, 16, 1024);
+                    mma_bf16(tO, da, db, id_pv, (i > 0 || kk > 0) ? 1u : 0u);
+                }
+                mma_commit(empty(st));
+                mma_commit(p_empty(i & 1));
+            }
+            mma_commit(o_full);
+        }
+        __syncwarp();
+    } else {
+        // ---------------- softmax / epilogue: thread tid owns TMEM lane tid
+        const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+        float mx[G], sum[G];
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            mx[h] = -INFINITY;
+            sum[h] = 0.f;
+        }
+        bool ok = __all_sync(0xffffffffu, mbar_wait(s_full, 0, abort_flag));
+        fence_after_sync();
+        if (ok) {
+            for (int i = 0; i < n; ++i) {
+                float v[NC];
+                tmem_ld<NC>(tS + lane_off + kN * i, v);
+                if (t0 + i * kTile + tid < t1) {
+#pragma unroll
+                    for (int h = 0; h < G; ++h) mx[h] = fmaxf(mx[h], v[h] * a.scale_log2);
+                }
+            }
+        }
+        // split max per head over the 128 softmax threads
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            float m = mx[h];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+            if (lane == 0) red[warp * kN + h] = m;
+        }
+        __syncwarp();
+        softmax_bar();
+#pragma unroll
+        for (int h = 0; h < G; ++h) mx[h] = fmaxf(fmaxf(red[h], red[kN + h]), fmaxf(red[2 * kN + h], red[3 * kN + h]));
+        softmax_bar();
+
+        const int64_t lbase = (((int64_t)b * a.n_layers + li) * H + (int64_t)g * G) * a.cap;
+        for (int i = 0; i < n && ok; ++i) {
+            if (i >= 2 && !(ok = __all_sync(0xffffffffu, mbar_wait(p_empty(i & 1), ((i >> 1) - 1) & 1, abort_flag))))
+                break;
+            float v[NC];
+            tmem_ld<NC>(tS + lane_off + kN * i, v);
+            const int tok = t0 + i * kTile + tid;
+            const bool valid = tok < t1;
+            unsigned char *pbuf = sm + kOffP + (i & 1) * kOpBytes + (tid >> 6) * (kN * 128);
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                const float z = v[h] * a.scale_log2;
+                float p = 0.f;
+                if (valid) {
+                    if (a.logits) a.logits[lbase + (int64_t)h * a.cap + tok] = z;
+                    p = exp2f(z - mx[h]);
+                    sum[h] += p;
+                }
+                *reinterpret_cast<__nv_bfloat16 *>(pbuf + sw128(h, tid & 63)) = __float2bfloat16_rn(p);
+            }
+            fence_async_smem();
+            mbar_arrive(p_full(i & 1));
+        }
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            float t = sum[h];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+            if (lane == 0) red[warp * kN + h] = t;
+        }
+        __syncwarp();
+        softmax_bar();
+#pragma unroll
+        for (int h = 0; h < G; ++h) sum[h] = red[h] + red[kN + h] + red[2 * kN + h] + red[3 * kN + h];
+
+        if (ok) ok = mbar_wait(o_full, 0, abort_flag);
+        ok = __all_sync(0xffffffffu, ok);
+        fence_after_sync();
+        if (ok) {
+            float o[NC];
+            tmem_ld<NC>(tO + lane_off, o);
+            const int64_t pbase = (((int64_t)b * a.n_layers + li) * H + (int64_t)g * G) * a.n_splits;
+#pragma unroll
+            for (int h = 0; h < G; ++h) a.part_o[((pbase + (int64_t)h * a.n_splits) + s) * kD + tid] = o[h];
+            if (tid < G) {
+                float mm = -INFINITY, ss = 0.f;
+#pragma unroll
+                for (int h = 0; h < G; ++h)
+                    if (h == tid) {
+                        mm = mx[h];
+                        ss = sum[h];
+                    }
+                a.part_ml[((pbase + (int64_t)tid * a.n_splits) + s) * 2 + 0] = mm;
+                a.part_ml[((pbase + (int64_t)tid * a.n_splits) + s) * 2 + 1] = ss;
+            }
+        }
+    }
+    fence_before_sync();
+    __syncthreads();
+    if (warp == 0) {
+        fence_after_sync();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+    }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        cudaDriverEntryPointQueryResult q;
+        void *p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }
+    return fn;
+}
+
+bool make_map(CUtensorMap *m, const void *pool, uint64_t rows, int rows_per_box) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)kD * 2};
+    cuuint32_t box[2] = {64u, (cuuint32_t)rows_per_box};
+    cuuint32_t es[2] = {1u, 1u};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(pool), dims, strides, box, es,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int G>
+cudaError_t launch_tc_g(const CUtensorMap &mk, const CUtensorMap &mv, const TcArgs &t, dim3 grid, cudaStream_t st) {
+    static bool attr = false;
+    if (!attr) {
+        cudaError_t e = cudaFuncSetAttribute(attend_tc_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        if (e != cudaSuccess) return e;
+        attr = true;
+    }
+    attend_tc_kernel<G><<<grid, kThreads, kSmemBytes, st>>>(mk, mv, t);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int tc_max_split_tokens() { return kMaxTiles * kTile; }
+
+bool tc_supported(int dtype, int head_dim, int group, int page_size) {
+    if (dtype != IKV_BF16 || head_dim != kD) return false;
+    if (!(group == 1 || group == 2 || group == 4 || group == 7 || group == 8)) return false;
+    if (page_size % 128 == 0) return true;
+    return page_size >= 8 && 128 % page_size == 0;
+}
+
+cudaError_t launch_attend_tc(const AttendArgs &a, int group, cudaStream_t st) {
+    const int rpb = a.pv.page_size >= kTile ? kTile : a.pv.page_size;
+    // rows of every layer the launch can touch: [layers][num_pages][kv_heads][page_size]
+    const uint64_t rows = (uint64_t)(a.layer0 + a.n_layers) * a.pv.num_pages * a.pv.kv_heads * a.pv.page_size;
+    CUtensorMap mk, mv;
+    if (!make_map(&mk, a.k, rows, rpb) || !make_map(&mv, a.v, rows, rpb)) return cudaErrorInvalidValue;
+    TcArgs t{};
+    t.len = a.len;
+    t.block_table = a.pv.block_table;
+    t.num_pages = a.pv.num_pages;
+    t.page_size = a.pv.page_size;
+    t.max_pages = a.pv.max_pages;
+    t.kv_heads = a.pv.kv_heads;
+    t.rows_per_box = rpb;
+    t.q = reinterpret_cast<const __nv_bfloat16 *>(a.q);
+    t.batch = a.batch;
+    t.q_heads = a.q_heads;
+    t.layer0 = a.layer0;
+    t.n_layers = a.n_layers;
+    t.split_tokens = a.split_tokens;
+    t.n_splits = a.n_splits;
+    t.cap = a.cap;
+    t.scale_log2 = a.scale_log2;
+    t.logits = a.logits;
+    t.part_ml = a.part_ml;
+    t.part_o = a.part_o;
+    dim3 grid(a.n_splits, a.pv.kv_heads, a.batch * a.n_layers);
+    cudaError_t e;
+    switch (group) {
+        case 1: e = launch_tc_g<1>(mk, mv, t, grid, st); break;
+        case 2: e = launch_tc_g<2>(mk, mv, t, grid, st); break;
+        case 4: e = launch_tc_g<4>(mk, mv, t, grid, st); break;
+        case 7: e = launch_tc_g<7>(mk, mv, t, grid, st); break;
+        case 8: e = launch_tc_g<8>(mk, mv, t, grid, st); break;
+        default: return cudaErrorInvalidValue;
+    }
+    note_launch();
+    return e;
+}
+
+}  // namespace ikv
+
+extern "C" ikv_status ikv_device_status(uint32_t *flags) {
+    if (!flags) return ikv::report(IKV_ERR_ARG, "flags is NULL");
+    unsigned int v = 0, z = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(&v, ikv::g_tc_error, sizeof(v));
+    if (e == cudaSuccess) e = cudaMemcpyToSymbol(ikv::g_tc_error, &z, sizeof(z));
+    if (e != cudaSuccess) return ikv::report(IKV_ERR_CUDA, "ikv_device_status: %s", cudaGetErrorString(e));
+    *flags = v;
+    return IKV_OK;
+}

@@ -67,6 +67,11 @@ struct ScoreArgs {
     int32_t elig[kMaxLayersPerScorePass];
 };
 
+// tensor-core attention (bf16, head_dim 128): attend_tc.cu
+bool tc_supported(int dtype, int head_dim, int group, int page_size);
+int tc_max_split_tokens();
+cudaError_t launch_attend_tc(const AttendArgs &a, int group, cudaStream_t st);
+
 // launchers (return cudaError_t of the launch)
 cudaError_t launch_attend(const AttendArgs &a, int dtype, int head_dim, int group, cudaStream_t st);
 cudaError_t launch_combine(const CombineArgs &a, int dtype, cudaStream_t st);

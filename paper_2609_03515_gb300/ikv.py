@@ -61,6 +61,7 @@ def _load():
     sigs = {
         "ikv_last_error": ([], ctypes.c_char_p),
         "ikv_launch_count": ([], ctypes.c_int64),
+        "ikv_device_status": ([ctypes.POINTER(ctypes.c_uint32)], I32),
         "ikv_attend_workspace_size": ([SP, CP, ctypes.POINTER(SZ)], I32),
         "ikv_decode_attend_score": ([SP, CP, I32, P, P, P, P, F32, P, SZ, P], I32),
         "ikv_static_scratch_bytes": ([], SZ),
@@ -110,6 +111,12 @@ def ikv_last_error() -> str:
 
 def ikv_launch_count() -> int:
     return int(_lib.ikv_launch_count())
+
+
+def ikv_device_status() -> int:
+    v = ctypes.c_uint32(0)
+    _check(_lib.ikv_device_status(ctypes.byref(v)), "ikv_device_status")
+    return int(v.value)
 
 
 def ikv_attend_workspace_size(shape: ikv_shape, cache: ikv_cache) -> int:

@@ -181,4 +181,5 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
                     ov_rows = st.V[l][g][order]
                     rep.kv_err = max(rep.kv_err, float(np.max(np.abs(gk - ok_rows))), float(np.max(np.abs(gv - ov_rows))))
         reports.append(rep)
+    assert ikv.ikv_device_status() == 0
     return reports

@@ -60,20 +60,24 @@ def test_device_generator_matches_host_bits():
 
 # ------------------------------------------------------------------ attention + score
 ATT_CASES = [
-    # dtype, d, H, Hkv, lengths, gran
-    (gen.F32, 64, 4, 2, [512, 37, 1], ikv.IKV_GRAN_SEQ),
-    (gen.BF16, 128, 32, 8, [700, 64, 1500], ikv.IKV_GRAN_SEQ),
-    (gen.BF16, 128, 28, 4, [333, 1025], ikv.IKV_GRAN_SEQ),
-    (gen.BF16, 128, 28, 4, [333, 1025], ikv.IKV_GRAN_KVHEAD),
-    (gen.BF16, 64, 8, 8, [129, 3000], ikv.IKV_GRAN_SEQ),
-    (gen.F32, 128, 16, 2, [65, 2100], ikv.IKV_GRAN_KVHEAD),
-    (gen.BF16, 128, 16, 16, [5000], ikv.IKV_GRAN_SEQ),
+    # dtype, d, H, Hkv, lengths, gran, page_size   (bf16 / d=128 / page 8..128 | 128k -> tensor-core kernel)
+    (gen.F32, 64, 4, 2, [512, 37, 1], ikv.IKV_GRAN_SEQ, 64),
+    (gen.BF16, 128, 32, 8, [700, 64, 1500], ikv.IKV_GRAN_SEQ, 64),
+    (gen.BF16, 128, 32, 8, [700, 129, 4100], ikv.IKV_GRAN_SEQ, 16),
+    (gen.BF16, 128, 32, 8, [1, 127, 128, 2000], ikv.IKV_GRAN_SEQ, 256),
+    (gen.BF16, 128, 32, 8, [700, 64, 1500], ikv.IKV_GRAN_SEQ, 48),      # page size 48: CUDA-core kernel
+    (gen.BF16, 128, 28, 4, [333, 1025], ikv.IKV_GRAN_SEQ, 64),
+    (gen.BF16, 128, 28, 4, [333, 1025], ikv.IKV_GRAN_KVHEAD, 32),
+    (gen.BF16, 64, 8, 8, [129, 3000], ikv.IKV_GRAN_SEQ, 64),
+    (gen.F32, 128, 16, 2, [65, 2100], ikv.IKV_GRAN_KVHEAD, 64),
+    (gen.BF16, 128, 16, 16, [5000], ikv.IKV_GRAN_SEQ, 64),
+    (gen.BF16, 128, 16, 8, [30000], ikv.IKV_GRAN_SEQ, 128),            # 2 heads per group, long split
 ]
 
 
-@pytest.mark.parametrize("dt,d,H,Hkv,lens,gran", ATT_CASES)
-def test_decode_attend_score_matches_oracle(dt, d, H, Hkv, lens, gran):
-    w = gen.Workload("a", len(lens), 3, H, Hkv, d, lens, 1, dtype=dt, seed=21, page_size=64)
+@pytest.mark.parametrize("dt,d,H,Hkv,lens,gran,ps", ATT_CASES)
+def test_decode_attend_score_matches_oracle(dt, d, H, Hkv, lens, gran, ps):
+    w = gen.Workload("a", len(lens), 3, H, Hkv, d, lens, 1, dtype=dt, seed=21, page_size=ps)
     u = w.u_table()
     c = make_cache(w, gran, page_perm_seed=5)
     fill_device(c, w, torch.from_numpy(u).cuda())
@@ -90,6 +94,7 @@ def test_decode_attend_score_matches_oracle(dt, d, H, Hkv, lens, gran):
     alpha = 0.85
     ikv.ikv_decode_attend_score(c.shape(), cch, layer, q, out, score, ema, alpha, ws, ws.numel())
     torch.cuda.synchronize()
+    assert ikv.ikv_device_status() == 0
     q64 = as_f64(q_h, w)
     tol_out = 2e-2 if dt == gen.BF16 else 1e-4
     R = c.rows_per_seq
