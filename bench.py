@@ -72,7 +72,7 @@ def rank_seed(base_seed: int, rank: int) -> int:
     return base_seed + 1000 * rank
 
 
-ATTEND_KERNEL_REV = "attend_v1"
+ATTEND_KERNEL_REV = "attend_tc_v1"
 
 
 def profiled_traffic(workload: str):
@@ -80,7 +80,7 @@ def profiled_traffic(workload: str):
     or None when that summary was taken on another kernel revision or workload."""
     import re
 
-    path = os.path.join(ROOT, "profiles", f"attend_split_kernel__{workload}.md")
+    path = os.path.join(ROOT, "profiles", f"attend_tc_kernel__{workload}.md")
     if not os.path.exists(path):
         return None
     txt = open(path).read()
@@ -420,8 +420,10 @@ def run_ours(args):
     full = run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, True, dist)
     modes = {}
     if not args.no_modes:
-        for name, ww in (("lazy4", w.with_(refresh_period=4)), ("score_free", w.with_(score_free=True))):
-            r = run_mode(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, False, dist)
+        for name, ww, cm in (("lazy4", w.with_(refresh_period=4), compact_mode),
+                             ("score_free", w.with_(score_free=True), compact_mode),
+                             ("full_holefill", w, ikv.IKV_COMPACT_HOLEFILL)):
+            r = run_mode(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, False, dist)
             modes[name] = r
     qs_pin = qs_t.pin_memory()
     kn_pin = kn_dev.cpu().pin_memory()
@@ -464,7 +466,7 @@ def run_ours(args):
                    "l2": "inputs exceed L2 (K/V working set %.0f MB > 129 MB), no flush" % (kv_bytes / 1e6),
                    "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                     "traffic": traffic, "kernel": "attend_split_kernel", "peak_kind": peak_kind,
+                     "traffic": traffic, "kernel": "attend_tc_kernel", "peak_kind": peak_kind,
                      "bytes_per_launch": kv_bytes + q_bytes, "ms_per_launch": att_ms},
         "kernel_ms_per_step": full["kernel_ms"],
         "cpu_baseline": cpu,
@@ -476,6 +478,8 @@ def run_ours(args):
     }
     if modes:
         line["speedup_vs_full"] = {k: (w.batch * K * world / (v["ms"] / 1e3)) / value for k, v in modes.items()}
+        line["modes_note"] = ("lazy4 / score_free: same inputs, stable compaction; full_holefill: full refresh with "
+                              "hole-fill compaction (same kept sets, survivors not kept in order)")
     print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()

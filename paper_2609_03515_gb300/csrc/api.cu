@@ -99,7 +99,7 @@ PagedView view_of(const ikv_shape *s, const ikv_cache *c) {
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct AttendWs {
-    size_t part_ml, part_o, lse2, logits, end;
+    size_t part_ml, part_o, lse2, arrivals, logits, end;
 };
 
 AttendWs attend_ws(const ikv_shape *s, int32_t cap, int n_layers, bool logits) {
@@ -112,6 +112,8 @@ AttendWs attend_ws(const ikv_shape *s, int32_t cap, int n_layers, bool logits) {
     off = align256(off + bhl * kMaxSplits * s->head_dim * sizeof(float));
     w.lse2 = off;
     off = align256(off + bhl * sizeof(float));
+    w.arrivals = off;
+    off = align256(off + (size_t)s->batch * n_layers * s->kv_heads * sizeof(int32_t));
     w.logits = off;
     if (logits) off = align256(off + bhl * (size_t)cap * sizeof(float));
     w.end = off;
@@ -173,7 +175,8 @@ void choose_splits(const ikv_shape *s, int n_layers, int32_t max_len, int granul
 // attention (+ combine) over layers [layer0, layer0 + n_layers)
 ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, int32_t n_layers, int32_t max_len,
                       const void *q, void *out, void *ws, const AttendWs &w, bool logits, int32_t *split_out,
-                      int32_t *nsplit_out, cudaStream_t st, const ikv_timing *tm = nullptr) {
+                      int32_t *nsplit_out, cudaStream_t st, const ikv_timing *tm = nullptr,
+                      bool counters_zeroed = false) {
     AttendArgs a{};
     a.k = c->k;
     a.v = c->v;
@@ -197,26 +200,32 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
     a.cap = cap_of(c);
     a.part_ml = at<float>(ws, w.part_ml);
     a.part_o = at<float>(ws, w.part_o);
-    if (max_len > 0) {
-        if (tc)
-            IKV_TRY_CUDA(launch_attend_tc(a, group, st), "tensor-core attend launch");
-        else
-            IKV_TRY_CUDA(launch_attend(a, s->dtype, s->head_dim, group, st), "attend launch");
+    if (tc) {
+        // fused combine: the last split of each unit writes out and lse2
+        int32_t *arr = at<int32_t>(ws, w.arrivals);
+        if (!counters_zeroed)
+            IKV_TRY_CUDA(cudaMemsetAsync(arr, 0, sizeof(int32_t) * (size_t)s->batch * n_layers * s->kv_heads, st),
+                         "cudaMemsetAsync");
+        TcOutputs o{out, at<float>(ws, w.lse2), arr};
+        if (max_len > 0) IKV_TRY_CUDA(launch_attend_tc(a, o, group, st), "tensor-core attend launch");
+        if (tm && tm->attend_end) IKV_TRY_CUDA(cudaEventRecord(tm->attend_end, st), "cudaEventRecord");
+    } else {
+        if (max_len > 0) IKV_TRY_CUDA(launch_attend(a, s->dtype, s->head_dim, group, st), "attend launch");
+        if (tm && tm->attend_end) IKV_TRY_CUDA(cudaEventRecord(tm->attend_end, st), "cudaEventRecord");
+        CombineArgs cb{};
+        cb.len = c->len;
+        cb.batch = s->batch;
+        cb.q_heads = s->q_heads;
+        cb.n_layers = n_layers;
+        cb.split_tokens = a.split_tokens;
+        cb.n_splits = a.n_splits;
+        cb.head_dim = s->head_dim;
+        cb.part_ml = a.part_ml;
+        cb.part_o = a.part_o;
+        cb.out = out;
+        cb.lse2 = at<float>(ws, w.lse2);
+        IKV_TRY_CUDA(launch_combine(cb, s->dtype, st), "combine launch");
     }
-    if (tm && tm->attend_end) IKV_TRY_CUDA(cudaEventRecord(tm->attend_end, st), "cudaEventRecord");
-    CombineArgs cb{};
-    cb.len = c->len;
-    cb.batch = s->batch;
-    cb.q_heads = s->q_heads;
-    cb.n_layers = n_layers;
-    cb.split_tokens = a.split_tokens;
-    cb.n_splits = a.n_splits;
-    cb.head_dim = s->head_dim;
-    cb.part_ml = a.part_ml;
-    cb.part_o = a.part_o;
-    cb.out = out;
-    cb.lse2 = at<float>(ws, w.lse2);
-    IKV_TRY_CUDA(launch_combine(cb, s->dtype, st), "combine launch");
     if (split_out) *split_out = a.split_tokens;
     if (nsplit_out) *nsplit_out = a.n_splits;
     return IKV_OK;
@@ -383,7 +392,8 @@ ikv_status ikv_compact_kv(const ikv_shape *shape, ikv_cache *cache, const int32_
 }
 
 static ikv_status append_impl(const ikv_shape *shape, ikv_cache *cache, const void *k_new, const void *v_new,
-                              float *ema, int32_t init_mean, int32_t *done, cudaStream_t stream) {
+                              float *ema, int32_t init_mean, int32_t *done, cudaStream_t stream,
+                              bool counters_zeroed = false) {
     AppendArgs a{};
     a.k = cache->k;
     a.v = cache->v;
@@ -401,7 +411,8 @@ static ikv_status append_impl(const ikv_shape *shape, ikv_cache *cache, const vo
     a.ema = ema;
     a.init_mean = ema ? init_mean : 0;
     a.done = done;
-    IKV_TRY_CUDA(cudaMemsetAsync(done, 0, sizeof(int32_t) * shape->batch, stream), "cudaMemsetAsync");
+    if (!counters_zeroed)
+        IKV_TRY_CUDA(cudaMemsetAsync(done, 0, sizeof(int32_t) * shape->batch, stream), "cudaMemsetAsync");
     IKV_TRY_CUDA(launch_append(a, stream), "append launch");
     return IKV_OK;
 }
@@ -462,11 +473,18 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     const int32_t L1 = cache->max_len + 1;
     const ikv_timing *tm = p->timing;
 
+    // control words (append and split-arrival counters) start at zero
+    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.at.arrivals), 0, w.at.logits - w.at.arrivals, stream),
+                 "cudaMemsetAsync");
+    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.done), 0, sizeof(int32_t) * shape->batch, stream),
+                 "cudaMemsetAsync");
     if (tm && (e = record(tm->begin, stream))) return e;
     const int32_t init_mean = refresh ? (p->refresh_init == IKV_INIT_MEAN) : 1;
-    if ((e = append_impl(shape, cache, k_new, v_new, ema, init_mean, at<int32_t>(ws, w.done), stream))) return e;
+    if ((e = append_impl(shape, cache, k_new, v_new, ema, init_mean, at<int32_t>(ws, w.done), stream, true)))
+        return e;
     if (tm && (e = record(tm->append_end, stream))) return e;
-    if ((e = run_attend(shape, cache, 0, shape->layers, L1, q, out, ws, w.at, scoring, nullptr, nullptr, stream, tm)))
+    if ((e = run_attend(shape, cache, 0, shape->layers, L1, q, out, ws, w.at, scoring, nullptr, nullptr, stream, tm,
+                        true)))
         return e;
     if (tm && (e = record(tm->combine_end, stream))) return e;
     if (scoring && (e = run_score(shape, cache, shape->layers, elig, n_elig, L1, ws, w.at, p->alpha, ema, nullptr, stream)))

@@ -48,7 +48,7 @@ constexpr int kOffBar = kOffRed + 4 * kN * 4;
 // barriers: full[kNst], empty[kNst], s_full, p_full[2], p_empty[2], o_full
 constexpr int kNumBar = 2 * kNst + 6;
 constexpr int kOffMisc = kOffBar + kNumBar * 8;
-constexpr int kSmemBytes = kOffMisc + 16 + 1024;   // + slack for 1024-byte alignment
+constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // misc: tmem slot, abort flag, last-split flag   // + slack for 1024-byte alignment
 
 enum : unsigned { kErrTimeout = 1u };
 
@@ -61,6 +61,9 @@ struct TcArgs {
     float scale_log2;
     float *logits;              // may be null
     float *part_ml, *part_o;
+    __nv_bfloat16 *out;         // [n_layers][batch][H][128]
+    float *lse2;                // [batch][n_layers][H]
+    int32_t *arrivals;          // [batch][n_layers][kv_heads], zero on entry, left zero
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -190,9 +193,18 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int l = a.layer0 + li;
     const int L = a.len[b];
     const int t0 = s * a.split_tokens;
-    if (t0 >= L) return;
+    if (t0 >= L) {
+        if (s == 0) {  // empty sequence: zero output, log-sum-exp -inf
+            for (int i = threadIdx.x; i < G * kD; i += kThreads)
+                a.out[(((int64_t)li * a.batch + b) * a.q_heads + (int64_t)g * G) * kD + i] = __float2bfloat16_rn(0.f);
+            if (threadIdx.x < G)
+                a.lse2[((int64_t)b * a.n_layers + li) * a.q_heads + (int64_t)g * G + threadIdx.x] = -INFINITY;
+        }
+        return;
+    }
     const int t1 = min(t0 + a.split_tokens, L);
     const int n = (t1 - t0 + kTile - 1) / kTile;
+    const int ns_active = (L + a.split_tokens - 1) / a.split_tokens;
     if (n > kMaxTiles) {  // the host sizes splits to fit TMEM; refuse rather than overrun
         if (threadIdx.x == 0) atomicOr(&g_tc_error, 2u);
         return;
@@ -407,6 +419,34 @@ __global__ void __launch_bounds__(kThreads, 2)
                 a.part_ml[((pbase + (int64_t)tid * a.n_splits) + s) * 2 + 1] = ss;
             }
         }
+        // The last split of (sequence, layer, kv head) to finish merges every
+        // split's partial into the output and the per-head log-sum-exp.  Arrival
+        // counter only: no CTA waits for another.
+        __threadfence();
+        __syncwarp();
+        softmax_bar();
+        int *last_flag = reinterpret_cast<int *>(sm + kOffMisc + 8);
+        const int64_t unit = ((int64_t)b * a.n_layers + li) * a.kv_heads + g;
+        if (tid == 0) *last_flag = (atomicAdd(&a.arrivals[unit], 1) == ns_active - 1) ? 1 : 0;
+        softmax_bar();
+        if (*last_flag && ok) {
+            __threadfence();
+            const int64_t pbase = (((int64_t)b * a.n_layers + li) * H + (int64_t)g * G) * a.n_splits;
+            for (int h = 0; h < G; ++h) {
+                const float *ml = a.part_ml + (pbase + (int64_t)h * a.n_splits) * 2;
+                float M = -INFINITY;
+                for (int q = 0; q < ns_active; ++q) M = fmaxf(M, __ldcg(ml + 2 * q));
+                float wsum = 0.f, acc = 0.f;
+                for (int q = 0; q < ns_active; ++q) {
+                    const float w = exp2f(__ldcg(ml + 2 * q) - M);
+                    wsum += __ldcg(ml + 2 * q + 1) * w;
+                    acc += __ldcg(a.part_o + ((pbase + (int64_t)h * a.n_splits) + q) * kD + tid) * w;
+                }
+                a.out[(((int64_t)li * a.batch + b) * H + (int64_t)g * G + h) * kD + tid] = __float2bfloat16_rn(acc / wsum);
+                if (tid == 0) a.lse2[((int64_t)b * a.n_layers + li) * H + (int64_t)g * G + h] = M + log2f(wsum);
+            }
+            if (tid == 0) a.arrivals[unit] = 0;
+        }
     }
     fence_before_sync();
     __syncthreads();
@@ -464,7 +504,7 @@ bool tc_supported(int dtype, int head_dim, int group, int page_size) {
     return page_size >= 8 && 128 % page_size == 0;
 }
 
-cudaError_t launch_attend_tc(const AttendArgs &a, int group, cudaStream_t st) {
+cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group, cudaStream_t st) {
     const int rpb = a.pv.page_size >= kTile ? kTile : a.pv.page_size;
     // rows of every layer the launch can touch: [layers][num_pages][kv_heads][page_size]
     const uint64_t rows = (uint64_t)(a.layer0 + a.n_layers) * a.pv.num_pages * a.pv.kv_heads * a.pv.page_size;
@@ -490,6 +530,9 @@ cudaError_t launch_attend_tc(const AttendArgs &a, int group, cudaStream_t st) {
     t.logits = a.logits;
     t.part_ml = a.part_ml;
     t.part_o = a.part_o;
+    t.out = reinterpret_cast<__nv_bfloat16 *>(o.out);
+    t.lse2 = o.lse2;
+    t.arrivals = o.arrivals;
     dim3 grid(a.n_splits, a.pv.kv_heads, a.batch * a.n_layers);
     cudaError_t e;
     switch (group) {

@@ -70,7 +70,13 @@ struct ScoreArgs {
 // tensor-core attention (bf16, head_dim 128): attend_tc.cu
 bool tc_supported(int dtype, int head_dim, int group, int page_size);
 int tc_max_split_tokens();
-cudaError_t launch_attend_tc(const AttendArgs &a, int group, cudaStream_t st);
+// the tensor-core kernel also merges its splits (last CTA of each unit)
+struct TcOutputs {
+    void *out;                  // [n_layers][batch][H][128] bf16
+    float *lse2;                // [batch][n_layers][H]
+    int32_t *arrivals;          // [batch][n_layers][kv_heads] zeroed before the launch
+};
+cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group, cudaStream_t st);
 
 // launchers (return cudaError_t of the launch)
 cudaError_t launch_attend(const AttendArgs &a, int dtype, int head_dim, int group, cudaStream_t st);
