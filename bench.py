@@ -72,7 +72,7 @@ def rank_seed(base_seed: int, rank: int) -> int:
     return base_seed + 1000 * rank
 
 
-ATTEND_KERNEL_REV = "attend_tc_v1"
+ATTEND_KERNEL_REV = "attend_tc_v2"
 
 
 def profiled_traffic(workload: str):

@@ -98,6 +98,8 @@ PagedView view_of(const ikv_shape *s, const ikv_cache *c) {
 // ---- workspace layout ------------------------------------------------------
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
+int32_t logit_stride(int32_t cap) { return (cap + 127) / 128 * 128; }
+
 struct AttendWs {
     size_t part_ml, part_o, lse2, arrivals, logits, end;
 };
@@ -115,7 +117,7 @@ AttendWs attend_ws(const ikv_shape *s, int32_t cap, int n_layers, bool logits) {
     w.arrivals = off;
     off = align256(off + (size_t)s->batch * n_layers * s->kv_heads * sizeof(int32_t));
     w.logits = off;
-    if (logits) off = align256(off + bhl * (size_t)cap * sizeof(float));
+    if (logits) off = align256(off + bhl * (size_t)logit_stride(cap) * sizeof(float));
     w.end = off;
     return w;
 }
@@ -191,13 +193,17 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
     const uint64_t pool_rows = (uint64_t)(layer0 + n_layers) * c->num_pages * s->kv_heads * c->page_size;
     const bool tc = tc_supported(s->dtype, s->head_dim, group, c->page_size) &&
                     (int64_t)max_len <= (int64_t)kMaxSplits * tc_max_split_tokens() && pool_rows < (1ull << 31);
-    if (tc)
-        choose_splits(s, n_layers, max_len, 128, tc_max_split_tokens(), &a.split_tokens, &a.n_splits);
-    else
+    if (tc) {
+        int32_t it = 0, nc = 0;
+        tc_plan(max_len, (int64_t)s->batch * n_layers * s->kv_heads, sm_count(), &it, &nc);
+        a.split_tokens = it * 128;
+        a.n_splits = nc;
+    } else
         choose_splits(s, n_layers, max_len, kTileTokens, 1 << 30, &a.split_tokens, &a.n_splits);
     a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)s->head_dim));
     a.logits = logits ? at<float>(ws, w.logits) : nullptr;
     a.cap = cap_of(c);
+    a.lstride = logit_stride(a.cap);
     a.part_ml = at<float>(ws, w.part_ml);
     a.part_o = at<float>(ws, w.part_o);
     if (tc) {
@@ -207,7 +213,7 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
             IKV_TRY_CUDA(cudaMemsetAsync(arr, 0, sizeof(int32_t) * (size_t)s->batch * n_layers * s->kv_heads, st),
                          "cudaMemsetAsync");
         TcOutputs o{out, at<float>(ws, w.lse2), arr};
-        if (max_len > 0) IKV_TRY_CUDA(launch_attend_tc(a, o, group, st), "tensor-core attend launch");
+        if (max_len > 0) IKV_TRY_CUDA(launch_attend_tc(a, o, group, sm_count(), st), "tensor-core attend launch");
         if (tm && tm->attend_end) IKV_TRY_CUDA(cudaEventRecord(tm->attend_end, st), "cudaEventRecord");
     } else {
         if (max_len > 0) IKV_TRY_CUDA(launch_attend(a, s->dtype, s->head_dim, group, st), "attend launch");
@@ -244,6 +250,7 @@ ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, c
         sa.n_layers = n_layers;
         sa.cap = cap_of(c);
         sa.logits = at<float>(ws, w.logits);
+        sa.lstride = logit_stride(cap_of(c));
         sa.lse2 = at<float>(ws, w.lse2);
         sa.n_elig = n_elig - k0 < kMaxLayersPerScorePass ? n_elig - k0 : kMaxLayersPerScorePass;
         for (int k = 0; k < sa.n_elig; ++k) sa.elig[k] = elig[k0 + k];

@@ -225,7 +225,7 @@ __global__ void __launch_bounds__(kAttendThreads, 2) attend_split_kernel(const A
                       red[(3 * G + h) * C::TT + j];
             if (j < nv) {
                 if (LOGITS)
-                    a.logits[((((int64_t)b * a.n_layers + li) * H) + g * G + h) * (int64_t)a.cap + tbase + j] = z;
+                    a.logits[((((int64_t)b * a.n_layers + li) * H) + g * G + h) * (int64_t)a.lstride + tbase + j] = z;
             } else {
                 z = -INFINITY;
             }

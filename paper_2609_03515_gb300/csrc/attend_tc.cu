@@ -1,8 +1,12 @@
 // Tensor-core split-K decode attention with logits, bf16, head_dim 128 (sm_103a).
 //
-// Same contract as attend_split_kernel (one CTA per split, kv head, sequence x
-// layer; writes log2-domain logits and per-split (max, sum, O) partials), built
-// from Blackwell pieces:
+// The cache of every (sequence, layer, kv head) unit is cut into chunks of up to
+// 15 tiles of 128 tokens; one CTA handles one chunk (the G query heads of its
+// kv head), writes that chunk's log2-domain logits and its (max, sum, O)
+// partial, and the unit's last chunk to finish merges the partials into the
+// output and the per-head log-sum-exp (arrival counter, no waiting).  The 1-D
+// grid is chunk-major, so every unit's short remainder chunk is dispatched last
+// and fills the final wave.  Two CTAs share an SM.  Built from Blackwell pieces:
 //   * TMA (cp.async.bulk.tensor.2d, 128-byte swizzle) streams 128-token K and V
 //     tiles out of the paged pool (one box per page segment and 64-column half)
 //     into a 3-stage ring guarded by mbarriers;
@@ -10,8 +14,8 @@
 //       S_i[128 tokens x 16] = K_i[128 x 128] . Q^T[128 x 16]   (Q: G heads, zero-padded to 16)
 //       O[128 dims x 16]    += V_i^T[128 x 128] . P_i^T[128 x 16]
 //     with K-major operands for QK and an MN-major (transposed) V for PV;
-//   * the softmax runs as two sweeps over the S tiles kept in TMEM: the split
-//     maximum per head, then exp2, logits write-out, row sums and the bf16 P
+//   * the softmax runs as two sweeps over the S tiles kept in TMEM: the chunk
+//     maximum per head, then logits write-out, exp2, row sums and the bf16 P
 //     operand (double-buffered in shared memory) that feeds the PV MMA.
 // Warp roles (192 threads): warps 0-3 own TMEM lanes 0-127 (softmax, epilogue),
 // warp 4 issues TMA loads, warp 5 issues MMAs.  Every mbarrier wait is bounded;
@@ -59,7 +63,8 @@ struct TcArgs {
     const __nv_bfloat16 *q;     // q + ((li*batch + b)*H + h)*128
     int32_t batch, q_heads, layer0, n_layers, split_tokens, n_splits, cap;
     float scale_log2;
-    float *logits;              // may be null
+    float *logits;              // may be null; rows of lstride floats
+    int32_t lstride;            // logits row stride, a multiple of 128
     float *part_ml, *part_o;
     __nv_bfloat16 *out;         // [n_layers][batch][H][128]
     float *lse2;                // [batch][n_layers][H]
@@ -188,8 +193,13 @@ __global__ void __launch_bounds__(kThreads, 2)
     unsigned char *sm = smem_raw + (base - raw);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int s = blockIdx.x, g = blockIdx.y;
-    const int b = blockIdx.z % a.batch, li = blockIdx.z / a.batch;
+    // 1-D grid, chunk-major: CTA i handles chunk i / n_units of unit i % n_units, so every
+    // unit's short remainder chunk is dispatched last and fills the final wave
+    const int n_units = a.batch * a.n_layers * a.kv_heads;
+    const int s = blockIdx.x / n_units;
+    const int unit_id = blockIdx.x % n_units;
+    const int g = unit_id % a.kv_heads;
+    const int b = (unit_id / a.kv_heads) % a.batch, li = (unit_id / a.kv_heads) / a.batch;
     const int l = a.layer0 + li;
     const int L = a.len[b];
     const int t0 = s * a.split_tokens;
@@ -265,20 +275,24 @@ __global__ void __launch_bounds__(kThreads, 2)
         // ---------------- TMA producer
         if (lane == 0) {
             const int boxes = kTile / a.rows_per_box;
+            // pool row of box bx of load j (loads 0..n-1: K tiles, n..2n-1: V tiles)
+            auto box_row = [&](int j, int bx) {
+                const int tile = j < n ? j : j - n;
+                const int tok = t0 + tile * kTile + bx * a.rows_per_box;
+                int lp = tok / a.page_size;
+                if (lp >= a.max_pages) lp = a.max_pages - 1;
+                const int page = a.block_table[(int64_t)b * a.max_pages + lp];
+                return ((l * a.num_pages + page) * a.kv_heads + g) * a.page_size + tok % a.page_size;
+            };
             int issued = 0;
             for (int j = 0; j < 2 * n; ++j) {
                 const int st = j % kNst;
                 if (j >= kNst && !mbar_wait(empty(st), ((j / kNst) - 1) & 1, abort_flag)) break;
                 mbar_expect_tx(full(st), kStage);
-                const int tile = j < n ? j : j - n;
                 const CUtensorMap *tm = j < n ? &tmK : &tmV;
                 const uint32_t dst = base + st * kStage;
                 for (int bx = 0; bx < boxes; ++bx) {
-                    const int tok = t0 + tile * kTile + bx * a.rows_per_box;
-                    int lp = tok / a.page_size;
-                    if (lp >= a.max_pages) lp = a.max_pages - 1;
-                    const int page = a.block_table[(int64_t)b * a.max_pages + lp];
-                    const int row = ((l * a.num_pages + page) * a.kv_heads + g) * a.page_size + tok % a.page_size;
+                    const int row = box_row(j, bx);
                     tma_load_2d(dst + bx * a.rows_per_box * 128, tm, 0, row, full(st));
                     tma_load_2d(dst + kHalf + bx * a.rows_per_box * 128, tm, 64, row, full(st));
                 }
@@ -339,6 +353,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         bool ok = __all_sync(0xffffffffu, mbar_wait(s_full, 0, abort_flag));
         fence_after_sync();
+        // sweep 1: split maximum
         if (ok) {
             for (int i = 0; i < n; ++i) {
                 float v[NC];
@@ -363,7 +378,10 @@ __global__ void __launch_bounds__(kThreads, 2)
         for (int h = 0; h < G; ++h) mx[h] = fmaxf(fmaxf(red[h], red[kN + h]), fmaxf(red[2 * kN + h], red[3 * kN + h]));
         softmax_bar();
 
-        const int64_t lbase = (((int64_t)b * a.n_layers + li) * H + (int64_t)g * G) * a.cap;
+        // sweep 2: logits write-out, exp2, row sums and the P operand of each tile.  The
+        // logits stores sit here, interleaved with the V stream; issued as a burst in
+        // sweep 1 they measured slower.
+        const int64_t lbase = (((int64_t)b * a.n_layers + li) * H + (int64_t)g * G) * a.lstride;
         for (int i = 0; i < n && ok; ++i) {
             if (i >= 2 && !(ok = __all_sync(0xffffffffu, mbar_wait(p_empty(i & 1), ((i >> 1) - 1) & 1, abort_flag))))
                 break;
@@ -377,7 +395,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 const float z = v[h] * a.scale_log2;
                 float p = 0.f;
                 if (valid) {
-                    if (a.logits) a.logits[lbase + (int64_t)h * a.cap + tok] = z;
+                    if (a.logits) a.logits[lbase + (int64_t)h * a.lstride + tok] = z;
                     p = exp2f(z - mx[h]);
                     sum[h] += p;
                 }
@@ -432,18 +450,49 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (*last_flag && ok) {
             __threadfence();
             const int64_t pbase = (((int64_t)b * a.n_layers + li) * H + (int64_t)g * G) * a.n_splits;
+            // online merge over the unit's splits, four splits x all heads per round so that
+            // every load of a round is in flight at once
+            float M[G], ws[G], acc[G];
+#pragma unroll
             for (int h = 0; h < G; ++h) {
-                const float *ml = a.part_ml + (pbase + (int64_t)h * a.n_splits) * 2;
-                float M = -INFINITY;
-                for (int q = 0; q < ns_active; ++q) M = fmaxf(M, __ldcg(ml + 2 * q));
-                float wsum = 0.f, acc = 0.f;
-                for (int q = 0; q < ns_active; ++q) {
-                    const float w = exp2f(__ldcg(ml + 2 * q) - M);
-                    wsum += __ldcg(ml + 2 * q + 1) * w;
-                    acc += __ldcg(a.part_o + ((pbase + (int64_t)h * a.n_splits) + q) * kD + tid) * w;
+                M[h] = -INFINITY;
+                ws[h] = 0.f;
+                acc[h] = 0.f;
+            }
+            constexpr int MQ = G <= 4 ? 4 : 2;  // chunks per round (register budget)
+            for (int q0 = 0; q0 < ns_active; q0 += MQ) {
+                float mq[MQ][G], lq[MQ][G], oq[MQ][G];
+#pragma unroll
+                for (int j = 0; j < MQ; ++j)
+#pragma unroll
+                    for (int h = 0; h < G; ++h) {
+                        const int q = q0 + j;
+                        const int64_t slot = pbase + (int64_t)h * a.n_splits + q;
+                        mq[j][h] = q < ns_active ? __ldcg(a.part_ml + slot * 2) : -INFINITY;
+                        lq[j][h] = q < ns_active ? __ldcg(a.part_ml + slot * 2 + 1) : 0.f;
+                        oq[j][h] = q < ns_active ? __ldcg(a.part_o + slot * kD + tid) : 0.f;
+                    }
+#pragma unroll
+                for (int h = 0; h < G; ++h) {
+                    float mn = M[h];
+#pragma unroll
+                    for (int j = 0; j < MQ; ++j) mn = fmaxf(mn, mq[j][h]);
+                    const float sc = exp2f(M[h] - mn);  // 0 while M is -inf
+                    ws[h] *= sc;
+                    acc[h] *= sc;
+#pragma unroll
+                    for (int j = 0; j < MQ; ++j) {
+                        const float wq = exp2f(mq[j][h] - mn);  // 0 for padding slots
+                        ws[h] += lq[j][h] * wq;
+                        acc[h] += oq[j][h] * wq;
+                    }
+                    M[h] = mn;
                 }
-                a.out[(((int64_t)li * a.batch + b) * H + (int64_t)g * G + h) * kD + tid] = __float2bfloat16_rn(acc / wsum);
-                if (tid == 0) a.lse2[((int64_t)b * a.n_layers + li) * H + (int64_t)g * G + h] = M + log2f(wsum);
+            }
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                a.out[(((int64_t)li * a.batch + b) * H + (int64_t)g * G + h) * kD + tid] = __float2bfloat16_rn(acc[h] / ws[h]);
+                if (tid == 0) a.lse2[((int64_t)b * a.n_layers + li) * H + (int64_t)g * G + h] = M[h] + log2f(ws[h]);
             }
             if (tid == 0) a.arrivals[unit] = 0;
         }
@@ -497,6 +546,25 @@ cudaError_t launch_tc_g(const CUtensorMap &mk, const CUtensorMap &mv, const TcAr
 
 int tc_max_split_tokens() { return kMaxTiles * kTile; }
 
+#ifndef IKV_TC_WAVES
+#define IKV_TC_WAVES 2
+#endif
+// Chunking of the flattened (unit, tile) work for lengths up to max_len: enough
+// chunks for about IKV_TC_WAVES waves of two CTAs per SM, each chunk 1..15 tiles,
+// at most kMaxSplits chunks per unit.
+void tc_plan(int32_t max_len, int64_t units, int sms, int32_t *item_tiles, int32_t *n_chunks) {
+    const int64_t tiles = ((int64_t)max_len + kTile - 1) / kTile;
+    const int64_t target = (int64_t)2 * sms * IKV_TC_WAVES;
+    int64_t c = (units * tiles + target - 1) / target;
+    const int64_t cmin = (tiles + kMaxSplits - 1) / kMaxSplits;
+    if (c < cmin) c = cmin;
+    if (c < 1) c = 1;
+    if (c > kMaxTiles) c = kMaxTiles;
+    *item_tiles = (int32_t)c;
+    const int64_t n = (tiles + c - 1) / c;
+    *n_chunks = (int32_t)(n < 1 ? 1 : n);
+}
+
 bool tc_supported(int dtype, int head_dim, int group, int page_size) {
     if (dtype != IKV_BF16 || head_dim != kD) return false;
     if (!(group == 1 || group == 2 || group == 4 || group == 7 || group == 8)) return false;
@@ -504,7 +572,8 @@ bool tc_supported(int dtype, int head_dim, int group, int page_size) {
     return page_size >= 8 && 128 % page_size == 0;
 }
 
-cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group, cudaStream_t st) {
+cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group, int sms, cudaStream_t st) {
+    (void)sms;
     const int rpb = a.pv.page_size >= kTile ? kTile : a.pv.page_size;
     // rows of every layer the launch can touch: [layers][num_pages][kv_heads][page_size]
     const uint64_t rows = (uint64_t)(a.layer0 + a.n_layers) * a.pv.num_pages * a.pv.kv_heads * a.pv.page_size;
@@ -528,12 +597,13 @@ cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group,
     t.cap = a.cap;
     t.scale_log2 = a.scale_log2;
     t.logits = a.logits;
+    t.lstride = a.lstride;
     t.part_ml = a.part_ml;
     t.part_o = a.part_o;
     t.out = reinterpret_cast<__nv_bfloat16 *>(o.out);
     t.lse2 = o.lse2;
     t.arrivals = o.arrivals;
-    dim3 grid(a.n_splits, a.pv.kv_heads, a.batch * a.n_layers);
+    dim3 grid(a.n_splits * a.pv.kv_heads * a.batch * a.n_layers);
     cudaError_t e;
     switch (group) {
         case 1: e = launch_tc_g<1>(mk, mv, t, grid, st); break;

@@ -11,7 +11,7 @@ namespace ikv {
 
 constexpr int kTileTokens = 64;    // K/V rows staged per attention tile
 constexpr int kAttendThreads = 128;
-constexpr int kMaxSplits = 64;     // split-K partitions per (seq, layer, kv head)
+constexpr int kMaxSplits = 128;    // split-K partitions per (seq, layer, kv head)
 constexpr int kMinSplitTokens = 256;
 constexpr int kMaxLayersPerScorePass = 32;
 constexpr int kMaxLayers = 512;
@@ -40,8 +40,9 @@ struct AttendArgs {
     int32_t batch, q_heads, layer0, n_layers;
     int32_t split_tokens, n_splits;
     float scale_log2;           // log2(e) / sqrt(d)
-    float *logits;              // [batch][n_layers][H][cap] log2-domain logits, or null
+    float *logits;              // [batch][n_layers][H][lstride] log2-domain logits, or null
     int32_t cap;
+    int32_t lstride;            // logits row stride: cap rounded up to a multiple of 128
     float *part_ml;             // [batch][n_layers][H][n_splits][2]  (running max, sum) in log2 domain
     float *part_o;              // [batch][n_layers][H][n_splits][D]  unnormalised partial output
 };
@@ -57,7 +58,8 @@ struct CombineArgs {
 struct ScoreArgs {
     const int32_t *len;         // [batch]
     int32_t batch, q_heads, kv_heads, rows_per_seq, n_layers, cap;
-    const float *logits;        // [batch][n_layers][H][cap]
+    const float *logits;        // [batch][n_layers][H][lstride]
+    int32_t lstride;
     const float *lse2;          // [batch][n_layers][H]
     int32_t n_elig;             // eligible local layers, in ascending order
     const int32_t *elig_dev;    // unused placeholder
@@ -76,7 +78,8 @@ struct TcOutputs {
     float *lse2;                // [batch][n_layers][H]
     int32_t *arrivals;          // [batch][n_layers][kv_heads] zeroed before the launch
 };
-cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group, cudaStream_t st);
+void tc_plan(int32_t max_len, int64_t units, int sms, int32_t *item_tiles, int32_t *n_chunks);
+cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group, int sms, cudaStream_t st);
 
 // launchers (return cudaError_t of the launch)
 cudaError_t launch_attend(const AttendArgs &a, int dtype, int head_dim, int group, cudaStream_t st);

@@ -38,12 +38,12 @@ __global__ void __launch_bounds__(kScoreWarps * 32) score_ema_kernel(const Score
     const float inv = 1.f / (float)nh;
     if (warp < a.n_elig) {
         const int li = a.elig[warp];
-        const float *zl = a.logits + (((int64_t)b * a.n_layers + li) * H) * (int64_t)a.cap;
+        const float *zl = a.logits + (((int64_t)b * a.n_layers + li) * H) * (int64_t)a.lstride;
         const float *ll = a.lse2 + ((int64_t)b * a.n_layers + li) * H;
         float acc = 0.f;
         if (valid) {
 #pragma unroll 8
-            for (int h = h0; h < h0 + nh; ++h) acc += exp2f(zl[(int64_t)h * a.cap + i] - ll[h]);
+            for (int h = h0; h < h0 + nh; ++h) acc += exp2f(zl[(int64_t)h * a.lstride + i] - ll[h]);
         }
         sl[warp][lane] = acc * inv;
     }
