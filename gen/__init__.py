@@ -84,6 +84,7 @@ def host_lib():
         lib.ikvgen_u_table.argtypes = [U64, I32, I32, I32, P]
         lib.ikvgen_kv_block.argtypes = [ctypes.POINTER(Spec), P, I32, I32, I64, I64, I32, P, P]
         lib.ikvgen_heavy_flags.argtypes = [ctypes.POINTER(Spec), I32, I64, I64, P]
+        lib.ikvgen_kv_rows_at.argtypes = [ctypes.POINTER(Spec), P, I32, I32, P, I64, I32, P, P]
         lib.ikvgen_queries.argtypes = [U64, I32, I32, I32, I32, I32, P, I32, I32, I32, I32, P]
         lib.ikvgen_lengths.argtypes = [U64, I32, I32, I32, P]
         lib.ikvgen_normals.argtypes = [U64, U64, I64, P]
@@ -185,6 +186,22 @@ class Workload:
             v = np.empty(shape, np.float32)
         host_lib().ikvgen_kv_block(ctypes.byref(sp), _ptr(u), b, layer, p0, count, dt, _ptr(k), _ptr(v))
         if dt == BF16:
+            return bf16_to_f32(k), bf16_to_f32(v)
+        return k, v
+
+    def kv_rows(self, b: int, layer: int, positions, u: Optional[np.ndarray] = None):
+        """Keys and values [kv_heads][count][d] at arbitrary original positions (float32
+        arrays holding exactly the stored values)."""
+        u = self.u_table() if u is None else u
+        pos = np.ascontiguousarray(np.asarray(positions, dtype=np.int64))
+        n = pos.shape[0]
+        shape = (self.kv_heads, n, self.head_dim)
+        dt = np.uint16 if self.dtype == BF16 else np.float32
+        k = np.empty(shape, dt)
+        v = np.empty(shape, dt)
+        sp = self.spec()
+        host_lib().ikvgen_kv_rows_at(ctypes.byref(sp), _ptr(u), b, layer, _ptr(pos), n, self.dtype, _ptr(k), _ptr(v))
+        if self.dtype == BF16:
             return bf16_to_f32(k), bf16_to_f32(v)
         return k, v
 

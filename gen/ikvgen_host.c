@@ -51,6 +51,25 @@ void ikvgen_kv_block(const ikvgen_spec *s, const float *u, int32_t b, int32_t l,
         }
 }
 
+/* Keys and values of sequence b, layer l at the listed positions (any order).
+ * out_k / out_v: [kv_heads][count][d] (either may be NULL). */
+void ikvgen_kv_rows_at(const ikvgen_spec *s, const float *u, int32_t b, int32_t l, const int64_t *positions,
+                       int64_t count, int32_t dtype, void *out_k, void *out_v) {
+    const int32_t d = s->head_dim;
+#pragma omp parallel for schedule(static) collapse(2)
+    for (int32_t g = 0; g < s->kv_heads; ++g)
+        for (int64_t i = 0; i < count; ++i) {
+            int64_t p = positions[i];
+            int heavy = ikvgen_is_heavy(s, b, p);
+            const float *ug = u + ((int64_t)l * s->kv_heads + g) * d;
+            int64_t base = ((int64_t)g * count + i) * d;
+            for (int32_t e = 0; e < d; ++e) {
+                if (out_k) store(out_k, base + e, ikvgen_key_elem(s, b, l, g, p, e, heavy, ug[e]), dtype);
+                if (out_v) store(out_v, base + e, ikvgen_value_elem(s, b, l, g, p, e), dtype);
+            }
+        }
+}
+
 /* Heavy-position flags for positions [p0, p0+count) of sequence b. */
 void ikvgen_heavy_flags(const ikvgen_spec *s, int32_t b, int64_t p0, int64_t count, uint8_t *out) {
     for (int64_t i = 0; i < count; ++i) out[i] = (uint8_t)ikvgen_is_heavy(s, b, p0 + i);

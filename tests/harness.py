@@ -183,3 +183,80 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
         reports.append(rep)
     assert ikv.ikv_device_status() == 0
     return reports
+
+
+def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1), page_perm_seed: Optional[int] = 7):
+    """Full-size lock-step for a few sequences of a workload (GRAN_SEQ).
+
+    The GPU decodes the whole batch at its real size (device-generated prefill, the
+    same launch configuration as the benchmark).  For each sampled sequence the
+    oracle keeps only (original positions, utilities) and, layer by layer,
+    regenerates the cached K/V rows from the seeded generator by position -- so a
+    32k x 32-layer fp64 cache never has to exist at once.  Sequences are independent,
+    so sampling them checks the full-batch run."""
+    T = steps
+    u = w.u_table()
+    u_dev = torch.from_numpy(u).cuda()
+    c = make_cache(w, ikv.IKV_GRAN_SEQ, page_perm_seed)
+    fill_device(c, w, u_dev)
+    op = O.Params(alpha=w.alpha, refresh_period=w.refresh_period, score_free=w.score_free)
+    p = c.params(w.alpha, w.refresh_period, w.score_free)
+    ws = c.step_workspace()
+    qs = w.queries(1, T + 1, u)
+    budgets = w.budgets()
+    lens = list(w.prefill)
+    out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
+    sp = w.spec()
+    L0_dev = torch.tensor(w.prefill, dtype=torch.int32, device="cuda")
+    kn = torch.empty((1, w.layers, w.batch, w.kv_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
+    vn = torch.empty_like(kn)
+    state = {b: {"pos": np.arange(w.prefill[b], dtype=np.int64), "m": np.zeros(w.prefill[b])} for b in seqs}
+    reports = []
+    for t in range(1, T + 1):
+        assert gen.cuda_lib().ikvgen_fill_tokens_cuda(ctypes.byref(sp), u_dev.data_ptr(), L0_dev.data_ptr(), t, t + 1,
+                                                      w.dtype, kn.data_ptr(), vn.data_ptr(),
+                                                      torch.cuda.current_stream().cuda_stream) == 0
+        ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, to_device(qs[t - 1], w), kn[0], vn[0], out, ws,
+                     ws.numel())
+        lens = [min(L + 1, B) if L + 1 > B else L + 1 for L, B in zip(lens, budgets)]
+        torch.cuda.synchronize()
+        refresh = O.is_refresh(t, w.refresh_period, w.score_free)
+        rep = StepReport(t=t, refresh=refresh)
+        q64 = as_f64(qs[t - 1], w)
+        len_h = c.len.cpu().numpy()
+        for b in seqs:
+            st = state[b]
+            # append (Appendix "New token insertion"; 0 on refresh steps)
+            st["m"] = np.append(st["m"], O.new_token_state(st["m"], refresh, op.refresh_init))
+            st["pos"] = np.append(st["pos"], w.prefill[b] + t - 1)
+            out_b = out[:, b].float().cpu().numpy()
+            for l in range(w.layers):
+                k, v = w.kv_rows(b, l, st["pos"], u)
+                a_, o_ = O.last_query_attention(q64[l, b], [x.astype(np.float64) for x in k],
+                                                [x.astype(np.float64) for x in v])
+                rep.out_err = max(rep.out_err, float(np.max(np.abs(out_b[l] - o_))))
+                if refresh:
+                    st["m"] = O.ema_update(st["m"], O.pooled_score(a_, O.GRAN_SEQ, w.kv_heads)[0], op.alpha)
+            n = int(len_h[b])
+            assert n == min(st["pos"].shape[0], budgets[b])
+            gpos = c.pos[b, :n].cpu().numpy().astype(np.int64)
+            gm = c.ema[b, :n].cpu().numpy()
+            slot_of = {int(pp): i for i, pp in enumerate(st["pos"])}
+            oslots = np.array([slot_of[int(pp)] for pp in gpos])
+            kept = np.zeros(st["pos"].shape[0], bool)
+            kept[oslots] = True
+            ok, _ = boundary_ok(st["m"], kept, budgets[b])
+            rep.set_ok &= ok
+            rep.strict_set_equal &= set(O.select_keep(st["m"], budgets[b]).tolist()) == set(oslots.tolist())
+            rep.m_err = max(rep.m_err, float(np.max(np.abs(gm - st["m"][oslots]))))
+            keep = np.sort(oslots)
+            st["m"], st["pos"] = st["m"][keep], st["pos"][keep]
+            for l in check_layers:
+                lk, lv = w.kv_rows(b, l % w.layers, gpos, u)
+                for g in range(w.kv_heads):
+                    gk = c.gather(c.k, b, l % w.layers, g, n).float().cpu().numpy()
+                    gv = c.gather(c.v, b, l % w.layers, g, n).float().cpu().numpy()
+                    rep.kv_err = max(rep.kv_err, float(np.max(np.abs(gk - lk[g]))), float(np.max(np.abs(gv - lv[g]))))
+        reports.append(rep)
+    assert ikv.ikv_device_status() == 0
+    return reports

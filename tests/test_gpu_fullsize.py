@@ -1,0 +1,46 @@
+"""Parity at the five workloads' full sizes (GPU only).
+
+The GPU runs each workload at its real shape in the benchmark's launch
+configuration; the oracle follows sampled sequences (sequences are independent)
+for the first decode steps, including step 1, which scores the whole prefill
+and evicts ~90% of it.  Per step: attention outputs of every layer and head
+(bf16: 2e-2), the kept set under the 1e-4 boundary rule, the kept utilities
+(1e-3), and the compacted K/V rows of the first and last layer bit for bit.
+"""
+import pytest
+
+import gen
+from harness import run_fullsize_sampled
+
+pytestmark = pytest.mark.gpu
+
+
+def _check(reps):
+    for r in reps:
+        assert r.set_ok, r
+        assert r.out_err < 2e-2, r
+        assert r.m_err < 1e-3, r
+        assert r.kv_err == 0.0, r
+
+
+@pytest.mark.timeout(1200)
+def test_config1_llama_b1_32k_full_refresh():
+    _check(run_fullsize_sampled(gen.config(1), seqs=[0], steps=3))
+
+
+@pytest.mark.timeout(1200)
+def test_config2_llama_b16_ragged_lazy4():
+    # steps 1 and 5 refresh, 2-4 carry the state (Eq. 6); two of the sixteen sequences followed
+    _check(run_fullsize_sampled(gen.config(2), seqs=[0, 11], steps=5))
+
+
+@pytest.mark.timeout(1200)
+def test_config3_llama_b8_64k_score_free():
+    _check(run_fullsize_sampled(gen.config(3), seqs=[5], steps=3))
+
+
+@pytest.mark.timeout(1200)
+def test_config4_qwen_b32_16k_sweep_point():
+    # one point of the sweep: budget 25%, alpha 0.5, Lazy refresh period 2
+    w = gen.config(4).with_(budget_frac=0.25, alpha=0.5, refresh_period=2)
+    _check(run_fullsize_sampled(w, seqs=[31], steps=3))
