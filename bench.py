@@ -45,7 +45,9 @@ def parse():
     ap.add_argument("--config", type=int, default=1)
     ap.add_argument("--no-modes", action="store_true", help="skip the Lazy4 / Score-Free lines")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline")
-    ap.add_argument("--compact", default="stable", choices=["stable", "holefill"])
+    ap.add_argument("--compact", default="short", choices=["short", "stable", "holefill"],
+                    help="short: order-preserving, moves the shorter side (default); stable: always shifts "
+                         "the suffix left; holefill: moves survivors into holes (order not kept)")
     ap.add_argument("--cpu-steps", type=int, default=0, help="oracle steps in the CPU sample (0 = auto)")
     return ap.parse_args()
 
@@ -245,7 +247,8 @@ def reset(c, w, u_dev):
 
 
 def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_detail: bool, dist):
-    """Warm-up then K timed steps of one schedule; returns a dict of measurements."""
+    """Warm-up then K timed steps of one schedule, launched eagerly; returns a dict of
+    measurements (with per-kernel CUDA-event times when want_detail)."""
     import torch
 
     from paper_2609_03515_gb300 import ikv
@@ -285,7 +288,6 @@ def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_d
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
-    clocks = ClockSampler(torch.cuda.current_device()) if want_detail else None
     launches0 = ikv.ikv_launch_count()
     start.record(stream)
     for i in range(K):
@@ -296,13 +298,80 @@ def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_d
     ms = max_over_ranks(start.elapsed_time(stop), dist, c.k.device)
     res = {"ms": ms, "launches": launches, "lens": lens}
     if want_detail:
-        res["clocks"] = clocks.stop()
         names = ["append", "attend", "combine", "score_ema", "select", "compact"]
         per = {n: [] for n in names}
         for e in evs:
             for j, n in enumerate(names):
                 per[n].append(e[j].elapsed_time(e[j + 1]))
         res["kernel_ms"] = {n: sum(v) / len(v) for n, v in per.items()}
+    return res
+
+
+def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, sample_clocks: bool):
+    """The same schedule with each steady-state step replayed from a captured CUDA graph.
+
+    After the eager warm-up (decode step 1 evicts ~90% of the prefill, later steps hold
+    the budget), one graph per step kind (refresh / carry-over, Eq. 6) is captured
+    around ikv_step with fixed input buffers; every timed step copies its inputs into
+    those buffers (one device-to-device copy each) and replays the graph of its kind."""
+    import torch
+
+    from paper_2609_03515_gb300 import ikv
+
+    reset(c, w, u_dev)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode)
+    budgets = w.budgets()
+    lens = list(w.prefill)
+    dev = c.k.device
+    out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=c.torch_dtype, device=dev)
+    q_buf, kn_buf, vn_buf = torch.empty_like(qs_dev[0]), torch.empty_like(kn_dev[0]), torch.empty_like(vn_dev[0])
+    W, K = args.warmup, args.steps
+    for t in range(1, W + 1):
+        ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws,
+                     ws.numel(), torch.cuda.current_stream())
+        lens = [min(L + 1, B) if L + 1 > B else L + 1 for L, B in zip(lens, budgets)]
+    torch.cuda.synchronize()
+    steady = c.cache(max(lens))
+
+    def refresh(t):
+        return t == 1 if w.score_free else (t - 1) % w.refresh_period == 0
+
+    graphs = {}
+    n0 = ikv.ikv_launch_count()
+    for i in range(K):
+        t = W + 1 + i
+        kind = refresh(t)
+        if kind in graphs:
+            continue
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="thread_local"):
+            ikv.ikv_step(c.shape(), p, steady, c.ema, t, q_buf, kn_buf, vn_buf, out, ws, ws.numel(),
+                         torch.cuda.current_stream())
+        graphs[kind] = (g, ikv.ikv_launch_count() - n0)
+        n0 = ikv.ikv_launch_count()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(torch.cuda.current_device()) if sample_clocks else None
+    launches = 0
+    start.record(stream)
+    for i in range(K):
+        t = W + 1 + i
+        q_buf.copy_(qs_dev[t - 1], non_blocking=True)
+        kn_buf.copy_(kn_dev[t - 1], non_blocking=True)
+        vn_buf.copy_(vn_dev[t - 1], non_blocking=True)
+        g, nl = graphs[refresh(t)]
+        g.replay()
+        launches += nl
+    stop.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(start.elapsed_time(stop), dist, dev)
+    res = {"ms": ms, "launches": launches}
+    if sample_clocks:
+        res["clocks"] = clocks.stop()
     return res
 
 
@@ -383,7 +452,8 @@ def run_ours(args):
     total_steps = args.warmup + args.steps
     if total_steps > w.steps:
         w = w.with_(steps=total_steps)
-    compact_mode = ikv.IKV_COMPACT_STABLE if args.compact == "stable" else ikv.IKV_COMPACT_HOLEFILL
+    compact_mode = {"short": ikv.IKV_COMPACT_STABLE_SHORT, "stable": ikv.IKV_COMPACT_STABLE,
+                    "holefill": ikv.IKV_COMPACT_HOLEFILL}[args.compact]
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
@@ -417,14 +487,17 @@ def run_ours(args):
     assert rc == 0
     torch.cuda.synchronize()
 
-    full = run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, True, dist)
+    eager = run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, True, dist)
+    full = run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, True)
     modes = {}
     if not args.no_modes:
         for name, ww, cm in (("lazy4", w.with_(refresh_period=4), compact_mode),
                              ("score_free", w.with_(score_free=True), compact_mode),
-                             ("full_holefill", w, ikv.IKV_COMPACT_HOLEFILL)):
-            r = run_mode(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, False, dist)
-            modes[name] = r
+                             ("full_stable_left", w, ikv.IKV_COMPACT_STABLE),
+                             ("full_holefill", w, ikv.IKV_COMPACT_HOLEFILL),
+                             ("lazy4_holefill", w.with_(refresh_period=4), ikv.IKV_COMPACT_HOLEFILL),
+                             ("score_free_holefill", w.with_(score_free=True), ikv.IKV_COMPACT_HOLEFILL)):
+            modes[name] = run_mode_graph(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, dist, False)
     qs_pin = qs_t.pin_memory()
     kn_pin = kn_dev.cpu().pin_memory()
     vn_pin = vn_dev.cpu().pin_memory()
@@ -443,7 +516,7 @@ def run_ours(args):
     esz = 2 if w.dtype == gen.BF16 else 4
     kv_bytes = sum(L) * w.layers * w.kv_heads * w.head_dim * 2 * esz
     q_bytes = w.layers * w.batch * w.q_heads * w.head_dim * esz
-    att_ms = full["kernel_ms"]["attend"]
+    att_ms = eager["kernel_ms"]["attend"]
     achieved = (kv_bytes + q_bytes) / (att_ms / 1e3) / 1e9
     traffic = profiled_traffic(w.name)
     line = {
@@ -463,12 +536,15 @@ def run_ours(args):
                    "kv_heads": w.kv_heads, "head_dim": w.head_dim, "prefill": w.prefill[0] if w.batch == 1 else w.prefill,
                    "budget": w.budgets(), "alpha": w.alpha, "refresh": "full", "compaction": args.compact,
                    "timed_steps": f"decode steps {args.warmup + 1}..{args.warmup + K} (steady state; step 1 in warm-up)",
+                   "launch": "CUDA graph per step kind, inputs staged by one device copy each",
                    "l2": "inputs exceed L2 (K/V working set %.0f MB > 129 MB), no flush" % (kv_bytes / 1e6),
                    "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                      "traffic": traffic, "kernel": "attend_tc_kernel", "peak_kind": peak_kind,
                      "bytes_per_launch": kv_bytes + q_bytes, "ms_per_launch": att_ms},
-        "kernel_ms_per_step": full["kernel_ms"],
+        "kernel_ms_per_step": eager["kernel_ms"],
+        "eager": {"value": job_throughput(w.batch * K, world, eager["ms"]), "ms_per_step": eager["ms"] / K,
+                  "note": "same steps launched one by one (per-kernel events above come from this run)"},
         "cpu_baseline": cpu,
         "e2e": {"value": w.batch * K * world / (e2e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
@@ -478,8 +554,9 @@ def run_ours(args):
     }
     if modes:
         line["speedup_vs_full"] = {k: (w.batch * K * world / (v["ms"] / 1e3)) / value for k, v in modes.items()}
-        line["modes_note"] = ("lazy4 / score_free: same inputs, stable compaction; full_holefill: full refresh with "
-                              "hole-fill compaction (same kept sets, survivors not kept in order)")
+        line["modes_note"] = ("lazy4 / score_free: same inputs and compaction as the headline; full_stable_left: "
+                              "stable compaction that always shifts the suffix left; *_holefill: hole-fill "
+                              "compaction (same kept sets, survivors not kept in order)")
     print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()

@@ -33,10 +33,12 @@
  * Paged K/V layout
  * ----------------
  *  k, v: [layers][num_pages][kv_heads][page_size][head_dim] (dtype).
- *  Sequence b owns logical pages 0..max_pages-1 mapped through
- *  block_table[b][p] to physical pages; its cache slot j lives in logical page
- *  j / page_size at offset j % page_size.  cap = max_pages * page_size is the
- *  slot capacity of a row.  Slots 0..len[b]-1 are valid.
+ *  Sequence b owns a slot space of cap = max_pages * page_size slots; slot p of
+ *  it lives in physical page block_table[b][p / page_size] at offset
+ *  p % page_size.  The sequence's cache slot j (j = 0..len[b]-1) is slot
+ *  start[b] + j of that space (start == NULL means 0 for every sequence);
+ *  start[b] + len[b] <= cap always.  Every block_table entry must name a valid
+ *  page.
  *
  * Utility rows
  * ------------
@@ -71,7 +73,7 @@ typedef enum {
 
 enum { IKV_F32 = 0, IKV_BF16 = 1 };
 enum { IKV_GRAN_SEQ = 0, IKV_GRAN_KVHEAD = 1 };
-enum { IKV_COMPACT_STABLE = 0, IKV_COMPACT_HOLEFILL = 1 };
+enum { IKV_COMPACT_STABLE = 0, IKV_COMPACT_HOLEFILL = 1, IKV_COMPACT_STABLE_SHORT = 2 };
 enum { IKV_INIT_ZERO = 0, IKV_INIT_MEAN = 1 };
 
 typedef struct {
@@ -90,6 +92,8 @@ typedef struct {
     int32_t *pos;                /* [rows][cap] original token position per slot (device) */
     int32_t *next_pos;           /* [batch] position given to the next appended token (device) */
     int32_t max_len;             /* HOST-side upper bound on every len[b]; sizes launch grids */
+    int32_t *start;              /* [batch] slot of cache slot 0 (device), or NULL = 0; moved
+                                    only by IKV_COMPACT_STABLE_SHORT */
 } ikv_cache;
 
 /* Optional per-kernel CUDA events recorded on the call's stream by ikv_step
@@ -204,9 +208,14 @@ ikv_status ikv_select_budget(int32_t rows, int32_t cap, const float *util, const
  * len[b] = keep_len[r].  IKV_COMPACT_STABLE preserves the survivors' order
  * (moves only the shifted suffix); IKV_COMPACT_HOLEFILL moves survivors that
  * sit at slots >= keep_len into the evicted slots below keep_len, keeping the
- * same set but not its order (fewer moved rows).
+ * same set but not its order (fewer moved rows).  IKV_COMPACT_STABLE_SHORT
+ * also preserves the order but moves whichever side of the evicted slots is
+ * shorter: the suffix left (start unchanged) or the prefix right (start[b]
+ * grows by the number evicted), chosen per sequence, and only while the slot
+ * space keeps room for the next append (needs cache->start; sequences with
+ * several utility rows always compact left).
  *  keep/keep_len as produced by ikv_select_budget.  ws: at least
- *  ikv_compact_workspace_size() bytes (0 for the stable mode).
+ *  ikv_compact_workspace_size() bytes.
  * ------------------------------------------------------------------------- */
 ikv_status ikv_compact_workspace_size(const ikv_shape *shape, const ikv_cache *cache, int32_t mode, size_t *bytes);
 ikv_status ikv_compact_kv(const ikv_shape *shape, ikv_cache *cache, const int32_t *keep, const int32_t *keep_len,

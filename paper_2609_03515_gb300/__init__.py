@@ -51,6 +51,7 @@ class DecodeCache:
         self.pos = torch.zeros((self.rows, self.cap), dtype=torch.int32, device=device)
         self.ema = torch.zeros((self.rows, self.cap), dtype=torch.float32, device=device)
         self.budget = torch.zeros(batch, dtype=torch.int32, device=device)
+        self.start = torch.zeros(batch, dtype=torch.int32, device=device)
         self.max_len = 0
 
     # ---- ABI structs ------------------------------------------------------
@@ -62,7 +63,7 @@ class DecodeCache:
         ml = self.max_len if max_len is None else max_len
         return ikv.ikv_cache(self.k.data_ptr(), self.v.data_ptr(), self.block_table.data_ptr(), self.num_pages,
                              self.page_size, self.max_pages, self.len.data_ptr(), self.pos.data_ptr(),
-                             self.next_pos.data_ptr(), ml)
+                             self.next_pos.data_ptr(), ml, self.start.data_ptr())
 
     @property
     def rows_per_seq(self) -> int:
@@ -78,11 +79,12 @@ class DecodeCache:
         ar = torch.arange(self.cap, dtype=torch.int32, device=dev)
         self.pos.copy_(ar.expand(self.rows, self.cap))
         self.ema.zero_()
+        self.start.zero_()
         self.max_len = max(lengths)
 
-    def slot_rows(self, b: int, layer: int, g: int, n: int) -> torch.Tensor:
-        """K/V rows [n][head_dim] of slots 0..n-1 of (b, layer, g), gathered through the block table."""
-        slots = torch.arange(n, device=self.k.device)
+    def slot_rows(self, b: int, layer: int, g: int, n: int):
+        """(pages, offsets) of cache slots 0..n-1 of sequence b (through start and the block table)."""
+        slots = torch.arange(n, device=self.k.device) + int(self.start[b].item())
         pages = self.block_table[b, (slots // self.page_size).long()].long()
         return pages, slots % self.page_size
 
@@ -92,7 +94,8 @@ class DecodeCache:
 
     def scatter(self, pool: torch.Tensor, b: int, layer: int, g: int, rows: torch.Tensor, start: int = 0) -> None:
         n = rows.shape[0]
-        slots = torch.arange(start, start + n, device=pool.device)
+        s0 = start + int(self.start[b].item())
+        slots = torch.arange(s0, s0 + n, device=pool.device)
         pages = self.block_table[b, (slots // self.page_size).long()].long()
         pool[layer, pages, g, slots % self.page_size] = rows.to(pool.dtype)
 

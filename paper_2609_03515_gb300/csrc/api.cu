@@ -87,6 +87,7 @@ int32_t cap_of(const ikv_cache *c) { return c->page_size * c->max_pages; }
 PagedView view_of(const ikv_shape *s, const ikv_cache *c) {
     PagedView v;
     v.block_table = c->block_table;
+    v.start = c->start;
     v.num_pages = c->num_pages;
     v.page_size = c->page_size;
     v.max_pages = c->max_pages;
@@ -124,7 +125,7 @@ AttendWs attend_ws(const ikv_shape *s, int32_t cap, int n_layers, bool logits) {
 
 struct StepWs {
     AttendWs at;
-    size_t keep, keep_len, done, moves, n_moves, end;
+    size_t keep, keep_len, done, cdone, moves, n_moves, end;
 };
 
 StepWs step_ws(const ikv_shape *s, int32_t cap) {
@@ -136,8 +137,9 @@ StepWs step_ws(const ikv_shape *s, int32_t cap) {
     off = align256(off + R * cap * sizeof(int32_t));
     w.keep_len = off;
     off = align256(off + R * sizeof(int32_t));
-    w.done = off;
-    off = align256(off + (size_t)s->batch * sizeof(int32_t));
+    w.done = off;  // append arrivals, then compaction arrivals: one control block
+    w.cdone = off + (size_t)s->batch * sizeof(int32_t);
+    off = align256(off + 2 * (size_t)s->batch * sizeof(int32_t));
     w.moves = off;
     off = align256(off + R * cap * 2 * sizeof(int32_t));
     w.n_moves = off;
@@ -192,10 +194,11 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
     const int group = s->q_heads / s->kv_heads;
     const uint64_t pool_rows = (uint64_t)(layer0 + n_layers) * c->num_pages * s->kv_heads * c->page_size;
     const bool tc = tc_supported(s->dtype, s->head_dim, group, c->page_size) &&
-                    (int64_t)max_len <= (int64_t)kMaxSplits * tc_max_split_tokens() && pool_rows < (1ull << 31);
+                    (int64_t)max_len + 127 <= (int64_t)kMaxSplits * tc_max_split_tokens() && pool_rows < (1ull << 31);
     if (tc) {
         int32_t it = 0, nc = 0;
-        tc_plan(max_len, (int64_t)s->batch * n_layers * s->kv_heads, sm_count(), &it, &nc);
+        // a start offset may put the first valid row anywhere in its 128-slot tile
+        tc_plan(max_len + 127, (int64_t)s->batch * n_layers * s->kv_heads, sm_count(), &it, &nc);
         a.split_tokens = it * 128;
         a.n_splits = nc;
     } else
@@ -347,18 +350,18 @@ ikv_status ikv_compact_workspace_size(const ikv_shape *shape, const ikv_cache *c
     if (e) return e;
     if ((e = check_cache(shape, cache, false))) return e;
     if (!bytes) return fail(IKV_ERR_ARG, "bytes is NULL");
-    if (mode == IKV_COMPACT_STABLE) {
-        *bytes = 0;
-        return IKV_OK;
-    }
-    if (mode != IKV_COMPACT_HOLEFILL) return fail(IKV_ERR_ARG, "unknown compact mode %d", mode);
+    if (mode != IKV_COMPACT_STABLE && mode != IKV_COMPACT_HOLEFILL && mode != IKV_COMPACT_STABLE_SHORT)
+        return fail(IKV_ERR_ARG, "unknown compact mode %d", mode);
     const size_t R = (size_t)shape->batch * rows_per_seq(shape);
-    *bytes = align256(R * cap_of(cache) * 2 * sizeof(int32_t)) + align256(R * sizeof(int32_t));
+    *bytes = align256((size_t)shape->batch * sizeof(int32_t));  // arrival counters
+    if (mode == IKV_COMPACT_HOLEFILL)
+        *bytes += align256(R * cap_of(cache) * 2 * sizeof(int32_t)) + align256(R * sizeof(int32_t));
     return IKV_OK;
 }
 
 static ikv_status compact_impl(const ikv_shape *shape, ikv_cache *cache, const int32_t *keep, const int32_t *keep_len,
-                               float *ema, int32_t mode, int32_t *moves, int32_t *n_moves, cudaStream_t stream) {
+                               float *ema, int32_t mode, int32_t *moves, int32_t *n_moves, int32_t *done,
+                               cudaStream_t stream) {
     CompactArgs a{};
     a.k = cache->k;
     a.v = cache->v;
@@ -368,8 +371,11 @@ static ikv_status compact_impl(const ikv_shape *shape, ikv_cache *cache, const i
     a.rows_per_seq = rows_per_seq(shape);
     a.cap = cap_of(cache);
     a.elem_bytes = elem_bytes(shape);
+    a.mode = mode;
     a.len = cache->len;
     a.pos = cache->pos;
+    a.start = cache->start;
+    a.done = done;
     a.ema = ema;
     a.keep = keep;
     a.keep_len = keep_len;
@@ -388,14 +394,19 @@ ikv_status ikv_compact_kv(const ikv_shape *shape, ikv_cache *cache, const int32_
     if (!keep || !keep_len) return fail(IKV_ERR_ARG, "keep/keep_len is NULL");
     size_t need = 0;
     if ((e = ikv_compact_workspace_size(shape, cache, mode, &need))) return e;
+    if (mode == IKV_COMPACT_STABLE_SHORT && !cache->start)
+        return fail(IKV_ERR_ARG, "IKV_COMPACT_STABLE_SHORT needs cache->start");
+    if (!ws || ws_bytes < need) return fail(IKV_ERR_WORKSPACE, "workspace needs %zu bytes", need);
+    int32_t *done = at<int32_t>(ws, 0);
+    const size_t off = align256((size_t)shape->batch * sizeof(int32_t));
     int32_t *moves = nullptr, *n_moves = nullptr;
     if (mode == IKV_COMPACT_HOLEFILL) {
-        if (!ws || ws_bytes < need) return fail(IKV_ERR_WORKSPACE, "workspace needs %zu bytes", need);
         const size_t R = (size_t)shape->batch * rows_per_seq(shape);
-        moves = at<int32_t>(ws, 0);
-        n_moves = at<int32_t>(ws, align256(R * cap_of(cache) * 2 * sizeof(int32_t)));
+        moves = at<int32_t>(ws, off);
+        n_moves = at<int32_t>(ws, off + align256(R * cap_of(cache) * 2 * sizeof(int32_t)));
     }
-    return compact_impl(shape, cache, keep, keep_len, ema, mode, moves, n_moves, stream);
+    IKV_TRY_CUDA(cudaMemsetAsync(done, 0, sizeof(int32_t) * shape->batch, stream), "cudaMemsetAsync");
+    return compact_impl(shape, cache, keep, keep_len, ema, mode, moves, n_moves, done, stream);
 }
 
 static ikv_status append_impl(const ikv_shape *shape, ikv_cache *cache, const void *k_new, const void *v_new,
@@ -462,8 +473,11 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     if (t < 1) return fail(IKV_ERR_ARG, "t is 1-based (got %d)", t);
     if (!(p->alpha >= 0.f && p->alpha <= 1.f)) return fail(IKV_ERR_ARG, "alpha must be in [0, 1]");
     if (p->refresh_period < 1) return fail(IKV_ERR_ARG, "refresh_period must be >= 1");
-    if (p->compact_mode != IKV_COMPACT_STABLE && p->compact_mode != IKV_COMPACT_HOLEFILL)
+    if (p->compact_mode != IKV_COMPACT_STABLE && p->compact_mode != IKV_COMPACT_HOLEFILL &&
+        p->compact_mode != IKV_COMPACT_STABLE_SHORT)
         return fail(IKV_ERR_ARG, "unknown compact mode %d", p->compact_mode);
+    if (p->compact_mode == IKV_COMPACT_STABLE_SHORT && !cache->start)
+        return fail(IKV_ERR_ARG, "IKV_COMPACT_STABLE_SHORT needs cache->start");
     if (p->refresh_init != IKV_INIT_ZERO && p->refresh_init != IKV_INIT_MEAN)
         return fail(IKV_ERR_ARG, "unknown refresh_init %d", p->refresh_init);
     const int32_t cap = cap_of(cache);
@@ -483,7 +497,7 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     // control words (append and split-arrival counters) start at zero
     IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.at.arrivals), 0, w.at.logits - w.at.arrivals, stream),
                  "cudaMemsetAsync");
-    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.done), 0, sizeof(int32_t) * shape->batch, stream),
+    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.done), 0, 2 * sizeof(int32_t) * shape->batch, stream),
                  "cudaMemsetAsync");
     if (tm && (e = record(tm->begin, stream))) return e;
     const int32_t init_mean = refresh ? (p->refresh_init == IKV_INIT_MEAN) : 1;
@@ -503,7 +517,7 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
                  "select launch");
     if (tm && (e = record(tm->select_end, stream))) return e;
     if ((e = compact_impl(shape, cache, at<int32_t>(ws, w.keep), at<int32_t>(ws, w.keep_len), ema, p->compact_mode,
-                          at<int32_t>(ws, w.moves), at<int32_t>(ws, w.n_moves), stream)))
+                          at<int32_t>(ws, w.moves), at<int32_t>(ws, w.n_moves), at<int32_t>(ws, w.cdone), stream)))
         return e;
     if (tm && (e = record(tm->end, stream))) return e;
     return IKV_OK;

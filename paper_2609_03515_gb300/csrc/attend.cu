@@ -119,6 +119,7 @@ __global__ void __launch_bounds__(kAttendThreads, 2) attend_split_kernel(const A
     const int b = blockIdx.z % a.batch, li = blockIdx.z / a.batch;
     const int l = a.layer0 + li;
     const int L = a.len[b];
+    const int S0 = a.pv.start_of(b);
     const int t0 = s * a.split_tokens;
     if (t0 >= L) return;
     const int t1 = min(t0 + a.split_tokens, L);
@@ -137,7 +138,7 @@ __global__ void __launch_bounds__(kAttendThreads, 2) attend_split_kernel(const A
             const int j = idx / C::CPR, c = idx % C::CPR;
             const int tok = base + j;
             if (tok < t1) {
-                const int64_t row = a.pv.row(b, l, g, tok);
+                const int64_t row = a.pv.row_phys(b, l, g, S0 + tok);
                 const int off = j * C::kRowBytes + ((c ^ (j & 7)) << 4);
                 cp_async16(st + off, kbase + row * C::kRowBytes + c * 16);
                 cp_async16(st + C::kTileBytes + off, vbase + row * C::kRowBytes + c * 16);

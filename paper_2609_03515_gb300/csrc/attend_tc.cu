@@ -59,6 +59,7 @@ enum : unsigned { kErrTimeout = 1u };
 struct TcArgs {
     const int32_t *len;
     const int32_t *block_table;
+    const int32_t *start;       // [batch] physical slot of logical slot 0, or null
     int32_t num_pages, page_size, max_pages, kv_heads, rows_per_box;
     const __nv_bfloat16 *q;     // q + ((li*batch + b)*H + h)*128
     int32_t batch, q_heads, layer0, n_layers, split_tokens, n_splits, cap;
@@ -201,9 +202,14 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int g = unit_id % a.kv_heads;
     const int b = (unit_id / a.kv_heads) % a.batch, li = (unit_id / a.kv_heads) / a.batch;
     const int l = a.layer0 + li;
+    // The unit's valid rows are physical slots [S0, S0 + L).  Chunks cut the 128-aligned
+    // physical tiles covering them (TMA boxes stay page aligned); rows outside are masked.
     const int L = a.len[b];
-    const int t0 = s * a.split_tokens;
-    if (t0 >= L) {
+    const int S0 = a.start ? a.start[b] : 0;
+    const int ft = S0 / kTile;
+    const int nt_unit = L > 0 ? (S0 + L + kTile - 1) / kTile - ft : 0;
+    const int item = a.split_tokens / kTile;  // tiles per chunk
+    if (s * item >= nt_unit) {
         if (s == 0) {  // empty sequence: zero output, log-sum-exp -inf
             for (int i = threadIdx.x; i < G * kD; i += kThreads)
                 a.out[(((int64_t)li * a.batch + b) * a.q_heads + (int64_t)g * G) * kD + i] = __float2bfloat16_rn(0.f);
@@ -212,9 +218,10 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         return;
     }
-    const int t1 = min(t0 + a.split_tokens, L);
-    const int n = (t1 - t0 + kTile - 1) / kTile;
-    const int ns_active = (L + a.split_tokens - 1) / a.split_tokens;
+    const int n = min(item, nt_unit - s * item);           // tiles of this chunk
+    const int t0 = (ft + s * item) * kTile;                  // physical slot of its first row
+    const int lo = max(t0, S0), t1 = min(t0 + n * kTile, S0 + L);  // its valid rows [lo, t1)
+    const int ns_active = (nt_unit + item - 1) / item;
     if (n > kMaxTiles) {  // the host sizes splits to fit TMEM; refuse rather than overrun
         if (threadIdx.x == 0) atomicOr(&g_tc_error, 2u);
         return;
@@ -358,7 +365,8 @@ __global__ void __launch_bounds__(kThreads, 2)
             for (int i = 0; i < n; ++i) {
                 float v[NC];
                 tmem_ld<NC>(tS + lane_off + kN * i, v);
-                if (t0 + i * kTile + tid < t1) {
+                const int tok = t0 + i * kTile + tid;
+                if (tok >= lo && tok < t1) {
 #pragma unroll
                     for (int h = 0; h < G; ++h) mx[h] = fmaxf(mx[h], v[h] * a.scale_log2);
                 }
@@ -388,14 +396,14 @@ __global__ void __launch_bounds__(kThreads, 2)
             float v[NC];
             tmem_ld<NC>(tS + lane_off + kN * i, v);
             const int tok = t0 + i * kTile + tid;
-            const bool valid = tok < t1;
+            const bool valid = tok >= lo && tok < t1;
             unsigned char *pbuf = sm + kOffP + (i & 1) * kOpBytes + (tid >> 6) * (kN * 128);
 #pragma unroll
             for (int h = 0; h < G; ++h) {
                 const float z = v[h] * a.scale_log2;
                 float p = 0.f;
                 if (valid) {
-                    if (a.logits) a.logits[lbase + (int64_t)h * a.lstride + tok] = z;
+                    if (a.logits) a.logits[lbase + (int64_t)h * a.lstride + (tok - S0)] = z;
                     p = exp2f(z - mx[h]);
                     sum[h] += p;
                 }
@@ -582,6 +590,7 @@ cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group,
     TcArgs t{};
     t.len = a.len;
     t.block_table = a.pv.block_table;
+    t.start = a.pv.start;
     t.num_pages = a.pv.num_pages;
     t.page_size = a.pv.page_size;
     t.max_pages = a.pv.max_pages;

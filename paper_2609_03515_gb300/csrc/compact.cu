@@ -1,14 +1,19 @@
 // In-place gather compaction of the paged K/V after eviction, and the append
 // of each step's new token.
 //
-// Stable mode: slot j <- slot keep[j] for j < n, keep ascending, so keep[j] >= j
-// and once keep[j] != j every later slot moves too: only the suffix from the
-// first moved slot j* is touched.  One CTA per (sequence, layer, kv head) walks
-// that suffix in ascending 32-row tiles through a 4-stage cp.async ring.  A
-// tile's sources are >= its first destination, and every earlier tile's
-// destinations lie below that, so reading ahead of the writes is safe; within
-// a tile all reads land (wait + barrier) before any write.  Extra CTAs per row
-// move the utility and position arrays the same way and set len = n.
+// Stable mode: logical slot j <- logical slot keep[j] for j < n; keep ascending,
+// so keep[j] >= j and once keep[j] != j every later slot moves too: only the
+// suffix from the first moved slot is touched.  One CTA per (sequence, layer,
+// kv head) walks that suffix in ascending 32-row tiles through a 4-stage
+// cp.async ring.  A tile's sources are >= its first destination, and every
+// earlier tile's destinations lie below that, so reading ahead of the writes is
+// safe; within a tile all reads land (wait + barrier) before any write.
+// Shorter-side stable mode: with D = len - n evictions, keep[j] - j rises from 0
+// to at most D, so either the suffix moves left (start kept) or the prefix before
+// the first slot with keep[j] = j + D moves right by its gap (start += D) --
+// whichever moves fewer rows.  The right move walks descending tiles, the mirror
+// image of the left one.  Survivors keep their order either way.  Extra CTAs per
+// row gather the utility and position arrays (logical slots, always left).
 //
 // Hole-fill mode: survivors at slots >= n move into the evicted slots below n
 // (k-th hole <- k-th such survivor).  Sources and destinations are disjoint,
@@ -52,6 +57,9 @@ __device__ __forceinline__ float block_sum(float v, float *scratch) {
     return r;
 }
 
+// Stable compaction of one sequence's rows (see the file comment).  Every CTA of
+// sequence b reads len[b] and start[b] first; the last CTA of b to arrive writes
+// the new values, so no CTA sees them early.
 __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const CompactArgs a) {
     extern __shared__ __align__(16) unsigned char cbuf[];
     __shared__ int scratch[32];
@@ -59,94 +67,140 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
     const int b = blockIdx.y, x = blockIdx.x;
     const int kvh = a.pv.kv_heads;
     const int nkv = a.layers * kvh;
+    const int L = a.len[b];
+    const int S = a.start ? a.start[b] : 0;
+    // shorter-side decision, identical in every CTA of b (it depends on row b only;
+    // rows of several KV heads share b's slot space, so they always compact left)
+    int new_start = S;
+    int right_moves = 0;  // prefix [0, right_moves) moves right when > 0
+    const int r0 = b * a.rows_per_seq;
+    const int n0 = a.keep_len[r0];
+    const int32_t *kp0 = a.keep + (int64_t)r0 * a.cap;
+    if (a.mode == IKV_COMPACT_STABLE_SHORT && a.rows_per_seq == 1 && a.start && n0 < L) {
+        const int D = L - n0;  // evicted slots: the prefix shifts right by D
+        int jl = n0, jr = n0;
+        for (int j = tid; j < n0; j += kCompThreads) {
+            const int kj = kp0[j];
+            if (kj != j) jl = min(jl, j);          // left: the suffix from jl moves
+            if (kj - j == D) jr = min(jr, j);      // right: the prefix before jr moves
+        }
+        jl = block_min_int(jl, scratch);
+        jr = block_min_int(jr, scratch);
+        if (jr < n0 - jl && S + D + n0 + 1 <= a.cap) {  // room for the next append
+            new_start = S + D;
+            right_moves = jr;
+        }
+    }
     if (x < nkv) {
         const int l = x / kvh, g = x % kvh;
         const int r = b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g);
         const int n = a.keep_len[r];
         const int32_t *kp = a.keep + (int64_t)r * a.cap;
-        int first = n;
-        for (int j = tid; j < n; j += kCompThreads)
-            if (kp[j] != j) first = min(first, j);
-        const int jstar = block_min_int(first, scratch);
-        if (jstar >= n) return;
-        const int rowB = a.pv.head_dim * a.elem_bytes;
-        const int CPR = rowB >> 4;
-        const int stageB = 2 * kCompRows * rowB;
-        const int n_tiles = (n - jstar + kCompRows - 1) / kCompRows;
-        unsigned char *kb = reinterpret_cast<unsigned char *>(a.k);
-        unsigned char *vb = reinterpret_cast<unsigned char *>(a.v);
-        auto issue = [&](int tile) {
-            unsigned char *st = cbuf + (tile % kCompStages) * stageB;
-            for (int idx = tid; idx < kCompRows * CPR; idx += kCompThreads) {
-                const int jj = idx / CPR, c = idx % CPR;
-                const int j = jstar + tile * kCompRows + jj;
-                if (j < n) {
-                    const int64_t src = a.pv.row(b, l, g, kp[j]);
-                    cp_async16(st + jj * rowB + c * 16, kb + src * rowB + c * 16);
-                    cp_async16(st + (kCompRows + jj) * rowB + c * 16, vb + src * rowB + c * 16);
+        int j0 = 0, j1 = 0;  // rows [j0, j1) move
+        const bool right = right_moves > 0;
+        if (right) {
+            j1 = right_moves;
+        } else {
+            int first = n;
+            for (int j = tid; j < n; j += kCompThreads)
+                if (kp[j] != j) first = min(first, j);
+            j0 = block_min_int(first, scratch);
+            j1 = n;
+        }
+        if (j0 < j1) {
+            const int rowB = a.pv.head_dim * a.elem_bytes;
+            const int CPR = rowB >> 4;
+            const int stageB = 2 * kCompRows * rowB;
+            const int n_tiles = (j1 - j0 + kCompRows - 1) / kCompRows;
+            unsigned char *kb = reinterpret_cast<unsigned char *>(a.k);
+            unsigned char *vb = reinterpret_cast<unsigned char *>(a.v);
+            // tile k covers rows [jb, jb + kCompRows) ascending (left) or descending (right)
+            auto tile_base = [&](int tile) { return right ? j1 - (tile + 1) * kCompRows : j0 + tile * kCompRows; };
+            auto issue = [&](int tile) {
+                unsigned char *st = cbuf + (tile % kCompStages) * stageB;
+                const int jb = tile_base(tile);
+                for (int idx = tid; idx < kCompRows * CPR; idx += kCompThreads) {
+                    const int jj = idx / CPR, c = idx % CPR;
+                    const int j = jb + jj;
+                    if (j >= j0 && j < j1) {
+                        const int64_t src = a.pv.row_phys(b, l, g, S + kp[j]);
+                        cp_async16(st + jj * rowB + c * 16, kb + src * rowB + c * 16);
+                        cp_async16(st + (kCompRows + jj) * rowB + c * 16, vb + src * rowB + c * 16);
+                    }
+                }
+            };
+#pragma unroll
+            for (int i = 0; i < kCompStages - 1; ++i) {
+                if (i < n_tiles) issue(i);
+                cp_async_commit();
+            }
+            for (int tile = 0; tile < n_tiles; ++tile) {
+                __syncthreads();  // the stage about to be refilled was written out last iteration
+                if (tile + kCompStages - 1 < n_tiles) issue(tile + kCompStages - 1);
+                cp_async_commit();
+                cp_async_wait<kCompStages - 1>();
+                __syncthreads();  // every read of this tile has landed before any write
+                const unsigned char *st = cbuf + (tile % kCompStages) * stageB;
+                const int jb = tile_base(tile);
+                for (int idx = tid; idx < kCompRows * CPR; idx += kCompThreads) {
+                    const int jj = idx / CPR, c = idx % CPR;
+                    const int j = jb + jj;
+                    if (j >= j0 && j < j1) {
+                        const int64_t dst = a.pv.row_phys(b, l, g, new_start + j);
+                        *reinterpret_cast<uint4 *>(kb + dst * rowB + c * 16) =
+                            *reinterpret_cast<const uint4 *>(st + jj * rowB + c * 16);
+                        *reinterpret_cast<uint4 *>(vb + dst * rowB + c * 16) =
+                            *reinterpret_cast<const uint4 *>(st + (kCompRows + jj) * rowB + c * 16);
+                    }
                 }
             }
-        };
-#pragma unroll
-        for (int i = 0; i < kCompStages - 1; ++i) {
-            if (i < n_tiles) issue(i);
-            cp_async_commit();
+            cp_async_wait<0>();
         }
-        for (int tile = 0; tile < n_tiles; ++tile) {
-            __syncthreads();  // the stage about to be refilled was written out last iteration
-            if (tile + kCompStages - 1 < n_tiles) issue(tile + kCompStages - 1);
-            cp_async_commit();
-            cp_async_wait<kCompStages - 1>();
-            __syncthreads();  // every read of this tile has landed before any write
-            const unsigned char *st = cbuf + (tile % kCompStages) * stageB;
-            for (int idx = tid; idx < kCompRows * CPR; idx += kCompThreads) {
-                const int jj = idx / CPR, c = idx % CPR;
-                const int j = jstar + tile * kCompRows + jj;
-                if (j < n) {
-                    const int64_t dst = a.pv.row(b, l, g, j);
-                    *reinterpret_cast<uint4 *>(kb + dst * rowB + c * 16) =
-                        *reinterpret_cast<const uint4 *>(st + jj * rowB + c * 16);
-                    *reinterpret_cast<uint4 *>(vb + dst * rowB + c * 16) =
-                        *reinterpret_cast<const uint4 *>(st + (kCompRows + jj) * rowB + c * 16);
+    } else {
+        // utility / position rows: always the plain stable gather of logical slots
+        const int rr = x - nkv;
+        const int r = b * a.rows_per_seq + rr;
+        const int n = a.keep_len[r];
+        const int32_t *kp = a.keep + (int64_t)r * a.cap;
+        int32_t *pos = a.pos + (int64_t)r * a.cap;
+        float *ema = a.ema ? a.ema + (int64_t)r * a.cap : nullptr;
+        constexpr int PER = 16;
+        for (int base = 0; base < n; base += kCompThreads * PER) {
+            int32_t pv[PER];
+            float ev[PER];
+            int src[PER];
+#pragma unroll
+            for (int u = 0; u < PER; ++u) {
+                const int j = base + u * kCompThreads + tid;
+                src[u] = j < n ? kp[j] : j;
+                if (j < n && src[u] != j) {
+                    pv[u] = pos[src[u]];
+                    ev[u] = ema ? ema[src[u]] : 0.f;
                 }
             }
-        }
-        cp_async_wait<0>();
-        return;
-    }
-    // utility / position rows
-    const int rr = x - nkv;
-    const int r = b * a.rows_per_seq + rr;
-    const int n = a.keep_len[r];
-    const int32_t *kp = a.keep + (int64_t)r * a.cap;
-    int32_t *pos = a.pos + (int64_t)r * a.cap;
-    float *ema = a.ema ? a.ema + (int64_t)r * a.cap : nullptr;
-    constexpr int PER = 16;
-    for (int base = 0; base < n; base += kCompThreads * PER) {
-        int32_t pv[PER];
-        float ev[PER];
-        int src[PER];
+            __syncthreads();
 #pragma unroll
-        for (int u = 0; u < PER; ++u) {
-            const int j = base + u * kCompThreads + tid;
-            src[u] = j < n ? kp[j] : j;
-            if (j < n && src[u] != j) {
-                pv[u] = pos[src[u]];
-                ev[u] = ema ? ema[src[u]] : 0.f;
+            for (int u = 0; u < PER; ++u) {
+                const int j = base + u * kCompThreads + tid;
+                if (j < n && src[u] != j) {
+                    pos[j] = pv[u];
+                    if (ema) ema[j] = ev[u];
+                }
             }
+            __syncthreads();
         }
-        __syncthreads();
-#pragma unroll
-        for (int u = 0; u < PER; ++u) {
-            const int j = base + u * kCompThreads + tid;
-            if (j < n && src[u] != j) {
-                pos[j] = pv[u];
-                if (ema) ema[j] = ev[u];
-            }
-        }
-        __syncthreads();
     }
-    if (rr == 0 && tid == 0) a.len[b] = n;
+    // publish len / start once every CTA of b has read them
+    __syncthreads();
+    if (tid == 0) {
+        __threadfence();
+        if (atomicAdd(&a.done[b], 1) == (int)gridDim.x - 1) {
+            __threadfence();
+            a.len[b] = n0;
+            if (a.start) a.start[b] = new_start;
+            a.done[b] = 0;
+        }
+    }
 }
 
 // Hole-fill move list of one row: for every evicted slot h < n (the k-th such),
@@ -190,14 +244,15 @@ __global__ void __launch_bounds__(kCompThreads) holefill_move_kernel(const Compa
         const int r = b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g);
         const int nm = a.n_moves[r];
         const int32_t *mv = a.moves + (int64_t)r * a.cap * 2;
+        const int S = a.pv.start_of(b);
         const int rowB = a.pv.head_dim * a.elem_bytes;
         const int CPR = rowB >> 4;
         unsigned char *kb = reinterpret_cast<unsigned char *>(a.k);
         unsigned char *vb = reinterpret_cast<unsigned char *>(a.v);
         for (int idx = tid; idx < nm * CPR; idx += kCompThreads) {
             const int m = idx / CPR, c = idx % CPR;
-            const int64_t src = a.pv.row(b, l, g, mv[2 * m]);
-            const int64_t dst = a.pv.row(b, l, g, mv[2 * m + 1]);
+            const int64_t src = a.pv.row_phys(b, l, g, S + mv[2 * m]);
+            const int64_t dst = a.pv.row_phys(b, l, g, S + mv[2 * m + 1]);
             *reinterpret_cast<uint4 *>(kb + dst * rowB + c * 16) = *reinterpret_cast<const uint4 *>(kb + src * rowB + c * 16);
             *reinterpret_cast<uint4 *>(vb + dst * rowB + c * 16) = *reinterpret_cast<const uint4 *>(vb + src * rowB + c * 16);
         }
@@ -228,11 +283,12 @@ __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a
     const int tid = threadIdx.x;
     const int b = blockIdx.y;
     const int L = a.len[b];
+    const int S = a.pv.start_of(b);
     const int kvh = a.pv.kv_heads;
     const int nkv = a.layers * kvh;
     const int rowB = a.pv.head_dim * a.elem_bytes;
     const int CPR = rowB >> 4;
-    if (L < a.cap) {
+    if (S + L < a.cap) {
         unsigned char *kb = reinterpret_cast<unsigned char *>(a.k);
         unsigned char *vb = reinterpret_cast<unsigned char *>(a.v);
         const unsigned char *kn = reinterpret_cast<const unsigned char *>(a.k_new);
@@ -242,7 +298,7 @@ __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a
             if (x < nkv) {
                 const int l = x / kvh, g = x % kvh;
                 const int64_t src = (((int64_t)l * a.batch + b) * kvh + g) * rowB + c * 16;
-                const int64_t dst = a.pv.row(b, l, g, L) * rowB + c * 16;
+                const int64_t dst = a.pv.row_phys(b, l, g, S + L) * rowB + c * 16;
                 *reinterpret_cast<uint4 *>(kb + dst) = *reinterpret_cast<const uint4 *>(kn + src);
                 *reinterpret_cast<uint4 *>(vb + dst) = *reinterpret_cast<const uint4 *>(vn + src);
             }
@@ -270,7 +326,7 @@ __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a
         const int prev = atomicAdd(&a.done[b], 1);
         if (prev == (int)gridDim.x - 1) {
             __threadfence();
-            if (L < a.cap) {
+            if (S + L < a.cap) {
                 a.len[b] = L + 1;
                 a.next_pos[b] = a.next_pos[b] + 1;
             }
@@ -285,8 +341,13 @@ cudaError_t launch_compact(const CompactArgs &a, int mode, cudaStream_t st) {
     dim3 grid(a.layers * a.pv.kv_heads + a.rows_per_seq, a.batch);
     if (mode == IKV_COMPACT_STABLE) {
         const int smem = kCompStages * 2 * kCompRows * a.pv.head_dim * a.elem_bytes;
-        cudaError_t e = cudaFuncSetAttribute(compact_stable_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        if (e != cudaSuccess) return e;
+        static int attr_smem = 0;  // raise the dynamic shared-memory limit once per size
+        if (smem > attr_smem) {
+            cudaError_t e =
+                cudaFuncSetAttribute(compact_stable_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+            if (e != cudaSuccess) return e;
+            attr_smem = smem;
+        }
         compact_stable_kernel<<<grid, kCompThreads, smem, st>>>(a);
         note_launch();
         return cudaGetLastError();

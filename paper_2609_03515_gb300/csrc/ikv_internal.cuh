@@ -23,12 +23,16 @@ void note_launch(int n = 1);
 ikv_status report(ikv_status s, const char *fmt, ...);
 
 // Where a (sequence, slot) row of layer l / kv head g lives in the paged pool.
+// Logical slot j of sequence b is physical slot start[b] + j of its slot space
+// [0, cap); physical slot p lives in page block_table[b][p / page_size].
 struct PagedView {
     const int32_t *block_table;
+    const int32_t *start;       // [batch] or null (all zero)
     int32_t num_pages, page_size, max_pages, kv_heads, head_dim;
-    __device__ __forceinline__ int64_t row(int32_t b, int32_t l, int32_t g, int32_t slot) const {
-        const int32_t page = block_table[(int64_t)b * max_pages + slot / page_size];
-        return (((int64_t)l * num_pages + page) * kv_heads + g) * page_size + slot % page_size;
+    __device__ __forceinline__ int32_t start_of(int32_t b) const { return start ? start[b] : 0; }
+    __device__ __forceinline__ int64_t row_phys(int32_t b, int32_t l, int32_t g, int32_t phys) const {
+        const int32_t page = block_table[(int64_t)b * max_pages + phys / page_size];
+        return (((int64_t)l * num_pages + page) * kv_heads + g) * page_size + phys % page_size;
     }
 };
 
@@ -94,7 +98,10 @@ struct CompactArgs {
     void *k, *v;
     PagedView pv;
     int32_t batch, layers, rows_per_seq, cap, elem_bytes;
+    int32_t mode;               // IKV_COMPACT_*
     int32_t *len, *pos;
+    int32_t *start;             // [batch] or null; advanced by the shorter-side mode
+    int32_t *done;              // [batch] arrival counters, zero on entry; reset by the last CTA
     float *ema;
     const int32_t *keep, *keep_len;
     int32_t *moves;             // hole-fill: [rows][cap][2] (src, dst), null for stable

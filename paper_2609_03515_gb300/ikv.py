@@ -17,7 +17,7 @@ LIB_PATH = os.path.join(HERE, "libikv.so")
 IKV_OK, IKV_ERR_ARG, IKV_ERR_SHAPE, IKV_ERR_ALIGN, IKV_ERR_WORKSPACE, IKV_ERR_UNSUPPORTED, IKV_ERR_CUDA = range(7)
 IKV_F32, IKV_BF16 = 0, 1
 IKV_GRAN_SEQ, IKV_GRAN_KVHEAD = 0, 1
-IKV_COMPACT_STABLE, IKV_COMPACT_HOLEFILL = 0, 1
+IKV_COMPACT_STABLE, IKV_COMPACT_HOLEFILL, IKV_COMPACT_STABLE_SHORT = 0, 1, 2
 IKV_INIT_ZERO, IKV_INIT_MEAN = 0, 1
 
 P = ctypes.c_void_p
@@ -33,7 +33,7 @@ class ikv_shape(ctypes.Structure):
 
 class ikv_cache(ctypes.Structure):
     _fields_ = [("k", P), ("v", P), ("block_table", P), ("num_pages", I32), ("page_size", I32), ("max_pages", I32),
-                ("len", P), ("pos", P), ("next_pos", P), ("max_len", I32)]
+                ("len", P), ("pos", P), ("next_pos", P), ("max_len", I32), ("start", P)]
 
 
 class ikv_timing(ctypes.Structure):

@@ -185,7 +185,8 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
     return reports
 
 
-def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1), page_perm_seed: Optional[int] = 7):
+def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1), page_perm_seed: Optional[int] = 7,
+                         compact_mode: int = ikv.IKV_COMPACT_STABLE):
     """Full-size lock-step for a few sequences of a workload (GRAN_SEQ).
 
     The GPU decodes the whole batch at its real size (device-generated prefill, the
@@ -200,7 +201,7 @@ def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1)
     c = make_cache(w, ikv.IKV_GRAN_SEQ, page_perm_seed)
     fill_device(c, w, u_dev)
     op = O.Params(alpha=w.alpha, refresh_period=w.refresh_period, score_free=w.score_free)
-    p = c.params(w.alpha, w.refresh_period, w.score_free)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode)
     ws = c.step_workspace()
     qs = w.queries(1, T + 1, u)
     budgets = w.budgets()

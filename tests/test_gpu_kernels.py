@@ -209,7 +209,7 @@ def test_select_kvhead_rows_share_length():
 
 
 # ------------------------------------------------------------------ compaction and append
-@pytest.mark.parametrize("mode", [ikv.IKV_COMPACT_STABLE, ikv.IKV_COMPACT_HOLEFILL])
+@pytest.mark.parametrize("mode", [ikv.IKV_COMPACT_STABLE, ikv.IKV_COMPACT_HOLEFILL, ikv.IKV_COMPACT_STABLE_SHORT])
 @pytest.mark.parametrize("gran", [ikv.IKV_GRAN_SEQ, ikv.IKV_GRAN_KVHEAD])
 def test_compact_matches_oracle_eviction(mode, gran):
     w = gen.Workload("c", 3, 2, 8, 2, 128, [1000, 3278, 70], 1, dtype=gen.BF16, seed=31, page_size=16)
@@ -249,7 +249,7 @@ def test_compact_matches_oracle_eviction(mode, gran):
         n = st.length
         for rr in range(R):
             gp = pos[b * R + rr, :n]
-            if mode == ikv.IKV_COMPACT_STABLE:
+            if mode != ikv.IKV_COMPACT_HOLEFILL:
                 assert np.array_equal(gp, st.pos[rr])
                 assert np.array_equal(ema[b * R + rr, :n], st.m[rr].astype(np.float32))
             else:
@@ -289,3 +289,34 @@ def test_append_token(init_mean):
             for l in range(w.layers):
                 assert np.array_equal(c.gather(c.k, b, l, g, L + 1)[L].cpu().numpy(), kn[l, b, g])
                 assert np.array_equal(c.gather(c.v, b, l, g, L + 1)[L].cpu().numpy(), vn[l, b, g])
+
+
+def test_compact_short_side_moves_the_prefix():
+    """Shorter-side stable compaction: an eviction near the front moves the prefix right
+    and advances start; one near the back moves the suffix left; order is kept."""
+    w = gen.Workload("c", 2, 2, 8, 2, 128, [3278, 3278], 1, dtype=gen.BF16, seed=33, page_size=64)
+    u = w.u_table()
+    c = make_cache(w, page_perm_seed=2)
+    fill_device(c, w, torch.from_numpy(u).cuda())
+    util = np.ones((2, c.cap), np.float32)
+    util[0, 5] = 0.0       # evict slot 5 of sequence 0: 5 rows before it, 3272 after
+    util[1, 3000] = 0.0    # evict slot 3000 of sequence 1: 277 rows after it
+    c.ema.copy_(torch.from_numpy(util).cuda())
+    c.budget.fill_(3277)
+    keep = torch.empty((2, c.cap), dtype=torch.int32, device="cuda")
+    keep_len = torch.empty((2,), dtype=torch.int32, device="cuda")
+    ikv.ikv_select_budget(2, c.cap, c.ema, c.len, 1, c.budget, keep, keep_len)
+    cch = c.cache(3278)
+    nws = ikv.ikv_compact_workspace_size(c.shape(), cch, ikv.IKV_COMPACT_STABLE_SHORT)
+    ws = torch.empty(nws, dtype=torch.uint8, device="cuda")
+    ikv.ikv_compact_kv(c.shape(), cch, keep, keep_len, c.ema, ikv.IKV_COMPACT_STABLE_SHORT, ws, nws)
+    torch.cuda.synchronize()
+    assert c.start.cpu().tolist() == [1, 0] and c.len.cpu().tolist() == [3277, 3277]
+    for b, ev in ((0, 5), (1, 3000)):
+        want_pos = [p for p in range(3278) if p != ev]
+        assert c.pos[b, :3277].cpu().tolist() == want_pos
+        for l in range(2):
+            k, v = w.kv_rows(b, l, np.array(want_pos), u)
+            for g in range(2):
+                assert np.array_equal(c.gather(c.k, b, l, g, 3277).float().cpu().numpy(), k[g])
+                assert np.array_equal(c.gather(c.v, b, l, g, 3277).float().cpu().numpy(), v[g])

@@ -68,6 +68,15 @@ def test_holefill_keeps_the_same_sets():
     _assert(run_lockstep(small_llama(steps=6), compact_mode=ikv.IKV_COMPACT_HOLEFILL), 2e-2)
 
 
+def test_short_side_compaction_trajectory():
+    """Shorter-side stable compaction moves start, so the attention sees tiles that do
+    not start at slot 0 of the slot space; results must not change."""
+    _assert(run_lockstep(small_llama(steps=10), compact_mode=ikv.IKV_COMPACT_STABLE_SHORT), 2e-2)
+    _assert(run_lockstep(gen.config(0), compact_mode=ikv.IKV_COMPACT_STABLE_SHORT), 1e-4, strict_fraction=1.0)
+    _assert(run_lockstep(small_llama(steps=6, score_free=True, page_size=16),
+                         compact_mode=ikv.IKV_COMPACT_STABLE_SHORT), 2e-2)
+
+
 def test_sparse_layer_mask_and_mean_init_on_refresh():
     w = small_llama(steps=5, layers=4)
     _assert(run_lockstep(w, layer_eligible=[1, 0, 1, 0], refresh_init=ikv.IKV_INIT_MEAN), 2e-2)
