@@ -25,6 +25,7 @@ namespace {
 
 constexpr int kCompThreads = 256;
 constexpr int kCompRows = 32;
+constexpr int kRelocateSlack = 128;  // slots a relocation to slot 0 must free
 constexpr int kCompStages = 4;
 
 __device__ __forceinline__ void cp_async16(void *smem, const void *gmem) {
@@ -70,14 +71,14 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
     const int L = a.len[b];
     const int S = a.start ? a.start[b] : 0;
     // shorter-side decision, identical in every CTA of b (it depends on row b only;
-    // rows of several KV heads share b's slot space, so they always compact left)
+    // rows of several KV heads share b's slot space, so they always compact left).
+    // K/V row j lands at physical slot new_start + j; it moves iff S + kp[j] differs.
     int new_start = S;
-    int right_moves = 0;  // prefix [0, right_moves) moves right when > 0
     const int r0 = b * a.rows_per_seq;
     const int n0 = a.keep_len[r0];
     const int32_t *kp0 = a.keep + (int64_t)r0 * a.cap;
     if (a.mode == IKV_COMPACT_STABLE_SHORT && a.rows_per_seq == 1 && a.start && n0 < L) {
-        const int D = L - n0;  // evicted slots: the prefix shifts right by D
+        const int D = L - n0;  // evicted slots: the prefix may shift right by D
         int jl = n0, jr = n0;
         for (int j = tid; j < n0; j += kCompThreads) {
             const int kj = kp0[j];
@@ -86,9 +87,11 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
         }
         jl = block_min_int(jl, scratch);
         jr = block_min_int(jr, scratch);
-        if (jr < n0 - jl && S + D + n0 + 1 <= a.cap) {  // room for the next append
-            new_start = S + D;
-            right_moves = jr;
+        if (jr < n0 - jl) {
+            if (S + D + n0 + 1 <= a.cap)                        // room for the next append
+                new_start = S + D;
+            else if (S > 0 && a.cap - (n0 + 1) >= kRelocateSlack)  // out of room: move all rows
+                new_start = 0;                                 // to slot 0 once, regaining it
         }
     }
     if (x < nkv) {
@@ -96,17 +99,15 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
         const int r = b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g);
         const int n = a.keep_len[r];
         const int32_t *kp = a.keep + (int64_t)r * a.cap;
-        int j0 = 0, j1 = 0;  // rows [j0, j1) move
-        const bool right = right_moves > 0;
-        if (right) {
-            j1 = right_moves;
-        } else {
-            int first = n;
-            for (int j = tid; j < n; j += kCompThreads)
-                if (kp[j] != j) first = min(first, j);
-            j0 = block_min_int(first, scratch);
-            j1 = n;
-        }
+        const int shift = new_start - S;
+        // right (shift > 0): rows [0, j1) move, j1 the first row already in place (kp[j] = j + shift);
+        // left (shift <= 0): rows [j0, n) move, j0 the first row not in place
+        const bool right = shift > 0;
+        int first = n;
+        for (int j = tid; j < n; j += kCompThreads)
+            if ((kp[j] == j + shift) == right) first = min(first, j);
+        first = block_min_int(first, scratch);
+        const int j0 = right ? 0 : first, j1 = right ? first : n;
         if (j0 < j1) {
             const int rowB = a.pv.head_dim * a.elem_bytes;
             const int CPR = rowB >> 4;
@@ -339,7 +340,7 @@ __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a
 
 cudaError_t launch_compact(const CompactArgs &a, int mode, cudaStream_t st) {
     dim3 grid(a.layers * a.pv.kv_heads + a.rows_per_seq, a.batch);
-    if (mode == IKV_COMPACT_STABLE) {
+    if (mode == IKV_COMPACT_STABLE || mode == IKV_COMPACT_STABLE_SHORT) {
         const int smem = kCompStages * 2 * kCompRows * a.pv.head_dim * a.elem_bytes;
         static int attr_smem = 0;  // raise the dynamic shared-memory limit once per size
         if (smem > attr_smem) {

@@ -115,6 +115,41 @@ def test_decode_attend_score_matches_oracle(dt, d, H, Hkv, lens, gran, ps):
             assert torch.equal(ema[r, L:], ema0[r, L:])
 
 
+@pytest.mark.parametrize("ps,starts,lens", [
+    (64, [37, 128, 1000, 0], [700, 129, 4100, 1]),    # tensor-core kernel, chunks cut physical tiles
+    (16, [5, 250], [2000, 17]),
+    (48, [100, 3], [1500, 64]),                          # CUDA-core kernel
+])
+def test_decode_attend_score_with_start_offset(ps, starts, lens):
+    """Logical slot j of sequence b lives at physical slot start[b] + j; scores land at j."""
+    fill = [s + L for s, L in zip(starts, lens)]
+    w = gen.Workload("a", len(lens), 2, 32, 8, 128, fill, 1, dtype=gen.BF16, seed=22, page_size=ps)
+    u = w.u_table()
+    c = make_cache(w, page_perm_seed=9)
+    fill_device(c, w, torch.from_numpy(u).cuda())      # physical slot p holds position p
+    c.start.copy_(torch.tensor(starts, dtype=torch.int32))
+    c.len.copy_(torch.tensor(lens, dtype=torch.int32))
+    layer = 1
+    q_h = w.queries(1, 2, u)[0, layer]
+    q = to_device(q_h, w)
+    out = torch.empty((w.batch, 32, 128), dtype=q.dtype, device="cuda")
+    score = torch.full((c.rows, c.cap), -7.0, device="cuda")
+    ema = torch.zeros((c.rows, c.cap), device="cuda")
+    cch = c.cache(max(lens))
+    ws = torch.empty(ikv.ikv_attend_workspace_size(c.shape(), cch), dtype=torch.uint8, device="cuda")
+    ikv.ikv_decode_attend_score(c.shape(), cch, layer, q, out, score, ema, 0.5, ws, ws.numel())
+    torch.cuda.synchronize()
+    assert ikv.ikv_device_status() == 0
+    q64 = as_f64(q_h, w)
+    for b, (S, L) in enumerate(zip(starts, lens)):
+        k, v = w.kv_block(b, layer, S, L, u)
+        a, o = O.last_query_attention(q64[b], [x.astype(np.float64) for x in k], [x.astype(np.float64) for x in v])
+        assert np.max(np.abs(out[b].float().cpu().numpy() - o)) < 2e-2
+        sc = O.pooled_score(a, O.GRAN_SEQ, 8)[0]
+        assert np.max(np.abs(score[b, :L].cpu().numpy() - sc)) < 2e-5
+        assert torch.all(score[b, L:] == -7.0)
+
+
 def test_decode_attend_without_score_leaves_state():
     w = gen.Workload("a", 2, 1, 32, 8, 128, [900, 50], 1, dtype=gen.BF16, seed=2)
     u = w.u_table()
@@ -320,3 +355,45 @@ def test_compact_short_side_moves_the_prefix():
             for g in range(2):
                 assert np.array_equal(c.gather(c.k, b, l, g, 3277).float().cpu().numpy(), k[g])
                 assert np.array_equal(c.gather(c.v, b, l, g, 3277).float().cpu().numpy(), v[g])
+
+
+def test_compact_short_side_relocates_and_skips_in_place():
+    """Shorter-side compaction at the end of the slot space: (0) the prefix would move right
+    but has no room, so every row moves to slot 0 once; (1) the oldest row is evicted, so
+    start advances with no row moved; (2) no room and too little slack to relocate, so the
+    suffix moves left and start stays."""
+    w = gen.Workload("c", 3, 2, 8, 2, 128, [3520] * 3, 1, dtype=gen.BF16, seed=34, page_size=64)
+    u = w.u_table()
+    c = DecodeCache(3, 2, 8, 2, 128, 3520, dtype=ikv.IKV_BF16, page_size=64, page_perm_seed=5)
+    assert c.cap == 3520
+    fill_device(c, w, torch.from_numpy(u).cuda())  # physical slot p holds position p
+    S, L, ev = [244, 100, 70], [3276, 3276, 3450], [5, 0, 5]
+    c.start.copy_(torch.tensor(S, dtype=torch.int32))
+    c.len.copy_(torch.tensor(L, dtype=torch.int32))
+    c.budget.copy_(torch.tensor([x - 1 for x in L], dtype=torch.int32))
+    util = np.ones((3, c.cap), np.float32)
+    pos = np.zeros((3, c.cap), np.int32)
+    for b in range(3):
+        util[b, ev[b]] = 0.0
+        pos[b, :L[b]] = np.arange(S[b], S[b] + L[b])
+    c.ema.copy_(torch.from_numpy(util).cuda())
+    c.pos.copy_(torch.from_numpy(pos).cuda())
+    keep = torch.empty((3, c.cap), dtype=torch.int32, device="cuda")
+    keep_len = torch.empty((3,), dtype=torch.int32, device="cuda")
+    ikv.ikv_select_budget(3, c.cap, c.ema, c.len, 1, c.budget, keep, keep_len)
+    cch = c.cache(max(L))
+    nws = ikv.ikv_compact_workspace_size(c.shape(), cch, ikv.IKV_COMPACT_STABLE_SHORT)
+    ws = torch.empty(nws, dtype=torch.uint8, device="cuda")
+    ikv.ikv_compact_kv(c.shape(), cch, keep, keep_len, c.ema, ikv.IKV_COMPACT_STABLE_SHORT, ws, nws)
+    torch.cuda.synchronize()
+    assert c.start.cpu().tolist() == [0, 101, 70]
+    assert c.len.cpu().tolist() == [x - 1 for x in L]
+    for b in range(3):
+        n = L[b] - 1
+        want_pos = [S[b] + j for j in range(L[b]) if j != ev[b]]
+        assert c.pos[b, :n].cpu().tolist() == want_pos
+        for l in range(2):
+            k, v = w.kv_rows(b, l, np.array(want_pos), u)
+            for g in range(2):
+                assert np.array_equal(c.gather(c.k, b, l, g, n).float().cpu().numpy(), k[g])
+                assert np.array_equal(c.gather(c.v, b, l, g, n).float().cpu().numpy(), v[g])
