@@ -74,7 +74,7 @@ def rank_seed(base_seed: int, rank: int) -> int:
     return base_seed + 1000 * rank
 
 
-ATTEND_KERNEL_REV = "attend_tc_v2"
+ATTEND_KERNEL_REV = "attend_tc_v3"
 
 
 def profiled_traffic(workload: str):

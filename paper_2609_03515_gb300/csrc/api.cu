@@ -260,7 +260,7 @@ ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, c
         sa.alpha = alpha;
         sa.ema = ema;
         sa.score = score;
-        IKV_TRY_CUDA(launch_score_ema(sa, max_len, st), "score launch");
+        IKV_TRY_CUDA(launch_score_ema(sa, max_len, sm_count(), st), "score launch");
     }
     return IKV_OK;
 }

@@ -88,7 +88,7 @@ cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group,
 // launchers (return cudaError_t of the launch)
 cudaError_t launch_attend(const AttendArgs &a, int dtype, int head_dim, int group, cudaStream_t st);
 cudaError_t launch_combine(const CombineArgs &a, int dtype, cudaStream_t st);
-cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, cudaStream_t st);
+cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, int sms, cudaStream_t st);
 cudaError_t launch_ema_update(int32_t rows, int32_t cap, float *ema, const float *score, const int32_t *len,
                               int32_t rows_per_seq, float alpha, int32_t max_len, cudaStream_t st);
 cudaError_t launch_select(int32_t rows, int32_t cap, const float *util, const int32_t *len, int32_t rows_per_seq,
