@@ -74,21 +74,22 @@ def rank_seed(base_seed: int, rank: int) -> int:
     return base_seed + 1000 * rank
 
 
-ATTEND_KERNEL_REV = "attend_tc_v3"
+# revision of each attention kernel; a committed ncu summary counts only for its own revision
+ATTEND_KERNEL_REV = {"attend_tc_kernel": "attend_tc_v3", "attend_split_kernel": "attend_split_v2"}
 
 
-def profiled_traffic(workload: str):
+def profiled_traffic(kernel: str, workload: str):
     """DRAM bytes per launch of the attention kernel from the committed ncu summary,
     or None when that summary was taken on another kernel revision or workload."""
     import re
 
-    path = os.path.join(ROOT, "profiles", f"attend_tc_kernel__{workload}.md")
+    path = os.path.join(ROOT, "profiles", f"{kernel}__{workload}.md")
     if not os.path.exists(path):
         return None
     txt = open(path).read()
     rev = re.search(r"^kernel_rev:\s*(\S+)", txt, re.M)
     tb = re.search(r"^traffic_bytes_per_launch:\s*(\d+)", txt, re.M)
-    if not rev or not tb or rev.group(1) != ATTEND_KERNEL_REV:
+    if not rev or not tb or rev.group(1) != ATTEND_KERNEL_REV.get(kernel):
         return None
     return int(tb.group(1))
 
@@ -376,7 +377,11 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
 
 
 def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist):
-    """Same steps through the C ABI, inputs from pinned host memory and the output read back every step."""
+    """Same steps through the C ABI, inputs from pinned host memory and the output read back every step.
+
+    Two buffer sets and a copy stream: the upload of step t+1's inputs and the read-back
+    of step t-1's output run while step t computes.  Every step's copies lie inside the
+    timed region (the compute stream waits for the copy stream before the stop event)."""
     import torch
 
     from paper_2609_03515_gb300 import ikv
@@ -386,37 +391,59 @@ def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist):
     budgets = w.budgets()
     lens = list(w.prefill)
     dev = c.k.device
-    q_d = torch.empty(qs_h.shape[1:], dtype=qs_h.dtype, device=dev)
-    kn_d = torch.empty(kn_h.shape[1:], dtype=kn_h.dtype, device=dev)
-    vn_d = torch.empty_like(kn_d)
-    out_d = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=c.torch_dtype, device=dev)
-    out_h = torch.empty(out_d.shape, dtype=out_d.dtype, pin_memory=True)
-    stream = torch.cuda.current_stream()
+    q_d = [torch.empty(qs_h.shape[1:], dtype=qs_h.dtype, device=dev) for _ in range(2)]
+    kn_d = [torch.empty(kn_h.shape[1:], dtype=kn_h.dtype, device=dev) for _ in range(2)]
+    vn_d = [torch.empty(kn_h.shape[1:], dtype=kn_h.dtype, device=dev) for _ in range(2)]
+    oshape = (w.layers, w.batch, w.q_heads, w.head_dim)
+    out_d = [torch.empty(oshape, dtype=c.torch_dtype, device=dev) for _ in range(2)]
+    out_h = [torch.empty(oshape, dtype=c.torch_dtype, pin_memory=True) for _ in range(2)]
+    comp = torch.cuda.current_stream()
+    cs = torch.cuda.Stream(device=dev)
+    in_ready = [torch.cuda.Event() for _ in range(2)]
+    done = [torch.cuda.Event() for _ in range(2)]
 
-    def step(t):
+    def upload(t):
+        i = t % 2
+        with torch.cuda.stream(cs):
+            q_d[i].copy_(qs_h[t - 1], non_blocking=True)
+            kn_d[i].copy_(kn_h[t - 1], non_blocking=True)
+            vn_d[i].copy_(vn_h[t - 1], non_blocking=True)
+            in_ready[i].record(cs)
+
+    def run(t0, n):
+        """Steps t0 .. t0+n-1; the upload of t0 is issued here, the last read-back is waited for."""
         nonlocal lens
-        q_d.copy_(qs_h[t - 1], non_blocking=True)
-        kn_d.copy_(kn_h[t - 1], non_blocking=True)
-        vn_d.copy_(vn_h[t - 1], non_blocking=True)
-        ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, q_d, kn_d, vn_d, out_d, ws, ws.numel(), stream)
-        out_h.copy_(out_d, non_blocking=True)
-        lens = [min(L + 1, B) if L + 1 > B else L + 1 for L, B in zip(lens, budgets)]
+        cs.wait_stream(comp)
+        upload(t0)
+        for t in range(t0, t0 + n):
+            i = t % 2
+            if t + 1 < t0 + n:
+                if t + 1 >= t0 + 2:
+                    cs.wait_event(done[(t + 1) % 2])   # step t-1 has read the buffers step t+1 reuses
+                upload(t + 1)
+            comp.wait_event(in_ready[i])
+            ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, q_d[i], kn_d[i], vn_d[i], out_d[i], ws,
+                         ws.numel(), comp)
+            done[i].record(comp)
+            with torch.cuda.stream(cs):
+                cs.wait_event(done[i])
+                out_h[i].copy_(out_d[i], non_blocking=True)
+            lens = [min(L + 1, B) if L + 1 > B else L + 1 for L, B in zip(lens, budgets)]
+        comp.wait_stream(cs)
 
     W, K = args.warmup, args.steps
-    for t in range(1, W + 1):
-        step(t)
+    run(1, W)
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    start.record(stream)
-    for i in range(K):
-        step(W + 1 + i)
-    stop.record(stream)
+    start.record(comp)
+    run(W + 1, K)
+    stop.record(comp)
     torch.cuda.synchronize()
     ms = max_over_ranks(start.elapsed_time(stop), dist, dev)
-    h2d = (q_d.numel() + kn_d.numel() + vn_d.numel()) * q_d.element_size()
-    d2h = out_d.numel() * out_d.element_size()
+    h2d = (q_d[0].numel() + kn_d[0].numel() + vn_d[0].numel()) * q_d[0].element_size()
+    d2h = out_d[0].numel() * out_d[0].element_size()
     return ms, h2d, d2h
 
 
@@ -518,7 +545,11 @@ def run_ours(args):
     q_bytes = w.layers * w.batch * w.q_heads * w.head_dim * esz
     att_ms = eager["kernel_ms"]["attend"]
     achieved = (kv_bytes + q_bytes) / (att_ms / 1e3) / 1e9
-    traffic = profiled_traffic(w.name)
+    att_path = ikv.ikv_attend_path(c.shape(), c.cache(max(L)))
+    att_kernel = "attend_tc_kernel" if att_path == ikv.IKV_PATH_TENSOR_CORE else "attend_split_kernel"
+    traffic = profiled_traffic(att_kernel, w.name)
+    l2_note = ("inputs exceed L2 (K/V working set %.0f MB > 129 MB), no flush" % (kv_bytes / 1e6) if kv_bytes > 129e6
+               else "K/V working set %.2f MB stays in L2 (launch-bound case), no flush" % (kv_bytes / 1e6))
     line = {
         "metric": METRIC,
         "value": value,
@@ -537,10 +568,10 @@ def run_ours(args):
                    "budget": w.budgets(), "alpha": w.alpha, "refresh": "full", "compaction": args.compact,
                    "timed_steps": f"decode steps {args.warmup + 1}..{args.warmup + K} (steady state; step 1 in warm-up)",
                    "launch": "CUDA graph per step kind, inputs staged by one device copy each",
-                   "l2": "inputs exceed L2 (K/V working set %.0f MB > 129 MB), no flush" % (kv_bytes / 1e6),
+                   "l2": l2_note,
                    "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                     "traffic": traffic, "kernel": "attend_tc_kernel", "peak_kind": peak_kind,
+                     "traffic": traffic, "kernel": att_kernel, "peak_kind": peak_kind,
                      "bytes_per_launch": kv_bytes + q_bytes, "ms_per_launch": att_ms},
         "kernel_ms_per_step": eager["kernel_ms"],
         "eager": {"value": job_throughput(w.batch * K, world, eager["ms"]), "ms_per_step": eager["ms"] / K,

@@ -111,7 +111,9 @@ typedef struct {
     int32_t score_free;             /* 1: score at step 1 only, then freeze (Sec. 3.2) */
     const int32_t *budget;          /* [batch] decode budget B per sequence (device) */
     const uint8_t *layer_eligible;  /* HOST [layers] 0/1, NULL = all layers eligible */
-    int32_t compact_mode;           /* IKV_COMPACT_STABLE (order-preserving) | IKV_COMPACT_HOLEFILL */
+    int32_t compact_mode;           /* IKV_COMPACT_STABLE (order-preserving, suffix moves left) |
+                                       IKV_COMPACT_STABLE_SHORT (order-preserving, shorter side moves;
+                                       needs cache->start) | IKV_COMPACT_HOLEFILL (set only) */
     int32_t refresh_init;           /* utility of a token appended on a refresh step:
                                        IKV_INIT_ZERO (m_0 = 0 rule) | IKV_INIT_MEAN */
     const ikv_timing *timing;       /* nullable */
@@ -128,6 +130,17 @@ int64_t ikv_launch_count(void);
  * attention kernel ran out (the kernel abandoned its work and returned);
  * bit 1: a split longer than the kernel's TMEM budget reached the device. */
 ikv_status ikv_device_status(uint32_t *flags);
+
+/* Which decode-attention kernel ikv_decode_attend_score and ikv_step launch for
+ * this shape and cache (all layers, cache->max_len):
+ * IKV_PATH_TENSOR_CORE -- TMA-staged K/V tiles, tcgen05 QK^T and PV with TMEM
+ *   accumulators; bf16, head_dim 128, group size 1, 2, 4, 7 or 8, page_size a
+ *   divisor of 128 (>= 8) or a multiple of 128;
+ * IKV_PATH_CUDA_CORE -- split-K flash decoding on the CUDA cores plus a combine
+ *   kernel; every other supported shape.
+ * Host only; launches nothing.  *path receives the value. */
+enum { IKV_PATH_CUDA_CORE = 0, IKV_PATH_TENSOR_CORE = 1 };
+ikv_status ikv_attend_path(const ikv_shape *shape, const ikv_cache *cache, int32_t *path);
 
 /* ---------------------------------------------------------------------------
  * ikv_decode_attend_score -- one layer of decode attention plus its score.

@@ -177,6 +177,16 @@ void choose_splits(const ikv_shape *s, int n_layers, int32_t max_len, int granul
 }
 
 // attention (+ combine) over layers [layer0, layer0 + n_layers)
+// The tensor-core kernel serves bf16, d = 128, groups {1,2,4,7,8}, page sizes that tile
+// 128 rows, and pools whose rows a 32-bit TMA coordinate reaches; the split-K CUDA-core
+// kernel serves the rest.
+static bool use_tc(const ikv_shape *s, const ikv_cache *c, int32_t layers_touched, int32_t max_len) {
+    const int group = s->q_heads / s->kv_heads;
+    const uint64_t pool_rows = (uint64_t)layers_touched * c->num_pages * s->kv_heads * c->page_size;
+    return tc_supported(s->dtype, s->head_dim, group, c->page_size) &&
+           (int64_t)max_len + 127 <= (int64_t)kMaxSplits * tc_max_split_tokens() && pool_rows < (1ull << 31);
+}
+
 ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, int32_t n_layers, int32_t max_len,
                       const void *q, void *out, void *ws, const AttendWs &w, bool logits, int32_t *split_out,
                       int32_t *nsplit_out, cudaStream_t st, const ikv_timing *tm = nullptr,
@@ -192,9 +202,7 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
     a.layer0 = layer0;
     a.n_layers = n_layers;
     const int group = s->q_heads / s->kv_heads;
-    const uint64_t pool_rows = (uint64_t)(layer0 + n_layers) * c->num_pages * s->kv_heads * c->page_size;
-    const bool tc = tc_supported(s->dtype, s->head_dim, group, c->page_size) &&
-                    (int64_t)max_len + 127 <= (int64_t)kMaxSplits * tc_max_split_tokens() && pool_rows < (1ull << 31);
+    const bool tc = use_tc(s, c, layer0 + n_layers, max_len);
     if (tc) {
         int32_t it = 0, nc = 0;
         // a start offset may put the first valid row anywhere in its 128-slot tile
@@ -297,6 +305,16 @@ ikv_status ikv_attend_workspace_size(const ikv_shape *shape, const ikv_cache *ca
     if ((e = check_cache(shape, cache, false))) return e;
     if (!bytes) return fail(IKV_ERR_ARG, "bytes is NULL");
     *bytes = attend_ws(shape, cap_of(cache), 1, true).end;
+    return IKV_OK;
+}
+
+ikv_status ikv_attend_path(const ikv_shape *shape, const ikv_cache *cache, int32_t *path) {
+    g_err[0] = 0;
+    ikv_status e = check_shape(shape);
+    if (e) return e;
+    if ((e = check_cache(shape, cache, false))) return e;
+    if (!path) return fail(IKV_ERR_ARG, "path is NULL");
+    *path = use_tc(shape, cache, shape->layers, cache->max_len) ? IKV_PATH_TENSOR_CORE : IKV_PATH_CUDA_CORE;
     return IKV_OK;
 }
 

@@ -19,6 +19,7 @@ IKV_F32, IKV_BF16 = 0, 1
 IKV_GRAN_SEQ, IKV_GRAN_KVHEAD = 0, 1
 IKV_COMPACT_STABLE, IKV_COMPACT_HOLEFILL, IKV_COMPACT_STABLE_SHORT = 0, 1, 2
 IKV_INIT_ZERO, IKV_INIT_MEAN = 0, 1
+IKV_PATH_CUDA_CORE, IKV_PATH_TENSOR_CORE = 0, 1
 
 P = ctypes.c_void_p
 I32 = ctypes.c_int32
@@ -62,6 +63,7 @@ def _load():
         "ikv_last_error": ([], ctypes.c_char_p),
         "ikv_launch_count": ([], ctypes.c_int64),
         "ikv_device_status": ([ctypes.POINTER(ctypes.c_uint32)], I32),
+        "ikv_attend_path": ([SP, CP, ctypes.POINTER(I32)], I32),
         "ikv_attend_workspace_size": ([SP, CP, ctypes.POINTER(SZ)], I32),
         "ikv_decode_attend_score": ([SP, CP, I32, P, P, P, P, F32, P, SZ, P], I32),
         "ikv_static_scratch_bytes": ([], SZ),
@@ -116,6 +118,12 @@ def ikv_launch_count() -> int:
 def ikv_device_status() -> int:
     v = ctypes.c_uint32(0)
     _check(_lib.ikv_device_status(ctypes.byref(v)), "ikv_device_status")
+    return int(v.value)
+
+
+def ikv_attend_path(shape: ikv_shape, cache: ikv_cache) -> int:
+    v = I32(0)
+    _check(_lib.ikv_attend_path(ctypes.byref(shape), ctypes.byref(cache), ctypes.byref(v)), "ikv_attend_path")
     return int(v.value)
 
 

@@ -115,6 +115,21 @@ def test_other_entry_points_reject_nulls(lib):
                           None) == lib.IKV_ERR_WORKSPACE
 
 
+def test_attend_path_query(lib):
+    """Which attention kernel a shape gets is decided on the host (no launch)."""
+    def path(shape_kw, cache_kw):
+        return lib.ikv_attend_path(_shape(lib, **shape_kw), _cache(lib, **cache_kw))
+    bf = dict(dtype=lib.IKV_BF16, head_dim=128, q_heads=32, kv_heads=8)
+    assert path({}, {}) == lib.IKV_PATH_CUDA_CORE                                  # fp32, d = 64
+    assert path(bf, {}) == lib.IKV_PATH_TENSOR_CORE                                # bf16, d = 128, G = 4, page 64
+    assert path(dict(bf, q_heads=28, kv_heads=4), {}) == lib.IKV_PATH_TENSOR_CORE  # G = 7
+    assert path(bf, dict(page_size=256, max_pages=1)) == lib.IKV_PATH_TENSOR_CORE
+    assert path(bf, dict(page_size=48, max_pages=4, max_len=100)) == lib.IKV_PATH_CUDA_CORE
+    assert path(dict(bf, head_dim=64), {}) == lib.IKV_PATH_CUDA_CORE               # bf16, d = 64
+    with pytest.raises(lib.IKVError):
+        path(dict(bf, q_heads=5, kv_heads=2), {})
+
+
 def test_product_package_does_not_reference_the_oracle():
     """The CUDA path and its binding never import or link the CPU oracle."""
     pkg = os.path.join(ROOT, "paper_2609_03515_gb300")
