@@ -48,6 +48,11 @@ def parse():
     ap.add_argument("--compact", default="short", choices=["short", "stable", "holefill"],
                     help="short: order-preserving, moves the shorter side (default); stable: always shifts "
                          "the suffix left; holefill: moves survivors into holes (order not kept)")
+    ap.add_argument("--max-holes", type=int, default=128,
+                    help="deferred compaction: evicted slots stay marked dead until a sequence holds more "
+                         "than this many (0 = compact on every eviction)")
+    ap.add_argument("--mode-kernels", action="store_true",
+                    help="also run every mode eagerly and report its per-kernel times")
     ap.add_argument("--cpu-steps", type=int, default=0, help="oracle steps in the CPU sample (0 = auto)")
     return ap.parse_args()
 
@@ -76,6 +81,13 @@ def rank_seed(base_seed: int, rank: int) -> int:
 
 # revision of each attention kernel; a committed ncu summary counts only for its own revision
 ATTEND_KERNEL_REV = {"attend_tc_kernel": "attend_tc_v3", "attend_split_kernel": "attend_split_v2"}
+
+
+def schedule_name(w) -> str:
+    """The refresh schedule of a workload: full, lazy<r> (Eq. 6) or score_free."""
+    if w.score_free:
+        return "score_free"
+    return "full" if w.refresh_period == 1 else f"lazy{w.refresh_period}"
 
 
 def profiled_traffic(kernel: str, workload: str):
@@ -247,29 +259,29 @@ def reset(c, w, u_dev):
     torch.cuda.synchronize()
 
 
-def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_detail: bool, dist):
+def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_detail: bool, dist, mh: int = 0):
     """Warm-up then K timed steps of one schedule, launched eagerly; returns a dict of
     measurements (with per-kernel CUDA-event times when want_detail)."""
     import torch
 
-    from paper_2609_03515_gb300 import ikv
+    from paper_2609_03515_gb300 import ikv, step_lengths
 
     reset(c, w, u_dev)
-    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh)
     budgets = w.budgets()
-    lens = list(w.prefill)
+    lens, live = list(w.prefill), list(w.prefill)
     out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=c.torch_dtype, device=c.k.device)
     stream = torch.cuda.current_stream()
 
     def step(t, timing=None):
-        nonlocal lens
+        nonlocal lens, live
         if timing is not None:
             p.timing = ctypes.pointer(timing)
         else:
             p.timing = None
         ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws,
                      ws.numel(), stream)
-        lens = [min(L + 1, B) if L + 1 > B else L + 1 for L, B in zip(lens, budgets)]
+        lens, live = step_lengths(lens, live, budgets, mh)
 
     W, K = args.warmup, args.steps
     for t in range(1, W + 1):
@@ -308,7 +320,8 @@ def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_d
     return res
 
 
-def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, sample_clocks: bool):
+def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, sample_clocks: bool,
+                   mh: int = 0):
     """The same schedule with each steady-state step replayed from a captured CUDA graph.
 
     After the eager warm-up (decode step 1 evicts ~90% of the prefill, later steps hold
@@ -317,12 +330,13 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     those buffers (one device-to-device copy each) and replays the graph of its kind."""
     import torch
 
-    from paper_2609_03515_gb300 import ikv
+    from paper_2609_03515_gb300 import ikv, step_lengths
 
     reset(c, w, u_dev)
-    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh)
     budgets = w.budgets()
-    lens = list(w.prefill)
+    assert all(L0 >= B for L0, B in zip(w.prefill, budgets)), "graph replay assumes every sequence at its budget"
+    lens, live = list(w.prefill), list(w.prefill)
     dev = c.k.device
     out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=c.torch_dtype, device=dev)
     q_buf, kn_buf, vn_buf = torch.empty_like(qs_dev[0]), torch.empty_like(kn_dev[0]), torch.empty_like(vn_dev[0])
@@ -330,9 +344,11 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     for t in range(1, W + 1):
         ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws,
                      ws.numel(), torch.cuda.current_stream())
-        lens = [min(L + 1, B) if L + 1 > B else L + 1 for L, B in zip(lens, budgets)]
+        lens, live = step_lengths(lens, live, budgets, mh)
     torch.cuda.synchronize()
-    steady = c.cache(max(lens))
+    # one graph serves every later step, so its max_len bounds them all: the budget plus
+    # the dead slots deferred compaction may hold
+    steady = c.cache(min(c.cap - 1, max(max(lens), max(budgets) + mh)))
 
     def refresh(t):
         return t == 1 if w.score_free else (t - 1) % w.refresh_period == 0
@@ -376,7 +392,7 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     return res
 
 
-def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist):
+def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist, mh: int = 0):
     """Same steps through the C ABI, inputs from pinned host memory and the output read back every step.
 
     Two buffer sets and a copy stream: the upload of step t+1's inputs and the read-back
@@ -384,12 +400,12 @@ def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist):
     timed region (the compute stream waits for the copy stream before the stop event)."""
     import torch
 
-    from paper_2609_03515_gb300 import ikv
+    from paper_2609_03515_gb300 import ikv, step_lengths
 
     reset(c, w, u_dev)
-    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh)
     budgets = w.budgets()
-    lens = list(w.prefill)
+    lens, live = list(w.prefill), list(w.prefill)
     dev = c.k.device
     q_d = [torch.empty(qs_h.shape[1:], dtype=qs_h.dtype, device=dev) for _ in range(2)]
     kn_d = [torch.empty(kn_h.shape[1:], dtype=kn_h.dtype, device=dev) for _ in range(2)]
@@ -412,7 +428,7 @@ def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist):
 
     def run(t0, n):
         """Steps t0 .. t0+n-1; the upload of t0 is issued here, the last read-back is waited for."""
-        nonlocal lens
+        nonlocal lens, live
         cs.wait_stream(comp)
         upload(t0)
         for t in range(t0, t0 + n):
@@ -428,7 +444,7 @@ def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist):
             with torch.cuda.stream(cs):
                 cs.wait_event(done[i])
                 out_h[i].copy_(out_d[i], non_blocking=True)
-            lens = [min(L + 1, B) if L + 1 > B else L + 1 for L, B in zip(lens, budgets)]
+            lens, live = step_lengths(lens, live, budgets, mh)
         comp.wait_stream(cs)
 
     W, K = args.warmup, args.steps
@@ -471,7 +487,7 @@ def run_ours(args):
         __graft_entry__.build()
     if dist:
         dist.barrier()
-    from paper_2609_03515_gb300 import ikv
+    from paper_2609_03515_gb300 import ikv, step_lengths
 
     w = gen.config(args.config)
     # each rank decodes its own independent sequences (distinct seed per rank)
@@ -514,21 +530,39 @@ def run_ours(args):
     assert rc == 0
     torch.cuda.synchronize()
 
-    eager = run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, True, dist)
-    full = run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, True)
+    mh = args.max_holes
+    eager = run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, True, dist, mh)
+    full = run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, True, mh)
+    head_sched = schedule_name(w)
     modes = {}
+    mode_kernels = {}
     if not args.no_modes:
-        for name, ww, cm in (("lazy4", w.with_(refresh_period=4), compact_mode),
-                             ("score_free", w.with_(score_free=True), compact_mode),
-                             ("full_stable_left", w, ikv.IKV_COMPACT_STABLE),
-                             ("full_holefill", w, ikv.IKV_COMPACT_HOLEFILL),
-                             ("lazy4_holefill", w.with_(refresh_period=4), ikv.IKV_COMPACT_HOLEFILL),
-                             ("score_free_holefill", w.with_(score_free=True), ikv.IKV_COMPACT_HOLEFILL)):
-            modes[name] = run_mode_graph(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, dist, False)
+        full_w = w.with_(refresh_period=1, score_free=False)
+        lazy_w = w.with_(refresh_period=4, score_free=False)
+        sf_w = w.with_(refresh_period=1, score_free=True)
+        variants = (("full", full_w, compact_mode, mh),
+                    ("lazy4", lazy_w, compact_mode, mh),
+                    ("score_free", sf_w, compact_mode, mh),
+                    ("full_every_step", full_w, compact_mode, 0),
+                    ("lazy4_every_step", lazy_w, compact_mode, 0),
+                    ("score_free_every_step", sf_w, compact_mode, 0),
+                    ("full_stable_left", full_w, ikv.IKV_COMPACT_STABLE, 0),
+                    ("full_holefill", full_w, ikv.IKV_COMPACT_HOLEFILL, 0),
+                    ("lazy4_holefill", lazy_w, ikv.IKV_COMPACT_HOLEFILL, 0),
+                    ("score_free_holefill", sf_w, ikv.IKV_COMPACT_HOLEFILL, 0))
+        for name, ww, cm, vmh in variants:
+            if name == head_sched and cm == compact_mode and vmh == mh:
+                modes[name] = full           # the headline run is this mode
+                continue
+            modes[name] = run_mode_graph(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, dist, False, vmh)
+        if args.mode_kernels:
+            for name, ww, cm, vmh in variants:
+                mode_kernels[name] = run_mode(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, True, dist,
+                                              vmh)["kernel_ms"]
     qs_pin = qs_t.pin_memory()
     kn_pin = kn_dev.cpu().pin_memory()
     vn_pin = vn_dev.cpu().pin_memory()
-    e2e_ms, h2d, d2h = run_e2e(args, w, c, u_dev, ws, compact_mode, qs_pin, kn_pin, vn_pin, dist)
+    e2e_ms, h2d, d2h = run_e2e(args, w, c, u_dev, ws, compact_mode, qs_pin, kn_pin, vn_pin, dist, mh)
 
     K = args.steps
     value = job_throughput(w.batch * K, world, full["ms"])
@@ -565,7 +599,7 @@ def run_ours(args):
         "data": "synthetic",
         "config": {"workload": w.name, "batch_per_gpu": w.batch, "layers": w.layers, "q_heads": w.q_heads,
                    "kv_heads": w.kv_heads, "head_dim": w.head_dim, "prefill": w.prefill[0] if w.batch == 1 else w.prefill,
-                   "budget": w.budgets(), "alpha": w.alpha, "refresh": "full", "compaction": args.compact,
+                   "budget": w.budgets(), "alpha": w.alpha, "refresh": head_sched, "compaction": args.compact, "max_holes": mh,
                    "timed_steps": f"decode steps {args.warmup + 1}..{args.warmup + K} (steady state; step 1 in warm-up)",
                    "launch": "CUDA graph per step kind, inputs staged by one device copy each",
                    "l2": l2_note,
@@ -581,13 +615,18 @@ def run_ours(args):
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": full["launches"],
         "clocks": full["clocks"],
-        "modes": {"full": value, **{k: w.batch * K * world / (v["ms"] / 1e3) for k, v in modes.items()}},
+        "modes": {k: w.batch * K * world / (v["ms"] / 1e3) for k, v in modes.items()},
     }
     if modes:
-        line["speedup_vs_full"] = {k: (w.batch * K * world / (v["ms"] / 1e3)) / value for k, v in modes.items()}
-        line["modes_note"] = ("lazy4 / score_free: same inputs and compaction as the headline; full_stable_left: "
-                              "stable compaction that always shifts the suffix left; *_holefill: hole-fill "
-                              "compaction (same kept sets, survivors not kept in order)")
+        full_v = line["modes"]["full"]
+        line["speedup_vs_full"] = {k: v / full_v for k, v in line["modes"].items() if k != "full"}
+        if mode_kernels:
+            line["mode_kernel_ms_per_step"] = mode_kernels
+        line["modes_note"] = ("full / lazy4 / score_free: refresh every step / every 4th step (Eq. 6) / step 1 "
+                              "only, same inputs and compaction as the headline; *_every_step: the same "
+                              "compaction run on every eviction (max_holes 0); full_stable_left: stable "
+                              "compaction that always shifts the suffix left, every step; *_holefill: hole-fill "
+                              "compaction every step (same kept sets, survivors not kept in order)")
     print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()

@@ -88,12 +88,18 @@ typedef struct {
     int32_t num_pages;           /* physical pages per layer in the pools */
     int32_t page_size;           /* slots per page, >= 1 */
     int32_t max_pages;           /* logical pages per sequence; cap = max_pages * page_size */
-    int32_t *len;                /* [batch] valid slots per sequence (device) */
-    int32_t *pos;                /* [rows][cap] original token position per slot (device) */
+    int32_t *len;                /* [batch] slots in use per sequence (device); with dead_slots
+                                    set this counts dead slots too */
+    int32_t *pos;                /* [rows][cap] original token position per slot (device);
+                                    -1 marks a dead slot (see dead_slots) */
     int32_t *next_pos;           /* [batch] position given to the next appended token (device) */
     int32_t max_len;             /* HOST-side upper bound on every len[b]; sizes launch grids */
     int32_t *start;              /* [batch] slot of cache slot 0 (device), or NULL = 0; moved
                                     only by IKV_COMPACT_STABLE_SHORT */
+    int32_t dead_slots;          /* nonzero: slots whose pos is < 0 are dead -- evicted but not yet
+                                    compacted away (ikv_params.max_holes).  Attention, scores,
+                                    selection and the mean-utility append then skip them.
+                                    0: every slot below len is live (pos is not read for it). */
 } ikv_cache;
 
 /* Optional per-kernel CUDA events recorded on the call's stream by ikv_step
@@ -117,6 +123,15 @@ typedef struct {
     int32_t refresh_init;           /* utility of a token appended on a refresh step:
                                        IKV_INIT_ZERO (m_0 = 0 rule) | IKV_INIT_MEAN */
     const ikv_timing *timing;       /* nullable */
+    int32_t max_holes;              /* deferred compaction: 0 = compact on every eviction.  > 0:
+                                       an evicted slot is only marked dead (pos = -1) while the
+                                       sequence's dead slots stay <= max_holes; the step that
+                                       would exceed it compacts (compact_mode) and clears them.
+                                       The kept set and its order are the same either way; the
+                                       attention reads up to max_holes extra (masked) slots, and
+                                       rows move once per ~max_holes evictions instead of every
+                                       step.  Needs pos; len then counts dead slots, so the
+                                       caller's max_len bound is max(budget) + max_holes. */
 } ikv_params;
 
 /* Message for the last error on this thread ("" if none). */
@@ -128,7 +143,8 @@ int64_t ikv_launch_count(void);
 /* Device-side error word of the current device, then cleared (synchronises
  * the device).  0 = no error.  Bit 0: a bounded wait inside the tensor-core
  * attention kernel ran out (the kernel abandoned its work and returned);
- * bit 1: a split longer than the kernel's TMEM budget reached the device. */
+ * bit 1: a split longer than the kernel's TMEM budget reached the device;
+ * bit 2: an append found no free slot (start + len = cap) and was dropped. */
 ikv_status ikv_device_status(uint32_t *flags);
 
 /* Which decode-attention kernel ikv_decode_attend_score and ikv_step launch for
@@ -154,7 +170,9 @@ ikv_status ikv_attend_path(const ikv_shape *shape, const ikv_cache *cache, int32
  * (all q_heads for IKV_GRAN_SEQ, the KV head's group for IKV_GRAN_KVHEAD).
  * If ema != NULL the EMA of Eq. 4 is applied in place for i < len[b]:
  *     ema[r][i] = alpha * ema[r][i] + (1 - alpha) * score_i
- * which is one layer of the Appendix's layer-sequential update.
+ * which is one layer of the Appendix's layer-sequential update.  With
+ * cache->dead_slots set, dead slots (pos[r][i] < 0, r the row of (b, g)) are
+ * left out of the softmax: their probability and score are 0.
  *
  *  q, out: [batch][q_heads][head_dim] (dtype).  score, ema: [rows][cap] fp32.
  *  ws: at least ikv_attend_workspace_size() bytes.
@@ -200,16 +218,19 @@ ikv_status ikv_ema_update(int32_t rows, int32_t cap, float *ema, const float *sc
  * ikv_select_budget -- which tokens survive (Sec. 3: evict the lowest m_t(i)
  * whenever the cache exceeds B).
  *
- * For row r with L = len[r / rows_per_seq] and B = budget[r / rows_per_seq]:
- * if L <= B every slot is kept (keep[r][j] = j, keep_len[r] = L); otherwise
- * keep[r][0..B) lists, in ascending slot order, the B slots with the largest
- * util[r][i] (i < L).  Ties keep the lower slot; -0.0 equals +0.0; NaN ranks
- * below every number.  Bit-exact: the result depends only on the fp32 values.
- *  util: [rows][cap] fp32; keep: [rows][cap] int32; keep_len: [rows] int32.
+ * For row r with L = len[r / rows_per_seq] and B = budget[r / rows_per_seq],
+ * the live slots are i < L (with pos != NULL: those with pos[r][i] >= 0; dead
+ * slots are never kept).  If at most B slots are live, all of them are kept;
+ * otherwise the B live slots with the largest util[r][i].  keep[r][0..n) lists
+ * them in ascending slot order, keep_len[r] = n.  Ties keep the lower slot;
+ * -0.0 equals +0.0; NaN ranks below every number.  Bit-exact: the result
+ * depends only on the fp32 values.
+ *  util: [rows][cap] fp32; pos: [rows][cap] int32 or NULL; keep: [rows][cap]
+ *  int32; keep_len: [rows] int32.
  * ------------------------------------------------------------------------- */
 ikv_status ikv_select_budget(int32_t rows, int32_t cap, const float *util, const int32_t *len,
-                             int32_t rows_per_seq, const int32_t *budget, int32_t *keep, int32_t *keep_len,
-                             cudaStream_t stream);
+                             int32_t rows_per_seq, const int32_t *budget, const int32_t *pos, int32_t *keep,
+                             int32_t *keep_len, cudaStream_t stream);
 
 /* ---------------------------------------------------------------------------
  * ikv_compact_kv -- in-place gather compaction after eviction ("cache
@@ -239,9 +260,10 @@ ikv_status ikv_compact_kv(const ikv_shape *shape, ikv_cache *cache, const int32_
  *
  * Writes k_new/v_new ([layers][batch][kv_heads][head_dim]) into slot len[b]
  * of every layer, sets pos[r][len[b]] = next_pos[b], and gives the token the
- * utility 0 (init_mean == 0) or the mean utility of the existing len[b]
- * tokens of its row (init_mean == 1, Appendix "New token insertion during
- * non-refresh steps").  Then len[b] += 1 and next_pos[b] += 1.
+ * utility 0 (init_mean == 0) or the mean utility of the existing live tokens
+ * of its row (init_mean == 1, Appendix "New token insertion during non-refresh
+ * steps"; dead slots excluded when cache->dead_slots).  Then len[b] += 1 and
+ * next_pos[b] += 1.
  * Fails with IKV_ERR_SHAPE (host) if max_len + 1 > cap.
  * ------------------------------------------------------------------------- */
 ikv_status ikv_append_token(const ikv_shape *shape, ikv_cache *cache, const void *k_new, const void *v_new,
@@ -257,12 +279,16 @@ ikv_status ikv_append_token(const ikv_shape *shape, ikv_cache *cache, const void
  *   4. refresh steps only: for each eligible layer in ascending order,
  *      ema = alpha * ema + (1 - alpha) * s_layer  (Eq. 1, Eq. 4, Appendix
  *      "Layer scoring"); off-refresh steps leave ema untouched (Eq. 6)
- *   5. if len[b] > budget[b]: keep the budget[b] highest utilities and compact
- *      (Appendix "Eviction on non-refresh steps": also on off-refresh steps)
+ *   5. if more than budget[b] slots are live: keep the budget[b] highest
+ *      utilities and compact, or with max_holes > 0 mark the evicted slots dead
+ *      until their number would exceed max_holes (Appendix "Eviction on
+ *      non-refresh steps": also on off-refresh steps)
  *  q: [layers][batch][q_heads][head_dim]; k_new, v_new: [layers][batch][kv_heads][head_dim];
  *  out: [layers][batch][q_heads][head_dim] (all dtype).  ema: [rows][cap] fp32.
  *  cache->max_len bounds len[] BEFORE the append; the step needs max_len + 1 <= cap.
- *  After the step the caller should lower max_len to max(budget) if it tracks it.
+ *  After the step the caller should lower max_len to max(budget) (+ max_holes)
+ *  if it tracks it.  With max_holes > 0 the step treats the cache as holding
+ *  dead slots whatever cache->dead_slots says.
  * ------------------------------------------------------------------------- */
 ikv_status ikv_step_workspace_size(const ikv_shape *shape, const ikv_cache *cache, size_t *bytes);
 ikv_status ikv_step(const ikv_shape *shape, const ikv_params *params, ikv_cache *cache, float *ema, int32_t t,

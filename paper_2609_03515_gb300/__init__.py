@@ -14,7 +14,27 @@ import torch
 
 from . import ikv
 
-__all__ = ["ikv", "DecodeCache"]
+__all__ = ["ikv", "DecodeCache", "step_lengths"]
+
+
+def step_lengths(lens: Sequence[int], live: Sequence[int], budgets: Sequence[int], max_holes: int = 0):
+    """Host mirror of one ikv_step's length bookkeeping, for sizing max_len.
+
+    lens: slots in use per sequence (len[b], dead slots included); live: live slots.
+    The step appends one token; if more than budget[b] slots are then live, it keeps
+    budget[b] of them.  The evicted slots are only marked dead while the dead slots
+    stay <= max_holes (> 0); otherwise the sequence is compacted to its live slots.
+    Returns the (lens, live) after the step."""
+    out_l, out_v = [], []
+    for L, n, B in zip(lens, live, budgets):
+        L, n = L + 1, n + 1
+        kept = min(n, B)
+        if max_holes > 0 and L - kept <= max_holes:
+            out_l.append(L)
+        else:
+            out_l.append(kept)
+        out_v.append(kept)
+    return out_l, out_v
 
 
 class DecodeCache:
@@ -22,8 +42,9 @@ class DecodeCache:
 
     k, v:        [layers][num_pages][kv_heads][page_size][head_dim] (bf16 or fp32)
     block_table: [batch][max_pages] int32 physical page of each logical page
-    len:         [batch] int32;  next_pos: [batch] int32
-    pos, ema:    [rows][cap] int32 / fp32, rows = batch (per-sequence state) or batch * kv_heads
+    len:         [batch] int32 slots in use (dead slots included);  next_pos: [batch] int32
+    pos, ema:    [rows][cap] int32 / fp32, rows = batch (per-sequence state) or batch * kv_heads;
+                 pos = -1 marks a dead slot (deferred compaction)
     budget:      [batch] int32
     """
 
@@ -59,11 +80,11 @@ class DecodeCache:
         return ikv.ikv_shape(self.batch, self.layers, self.q_heads, self.kv_heads, self.head_dim, self.dtype,
                              self.granularity)
 
-    def cache(self, max_len: Optional[int] = None) -> ikv.ikv_cache:
+    def cache(self, max_len: Optional[int] = None, dead_slots: bool = False) -> ikv.ikv_cache:
         ml = self.max_len if max_len is None else max_len
         return ikv.ikv_cache(self.k.data_ptr(), self.v.data_ptr(), self.block_table.data_ptr(), self.num_pages,
                              self.page_size, self.max_pages, self.len.data_ptr(), self.pos.data_ptr(),
-                             self.next_pos.data_ptr(), ml, self.start.data_ptr())
+                             self.next_pos.data_ptr(), ml, self.start.data_ptr(), 1 if dead_slots else 0)
 
     @property
     def rows_per_seq(self) -> int:
@@ -105,7 +126,7 @@ class DecodeCache:
 
     def params(self, alpha: float, refresh_period: int = 1, score_free: bool = False,
                compact_mode: int = ikv.IKV_COMPACT_STABLE, refresh_init: int = ikv.IKV_INIT_ZERO,
-               layer_eligible: Optional[Sequence[int]] = None) -> ikv.ikv_params:
+               layer_eligible: Optional[Sequence[int]] = None, max_holes: int = 0) -> ikv.ikv_params:
         p = ikv.ikv_params()
         p.alpha = alpha
         p.refresh_period = refresh_period
@@ -116,6 +137,7 @@ class DecodeCache:
             p.layer_eligible = ctypes_addr(self._elig)
         p.compact_mode = compact_mode
         p.refresh_init = refresh_init
+        p.max_holes = max_holes
         return p
 
 

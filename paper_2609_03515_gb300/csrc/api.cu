@@ -72,6 +72,7 @@ ikv_status check_cache(const ikv_shape *s, const ikv_cache *c, bool need_pos) {
     if (!c) return fail(IKV_ERR_ARG, "cache is NULL");
     if (!c->k || !c->v || !c->block_table || !c->len) return fail(IKV_ERR_ARG, "cache k/v/block_table/len is NULL");
     if (need_pos && (!c->pos || !c->next_pos)) return fail(IKV_ERR_ARG, "cache pos/next_pos is NULL");
+    if (c->dead_slots && !c->pos) return fail(IKV_ERR_ARG, "dead_slots needs cache->pos");
     if (!aligned16(c->k) || !aligned16(c->v)) return fail(IKV_ERR_ALIGN, "K/V pools must be 16-byte aligned");
     if (c->page_size <= 0 || c->max_pages <= 0 || c->num_pages <= 0)
         return fail(IKV_ERR_SHAPE, "page_size/max_pages/num_pages must be positive");
@@ -217,6 +218,8 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
     a.lstride = logit_stride(a.cap);
     a.part_ml = at<float>(ws, w.part_ml);
     a.part_o = at<float>(ws, w.part_o);
+    a.pos = c->dead_slots ? c->pos : nullptr;
+    a.rows_per_seq = rows_per_seq(s);
     if (tc) {
         // fused combine: the last split of each unit writes out and lse2
         int32_t *arr = at<int32_t>(ws, w.arrivals);
@@ -353,12 +356,14 @@ ikv_status ikv_ema_update(int32_t rows, int32_t cap, float *ema, const float *sc
 }
 
 ikv_status ikv_select_budget(int32_t rows, int32_t cap, const float *util, const int32_t *len, int32_t rows_per_seq_,
-                             const int32_t *budget, int32_t *keep, int32_t *keep_len, cudaStream_t stream) {
+                             const int32_t *budget, const int32_t *pos, int32_t *keep, int32_t *keep_len,
+                             cudaStream_t stream) {
     g_err[0] = 0;
     if (rows < 0 || cap < 0 || rows_per_seq_ <= 0) return fail(IKV_ERR_SHAPE, "rows/cap/rows_per_seq out of range");
     if (rows > 0 && (!util || !len || !budget || !keep || !keep_len))
         return fail(IKV_ERR_ARG, "util/len/budget/keep/keep_len is NULL");
-    IKV_TRY_CUDA(launch_select(rows, cap, util, len, rows_per_seq_, budget, keep, keep_len, stream), "select launch");
+    IKV_TRY_CUDA(launch_select(rows, cap, util, len, rows_per_seq_, budget, pos, keep, keep_len, stream),
+                 "select launch");
     return IKV_OK;
 }
 
@@ -379,7 +384,7 @@ ikv_status ikv_compact_workspace_size(const ikv_shape *shape, const ikv_cache *c
 
 static ikv_status compact_impl(const ikv_shape *shape, ikv_cache *cache, const int32_t *keep, const int32_t *keep_len,
                                float *ema, int32_t mode, int32_t *moves, int32_t *n_moves, int32_t *done,
-                               cudaStream_t stream) {
+                               cudaStream_t stream, int32_t max_holes = 0) {
     CompactArgs a{};
     a.k = cache->k;
     a.v = cache->v;
@@ -399,6 +404,7 @@ static ikv_status compact_impl(const ikv_shape *shape, ikv_cache *cache, const i
     a.keep_len = keep_len;
     a.moves = moves;
     a.n_moves = n_moves;
+    a.max_holes = max_holes;
     IKV_TRY_CUDA(launch_compact(a, mode, stream), "compact launch");
     return IKV_OK;
 }
@@ -446,6 +452,7 @@ static ikv_status append_impl(const ikv_shape *shape, ikv_cache *cache, const vo
     a.next_pos = cache->next_pos;
     a.ema = ema;
     a.init_mean = ema ? init_mean : 0;
+    a.dead_slots = cache->dead_slots ? 1 : 0;
     a.done = done;
     if (!counters_zeroed)
         IKV_TRY_CUDA(cudaMemsetAsync(done, 0, sizeof(int32_t) * shape->batch, stream), "cudaMemsetAsync");
@@ -498,6 +505,11 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
         return fail(IKV_ERR_ARG, "IKV_COMPACT_STABLE_SHORT needs cache->start");
     if (p->refresh_init != IKV_INIT_ZERO && p->refresh_init != IKV_INIT_MEAN)
         return fail(IKV_ERR_ARG, "unknown refresh_init %d", p->refresh_init);
+    if (p->max_holes < 0) return fail(IKV_ERR_ARG, "max_holes must be >= 0");
+    // with deferred compaction every kernel of the step treats pos < 0 as a dead slot
+    ikv_cache cv = *cache;
+    if (p->max_holes > 0) cv.dead_slots = 1;
+    cache = &cv;
     const int32_t cap = cap_of(cache);
     if (cache->max_len + 1 > cap) return fail(IKV_ERR_SHAPE, "no free slot: max_len + 1 > cap");
     const StepWs w = step_ws(shape, cap);
@@ -530,12 +542,14 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
         return e;
     if (tm && (e = record(tm->score_end, stream))) return e;
     const int32_t R = shape->batch * rows_per_seq(shape);
-    IKV_TRY_CUDA(launch_select(R, cap, ema, cache->len, rows_per_seq(shape), p->budget, at<int32_t>(ws, w.keep),
+    IKV_TRY_CUDA(launch_select(R, cap, ema, cache->len, rows_per_seq(shape), p->budget,
+                               cache->dead_slots ? cache->pos : nullptr, at<int32_t>(ws, w.keep),
                                at<int32_t>(ws, w.keep_len), stream),
                  "select launch");
     if (tm && (e = record(tm->select_end, stream))) return e;
     if ((e = compact_impl(shape, cache, at<int32_t>(ws, w.keep), at<int32_t>(ws, w.keep_len), ema, p->compact_mode,
-                          at<int32_t>(ws, w.moves), at<int32_t>(ws, w.n_moves), at<int32_t>(ws, w.cdone), stream)))
+                          at<int32_t>(ws, w.moves), at<int32_t>(ws, w.n_moves), at<int32_t>(ws, w.cdone), stream,
+                          p->max_holes)))
         return e;
     if (tm && (e = record(tm->end, stream))) return e;
     return IKV_OK;

@@ -120,6 +120,7 @@ __global__ void __launch_bounds__(kAttendThreads, 2) attend_split_kernel(const A
     const int l = a.layer0 + li;
     const int L = a.len[b];
     const int S0 = a.pv.start_of(b);
+    const int32_t *prow = a.pos ? a.pos + ((int64_t)b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g)) * a.cap : nullptr;
     const int t0 = s * a.split_tokens;
     if (t0 >= L) return;
     const int t1 = min(t0 + a.split_tokens, L);
@@ -219,12 +220,13 @@ __global__ void __launch_bounds__(kAttendThreads, 2) attend_split_kernel(const A
         }
         __syncthreads();
 
-        // ---- logits of this tile (log2 domain), masked tail
+        // ---- logits of this tile (log2 domain), masked tail and dead slots (-inf)
         for (int idx = tid; idx < G * C::TT; idx += kAttendThreads) {
             const int h = idx / C::TT, j = idx % C::TT;
             float z = red[(0 * G + h) * C::TT + j] + red[(1 * G + h) * C::TT + j] + red[(2 * G + h) * C::TT + j] +
                       red[(3 * G + h) * C::TT + j];
             if (j < nv) {
+                if (prow && prow[tbase + j] < 0) z = -INFINITY;
                 if (LOGITS)
                     a.logits[((((int64_t)b * a.n_layers + li) * H) + g * G + h) * (int64_t)a.lstride + tbase + j] = z;
             } else {
@@ -240,8 +242,9 @@ __global__ void __launch_bounds__(kAttendThreads, 2) attend_split_kernel(const A
             const float mx = warp_max(fmaxf(za, zb));
             const float m_old = m_run[h];
             const float m_new = fmaxf(m_old, mx);
-            const float corr = exp2f(m_old - m_new);
-            const float pa = exp2f(za - m_new), pb = exp2f(zb - m_new);
+            const float m_ref = m_new == -INFINITY ? 0.f : m_new;  // every slot so far dead: nothing to scale
+            const float corr = exp2f(m_old - m_ref);
+            const float pa = exp2f(za - m_ref), pb = exp2f(zb - m_ref);
             const float sum = warp_sum(pa + pb);
             p_s[lane * C::GP + h] = pa;
             p_s[(lane + 32) * C::GP + h] = pb;
@@ -316,17 +319,18 @@ __global__ void __launch_bounds__(128) combine_kernel(const CombineArgs a) {
     const float *ml = a.part_ml + pbase * 2;
     float M = -INFINITY;
     for (int s = 0; s < ns; ++s) M = fmaxf(M, ml[2 * s]);
+    const float Mref = M == -INFINITY ? 0.f : M;  // splits whose slots are all dead carry -inf
     float wsum = 0.f;
-    for (int s = 0; s < ns; ++s) wsum += ml[2 * s + 1] * exp2f(ml[2 * s] - M);
-    const float inv = ns > 0 ? 1.f / wsum : 0.f;
+    for (int s = 0; s < ns; ++s) wsum += ml[2 * s + 1] * exp2f(ml[2 * s] - Mref);
+    const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
     const int64_t obase = (((int64_t)li * a.batch + b) * a.q_heads + h) * D;
     for (int e = threadIdx.x; e < D; e += blockDim.x) {
         float acc = 0.f;
-        for (int s = 0; s < ns; ++s) acc += a.part_o[(pbase + s) * D + e] * exp2f(ml[2 * s] - M);
+        for (int s = 0; s < ns; ++s) acc += a.part_o[(pbase + s) * D + e] * exp2f(ml[2 * s] - Mref);
         Chunk<T>::store(a.out, obase + e, acc * inv);
     }
     if (a.lse2 && threadIdx.x == 0)
-        a.lse2[((int64_t)b * a.n_layers + li) * a.q_heads + h] = ns > 0 ? M + log2f(wsum) : -INFINITY;
+        a.lse2[((int64_t)b * a.n_layers + li) * a.q_heads + h] = wsum > 0.f ? M + log2f(wsum) : -INFINITY;
 }
 
 template <typename T, int D, int G>

@@ -70,6 +70,8 @@ struct TcArgs {
     __nv_bfloat16 *out;         // [n_layers][batch][H][128]
     float *lse2;                // [batch][n_layers][H]
     int32_t *arrivals;          // [batch][n_layers][kv_heads], zero on entry, left zero
+    const int32_t *pos;         // [rows][cap], -1 at dead slots; null: every slot below len is live
+    int32_t rows_per_seq;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -358,15 +360,25 @@ __global__ void __launch_bounds__(kThreads, 2)
             mx[h] = -INFINITY;
             sum[h] = 0.f;
         }
+        // bit i: this thread's row of tile i is a valid, live slot.  The liveness of every
+        // tile is fetched before the wait for the QK products, so its latency is hidden.
+        uint32_t live_bits = 0u;
+        {
+            const int32_t *prow =
+                a.pos ? a.pos + ((int64_t)b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g)) * a.cap : nullptr;
+            for (int i = 0; i < n; ++i) {
+                const int tok = t0 + i * kTile + tid;  // physical slot; logical slot tok - S0
+                if (tok >= lo && tok < t1 && (!prow || __ldg(prow + (tok - S0)) >= 0)) live_bits |= 1u << i;
+            }
+        }
         bool ok = __all_sync(0xffffffffu, mbar_wait(s_full, 0, abort_flag));
         fence_after_sync();
-        // sweep 1: split maximum
+        // sweep 1: split maximum (-inf for a head when every row of the chunk is dead)
         if (ok) {
             for (int i = 0; i < n; ++i) {
                 float v[NC];
                 tmem_ld<NC>(tS + lane_off + kN * i, v);
-                const int tok = t0 + i * kTile + tid;
-                if (tok >= lo && tok < t1) {
+                if ((live_bits >> i) & 1u) {
 #pragma unroll
                     for (int h = 0; h < G; ++h) mx[h] = fmaxf(mx[h], v[h] * a.scale_log2);
                 }
@@ -397,13 +409,14 @@ __global__ void __launch_bounds__(kThreads, 2)
             tmem_ld<NC>(tS + lane_off + kN * i, v);
             const int tok = t0 + i * kTile + tid;
             const bool valid = tok >= lo && tok < t1;
+            const bool live = (live_bits >> i) & 1u;  // valid and not dead
             unsigned char *pbuf = sm + kOffP + (i & 1) * kOpBytes + (tid >> 6) * (kN * 128);
 #pragma unroll
             for (int h = 0; h < G; ++h) {
                 const float z = v[h] * a.scale_log2;
                 float p = 0.f;
-                if (valid) {
-                    if (a.logits) a.logits[lbase + (int64_t)h * a.lstride + (tok - S0)] = z;
+                if (valid && a.logits) a.logits[lbase + (int64_t)h * a.lstride + (tok - S0)] = live ? z : -INFINITY;
+                if (live) {  // mx[h] is finite here: it covers this row
                     p = exp2f(z - mx[h]);
                     sum[h] += p;
                 }
@@ -485,12 +498,15 @@ __global__ void __launch_bounds__(kThreads, 2)
                     float mn = M[h];
 #pragma unroll
                     for (int j = 0; j < MQ; ++j) mn = fmaxf(mn, mq[j][h]);
-                    const float sc = exp2f(M[h] - mn);  // 0 while M is -inf
+                    // chunks whose rows are all dead carry max -inf and sum 0; while every
+                    // chunk so far is such, mn stays -inf and nothing accumulates
+                    const float mref = mn == -INFINITY ? 0.f : mn;
+                    const float sc = exp2f(M[h] - mref);  // 0 while M is -inf
                     ws[h] *= sc;
                     acc[h] *= sc;
 #pragma unroll
                     for (int j = 0; j < MQ; ++j) {
-                        const float wq = exp2f(mq[j][h] - mn);  // 0 for padding slots
+                        const float wq = exp2f(mq[j][h] - mref);  // 0 for padding and all-dead chunks
                         ws[h] += lq[j][h] * wq;
                         acc[h] += oq[j][h] * wq;
                     }
@@ -499,8 +515,11 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
 #pragma unroll
             for (int h = 0; h < G; ++h) {
-                a.out[(((int64_t)li * a.batch + b) * H + (int64_t)g * G + h) * kD + tid] = __float2bfloat16_rn(acc[h] / ws[h]);
-                if (tid == 0) a.lse2[((int64_t)b * a.n_layers + li) * H + (int64_t)g * G + h] = M[h] + log2f(ws[h]);
+                const bool any = ws[h] > 0.f;  // false only if every slot of the unit is dead
+                a.out[(((int64_t)li * a.batch + b) * H + (int64_t)g * G + h) * kD + tid] =
+                    __float2bfloat16_rn(any ? acc[h] / ws[h] : 0.f);
+                if (tid == 0)
+                    a.lse2[((int64_t)b * a.n_layers + li) * H + (int64_t)g * G + h] = any ? M[h] + log2f(ws[h]) : -INFINITY;
             }
             if (tid == 0) a.arrivals[unit] = 0;
         }
@@ -612,6 +631,8 @@ cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group,
     t.out = reinterpret_cast<__nv_bfloat16 *>(o.out);
     t.lse2 = o.lse2;
     t.arrivals = o.arrivals;
+    t.pos = a.pos;
+    t.rows_per_seq = a.rows_per_seq;
     dim3 grid(a.n_splits * a.pv.kv_heads * a.batch * a.n_layers);
     cudaError_t e;
     switch (group) {
@@ -633,7 +654,9 @@ extern "C" ikv_status ikv_device_status(uint32_t *flags) {
     unsigned int v = 0, z = 0;
     cudaError_t e = cudaMemcpyFromSymbol(&v, ikv::g_tc_error, sizeof(v));
     if (e == cudaSuccess) e = cudaMemcpyToSymbol(ikv::g_tc_error, &z, sizeof(z));
+    unsigned int ap = 0;
+    if (e == cudaSuccess) e = ikv::read_clear_append_error(&ap);
     if (e != cudaSuccess) return ikv::report(IKV_ERR_CUDA, "ikv_device_status: %s", cudaGetErrorString(e));
-    *flags = v;
+    *flags = v | (ap ? 4u : 0u);
     return IKV_OK;
 }

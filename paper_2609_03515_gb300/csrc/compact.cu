@@ -12,8 +12,12 @@
 // to at most D, so either the suffix moves left (start kept) or the prefix before
 // the first slot with keep[j] = j + D moves right by its gap (start += D) --
 // whichever moves fewer rows.  The right move walks descending tiles, the mirror
-// image of the left one.  Survivors keep their order either way.  Extra CTAs per
-// row gather the utility and position arrays (logical slots, always left).
+// image of the left one.  start only grows that way, so when the right move
+// finds no room for the next append before cap, every row moves to slot 0 once
+// (an ascending left move with start = 0), provided that frees at least 128
+// slots of room; otherwise the suffix moves left.  Survivors keep their order
+// in every case.  Extra CTAs per row gather the utility and position arrays
+// (logical slots, always left).
 //
 // Hole-fill mode: survivors at slots >= n move into the evicted slots below n
 // (k-th hole <- k-th such survivor).  Sources and destinations are disjoint,
@@ -58,6 +62,28 @@ __device__ __forceinline__ float block_sum(float v, float *scratch) {
     return r;
 }
 
+// Deferred compaction: sequence b only marks its evicted slots dead while its dead
+// slots (the ones already dead plus this step's evictions: len - kept) stay within
+// max_holes.  Every row of b keeps the same number of slots, so row b * rps decides.
+// A sequence whose slot space has no room left for the next append (start + len
+// = cap) compacts instead.
+__device__ __forceinline__ bool defer_of(const CompactArgs &a, int b, int L, int S) {
+    return a.max_holes > 0 && L - a.keep_len[b * a.rows_per_seq] <= a.max_holes && S + L < a.cap;
+}
+
+// pos = -1 at every slot below L of row r that keep[r] does not list (runs of
+// slots between consecutive kept slots; keep is ascending).
+__device__ __forceinline__ void mark_dead_row(const CompactArgs &a, int r, int L) {
+    const int n = a.keep_len[r];
+    const int32_t *kp = a.keep + (int64_t)r * a.cap;
+    int32_t *pos = a.pos + (int64_t)r * a.cap;
+    for (int i = threadIdx.x; i <= n; i += blockDim.x) {
+        const int lo = i == 0 ? 0 : kp[i - 1] + 1;
+        const int hi = i == n ? L : kp[i];
+        for (int j = lo; j < hi; ++j) pos[j] = -1;
+    }
+}
+
 // Stable compaction of one sequence's rows (see the file comment).  Every CTA of
 // sequence b reads len[b] and start[b] first; the last CTA of b to arrive writes
 // the new values, so no CTA sees them early.
@@ -70,6 +96,10 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
     const int nkv = a.layers * kvh;
     const int L = a.len[b];
     const int S = a.start ? a.start[b] : 0;
+    if (defer_of(a, b, L, S)) {  // nothing moves; len, start and the arrival counter stay as they are
+        if (x >= nkv) mark_dead_row(a, b * a.rows_per_seq + (x - nkv), L);
+        return;
+    }
     // shorter-side decision, identical in every CTA of b (it depends on row b only;
     // rows of several KV heads share b's slot space, so they always compact left).
     // K/V row j lands at physical slot new_start + j; it moves iff S + kp[j] differs.
@@ -87,13 +117,17 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
         }
         jl = block_min_int(jl, scratch);
         jr = block_min_int(jr, scratch);
+        // room for the appends until the next compaction: one, plus max_holes deferred ones
+        const int need = n0 + 1 + max(a.max_holes, 0);
         if (jr < n0 - jl) {
-            if (S + D + n0 + 1 <= a.cap)                        // room for the next append
+            if (S + D + need <= a.cap)                              // the prefix moves right
                 new_start = S + D;
-            else if (S > 0 && a.cap - (n0 + 1) >= kRelocateSlack)  // out of room: move all rows
-                new_start = 0;                                 // to slot 0 once, regaining it
+            else if (S > 0 && a.cap - need >= kRelocateSlack)       // out of room: move all rows
+                new_start = 0;                                      // to slot 0 once, regaining it
         }
     }
+    // whatever the mode, the next append must find a free slot: else move every row to slot 0
+    if (a.start && new_start + n0 + 1 > a.cap) new_start = 0;
     if (x < nkv) {
         const int l = x / kvh, g = x % kvh;
         const int r = b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g);
@@ -205,32 +239,44 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
 }
 
 // Hole-fill move list of one row: for every evicted slot h < n (the k-th such),
-// move the k-th survivor found at a slot >= n into it.
-__global__ void holefill_plan_kernel(const CompactArgs a) {
+// move the k-th survivor found at a slot >= n into it.  keep is ascending, so the
+// gap g_j = keep[j] - j is non-decreasing over the `below` survivors < n; the
+// holes just before keep[j] are the g_j - g_{j-1} slots keep[j] - g_j + k for
+// hole indices k in [g_{j-1}, g_j), and the holes after the last of them are the
+// slots below + k.  One coalesced pass over keep, no searching.
+constexpr int kPlanThreads = 1024;
+
+__global__ void __launch_bounds__(kPlanThreads) holefill_plan_kernel(const CompactArgs a) {
+    __shared__ int below_s;
     const int r = blockIdx.x;
     const int n = a.keep_len[r];
     const int32_t *kp = a.keep + (int64_t)r * a.cap;
-    // survivors below n: lower_bound(kp, n)
-    int lo = 0, hi = n;
-    while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if (kp[mid] < n) lo = mid + 1; else hi = mid;
+    if (defer_of(a, r / a.rows_per_seq, a.len[r / a.rows_per_seq], a.pv.start_of(r / a.rows_per_seq))) {
+        // decided here, before len changes
+        if (threadIdx.x == 0) a.n_moves[r] = -1;
+        return;
     }
-    const int below = lo;
-    const int n_tail = n - below;
+    if (threadIdx.x == 0) below_s = 0;
+    __syncthreads();
+    int cnt = 0;
+    for (int j = threadIdx.x; j < n; j += kPlanThreads) cnt += kp[j] < n;
+    if (cnt) atomicAdd(&below_s, cnt);
+    __syncthreads();
+    const int below = below_s;       // survivors already below n
+    const int n_tail = n - below;    // survivors at slots >= n = holes below n
     int32_t *mv = a.moves + (int64_t)r * a.cap * 2;
-    for (int h = threadIdx.x; h < n; h += blockDim.x) {
-        int l2 = 0, h2 = below;  // entries < h among kp[0..below)
-        while (l2 < h2) {
-            const int mid = (l2 + h2) >> 1;
-            if (kp[mid] < h) l2 = mid + 1; else h2 = mid;
+    for (int j = threadIdx.x; j < below; j += kPlanThreads) {
+        const int kj = kp[j];
+        const int g = kj - j, gp = j ? kp[j - 1] - (j - 1) : 0;
+        for (int k = gp; k < g; ++k) {
+            mv[2 * k] = kp[below + k];
+            mv[2 * k + 1] = kj - g + k;
         }
-        const bool kept = l2 < below && kp[l2] == h;
-        if (!kept) {
-            const int hole = h - l2;
-            mv[2 * hole] = kp[below + hole];
-            mv[2 * hole + 1] = h;
-        }
+    }
+    const int g_last = below ? kp[below - 1] - (below - 1) : 0;
+    for (int k = g_last + threadIdx.x; k < n_tail; k += kPlanThreads) {
+        mv[2 * k] = kp[below + k];
+        mv[2 * k + 1] = below + k;
     }
     if (threadIdx.x == 0) a.n_moves[r] = n_tail;
 }
@@ -243,7 +289,7 @@ __global__ void __launch_bounds__(kCompThreads) holefill_move_kernel(const Compa
     if (x < nkv) {
         const int l = x / kvh, g = x % kvh;
         const int r = b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g);
-        const int nm = a.n_moves[r];
+        const int nm = a.n_moves[r];  // -1: deferred, nothing moves
         const int32_t *mv = a.moves + (int64_t)r * a.cap * 2;
         const int S = a.pv.start_of(b);
         const int rowB = a.pv.head_dim * a.elem_bytes;
@@ -262,6 +308,10 @@ __global__ void __launch_bounds__(kCompThreads) holefill_move_kernel(const Compa
     const int rr = x - nkv;
     const int r = b * a.rows_per_seq + rr;
     const int nm = a.n_moves[r];
+    if (nm < 0) {  // deferred: mark this step's evictions dead; len stays
+        mark_dead_row(a, r, a.len[b]);
+        return;
+    }
     const int32_t *mv = a.moves + (int64_t)r * a.cap * 2;
     int32_t *pos = a.pos + (int64_t)r * a.cap;
     float *ema = a.ema ? a.ema + (int64_t)r * a.cap : nullptr;
@@ -278,6 +328,12 @@ __global__ void __launch_bounds__(kCompThreads) holefill_move_kernel(const Compa
 // the last CTA of sequence b to arrive advances len[b] and next_pos[b] (every
 // CTA reads len[b] before it arrives, so nobody sees the new value early).
 constexpr int kAppendRows = 8;
+
+}  // namespace
+
+__device__ unsigned int g_append_error = 0;  // bit 0: an append found no free slot (start + len = cap)
+
+namespace {
 
 __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a) {
     __shared__ float scratch[32];
@@ -310,9 +366,16 @@ __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a
                 const int64_t r = (int64_t)b * a.rows_per_seq + rr;
                 float init = 0.f;
                 if (a.init_mean && L > 0) {
-                    float s = 0.f;
-                    for (int i = tid; i < L; i += kCompThreads) s += a.ema[r * a.cap + i];
-                    init = block_sum(s, scratch) / (float)L;
+                    float s = 0.f, c = 0.f;
+                    const int32_t *pr = a.pos + r * a.cap;
+                    for (int i = tid; i < L; i += kCompThreads)
+                        if (!a.dead_slots || pr[i] >= 0) {  // the mean over live slots only
+                            s += a.ema[r * a.cap + i];
+                            c += 1.f;
+                        }
+                    s = block_sum(s, scratch);
+                    c = a.dead_slots ? block_sum(c, scratch) : (float)L;
+                    init = c > 0.f ? s / c : 0.f;
                 }
                 if (tid == 0) {
                     if (a.ema) a.ema[r * a.cap + L] = init;
@@ -330,6 +393,8 @@ __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a
             if (S + L < a.cap) {
                 a.len[b] = L + 1;
                 a.next_pos[b] = a.next_pos[b] + 1;
+            } else {
+                atomicOr(&g_append_error, 1u);  // the token was not stored; ikv_device_status reports it
             }
             a.done[b] = 0;
         }
@@ -353,11 +418,18 @@ cudaError_t launch_compact(const CompactArgs &a, int mode, cudaStream_t st) {
         note_launch();
         return cudaGetLastError();
     }
-    holefill_plan_kernel<<<a.batch * a.rows_per_seq, 256, 0, st>>>(a);
+    holefill_plan_kernel<<<a.batch * a.rows_per_seq, kPlanThreads, 0, st>>>(a);
     note_launch();
     holefill_move_kernel<<<grid, kCompThreads, 0, st>>>(a);
     note_launch();
     return cudaGetLastError();
+}
+
+cudaError_t read_clear_append_error(unsigned int *v) {
+    unsigned int z = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(v, g_append_error, sizeof(*v));
+    if (e == cudaSuccess) e = cudaMemcpyToSymbol(g_append_error, &z, sizeof(z));
+    return e;
 }
 
 cudaError_t launch_append(const AppendArgs &a, cudaStream_t st) {

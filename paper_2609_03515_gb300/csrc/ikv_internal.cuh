@@ -49,6 +49,8 @@ struct AttendArgs {
     int32_t lstride;            // logits row stride: cap rounded up to a multiple of 128
     float *part_ml;             // [batch][n_layers][H][n_splits][2]  (running max, sum) in log2 domain
     float *part_o;              // [batch][n_layers][H][n_splits][D]  unnormalised partial output
+    const int32_t *pos;         // [rows][cap] with -1 at dead slots, or null (every slot below len live)
+    int32_t rows_per_seq;       // utility rows per sequence (row of (b, g): b * rows_per_seq + g or b)
 };
 
 struct CombineArgs {
@@ -92,7 +94,8 @@ cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, int sms, cudaS
 cudaError_t launch_ema_update(int32_t rows, int32_t cap, float *ema, const float *score, const int32_t *len,
                               int32_t rows_per_seq, float alpha, int32_t max_len, cudaStream_t st);
 cudaError_t launch_select(int32_t rows, int32_t cap, const float *util, const int32_t *len, int32_t rows_per_seq,
-                          const int32_t *budget, int32_t *keep, int32_t *keep_len, cudaStream_t st);
+                          const int32_t *budget, const int32_t *pos, int32_t *keep, int32_t *keep_len,
+                          cudaStream_t st);
 
 struct CompactArgs {
     void *k, *v;
@@ -106,6 +109,8 @@ struct CompactArgs {
     const int32_t *keep, *keep_len;
     int32_t *moves;             // hole-fill: [rows][cap][2] (src, dst), null for stable
     int32_t *n_moves;           // hole-fill: [rows]
+    int32_t max_holes;          // > 0: while a sequence's dead slots stay <= max_holes, mark
+                                // the evicted slots dead (pos = -1) instead of compacting
 };
 cudaError_t launch_compact(const CompactArgs &a, int mode, cudaStream_t st);
 
@@ -117,8 +122,11 @@ struct AppendArgs {
     int32_t *len, *pos, *next_pos;
     float *ema;
     int32_t init_mean;
+    int32_t dead_slots;         // the mean initialisation skips slots with pos < 0
     int32_t *done;              // [batch] arrival counters, zero on entry; reset by the last CTA
 };
 cudaError_t launch_append(const AppendArgs &a, cudaStream_t st);
+// reads and clears the append kernel's device error word (bit 0: no free slot)
+cudaError_t read_clear_append_error(unsigned int *v);
 
 }  // namespace ikv

@@ -2,15 +2,17 @@
 // lowest m whenever the cache exceeds B).
 //
 // One 1024-thread CTA per utility row.  Utilities map to order-preserving
-// 32-bit keys (sign-flipped IEEE bits; -0.0 folded onto +0.0; NaN -> 0, the
-// lowest key).  General case: an MSB-first radix select with 8-bit digits
-// (four passes, warp-aggregated shared-memory histograms) finds the exact B-th
-// largest key theta and how many theta-valued slots survive; one more pass
-// writes the kept slots in ascending order (two block scans per 1024-slot
-// chunk), keeping the lowest slots among keys equal to theta.  Steady-state
-// case L == B + 1: a single pass finds the one slot to evict (lowest key, and
-// among equal keys the highest slot).  The result depends only on the fp32
-// values, so it is bit-exact against any correct sort.
+// 32-bit keys (sign-flipped IEEE bits; -0.0 folded onto +0.0; NaN -> 1, below
+// every number).  Dead slots (pos < 0, deferred compaction) get key 0: below
+// every live key, never kept, not counted against B.  General case: an
+// MSB-first radix select with 8-bit digits (four passes, warp-aggregated
+// shared-memory histograms) finds the exact B-th largest key theta and how
+// many theta-valued slots survive; one more pass writes the kept slots in
+// ascending order (two block scans per 1024-slot chunk), keeping the lowest
+// slots among keys equal to theta.  Steady-state case, one live slot too many:
+// a single pass finds the slot to evict (lowest key, and among equal keys the
+// highest slot).  The result depends only on the fp32 values, so it is
+// bit-exact against any correct sort.
 #include "ikv_internal.cuh"
 
 namespace ikv {
@@ -20,10 +22,11 @@ constexpr int kSelThreads = 1024;
 
 __device__ __forceinline__ uint32_t ord_key(float f) {
     uint32_t u = __float_as_uint(f);
-    if ((u & 0x7FFFFFFFu) > 0x7F800000u) return 0u;  // NaN: lowest
+    if ((u & 0x7FFFFFFFu) > 0x7F800000u) return 1u;  // NaN: below every number (-inf maps to 0x007FFFFF)
     if ((u & 0x7FFFFFFFu) == 0u) u = 0u;              // -0.0 == +0.0
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
+constexpr uint32_t kDeadKey = 0u;  // dead slots: below every live key, never kept
 
 // exclusive scan of one value per thread across the block; returns (exclusive, total)
 __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t *warp_tot, uint32_t &total) {
@@ -54,12 +57,13 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t *warp_t
 
 __global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const float *__restrict__ util,
                                                               const int32_t *__restrict__ len, int32_t rps,
-                                                              const int32_t *__restrict__ budget, int32_t *keep,
+                                                              const int32_t *__restrict__ budget,
+                                                              const int32_t *__restrict__ pos, int32_t *keep,
                                                               int32_t *keep_len) {
     __shared__ uint32_t hist[256];
     __shared__ uint32_t warp_tot[32];
     __shared__ unsigned long long s_min[32];
-    __shared__ uint32_t s_digit, s_above;
+    __shared__ uint32_t s_digit, s_above, s_live;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int r = blockIdx.x;
@@ -67,11 +71,41 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const 
     int B = budget[r / rps];
     if (B < 0) B = 0;
     const float *u = util + (int64_t)r * cap;
+    const int32_t *pr = pos ? pos + (int64_t)r * cap : nullptr;
     int32_t *kp = keep + (int64_t)r * cap;
+    auto live = [&](int i) { return !pr || pr[i] >= 0; };
+    auto key_at = [&](int i) { return live(i) ? ord_key(u[i]) : kDeadKey; };
+    // every slot i < L for which keep_if(i) holds, in ascending order (block scans)
+    auto write_kept = [&](auto keep_if) {
+        uint32_t run = 0u;
+        for (int base = 0; base < L; base += kSelThreads) {
+            const int i = base + tid;
+            const uint32_t kf = (i < L && keep_if(i)) ? 1u : 0u;
+            uint32_t tot;
+            const uint32_t at = block_excl_scan(kf, warp_tot, tot);
+            if (kf) kp[run + at] = i;
+            run += tot;
+        }
+    };
 
-    if (L <= B) {
-        for (int j = tid; j < L; j += kSelThreads) kp[j] = j;
-        if (tid == 0) keep_len[r] = L;
+    int n_live = L;
+    if (pr) {
+        if (tid == 0) s_live = 0u;
+        __syncthreads();
+        uint32_t c = 0u;
+        for (int i = tid; i < L; i += kSelThreads) c += pr[i] >= 0;
+        if (c) atomicAdd(&s_live, c);
+        __syncthreads();
+        n_live = (int)s_live;
+    }
+
+    if (n_live <= B) {
+        if (n_live == L) {
+            for (int j = tid; j < L; j += kSelThreads) kp[j] = j;
+        } else {
+            write_kept([&](int i) { return live(i); });
+        }
+        if (tid == 0) keep_len[r] = n_live;
         return;
     }
     if (B == 0) {
@@ -79,10 +113,11 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const 
         return;
     }
 
-    if (L == B + 1) {
-        // evict exactly one: minimum of (key, ~slot)
+    if (n_live == B + 1) {
+        // evict exactly one: minimum of (key, ~slot) over the live slots
         unsigned long long best = ~0ull;
         for (int i = tid; i < L; i += kSelThreads) {
+            if (!live(i)) continue;
             const unsigned long long v = ((unsigned long long)ord_key(u[i]) << 32) | (uint32_t)(~(uint32_t)i);
             best = v < best ? v : best;
         }
@@ -104,11 +139,18 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const 
         }
         __syncthreads();
         const int ev = (int)(~(uint32_t)(s_min[0] & 0xFFFFFFFFull));
-        for (int j = tid; j < B; j += kSelThreads) kp[j] = j < ev ? j : j + 1;
+        if (n_live == L) {
+            for (int j = tid; j < B; j += kSelThreads) kp[j] = j < ev ? j : j + 1;
+        } else {
+            write_kept([&](int i) { return i != ev && live(i); });
+        }
         if (tid == 0) keep_len[r] = B;
         return;
     }
 
+    // general case: B < n_live - 1.  Dead slots carry the lowest key, and more than B
+    // live keys lie above it, so the B-th largest key theta is live and no dead slot
+    // is ever kept.
     uint32_t prefix = 0u, mask = 0u, k = (uint32_t)B;
     for (int pass = 0; pass < 4; ++pass) {
         const int shift = 24 - 8 * pass;
@@ -118,7 +160,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const 
             const int i = base + tid;
             uint32_t digit = 0xFFFFu;
             if (i < L) {
-                const uint32_t key = ord_key(u[i]);
+                const uint32_t key = key_at(i);
                 if ((key & mask) == prefix) digit = (key >> shift) & 0xFFu;
             }
             const uint32_t peers = __match_any_sync(0xffffffffu, digit);
@@ -163,7 +205,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const 
         const int i = base + tid;
         uint32_t key = 0u;
         bool in = i < L;
-        if (in) key = ord_key(u[i]);
+        if (in) key = key_at(i);
         const uint32_t gt = (in && key > theta) ? 1u : 0u;
         const uint32_t eq = (in && key == theta) ? 1u : 0u;
         uint32_t eq_tot, kp_tot;
@@ -180,9 +222,10 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const 
 }  // namespace
 
 cudaError_t launch_select(int32_t rows, int32_t cap, const float *util, const int32_t *len, int32_t rows_per_seq,
-                          const int32_t *budget, int32_t *keep, int32_t *keep_len, cudaStream_t st) {
+                          const int32_t *budget, const int32_t *pos, int32_t *keep, int32_t *keep_len,
+                          cudaStream_t st) {
     if (rows <= 0) return cudaSuccess;
-    select_kernel<<<rows, kSelThreads, 0, st>>>(cap, util, len, rows_per_seq, budget, keep, keep_len);
+    select_kernel<<<rows, kSelThreads, 0, st>>>(cap, util, len, rows_per_seq, budget, pos, keep, keep_len);
     note_launch();
     return cudaGetLastError();
 }

@@ -34,7 +34,7 @@ class ikv_shape(ctypes.Structure):
 
 class ikv_cache(ctypes.Structure):
     _fields_ = [("k", P), ("v", P), ("block_table", P), ("num_pages", I32), ("page_size", I32), ("max_pages", I32),
-                ("len", P), ("pos", P), ("next_pos", P), ("max_len", I32), ("start", P)]
+                ("len", P), ("pos", P), ("next_pos", P), ("max_len", I32), ("start", P), ("dead_slots", I32)]
 
 
 class ikv_timing(ctypes.Structure):
@@ -45,7 +45,7 @@ class ikv_timing(ctypes.Structure):
 class ikv_params(ctypes.Structure):
     _fields_ = [("alpha", F32), ("refresh_period", I32), ("score_free", I32), ("budget", P),
                 ("layer_eligible", P), ("compact_mode", I32), ("refresh_init", I32),
-                ("timing", ctypes.POINTER(ikv_timing))]
+                ("timing", ctypes.POINTER(ikv_timing)), ("max_holes", I32)]
 
 
 class IKVError(RuntimeError):
@@ -69,7 +69,7 @@ def _load():
         "ikv_static_scratch_bytes": ([], SZ),
         "ikv_decode_attend_score_static": ([SP, CP, I32, P, P, P, P, F32, P], I32),
         "ikv_ema_update": ([I32, I32, P, P, P, I32, F32, P], I32),
-        "ikv_select_budget": ([I32, I32, P, P, I32, P, P, P, P], I32),
+        "ikv_select_budget": ([I32, I32, P, P, I32, P, P, P, P, P], I32),
         "ikv_compact_workspace_size": ([SP, CP, I32, ctypes.POINTER(SZ)], I32),
         "ikv_compact_kv": ([SP, CP, P, P, P, I32, P, SZ, P], I32),
         "ikv_append_token": ([SP, CP, P, P, P, I32, P, SZ, P], I32),
@@ -154,9 +154,9 @@ def ikv_ema_update(rows, cap, ema, score, length, rows_per_seq, alpha, stream=No
            "ikv_ema_update")
 
 
-def ikv_select_budget(rows, cap, util, length, rows_per_seq, budget, keep, keep_len, stream=None) -> None:
-    _check(_lib.ikv_select_budget(rows, cap, _p(util), _p(length), rows_per_seq, _p(budget), _p(keep), _p(keep_len),
-                                  _stream(stream)), "ikv_select_budget")
+def ikv_select_budget(rows, cap, util, length, rows_per_seq, budget, pos, keep, keep_len, stream=None) -> None:
+    _check(_lib.ikv_select_budget(rows, cap, _p(util), _p(length), rows_per_seq, _p(budget), _p(pos), _p(keep),
+                                  _p(keep_len), _stream(stream)), "ikv_select_budget")
 
 
 def ikv_compact_workspace_size(shape, cache, mode) -> int:

@@ -19,7 +19,7 @@ import torch
 
 import gen
 import oracle as O
-from paper_2609_03515_gb300 import DecodeCache, ikv
+from paper_2609_03515_gb300 import DecodeCache, ikv, step_lengths
 
 GAP = 1e-4          # retained-set boundary rule
 TOL_M = 1e-3        # utilities, fp32 vs fp64
@@ -112,9 +112,17 @@ class StepReport:
     refresh: bool = True
 
 
+STABLE_MODES = (ikv.IKV_COMPACT_STABLE, ikv.IKV_COMPACT_STABLE_SHORT)
+
+
+def live_slots(pos_row: np.ndarray, n: int) -> np.ndarray:
+    """Logical slots below n that hold a live token (pos >= 0; -1 marks a dead slot)."""
+    return np.nonzero(pos_row[:n] >= 0)[0]
+
+
 def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: int = ikv.IKV_COMPACT_STABLE,
                  steps: Optional[int] = None, kv_check_layers=(0, -1), page_perm_seed: Optional[int] = 7,
-                 refresh_init: int = ikv.IKV_INIT_ZERO, layer_eligible=None) -> List[StepReport]:
+                 refresh_init: int = ikv.IKV_INIT_ZERO, layer_eligible=None, max_holes: int = 0) -> List[StepReport]:
     T = w.steps if steps is None else steps
     u = w.u_table()
     c = make_cache(w, gran, page_perm_seed)
@@ -124,11 +132,11 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
                   granularity=O.GRAN_SEQ if gran == ikv.IKV_GRAN_SEQ else O.GRAN_KVHEAD,
                   layer_mask=None if layer_eligible is None else [bool(x) for x in layer_eligible],
                   refresh_init="zero" if refresh_init == ikv.IKV_INIT_ZERO else "mean")
-    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, refresh_init, layer_eligible)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, refresh_init, layer_eligible, max_holes)
     ws = c.step_workspace()
     qs = w.queries(1, T + 1, u)
     budgets = w.budgets()
-    lens = list(w.prefill)
+    lens, live = list(w.prefill), list(w.prefill)
     out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
     tol_out = TOL_OUT_BF16 if w.dtype == gen.BF16 else TOL_OUT_F32
     reports = []
@@ -137,7 +145,7 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
         kn, vn = w.new_tokens(t, u)
         ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, to_device(qs[t - 1], w), to_device(kn, w),
                      to_device(vn, w), out, ws, ws.numel())
-        lens = [min(L + 1, B) if L + 1 > B else L + 1 for L, B in zip(lens, budgets)]
+        lens, live = step_lengths(lens, live, budgets, max_holes)
         torch.cuda.synchronize()
         out_h = out.float().cpu().numpy()
         ema_h = c.ema.cpu().numpy()
@@ -150,13 +158,17 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
             O.append_token(st, kn[:, b], vn[:, b], refresh, op)
             o_out = O.attend_and_score(st, q64[:, b], refresh, op)
             rep.out_err = max(rep.out_err, float(np.max(np.abs(out_h[:, b] - o_out))))
-            assert len_h[b] == min(st.length, budgets[b]), (t, b, len_h[b], st.length)
+            assert len_h[b] == lens[b], (t, b, len_h[b], lens[b])
             keeps = []
             for rr in range(R):
                 r = b * R + rr
-                n = int(len_h[b])
-                gpos = pos_h[r, :n]
-                gm = ema_h[r, :n]
+                ls = live_slots(pos_h[r], int(len_h[b]))
+                n = len(ls)
+                assert n == min(st.length, budgets[b]), (t, b, n, st.length)
+                gpos = pos_h[r, ls]
+                gm = ema_h[r, ls]
+                if compact_mode in STABLE_MODES:  # survivors keep their order (R5)
+                    assert np.all(np.diff(gpos) > 0), (t, b, rr)
                 slot_of = {int(pp): i for i, pp in enumerate(st.pos[rr])}
                 assert len(set(gpos.tolist())) == n
                 oslots = np.array([slot_of[int(pp)] for pp in gpos])
@@ -173,10 +185,10 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
             for l in kv_check_layers:
                 for g in range(w.kv_heads):
                     rr = 0 if R == 1 else g
-                    n = int(len_h[b])
-                    gk = c.gather(c.k, b, l % w.layers, g, n).float().cpu().numpy()
-                    gv = c.gather(c.v, b, l % w.layers, g, n).float().cpu().numpy()
-                    order = np.argsort(np.argsort(pos_h[b * R + rr, :n]))  # gpu slot -> rank by position
+                    ls = live_slots(pos_h[b * R + rr], int(len_h[b]))
+                    gk = c.gather(c.k, b, l % w.layers, g, int(len_h[b])).float().cpu().numpy()[ls]
+                    gv = c.gather(c.v, b, l % w.layers, g, int(len_h[b])).float().cpu().numpy()[ls]
+                    order = np.argsort(np.argsort(pos_h[b * R + rr, ls]))  # gpu live slot -> rank by position
                     ok_rows = st.K[l][g][order]
                     ov_rows = st.V[l][g][order]
                     rep.kv_err = max(rep.kv_err, float(np.max(np.abs(gk - ok_rows))), float(np.max(np.abs(gv - ov_rows))))
@@ -186,7 +198,7 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
 
 
 def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1), page_perm_seed: Optional[int] = 7,
-                         compact_mode: int = ikv.IKV_COMPACT_STABLE):
+                         compact_mode: int = ikv.IKV_COMPACT_STABLE, max_holes: int = 0):
     """Full-size lock-step for a few sequences of a workload (GRAN_SEQ).
 
     The GPU decodes the whole batch at its real size (device-generated prefill, the
@@ -201,11 +213,11 @@ def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1)
     c = make_cache(w, ikv.IKV_GRAN_SEQ, page_perm_seed)
     fill_device(c, w, u_dev)
     op = O.Params(alpha=w.alpha, refresh_period=w.refresh_period, score_free=w.score_free)
-    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=max_holes)
     ws = c.step_workspace()
     qs = w.queries(1, T + 1, u)
     budgets = w.budgets()
-    lens = list(w.prefill)
+    lens, live = list(w.prefill), list(w.prefill)
     out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
     sp = w.spec()
     L0_dev = torch.tensor(w.prefill, dtype=torch.int32, device="cuda")
@@ -219,7 +231,7 @@ def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1)
                                                       torch.cuda.current_stream().cuda_stream) == 0
         ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, to_device(qs[t - 1], w), kn[0], vn[0], out, ws,
                      ws.numel())
-        lens = [min(L + 1, B) if L + 1 > B else L + 1 for L, B in zip(lens, budgets)]
+        lens, live = step_lengths(lens, live, budgets, max_holes)
         torch.cuda.synchronize()
         refresh = O.is_refresh(t, w.refresh_period, w.score_free)
         rep = StepReport(t=t, refresh=refresh)
@@ -238,10 +250,14 @@ def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1)
                 rep.out_err = max(rep.out_err, float(np.max(np.abs(out_b[l] - o_))))
                 if refresh:
                     st["m"] = O.ema_update(st["m"], O.pooled_score(a_, O.GRAN_SEQ, w.kv_heads)[0], op.alpha)
-            n = int(len_h[b])
+            assert len_h[b] == lens[b]
+            ls = live_slots(c.pos[b, :int(len_h[b])].cpu().numpy(), int(len_h[b]))
+            n = len(ls)
             assert n == min(st["pos"].shape[0], budgets[b])
-            gpos = c.pos[b, :n].cpu().numpy().astype(np.int64)
-            gm = c.ema[b, :n].cpu().numpy()
+            gpos = c.pos[b, :int(len_h[b])].cpu().numpy().astype(np.int64)[ls]
+            gm = c.ema[b, :int(len_h[b])].cpu().numpy()[ls]
+            if compact_mode in STABLE_MODES:
+                assert np.all(np.diff(gpos) > 0)
             slot_of = {int(pp): i for i, pp in enumerate(st["pos"])}
             oslots = np.array([slot_of[int(pp)] for pp in gpos])
             kept = np.zeros(st["pos"].shape[0], bool)
@@ -255,8 +271,8 @@ def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1)
             for l in check_layers:
                 lk, lv = w.kv_rows(b, l % w.layers, gpos, u)
                 for g in range(w.kv_heads):
-                    gk = c.gather(c.k, b, l % w.layers, g, n).float().cpu().numpy()
-                    gv = c.gather(c.v, b, l % w.layers, g, n).float().cpu().numpy()
+                    gk = c.gather(c.k, b, l % w.layers, g, int(len_h[b])).float().cpu().numpy()[ls]
+                    gv = c.gather(c.v, b, l % w.layers, g, int(len_h[b])).float().cpu().numpy()[ls]
                     rep.kv_err = max(rep.kv_err, float(np.max(np.abs(gk - lk[g]))), float(np.max(np.abs(gv - lv[g]))))
         reports.append(rep)
     assert ikv.ikv_device_status() == 0

@@ -97,9 +97,40 @@ def test_step_rejects_bad_schedule_and_workspace(lib):
                           16, 1 << 40, None) == lib.IKV_ERR_SHAPE
 
 
+def test_deferred_compaction_arguments(lib):
+    shp, cch = _shape(lib), _cache(lib)
+    p = lib.ikv_params()
+    p.alpha, p.refresh_period, p.budget, p.max_holes = 0.9, 1, 16, -1
+    assert lib.raw_status("ikv_step", ctypes.byref(shp), ctypes.byref(p), ctypes.byref(cch), 16, 1, 16, 16, 16, 16,
+                          16, 1 << 40, None) == lib.IKV_ERR_ARG
+    nopos = _cache(lib, pos=0, dead_slots=1)
+    n = lib.SZ(0)
+    assert lib.raw_status("ikv_attend_workspace_size", ctypes.byref(shp), ctypes.byref(nopos),
+                          ctypes.byref(n)) == lib.IKV_ERR_ARG
+
+
+def test_step_lengths_mirror():
+    """Host bookkeeping of len (dead slots included) and live slots across steps."""
+    from paper_2609_03515_gb300 import step_lengths
+    # compact every step: len = live = min(L + 1, B)
+    assert step_lengths([100, 10], [100, 10], [50, 20]) == ([50, 11], [50, 11])
+    # deferred: one eviction per step adds a dead slot until more than max_holes would be dead
+    lens, live = [50], [50]
+    seen = []
+    for _ in range(7):
+        lens, live = step_lengths(lens, live, [50], max_holes=3)
+        seen.append(lens[0])
+        assert live == [50]
+    assert seen == [51, 52, 53, 50, 51, 52, 53]
+    # the first step evicts far more than max_holes: compacted at once
+    assert step_lengths([1000], [1000], [100], max_holes=8) == ([100], [100])
+    # below the budget nothing is evicted or marked
+    assert step_lengths([10], [10], [100], max_holes=8) == ([11], [11])
+
+
 def test_other_entry_points_reject_nulls(lib):
-    assert lib.raw_status("ikv_select_budget", 2, 8, None, 16, 1, 16, 16, 16, None) == lib.IKV_ERR_ARG
-    assert lib.raw_status("ikv_select_budget", -1, 8, 16, 16, 1, 16, 16, 16, None) == lib.IKV_ERR_SHAPE
+    assert lib.raw_status("ikv_select_budget", 2, 8, None, 16, 1, 16, None, 16, 16, None) == lib.IKV_ERR_ARG
+    assert lib.raw_status("ikv_select_budget", -1, 8, 16, 16, 1, 16, None, 16, 16, None) == lib.IKV_ERR_SHAPE
     assert lib.raw_status("ikv_ema_update", 2, 8, 16, None, 16, 1, ctypes.c_float(0.5), None) == lib.IKV_ERR_ARG
     assert lib.raw_status("ikv_ema_update", 2, 8, 16, 16, 16, 1, ctypes.c_float(-0.5), None) == lib.IKV_ERR_ARG
     shp, cch = _shape(lib), _cache(lib)

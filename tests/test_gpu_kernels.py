@@ -150,6 +150,51 @@ def test_decode_attend_score_with_start_offset(ps, starts, lens):
         assert torch.all(score[b, L:] == -7.0)
 
 
+@pytest.mark.parametrize("ps", [64, 48])   # tensor-core kernel, CUDA-core kernel
+def test_decode_attend_score_skips_dead_slots(ps):
+    """Dead slots (pos < 0) leave the softmax: the output and scores are the oracle's over
+    the live slots, dead slots score 0.  Sequence 0 has every chunk of its first 4000 slots
+    dead, sequence 1 keeps a single live slot, sequence 2 scattered holes."""
+    lens = [6000, 900, 3000]
+    w = gen.Workload("a", 3, 2, 32, 8, 128, lens, 1, dtype=gen.BF16, seed=23, page_size=ps)
+    u = w.u_table()
+    c = make_cache(w, page_perm_seed=4)
+    fill_device(c, w, torch.from_numpy(u).cuda())
+    rng = np.random.default_rng(15)
+    pos = c.pos.cpu().numpy()
+    pos[0, :4000] = -1
+    pos[1, :900] = -1
+    pos[1, 457] = 457
+    pos[2, :3000][rng.random(3000) < 0.2] = -1
+    c.pos.copy_(torch.from_numpy(pos).cuda())
+    layer = 1
+    q_h = w.queries(1, 2, u)[0, layer]
+    q = to_device(q_h, w)
+    out = torch.empty((3, 32, 128), dtype=q.dtype, device="cuda")
+    score = torch.full((c.rows, c.cap), -7.0, device="cuda")
+    ema0 = torch.from_numpy(rng.random((c.rows, c.cap)).astype(np.float32)).cuda()
+    ema = ema0.clone()
+    cch = c.cache(max(lens), dead_slots=True)
+    ws = torch.empty(ikv.ikv_attend_workspace_size(c.shape(), cch), dtype=torch.uint8, device="cuda")
+    alpha = 0.75
+    ikv.ikv_decode_attend_score(c.shape(), cch, layer, q, out, score, ema, alpha, ws, ws.numel())
+    torch.cuda.synchronize()
+    assert ikv.ikv_device_status() == 0
+    q64 = as_f64(q_h, w)
+    for b, L in enumerate(lens):
+        live = np.nonzero(pos[b, :L] >= 0)[0]
+        k, v = w.kv_rows(b, layer, live, u)
+        a_, o = O.last_query_attention(q64[b], [x.astype(np.float64) for x in k], [x.astype(np.float64) for x in v])
+        assert np.max(np.abs(out[b].float().cpu().numpy() - o)) < 2e-2
+        sc = O.pooled_score(a_, O.GRAN_SEQ, 8)[0]
+        got = score[b, :L].cpu().numpy()
+        assert np.max(np.abs(got[live] - sc)) < 2e-5
+        dead = pos[b, :L] < 0
+        assert np.all(got[dead] == 0.0)
+        e0 = ema0[b, :L].cpu().numpy()
+        assert np.array_equal(ema[b, :L].cpu().numpy()[dead], (np.float32(alpha) * e0[dead]).astype(np.float32))
+
+
 def test_decode_attend_without_score_leaves_state():
     w = gen.Workload("a", 2, 1, 32, 8, 128, [900, 50], 1, dtype=gen.BF16, seed=2)
     u = w.u_table()
@@ -185,12 +230,13 @@ def test_ema_update_matches_eq4():
 
 
 # ------------------------------------------------------------------ selection
-def _select_gpu(util: np.ndarray, lens, budgets, rps=1):
+def _select_gpu(util: np.ndarray, lens, budgets, rps=1, pos=None):
     rows, cap = util.shape
     keep = torch.full((rows, cap), -1, dtype=torch.int32, device="cuda")
     keep_len = torch.full((rows,), -1, dtype=torch.int32, device="cuda")
+    pos_d = None if pos is None else torch.from_numpy(np.ascontiguousarray(pos, dtype=np.int32)).cuda()
     ikv.ikv_select_budget(rows, cap, torch.from_numpy(util).cuda(), torch.tensor(lens, dtype=torch.int32).cuda(), rps,
-                          torch.tensor(budgets, dtype=torch.int32).cuda(), keep, keep_len)
+                          torch.tensor(budgets, dtype=torch.int32).cuda(), pos_d, keep, keep_len)
     torch.cuda.synchronize()
     return keep.cpu().numpy(), keep_len.cpu().numpy()
 
@@ -227,6 +273,33 @@ def test_select_ties_and_special_values():
     _check_select(np.full((2, 3000), 0.125, np.float32), [3000, 2999], [100, 2998])
 
 
+def test_select_skips_dead_slots():
+    """Dead slots (pos < 0, deferred compaction) are never kept and not counted: the kept
+    set is the oracle's selection over the live slots, mapped back to their slots."""
+    rng = np.random.default_rng(12)
+    cap = 9000
+    pool = np.array([0.0, 0.25, 0.5, 1.0, -np.inf, np.nan, 1e-30], np.float32)
+    lens = [8000, 8000, 8000, 3278, 3278, 300, 5, 4097]
+    dead_frac = [0.01, 0.3, 0.0, 0.02, 0.5, 0.9, 0.4, 0.25]
+    rows = len(lens)
+    util = (rng.random((rows, cap)) ** 4).astype(np.float32)
+    util[1] = pool[rng.integers(0, len(pool), cap)]            # ties and special values among live slots
+    pos = np.tile(np.arange(cap, dtype=np.int32), (rows, 1))
+    n_live = []
+    for r in range(rows):
+        dead = rng.random(lens[r]) < dead_frac[r]
+        pos[r, :lens[r]][dead] = -1
+        n_live.append(int((~dead).sum()))
+    # budgets: more than the live count, exactly one too many, and the general case
+    budgets = [n_live[0] - 1, 1000, n_live[2] - 1, 3277, n_live[4] + 5, 10, n_live[6] - 1, 100]
+    keep, keep_len = _select_gpu(util, lens, budgets, 1, pos)
+    for r in range(rows):
+        live = np.nonzero(pos[r, :lens[r]] >= 0)[0]
+        want = live[O.select_keep(util[r, live].astype(np.float64), budgets[r])]
+        assert keep_len[r] == len(want), (r, keep_len[r], len(want))
+        assert np.array_equal(keep[r, :len(want)], np.sort(want)), r
+
+
 def test_select_scale_invariance_on_gpu():
     """Corollary 2: uniform positive scaling does not change the kept set."""
     rng = np.random.default_rng(10)
@@ -260,7 +333,7 @@ def test_compact_matches_oracle_eviction(mode, gran):
     c.budget.copy_(torch.tensor(budgets, dtype=torch.int32).cuda())
     keep = torch.empty((c.rows, c.cap), dtype=torch.int32, device="cuda")
     keep_len = torch.empty((c.rows,), dtype=torch.int32, device="cuda")
-    ikv.ikv_select_budget(c.rows, c.cap, c.ema, c.len, c.rows_per_seq, c.budget, keep, keep_len)
+    ikv.ikv_select_budget(c.rows, c.cap, c.ema, c.len, c.rows_per_seq, c.budget, None, keep, keep_len)
     cch = c.cache(3278)
     nws = ikv.ikv_compact_workspace_size(c.shape(), cch, mode)
     ws = torch.empty(max(nws, 1), dtype=torch.uint8, device="cuda")
@@ -326,6 +399,33 @@ def test_append_token(init_mean):
                 assert np.array_equal(c.gather(c.v, b, l, g, L + 1)[L].cpu().numpy(), vn[l, b, g])
 
 
+def test_append_mean_skips_dead_slots():
+    """With dead slots the new token's utility is the mean over the live slots only."""
+    w = gen.Workload("p", 2, 2, 8, 2, 64, [300, 40], 1, dtype=gen.F32, seed=42, page_size=64)
+    u = w.u_table()
+    c = make_cache(w, ikv.IKV_GRAN_KVHEAD)
+    fill_device(c, w, torch.from_numpy(u).cuda())
+    rng = np.random.default_rng(14)
+    m0 = rng.random((c.rows, c.cap)).astype(np.float32)
+    pos = c.pos.cpu().numpy()
+    for r in range(c.rows):
+        pos[r, :w.prefill[r // w.kv_heads]][rng.random(w.prefill[r // w.kv_heads]) < 0.3] = -1
+    c.pos.copy_(torch.from_numpy(pos).cuda())
+    c.ema.copy_(torch.from_numpy(m0).cuda())
+    kn, vn = w.new_tokens(1, u)
+    ws = torch.empty(4096, dtype=torch.uint8, device="cuda")
+    ikv.ikv_append_token(c.shape(), c.cache(300, dead_slots=True), to_device(kn, w), to_device(vn, w), c.ema, 1, ws,
+                         4096)
+    torch.cuda.synchronize()
+    assert c.len.cpu().tolist() == [301, 41]
+    for r in range(c.rows):
+        L = w.prefill[r // w.kv_heads]
+        live = pos[r, :L] >= 0
+        want = O.new_token_state(m0[r, :L][live].astype(np.float64), refresh=False, refresh_init="zero")
+        assert abs(float(c.ema[r, L]) - want) < 1e-6
+        assert int(c.pos[r, L]) == L
+
+
 def test_compact_short_side_moves_the_prefix():
     """Shorter-side stable compaction: an eviction near the front moves the prefix right
     and advances start; one near the back moves the suffix left; order is kept."""
@@ -340,7 +440,7 @@ def test_compact_short_side_moves_the_prefix():
     c.budget.fill_(3277)
     keep = torch.empty((2, c.cap), dtype=torch.int32, device="cuda")
     keep_len = torch.empty((2,), dtype=torch.int32, device="cuda")
-    ikv.ikv_select_budget(2, c.cap, c.ema, c.len, 1, c.budget, keep, keep_len)
+    ikv.ikv_select_budget(2, c.cap, c.ema, c.len, 1, c.budget, None, keep, keep_len)
     cch = c.cache(3278)
     nws = ikv.ikv_compact_workspace_size(c.shape(), cch, ikv.IKV_COMPACT_STABLE_SHORT)
     ws = torch.empty(nws, dtype=torch.uint8, device="cuda")
@@ -380,7 +480,7 @@ def test_compact_short_side_relocates_and_skips_in_place():
     c.pos.copy_(torch.from_numpy(pos).cuda())
     keep = torch.empty((3, c.cap), dtype=torch.int32, device="cuda")
     keep_len = torch.empty((3,), dtype=torch.int32, device="cuda")
-    ikv.ikv_select_budget(3, c.cap, c.ema, c.len, 1, c.budget, keep, keep_len)
+    ikv.ikv_select_budget(3, c.cap, c.ema, c.len, 1, c.budget, None, keep, keep_len)
     cch = c.cache(max(L))
     nws = ikv.ikv_compact_workspace_size(c.shape(), cch, ikv.IKV_COMPACT_STABLE_SHORT)
     ws = torch.empty(nws, dtype=torch.uint8, device="cuda")

@@ -99,3 +99,18 @@ def test_budget_edges():
 def test_alpha_zero_and_one():
     _assert(run_lockstep(small_llama(alpha=0.0, steps=3, layers=2)), 2e-2)
     _assert(run_lockstep(small_llama(alpha=1.0, steps=3, layers=2)), 2e-2)
+
+
+def test_deferred_compaction_trajectories():
+    """max_holes > 0: evicted slots are only marked dead until the sequence holds more
+    than max_holes of them, then the cache is compacted.  The kept set, its order, the
+    utilities and the outputs must match the oracle (which compacts every step) on every
+    step, across compactions and under every schedule and compaction mode."""
+    _assert(run_lockstep(gen.config(0), max_holes=3), 1e-4, strict_fraction=1.0)
+    _assert(run_lockstep(small_llama(steps=12), max_holes=4), 2e-2)
+    _assert(run_lockstep(small_llama(steps=12, refresh_period=3), compact_mode=ikv.IKV_COMPACT_STABLE_SHORT,
+                         max_holes=5), 2e-2)
+    _assert(run_lockstep(small_llama(steps=10, score_free=True, page_size=16), max_holes=3), 2e-2)
+    _assert(run_lockstep(small_llama(steps=8), gran=ikv.IKV_GRAN_KVHEAD, max_holes=3), 2e-2)
+    _assert(run_lockstep(small_llama(steps=8), compact_mode=ikv.IKV_COMPACT_HOLEFILL, max_holes=3), 2e-2)
+    _assert(run_lockstep(small_llama(steps=8, refresh_period=2), refresh_init=ikv.IKV_INIT_MEAN, max_holes=64), 2e-2)
