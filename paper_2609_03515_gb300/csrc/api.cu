@@ -362,7 +362,9 @@ ikv_status ikv_select_budget(int32_t rows, int32_t cap, const float *util, const
     if (rows < 0 || cap < 0 || rows_per_seq_ <= 0) return fail(IKV_ERR_SHAPE, "rows/cap/rows_per_seq out of range");
     if (rows > 0 && (!util || !len || !budget || !keep || !keep_len))
         return fail(IKV_ERR_ARG, "util/len/budget/keep/keep_len is NULL");
-    IKV_TRY_CUDA(launch_select(rows, cap, util, len, rows_per_seq_, budget, pos, keep, keep_len, stream),
+    // max_holes 0: the kernel never writes pos here
+    IKV_TRY_CUDA(launch_select(rows, cap, util, len, rows_per_seq_, budget, const_cast<int32_t *>(pos), keep,
+                               keep_len, DeferArgs{0, cap, nullptr}, stream),
                  "select launch");
     return IKV_OK;
 }
@@ -544,7 +546,7 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     const int32_t R = shape->batch * rows_per_seq(shape);
     IKV_TRY_CUDA(launch_select(R, cap, ema, cache->len, rows_per_seq(shape), p->budget,
                                cache->dead_slots ? cache->pos : nullptr, at<int32_t>(ws, w.keep),
-                               at<int32_t>(ws, w.keep_len), stream),
+                               at<int32_t>(ws, w.keep_len), DeferArgs{p->max_holes, cap, cache->start}, stream),
                  "select launch");
     if (tm && (e = record(tm->select_end, stream))) return e;
     if ((e = compact_impl(shape, cache, at<int32_t>(ws, w.keep), at<int32_t>(ws, w.keep_len), ema, p->compact_mode,

@@ -94,6 +94,7 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
     const int b = blockIdx.y, x = blockIdx.x;
     const int kvh = a.pv.kv_heads;
     const int nkv = a.layers * kvh;
+    if (a.keep_len[b * a.rows_per_seq] < 0) return;  // selection marked the victim dead: nothing to do
     const int L = a.len[b];
     const int S = a.start ? a.start[b] : 0;
     if (defer_of(a, b, L, S)) {  // nothing moves; len, start and the arrival counter stay as they are
@@ -250,6 +251,7 @@ __global__ void __launch_bounds__(kPlanThreads) holefill_plan_kernel(const Compa
     __shared__ int below_s;
     const int r = blockIdx.x;
     const int n = a.keep_len[r];
+    if (n < 0) return;  // selection marked the victim dead: nothing to do
     const int32_t *kp = a.keep + (int64_t)r * a.cap;
     if (defer_of(a, r / a.rows_per_seq, a.len[r / a.rows_per_seq], a.pv.start_of(r / a.rows_per_seq))) {
         // decided here, before len changes
@@ -286,6 +288,7 @@ __global__ void __launch_bounds__(kCompThreads) holefill_move_kernel(const Compa
     const int b = blockIdx.y, x = blockIdx.x;
     const int kvh = a.pv.kv_heads;
     const int nkv = a.layers * kvh;
+    if (a.keep_len[b * a.rows_per_seq] < 0) return;  // selection marked the victim dead: nothing to do
     if (x < nkv) {
         const int l = x / kvh, g = x % kvh;
         const int r = b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g);

@@ -93,8 +93,17 @@ cudaError_t launch_combine(const CombineArgs &a, int dtype, cudaStream_t st);
 cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, int sms, cudaStream_t st);
 cudaError_t launch_ema_update(int32_t rows, int32_t cap, float *ema, const float *score, const int32_t *len,
                               int32_t rows_per_seq, float alpha, int32_t max_len, cudaStream_t st);
+// Deferred compaction inside selection: when a row has exactly one slot too many and
+// the sequence may defer (len - budget <= max_holes and start + len < cap), select
+// marks the victim dead itself and writes keep_len = -1 - budget, which tells the
+// compaction kernels that nothing moves.  max_holes = 0 disables it.
+struct DeferArgs {
+    int32_t max_holes;
+    int32_t cap;
+    const int32_t *start;       // [batch] or null
+};
 cudaError_t launch_select(int32_t rows, int32_t cap, const float *util, const int32_t *len, int32_t rows_per_seq,
-                          const int32_t *budget, const int32_t *pos, int32_t *keep, int32_t *keep_len,
+                          const int32_t *budget, int32_t *pos, int32_t *keep, int32_t *keep_len, const DeferArgs &df,
                           cudaStream_t st);
 
 struct CompactArgs {

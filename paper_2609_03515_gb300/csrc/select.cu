@@ -57,9 +57,8 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t *warp_t
 
 __global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const float *__restrict__ util,
                                                               const int32_t *__restrict__ len, int32_t rps,
-                                                              const int32_t *__restrict__ budget,
-                                                              const int32_t *__restrict__ pos, int32_t *keep,
-                                                              int32_t *keep_len) {
+                                                              const int32_t *__restrict__ budget, int32_t *pos,
+                                                              int32_t *keep, int32_t *keep_len, DeferArgs df) {
     __shared__ uint32_t hist[256];
     __shared__ uint32_t warp_tot[32];
     __shared__ unsigned long long s_min[32];
@@ -71,7 +70,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const 
     int B = budget[r / rps];
     if (B < 0) B = 0;
     const float *u = util + (int64_t)r * cap;
-    const int32_t *pr = pos ? pos + (int64_t)r * cap : nullptr;
+    int32_t *pr = pos ? pos + (int64_t)r * cap : nullptr;
     int32_t *kp = keep + (int64_t)r * cap;
     auto live = [&](int i) { return !pr || pr[i] >= 0; };
     auto key_at = [&](int i) { return live(i) ? ord_key(u[i]) : kDeadKey; };
@@ -88,16 +87,37 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const 
         }
     };
 
-    int n_live = L;
-    if (pr) {
-        if (tid == 0) s_live = 0u;
-        __syncthreads();
-        uint32_t c = 0u;
-        for (int i = tid; i < L; i += kSelThreads) c += pr[i] >= 0;
-        if (c) atomicAdd(&s_live, c);
-        __syncthreads();
-        n_live = (int)s_live;
+    // one pass: the live count and the lowest (key, highest slot) among the live slots,
+    // which is the victim whenever exactly one slot must go
+    if (tid == 0) s_live = 0u;
+    __syncthreads();
+    uint32_t c = 0u;
+    unsigned long long best = ~0ull;
+    for (int i = tid; i < L; i += kSelThreads) {
+        if (!live(i)) continue;
+        ++c;
+        const unsigned long long v = ((unsigned long long)ord_key(u[i]) << 32) | (uint32_t)(~(uint32_t)i);
+        best = v < best ? v : best;
     }
+    if (pr && c) atomicAdd(&s_live, c);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const unsigned long long y = __shfl_xor_sync(0xffffffffu, best, o);
+        best = y < best ? y : best;
+    }
+    if (lane == 0) s_min[warp] = best;
+    __syncthreads();
+    if (warp == 0) {
+        best = s_min[lane];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const unsigned long long y = __shfl_xor_sync(0xffffffffu, best, o);
+            best = y < best ? y : best;
+        }
+        if (lane == 0) s_min[0] = best;
+    }
+    __syncthreads();
+    const int n_live = pr ? (int)s_live : L;
 
     if (n_live <= B) {
         if (n_live == L) {
@@ -114,31 +134,17 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const 
     }
 
     if (n_live == B + 1) {
-        // evict exactly one: minimum of (key, ~slot) over the live slots
-        unsigned long long best = ~0ull;
-        for (int i = tid; i < L; i += kSelThreads) {
-            if (!live(i)) continue;
-            const unsigned long long v = ((unsigned long long)ord_key(u[i]) << 32) | (uint32_t)(~(uint32_t)i);
-            best = v < best ? v : best;
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const unsigned long long y = __shfl_xor_sync(0xffffffffu, best, o);
-            best = y < best ? y : best;
-        }
-        if (lane == 0) s_min[warp] = best;
-        __syncthreads();
-        if (warp == 0) {
-            best = s_min[lane];
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                const unsigned long long y = __shfl_xor_sync(0xffffffffu, best, o);
-                best = y < best ? y : best;
-            }
-            if (lane == 0) s_min[0] = best;
-        }
-        __syncthreads();
         const int ev = (int)(~(uint32_t)(s_min[0] & 0xFFFFFFFFull));
+        const int b = r / rps;
+        if (pr && df.max_holes > 0 && L - B <= df.max_holes && (df.start ? df.start[b] : 0) + L < df.cap) {
+            // deferred compaction (the rule the compaction kernels apply): the victim is
+            // only marked dead, and keep_len < 0 tells compaction that nothing moves
+            if (tid == 0) {
+                pr[ev] = -1;
+                keep_len[r] = -1 - B;
+            }
+            return;
+        }
         if (n_live == L) {
             for (int j = tid; j < B; j += kSelThreads) kp[j] = j < ev ? j : j + 1;
         } else {
@@ -222,10 +228,10 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const 
 }  // namespace
 
 cudaError_t launch_select(int32_t rows, int32_t cap, const float *util, const int32_t *len, int32_t rows_per_seq,
-                          const int32_t *budget, const int32_t *pos, int32_t *keep, int32_t *keep_len,
+                          const int32_t *budget, int32_t *pos, int32_t *keep, int32_t *keep_len, const DeferArgs &df,
                           cudaStream_t st) {
     if (rows <= 0) return cudaSuccess;
-    select_kernel<<<rows, kSelThreads, 0, st>>>(cap, util, len, rows_per_seq, budget, pos, keep, keep_len);
+    select_kernel<<<rows, kSelThreads, 0, st>>>(cap, util, len, rows_per_seq, budget, pos, keep, keep_len, df);
     note_launch();
     return cudaGetLastError();
 }

@@ -24,25 +24,42 @@ def _check(reps):
         assert r.kv_err == 0.0, r
 
 
+# The benchmark's configuration: shorter-side stable compaction, deferred while a
+# sequence holds at most 128 dead slots.
+SHORT, BENCH_HOLES = ikv.IKV_COMPACT_STABLE_SHORT, 128
+
+
 @pytest.mark.timeout(1200)
 def test_config1_llama_b1_32k_full_refresh():
-    # the benchmark's configuration: shorter-side stable compaction
-    _check(run_fullsize_sampled(gen.config(1), seqs=[0], steps=4, compact_mode=ikv.IKV_COMPACT_STABLE_SHORT))
+    _check(run_fullsize_sampled(gen.config(1), seqs=[0], steps=4, compact_mode=SHORT, max_holes=BENCH_HOLES))
+
+
+@pytest.mark.timeout(1200)
+def test_config1_deferred_compaction_crossing():
+    # max_holes 3: steps 2-4 mark their evictions dead, step 5 compacts them away, 6-7 mark again
+    _check(run_fullsize_sampled(gen.config(1), seqs=[0], steps=7, compact_mode=SHORT, max_holes=3))
 
 
 @pytest.mark.timeout(1200)
 def test_config2_llama_b16_ragged_lazy4():
     # steps 1 and 5 refresh, 2-4 carry the state (Eq. 6); two of the sixteen sequences followed
-    _check(run_fullsize_sampled(gen.config(2), seqs=[0, 11], steps=5))
+    _check(run_fullsize_sampled(gen.config(2), seqs=[0, 11], steps=5, compact_mode=SHORT, max_holes=BENCH_HOLES))
 
 
 @pytest.mark.timeout(1200)
 def test_config3_llama_b8_64k_score_free():
-    _check(run_fullsize_sampled(gen.config(3), seqs=[5], steps=3))
+    _check(run_fullsize_sampled(gen.config(3), seqs=[5], steps=3, compact_mode=SHORT, max_holes=BENCH_HOLES))
 
 
 @pytest.mark.timeout(1200)
 def test_config4_qwen_b32_16k_sweep_point():
     # one point of the sweep: budget 25%, alpha 0.5, Lazy refresh period 2
     w = gen.config(4).with_(budget_frac=0.25, alpha=0.5, refresh_period=2)
-    _check(run_fullsize_sampled(w, seqs=[31], steps=3))
+    _check(run_fullsize_sampled(w, seqs=[31], steps=3, compact_mode=SHORT, max_holes=BENCH_HOLES))
+
+
+@pytest.mark.timeout(1200)
+def test_config4_every_step_compaction():
+    # the same workload with compaction on every eviction and the always-left stable shift
+    w = gen.config(4).with_(budget_frac=0.1)
+    _check(run_fullsize_sampled(w, seqs=[0], steps=3, compact_mode=ikv.IKV_COMPACT_STABLE))
