@@ -195,6 +195,73 @@ def test_decode_attend_score_skips_dead_slots(ps):
         assert np.array_equal(ema[b, :L].cpu().numpy()[dead], (np.float32(alpha) * e0[dead]).astype(np.float32))
 
 
+def _attend_case(w, c, layer, kv=None, u=None, alpha=0.5):
+    """Run one attention layer through the ABI and compare it with the oracle (GRAN_SEQ)."""
+    u = w.u_table() if u is None else u
+    q_h = w.queries(1, 2, u)[0, layer]
+    q = to_device(q_h, w)
+    out = torch.empty((w.batch, w.q_heads, w.head_dim), dtype=q.dtype, device="cuda")
+    score = torch.full((c.rows, c.cap), -7.0, device="cuda")
+    ema = torch.zeros((c.rows, c.cap), device="cuda")
+    cch = c.cache(max(w.prefill))
+    ws = torch.empty(ikv.ikv_attend_workspace_size(c.shape(), cch), dtype=torch.uint8, device="cuda")
+    ikv.ikv_decode_attend_score(c.shape(), cch, layer, q, out, score, ema, alpha, ws, ws.numel())
+    torch.cuda.synchronize()
+    assert ikv.ikv_device_status() == 0
+    q64 = as_f64(q_h, w)
+    for b, L in enumerate(w.prefill):
+        k, v = kv[b] if kv is not None else w.kv_block(b, layer, 0, L, u)
+        a_, o = O.last_query_attention(q64[b], [x.astype(np.float64) for x in k], [x.astype(np.float64) for x in v])
+        assert np.max(np.abs(out[b].float().cpu().numpy() - o)) < 2e-2, b
+        sc = O.pooled_score(a_, O.GRAN_SEQ, w.kv_heads)[0]
+        assert np.max(np.abs(score[b, :L].cpu().numpy() - sc)) < 2e-5, b
+
+
+def test_attend_dominant_late_logits():
+    """Keys deep inside long units are set along their head's query, so their logits
+    exceed every other by ~80 (log2 units): one slot takes nearly all of the softmax,
+    in a late chunk of the split, far from the first tiles."""
+    w = gen.Workload("r", 1, 2, 32, 8, 128, [40000], 1, dtype=gen.BF16, seed=24, page_size=64)
+    u = w.u_table()
+    c = make_cache(w, page_perm_seed=6)
+    fill_device(c, w, torch.from_numpy(u).cuda())
+    layer = 1
+    q_h = w.queries(1, 2, u)[0, layer]                      # [batch][H][d] bf16 bits
+    qf = gen.bf16_to_f32(q_h)
+    k, v = w.kv_block(0, layer, 0, 40000, u)
+    for slot, g in ((9000, 0), (21000, 3), (33333, 5), (39990, 7)):
+        k[g][slot] = gen.bf16_to_f32(gen.f32_to_bf16_bits((5.0 * qf[0, g * 4]).astype(np.float32)))
+    for g in range(8):
+        c.scatter(c.k, 0, layer, g, torch.from_numpy(k[g]).cuda())
+    _attend_case(w, c, layer, kv=[(k, v)], u=u)
+
+
+def test_attend_many_tiny_units():
+    """Units of 0..3 slots next to longer ones: one-tile chunks, mostly-masked tiles and an
+    empty sequence (zero output)."""
+    lens = [1, 2, 3, 0, 130, 1, 64]
+    w = gen.Workload("t", len(lens), 3, 16, 8, 128, lens, 1, dtype=gen.BF16, seed=26, page_size=16)
+    u = w.u_table()
+    c = make_cache(w, page_perm_seed=2)
+    fill_device(c, w, torch.from_numpy(u).cuda())
+    q_h = w.queries(1, 2, u)[0, 2]
+    q = to_device(q_h, w)
+    out = torch.full((w.batch, 16, 128), 7.0, dtype=q.dtype, device="cuda")
+    cch = c.cache(max(lens))
+    ws = torch.empty(ikv.ikv_attend_workspace_size(c.shape(), cch), dtype=torch.uint8, device="cuda")
+    ikv.ikv_decode_attend_score(c.shape(), cch, 2, q, out, None, None, 0.5, ws, ws.numel())
+    torch.cuda.synchronize()
+    assert ikv.ikv_device_status() == 0
+    q64 = as_f64(q_h, w)
+    for b, L in enumerate(lens):
+        if L == 0:
+            assert torch.all(out[b] == 0)
+            continue
+        k, v = w.kv_block(b, 2, 0, L, u)
+        _, o = O.last_query_attention(q64[b], [x.astype(np.float64) for x in k], [x.astype(np.float64) for x in v])
+        assert np.max(np.abs(out[b].float().cpu().numpy() - o)) < 2e-2, b
+
+
 def test_decode_attend_without_score_leaves_state():
     w = gen.Workload("a", 2, 1, 32, 8, 128, [900, 50], 1, dtype=gen.BF16, seed=2)
     u = w.u_table()
