@@ -107,6 +107,28 @@ def ema_update(m: np.ndarray, s: np.ndarray, alpha: float) -> np.ndarray:
     return alpha * m + (1.0 - alpha) * s
 
 
+def cumulative_update(m: np.ndarray, s: np.ndarray) -> np.ndarray:
+    """Eq. 3 (cumulative, H2O-style): m <- m + s."""
+    return m + s
+
+
+def single_step_update(m: np.ndarray, s: np.ndarray) -> np.ndarray:
+    """Eq. 2 (single-step): m <- s."""
+    return np.array(s, dtype=np.float64, copy=True)
+
+
+def aggregate(m: np.ndarray, s: np.ndarray, p: "Params") -> np.ndarray:
+    """One layer's update of the running utility under the configured rule (Eq. 2-4),
+    applied after every eligible layer in the Appendix's layer-sequential order."""
+    if p.aggregation == "ema":
+        return ema_update(m, s, p.alpha)
+    if p.aggregation == "cumulative":
+        return cumulative_update(m, s)
+    if p.aggregation == "single":
+        return single_step_update(m, s)
+    raise ValueError(p.aggregation)
+
+
 def layer_sequential_ema(m_prev: np.ndarray, layer_scores: Sequence[np.ndarray], alpha: float) -> np.ndarray:
     """Appendix "Layer scoring": m_{t,0} = m_{t-1,K}; m_{t,l} = alpha m_{t,l-1} + (1-alpha) s_{t,l}."""
     m = np.array(m_prev, dtype=np.float64, copy=True)
@@ -167,6 +189,7 @@ class Params:
     granularity: int = GRAN_SEQ
     layer_mask: Optional[List[bool]] = None   # eligible layers (R8)
     refresh_init: str = "zero"         # R3
+    aggregation: str = "ema"           # Eq. 4 (InertiaKV); "cumulative" (Eq. 3) or "single" (Eq. 2)
 
 
 @dataclass
@@ -244,7 +267,7 @@ def attend_and_score(st: SeqState, q_t: np.ndarray, refresh: bool, p: Params) ->
         eligible = p.layer_mask is None or p.layer_mask[l]
         if refresh and eligible:
             s = pooled_score(a, st.granularity, st.kv_heads)
-            st.m = ema_update(st.m, s, p.alpha)
+            st.m = aggregate(st.m, s, p)
     return np.stack(outs)
 
 

@@ -247,6 +247,45 @@ def test_alpha_zero_keeps_only_last_eligible_layer():
         assert np.max(np.abs(st.m[0] - want)) < 1e-15
 
 
+def test_cumulative_constant_stream_through_decode_loop():
+    """Eq. 3 under the layer-sequential update: uniform attention gives s = 1/L at every
+    layer and step, so after T refresh steps the surviving prefill tokens hold K T / L
+    (no forgetting), and the new token (K / L after its own step) is the one evicted."""
+    layers, kv, H, d, L0, T = 3, 2, 4, 8, 20, 5
+    K = [[np.zeros((L0, d)) for _ in range(kv)] for _ in range(layers)]
+    V = [[np.ones((L0, d)) for _ in range(kv)] for _ in range(layers)]
+    st = O.prefill_state(K, V, budget=L0)
+    p = O.Params(aggregation="cumulative")
+    rng = np.random.default_rng(9)
+    for t in range(1, T + 1):
+        q = rng.standard_normal((layers, H, d))
+        O.decode_step(st, t, q, np.zeros((layers, kv, d)), np.ones((layers, kv, d)), p)
+        assert st.length == L0
+    assert np.array_equal(st.pos[0], np.arange(L0))
+    assert np.max(np.abs(st.m[0] - layers * T / (L0 + 1))) < 1e-13
+
+
+def test_single_step_keeps_last_layer_and_equals_alpha_zero():
+    """Eq. 2: the utility is the last eligible layer's score -- the same as EMA with
+    alpha = 0 (bit for bit) -- whatever the earlier layers or steps contributed."""
+    layers, kv, H, d, L0, zs = 3, 1, 2, 4, 8, 1.5
+    spikes = [0, 3, 5]
+    K, V, q = _spike_layers(layers, kv, H, d, L0, spikes, zs)
+    for mask, last in (([True, True, True], 2), ([True, False, False], 0)):
+        st = O.prefill_state(K, V, budget=L0 + 1)
+        st.m[:] = 7.0  # any earlier state is discarded
+        ref = _clone(st)
+        O.decode_step(st, 1, q, np.zeros((layers, kv, d)), np.zeros((layers, kv, d)),
+                      O.Params(aggregation="single", layer_mask=mask))
+        O.decode_step(ref, 1, q, np.zeros((layers, kv, d)), np.zeros((layers, kv, d)),
+                      O.Params(alpha=0.0, layer_mask=mask))
+        den = math.exp(zs) + L0
+        want = np.full(L0 + 1, 1.0 / den)
+        want[spikes[last]] = math.exp(zs) / den
+        assert np.max(np.abs(st.m[0] - want)) < 1e-15
+        assert np.array_equal(st.m, ref.m)
+
+
 # ---------------------------------------------------------------- schedule
 def test_refresh_sets():
     assert [t for t in range(1, 14) if O.is_refresh(t, 4, False)] == [1, 5, 9, 13]
