@@ -75,6 +75,9 @@ enum { IKV_F32 = 0, IKV_BF16 = 1 };
 enum { IKV_GRAN_SEQ = 0, IKV_GRAN_KVHEAD = 1 };
 enum { IKV_COMPACT_STABLE = 0, IKV_COMPACT_HOLEFILL = 1, IKV_COMPACT_STABLE_SHORT = 2 };
 enum { IKV_INIT_ZERO = 0, IKV_INIT_MEAN = 1 };
+/* Temporal aggregation of the per-layer scores (Sec. 3.1): Eq. 4 EMA (InertiaKV),
+ * Eq. 3 cumulative sum (H2O-style), Eq. 2 single-step. */
+enum { IKV_AGG_EMA = 0, IKV_AGG_CUMULATIVE = 1, IKV_AGG_SINGLE_STEP = 2 };
 
 typedef struct {
     int32_t batch, layers, q_heads, kv_heads, head_dim;
@@ -132,6 +135,10 @@ typedef struct {
                                        rows move once per ~max_holes evictions instead of every
                                        step.  Needs pos; len then counts dead slots, so the
                                        caller's max_len bound is max(budget) + max_holes. */
+    int32_t agg_mode;               /* how each eligible layer's score updates the utility, in layer
+                                       order: IKV_AGG_EMA m = alpha m + (1 - alpha) s (Eq. 4, the
+                                       method; default) | IKV_AGG_CUMULATIVE m = m + s (Eq. 3) |
+                                       IKV_AGG_SINGLE_STEP m = s (Eq. 2) */
 } ikv_params;
 
 /* Message for the last error on this thread ("" if none). */
@@ -278,7 +285,8 @@ ikv_status ikv_append_token(const ikv_shape *shape, ikv_cache *cache, const void
  *   3. attention of every layer over all len[b] slots (the new token included)
  *   4. refresh steps only: for each eligible layer in ascending order,
  *      ema = alpha * ema + (1 - alpha) * s_layer  (Eq. 1, Eq. 4, Appendix
- *      "Layer scoring"); off-refresh steps leave ema untouched (Eq. 6)
+ *      "Layer scoring"; or Eq. 3 / Eq. 2 per agg_mode); off-refresh steps leave
+ *      ema untouched (Eq. 6)
  *   5. if more than budget[b] slots are live: keep the budget[b] highest
  *      utilities and compact, or with max_holes > 0 mark the evicted slots dead
  *      until their number would exceed max_holes (Appendix "Eviction on

@@ -126,7 +126,8 @@ class DecodeCache:
 
     def params(self, alpha: float, refresh_period: int = 1, score_free: bool = False,
                compact_mode: int = ikv.IKV_COMPACT_STABLE, refresh_init: int = ikv.IKV_INIT_ZERO,
-               layer_eligible: Optional[Sequence[int]] = None, max_holes: int = 0) -> ikv.ikv_params:
+               layer_eligible: Optional[Sequence[int]] = None, max_holes: int = 0,
+               agg_mode: int = ikv.IKV_AGG_EMA) -> ikv.ikv_params:
         p = ikv.ikv_params()
         p.alpha = alpha
         p.refresh_period = refresh_period
@@ -138,6 +139,7 @@ class DecodeCache:
         p.compact_mode = compact_mode
         p.refresh_init = refresh_init
         p.max_holes = max_holes
+        p.agg_mode = agg_mode
         return p
 
 

@@ -253,7 +253,7 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
 
 ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, const int32_t *elig, int n_elig,
                      int32_t max_len, void *ws, const AttendWs &w, float alpha, float *ema, float *score,
-                     cudaStream_t st) {
+                     cudaStream_t st, int32_t agg = IKV_AGG_EMA) {
     for (int k0 = 0; k0 < n_elig; k0 += kMaxLayersPerScorePass) {
         ScoreArgs sa{};
         sa.len = c->len;
@@ -269,6 +269,7 @@ ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, c
         sa.n_elig = n_elig - k0 < kMaxLayersPerScorePass ? n_elig - k0 : kMaxLayersPerScorePass;
         for (int k = 0; k < sa.n_elig; ++k) sa.elig[k] = elig[k0 + k];
         sa.alpha = alpha;
+        sa.agg = agg;
         sa.ema = ema;
         sa.score = score;
         IKV_TRY_CUDA(launch_score_ema(sa, max_len, sm_count(), st), "score launch");
@@ -508,6 +509,8 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     if (p->refresh_init != IKV_INIT_ZERO && p->refresh_init != IKV_INIT_MEAN)
         return fail(IKV_ERR_ARG, "unknown refresh_init %d", p->refresh_init);
     if (p->max_holes < 0) return fail(IKV_ERR_ARG, "max_holes must be >= 0");
+    if (p->agg_mode != IKV_AGG_EMA && p->agg_mode != IKV_AGG_CUMULATIVE && p->agg_mode != IKV_AGG_SINGLE_STEP)
+        return fail(IKV_ERR_ARG, "unknown agg_mode %d", p->agg_mode);
     // with deferred compaction every kernel of the step treats pos < 0 as a dead slot
     ikv_cache cv = *cache;
     if (p->max_holes > 0) cv.dead_slots = 1;
@@ -540,7 +543,8 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
                         true)))
         return e;
     if (tm && (e = record(tm->combine_end, stream))) return e;
-    if (scoring && (e = run_score(shape, cache, shape->layers, elig, n_elig, L1, ws, w.at, p->alpha, ema, nullptr, stream)))
+    if (scoring && (e = run_score(shape, cache, shape->layers, elig, n_elig, L1, ws, w.at, p->alpha, ema, nullptr, stream,
+                                  p->agg_mode)))
         return e;
     if (tm && (e = record(tm->score_end, stream))) return e;
     const int32_t R = shape->batch * rows_per_seq(shape);

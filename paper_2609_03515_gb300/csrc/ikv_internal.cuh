@@ -70,6 +70,7 @@ struct ScoreArgs {
     int32_t n_elig;             // eligible local layers, in ascending order
     const int32_t *elig_dev;    // unused placeholder
     float alpha;
+    int32_t agg;                // IKV_AGG_*: how each layer's score updates ema
     float *ema;                 // [rows][cap] or null
     float *score;               // [rows][cap] or null (only meaningful with one layer)
     int32_t elig[kMaxLayersPerScorePass];

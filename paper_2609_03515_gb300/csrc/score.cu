@@ -90,7 +90,12 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_ema_kernel(const Sc
         float sc = 0.f;
         for (int k = 0; k < a.n_elig; ++k) {
             sc = sl[k][threadIdx.x];
-            m = a.alpha * m + (1.f - a.alpha) * sc;
+            if (a.agg == IKV_AGG_EMA)
+                m = a.alpha * m + (1.f - a.alpha) * sc;  // Eq. 4
+            else if (a.agg == IKV_AGG_CUMULATIVE)
+                m += sc;                                  // Eq. 3
+            else
+                m = sc;                                   // Eq. 2
         }
         if (a.ema) a.ema[at] = m;
         if (a.score) a.score[at] = sc;

@@ -20,6 +20,7 @@ IKV_GRAN_SEQ, IKV_GRAN_KVHEAD = 0, 1
 IKV_COMPACT_STABLE, IKV_COMPACT_HOLEFILL, IKV_COMPACT_STABLE_SHORT = 0, 1, 2
 IKV_INIT_ZERO, IKV_INIT_MEAN = 0, 1
 IKV_PATH_CUDA_CORE, IKV_PATH_TENSOR_CORE = 0, 1
+IKV_AGG_EMA, IKV_AGG_CUMULATIVE, IKV_AGG_SINGLE_STEP = 0, 1, 2
 
 P = ctypes.c_void_p
 I32 = ctypes.c_int32
@@ -45,7 +46,7 @@ class ikv_timing(ctypes.Structure):
 class ikv_params(ctypes.Structure):
     _fields_ = [("alpha", F32), ("refresh_period", I32), ("score_free", I32), ("budget", P),
                 ("layer_eligible", P), ("compact_mode", I32), ("refresh_init", I32),
-                ("timing", ctypes.POINTER(ikv_timing)), ("max_holes", I32)]
+                ("timing", ctypes.POINTER(ikv_timing)), ("max_holes", I32), ("agg_mode", I32)]
 
 
 class IKVError(RuntimeError):

@@ -122,7 +122,8 @@ def live_slots(pos_row: np.ndarray, n: int) -> np.ndarray:
 
 def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: int = ikv.IKV_COMPACT_STABLE,
                  steps: Optional[int] = None, kv_check_layers=(0, -1), page_perm_seed: Optional[int] = 7,
-                 refresh_init: int = ikv.IKV_INIT_ZERO, layer_eligible=None, max_holes: int = 0) -> List[StepReport]:
+                 refresh_init: int = ikv.IKV_INIT_ZERO, layer_eligible=None, max_holes: int = 0,
+                 agg_mode: int = ikv.IKV_AGG_EMA) -> List[StepReport]:
     T = w.steps if steps is None else steps
     u = w.u_table()
     c = make_cache(w, gran, page_perm_seed)
@@ -131,8 +132,11 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
     op = O.Params(alpha=w.alpha, refresh_period=w.refresh_period, score_free=w.score_free,
                   granularity=O.GRAN_SEQ if gran == ikv.IKV_GRAN_SEQ else O.GRAN_KVHEAD,
                   layer_mask=None if layer_eligible is None else [bool(x) for x in layer_eligible],
-                  refresh_init="zero" if refresh_init == ikv.IKV_INIT_ZERO else "mean")
-    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, refresh_init, layer_eligible, max_holes)
+                  refresh_init="zero" if refresh_init == ikv.IKV_INIT_ZERO else "mean",
+                  aggregation={ikv.IKV_AGG_EMA: "ema", ikv.IKV_AGG_CUMULATIVE: "cumulative",
+                               ikv.IKV_AGG_SINGLE_STEP: "single"}[agg_mode])
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, refresh_init, layer_eligible, max_holes,
+                 agg_mode)
     ws = c.step_workspace()
     qs = w.queries(1, T + 1, u)
     budgets = w.budgets()

@@ -103,6 +103,9 @@ def test_deferred_compaction_arguments(lib):
     p.alpha, p.refresh_period, p.budget, p.max_holes = 0.9, 1, 16, -1
     assert lib.raw_status("ikv_step", ctypes.byref(shp), ctypes.byref(p), ctypes.byref(cch), 16, 1, 16, 16, 16, 16,
                           16, 1 << 40, None) == lib.IKV_ERR_ARG
+    p.max_holes, p.agg_mode = 0, 3   # no such aggregation rule
+    assert lib.raw_status("ikv_step", ctypes.byref(shp), ctypes.byref(p), ctypes.byref(cch), 16, 1, 16, 16, 16, 16,
+                          16, 1 << 40, None) == lib.IKV_ERR_ARG
     nopos = _cache(lib, pos=0, dead_slots=1)
     n = lib.SZ(0)
     assert lib.raw_status("ikv_attend_workspace_size", ctypes.byref(shp), ctypes.byref(nopos),

@@ -114,3 +114,15 @@ def test_deferred_compaction_trajectories():
     _assert(run_lockstep(small_llama(steps=8), gran=ikv.IKV_GRAN_KVHEAD, max_holes=3), 2e-2)
     _assert(run_lockstep(small_llama(steps=8), compact_mode=ikv.IKV_COMPACT_HOLEFILL, max_holes=3), 2e-2)
     _assert(run_lockstep(small_llama(steps=8, refresh_period=2), refresh_init=ikv.IKV_INIT_MEAN, max_holes=64), 2e-2)
+
+
+def test_cumulative_and_single_step_aggregation():
+    """Eq. 3 (cumulative) and Eq. 2 (single-step) in place of the EMA, under full refresh,
+    Lazy refresh and deferred compaction."""
+    cum, single = ikv.IKV_AGG_CUMULATIVE, ikv.IKV_AGG_SINGLE_STEP
+    _assert(run_lockstep(gen.config(0), agg_mode=cum), 1e-4, strict_fraction=1.0)
+    _assert(run_lockstep(small_llama(steps=8), agg_mode=cum), 2e-2)
+    _assert(run_lockstep(small_llama(steps=8, refresh_period=3), agg_mode=cum, max_holes=4), 2e-2)
+    _assert(run_lockstep(small_llama(steps=6), agg_mode=single), 2e-2)
+    _assert(run_lockstep(small_llama(steps=6), gran=ikv.IKV_GRAN_KVHEAD, agg_mode=single,
+                         compact_mode=ikv.IKV_COMPACT_STABLE_SHORT), 2e-2)
