@@ -42,6 +42,11 @@ Readings taken where the paper is silent (each also stated where it is used):
 * R6 (self-attention): the appended token is part of its own step's softmax.
 * R7 (scale): softmax scale ``1/sqrt(d)``; keys are used as stored.
 * R8 (eligible layers): all layers unless a layer mask says otherwise.
+* R9 (scorer variants, Appendix "Per-step scoring"): VNorm divides each value
+  row's l2 norm by the mean norm over the cached tokens of its (layer, KV head);
+  entropy weighting uses the normalized entropy H(s) / ln n of the layer's
+  pooled score distribution s over the n cached tokens (per utility row), and
+  weight 1 when n = 1 or when a head's values are all zero.
 """
 from __future__ import annotations
 
@@ -97,6 +102,35 @@ def pooled_score(a: np.ndarray, granularity: int, kv_heads: int) -> np.ndarray:
     if granularity == GRAN_SEQ:
         return a.mean(axis=0, keepdims=True)
     return a.reshape(kv_heads, H // kv_heads, L).mean(axis=1)
+
+
+def vnorm_weights(V_l: Sequence[np.ndarray]) -> np.ndarray:
+    """Appendix "Per-step scoring", VNorm: for each KV head g, the l2 norm of every cached
+    value row divided by the mean of those norms over the cached tokens.  [H_kv, L].
+    (All-zero values of a head: weight 1, reading R9.)"""
+    n = np.stack([np.sqrt(np.sum(np.asarray(v, np.float64) ** 2, axis=1)) for v in V_l])
+    mean = n.mean(axis=1, keepdims=True)
+    return np.where(mean > 0, n / np.where(mean > 0, mean, 1.0), 1.0)
+
+
+def vnorm_score(a: np.ndarray, V_l: Sequence[np.ndarray], granularity: int, kv_heads: int) -> np.ndarray:
+    """VNorm per-step score: each head's probabilities times its KV head's value-norm
+    weights, then pooled as in Eq. 1."""
+    H, L = a.shape
+    w = vnorm_weights(V_l)
+    return pooled_score(a * np.repeat(w, H // kv_heads, axis=0), granularity, kv_heads)
+
+
+def entropy_weight(s_row: np.ndarray) -> float:
+    """Entropy weighting: a layer's contribution is scaled by the normalized entropy of its
+    pooled score distribution (which sums to 1 over the cached tokens), H(s) / ln n;
+    1 when a single token is cached (reading R9)."""
+    s_row = np.asarray(s_row, np.float64)
+    n = s_row.size
+    if n <= 1:
+        return 1.0
+    p = s_row[s_row > 0]
+    return float(-np.sum(p * np.log(p)) / np.log(n))
 
 
 # --------------------------------------------------------------------------
@@ -190,6 +224,7 @@ class Params:
     layer_mask: Optional[List[bool]] = None   # eligible layers (R8)
     refresh_init: str = "zero"         # R3
     aggregation: str = "ema"           # Eq. 4 (InertiaKV); "cumulative" (Eq. 3) or "single" (Eq. 2)
+    scorer: str = "attention"          # Eq. 1; "vnorm" or "entropy" (Appendix "Per-step scoring")
 
 
 @dataclass
@@ -266,7 +301,12 @@ def attend_and_score(st: SeqState, q_t: np.ndarray, refresh: bool, p: Params) ->
         outs.append(o)
         eligible = p.layer_mask is None or p.layer_mask[l]
         if refresh and eligible:
-            s = pooled_score(a, st.granularity, st.kv_heads)
+            if p.scorer == "vnorm":
+                s = vnorm_score(a, st.V[l], st.granularity, st.kv_heads)
+            else:
+                s = pooled_score(a, st.granularity, st.kv_heads)
+            if p.scorer == "entropy":
+                s = s * np.array([[entropy_weight(row)] for row in s])
             st.m = aggregate(st.m, s, p)
     return np.stack(outs)
 

@@ -286,6 +286,85 @@ def test_single_step_keeps_last_layer_and_equals_alpha_zero():
         assert np.array_equal(st.m, ref.m)
 
 
+def test_vnorm_weights_bruteforce_and_invariances():
+    """VNorm (Appendix "Per-step scoring"): pure-Python norms and means; unit-norm values
+    leave Eq. 1 unchanged; scaling a KV head's values does not change the score."""
+    rng = np.random.default_rng(21)
+    H, kv, L, d = 6, 3, 9, 5
+    V = [rng.standard_normal((L, d)) for _ in range(kv)]
+    a = rng.random((H, L))
+    a /= a.sum(axis=1, keepdims=True)
+    got = O.vnorm_score(a, V, O.GRAN_SEQ, kv)[0]
+    G = H // kv
+    for i in range(L):
+        acc = 0.0
+        for h in range(H):
+            g = h // G
+            norms = [math.sqrt(sum(x * x for x in V[g][j])) for j in range(L)]
+            acc += a[h, i] * norms[i] / (sum(norms) / L)
+        assert abs(got[i] - acc / H) < 1e-14
+    unit = [v / np.linalg.norm(v, axis=1, keepdims=True) for v in V]
+    assert np.max(np.abs(O.vnorm_score(a, unit, O.GRAN_KVHEAD, kv) - O.pooled_score(a, O.GRAN_KVHEAD, kv))) < 1e-14
+    scaled = [v * c for v, c in zip(V, (0.5, 3.0, 7.0))]
+    assert np.max(np.abs(O.vnorm_score(a, scaled, O.GRAN_SEQ, kv) - got)) < 1e-14
+
+
+def test_entropy_weight_closed_forms():
+    """Entropy weighting: uniform scores have normalized entropy 1 (no change), a one-hot
+    distribution 0, and a two-point distribution (p, 1-p) over n tokens has
+    -(p ln p + (1-p) ln(1-p)) / ln n; brute force with math.log."""
+    assert abs(O.entropy_weight(np.full(37, 1 / 37)) - 1.0) < 1e-14
+    assert O.entropy_weight(np.eye(1, 12)[0]) == 0.0
+    assert O.entropy_weight(np.array([1.0])) == 1.0
+    p, n = 0.3, 8
+    s = np.zeros(n)
+    s[2], s[5] = p, 1 - p
+    assert abs(O.entropy_weight(s) - (-(p * math.log(p) + (1 - p) * math.log(1 - p)) / math.log(n))) < 1e-15
+    rng = np.random.default_rng(3)
+    r = rng.random(15)
+    r /= r.sum()
+    assert abs(O.entropy_weight(r) - sum(-x * math.log(x) for x in r) / math.log(15)) < 1e-14
+
+
+def test_entropy_scorer_through_decode_step():
+    """Uniform attention: entropy weight 1, so the step equals the plain scorer bit for
+    bit; a spiked layer contributes its score times its normalized entropy."""
+    layers, kv, H, d, L0, alpha = 2, 1, 2, 4, 10, 0.6
+    K = [[np.zeros((L0, d)) for _ in range(kv)] for _ in range(layers)]
+    V = [[np.ones((L0, d)) for _ in range(kv)] for _ in range(layers)]
+    q = np.ones((layers, H, d))
+    st, ref = O.prefill_state(K, V, budget=L0 + 1), O.prefill_state(K, V, budget=L0 + 1)
+    O.decode_step(st, 1, q, np.zeros((layers, kv, d)), np.ones((layers, kv, d)), O.Params(alpha=alpha, scorer="entropy"))
+    O.decode_step(ref, 1, q, np.zeros((layers, kv, d)), np.ones((layers, kv, d)), O.Params(alpha=alpha))
+    assert np.max(np.abs(st.m - ref.m)) < 1e-15
+    zs = 3.0
+    K2, V2, q2 = _spike_layers(1, 1, 2, 4, L0, [4], zs)
+    st2 = O.prefill_state(K2, V2, budget=L0 + 1)
+    O.decode_step(st2, 1, q2, np.zeros((1, 1, 4)), np.zeros((1, 1, 4)), O.Params(alpha=alpha, scorer="entropy"))
+    L = L0 + 1
+    s = np.full(L, 1.0 / (math.exp(zs) + L - 1))
+    s[4] = math.exp(zs) / (math.exp(zs) + L - 1)
+    w = -sum(x * math.log(x) for x in s) / math.log(L)
+    assert np.max(np.abs(st2.m[0] - (1 - alpha) * w * s)) < 1e-15
+
+
+def test_vnorm_scorer_through_decode_step():
+    """VNorm inside the decode loop: value rows of equal norm give the plain scores; one
+    value row twice as long doubles its token's weight relative to the mean norm."""
+    layers, kv, H, d, L0, alpha = 1, 1, 2, 4, 6, 0.5
+    K = [[np.zeros((L0, d))]]
+    V = [[np.ones((L0, d))]]
+    V[0][0][3] *= 2.0
+    q = np.ones((layers, H, d))
+    st = O.prefill_state(K, V, budget=L0 + 1)
+    O.decode_step(st, 1, q, np.zeros((layers, kv, d)), np.ones((layers, kv, d)), O.Params(alpha=alpha, scorer="vnorm"))
+    L = L0 + 1
+    norms = np.full(L, 2.0)
+    norms[3] = 4.0
+    want = (1 - alpha) * (1.0 / L) * norms / norms.mean()
+    assert np.max(np.abs(st.m[0] - want)) < 1e-15
+
+
 # ---------------------------------------------------------------- schedule
 def test_refresh_sets():
     assert [t for t in range(1, 14) if O.is_refresh(t, 4, False)] == [1, 5, 9, 13]
