@@ -78,6 +78,11 @@ enum { IKV_INIT_ZERO = 0, IKV_INIT_MEAN = 1 };
 /* Temporal aggregation of the per-layer scores (Sec. 3.1): Eq. 4 EMA (InertiaKV),
  * Eq. 3 cumulative sum (H2O-style), Eq. 2 single-step. */
 enum { IKV_AGG_EMA = 0, IKV_AGG_CUMULATIVE = 1, IKV_AGG_SINGLE_STEP = 2 };
+/* Per-step scorer (Appendix "Per-step scoring"): Eq. 1 head-pooled attention; VNorm
+ * (each head's probabilities times the l2 norm of the value row over the mean norm of
+ * its (layer, kv head)); entropy weighting (each layer's pooled score times the
+ * normalized entropy H(s) / ln n of that score over the n live slots, 1 if n = 1). */
+enum { IKV_SCORE_ATTENTION = 0, IKV_SCORE_VNORM = 1, IKV_SCORE_ENTROPY = 2 };
 
 typedef struct {
     int32_t batch, layers, q_heads, kv_heads, head_dim;
@@ -103,6 +108,11 @@ typedef struct {
                                     compacted away (ikv_params.max_holes).  Attention, scores,
                                     selection and the mean-utility append then skip them.
                                     0: every slot below len is live (pos is not read for it). */
+    float *vnorm;                /* [layers][batch][kv_heads][cap] l2 norm of each cached value row,
+                                    by logical slot (device), or NULL.  Needed by the VNorm scorer;
+                                    when set, ikv_append_token / ikv_step store the new row's norm and
+                                    compaction moves the norms with their rows.  Fill it once for the
+                                    prefill with ikv_value_norms. */
 } ikv_cache;
 
 /* Optional per-kernel CUDA events recorded on the call's stream by ikv_step
@@ -139,6 +149,8 @@ typedef struct {
                                        order: IKV_AGG_EMA m = alpha m + (1 - alpha) s (Eq. 4, the
                                        method; default) | IKV_AGG_CUMULATIVE m = m + s (Eq. 3) |
                                        IKV_AGG_SINGLE_STEP m = s (Eq. 2) */
+    int32_t scorer;                 /* IKV_SCORE_ATTENTION (Eq. 1, default) | IKV_SCORE_VNORM (needs
+                                       cache->vnorm) | IKV_SCORE_ENTROPY */
 } ikv_params;
 
 /* Message for the last error on this thread ("" if none). */
@@ -212,6 +224,15 @@ size_t ikv_static_scratch_bytes(void);
 ikv_status ikv_decode_attend_score_static(const ikv_shape *shape, const ikv_cache *cache, int32_t layer,
                                           const void *q, void *out, float *score, float *ema, float alpha,
                                           cudaStream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * ikv_value_norms -- l2 norm of every cached value row (Appendix "Per-step
+ * scoring", VNorm): cache->vnorm[l][b][g][j] = ||V[l][b][g][slot j]||_2 for every
+ * layer l, sequence b, KV head g and logical slot j < len[b] (through start and the
+ * block table).  Call once after the prefill; the append and compaction keep it
+ * current from then on.  Fails with IKV_ERR_ARG if cache->vnorm is NULL.
+ * ------------------------------------------------------------------------- */
+ikv_status ikv_value_norms(const ikv_shape *shape, const ikv_cache *cache, cudaStream_t stream);
 
 /* ---------------------------------------------------------------------------
  * ikv_ema_update -- Eq. 4 on a score array, in place.

@@ -50,7 +50,7 @@ class DecodeCache:
 
     def __init__(self, batch: int, layers: int, q_heads: int, kv_heads: int, head_dim: int, cap_tokens: int,
                  dtype: int = ikv.IKV_BF16, page_size: int = 64, granularity: int = ikv.IKV_GRAN_SEQ,
-                 device: str = "cuda", page_perm_seed: Optional[int] = None):
+                 device: str = "cuda", page_perm_seed: Optional[int] = None, value_norms: bool = False):
         self.batch, self.layers, self.q_heads, self.kv_heads, self.head_dim = batch, layers, q_heads, kv_heads, head_dim
         self.dtype, self.granularity, self.page_size = dtype, granularity, page_size
         self.max_pages = (cap_tokens + page_size - 1) // page_size
@@ -73,6 +73,9 @@ class DecodeCache:
         self.ema = torch.zeros((self.rows, self.cap), dtype=torch.float32, device=device)
         self.budget = torch.zeros(batch, dtype=torch.int32, device=device)
         self.start = torch.zeros(batch, dtype=torch.int32, device=device)
+        # per-slot value-row norms, for the VNorm scorer
+        self.vnorm = (torch.zeros((layers, batch, kv_heads, self.cap), dtype=torch.float32, device=device)
+                      if value_norms else None)
         self.max_len = 0
 
     # ---- ABI structs ------------------------------------------------------
@@ -84,7 +87,8 @@ class DecodeCache:
         ml = self.max_len if max_len is None else max_len
         return ikv.ikv_cache(self.k.data_ptr(), self.v.data_ptr(), self.block_table.data_ptr(), self.num_pages,
                              self.page_size, self.max_pages, self.len.data_ptr(), self.pos.data_ptr(),
-                             self.next_pos.data_ptr(), ml, self.start.data_ptr(), 1 if dead_slots else 0)
+                             self.next_pos.data_ptr(), ml, self.start.data_ptr(), 1 if dead_slots else 0,
+                             self.vnorm.data_ptr() if self.vnorm is not None else None)
 
     @property
     def rows_per_seq(self) -> int:
@@ -127,7 +131,7 @@ class DecodeCache:
     def params(self, alpha: float, refresh_period: int = 1, score_free: bool = False,
                compact_mode: int = ikv.IKV_COMPACT_STABLE, refresh_init: int = ikv.IKV_INIT_ZERO,
                layer_eligible: Optional[Sequence[int]] = None, max_holes: int = 0,
-               agg_mode: int = ikv.IKV_AGG_EMA) -> ikv.ikv_params:
+               agg_mode: int = ikv.IKV_AGG_EMA, scorer: int = ikv.IKV_SCORE_ATTENTION) -> ikv.ikv_params:
         p = ikv.ikv_params()
         p.alpha = alpha
         p.refresh_period = refresh_period
@@ -140,6 +144,7 @@ class DecodeCache:
         p.refresh_init = refresh_init
         p.max_holes = max_holes
         p.agg_mode = agg_mode
+        p.scorer = scorer
         return p
 
 

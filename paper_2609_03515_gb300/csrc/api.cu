@@ -126,7 +126,7 @@ AttendWs attend_ws(const ikv_shape *s, int32_t cap, int n_layers, bool logits) {
 
 struct StepWs {
     AttendWs at;
-    size_t keep, keep_len, done, cdone, moves, n_moves, end;
+    size_t keep, keep_len, done, cdone, moves, n_moves, sbuf, epart, vmean, end;
 };
 
 StepWs step_ws(const ikv_shape *s, int32_t cap) {
@@ -145,6 +145,14 @@ StepWs step_ws(const ikv_shape *s, int32_t cap) {
     off = align256(off + R * cap * 2 * sizeof(int32_t));
     w.n_moves = off;
     off = align256(off + R * sizeof(int32_t));
+    // scorer variants: entropy pass buffers and VNorm means
+    const size_t blk_max = ((size_t)cap + 31) / 32;
+    w.sbuf = off;
+    off = align256(off + R * s->layers * (size_t)logit_stride(cap) * sizeof(float));
+    w.epart = off;
+    off = align256(off + R * (s->layers + 1) * blk_max * sizeof(float));
+    w.vmean = off;
+    off = align256(off + (size_t)s->batch * s->layers * s->kv_heads * sizeof(float));
     w.end = off;
     return w;
 }
@@ -251,29 +259,51 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
     return IKV_OK;
 }
 
+// Scorer-variant scratch of ikv_step (null for the per-layer entry points, which
+// score with Eq. 1 only).
+struct ScorerWs {
+    float *sbuf = nullptr, *epart = nullptr, *vmean = nullptr;
+};
+
 ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, const int32_t *elig, int n_elig,
                      int32_t max_len, void *ws, const AttendWs &w, float alpha, float *ema, float *score,
-                     cudaStream_t st, int32_t agg = IKV_AGG_EMA) {
+                     cudaStream_t st, int32_t agg = IKV_AGG_EMA, int32_t scorer = IKV_SCORE_ATTENTION,
+                     const ScorerWs &sw = ScorerWs{}) {
+    ScoreArgs base{};
+    base.len = c->len;
+    base.batch = s->batch;
+    base.q_heads = s->q_heads;
+    base.kv_heads = s->kv_heads;
+    base.rows_per_seq = rows_per_seq(s);
+    base.n_layers = n_layers;
+    base.cap = cap_of(c);
+    base.logits = at<float>(ws, w.logits);
+    base.lstride = logit_stride(cap_of(c));
+    base.lse2 = at<float>(ws, w.lse2);
+    base.alpha = alpha;
+    base.agg = agg;
+    base.ema = ema;
+    base.score = score;
+    base.layer0 = 0;
+    base.scorer = scorer;
+    base.vnorm = c->vnorm;
+    base.vmean = sw.vmean;
+    base.pos = c->dead_slots ? c->pos : nullptr;
+    base.sbuf = sw.sbuf;
+    base.epart = sw.epart;
+    base.n_elig_total = n_elig;
+    int V = 1;
+    base.nblk = score_blocks(base, max_len, sm_count(), &V);
+    base.blk_tok = 32 * V;
+    if (scorer == IKV_SCORE_VNORM) IKV_TRY_CUDA(launch_vnorm_mean(base, st), "vnorm mean launch");
     for (int k0 = 0; k0 < n_elig; k0 += kMaxLayersPerScorePass) {
-        ScoreArgs sa{};
-        sa.len = c->len;
-        sa.batch = s->batch;
-        sa.q_heads = s->q_heads;
-        sa.kv_heads = s->kv_heads;
-        sa.rows_per_seq = rows_per_seq(s);
-        sa.n_layers = n_layers;
-        sa.cap = cap_of(c);
-        sa.logits = at<float>(ws, w.logits);
-        sa.lstride = logit_stride(cap_of(c));
-        sa.lse2 = at<float>(ws, w.lse2);
+        ScoreArgs sa = base;
         sa.n_elig = n_elig - k0 < kMaxLayersPerScorePass ? n_elig - k0 : kMaxLayersPerScorePass;
+        sa.k0 = k0;
         for (int k = 0; k < sa.n_elig; ++k) sa.elig[k] = elig[k0 + k];
-        sa.alpha = alpha;
-        sa.agg = agg;
-        sa.ema = ema;
-        sa.score = score;
         IKV_TRY_CUDA(launch_score_ema(sa, max_len, sm_count(), st), "score launch");
     }
+    if (scorer == IKV_SCORE_ENTROPY) IKV_TRY_CUDA(launch_entropy_fold(base, max_len, st), "entropy fold launch");
     return IKV_OK;
 }
 
@@ -346,6 +376,18 @@ ikv_status ikv_decode_attend_score(const ikv_shape *shape, const ikv_cache *cach
     return IKV_OK;
 }
 
+ikv_status ikv_value_norms(const ikv_shape *shape, const ikv_cache *cache, cudaStream_t stream) {
+    g_err[0] = 0;
+    ikv_status e = check_shape(shape);
+    if (e) return e;
+    if ((e = check_cache(shape, cache, false))) return e;
+    if (!cache->vnorm) return fail(IKV_ERR_ARG, "cache->vnorm is NULL");
+    IKV_TRY_CUDA(launch_value_norms(cache->v, view_of(shape, cache), cache->len, shape->batch, shape->layers,
+                                    cap_of(cache), shape->dtype, cache->vnorm, stream),
+                 "value norms launch");
+    return IKV_OK;
+}
+
 ikv_status ikv_ema_update(int32_t rows, int32_t cap, float *ema, const float *score, const int32_t *len,
                           int32_t rows_per_seq_, float alpha, cudaStream_t stream) {
     g_err[0] = 0;
@@ -408,6 +450,7 @@ static ikv_status compact_impl(const ikv_shape *shape, ikv_cache *cache, const i
     a.moves = moves;
     a.n_moves = n_moves;
     a.max_holes = max_holes;
+    a.vnorm = cache->vnorm;
     IKV_TRY_CUDA(launch_compact(a, mode, stream), "compact launch");
     return IKV_OK;
 }
@@ -457,6 +500,7 @@ static ikv_status append_impl(const ikv_shape *shape, ikv_cache *cache, const vo
     a.init_mean = ema ? init_mean : 0;
     a.dead_slots = cache->dead_slots ? 1 : 0;
     a.done = done;
+    a.vnorm = cache->vnorm;
     if (!counters_zeroed)
         IKV_TRY_CUDA(cudaMemsetAsync(done, 0, sizeof(int32_t) * shape->batch, stream), "cudaMemsetAsync");
     IKV_TRY_CUDA(launch_append(a, stream), "append launch");
@@ -511,6 +555,9 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     if (p->max_holes < 0) return fail(IKV_ERR_ARG, "max_holes must be >= 0");
     if (p->agg_mode != IKV_AGG_EMA && p->agg_mode != IKV_AGG_CUMULATIVE && p->agg_mode != IKV_AGG_SINGLE_STEP)
         return fail(IKV_ERR_ARG, "unknown agg_mode %d", p->agg_mode);
+    if (p->scorer != IKV_SCORE_ATTENTION && p->scorer != IKV_SCORE_VNORM && p->scorer != IKV_SCORE_ENTROPY)
+        return fail(IKV_ERR_ARG, "unknown scorer %d", p->scorer);
+    if (p->scorer == IKV_SCORE_VNORM && !cache->vnorm) return fail(IKV_ERR_ARG, "IKV_SCORE_VNORM needs cache->vnorm");
     // with deferred compaction every kernel of the step treats pos < 0 as a dead slot
     ikv_cache cv = *cache;
     if (p->max_holes > 0) cv.dead_slots = 1;
@@ -543,8 +590,12 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
                         true)))
         return e;
     if (tm && (e = record(tm->combine_end, stream))) return e;
+    ScorerWs sw;
+    sw.sbuf = at<float>(ws, w.sbuf);
+    sw.epart = at<float>(ws, w.epart);
+    sw.vmean = at<float>(ws, w.vmean);
     if (scoring && (e = run_score(shape, cache, shape->layers, elig, n_elig, L1, ws, w.at, p->alpha, ema, nullptr, stream,
-                                  p->agg_mode)))
+                                  p->agg_mode, p->scorer, sw)))
         return e;
     if (tm && (e = record(tm->score_end, stream))) return e;
     const int32_t R = shape->batch * rows_per_seq(shape);

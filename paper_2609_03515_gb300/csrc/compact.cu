@@ -62,6 +62,31 @@ __device__ __forceinline__ float block_sum(float v, float *scratch) {
     return r;
 }
 
+// Logical gather of one per-slot row in place: row[j] <- row[kp[j]] for j < n (kp
+// ascending, kp[j] >= j).  Chunk by chunk, every read lands before any write; a
+// later chunk's sources lie at or after its own slots, above every earlier write.
+template <typename T>
+__device__ __forceinline__ void gather_row(T *row, const int32_t *kp, int n) {
+    constexpr int PER = 16;
+    for (int base = 0; base < n; base += kCompThreads * PER) {
+        T val[PER];
+        int src[PER];
+#pragma unroll
+        for (int u = 0; u < PER; ++u) {
+            const int j = base + u * kCompThreads + (int)threadIdx.x;
+            src[u] = j < n ? kp[j] : j;
+            if (j < n && src[u] != j) val[u] = row[src[u]];
+        }
+        __syncthreads();
+#pragma unroll
+        for (int u = 0; u < PER; ++u) {
+            const int j = base + u * kCompThreads + (int)threadIdx.x;
+            if (j < n && src[u] != j) row[j] = val[u];
+        }
+        __syncthreads();
+    }
+}
+
 // Deferred compaction: sequence b only marks its evicted slots dead while its dead
 // slots (the ones already dead plus this step's evictions: len - kept) stay within
 // max_holes.  Every row of b keeps the same number of slots, so row b * rps decides.
@@ -192,6 +217,7 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
             }
             cp_async_wait<0>();
         }
+        if (a.vnorm) gather_row(a.vnorm + (((int64_t)l * a.batch + b) * kvh + g) * a.cap, kp, n);
     } else {
         // utility / position rows: always the plain stable gather of logical slots
         const int rr = x - nkv;
@@ -299,6 +325,10 @@ __global__ void __launch_bounds__(kCompThreads) holefill_move_kernel(const Compa
         const int CPR = rowB >> 4;
         unsigned char *kb = reinterpret_cast<unsigned char *>(a.k);
         unsigned char *vb = reinterpret_cast<unsigned char *>(a.v);
+        if (a.vnorm) {
+            float *vn = a.vnorm + (((int64_t)l * a.batch + b) * kvh + g) * a.cap;
+            for (int m = tid; m < nm; m += kCompThreads) vn[mv[2 * m + 1]] = vn[mv[2 * m]];
+        }
         for (int idx = tid; idx < nm * CPR; idx += kCompThreads) {
             const int m = idx / CPR, c = idx % CPR;
             const int64_t src = a.pv.row_phys(b, l, g, S + mv[2 * m]);
@@ -361,6 +391,23 @@ __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a
                 const int64_t dst = a.pv.row_phys(b, l, g, S + L) * rowB + c * 16;
                 *reinterpret_cast<uint4 *>(kb + dst) = *reinterpret_cast<const uint4 *>(kn + src);
                 *reinterpret_cast<uint4 *>(vb + dst) = *reinterpret_cast<const uint4 *>(vn + src);
+            }
+        }
+        if (a.vnorm) {  // l2 norm of the new value row: warp w takes the CTA's row w
+            const int x = blockIdx.x * kAppendRows + (tid >> 5), lane = tid & 31;
+            if ((tid >> 5) < kAppendRows && x < nkv) {
+                const int l = x / kvh, g = x % kvh;
+                const int64_t e0 = (((int64_t)l * a.batch + b) * kvh + g) * a.pv.head_dim;
+                float sq = 0.f;
+                for (int e = lane; e < a.pv.head_dim; e += 32) {
+                    const float xv = a.elem_bytes == 2
+                                         ? __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(a.v_new)[e0 + e])
+                                         : reinterpret_cast<const float *>(a.v_new)[e0 + e];
+                    sq += xv * xv;
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+                if (lane == 0) a.vnorm[(((int64_t)l * a.batch + b) * kvh + g) * a.cap + L] = sqrtf(sq);
             }
         }
         if (blockIdx.x == 0) {

@@ -74,6 +74,17 @@ struct ScoreArgs {
     float *ema;                 // [rows][cap] or null
     float *score;               // [rows][cap] or null (only meaningful with one layer)
     int32_t elig[kMaxLayersPerScorePass];
+    int32_t layer0;             // model layer of local layer 0 (vnorm indexing)
+    int32_t scorer;             // IKV_SCORE_*
+    const float *vnorm;         // VNorm: [layers][batch][kv_heads][cap] value-row norms
+    float *vmean;               // VNorm: [batch][n_layers][kv_heads] mean norm over live slots
+    const int32_t *pos;         // [rows][cap], -1 at dead slots, or null (all slots below len live)
+    float *sbuf;                // entropy: [rows][n_elig_total][lstride] pooled scores
+    float *epart;               // entropy: [rows][n_elig_total + 1][nblk] partial entropies, live counts
+    int32_t nblk;               // entropy: token blocks of the score pass (partials row stride)
+    int32_t blk_tok;            // entropy: tokens per block of the score pass
+    int32_t k0;                 // eligible-layer index of this pass's first layer
+    int32_t n_elig_total;       // eligible layers over all passes
 };
 
 // tensor-core attention (bf16, head_dim 128): attend_tc.cu
@@ -92,6 +103,12 @@ cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group,
 cudaError_t launch_attend(const AttendArgs &a, int dtype, int head_dim, int group, cudaStream_t st);
 cudaError_t launch_combine(const CombineArgs &a, int dtype, cudaStream_t st);
 cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, int sms, cudaStream_t st);
+// token blocks (and tokens per lane V) the score pass uses for max_len
+int score_blocks(const ScoreArgs &a, int32_t max_len, int sms, int *V);
+cudaError_t launch_entropy_fold(const ScoreArgs &a, int32_t max_len, cudaStream_t st);
+cudaError_t launch_vnorm_mean(const ScoreArgs &a, cudaStream_t st);
+cudaError_t launch_value_norms(const void *v, const PagedView &pv, const int32_t *len, int32_t batch, int32_t layers,
+                               int32_t cap, int dtype, float *vnorm, cudaStream_t st);
 cudaError_t launch_ema_update(int32_t rows, int32_t cap, float *ema, const float *score, const int32_t *len,
                               int32_t rows_per_seq, float alpha, int32_t max_len, cudaStream_t st);
 // Deferred compaction inside selection: when a row has exactly one slot too many and
@@ -121,6 +138,7 @@ struct CompactArgs {
     int32_t *n_moves;           // hole-fill: [rows]
     int32_t max_holes;          // > 0: while a sequence's dead slots stay <= max_holes, mark
                                 // the evicted slots dead (pos = -1) instead of compacting
+    float *vnorm;               // [layers][batch][kv_heads][cap] value-row norms moved with the rows, or null
 };
 cudaError_t launch_compact(const CompactArgs &a, int mode, cudaStream_t st);
 
@@ -134,6 +152,7 @@ struct AppendArgs {
     int32_t init_mean;
     int32_t dead_slots;         // the mean initialisation skips slots with pos < 0
     int32_t *done;              // [batch] arrival counters, zero on entry; reset by the last CTA
+    float *vnorm;               // [layers][batch][kv_heads][cap]: the new row's norm is stored, or null
 };
 cudaError_t launch_append(const AppendArgs &a, cudaStream_t st);
 // reads and clears the append kernel's device error word (bit 0: no free slot)

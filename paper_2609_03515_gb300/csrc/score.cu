@@ -1,13 +1,15 @@
-// Eq. 1 score and the layer-sequential EMA of Eq. 4 (Appendix "Layer scoring"),
-// fused with the softmax normalisation.
+// Eq. 1 score and the layer-sequential aggregation of Eq. 2-4 (Appendix "Layer
+// scoring"), fused with the softmax normalisation; the VNorm and entropy-weighted
+// scorers of the Appendix "Per-step scoring"; value-row norms for VNorm.
 //
-// score_ema_kernel: one CTA per (32-token chunk, utility row), one warp per
-// eligible layer (up to 32 per pass), lanes over tokens.  Warp l computes
-// s_l(i) = mean over the row's heads of p_h(i) = exp2(z_h(i) - lse2_h) from
-// the attention kernel's log2-domain logits and log-sum-exp; warp 0 then folds
-// the layers into the utility in ascending layer order,
-// m = alpha m + (1 - alpha) s_l.  More than 32 eligible layers take several
-// passes, launched in order.
+// score_kernel: one CTA per (32 V tokens, utility row), one warp per eligible layer
+// (up to 32 per pass, passes launched in layer order), V consecutive tokens per lane.
+// Warp l computes s_l(i) = mean over the row's heads of p_h(i) = exp2(z_h(i) - lse2_h)
+// from the attention kernel's log2-domain logits and log-sum-exp (VNorm: each head's
+// p_h(i) times its KV head's value-norm weight); the CTA's first 32 V threads then fold
+// the layers into the utility in ascending order.  The entropy scorer needs every
+// token of a layer before its weight is known, so its first pass only stores s_l and
+// per-block partial entropies, and entropy_fold_kernel applies the weights and folds.
 #include "ikv_internal.cuh"
 
 namespace ikv {
@@ -23,16 +25,24 @@ __device__ __forceinline__ float vget(float x, int) { return x; }
 __device__ __forceinline__ float vget(float2 x, int v) { return v == 0 ? x.x : x.y; }
 __device__ __forceinline__ float vget(float4 x, int v) { return v == 0 ? x.x : v == 1 ? x.y : v == 2 ? x.z : x.w; }
 
-// CTA = 32 V tokens x up to 32 layers.  Warp w computes s_l(i) of eligible
-// layer k0 + w for the CTA's tokens (mean over the row's heads of
-// exp2(z - lse2)), V consecutive tokens per lane; the CTA's first 32 V
-// threads then fold the layers into the utility in ascending order.  The
-// pass is latency bound: every head of a batch of 32 / V is loaded before any
-// is used, the per-head log-sum-exp travels by shuffle, and the utility is
-// fetched before the loads.  V > 1 reads each head row in 256- or 512-byte
-// runs, which DRAM serves far better than scattered 128-byte pieces.
-template <int V>
-__global__ void __launch_bounds__(kScoreWarps * 32, 1) score_ema_kernel(const ScoreArgs a) {
+__device__ __forceinline__ float aggregate(float m, float s, int agg, float alpha) {
+    if (agg == IKV_AGG_EMA) return alpha * m + (1.f - alpha) * s;  // Eq. 4
+    if (agg == IKV_AGG_CUMULATIVE) return m + s;                    // Eq. 3
+    return s;                                                       // Eq. 2
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// The pass is latency bound: every head of a batch of 32 / V is loaded before any
+// is used, the per-head log-sum-exp travels by shuffle, and the utility is fetched
+// before the loads.  V > 1 reads each head row in 256- or 512-byte runs, which DRAM
+// serves far better than scattered 128-byte pieces.
+template <int V, int SCORER>
+__global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreArgs a) {
     using VT = typename VecF<V>::T;
     constexpr int kTok = 32 * V;   // tokens per CTA
     constexpr int kHB = 32 / V;    // heads per load batch (32 registers of loads)
@@ -49,13 +59,13 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_ema_kernel(const Sc
         nh = a.q_heads / a.kv_heads;
         h0 = (r % a.rows_per_seq) * nh;
     }
-    const int H = a.q_heads;
+    const int H = a.q_heads, G = a.q_heads / a.kv_heads;
     const float inv = 1.f / (float)nh;
     const int fi = i0 + (int)threadIdx.x;  // token folded by this thread (threads < kTok)
     const bool folds = threadIdx.x < kTok && fi < L;
     const int64_t at = (int64_t)r * a.cap + fi;
     float m = 0.f;
-    if (folds && a.ema) m = a.ema[at];
+    if (SCORER != IKV_SCORE_ENTROPY && folds && a.ema) m = a.ema[at];
     if (warp < a.n_elig) {
         const int li = a.elig[warp];
         // row padding keeps i0 + kTok <= lstride, so the vector loads stay inside the row
@@ -77,28 +87,130 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_ema_kernel(const Sc
             for (int j = 0; j < kHB; ++j) {
                 const float lj = __shfl_sync(0xffffffffu, lse_lane, j);
                 if (il < L && j < nb) {
+                    float w[V];
 #pragma unroll
-                    for (int v = 0; v < V; ++v) acc[v] += exp2f(vget(z[j], v) - lj);
+                    for (int v = 0; v < V; ++v) w[v] = 1.f;
+                    if (SCORER == IKV_SCORE_VNORM) {
+                        // value-norm weight of this head's KV head: norm over the unit's mean norm
+                        const int g = (h0 + hb + j) / G;
+                        const int64_t u = ((int64_t)b * a.n_layers + li) * a.kv_heads + g;
+                        const float mean = a.vmean[u];
+                        const float *vn = a.vnorm + (((int64_t)(a.layer0 + li) * a.batch + b) * a.kv_heads + g) * a.cap;
+#pragma unroll
+                        for (int v = 0; v < V; ++v)
+                            w[v] = mean > 0.f ? (il + v < L ? __ldg(vn + il + v) : 0.f) / mean : 1.f;
+                    }
+#pragma unroll
+                    for (int v = 0; v < V; ++v) acc[v] += exp2f(vget(z[j], v) - lj) * w[v];
                 }
             }
         }
 #pragma unroll
         for (int v = 0; v < V; ++v) sl[warp][lane * V + v] = acc[v] * inv;
+        if (SCORER == IKV_SCORE_ENTROPY) {
+            // the layer's pooled scores, and this block's share of -sum s ln s over them
+            const int k = a.k0 + warp;
+            float e = 0.f;
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int i = il + v;
+                const float s = acc[v] * inv;
+                if (i < L) {
+                    a.sbuf[((int64_t)r * a.n_elig_total + k) * a.lstride + i] = s;
+                    if (s > 0.f) e -= s * logf(s);
+                }
+            }
+            e = warp_sum(e);
+            if (lane == 0) a.epart[((int64_t)r * (a.n_elig_total + 1) + k) * a.nblk + blockIdx.x] = e;
+        }
+    }
+    if (SCORER == IKV_SCORE_ENTROPY) {
+        if (warp == 0) {  // live slots of this block (the entropy normalisation is ln of their count)
+            float c = 0.f;
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int i = il + v;
+                if (i < L && (!a.pos || a.pos[(int64_t)r * a.cap + i] >= 0)) c += 1.f;
+            }
+            c = warp_sum(c);
+            if (lane == 0) a.epart[((int64_t)r * (a.n_elig_total + 1) + a.n_elig_total) * a.nblk + blockIdx.x] = c;
+        }
+        return;
     }
     __syncthreads();
     if (folds) {
         float sc = 0.f;
         for (int k = 0; k < a.n_elig; ++k) {
             sc = sl[k][threadIdx.x];
-            if (a.agg == IKV_AGG_EMA)
-                m = a.alpha * m + (1.f - a.alpha) * sc;  // Eq. 4
-            else if (a.agg == IKV_AGG_CUMULATIVE)
-                m += sc;                                  // Eq. 3
-            else
-                m = sc;                                   // Eq. 2
+            m = aggregate(m, sc, a.agg, a.alpha);
         }
         if (a.ema) a.ema[at] = m;
         if (a.score) a.score[at] = sc;
+    }
+}
+
+// Entropy weighting, second pass: the normalised entropy w_k = H(s_k) / ln n of every
+// eligible layer's pooled score distribution (n live slots; 1 when n <= 1), then the
+// layer-sequential fold of w_k s_k(i) for this CTA's tokens.
+constexpr int kFoldThreads = 256;
+__global__ void __launch_bounds__(kFoldThreads) entropy_fold_kernel(const ScoreArgs a) {
+    __shared__ float wk[kMaxLayers];
+    __shared__ float n_live;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int r = blockIdx.y;
+    const int L = a.len[r / a.rows_per_seq];
+    const int i = blockIdx.x * kFoldThreads + threadIdx.x;
+    if ((int)(blockIdx.x * kFoldThreads) >= L) return;
+    const int NE = a.n_elig_total;
+    const float *ep = a.epart + (int64_t)r * (NE + 1) * a.nblk;
+    const int nb = (L + a.blk_tok - 1) / a.blk_tok;  // the blocks the first pass wrote for this row
+    if (warp == 0) {
+        float c = 0.f;
+        for (int j = lane; j < nb; j += 32) c += ep[(int64_t)NE * a.nblk + j];
+        c = warp_sum(c);
+        if (lane == 0) n_live = c;
+    }
+    __syncthreads();
+    const float n = n_live;
+    for (int k = warp; k < NE; k += kFoldThreads / 32) {
+        float e = 0.f;
+        for (int j = lane; j < nb; j += 32) e += ep[(int64_t)k * a.nblk + j];
+        e = warp_sum(e);
+        if (lane == 0) wk[k] = n > 1.5f ? e / logf(n) : 1.f;
+    }
+    __syncthreads();
+    if (i >= L) return;
+    const int64_t at = (int64_t)r * a.cap + i;
+    float m = a.ema[at];
+    for (int k = 0; k < NE; ++k)
+        m = aggregate(m, wk[k] * a.sbuf[((int64_t)r * NE + k) * a.lstride + i], a.agg, a.alpha);
+    a.ema[at] = m;
+}
+
+// Mean value-row norm of every (sequence, layer, kv head) over its live slots.
+constexpr int kMeanThreads = 256;
+__global__ void __launch_bounds__(kMeanThreads) vnorm_mean_kernel(const ScoreArgs a) {
+    __shared__ float red[2][kMeanThreads / 32];
+    const int u = blockIdx.x;  // (b * n_layers + li) * kv_heads + g
+    const int g = u % a.kv_heads, li = (u / a.kv_heads) % a.n_layers, b = u / a.kv_heads / a.n_layers;
+    const int L = a.len[b];
+    const int r = b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g);
+    const float *vn = a.vnorm + (((int64_t)(a.layer0 + li) * a.batch + b) * a.kv_heads + g) * a.cap;
+    float s = 0.f, c = 0.f;
+    for (int i = threadIdx.x; i < L; i += kMeanThreads)
+        if (!a.pos || a.pos[(int64_t)r * a.cap + i] >= 0) {
+            s += vn[i];
+            c += 1.f;
+        }
+    s = warp_sum(s);
+    c = warp_sum(c);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (lane == 0) red[0][warp] = s, red[1][warp] = c;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float ts = 0.f, tc = 0.f;
+        for (int w = 0; w < kMeanThreads / 32; ++w) ts += red[0][w], tc += red[1][w];
+        a.vmean[u] = tc > 0.f ? ts / tc : 0.f;
     }
 }
 
@@ -112,21 +224,90 @@ __global__ void ema_update_kernel(int32_t cap, float *ema, const float *score, c
     }
 }
 
+// l2 norm of every cached value row: one warp per (layer, sequence, kv head, slot).
+template <typename T>
+__global__ void value_norms_kernel(const T *v, PagedView pv, const int32_t *len, int32_t batch, int32_t layers,
+                                   int32_t cap, float *vnorm) {
+    const int lane = threadIdx.x & 31;
+    const int64_t wid = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const int64_t units = (int64_t)layers * batch * pv.kv_heads;
+    const int64_t u = wid / cap;
+    const int j = (int)(wid % cap);
+    if (u >= units) return;
+    const int g = (int)(u % pv.kv_heads), b = (int)((u / pv.kv_heads) % batch), l = (int)(u / pv.kv_heads / batch);
+    if (j >= len[b]) return;
+    const T *row = v + pv.row_phys(b, l, g, pv.start_of(b) + j) * pv.head_dim;
+    float s = 0.f;
+    for (int e = lane; e < pv.head_dim; e += 32) {
+        const float x = static_cast<float>(row[e]);
+        s += x * x;
+    }
+    s = warp_sum(s);
+    if (lane == 0) vnorm[u * cap + j] = sqrtf(s);
+}
+
 }  // namespace
 
-cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, int sms, cudaStream_t st) {
-    if (max_len <= 0 || a.n_elig <= 0) return cudaSuccess;
+int score_blocks(const ScoreArgs &a, int32_t max_len, int sms, int *V) {
     // widest token vector that still gives every SM two CTAs
     const int64_t rows = (int64_t)a.batch * a.rows_per_seq;
     auto ctas = [&](int tok) { return rows * ((max_len + tok - 1) / tok); };
-    const int V = ctas(128) >= 2 * sms ? 4 : ctas(64) >= 2 * sms ? 2 : 1;
-    dim3 grid((max_len + 32 * V - 1) / (32 * V), (unsigned)rows);
+    *V = ctas(128) >= 2 * sms ? 4 : ctas(64) >= 2 * sms ? 2 : 1;
+    return (max_len + 32 * *V - 1) / (32 * *V);
+}
+
+template <int SCORER>
+static void launch_score_t(const ScoreArgs &a, dim3 grid, int V, cudaStream_t st) {
     if (V == 4)
-        score_ema_kernel<4><<<grid, kScoreWarps * 32, 0, st>>>(a);
+        score_kernel<4, SCORER><<<grid, kScoreWarps * 32, 0, st>>>(a);
     else if (V == 2)
-        score_ema_kernel<2><<<grid, kScoreWarps * 32, 0, st>>>(a);
+        score_kernel<2, SCORER><<<grid, kScoreWarps * 32, 0, st>>>(a);
     else
-        score_ema_kernel<1><<<grid, kScoreWarps * 32, 0, st>>>(a);
+        score_kernel<1, SCORER><<<grid, kScoreWarps * 32, 0, st>>>(a);
+}
+
+cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, int sms, cudaStream_t st) {
+    if (max_len <= 0 || a.n_elig <= 0) return cudaSuccess;
+    int V = 1;
+    const int nblk = score_blocks(a, max_len, sms, &V);
+    dim3 grid(nblk, (unsigned)(a.batch * a.rows_per_seq));
+    if (a.scorer == IKV_SCORE_VNORM)
+        launch_score_t<IKV_SCORE_VNORM>(a, grid, V, st);
+    else if (a.scorer == IKV_SCORE_ENTROPY)
+        launch_score_t<IKV_SCORE_ENTROPY>(a, grid, V, st);
+    else
+        launch_score_t<IKV_SCORE_ATTENTION>(a, grid, V, st);
+    note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_entropy_fold(const ScoreArgs &a, int32_t max_len, cudaStream_t st) {
+    if (max_len <= 0 || a.n_elig_total <= 0) return cudaSuccess;
+    dim3 grid((max_len + kFoldThreads - 1) / kFoldThreads, (unsigned)(a.batch * a.rows_per_seq));
+    entropy_fold_kernel<<<grid, kFoldThreads, 0, st>>>(a);
+    note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_vnorm_mean(const ScoreArgs &a, cudaStream_t st) {
+    const int units = a.batch * a.n_layers * a.kv_heads;
+    if (units <= 0) return cudaSuccess;
+    vnorm_mean_kernel<<<units, kMeanThreads, 0, st>>>(a);
+    note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_value_norms(const void *v, const PagedView &pv, const int32_t *len, int32_t batch, int32_t layers,
+                               int32_t cap, int dtype, float *vnorm, cudaStream_t st) {
+    const int64_t warps = (int64_t)layers * batch * pv.kv_heads * cap;
+    if (warps <= 0) return cudaSuccess;
+    const int64_t blocks = (warps + 7) / 8;
+    if (dtype == IKV_BF16)
+        value_norms_kernel<__nv_bfloat16><<<(unsigned)blocks, 256, 0, st>>>(
+            reinterpret_cast<const __nv_bfloat16 *>(v), pv, len, batch, layers, cap, vnorm);
+    else
+        value_norms_kernel<float><<<(unsigned)blocks, 256, 0, st>>>(reinterpret_cast<const float *>(v), pv, len,
+                                                                    batch, layers, cap, vnorm);
     note_launch();
     return cudaGetLastError();
 }

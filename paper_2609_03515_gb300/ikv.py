@@ -21,6 +21,7 @@ IKV_COMPACT_STABLE, IKV_COMPACT_HOLEFILL, IKV_COMPACT_STABLE_SHORT = 0, 1, 2
 IKV_INIT_ZERO, IKV_INIT_MEAN = 0, 1
 IKV_PATH_CUDA_CORE, IKV_PATH_TENSOR_CORE = 0, 1
 IKV_AGG_EMA, IKV_AGG_CUMULATIVE, IKV_AGG_SINGLE_STEP = 0, 1, 2
+IKV_SCORE_ATTENTION, IKV_SCORE_VNORM, IKV_SCORE_ENTROPY = 0, 1, 2
 
 P = ctypes.c_void_p
 I32 = ctypes.c_int32
@@ -35,7 +36,8 @@ class ikv_shape(ctypes.Structure):
 
 class ikv_cache(ctypes.Structure):
     _fields_ = [("k", P), ("v", P), ("block_table", P), ("num_pages", I32), ("page_size", I32), ("max_pages", I32),
-                ("len", P), ("pos", P), ("next_pos", P), ("max_len", I32), ("start", P), ("dead_slots", I32)]
+                ("len", P), ("pos", P), ("next_pos", P), ("max_len", I32), ("start", P), ("dead_slots", I32),
+                ("vnorm", P)]
 
 
 class ikv_timing(ctypes.Structure):
@@ -46,7 +48,8 @@ class ikv_timing(ctypes.Structure):
 class ikv_params(ctypes.Structure):
     _fields_ = [("alpha", F32), ("refresh_period", I32), ("score_free", I32), ("budget", P),
                 ("layer_eligible", P), ("compact_mode", I32), ("refresh_init", I32),
-                ("timing", ctypes.POINTER(ikv_timing)), ("max_holes", I32), ("agg_mode", I32)]
+                ("timing", ctypes.POINTER(ikv_timing)), ("max_holes", I32), ("agg_mode", I32),
+                ("scorer", I32)]
 
 
 class IKVError(RuntimeError):
@@ -70,6 +73,7 @@ def _load():
         "ikv_static_scratch_bytes": ([], SZ),
         "ikv_decode_attend_score_static": ([SP, CP, I32, P, P, P, P, F32, P], I32),
         "ikv_ema_update": ([I32, I32, P, P, P, I32, F32, P], I32),
+        "ikv_value_norms": ([SP, CP, P], I32),
         "ikv_select_budget": ([I32, I32, P, P, I32, P, P, P, P, P], I32),
         "ikv_compact_workspace_size": ([SP, CP, I32, ctypes.POINTER(SZ)], I32),
         "ikv_compact_kv": ([SP, CP, P, P, P, I32, P, SZ, P], I32),
@@ -153,6 +157,10 @@ def ikv_decode_attend_score_static(shape, cache, layer, q, out, score, ema, alph
 def ikv_ema_update(rows, cap, ema, score, length, rows_per_seq, alpha, stream=None) -> None:
     _check(_lib.ikv_ema_update(rows, cap, _p(ema), _p(score), _p(length), rows_per_seq, alpha, _stream(stream)),
            "ikv_ema_update")
+
+
+def ikv_value_norms(shape, cache, stream=None) -> None:
+    _check(_lib.ikv_value_norms(ctypes.byref(shape), ctypes.byref(cache), _stream(stream)), "ikv_value_norms")
 
 
 def ikv_select_budget(rows, cap, util, length, rows_per_seq, budget, pos, keep, keep_len, stream=None) -> None:

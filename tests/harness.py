@@ -32,10 +32,10 @@ def torch_dtype(w: gen.Workload):
 
 
 def make_cache(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, page_perm_seed: Optional[int] = 7,
-               extra_cap: int = 0) -> DecodeCache:
+               extra_cap: int = 0, value_norms: bool = False) -> DecodeCache:
     c = DecodeCache(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.cap + extra_cap,
                     dtype=ikv.IKV_BF16 if w.dtype == gen.BF16 else ikv.IKV_F32, page_size=w.page_size,
-                    granularity=gran, page_perm_seed=page_perm_seed)
+                    granularity=gran, page_perm_seed=page_perm_seed, value_norms=value_norms)
     c.set_prefill(w.prefill, w.budgets())
     return c
 
@@ -123,20 +123,24 @@ def live_slots(pos_row: np.ndarray, n: int) -> np.ndarray:
 def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: int = ikv.IKV_COMPACT_STABLE,
                  steps: Optional[int] = None, kv_check_layers=(0, -1), page_perm_seed: Optional[int] = 7,
                  refresh_init: int = ikv.IKV_INIT_ZERO, layer_eligible=None, max_holes: int = 0,
-                 agg_mode: int = ikv.IKV_AGG_EMA) -> List[StepReport]:
+                 agg_mode: int = ikv.IKV_AGG_EMA, scorer: int = ikv.IKV_SCORE_ATTENTION) -> List[StepReport]:
     T = w.steps if steps is None else steps
     u = w.u_table()
-    c = make_cache(w, gran, page_perm_seed)
+    c = make_cache(w, gran, page_perm_seed, value_norms=scorer == ikv.IKV_SCORE_VNORM)
     kv = fill_host(c, w, u)
+    if c.vnorm is not None:
+        ikv.ikv_value_norms(c.shape(), c.cache(max(w.prefill)))
     sts = oracle_states(w, kv, gran)
     op = O.Params(alpha=w.alpha, refresh_period=w.refresh_period, score_free=w.score_free,
                   granularity=O.GRAN_SEQ if gran == ikv.IKV_GRAN_SEQ else O.GRAN_KVHEAD,
                   layer_mask=None if layer_eligible is None else [bool(x) for x in layer_eligible],
                   refresh_init="zero" if refresh_init == ikv.IKV_INIT_ZERO else "mean",
                   aggregation={ikv.IKV_AGG_EMA: "ema", ikv.IKV_AGG_CUMULATIVE: "cumulative",
-                               ikv.IKV_AGG_SINGLE_STEP: "single"}[agg_mode])
+                               ikv.IKV_AGG_SINGLE_STEP: "single"}[agg_mode],
+                  scorer={ikv.IKV_SCORE_ATTENTION: "attention", ikv.IKV_SCORE_VNORM: "vnorm",
+                          ikv.IKV_SCORE_ENTROPY: "entropy"}[scorer])
     p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, refresh_init, layer_eligible, max_holes,
-                 agg_mode)
+                 agg_mode, scorer)
     ws = c.step_workspace()
     qs = w.queries(1, T + 1, u)
     budgets = w.budgets()

@@ -106,6 +106,13 @@ def test_deferred_compaction_arguments(lib):
     p.max_holes, p.agg_mode = 0, 3   # no such aggregation rule
     assert lib.raw_status("ikv_step", ctypes.byref(shp), ctypes.byref(p), ctypes.byref(cch), 16, 1, 16, 16, 16, 16,
                           16, 1 << 40, None) == lib.IKV_ERR_ARG
+    p.agg_mode, p.scorer = 0, 5   # no such scorer
+    assert lib.raw_status("ikv_step", ctypes.byref(shp), ctypes.byref(p), ctypes.byref(cch), 16, 1, 16, 16, 16, 16,
+                          16, 1 << 40, None) == lib.IKV_ERR_ARG
+    p.scorer = lib.IKV_SCORE_VNORM   # VNorm without value norms in the cache
+    assert lib.raw_status("ikv_step", ctypes.byref(shp), ctypes.byref(p), ctypes.byref(cch), 16, 1, 16, 16, 16, 16,
+                          16, 1 << 40, None) == lib.IKV_ERR_ARG
+    assert lib.raw_status("ikv_value_norms", ctypes.byref(shp), ctypes.byref(cch), None) == lib.IKV_ERR_ARG
     nopos = _cache(lib, pos=0, dead_slots=1)
     n = lib.SZ(0)
     assert lib.raw_status("ikv_attend_workspace_size", ctypes.byref(shp), ctypes.byref(nopos),

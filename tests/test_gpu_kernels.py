@@ -280,6 +280,25 @@ def test_decode_attend_without_score_leaves_state():
         assert np.max(np.abs(out[b].float().cpu().numpy() - o)) < 2e-2
 
 
+def test_value_norms_match_numpy():
+    """ikv_value_norms: the l2 norm of every cached value row, through start and a permuted
+    block table, for both dtypes."""
+    for dt, d, ps in ((gen.BF16, 128, 64), (gen.F32, 64, 16)):
+        w = gen.Workload("n", 3, 2, 8, 4, d, [300, 1, 777], 1, dtype=dt, seed=27, page_size=ps)
+        u = w.u_table()
+        c = make_cache(w, page_perm_seed=3, value_norms=True)
+        fill_device(c, w, torch.from_numpy(u).cuda())
+        ikv.ikv_value_norms(c.shape(), c.cache(777))
+        torch.cuda.synchronize()
+        got = c.vnorm.cpu().numpy()
+        for b, L in enumerate(w.prefill):
+            for l in range(2):
+                _, v = w.kv_block(b, l, 0, L, u)
+                for g in range(4):
+                    want = np.sqrt(np.sum(v[g].astype(np.float64) ** 2, axis=1))
+                    assert np.max(np.abs(got[l, b, g, :L] - want) / want) < 1e-5
+
+
 def test_ema_update_matches_eq4():
     rng = np.random.default_rng(4)
     rows, cap = 5, 1000

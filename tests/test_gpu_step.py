@@ -126,3 +126,21 @@ def test_cumulative_and_single_step_aggregation():
     _assert(run_lockstep(small_llama(steps=6), agg_mode=single), 2e-2)
     _assert(run_lockstep(small_llama(steps=6), gran=ikv.IKV_GRAN_KVHEAD, agg_mode=single,
                          compact_mode=ikv.IKV_COMPACT_STABLE_SHORT), 2e-2)
+
+
+def test_vnorm_and_entropy_scorers():
+    """The Appendix's VNorm and entropy-weighted scorers in place of Eq. 1, in lock-step with
+    the oracle.  VNorm reads value-row norms that the append stores and the compaction moves
+    (stable, shorter-side, hole-fill and deferred), so the trajectories also check those."""
+    vn, ent = ikv.IKV_SCORE_VNORM, ikv.IKV_SCORE_ENTROPY
+    _assert(run_lockstep(gen.config(0), scorer=vn), 1e-4, strict_fraction=1.0)
+    _assert(run_lockstep(gen.config(0), scorer=ent), 1e-4, strict_fraction=1.0)
+    _assert(run_lockstep(small_llama(steps=8), scorer=vn), 2e-2)
+    _assert(run_lockstep(small_llama(steps=8, refresh_period=3), scorer=vn, compact_mode=ikv.IKV_COMPACT_STABLE_SHORT,
+                         max_holes=3), 2e-2)
+    _assert(run_lockstep(small_llama(steps=6), scorer=vn, gran=ikv.IKV_GRAN_KVHEAD,
+                         compact_mode=ikv.IKV_COMPACT_HOLEFILL), 2e-2)
+    _assert(run_lockstep(small_llama(steps=8), scorer=ent), 2e-2)
+    _assert(run_lockstep(small_llama(steps=8, score_free=True), scorer=ent, max_holes=4), 2e-2)
+    _assert(run_lockstep(small_llama(steps=6), scorer=ent, gran=ikv.IKV_GRAN_KVHEAD,
+                         agg_mode=ikv.IKV_AGG_CUMULATIVE), 2e-2)
