@@ -239,7 +239,7 @@ def setup(w, device, compact_mode):
 
     c = DecodeCache(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.cap,
                     dtype=ikv.IKV_BF16 if w.dtype == gen.BF16 else ikv.IKV_F32, page_size=w.page_size,
-                    device=device, page_perm_seed=1)
+                    device=device, page_perm_seed=1, value_norms=True)
     return c
 
 
@@ -256,10 +256,15 @@ def reset(c, w, u_dev):
                                                c.max_pages, max(w.prefill), w.dtype,
                                                torch.cuda.current_stream().cuda_stream)
     assert rc == 0
+    if c.vnorm is not None:  # value-row norms of the prefill, for the VNorm scorer
+        from paper_2609_03515_gb300 import ikv
+
+        ikv.ikv_value_norms(c.shape(), c.cache(max(w.prefill)))
     torch.cuda.synchronize()
 
 
-def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_detail: bool, dist, mh: int = 0):
+def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_detail: bool, dist, mh: int = 0,
+             scorer: int = 0):
     """Warm-up then K timed steps of one schedule, launched eagerly; returns a dict of
     measurements (with per-kernel CUDA-event times when want_detail)."""
     import torch
@@ -267,7 +272,7 @@ def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_d
     from paper_2609_03515_gb300 import ikv, step_lengths
 
     reset(c, w, u_dev)
-    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh, scorer=scorer)
     budgets = w.budgets()
     lens, live = list(w.prefill), list(w.prefill)
     out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=c.torch_dtype, device=c.k.device)
@@ -321,7 +326,7 @@ def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_d
 
 
 def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, sample_clocks: bool,
-                   mh: int = 0):
+                   mh: int = 0, scorer: int = 0):
     """The same schedule with each steady-state step replayed from a captured CUDA graph.
 
     After the eager warm-up (decode step 1 evicts ~90% of the prefill, later steps hold
@@ -333,7 +338,7 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     from paper_2609_03515_gb300 import ikv, step_lengths
 
     reset(c, w, u_dev)
-    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh, scorer=scorer)
     budgets = w.budgets()
     assert all(L0 >= B for L0, B in zip(w.prefill, budgets)), "graph replay assumes every sequence at its budget"
     lens, live = list(w.prefill), list(w.prefill)
@@ -392,7 +397,7 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     return res
 
 
-def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist, mh: int = 0):
+def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist, mh: int = 0, scorer: int = 0):
     """Same steps through the C ABI, inputs from pinned host memory and the output read back every step.
 
     Two buffer sets and a copy stream: the upload of step t+1's inputs and the read-back
@@ -403,7 +408,7 @@ def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist, mh: int
     from paper_2609_03515_gb300 import ikv, step_lengths
 
     reset(c, w, u_dev)
-    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh, scorer=scorer)
     budgets = w.budgets()
     lens, live = list(w.prefill), list(w.prefill)
     dev = c.k.device
@@ -540,25 +545,28 @@ def run_ours(args):
         full_w = w.with_(refresh_period=1, score_free=False)
         lazy_w = w.with_(refresh_period=4, score_free=False)
         sf_w = w.with_(refresh_period=1, score_free=True)
-        variants = (("full", full_w, compact_mode, mh),
-                    ("lazy4", lazy_w, compact_mode, mh),
-                    ("score_free", sf_w, compact_mode, mh),
-                    ("full_every_step", full_w, compact_mode, 0),
-                    ("lazy4_every_step", lazy_w, compact_mode, 0),
-                    ("score_free_every_step", sf_w, compact_mode, 0),
-                    ("full_stable_left", full_w, ikv.IKV_COMPACT_STABLE, 0),
-                    ("full_holefill", full_w, ikv.IKV_COMPACT_HOLEFILL, 0),
-                    ("lazy4_holefill", lazy_w, ikv.IKV_COMPACT_HOLEFILL, 0),
-                    ("score_free_holefill", sf_w, ikv.IKV_COMPACT_HOLEFILL, 0))
-        for name, ww, cm, vmh in variants:
-            if name == head_sched and cm == compact_mode and vmh == mh:
+        att, vnm, ent = ikv.IKV_SCORE_ATTENTION, ikv.IKV_SCORE_VNORM, ikv.IKV_SCORE_ENTROPY
+        variants = (("full", full_w, compact_mode, mh, att),
+                    ("lazy4", lazy_w, compact_mode, mh, att),
+                    ("score_free", sf_w, compact_mode, mh, att),
+                    ("full_vnorm", full_w, compact_mode, mh, vnm),
+                    ("full_entropy", full_w, compact_mode, mh, ent),
+                    ("full_every_step", full_w, compact_mode, 0, att),
+                    ("lazy4_every_step", lazy_w, compact_mode, 0, att),
+                    ("score_free_every_step", sf_w, compact_mode, 0, att),
+                    ("full_stable_left", full_w, ikv.IKV_COMPACT_STABLE, 0, att),
+                    ("full_holefill", full_w, ikv.IKV_COMPACT_HOLEFILL, 0, att),
+                    ("lazy4_holefill", lazy_w, ikv.IKV_COMPACT_HOLEFILL, 0, att),
+                    ("score_free_holefill", sf_w, ikv.IKV_COMPACT_HOLEFILL, 0, att))
+        for name, ww, cm, vmh, sc in variants:
+            if name == head_sched and cm == compact_mode and vmh == mh and sc == att:
                 modes[name] = full           # the headline run is this mode
                 continue
-            modes[name] = run_mode_graph(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, dist, False, vmh)
+            modes[name] = run_mode_graph(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, dist, False, vmh, sc)
         if args.mode_kernels:
-            for name, ww, cm, vmh in variants:
+            for name, ww, cm, vmh, sc in variants:
                 mode_kernels[name] = run_mode(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, True, dist,
-                                              vmh)["kernel_ms"]
+                                              vmh, sc)["kernel_ms"]
     qs_pin = qs_t.pin_memory()
     kn_pin = kn_dev.cpu().pin_memory()
     vn_pin = vn_dev.cpu().pin_memory()
@@ -623,7 +631,8 @@ def run_ours(args):
         if mode_kernels:
             line["mode_kernel_ms_per_step"] = mode_kernels
         line["modes_note"] = ("full / lazy4 / score_free: refresh every step / every 4th step (Eq. 6) / step 1 "
-                              "only, same inputs and compaction as the headline; *_every_step: the same "
+                              "only, same inputs and compaction as the headline; full_vnorm / full_entropy: the "
+                              "VNorm and entropy-weighted scorers under full refresh; *_every_step: the same "
                               "compaction run on every eviction (max_holes 0); full_stable_left: stable "
                               "compaction that always shifts the suffix left, every step; *_holefill: hole-fill "
                               "compaction every step (same kept sets, survivors not kept in order)")

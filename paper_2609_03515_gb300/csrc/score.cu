@@ -47,6 +47,7 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
     constexpr int kTok = 32 * V;   // tokens per CTA
     constexpr int kHB = 32 / V;    // heads per load batch (32 registers of loads)
     __shared__ __align__(16) float sl[kMaxLayersPerScorePass][kTok];
+    extern __shared__ float wsm[];  // VNorm: per warp, [row's kv heads][kTok] value-norm weights
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int r = blockIdx.y;
     const int b = r / a.rows_per_seq;
@@ -71,6 +72,20 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
         // row padding keeps i0 + kTok <= lstride, so the vector loads stay inside the row
         const float *zp = a.logits + (((int64_t)b * a.n_layers + li) * H + h0) * (int64_t)a.lstride + il;
         const float *ll = a.lse2 + ((int64_t)b * a.n_layers + li) * H + h0;
+        const int g0 = h0 / G, ng = (nh + G - 1) / G;  // the row's kv heads
+        float *wv = wsm + (size_t)warp * ng * kTok;
+        if (SCORER == IKV_SCORE_VNORM) {
+            // every weight this warp needs, in one batch of loads: norm over the unit's mean norm
+            for (int gg = 0; gg < ng; ++gg) {
+                const int g = g0 + gg;
+                const float mean = a.vmean[((int64_t)b * a.n_layers + li) * a.kv_heads + g];
+                const float *vn = a.vnorm + (((int64_t)(a.layer0 + li) * a.batch + b) * a.kv_heads + g) * a.cap;
+#pragma unroll
+                for (int v = 0; v < V; ++v)
+                    wv[gg * kTok + lane * V + v] = mean > 0.f ? (il + v < L ? __ldg(vn + il + v) : 0.f) / mean : 1.f;
+            }
+            __syncwarp();
+        }
         float acc[V];
 #pragma unroll
         for (int v = 0; v < V; ++v) acc[v] = 0.f;
@@ -91,14 +106,9 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
 #pragma unroll
                     for (int v = 0; v < V; ++v) w[v] = 1.f;
                     if (SCORER == IKV_SCORE_VNORM) {
-                        // value-norm weight of this head's KV head: norm over the unit's mean norm
-                        const int g = (h0 + hb + j) / G;
-                        const int64_t u = ((int64_t)b * a.n_layers + li) * a.kv_heads + g;
-                        const float mean = a.vmean[u];
-                        const float *vn = a.vnorm + (((int64_t)(a.layer0 + li) * a.batch + b) * a.kv_heads + g) * a.cap;
+                        const float *wg = wv + ((h0 + hb + j) / G - g0) * kTok + lane * V;
 #pragma unroll
-                        for (int v = 0; v < V; ++v)
-                            w[v] = mean > 0.f ? (il + v < L ? __ldg(vn + il + v) : 0.f) / mean : 1.f;
+                        for (int v = 0; v < V; ++v) w[v] = wg[v];
                     }
 #pragma unroll
                     for (int v = 0; v < V; ++v) acc[v] += exp2f(vget(z[j], v) - lj) * w[v];
@@ -182,8 +192,14 @@ __global__ void __launch_bounds__(kFoldThreads) entropy_fold_kernel(const ScoreA
     if (i >= L) return;
     const int64_t at = (int64_t)r * a.cap + i;
     float m = a.ema[at];
-    for (int k = 0; k < NE; ++k)
-        m = aggregate(m, wk[k] * a.sbuf[((int64_t)r * NE + k) * a.lstride + i], a.agg, a.alpha);
+    for (int k0 = 0; k0 < NE; k0 += 16) {  // 16 layers' scores in flight, then folded in order
+        float sv[16];
+#pragma unroll
+        for (int u = 0; u < 16; ++u) sv[u] = k0 + u < NE ? a.sbuf[((int64_t)r * NE + k0 + u) * a.lstride + i] : 0.f;
+#pragma unroll
+        for (int u = 0; u < 16; ++u)
+            if (k0 + u < NE) m = aggregate(m, wk[k0 + u] * sv[u], a.agg, a.alpha);
+    }
     a.ema[at] = m;
 }
 
@@ -248,22 +264,41 @@ __global__ void value_norms_kernel(const T *v, PagedView pv, const int32_t *len,
 
 }  // namespace
 
+// VNorm weight staging: per warp, one kTok-token row per kv head of the utility row
+static size_t vnorm_smem(const ScoreArgs &a, int V) {
+    const int ng = a.rows_per_seq > 1 ? 1 : a.kv_heads;
+    return (size_t)kScoreWarps * ng * 32 * V * sizeof(float);
+}
+constexpr size_t kVnormSmemMax = 160 * 1024;
+
 int score_blocks(const ScoreArgs &a, int32_t max_len, int sms, int *V) {
     // widest token vector that still gives every SM two CTAs
     const int64_t rows = (int64_t)a.batch * a.rows_per_seq;
     auto ctas = [&](int tok) { return rows * ((max_len + tok - 1) / tok); };
-    *V = ctas(128) >= 2 * sms ? 4 : ctas(64) >= 2 * sms ? 2 : 1;
-    return (max_len + 32 * *V - 1) / (32 * *V);
+    int v = ctas(128) >= 2 * sms ? 4 : ctas(64) >= 2 * sms ? 2 : 1;
+    if (a.scorer == IKV_SCORE_VNORM)  // the weight staging must fit in shared memory
+        while (v > 1 && vnorm_smem(a, v) > kVnormSmemMax) v >>= 1;
+    *V = v;
+    return (max_len + 32 * v - 1) / (32 * v);
+}
+
+template <int V, int SCORER>
+static cudaError_t launch_score_v(const ScoreArgs &a, dim3 grid, cudaStream_t st) {
+    const size_t smem = SCORER == IKV_SCORE_VNORM ? vnorm_smem(a, V) : 0;
+    if (smem > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(score_kernel<V, SCORER>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)smem);
+        if (e != cudaSuccess) return e;
+    }
+    score_kernel<V, SCORER><<<grid, kScoreWarps * 32, smem, st>>>(a);
+    return cudaSuccess;
 }
 
 template <int SCORER>
-static void launch_score_t(const ScoreArgs &a, dim3 grid, int V, cudaStream_t st) {
-    if (V == 4)
-        score_kernel<4, SCORER><<<grid, kScoreWarps * 32, 0, st>>>(a);
-    else if (V == 2)
-        score_kernel<2, SCORER><<<grid, kScoreWarps * 32, 0, st>>>(a);
-    else
-        score_kernel<1, SCORER><<<grid, kScoreWarps * 32, 0, st>>>(a);
+static cudaError_t launch_score_t(const ScoreArgs &a, dim3 grid, int V, cudaStream_t st) {
+    if (V == 4) return launch_score_v<4, SCORER>(a, grid, st);
+    if (V == 2) return launch_score_v<2, SCORER>(a, grid, st);
+    return launch_score_v<1, SCORER>(a, grid, st);
 }
 
 cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, int sms, cudaStream_t st) {
@@ -271,12 +306,14 @@ cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, int sms, cudaS
     int V = 1;
     const int nblk = score_blocks(a, max_len, sms, &V);
     dim3 grid(nblk, (unsigned)(a.batch * a.rows_per_seq));
+    cudaError_t e;
     if (a.scorer == IKV_SCORE_VNORM)
-        launch_score_t<IKV_SCORE_VNORM>(a, grid, V, st);
+        e = launch_score_t<IKV_SCORE_VNORM>(a, grid, V, st);
     else if (a.scorer == IKV_SCORE_ENTROPY)
-        launch_score_t<IKV_SCORE_ENTROPY>(a, grid, V, st);
+        e = launch_score_t<IKV_SCORE_ENTROPY>(a, grid, V, st);
     else
-        launch_score_t<IKV_SCORE_ATTENTION>(a, grid, V, st);
+        e = launch_score_t<IKV_SCORE_ATTENTION>(a, grid, V, st);
+    if (e != cudaSuccess) return e;
     note_launch();
     return cudaGetLastError();
 }
