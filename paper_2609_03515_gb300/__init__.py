@@ -14,7 +14,19 @@ import torch
 
 from . import ikv
 
-__all__ = ["ikv", "DecodeCache", "step_lengths"]
+__all__ = ["ikv", "DecodeCache", "step_lengths", "auto_max_holes"]
+
+
+def auto_max_holes(budgets: Sequence[int]) -> int:
+    """A deferred-compaction threshold (ikv_params.max_holes) for sequences with these
+    budgets.  Holding on average max_holes / 2 dead slots makes the attention read that
+    many masked rows per step, and one compaction of about B rows (read + write) is
+    spread over max_holes steps; max_holes / 2 + 2 B / max_holes is smallest at
+    max_holes = 2 sqrt(B).  Rounded to a multiple of 8, at least 8."""
+    import math
+
+    b = sum(budgets) / max(1, len(budgets))
+    return max(8, int(round(2 * math.sqrt(b) / 8)) * 8)
 
 
 def step_lengths(lens: Sequence[int], live: Sequence[int], budgets: Sequence[int], max_holes: int = 0):

@@ -119,6 +119,18 @@ def test_deferred_compaction_arguments(lib):
                           ctypes.byref(n)) == lib.IKV_ERR_ARG
 
 
+def test_auto_max_holes():
+    """The deferred-compaction threshold minimises masked reads plus amortised compaction."""
+    from paper_2609_03515_gb300 import auto_max_holes
+    import math
+    for b in (51, 615, 1638, 3277, 6554):
+        mh = auto_max_holes([b])
+        assert mh % 8 == 0 and mh >= 8
+        cost = lambda m: m / 2 + 2 * b / m
+        assert cost(mh) <= 1.05 * cost(2 * math.sqrt(b))   # within 5 % of the continuous optimum
+    assert auto_max_holes([3277]) == 112 and auto_max_holes([6554]) == 160
+
+
 def test_step_lengths_mirror():
     """Host bookkeeping of len (dead slots included) and live slots across steps."""
     from paper_2609_03515_gb300 import step_lengths

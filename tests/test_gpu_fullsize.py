@@ -26,12 +26,17 @@ def _check(reps):
 
 # The benchmark's configuration: shorter-side stable compaction, deferred while a
 # sequence holds at most 128 dead slots.
-SHORT, BENCH_HOLES = ikv.IKV_COMPACT_STABLE_SHORT, 128
+SHORT = ikv.IKV_COMPACT_STABLE_SHORT
+
+
+def bench_holes(w):
+    return 128
 
 
 @pytest.mark.timeout(1200)
 def test_config1_llama_b1_32k_full_refresh():
-    _check(run_fullsize_sampled(gen.config(1), seqs=[0], steps=4, compact_mode=SHORT, max_holes=BENCH_HOLES))
+    w = gen.config(1)
+    _check(run_fullsize_sampled(w, seqs=[0], steps=4, compact_mode=SHORT, max_holes=bench_holes(w)))
 
 
 @pytest.mark.timeout(1200)
@@ -43,19 +48,21 @@ def test_config1_deferred_compaction_crossing():
 @pytest.mark.timeout(1200)
 def test_config2_llama_b16_ragged_lazy4():
     # steps 1 and 5 refresh, 2-4 carry the state (Eq. 6); two of the sixteen sequences followed
-    _check(run_fullsize_sampled(gen.config(2), seqs=[0, 11], steps=5, compact_mode=SHORT, max_holes=BENCH_HOLES))
+    w = gen.config(2)
+    _check(run_fullsize_sampled(w, seqs=[0, 11], steps=5, compact_mode=SHORT, max_holes=bench_holes(w)))
 
 
 @pytest.mark.timeout(1200)
 def test_config3_llama_b8_64k_score_free():
-    _check(run_fullsize_sampled(gen.config(3), seqs=[5], steps=3, compact_mode=SHORT, max_holes=BENCH_HOLES))
+    w = gen.config(3)
+    _check(run_fullsize_sampled(w, seqs=[5], steps=3, compact_mode=SHORT, max_holes=bench_holes(w)))
 
 
 @pytest.mark.timeout(1200)
 def test_config4_qwen_b32_16k_sweep_point():
     # one point of the sweep: budget 25%, alpha 0.5, Lazy refresh period 2
     w = gen.config(4).with_(budget_frac=0.25, alpha=0.5, refresh_period=2)
-    _check(run_fullsize_sampled(w, seqs=[31], steps=3, compact_mode=SHORT, max_holes=BENCH_HOLES))
+    _check(run_fullsize_sampled(w, seqs=[31], steps=3, compact_mode=SHORT, max_holes=bench_holes(w)))
 
 
 @pytest.mark.timeout(1200)
