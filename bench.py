@@ -335,9 +335,9 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     """The same schedule with each steady-state step replayed from a captured CUDA graph.
 
     After the eager warm-up (decode step 1 evicts ~90% of the prefill, later steps hold
-    the budget), one graph per step kind (refresh / carry-over, Eq. 6) is captured
-    around ikv_step with fixed input buffers; every timed step copies its inputs into
-    those buffers (one device-to-device copy each) and replays the graph of its kind."""
+    the budget), one graph per timed step t is captured around ikv_step(t) with that
+    step's resident inputs (q, k_new, v_new of step t), so replaying it does exactly what
+    the eager call would, with no staging copies; the timed region replays them in order."""
     import torch
 
     from paper_2609_03515_gb300 import ikv, step_lengths
@@ -349,32 +349,24 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     lens, live = list(w.prefill), list(w.prefill)
     dev = c.k.device
     out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=c.torch_dtype, device=dev)
-    q_buf, kn_buf, vn_buf = torch.empty_like(qs_dev[0]), torch.empty_like(kn_dev[0]), torch.empty_like(vn_dev[0])
     W, K = args.warmup, args.steps
     for t in range(1, W + 1):
         ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws,
                      ws.numel(), torch.cuda.current_stream())
         lens, live = step_lengths(lens, live, budgets, mh)
     torch.cuda.synchronize()
-    # one graph serves every later step, so its max_len bounds them all: the budget plus
-    # the dead slots deferred compaction may hold
+    # the graphs' max_len bounds every later step: the budget plus the dead slots
+    # deferred compaction may hold
     steady = c.cache(min(c.cap - 1, max(max(lens), max(budgets) + mh)))
-
-    def refresh(t):
-        return t == 1 if w.score_free else (t - 1) % w.refresh_period == 0
-
-    graphs = {}
+    graphs = []
     n0 = ikv.ikv_launch_count()
     for i in range(K):
         t = W + 1 + i
-        kind = refresh(t)
-        if kind in graphs:
-            continue
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, capture_error_mode="thread_local"):
-            ikv.ikv_step(c.shape(), p, steady, c.ema, t, q_buf, kn_buf, vn_buf, out, ws, ws.numel(),
-                         torch.cuda.current_stream())
-        graphs[kind] = (g, ikv.ikv_launch_count() - n0)
+            ikv.ikv_step(c.shape(), p, steady, c.ema, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws,
+                         ws.numel(), torch.cuda.current_stream())
+        graphs.append((g, ikv.ikv_launch_count() - n0))
         n0 = ikv.ikv_launch_count()
     torch.cuda.synchronize()
     stream = torch.cuda.current_stream()
@@ -385,12 +377,7 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     clocks = ClockSampler(torch.cuda.current_device()) if sample_clocks else None
     launches = 0
     start.record(stream)
-    for i in range(K):
-        t = W + 1 + i
-        q_buf.copy_(qs_dev[t - 1], non_blocking=True)
-        kn_buf.copy_(kn_dev[t - 1], non_blocking=True)
-        vn_buf.copy_(vn_dev[t - 1], non_blocking=True)
-        g, nl = graphs[refresh(t)]
+    for g, nl in graphs:
         g.replay()
         launches += nl
     stop.record(stream)
@@ -405,8 +392,8 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
 def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist, mh: int = 0, scorer: int = 0):
     """Same steps through the C ABI, inputs from pinned host memory and the output read back every step.
 
-    Two buffer sets and a copy stream: the upload of step t+1's inputs and the read-back
-    of step t-1's output run while step t computes.  Every step's copies lie inside the
+    Two buffer sets and one copy stream per direction: the upload of step t+1's inputs
+    and the read-back of step t-1's output run while step t computes.  Every step's copies lie inside the
     timed region (the compute stream waits for the copy stream before the stop event).
     After the eager warm-up, each timed step replays ikv_step from a CUDA graph captured
     for its kind (refresh / carry-over) and buffer set, so a stall of the host thread does
@@ -427,41 +414,48 @@ def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist, mh: int
     out_d = [torch.empty(oshape, dtype=c.torch_dtype, device=dev) for _ in range(2)]
     out_h = [torch.empty(oshape, dtype=c.torch_dtype, pin_memory=True) for _ in range(2)]
     comp = torch.cuda.current_stream()
-    cs = torch.cuda.Stream(device=dev)
+    up = torch.cuda.Stream(device=dev)    # host -> device uploads
+    down = torch.cuda.Stream(device=dev)  # device -> host read-backs (a separate copy engine)
     in_ready = [torch.cuda.Event() for _ in range(2)]
     done = [torch.cuda.Event() for _ in range(2)]
+    read = [torch.cuda.Event() for _ in range(2)]
 
     def upload(t):
         i = t % 2
-        with torch.cuda.stream(cs):
+        with torch.cuda.stream(up):
             q_d[i].copy_(qs_h[t - 1], non_blocking=True)
             kn_d[i].copy_(kn_h[t - 1], non_blocking=True)
             vn_d[i].copy_(vn_h[t - 1], non_blocking=True)
-            in_ready[i].record(cs)
+            in_ready[i].record(up)
 
     def run(t0, n):
         """Steps t0 .. t0+n-1; the upload of t0 is issued here, the last read-back is waited for."""
         nonlocal lens, live
-        cs.wait_stream(comp)
+        up.wait_stream(comp)
+        down.wait_stream(comp)
         upload(t0)
         for t in range(t0, t0 + n):
             i = t % 2
             if t + 1 < t0 + n:
                 if t + 1 >= t0 + 2:
-                    cs.wait_event(done[(t + 1) % 2])   # step t-1 has read the buffers step t+1 reuses
+                    up.wait_event(done[(t + 1) % 2])   # step t-1 has read the buffers step t+1 reuses
                 upload(t + 1)
             comp.wait_event(in_ready[i])
+            if t >= t0 + 2:
+                comp.wait_event(read[i])             # step t-2's output has been read back
             if graphs:
                 graphs[(refresh(t), i)].replay()
             else:
                 ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, q_d[i], kn_d[i], vn_d[i], out_d[i], ws,
                              ws.numel(), comp)
             done[i].record(comp)
-            with torch.cuda.stream(cs):
-                cs.wait_event(done[i])
+            with torch.cuda.stream(down):
+                down.wait_event(done[i])
                 out_h[i].copy_(out_d[i], non_blocking=True)
+                read[i].record(down)
             lens, live = step_lengths(lens, live, budgets, mh)
-        comp.wait_stream(cs)
+        comp.wait_stream(up)
+        comp.wait_stream(down)
 
     def refresh(t):
         return t == 1 if w.score_free else (t - 1) % w.refresh_period == 0
@@ -601,11 +595,11 @@ def run_ours(args):
     qs_pin = qs_t.pin_memory()
     kn_pin = kn_dev.cpu().pin_memory()
     vn_pin = vn_dev.cpu().pin_memory()
-    # three complete end-to-end runs, median reported: host-link bandwidth on the shared
+    # five complete end-to-end runs, median reported: host-link bandwidth on the shared
     # machine varies from run to run
-    e2e_runs = [run_e2e(args, w, c, u_dev, ws, compact_mode, qs_pin, kn_pin, vn_pin, dist, mh) for _ in range(3)]
+    e2e_runs = [run_e2e(args, w, c, u_dev, ws, compact_mode, qs_pin, kn_pin, vn_pin, dist, mh) for _ in range(5)]
     e2e_all = sorted(r[0] for r in e2e_runs)
-    e2e_ms, h2d, d2h = e2e_all[1], e2e_runs[0][1], e2e_runs[0][2]
+    e2e_ms, h2d, d2h = e2e_all[2], e2e_runs[0][1], e2e_runs[0][2]
 
     K = args.steps
     value = job_throughput(w.batch * K, world, full["ms"])
@@ -644,7 +638,7 @@ def run_ours(args):
                    "kv_heads": w.kv_heads, "head_dim": w.head_dim, "prefill": w.prefill[0] if w.batch == 1 else w.prefill,
                    "budget": w.budgets(), "alpha": w.alpha, "refresh": head_sched, "compaction": args.compact, "max_holes": mh,
                    "timed_steps": f"decode steps {args.warmup + 1}..{args.warmup + K} (steady state; step 1 in warm-up)",
-                   "launch": "CUDA graph per step kind, inputs staged by one device copy each",
+                   "launch": "one CUDA graph per timed step, captured on that step's resident inputs",
                    "l2": l2_note,
                    "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
@@ -656,7 +650,7 @@ def run_ours(args):
         "cpu_baseline": cpu,
         "e2e": {"value": w.batch * K * world / (e2e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "runs": [w.batch * K * world / (m / 1e3) for m in e2e_all],
-                "note": "median of three runs; inputs uploaded from pinned host memory and outputs read back "
+                "note": "median of five runs; inputs uploaded from pinned host memory and outputs read back "
                         "every step, overlapped with the previous / next step's compute"},
         "gpu_launches": full["launches"],
         "clocks": full["clocks"],

@@ -5,12 +5,17 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <optional>
 
 #include "ikv_internal.cuh"
 
 namespace ikv {
 
 static std::atomic<int64_t> g_launches{0};
+static thread_local int g_pdl = 0;
+bool pdl_enabled() { return g_pdl > 0; }
+PdlScope::PdlScope() { ++g_pdl; }
+PdlScope::~PdlScope() { --g_pdl; }
 void note_launch(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 
 namespace {
@@ -586,6 +591,10 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     if ((e = append_impl(shape, cache, k_new, v_new, ema, init_mean, at<int32_t>(ws, w.done), stream, true)))
         return e;
     if (tm && (e = record(tm->append_end, stream))) return e;
+    // the rest of the chain may overlap each kernel's ramp-up with its predecessor's tail
+    // (not when per-kernel events are recorded: those time each kernel alone)
+    std::optional<PdlScope> pdl;
+    if (!tm) pdl.emplace();
     if ((e = run_attend(shape, cache, 0, shape->layers, L1, q, out, ws, w.at, scoring, nullptr, nullptr, stream, tm,
                         true)))
         return e;

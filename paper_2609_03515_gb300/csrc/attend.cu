@@ -104,6 +104,7 @@ struct AttendCfg {
 template <typename T, int D, int G, bool LOGITS>
 __global__ void __launch_bounds__(kAttendThreads, 2) attend_split_kernel(const AttendArgs a) {
     using C = AttendCfg<T, D, G>;
+    pdl_wait();
     extern __shared__ __align__(128) unsigned char smem[];
     float *fs = reinterpret_cast<float *>(smem + C::kStageArea);
     float *q_s = fs + C::kQ;
@@ -310,6 +311,7 @@ __global__ void __launch_bounds__(kAttendThreads, 2) attend_split_kernel(const A
 
 template <typename T>
 __global__ void __launch_bounds__(128) combine_kernel(const CombineArgs a) {
+    pdl_wait();
     const int h = blockIdx.x;
     const int b = blockIdx.y % a.batch, li = blockIdx.y / a.batch;
     const int D = a.head_dim;
@@ -341,12 +343,12 @@ cudaError_t launch_attend_t(const AttendArgs &a, cudaStream_t st) {
         auto k = attend_split_kernel<T, D, G, true>;
         cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
         if (e != cudaSuccess) return e;
-        k<<<grid, kAttendThreads, C::kSmemBytes, st>>>(a);
+        { cudaError_t le = launch_k(k, grid, dim3(kAttendThreads), C::kSmemBytes, st, a); if (le != cudaSuccess) return le; }
     } else {
         auto k = attend_split_kernel<T, D, G, false>;
         cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
         if (e != cudaSuccess) return e;
-        k<<<grid, kAttendThreads, C::kSmemBytes, st>>>(a);
+        { cudaError_t le = launch_k(k, grid, dim3(kAttendThreads), C::kSmemBytes, st, a); if (le != cudaSuccess) return le; }
     }
     note_launch();
     return cudaGetLastError();
@@ -380,9 +382,9 @@ cudaError_t launch_attend(const AttendArgs &a, int dtype, int head_dim, int grou
 cudaError_t launch_combine(const CombineArgs &a, int dtype, cudaStream_t st) {
     dim3 grid(a.q_heads, a.batch * a.n_layers);
     if (dtype == IKV_BF16)
-        combine_kernel<__nv_bfloat16><<<grid, 128, 0, st>>>(a);
+        { cudaError_t le = launch_k(combine_kernel<__nv_bfloat16>, grid, dim3(128), 0, st, a); if (le != cudaSuccess) return le; }
     else
-        combine_kernel<float><<<grid, 128, 0, st>>>(a);
+        { cudaError_t le = launch_k(combine_kernel<float>, grid, dim3(128), 0, st, a); if (le != cudaSuccess) return le; }
     note_launch();
     return cudaGetLastError();
 }

@@ -190,6 +190,7 @@ template <int G>
 __global__ void __launch_bounds__(kThreads, 2)
     attend_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, const TcArgs a) {
     constexpr int NC = G <= 4 ? 4 : 8;  // TMEM columns read per S tile
+    pdl_wait();
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -565,8 +566,7 @@ cudaError_t launch_tc_g(const CUtensorMap &mk, const CUtensorMap &mv, const TcAr
         if (e != cudaSuccess) return e;
         attr = true;
     }
-    attend_tc_kernel<G><<<grid, kThreads, kSmemBytes, st>>>(mk, mv, t);
-    return cudaGetLastError();
+    return launch_k(attend_tc_kernel<G>, grid, dim3(kThreads), kSmemBytes, st, mk, mv, t);
 }
 
 }  // namespace

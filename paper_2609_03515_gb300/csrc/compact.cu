@@ -113,6 +113,7 @@ __device__ __forceinline__ void mark_dead_row(const CompactArgs &a, int r, int L
 // sequence b reads len[b] and start[b] first; the last CTA of b to arrive writes
 // the new values, so no CTA sees them early.
 __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const CompactArgs a) {
+    pdl_wait();
     extern __shared__ __align__(16) unsigned char cbuf[];
     __shared__ int scratch[32];
     const int tid = threadIdx.x;
@@ -274,6 +275,7 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
 constexpr int kPlanThreads = 1024;
 
 __global__ void __launch_bounds__(kPlanThreads) holefill_plan_kernel(const CompactArgs a) {
+    pdl_wait();
     __shared__ int below_s;
     const int r = blockIdx.x;
     const int n = a.keep_len[r];
@@ -310,6 +312,7 @@ __global__ void __launch_bounds__(kPlanThreads) holefill_plan_kernel(const Compa
 }
 
 __global__ void __launch_bounds__(kCompThreads) holefill_move_kernel(const CompactArgs a) {
+    pdl_wait();
     const int tid = threadIdx.x;
     const int b = blockIdx.y, x = blockIdx.x;
     const int kvh = a.pv.kv_heads;
@@ -369,6 +372,7 @@ __device__ unsigned int g_append_error = 0;  // bit 0: an append found no free s
 namespace {
 
 __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a) {
+    pdl_wait();
     __shared__ float scratch[32];
     const int tid = threadIdx.x;
     const int b = blockIdx.y;
@@ -464,15 +468,16 @@ cudaError_t launch_compact(const CompactArgs &a, int mode, cudaStream_t st) {
             if (e != cudaSuccess) return e;
             attr_smem = smem;
         }
-        compact_stable_kernel<<<grid, kCompThreads, smem, st>>>(a);
+        cudaError_t e = launch_k(compact_stable_kernel, grid, dim3(kCompThreads), smem, st, a);
         note_launch();
-        return cudaGetLastError();
+        return e != cudaSuccess ? e : cudaGetLastError();
     }
-    holefill_plan_kernel<<<a.batch * a.rows_per_seq, kPlanThreads, 0, st>>>(a);
+    cudaError_t e = launch_k(holefill_plan_kernel, dim3(a.batch * a.rows_per_seq), dim3(kPlanThreads), 0, st, a);
     note_launch();
-    holefill_move_kernel<<<grid, kCompThreads, 0, st>>>(a);
+    if (e != cudaSuccess) return e;
+    e = launch_k(holefill_move_kernel, grid, dim3(kCompThreads), 0, st, a);
     note_launch();
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t read_clear_append_error(unsigned int *v) {

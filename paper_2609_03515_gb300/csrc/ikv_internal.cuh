@@ -22,6 +22,40 @@ void note_launch(int n = 1);
 // Set the thread's ikv_last_error() message and return `s` (host).
 ikv_status report(ikv_status s, const char *fmt, ...);
 
+// Programmatic dependent launch.  While a PdlScope is alive on the issuing thread
+// (ikv_step, for the kernels after its first), kernels are launched with programmatic
+// stream serialisation: each may be scheduled while its predecessor drains.  Every
+// kernel of the library starts with pdl_wait() -- which returns once all predecessor
+// grids have completed and their memory is visible, and is a no-op for a normal launch
+// -- before it reads or writes anything, then lets its own dependents be scheduled.
+bool pdl_enabled();
+struct PdlScope {
+    PdlScope();
+    ~PdlScope();
+};
+__device__ __forceinline__ void pdl_wait() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+template <typename... KArgs, typename... Args>
+cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args... args) {
+    if (!pdl_enabled()) {
+        kernel<<<grid, block, smem, st>>>(args...);
+        return cudaGetLastError();
+    }
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // Where a (sequence, slot) row of layer l / kv head g lives in the paged pool.
 // Logical slot j of sequence b is physical slot start[b] + j of its slot space
 // [0, cap); physical slot p lives in page block_table[b][p / page_size].

@@ -44,6 +44,7 @@ __device__ __forceinline__ float warp_sum(float v) {
 template <int V, int SCORER>
 __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreArgs a) {
     using VT = typename VecF<V>::T;
+    pdl_wait();
     constexpr int kTok = 32 * V;   // tokens per CTA
     constexpr int kHB = 32 / V;    // heads per load batch (32 registers of loads)
     __shared__ __align__(16) float sl[kMaxLayersPerScorePass][kTok];
@@ -164,6 +165,7 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
 // layer-sequential fold of w_k s_k(i) for this CTA's tokens.
 constexpr int kFoldThreads = 256;
 __global__ void __launch_bounds__(kFoldThreads) entropy_fold_kernel(const ScoreArgs a) {
+    pdl_wait();
     __shared__ float wk[kMaxLayers];
     __shared__ float n_live;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -206,6 +208,7 @@ __global__ void __launch_bounds__(kFoldThreads) entropy_fold_kernel(const ScoreA
 // Mean value-row norm of every (sequence, layer, kv head) over its live slots.
 constexpr int kMeanThreads = 256;
 __global__ void __launch_bounds__(kMeanThreads) vnorm_mean_kernel(const ScoreArgs a) {
+    pdl_wait();
     __shared__ float red[2][kMeanThreads / 32];
     const int u = blockIdx.x;  // (b * n_layers + li) * kv_heads + g
     const int g = u % a.kv_heads, li = (u / a.kv_heads) % a.n_layers, b = u / a.kv_heads / a.n_layers;
@@ -290,8 +293,7 @@ static cudaError_t launch_score_v(const ScoreArgs &a, dim3 grid, cudaStream_t st
                                              (int)smem);
         if (e != cudaSuccess) return e;
     }
-    score_kernel<V, SCORER><<<grid, kScoreWarps * 32, smem, st>>>(a);
-    return cudaSuccess;
+    return launch_k(score_kernel<V, SCORER>, grid, dim3(kScoreWarps * 32), smem, st, a);
 }
 
 template <int SCORER>
@@ -321,17 +323,17 @@ cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, int sms, cudaS
 cudaError_t launch_entropy_fold(const ScoreArgs &a, int32_t max_len, cudaStream_t st) {
     if (max_len <= 0 || a.n_elig_total <= 0) return cudaSuccess;
     dim3 grid((max_len + kFoldThreads - 1) / kFoldThreads, (unsigned)(a.batch * a.rows_per_seq));
-    entropy_fold_kernel<<<grid, kFoldThreads, 0, st>>>(a);
+    cudaError_t e = launch_k(entropy_fold_kernel, grid, dim3(kFoldThreads), 0, st, a);
     note_launch();
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_vnorm_mean(const ScoreArgs &a, cudaStream_t st) {
     const int units = a.batch * a.n_layers * a.kv_heads;
     if (units <= 0) return cudaSuccess;
-    vnorm_mean_kernel<<<units, kMeanThreads, 0, st>>>(a);
+    cudaError_t e = launch_k(vnorm_mean_kernel, dim3(units), dim3(kMeanThreads), 0, st, a);
     note_launch();
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_value_norms(const void *v, const PagedView &pv, const int32_t *len, int32_t batch, int32_t layers,

@@ -59,6 +59,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(int32_t cap, const 
                                                               const int32_t *__restrict__ len, int32_t rps,
                                                               const int32_t *__restrict__ budget, int32_t *pos,
                                                               int32_t *keep, int32_t *keep_len, DeferArgs df) {
+    pdl_wait();
     __shared__ uint32_t hist[256];
     __shared__ uint32_t warp_tot[32];
     __shared__ unsigned long long s_min[32];
@@ -231,7 +232,9 @@ cudaError_t launch_select(int32_t rows, int32_t cap, const float *util, const in
                           const int32_t *budget, int32_t *pos, int32_t *keep, int32_t *keep_len, const DeferArgs &df,
                           cudaStream_t st) {
     if (rows <= 0) return cudaSuccess;
-    select_kernel<<<rows, kSelThreads, 0, st>>>(cap, util, len, rows_per_seq, budget, pos, keep, keep_len, df);
+    cudaError_t e = launch_k(select_kernel, dim3(rows), dim3(kSelThreads), 0, st, cap, util, len, rows_per_seq, budget,
+                             pos, keep, keep_len, df);
+    if (e != cudaSuccess) return e;
     note_launch();
     return cudaGetLastError();
 }
