@@ -83,7 +83,7 @@ def rank_seed(base_seed: int, rank: int) -> int:
 
 
 # revision of each attention kernel; a committed ncu summary counts only for its own revision
-ATTEND_KERNEL_REV = {"attend_tc_kernel": "attend_tc_v3", "attend_split_kernel": "attend_split_v2"}
+ATTEND_KERNEL_REV = {"attend_tc_kernel": "attend_tc_v5", "attend_split_kernel": "attend_split_v2"}
 
 
 def schedule_name(w) -> str:
@@ -330,14 +330,34 @@ def run_mode(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, want_d
     return res
 
 
+def split_step(c, p, cache, t, q, kn, vn, out, ws, stream, foreign=None):
+    """One decode step as a model issues it: ikv_step_begin, then per layer (after the
+    caller's own work for that layer, `foreign(l)`, if given) ikv_step_layer, then
+    ikv_step_end."""
+    from paper_2609_03515_gb300 import ikv
+
+    ikv.ikv_step_begin(c.shape(), p, cache, c.ema, t, ws, ws.numel(), stream)
+    for l in range(c.layers):
+        if foreign is None:
+            ikv.ikv_step_layer(c.shape(), p, cache, c.ema, t, l, q[l], kn[l], vn[l], out[l], ws, ws.numel(), stream)
+        else:
+            ql, kl, vl = foreign(l)
+            ikv.ikv_step_layer(c.shape(), p, cache, c.ema, t, l, ql, kl, vl, out[l], ws, ws.numel(), stream)
+    ikv.ikv_step_end(c.shape(), p, cache, c.ema, t, ws, ws.numel(), stream)
+
+
 def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, sample_clocks: bool,
-                   mh: int = 0, scorer: int = 0):
+                   mh: int = 0, scorer: int = 0, per_layer: str = ""):
     """The same schedule with each steady-state step replayed from a captured CUDA graph.
 
     After the eager warm-up (decode step 1 evicts ~90% of the prefill, later steps hold
     the budget), one graph per timed step t is captured around ikv_step(t) with that
     step's resident inputs (q, k_new, v_new of step t), so replaying it does exactly what
-    the eager call would, with no staging copies; the timed region replays them in order."""
+    the eager call would, with no staging copies; the timed region replays them in order.
+    per_layer "split": the step as ikv_step_begin / one ikv_step_layer per layer /
+    ikv_step_end; "foreign": the same, with the layer's q, k_new and v_new first copied
+    by PyTorch kernels into per-layer buffers (standing in for the projection that a
+    model runs before each layer's attention)."""
     import torch
 
     from paper_2609_03515_gb300 import ikv, step_lengths
@@ -350,9 +370,28 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     dev = c.k.device
     out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=c.torch_dtype, device=dev)
     W, K = args.warmup, args.steps
+    ql = torch.empty(qs_dev.shape[2:], dtype=qs_dev.dtype, device=dev)
+    kl = torch.empty(kn_dev.shape[2:], dtype=kn_dev.dtype, device=dev)
+    vl = torch.empty_like(kl)
+
+    def one(cache, t):
+        st = torch.cuda.current_stream()
+        if not per_layer:
+            ikv.ikv_step(c.shape(), p, cache, c.ema, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws,
+                         ws.numel(), st)
+            return
+
+        def foreign(l):
+            ql.copy_(qs_dev[t - 1, l])
+            kl.copy_(kn_dev[t - 1, l])
+            vl.copy_(vn_dev[t - 1, l])
+            return ql, kl, vl
+
+        split_step(c, p, cache, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws, st,
+                   foreign if per_layer == "foreign" else None)
+
     for t in range(1, W + 1):
-        ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws,
-                     ws.numel(), torch.cuda.current_stream())
+        one(c.cache(max(lens)), t)
         lens, live = step_lengths(lens, live, budgets, mh)
     torch.cuda.synchronize()
     # the graphs' max_len bounds every later step: the budget plus the dead slots
@@ -364,8 +403,7 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
         t = W + 1 + i
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, capture_error_mode="thread_local"):
-            ikv.ikv_step(c.shape(), p, steady, c.ema, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws,
-                         ws.numel(), torch.cuda.current_stream())
+            one(steady, t)
         graphs.append((g, ikv.ikv_launch_count() - n0))
         n0 = ikv.ikv_launch_count()
     torch.cuda.synchronize()
@@ -573,6 +611,10 @@ def run_ours(args):
     e2e_all = sorted(r[0] for r in e2e_runs)
     e2e_ms, h2d, d2h = e2e_all[2], e2e_runs[0][1], e2e_runs[0][2]
 
+    # the model-integration form: the same headline steps split per layer
+    per_layer = {k: run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, False, mh,
+                                   per_layer=k) for k in ("split", "foreign")}
+
     head_sched = schedule_name(w)
     modes = {}
     mode_kernels = {}
@@ -654,6 +696,16 @@ def run_ours(args):
                 "note": "median of five runs; inputs uploaded from pinned host memory and outputs read back "
                         "every step, overlapped with the previous / next step's compute"},
         "gpu_launches": full["launches"],
+        "per_layer": {
+            "value": job_throughput(w.batch * K, world, per_layer["split"]["ms"]),
+            "ms_per_step": per_layer["split"]["ms"] / K,
+            "vs_whole_step": full["ms"] / per_layer["split"]["ms"],
+            "gpu_launches": per_layer["split"]["launches"],
+            "with_foreign_copies": {"value": job_throughput(w.batch * K, world, per_layer["foreign"]["ms"]),
+                                    "ms_per_step": per_layer["foreign"]["ms"] / K},
+            "note": "the headline steps as ikv_step_begin / one ikv_step_layer per layer / ikv_step_end, one CUDA "
+                    "graph per step (PDL between the library's kernels); with_foreign_copies: each layer's q, "
+                    "k_new, v_new first copied by PyTorch kernels (3 per layer, not counted in gpu_launches)"},
         "clocks": full["clocks"],
         "modes": {k: w.batch * K * world / (v["ms"] / 1e3) for k, v in modes.items()},
     }

@@ -324,6 +324,40 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *params, ikv_cache 
                     const void *q, const void *k_new, const void *v_new, void *out, void *ws, size_t ws_bytes,
                     cudaStream_t stream);
 
+/* ---------------------------------------------------------------------------
+ * ikv_step_begin / ikv_step_layer / ikv_step_end -- ikv_step split at its layer
+ * boundary, for a model that has layer l's q, k_new and v_new only after layer
+ * l-1's attention output (Appendix "Layer scoring": the scores come from each
+ * layer's attention inside the forward pass).  Calling
+ *     ikv_step_begin(t); ikv_step_layer(t, 0); ...; ikv_step_layer(t, layers-1); ikv_step_end(t)
+ * on one stream does what ikv_step(t) does with the same arguments (results equal
+ * up to the rounding of the attention's split-K merge, which is partitioned per
+ * layer here).  Between the calls the stream may run other work that leaves the
+ * cache, ema and ws alone; the sequence may be captured in a CUDA graph.
+ *  - ikv_step_begin: step 2's bookkeeping -- reserves slot len[b] for the new token
+ *    (its position and utility, as ikv_append_token), len[b] += 1.  Its K/V rows
+ *    are written by ikv_step_layer.
+ *  - ikv_step_layer: writes k_new/v_new ([batch][kv_heads][head_dim], layer `layer`)
+ *    into the reserved slot and runs that layer's attention (step 3; out, q:
+ *    [batch][q_heads][head_dim]); on refresh steps an eligible layer also keeps its
+ *    attention logits in ws.  Every layer is called once, in ascending order.
+ *  - ikv_step_end: step 4 -- the kept scores of every eligible layer folded into ema
+ *    in ascending layer order, which is the order Eq. 4 prescribes; nothing reads ema
+ *    before the eviction -- and step 5 (selection, deferred or immediate compaction).
+ *  All three take the same shape, params, cache (max_len: the bound on len[]
+ *  before the append, as for ikv_step), ema, t and ws (ikv_step_workspace_size
+ *  bytes, which carries the step's state from call to call).  Argument errors are
+ *  reported by the call that sees them; nothing is launched then, and the step
+ *  cannot be continued.
+ * ------------------------------------------------------------------------- */
+ikv_status ikv_step_begin(const ikv_shape *shape, const ikv_params *params, ikv_cache *cache, float *ema, int32_t t,
+                          void *ws, size_t ws_bytes, cudaStream_t stream);
+ikv_status ikv_step_layer(const ikv_shape *shape, const ikv_params *params, ikv_cache *cache, float *ema, int32_t t,
+                          int32_t layer, const void *q, const void *k_new, const void *v_new, void *out, void *ws,
+                          size_t ws_bytes, cudaStream_t stream);
+ikv_status ikv_step_end(const ikv_shape *shape, const ikv_params *params, ikv_cache *cache, float *ema, int32_t t,
+                        void *ws, size_t ws_bytes, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

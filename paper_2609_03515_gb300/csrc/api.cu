@@ -131,7 +131,7 @@ AttendWs attend_ws(const ikv_shape *s, int32_t cap, int n_layers, bool logits) {
 
 struct StepWs {
     AttendWs at;
-    size_t keep, keep_len, done, cdone, moves, n_moves, sbuf, epart, vmean, end;
+    size_t keep, keep_len, done, cdone, moves, n_moves, sbuf, epart, vmean, slot, end;
 };
 
 StepWs step_ws(const ikv_shape *s, int32_t cap) {
@@ -158,6 +158,8 @@ StepWs step_ws(const ikv_shape *s, int32_t cap) {
     off = align256(off + R * (s->layers + 1) * blk_max * sizeof(float));
     w.vmean = off;
     off = align256(off + (size_t)s->batch * s->layers * s->kv_heads * sizeof(float));
+    w.slot = off;  // split step: each sequence's reserved slot
+    off = align256(off + (size_t)s->batch * sizeof(int32_t));
     w.end = off;
     return w;
 }
@@ -204,7 +206,8 @@ static bool use_tc(const ikv_shape *s, const ikv_cache *c, int32_t layers_touche
 ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, int32_t n_layers, int32_t max_len,
                       const void *q, void *out, void *ws, const AttendWs &w, bool logits, int32_t *split_out,
                       int32_t *nsplit_out, cudaStream_t st, const ikv_timing *tm = nullptr,
-                      bool counters_zeroed = false) {
+                      bool counters_zeroed = false, int32_t sc_layers = 0, int32_t sc_layer0 = 0,
+                      const AppendArgs *append = nullptr) {
     AttendArgs a{};
     a.k = c->k;
     a.v = c->v;
@@ -233,6 +236,18 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
     a.part_o = at<float>(ws, w.part_o);
     a.pos = c->dead_slots ? c->pos : nullptr;
     a.rows_per_seq = rows_per_seq(s);
+    a.sc_layers = sc_layers > 0 ? sc_layers : n_layers;
+    a.sc_layer0 = sc_layer0;
+    // split step: the new token's rows of this layer are stored by the tensor-core kernel
+    // itself, or by a copy kernel ahead of the CUDA-core one
+    if (append && tc) {
+        a.k_new = append->k_new;
+        a.v_new = append->v_new;
+        a.slot = append->slot;
+        a.vnorm = append->vnorm;
+    } else if (append) {
+        IKV_TRY_CUDA(launch_append_rows(*append, st), "append rows launch");
+    }
     if (tc) {
         // fused combine: the last split of each unit writes out and lse2
         int32_t *arr = at<int32_t>(ws, w.arrivals);
@@ -257,6 +272,8 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
         cb.part_o = a.part_o;
         cb.out = out;
         cb.lse2 = at<float>(ws, w.lse2);
+        cb.sc_layers = a.sc_layers;
+        cb.sc_layer0 = a.sc_layer0;
         IKV_TRY_CUDA(launch_combine(cb, s->dtype, st), "combine launch");
     }
     if (split_out) *split_out = a.split_tokens;
@@ -273,7 +290,7 @@ struct ScorerWs {
 ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, const int32_t *elig, int n_elig,
                      int32_t max_len, void *ws, const AttendWs &w, float alpha, float *ema, float *score,
                      cudaStream_t st, int32_t agg = IKV_AGG_EMA, int32_t scorer = IKV_SCORE_ATTENTION,
-                     const ScorerWs &sw = ScorerWs{}) {
+                     const ScorerWs &sw = ScorerWs{}, int32_t layer0 = 0) {
     ScoreArgs base{};
     base.len = c->len;
     base.batch = s->batch;
@@ -289,7 +306,7 @@ ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, c
     base.agg = agg;
     base.ema = ema;
     base.score = score;
-    base.layer0 = 0;
+    base.layer0 = layer0;
     base.scorer = scorer;
     base.vnorm = c->vnorm;
     base.vmean = sw.vmean;
@@ -486,7 +503,7 @@ ikv_status ikv_compact_kv(const ikv_shape *shape, ikv_cache *cache, const int32_
 
 static ikv_status append_impl(const ikv_shape *shape, ikv_cache *cache, const void *k_new, const void *v_new,
                               float *ema, int32_t init_mean, int32_t *done, cudaStream_t stream,
-                              bool counters_zeroed = false) {
+                              bool counters_zeroed = false, int32_t *slot = nullptr) {
     AppendArgs a{};
     a.k = cache->k;
     a.v = cache->v;
@@ -506,6 +523,7 @@ static ikv_status append_impl(const ikv_shape *shape, ikv_cache *cache, const vo
     a.dead_slots = cache->dead_slots ? 1 : 0;
     a.done = done;
     a.vnorm = cache->vnorm;
+    a.slot = slot;
     if (!counters_zeroed)
         IKV_TRY_CUDA(cudaMemsetAsync(done, 0, sizeof(int32_t) * shape->batch, stream), "cudaMemsetAsync");
     IKV_TRY_CUDA(launch_append(a, stream), "append launch");
@@ -526,27 +544,26 @@ ikv_status ikv_append_token(const ikv_shape *shape, ikv_cache *cache, const void
     return append_impl(shape, cache, k_new, v_new, ema, init_mean, at<int32_t>(ws, 0), stream);
 }
 
-ikv_status ikv_step_workspace_size(const ikv_shape *shape, const ikv_cache *cache, size_t *bytes) {
-    g_err[0] = 0;
-    ikv_status e = check_shape(shape);
-    if (e) return e;
-    if ((e = check_cache(shape, cache, false))) return e;
-    if (!bytes) return fail(IKV_ERR_ARG, "bytes is NULL");
-    *bytes = step_ws(shape, cap_of(cache)).end;
-    return IKV_OK;
-}
+// What every call of a decode step (ikv_step, or its begin / layer / end split) needs:
+// checked arguments, the cache as the step's kernels see it, the workspace layout
+// and the step's schedule.
+struct StepCtx {
+    ikv_cache cv;
+    StepWs w;
+    int32_t cap, L1, init_mean;
+    bool scoring;
+    int32_t elig[kMaxLayers];
+    int n_elig;
+    ScorerWs sw;
+};
 
-ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, int32_t t,
-                    const void *q, const void *k_new, const void *v_new, void *out, void *ws, size_t ws_bytes,
-                    cudaStream_t stream) {
-    g_err[0] = 0;
+static ikv_status prepare_step(const ikv_shape *shape, const ikv_params *p, const ikv_cache *cache, float *ema,
+                               int32_t t, void *ws, size_t ws_bytes, StepCtx *cx) {
     ikv_status e = check_shape(shape);
     if (e) return e;
     if ((e = check_cache(shape, cache, true))) return e;
     if (!p) return fail(IKV_ERR_ARG, "params is NULL");
-    if (!ema || !q || !k_new || !v_new || !out || !p->budget) return fail(IKV_ERR_ARG, "ema/q/k_new/v_new/out/budget is NULL");
-    if (!aligned16(q) || !aligned16(out) || !aligned16(k_new) || !aligned16(v_new))
-        return fail(IKV_ERR_ALIGN, "q/out/k_new/v_new must be 16-byte aligned");
+    if (!ema || !p->budget) return fail(IKV_ERR_ARG, "ema/budget is NULL");
     if (t < 1) return fail(IKV_ERR_ARG, "t is 1-based (got %d)", t);
     if (!(p->alpha >= 0.f && p->alpha <= 1.f)) return fail(IKV_ERR_ARG, "alpha must be in [0, 1]");
     if (p->refresh_period < 1) return fail(IKV_ERR_ARG, "refresh_period must be >= 1");
@@ -564,21 +581,63 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
         return fail(IKV_ERR_ARG, "unknown scorer %d", p->scorer);
     if (p->scorer == IKV_SCORE_VNORM && !cache->vnorm) return fail(IKV_ERR_ARG, "IKV_SCORE_VNORM needs cache->vnorm");
     // with deferred compaction every kernel of the step treats pos < 0 as a dead slot
-    ikv_cache cv = *cache;
-    if (p->max_holes > 0) cv.dead_slots = 1;
-    cache = &cv;
-    const int32_t cap = cap_of(cache);
-    if (cache->max_len + 1 > cap) return fail(IKV_ERR_SHAPE, "no free slot: max_len + 1 > cap");
-    const StepWs w = step_ws(shape, cap);
-    if (!ws || ws_bytes < w.end) return fail(IKV_ERR_WORKSPACE, "workspace needs %zu bytes", w.end);
-
+    cx->cv = *cache;
+    if (p->max_holes > 0) cx->cv.dead_slots = 1;
+    cx->cap = cap_of(cache);
+    if (cache->max_len + 1 > cx->cap) return fail(IKV_ERR_SHAPE, "no free slot: max_len + 1 > cap");
+    cx->w = step_ws(shape, cx->cap);
+    if (!ws || ws_bytes < cx->w.end) return fail(IKV_ERR_WORKSPACE, "workspace needs %zu bytes", cx->w.end);
     const bool refresh = p->score_free ? (t == 1) : ((t - 1) % p->refresh_period == 0);
-    int32_t elig[kMaxLayers];
-    int n_elig = 0;
+    cx->n_elig = 0;
     for (int l = 0; l < shape->layers; ++l)
-        if (!p->layer_eligible || p->layer_eligible[l]) elig[n_elig++] = l;
-    const bool scoring = refresh && n_elig > 0;
-    const int32_t L1 = cache->max_len + 1;
+        if (!p->layer_eligible || p->layer_eligible[l]) cx->elig[cx->n_elig++] = l;
+    cx->scoring = refresh && cx->n_elig > 0;
+    cx->L1 = cache->max_len + 1;
+    cx->init_mean = refresh ? (p->refresh_init == IKV_INIT_MEAN) : 1;
+    cx->sw.sbuf = at<float>(ws, cx->w.sbuf);
+    cx->sw.epart = at<float>(ws, cx->w.epart);
+    cx->sw.vmean = at<float>(ws, cx->w.vmean);
+    return IKV_OK;
+}
+
+// Step 5: selection, then deferred or immediate compaction.
+static ikv_status evict_impl(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, void *ws,
+                             const StepWs &w, cudaStream_t stream, const ikv_timing *tm) {
+    const int32_t cap = cap_of(cache);
+    const int32_t R = shape->batch * rows_per_seq(shape);
+    IKV_TRY_CUDA(launch_select(R, cap, ema, cache->len, rows_per_seq(shape), p->budget,
+                               cache->dead_slots ? cache->pos : nullptr, at<int32_t>(ws, w.keep),
+                               at<int32_t>(ws, w.keep_len), DeferArgs{p->max_holes, cap, cache->start}, stream),
+                 "select launch");
+    ikv_status e;
+    if (tm && (e = record(tm->select_end, stream))) return e;
+    return compact_impl(shape, cache, at<int32_t>(ws, w.keep), at<int32_t>(ws, w.keep_len), ema, p->compact_mode,
+                        at<int32_t>(ws, w.moves), at<int32_t>(ws, w.n_moves), at<int32_t>(ws, w.cdone), stream,
+                        p->max_holes);
+}
+
+ikv_status ikv_step_workspace_size(const ikv_shape *shape, const ikv_cache *cache, size_t *bytes) {
+    g_err[0] = 0;
+    ikv_status e = check_shape(shape);
+    if (e) return e;
+    if ((e = check_cache(shape, cache, false))) return e;
+    if (!bytes) return fail(IKV_ERR_ARG, "bytes is NULL");
+    *bytes = step_ws(shape, cap_of(cache)).end;
+    return IKV_OK;
+}
+
+ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, int32_t t,
+                    const void *q, const void *k_new, const void *v_new, void *out, void *ws, size_t ws_bytes,
+                    cudaStream_t stream) {
+    g_err[0] = 0;
+    StepCtx cx;
+    ikv_status e = prepare_step(shape, p, cache, ema, t, ws, ws_bytes, &cx);
+    if (e) return e;
+    if (!q || !k_new || !v_new || !out) return fail(IKV_ERR_ARG, "q/k_new/v_new/out is NULL");
+    if (!aligned16(q) || !aligned16(out) || !aligned16(k_new) || !aligned16(v_new))
+        return fail(IKV_ERR_ALIGN, "q/out/k_new/v_new must be 16-byte aligned");
+    cache = &cx.cv;
+    const StepWs &w = cx.w;
     const ikv_timing *tm = p->timing;
 
     // control words (append and split-arrival counters) start at zero
@@ -587,38 +646,88 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.done), 0, 2 * sizeof(int32_t) * shape->batch, stream),
                  "cudaMemsetAsync");
     if (tm && (e = record(tm->begin, stream))) return e;
-    const int32_t init_mean = refresh ? (p->refresh_init == IKV_INIT_MEAN) : 1;
-    if ((e = append_impl(shape, cache, k_new, v_new, ema, init_mean, at<int32_t>(ws, w.done), stream, true)))
+    if ((e = append_impl(shape, cache, k_new, v_new, ema, cx.init_mean, at<int32_t>(ws, w.done), stream, true)))
         return e;
     if (tm && (e = record(tm->append_end, stream))) return e;
     // the rest of the chain may overlap each kernel's ramp-up with its predecessor's tail
     // (not when per-kernel events are recorded: those time each kernel alone)
     std::optional<PdlScope> pdl;
     if (!tm) pdl.emplace();
-    if ((e = run_attend(shape, cache, 0, shape->layers, L1, q, out, ws, w.at, scoring, nullptr, nullptr, stream, tm,
-                        true)))
+    if ((e = run_attend(shape, cache, 0, shape->layers, cx.L1, q, out, ws, w.at, cx.scoring, nullptr, nullptr, stream,
+                        tm, true)))
         return e;
     if (tm && (e = record(tm->combine_end, stream))) return e;
-    ScorerWs sw;
-    sw.sbuf = at<float>(ws, w.sbuf);
-    sw.epart = at<float>(ws, w.epart);
-    sw.vmean = at<float>(ws, w.vmean);
-    if (scoring && (e = run_score(shape, cache, shape->layers, elig, n_elig, L1, ws, w.at, p->alpha, ema, nullptr, stream,
-                                  p->agg_mode, p->scorer, sw)))
+    if (cx.scoring && (e = run_score(shape, cache, shape->layers, cx.elig, cx.n_elig, cx.L1, ws, w.at, p->alpha, ema,
+                                     nullptr, stream, p->agg_mode, p->scorer, cx.sw)))
         return e;
     if (tm && (e = record(tm->score_end, stream))) return e;
-    const int32_t R = shape->batch * rows_per_seq(shape);
-    IKV_TRY_CUDA(launch_select(R, cap, ema, cache->len, rows_per_seq(shape), p->budget,
-                               cache->dead_slots ? cache->pos : nullptr, at<int32_t>(ws, w.keep),
-                               at<int32_t>(ws, w.keep_len), DeferArgs{p->max_holes, cap, cache->start}, stream),
-                 "select launch");
-    if (tm && (e = record(tm->select_end, stream))) return e;
-    if ((e = compact_impl(shape, cache, at<int32_t>(ws, w.keep), at<int32_t>(ws, w.keep_len), ema, p->compact_mode,
-                          at<int32_t>(ws, w.moves), at<int32_t>(ws, w.n_moves), at<int32_t>(ws, w.cdone), stream,
-                          p->max_holes)))
-        return e;
+    if ((e = evict_impl(shape, p, cache, ema, ws, w, stream, tm))) return e;
     if (tm && (e = record(tm->end, stream))) return e;
     return IKV_OK;
+}
+
+ikv_status ikv_step_begin(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, int32_t t,
+                          void *ws, size_t ws_bytes, cudaStream_t stream) {
+    g_err[0] = 0;
+    StepCtx cx;
+    ikv_status e = prepare_step(shape, p, cache, ema, t, ws, ws_bytes, &cx);
+    if (e) return e;
+    // control words start at zero (the attention leaves its arrival counters zero)
+    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, cx.w.at.arrivals), 0, cx.w.at.logits - cx.w.at.arrivals, stream),
+                 "cudaMemsetAsync");
+    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, cx.w.done), 0, 2 * sizeof(int32_t) * shape->batch, stream),
+                 "cudaMemsetAsync");
+    return append_impl(shape, &cx.cv, nullptr, nullptr, ema, cx.init_mean, at<int32_t>(ws, cx.w.done), stream, true,
+                       at<int32_t>(ws, cx.w.slot));
+}
+
+ikv_status ikv_step_layer(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, int32_t t,
+                          int32_t layer, const void *q, const void *k_new, const void *v_new, void *out, void *ws,
+                          size_t ws_bytes, cudaStream_t stream) {
+    g_err[0] = 0;
+    StepCtx cx;
+    ikv_status e = prepare_step(shape, p, cache, ema, t, ws, ws_bytes, &cx);
+    if (e) return e;
+    if (layer < 0 || layer >= shape->layers) return fail(IKV_ERR_ARG, "layer %d out of range", layer);
+    if (!q || !k_new || !v_new || !out) return fail(IKV_ERR_ARG, "q/k_new/v_new/out is NULL");
+    if (!aligned16(q) || !aligned16(out) || !aligned16(k_new) || !aligned16(v_new))
+        return fail(IKV_ERR_ALIGN, "q/out/k_new/v_new must be 16-byte aligned");
+    cache = &cx.cv;
+    PdlScope pdl;
+    AppendArgs a{};
+    a.k = cache->k;
+    a.v = cache->v;
+    a.pv = view_of(shape, cache);
+    a.batch = shape->batch;
+    a.layers = 1;
+    a.rows_per_seq = rows_per_seq(shape);
+    a.cap = cx.cap;
+    a.elem_bytes = elem_bytes(shape);
+    a.k_new = k_new;
+    a.v_new = v_new;
+    a.vnorm = cache->vnorm;
+    a.layer0 = layer;
+    a.slot = at<int32_t>(ws, cx.w.slot);
+    bool eligible = false;
+    for (int k = 0; k < cx.n_elig; ++k) eligible |= cx.elig[k] == layer;
+    // the new token's rows and one layer's attention; on refresh steps its logits and
+    // log-sum-exp land where the whole step's attention would put them, for
+    // ikv_step_end's score pass
+    return run_attend(shape, cache, layer, 1, cx.L1, q, out, ws, cx.w.at, cx.scoring && eligible, nullptr, nullptr,
+                      stream, nullptr, true, shape->layers, layer, &a);
+}
+
+ikv_status ikv_step_end(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, int32_t t,
+                        void *ws, size_t ws_bytes, cudaStream_t stream) {
+    g_err[0] = 0;
+    StepCtx cx;
+    ikv_status e = prepare_step(shape, p, cache, ema, t, ws, ws_bytes, &cx);
+    if (e) return e;
+    PdlScope pdl;
+    if (cx.scoring && (e = run_score(shape, &cx.cv, shape->layers, cx.elig, cx.n_elig, cx.L1, ws, cx.w.at, p->alpha,
+                                     ema, nullptr, stream, p->agg_mode, p->scorer, cx.sw)))
+        return e;
+    return evict_impl(shape, p, &cx.cv, ema, ws, cx.w, stream, nullptr);
 }
 
 }  // extern "C"

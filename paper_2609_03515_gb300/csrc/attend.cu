@@ -229,7 +229,8 @@ __global__ void __launch_bounds__(kAttendThreads, 2) attend_split_kernel(const A
             if (j < nv) {
                 if (prow && prow[tbase + j] < 0) z = -INFINITY;
                 if (LOGITS)
-                    a.logits[((((int64_t)b * a.n_layers + li) * H) + g * G + h) * (int64_t)a.lstride + tbase + j] = z;
+                    a.logits[((((int64_t)b * a.sc_layers + a.sc_layer0 + li) * H) + g * G + h) * (int64_t)a.lstride +
+                             tbase + j] = z;
             } else {
                 z = -INFINITY;
             }
@@ -332,7 +333,7 @@ __global__ void __launch_bounds__(128) combine_kernel(const CombineArgs a) {
         Chunk<T>::store(a.out, obase + e, acc * inv);
     }
     if (a.lse2 && threadIdx.x == 0)
-        a.lse2[((int64_t)b * a.n_layers + li) * a.q_heads + h] = wsum > 0.f ? M + log2f(wsum) : -INFINITY;
+        a.lse2[((int64_t)b * a.sc_layers + a.sc_layer0 + li) * a.q_heads + h] = wsum > 0.f ? M + log2f(wsum) : -INFINITY;
 }
 
 template <typename T, int D, int G>

@@ -64,14 +64,21 @@ struct TcArgs {
     const __nv_bfloat16 *q;     // q + ((li*batch + b)*H + h)*128
     int32_t batch, q_heads, layer0, n_layers, split_tokens, n_splits, cap;
     float scale_log2;
-    float *logits;              // may be null; rows of lstride floats
+    float *logits;              // may be null; [batch][sc_layers][H][lstride]
     int32_t lstride;            // logits row stride, a multiple of 128
     float *part_ml, *part_o;
     __nv_bfloat16 *out;         // [n_layers][batch][H][128]
-    float *lse2;                // [batch][n_layers][H]
+    float *lse2;                // [batch][sc_layers][H]
     int32_t *arrivals;          // [batch][n_layers][kv_heads], zero on entry, left zero
     const int32_t *pos;         // [rows][cap], -1 at dead slots; null: every slot below len is live
     int32_t rows_per_seq;
+    int32_t sc_layers, sc_layer0;  // local layer li is layer sc_layer0 + li of logits / lse2
+    // split step: the new token's K/V rows ([batch][kv_heads][128]) go to logical slot
+    // slot[b] (-1: none) before the attention reads it; vnorm (or null) gets its V norm
+    const __nv_bfloat16 *k_new, *v_new;
+    const int32_t *slot;
+    __nv_bfloat16 *k_pool, *v_pool;
+    float *vnorm;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -217,7 +224,8 @@ __global__ void __launch_bounds__(kThreads, 2)
             for (int i = threadIdx.x; i < G * kD; i += kThreads)
                 a.out[(((int64_t)li * a.batch + b) * a.q_heads + (int64_t)g * G) * kD + i] = __float2bfloat16_rn(0.f);
             if (threadIdx.x < G)
-                a.lse2[((int64_t)b * a.n_layers + li) * a.q_heads + (int64_t)g * G + threadIdx.x] = -INFINITY;
+                a.lse2[((int64_t)b * a.sc_layers + a.sc_layer0 + li) * a.q_heads + (int64_t)g * G + threadIdx.x] =
+                    -INFINITY;
         }
         return;
     }
@@ -243,19 +251,77 @@ __global__ void __launch_bounds__(kThreads, 2)
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(sm + kOffMisc);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + kOffMisc + 4);
 
-    if (tid == 0) {
-        for (int i = 0; i < kNst; ++i) {
-            mbar_init(full(i), 1);
-            mbar_init(empty(i), 1);
+    // pool row of box bx of load j (loads 0..n-1: K tiles, n..2n-1: V tiles)
+    const int boxes = kTile / a.rows_per_box;
+    auto box_row = [&](int j, int bx) {
+        const int tile = j < n ? j : j - n;
+        const int tok = t0 + tile * kTile + bx * a.rows_per_box;
+        int lp = tok / a.page_size;
+        if (lp >= a.max_pages) lp = a.max_pages - 1;
+        const int page = a.block_table[(int64_t)b * a.max_pages + lp];
+        return ((l * a.num_pages + page) * a.kv_heads + g) * a.page_size + tok % a.page_size;
+    };
+    auto issue = [&](int j) {
+        const int st = j % kNst;
+        mbar_expect_tx(full(st), kStage);
+        const CUtensorMap *tm = j < n ? &tmK : &tmV;
+        const uint32_t dst = base + st * kStage;
+        for (int bx = 0; bx < boxes; ++bx) {
+            const int row = box_row(j, bx);
+            tma_load_2d(dst + bx * a.rows_per_box * 128, tm, 0, row, full(st));
+            tma_load_2d(dst + kHalf + bx * a.rows_per_box * 128, tm, 64, row, full(st));
         }
-        mbar_init(s_full, 1);
-        mbar_init(p_full(0), 128);
-        mbar_init(p_full(1), 128);
-        mbar_init(p_empty(0), 1);
-        mbar_init(p_empty(1), 1);
-        mbar_init(o_full, 1);
-        *abort_flag = 0;
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    };
+    const int n_first = min(2 * n, kNst);  // loads issued before the CTA-wide barrier
+    if (warp == 4) {
+        // Split step: the CTA whose chunk holds the new token's slot stores the token's K
+        // and V rows into the cache (lanes 0-15: K, 16-31: V, 16 bytes each) before its
+        // TMA loads read that tile; the proxy fence orders the stores before them.
+        if (a.k_new) {
+            const int j = a.slot[b];
+            const int p = S0 + j;
+            if (j >= 0 && p >= t0 && p < t0 + n * kTile) {
+                const int page = a.block_table[(int64_t)b * a.max_pages + p / a.page_size];
+                const int64_t row = ((int64_t)(l * a.num_pages + page) * a.kv_heads + g) * a.page_size + p % a.page_size;
+                const bool isv = lane >= 16;
+                const int c = lane & 15;
+                const uint4 x = reinterpret_cast<const uint4 *>(isv ? a.v_new : a.k_new)[((int64_t)b * a.kv_heads + g) * 16 + c];
+                reinterpret_cast<uint4 *>(isv ? a.v_pool : a.k_pool)[row * 16 + c] = x;
+                float sq = 0.f;
+                if (isv) {
+                    const uint32_t w4[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const float lo = __uint_as_float(w4[k] << 16), hi = __uint_as_float(w4[k] & 0xffff0000u);
+                        sq += lo * lo + hi * hi;
+                    }
+                }
+#pragma unroll
+                for (int o = 8; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+                if (a.vnorm && lane == 16)
+                    a.vnorm[(((int64_t)l * a.batch + b) * a.kv_heads + g) * a.cap + j] = sqrtf(sq);
+                asm volatile("fence.proxy.async.global;" ::: "memory");
+            }
+            __syncwarp();
+        }
+        // the producer initialises the barriers and starts the K/V stream at once; the
+        // Q staging and TMEM allocation below overlap the loads' latency
+        if (lane == 0) {
+            for (int i = 0; i < kNst; ++i) {
+                mbar_init(full(i), 1);
+                mbar_init(empty(i), 1);
+            }
+            mbar_init(s_full, 1);
+            mbar_init(p_full(0), 128);
+            mbar_init(p_full(1), 128);
+            mbar_init(p_empty(0), 1);
+            mbar_init(p_empty(1), 1);
+            mbar_init(o_full, 1);
+            *abort_flag = 0;
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+            for (int j = 0; j < n_first; ++j) issue(j);
+        }
+        __syncwarp();
     }
     if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
@@ -284,28 +350,11 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (warp == 4) {
         // ---------------- TMA producer
         if (lane == 0) {
-            const int boxes = kTile / a.rows_per_box;
-            // pool row of box bx of load j (loads 0..n-1: K tiles, n..2n-1: V tiles)
-            auto box_row = [&](int j, int bx) {
-                const int tile = j < n ? j : j - n;
-                const int tok = t0 + tile * kTile + bx * a.rows_per_box;
-                int lp = tok / a.page_size;
-                if (lp >= a.max_pages) lp = a.max_pages - 1;
-                const int page = a.block_table[(int64_t)b * a.max_pages + lp];
-                return ((l * a.num_pages + page) * a.kv_heads + g) * a.page_size + tok % a.page_size;
-            };
-            int issued = 0;
-            for (int j = 0; j < 2 * n; ++j) {
+            int issued = n_first;
+            for (int j = n_first; j < 2 * n; ++j) {
                 const int st = j % kNst;
-                if (j >= kNst && !mbar_wait(empty(st), ((j / kNst) - 1) & 1, abort_flag)) break;
-                mbar_expect_tx(full(st), kStage);
-                const CUtensorMap *tm = j < n ? &tmK : &tmV;
-                const uint32_t dst = base + st * kStage;
-                for (int bx = 0; bx < boxes; ++bx) {
-                    const int row = box_row(j, bx);
-                    tma_load_2d(dst + bx * a.rows_per_box * 128, tm, 0, row, full(st));
-                    tma_load_2d(dst + kHalf + bx * a.rows_per_box * 128, tm, 64, row, full(st));
-                }
+                if (!mbar_wait(empty(st), ((j / kNst) - 1) & 1, abort_flag)) break;
+                issue(j);
                 issued = j + 1;
             }
             // drain: the last phase issued on each stage must have landed before the CTA exits
@@ -402,7 +451,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         // sweep 2: logits write-out, exp2, row sums and the P operand of each tile.  The
         // logits stores sit here, interleaved with the V stream; issued as a burst in
         // sweep 1 they measured slower.
-        const int64_t lbase = (((int64_t)b * a.n_layers + li) * H + (int64_t)g * G) * a.lstride;
+        const int64_t lbase = (((int64_t)b * a.sc_layers + a.sc_layer0 + li) * H + (int64_t)g * G) * a.lstride;
         for (int i = 0; i < n && ok; ++i) {
             if (i >= 2 && !(ok = __all_sync(0xffffffffu, mbar_wait(p_empty(i & 1), ((i >> 1) - 1) & 1, abort_flag))))
                 break;
@@ -472,55 +521,68 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (*last_flag && ok) {
             __threadfence();
             const int64_t pbase = (((int64_t)b * a.n_layers + li) * H + (int64_t)g * G) * a.n_splits;
-            // online merge over the unit's splits, four splits x all heads per round so that
-            // every load of a round is in flight at once
-            float M[G], ws[G], acc[G];
+            // split weights [G][n_splits] in the P buffers (every MMA has completed)
+            float *wq = reinterpret_cast<float *>(sm + kOffP);
+            // warp w merges heads w, w + 4: (1) the splits' (max, sum) pairs give the head's
+            // maximum M, each split's weight exp2(m - M) (0 for a split whose rows are all
+            // dead) and the total W; (2) lane i sums the weighted partial outputs of dims
+            // 4i .. 4i+3.  All loads of a phase are independent, so the merge costs a few
+            // L2 round trips whatever the number of splits.
+            for (int h = warp; h < G; h += 4) {
+                const float2 *ml = reinterpret_cast<const float2 *>(a.part_ml) + pbase + (int64_t)h * a.n_splits;
+                float mv[kMaxSplits / 32], lv[kMaxSplits / 32];
+                float M = -INFINITY;
 #pragma unroll
-            for (int h = 0; h < G; ++h) {
-                M[h] = -INFINITY;
-                ws[h] = 0.f;
-                acc[h] = 0.f;
-            }
-            constexpr int MQ = G <= 4 ? 4 : 2;  // chunks per round (register budget)
-            for (int q0 = 0; q0 < ns_active; q0 += MQ) {
-                float mq[MQ][G], lq[MQ][G], oq[MQ][G];
-#pragma unroll
-                for (int j = 0; j < MQ; ++j)
-#pragma unroll
-                    for (int h = 0; h < G; ++h) {
-                        const int q = q0 + j;
-                        const int64_t slot = pbase + (int64_t)h * a.n_splits + q;
-                        mq[j][h] = q < ns_active ? __ldcg(a.part_ml + slot * 2) : -INFINITY;
-                        lq[j][h] = q < ns_active ? __ldcg(a.part_ml + slot * 2 + 1) : 0.f;
-                        oq[j][h] = q < ns_active ? __ldcg(a.part_o + slot * kD + tid) : 0.f;
-                    }
-#pragma unroll
-                for (int h = 0; h < G; ++h) {
-                    float mn = M[h];
-#pragma unroll
-                    for (int j = 0; j < MQ; ++j) mn = fmaxf(mn, mq[j][h]);
-                    // chunks whose rows are all dead carry max -inf and sum 0; while every
-                    // chunk so far is such, mn stays -inf and nothing accumulates
-                    const float mref = mn == -INFINITY ? 0.f : mn;
-                    const float sc = exp2f(M[h] - mref);  // 0 while M is -inf
-                    ws[h] *= sc;
-                    acc[h] *= sc;
-#pragma unroll
-                    for (int j = 0; j < MQ; ++j) {
-                        const float wq = exp2f(mq[j][h] - mref);  // 0 for padding and all-dead chunks
-                        ws[h] += lq[j][h] * wq;
-                        acc[h] += oq[j][h] * wq;
-                    }
-                    M[h] = mn;
+                for (int k = 0; k < kMaxSplits / 32; ++k) {
+                    const int q = lane + 32 * k;
+                    const float2 x = q < ns_active ? __ldcg(ml + q) : make_float2(-INFINITY, 0.f);
+                    mv[k] = x.x;
+                    lv[k] = x.y;
+                    M = fmaxf(M, x.x);
                 }
-            }
 #pragma unroll
-            for (int h = 0; h < G; ++h) {
-                const bool any = ws[h] > 0.f;  // false only if every slot of the unit is dead
-                a.out[(((int64_t)li * a.batch + b) * H + (int64_t)g * G + h) * kD + tid] =
-                    __float2bfloat16_rn(any ? acc[h] / ws[h] : 0.f);
-                if (tid == 0)
-                    a.lse2[((int64_t)b * a.n_layers + li) * H + (int64_t)g * G + h] = any ? M[h] + log2f(ws[h]) : -INFINITY;
+                for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+                const float mref = M == -INFINITY ? 0.f : M;
+                float W = 0.f;
+#pragma unroll
+                for (int k = 0; k < kMaxSplits / 32; ++k) {
+                    const int q = lane + 32 * k;
+                    const float wk = exp2f(mv[k] - mref);
+                    W += lv[k] * wk;
+                    if (q < ns_active) wq[h * a.n_splits + q] = wk;
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) W += __shfl_xor_sync(0xffffffffu, W, o);
+                __syncwarp();
+                const float4 *po =
+                    reinterpret_cast<const float4 *>(a.part_o + (pbase + (int64_t)h * a.n_splits) * kD) + lane;
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int q0 = 0; q0 < ns_active; q0 += 8) {
+                    float4 ov[8];
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        ov[j] = q0 + j < ns_active ? __ldcg(po + (int64_t)(q0 + j) * (kD / 4))
+                                                   : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const float wj = q0 + j < ns_active ? wq[h * a.n_splits + q0 + j] : 0.f;
+                        acc.x += wj * ov[j].x;
+                        acc.y += wj * ov[j].y;
+                        acc.z += wj * ov[j].z;
+                        acc.w += wj * ov[j].w;
+                    }
+                }
+                const bool any = W > 0.f;  // false only if every slot of the unit is dead
+                __nv_bfloat162 r0 = __floats2bfloat162_rn(any ? acc.x / W : 0.f, any ? acc.y / W : 0.f);
+                __nv_bfloat162 r1 = __floats2bfloat162_rn(any ? acc.z / W : 0.f, any ? acc.w / W : 0.f);
+                uint2 packed;
+                packed.x = *reinterpret_cast<uint32_t *>(&r0);
+                packed.y = *reinterpret_cast<uint32_t *>(&r1);
+                *reinterpret_cast<uint2 *>(a.out + (((int64_t)li * a.batch + b) * H + (int64_t)g * G + h) * kD +
+                                           4 * lane) = packed;
+                if (lane == 0)
+                    a.lse2[((int64_t)b * a.sc_layers + a.sc_layer0 + li) * H + (int64_t)g * G + h] =
+                        any ? M + log2f(W) : -INFINITY;
             }
             if (tid == 0) a.arrivals[unit] = 0;
         }
@@ -583,6 +645,11 @@ void tc_plan(int32_t max_len, int64_t units, int sms, int32_t *item_tiles, int32
     const int64_t tiles = ((int64_t)max_len + kTile - 1) / kTile;
     const int64_t target = (int64_t)2 * sms * IKV_TC_WAVES;
     int64_t c = (units * tiles + target - 1) / target;
+    // A launch with few units (one layer of a small batch) whose chunks fit a single wave
+    // of resident CTAs takes the shortest chunks that still fit it: every CTA runs from
+    // the start and no short tail wave follows.
+    const int64_t per_unit = (int64_t)2 * sms / (units > 0 ? units : 1);
+    if (per_unit >= 1 && (tiles + per_unit - 1) / per_unit <= kMaxTiles) c = (tiles + per_unit - 1) / per_unit;
     const int64_t cmin = (tiles + kMaxSplits - 1) / kMaxSplits;
     if (c < cmin) c = cmin;
     if (c < 1) c = 1;
@@ -633,6 +700,14 @@ cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group,
     t.arrivals = o.arrivals;
     t.pos = a.pos;
     t.rows_per_seq = a.rows_per_seq;
+    t.sc_layers = a.sc_layers;
+    t.sc_layer0 = a.sc_layer0;
+    t.k_new = reinterpret_cast<const __nv_bfloat16 *>(a.k_new);
+    t.v_new = reinterpret_cast<const __nv_bfloat16 *>(a.v_new);
+    t.slot = a.slot;
+    t.k_pool = reinterpret_cast<__nv_bfloat16 *>(const_cast<void *>(a.k));
+    t.v_pool = reinterpret_cast<__nv_bfloat16 *>(const_cast<void *>(a.v));
+    t.vnorm = a.vnorm;
     dim3 grid(a.n_splits * a.pv.kv_heads * a.batch * a.n_layers);
     cudaError_t e;
     switch (group) {

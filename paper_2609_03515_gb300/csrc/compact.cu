@@ -382,7 +382,8 @@ __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a
     const int nkv = a.layers * kvh;
     const int rowB = a.pv.head_dim * a.elem_bytes;
     const int CPR = rowB >> 4;
-    if (S + L < a.cap) {
+    if (a.slot && blockIdx.x == 0 && tid == 0) a.slot[b] = S + L < a.cap ? L : -1;
+    if (S + L < a.cap && a.k_new) {
         unsigned char *kb = reinterpret_cast<unsigned char *>(a.k);
         unsigned char *vb = reinterpret_cast<unsigned char *>(a.v);
         const unsigned char *kn = reinterpret_cast<const unsigned char *>(a.k_new);
@@ -414,6 +415,8 @@ __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a
                 if (lane == 0) a.vnorm[(((int64_t)l * a.batch + b) * kvh + g) * a.cap + L] = sqrtf(sq);
             }
         }
+    }
+    if (S + L < a.cap) {
         if (blockIdx.x == 0) {
             const int np = a.next_pos[b];
             for (int rr = 0; rr < a.rows_per_seq; ++rr) {
@@ -455,6 +458,50 @@ __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a
     }
 }
 
+// Split step: the new token's rows of one layer into the slot ikv_step_begin reserved.
+// CTA (x, b) copies kv heads 8x .. 8x+7 of sequence b and stores their value-row norms.
+__global__ void __launch_bounds__(kCompThreads) append_rows_kernel(const AppendArgs a) {
+    pdl_wait();
+    const int tid = threadIdx.x;
+    const int b = blockIdx.y;
+    const int kvh = a.pv.kv_heads;
+    const int j = a.slot[b];
+    if (j < 0) return;  // no room: the begin call flagged the error and kept len
+    const int S = a.pv.start_of(b);
+    const int l = a.layer0;
+    const int rowB = a.pv.head_dim * a.elem_bytes;
+    const int CPR = rowB >> 4;
+    unsigned char *kb = reinterpret_cast<unsigned char *>(a.k);
+    unsigned char *vb = reinterpret_cast<unsigned char *>(a.v);
+    const unsigned char *kn = reinterpret_cast<const unsigned char *>(a.k_new);
+    const unsigned char *vn = reinterpret_cast<const unsigned char *>(a.v_new);
+    for (int idx = tid; idx < kAppendRows * CPR; idx += kCompThreads) {
+        const int g = blockIdx.x * kAppendRows + idx / CPR, c = idx % CPR;
+        if (g < kvh) {
+            const int64_t src = ((int64_t)b * kvh + g) * rowB + c * 16;
+            const int64_t dst = a.pv.row_phys(b, l, g, S + j) * rowB + c * 16;
+            *reinterpret_cast<uint4 *>(kb + dst) = *reinterpret_cast<const uint4 *>(kn + src);
+            *reinterpret_cast<uint4 *>(vb + dst) = *reinterpret_cast<const uint4 *>(vn + src);
+        }
+    }
+    if (a.vnorm) {
+        const int g = blockIdx.x * kAppendRows + (tid >> 5), lane = tid & 31;
+        if ((tid >> 5) < kAppendRows && g < kvh) {
+            const int64_t e0 = ((int64_t)b * kvh + g) * a.pv.head_dim;
+            float sq = 0.f;
+            for (int e = lane; e < a.pv.head_dim; e += 32) {
+                const float xv = a.elem_bytes == 2
+                                     ? __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(a.v_new)[e0 + e])
+                                     : reinterpret_cast<const float *>(a.v_new)[e0 + e];
+                sq += xv * xv;
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+            if (lane == 0) a.vnorm[(((int64_t)l * a.batch + b) * kvh + g) * a.cap + j] = sqrtf(sq);
+        }
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_compact(const CompactArgs &a, int mode, cudaStream_t st) {
@@ -489,10 +536,17 @@ cudaError_t read_clear_append_error(unsigned int *v) {
 
 cudaError_t launch_append(const AppendArgs &a, cudaStream_t st) {
     const int nkv = a.layers * a.pv.kv_heads;
-    dim3 grid((nkv + kAppendRows - 1) / kAppendRows, a.batch);
-    append_kernel<<<grid, kCompThreads, 0, st>>>(a);
+    dim3 grid(a.k_new ? (nkv + kAppendRows - 1) / kAppendRows : 1, a.batch);
+    cudaError_t e = launch_k(append_kernel, grid, dim3(kCompThreads), 0, st, a);
     note_launch();
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+cudaError_t launch_append_rows(const AppendArgs &a, cudaStream_t st) {
+    dim3 grid((a.pv.kv_heads + kAppendRows - 1) / kAppendRows, a.batch);
+    cudaError_t e = launch_k(append_rows_kernel, grid, dim3(kCompThreads), 0, st, a);
+    note_launch();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace ikv

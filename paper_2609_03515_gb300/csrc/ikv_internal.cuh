@@ -78,13 +78,22 @@ struct AttendArgs {
     int32_t batch, q_heads, layer0, n_layers;
     int32_t split_tokens, n_splits;
     float scale_log2;           // log2(e) / sqrt(d)
-    float *logits;              // [batch][n_layers][H][lstride] log2-domain logits, or null
+    float *logits;              // [batch][sc_layers][H][lstride] log2-domain logits, or null
     int32_t cap;
     int32_t lstride;            // logits row stride: cap rounded up to a multiple of 128
     float *part_ml;             // [batch][n_layers][H][n_splits][2]  (running max, sum) in log2 domain
     float *part_o;              // [batch][n_layers][H][n_splits][D]  unnormalised partial output
     const int32_t *pos;         // [rows][cap] with -1 at dead slots, or null (every slot below len live)
     int32_t rows_per_seq;       // utility rows per sequence (row of (b, g): b * rows_per_seq + g or b)
+    // logits and lse2 hold sc_layers layers per sequence; local layer li is their layer
+    // sc_layer0 + li (a per-layer launch writes into a whole step's arrays)
+    int32_t sc_layers, sc_layer0;
+    // tensor-core kernel, split step: the new token's rows of this (single) layer,
+    // [batch][kv_heads][D], stored into logical slot slot[b] (-1: none) before they are
+    // read; their V norms into vnorm (or null).  k_new null: no append.
+    const void *k_new, *v_new;
+    const int32_t *slot;
+    float *vnorm;
 };
 
 struct CombineArgs {
@@ -92,7 +101,8 @@ struct CombineArgs {
     int32_t batch, q_heads, n_layers, split_tokens, n_splits, head_dim;
     const float *part_ml, *part_o;
     void *out;                  // [n_layers][batch][H][D] (dtype)
-    float *lse2;                // [batch][n_layers][H] log2-sum-exp, or null
+    float *lse2;                // [batch][sc_layers][H] log2-sum-exp, or null
+    int32_t sc_layers, sc_layer0;
 };
 
 struct ScoreArgs {
@@ -127,7 +137,7 @@ int tc_max_split_tokens();
 // the tensor-core kernel also merges its splits (last CTA of each unit)
 struct TcOutputs {
     void *out;                  // [n_layers][batch][H][128] bf16
-    float *lse2;                // [batch][n_layers][H]
+    float *lse2;                // [batch][sc_layers][H]
     int32_t *arrivals;          // [batch][n_layers][kv_heads] zeroed before the launch
 };
 void tc_plan(int32_t max_len, int64_t units, int sms, int32_t *item_tiles, int32_t *n_chunks);
@@ -187,8 +197,14 @@ struct AppendArgs {
     int32_t dead_slots;         // the mean initialisation skips slots with pos < 0
     int32_t *done;              // [batch] arrival counters, zero on entry; reset by the last CTA
     float *vnorm;               // [layers][batch][kv_heads][cap]: the new row's norm is stored, or null
+    // split step: k_new == null makes launch_append do the bookkeeping only and record
+    // each sequence's reserved logical slot (-1: no room) in slot[b]; launch_append_rows
+    // then writes layer layer0's rows (k_new: [batch][kv_heads][D]) into that slot
+    int32_t layer0;
+    int32_t *slot;
 };
 cudaError_t launch_append(const AppendArgs &a, cudaStream_t st);
+cudaError_t launch_append_rows(const AppendArgs &a, cudaStream_t st);
 // reads and clears the append kernel's device error word (bit 0: no free slot)
 cudaError_t read_clear_append_error(unsigned int *v);
 

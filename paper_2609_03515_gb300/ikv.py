@@ -80,6 +80,9 @@ def _load():
         "ikv_append_token": ([SP, CP, P, P, P, I32, P, SZ, P], I32),
         "ikv_step_workspace_size": ([SP, CP, ctypes.POINTER(SZ)], I32),
         "ikv_step": ([SP, PP, CP, P, I32, P, P, P, P, P, SZ, P], I32),
+        "ikv_step_begin": ([SP, PP, CP, P, I32, P, SZ, P], I32),
+        "ikv_step_layer": ([SP, PP, CP, P, I32, I32, P, P, P, P, P, SZ, P], I32),
+        "ikv_step_end": ([SP, PP, CP, P, I32, P, SZ, P], I32),
     }
     for name, (args, res) in sigs.items():
         f = getattr(lib, name)
@@ -195,6 +198,22 @@ def ikv_step_workspace_size(shape, cache) -> int:
 def ikv_step(shape, params, cache, ema, t, q, k_new, v_new, out, ws, ws_bytes, stream=None) -> None:
     _check(_lib.ikv_step(ctypes.byref(shape), ctypes.byref(params), ctypes.byref(cache), _p(ema), t, _p(q), _p(k_new),
                          _p(v_new), _p(out), _p(ws), ws_bytes, _stream(stream)), "ikv_step")
+
+
+def ikv_step_begin(shape, params, cache, ema, t, ws, ws_bytes, stream=None) -> None:
+    _check(_lib.ikv_step_begin(ctypes.byref(shape), ctypes.byref(params), ctypes.byref(cache), _p(ema), t, _p(ws),
+                               ws_bytes, _stream(stream)), "ikv_step_begin")
+
+
+def ikv_step_layer(shape, params, cache, ema, t, layer, q, k_new, v_new, out, ws, ws_bytes, stream=None) -> None:
+    _check(_lib.ikv_step_layer(ctypes.byref(shape), ctypes.byref(params), ctypes.byref(cache), _p(ema), t, layer,
+                               _p(q), _p(k_new), _p(v_new), _p(out), _p(ws), ws_bytes, _stream(stream)),
+           "ikv_step_layer")
+
+
+def ikv_step_end(shape, params, cache, ema, t, ws, ws_bytes, stream=None) -> None:
+    _check(_lib.ikv_step_end(ctypes.byref(shape), ctypes.byref(params), ctypes.byref(cache), _p(ema), t, _p(ws),
+                             ws_bytes, _stream(stream)), "ikv_step_end")
 
 
 def raw_status(fn_name: str, *args) -> int:

@@ -120,10 +120,23 @@ def live_slots(pos_row: np.ndarray, n: int) -> np.ndarray:
     return np.nonzero(pos_row[:n] >= 0)[0]
 
 
+def decode_step(c: DecodeCache, p, cache, t: int, q, kn, vn, out, ws, per_layer: bool = False) -> None:
+    """One decode step through the C ABI: ikv_step, or its begin / per-layer / end split
+    (q, kn, vn, out: [layers][batch][...] device tensors)."""
+    if not per_layer:
+        ikv.ikv_step(c.shape(), p, cache, c.ema, t, q, kn, vn, out, ws, ws.numel())
+        return
+    ikv.ikv_step_begin(c.shape(), p, cache, c.ema, t, ws, ws.numel())
+    for l in range(c.layers):
+        ikv.ikv_step_layer(c.shape(), p, cache, c.ema, t, l, q[l], kn[l], vn[l], out[l], ws, ws.numel())
+    ikv.ikv_step_end(c.shape(), p, cache, c.ema, t, ws, ws.numel())
+
+
 def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: int = ikv.IKV_COMPACT_STABLE,
                  steps: Optional[int] = None, kv_check_layers=(0, -1), page_perm_seed: Optional[int] = 7,
                  refresh_init: int = ikv.IKV_INIT_ZERO, layer_eligible=None, max_holes: int = 0,
-                 agg_mode: int = ikv.IKV_AGG_EMA, scorer: int = ikv.IKV_SCORE_ATTENTION) -> List[StepReport]:
+                 agg_mode: int = ikv.IKV_AGG_EMA, scorer: int = ikv.IKV_SCORE_ATTENTION,
+                 per_layer: bool = False) -> List[StepReport]:
     T = w.steps if steps is None else steps
     u = w.u_table()
     c = make_cache(w, gran, page_perm_seed, value_norms=scorer == ikv.IKV_SCORE_VNORM)
@@ -151,8 +164,8 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
     R = c.rows_per_seq
     for t in range(1, T + 1):
         kn, vn = w.new_tokens(t, u)
-        ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, to_device(qs[t - 1], w), to_device(kn, w),
-                     to_device(vn, w), out, ws, ws.numel())
+        decode_step(c, p, c.cache(max(lens)), t, to_device(qs[t - 1], w), to_device(kn, w), to_device(vn, w), out,
+                    ws, per_layer)
         lens, live = step_lengths(lens, live, budgets, max_holes)
         torch.cuda.synchronize()
         out_h = out.float().cpu().numpy()
@@ -206,7 +219,7 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
 
 
 def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1), page_perm_seed: Optional[int] = 7,
-                         compact_mode: int = ikv.IKV_COMPACT_STABLE, max_holes: int = 0):
+                         compact_mode: int = ikv.IKV_COMPACT_STABLE, max_holes: int = 0, per_layer: bool = False):
     """Full-size lock-step for a few sequences of a workload (GRAN_SEQ).
 
     The GPU decodes the whole batch at its real size (device-generated prefill, the
@@ -237,8 +250,7 @@ def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1)
         assert gen.cuda_lib().ikvgen_fill_tokens_cuda(ctypes.byref(sp), u_dev.data_ptr(), L0_dev.data_ptr(), t, t + 1,
                                                       w.dtype, kn.data_ptr(), vn.data_ptr(),
                                                       torch.cuda.current_stream().cuda_stream) == 0
-        ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, to_device(qs[t - 1], w), kn[0], vn[0], out, ws,
-                     ws.numel())
+        decode_step(c, p, c.cache(max(lens)), t, to_device(qs[t - 1], w), kn[0], vn[0], out, ws, per_layer)
         lens, live = step_lengths(lens, live, budgets, max_holes)
         torch.cuda.synchronize()
         refresh = O.is_refresh(t, w.refresh_period, w.score_free)

@@ -97,6 +97,33 @@ def test_step_rejects_bad_schedule_and_workspace(lib):
                           16, 1 << 40, None) == lib.IKV_ERR_SHAPE
 
 
+def test_split_step_rejects_bad_arguments(lib):
+    """ikv_step_begin / _layer / _end check what ikv_step checks, plus the layer index."""
+    shp, cch = _shape(lib), _cache(lib)
+    p = lib.ikv_params()
+    p.alpha, p.refresh_period, p.budget = 0.9, 1, 16
+    P, S, C = ctypes.byref(p), ctypes.byref(shp), ctypes.byref(cch)
+    big = 1 << 40
+    assert lib.raw_status("ikv_step_begin", S, P, C, 16, 0, 16, big, None) == lib.IKV_ERR_ARG    # t is 1-based
+    assert lib.raw_status("ikv_step_begin", S, P, C, None, 1, 16, big, None) == lib.IKV_ERR_ARG  # no ema
+    assert lib.raw_status("ikv_step_begin", S, P, C, 16, 1, 16, 10, None) == lib.IKV_ERR_WORKSPACE
+    assert lib.raw_status("ikv_step_end", S, P, C, 16, 1, 0, 0, None) == lib.IKV_ERR_WORKSPACE
+    layer = lambda l, q=16, kn=16, out=16: lib.raw_status("ikv_step_layer", S, P, C, 16, 1, l, q, kn, 16, out, 16,
+                                                          big, None)
+    assert layer(2) == lib.IKV_ERR_ARG      # two layers: 0 and 1
+    assert layer(-1) == lib.IKV_ERR_ARG
+    assert layer(0, q=None) == lib.IKV_ERR_ARG
+    assert layer(0, kn=None) == lib.IKV_ERR_ARG
+    assert layer(1, out=8) == lib.IKV_ERR_ALIGN
+    p.refresh_period = 0
+    for fn in ("ikv_step_begin", "ikv_step_end"):
+        assert lib.raw_status(fn, S, P, C, 16, 1, 16, big, None) == lib.IKV_ERR_ARG
+    assert layer(0) == lib.IKV_ERR_ARG
+    p.refresh_period = 1
+    full = _cache(lib, max_len=256)  # no free slot for the new token
+    assert lib.raw_status("ikv_step_begin", S, P, ctypes.byref(full), 16, 1, 16, big, None) == lib.IKV_ERR_SHAPE
+
+
 def test_deferred_compaction_arguments(lib):
     shp, cch = _shape(lib), _cache(lib)
     p = lib.ikv_params()

@@ -70,3 +70,15 @@ def test_config4_every_step_compaction():
     # the same workload with compaction on every eviction and the always-left stable shift
     w = gen.config(4).with_(budget_frac=0.1)
     _check(run_fullsize_sampled(w, seqs=[0], steps=3, compact_mode=ikv.IKV_COMPACT_STABLE))
+
+
+@pytest.mark.timeout(1200)
+def test_config2_per_layer_split():
+    # the same workload stepped through ikv_step_begin / one ikv_step_layer per layer / ikv_step_end
+    w = gen.config(2)
+    _check(run_fullsize_sampled(w, seqs=[3], steps=5, compact_mode=SHORT, max_holes=bench_holes(w), per_layer=True))
+
+
+@pytest.mark.timeout(1200)
+def test_config1_per_layer_split():
+    _check(run_fullsize_sampled(gen.config(1), seqs=[0], steps=3, compact_mode=SHORT, max_holes=3, per_layer=True))

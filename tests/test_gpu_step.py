@@ -1,4 +1,5 @@
-"""Whole decode steps (ikv_step) in lock-step with the oracle (GPU only).
+"""Whole decode steps (ikv_step, or its begin / per-layer / end split) in lock-step
+with the oracle (GPU only).
 
 Each case runs several decode steps, with eviction on every step, and checks
 per step: attention outputs (bf16: 2e-2, fp32: 1e-4 absolute), utilities of
@@ -11,7 +12,7 @@ import pytest
 import torch
 
 import gen
-from harness import run_lockstep
+from harness import decode_step, make_cache, fill_host, run_lockstep, to_device
 from paper_2609_03515_gb300 import ikv
 
 pytestmark = pytest.mark.gpu
@@ -144,3 +145,60 @@ def test_vnorm_and_entropy_scorers():
     _assert(run_lockstep(small_llama(steps=8, score_free=True), scorer=ent, max_holes=4), 2e-2)
     _assert(run_lockstep(small_llama(steps=6), scorer=ent, gran=ikv.IKV_GRAN_KVHEAD,
                          agg_mode=ikv.IKV_AGG_CUMULATIVE), 2e-2)
+
+
+def test_per_layer_split_trajectories():
+    """ikv_step_begin, one ikv_step_layer per layer, ikv_step_end: the model-integration
+    form of the step (Appendix "Layer scoring": scores folded layer by layer inside the
+    forward pass), in lock-step with the oracle across schedules, row granularities,
+    compaction modes, deferral, aggregation rules and scorers."""
+    vn, ent = ikv.IKV_SCORE_VNORM, ikv.IKV_SCORE_ENTROPY
+    _assert(run_lockstep(gen.config(0), per_layer=True), 1e-4, strict_fraction=1.0)
+    _assert(run_lockstep(gen.config(0), max_holes=3, scorer=ent, per_layer=True), 1e-4, strict_fraction=1.0)
+    _assert(run_lockstep(small_llama(steps=8), per_layer=True), 2e-2)
+    _assert(run_lockstep(small_llama(steps=9, refresh_period=4), compact_mode=ikv.IKV_COMPACT_STABLE_SHORT,
+                         max_holes=3, per_layer=True), 2e-2)
+    _assert(run_lockstep(small_llama(steps=6, score_free=True, page_size=16), max_holes=4, per_layer=True), 2e-2)
+    _assert(run_lockstep(small_llama(steps=6), gran=ikv.IKV_GRAN_KVHEAD, compact_mode=ikv.IKV_COMPACT_HOLEFILL,
+                         per_layer=True), 2e-2)
+    _assert(run_lockstep(small_llama(steps=6, layers=4), layer_eligible=[0, 1, 1, 0],
+                         refresh_init=ikv.IKV_INIT_MEAN, agg_mode=ikv.IKV_AGG_CUMULATIVE, per_layer=True), 2e-2)
+    _assert(run_lockstep(small_llama(steps=6), scorer=vn, max_holes=3, per_layer=True), 2e-2)
+    _assert(run_lockstep(small_llama(steps=6, refresh_period=2), scorer=ent, per_layer=True), 2e-2)
+    w = gen.Workload(name="qwen-small", batch=2, layers=2, q_heads=28, kv_heads=4, head_dim=128, prefill=[700, 260],
+                     steps=5, dtype=gen.BF16, alpha=0.9, seed=9, page_size=32)
+    _assert(run_lockstep(w, per_layer=True), 2e-2)
+
+
+def test_per_layer_split_equals_whole_step():
+    """The split step and ikv_step on the same inputs give bit-identical caches, utilities
+    and outputs when the attention is partitioned alike: at these lengths (at most 3 tiles
+    of 128 slots per unit) both give every tile its own split, so the two differ only in
+    how the launches are cut."""
+    w = small_llama(steps=6, refresh_period=2, prefill=[100, 180, 250])
+    u = w.u_table()
+    caches = []
+    for per_layer in (False, True):
+        c = make_cache(w)
+        fill_host(c, w, u)
+        caches.append(c)
+    p = [c.params(w.alpha, w.refresh_period, False, ikv.IKV_COMPACT_STABLE_SHORT, max_holes=3) for c in caches]
+    ws = [c.step_workspace() for c in caches]
+    qs = w.queries(1, w.steps + 1, u)
+    outs = [torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+            for _ in caches]
+    max_len = max(w.prefill)
+    for t in range(1, w.steps + 1):
+        kn, vn = w.new_tokens(t, u)
+        for i, c in enumerate(caches):
+            decode_step(c, p[i], c.cache(max_len), t, to_device(qs[t - 1], w), to_device(kn, w), to_device(vn, w),
+                        outs[i], ws[i], per_layer=i == 1)
+        torch.cuda.synchronize()
+        a, b = caches
+        assert torch.equal(a.len, b.len) and torch.equal(a.start, b.start) and torch.equal(a.pos, b.pos), t
+        assert torch.equal(a.next_pos, b.next_pos), t
+        assert torch.equal(a.k, b.k) and torch.equal(a.v, b.v), t
+        assert torch.equal(a.ema, b.ema), t
+        assert torch.equal(outs[0], outs[1]), t
+        max_len = int(a.len.max())
+    assert ikv.ikv_device_status() == 0
