@@ -42,6 +42,15 @@ Readings taken where the paper is silent (each also stated where it is used):
 * R6 (self-attention): the appended token is part of its own step's softmax.
 * R7 (scale): softmax scale ``1/sqrt(d)``; keys are used as stored.
 * R8 (eligible layers): all layers unless a layer mask says otherwise.
+* R10 (per-layer immediate eviction, the Appendix "Layer scoring" hook read
+  literally): every layer, right after its own update of the state, evicts down
+  to the budget from the tokens that layer holds, by the state as it stands then
+  (m_{t,l}).  Layers then hold different token sets, so the state is indexed by
+  token position and shared by all layers.  A layer's update covers every live
+  position (held by at least one layer): a token the layer does not hold got no
+  attention there, so its score is 0 (Eq. 1) and Eq. 4 decays it.  The new
+  token's mean initialisation on non-refresh steps averages over the live
+  positions.  With one layer this is the base method exactly.
 * R9 (scorer variants, Appendix "Per-step scoring"): VNorm divides each value
   row's l2 norm by the mean norm over the cached tokens of its (layer, KV head);
   entropy weighting uses the normalized entropy H(s) / ln n of the layer's
@@ -341,3 +350,99 @@ def decode_step(st: SeqState, t: int, q_t: np.ndarray, k_new: np.ndarray, v_new:
     out = attend_and_score(st, q_t, refresh, p)
     evict(st)
     return out
+
+
+# --------------------------------------------------------------------------
+# Per-layer immediate eviction (reading R10)
+# --------------------------------------------------------------------------
+@dataclass
+class LayerwiseState:
+    """One sequence under per-layer eviction: layer l holds the tokens pos[l] (ascending
+    positions, slot order) with rows K[l][g], V[l][g] ([len(pos[l]), d]); m[p] is the
+    shared state of position p (every position ever appended; only live ones matter)."""
+
+    K: List[List[np.ndarray]]
+    V: List[List[np.ndarray]]
+    pos: List[np.ndarray]
+    m: np.ndarray
+    budget: int
+    next_pos: int
+
+    @property
+    def layers(self) -> int:
+        return len(self.K)
+
+    @property
+    def kv_heads(self) -> int:
+        return len(self.K[0])
+
+    def live(self) -> np.ndarray:
+        """Positions held by at least one layer, ascending."""
+        return np.unique(np.concatenate(self.pos))
+
+
+def layerwise_prefill_state(K, V, budget: int) -> LayerwiseState:
+    layers, kv = len(K), len(K[0])
+    L0 = K[0][0].shape[0]
+    return LayerwiseState(
+        K=[[np.array(K[l][g], np.float64) for g in range(kv)] for l in range(layers)],
+        V=[[np.array(V[l][g], np.float64) for g in range(kv)] for l in range(layers)],
+        pos=[np.arange(L0, dtype=np.int64) for _ in range(layers)],
+        m=np.zeros(L0), budget=budget, next_pos=L0)
+
+
+@dataclass
+class LayerTrace:
+    """What layer l's eviction saw: its held positions and their state m_{t,l}."""
+    pos: np.ndarray
+    m: np.ndarray
+    kept: np.ndarray
+
+
+def decode_step_layerwise(st: LayerwiseState, t: int, q_t: np.ndarray, k_new: np.ndarray, v_new: np.ndarray,
+                          p: Params, keep_override=None):
+    """One decode step under per-layer immediate eviction (reading R10).
+
+    q_t: [layers][H][d]; k_new, v_new: [layers][H_kv][d].  keep_override(l, trace) may
+    return the positions layer l keeps instead of its own top-B choice (lock-step tests).
+    Returns (attention outputs [layers][H][d], [LayerTrace per layer])."""
+    refresh = is_refresh(t, p.refresh_period, p.score_free)
+    # append: every layer gets the new token; its state is 0 on refresh steps (R3),
+    # else the mean over the live positions (Appendix "New token insertion", R10)
+    live = st.live()
+    if refresh and p.refresh_init == "zero":
+        init = 0.0
+    else:
+        init = float(np.mean(st.m[live])) if live.size else 0.0
+    st.m = np.append(st.m, init)
+    for l in range(st.layers):
+        for g in range(st.kv_heads):
+            st.K[l][g] = np.vstack([st.K[l][g], np.asarray(k_new[l][g], np.float64)[None]])
+            st.V[l][g] = np.vstack([st.V[l][g], np.asarray(v_new[l][g], np.float64)[None]])
+        st.pos[l] = np.append(st.pos[l], st.next_pos)
+    st.next_pos += 1
+    outs, traces = [], []
+    for l in range(st.layers):
+        a, o = last_query_attention(q_t[l], st.K[l], st.V[l])
+        outs.append(o)
+        eligible = p.layer_mask is None or p.layer_mask[l]
+        if refresh and eligible:
+            # Eq. 1 over the layer's own tokens; 0 for live positions it does not hold
+            s_pos = np.zeros_like(st.m)
+            s_pos[st.pos[l]] = pooled_score(a, GRAN_SEQ, st.kv_heads)[0]
+            live = st.live()
+            st.m[live] = ema_update(st.m[live], s_pos[live], p.alpha)
+        m_l = st.m[st.pos[l]]
+        keep = select_keep(m_l, st.budget)
+        tr = LayerTrace(pos=st.pos[l].copy(), m=m_l.copy(), kept=st.pos[l][keep])
+        if keep_override is not None:
+            kp = keep_override(l, tr)
+            if kp is not None:
+                keep = np.searchsorted(st.pos[l], np.sort(np.asarray(kp, np.int64)))
+                tr.kept = st.pos[l][keep]
+        traces.append(tr)
+        st.pos[l] = st.pos[l][keep]
+        for g in range(st.kv_heads):
+            st.K[l][g] = st.K[l][g][keep]
+            st.V[l][g] = st.V[l][g][keep]
+    return np.stack(outs), traces

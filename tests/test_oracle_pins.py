@@ -545,3 +545,122 @@ def test_new_token_can_be_evicted_same_step():
     O.append_token(st, np.zeros((1, 1, 2)), np.zeros((1, 1, 2)), False, O.Params())
     O.evict(st)  # mean 1.0 ties every survivor; the new token holds the highest slot
     assert st.pos[0].tolist() == [0, 1, 2, 4]
+
+
+# ------------------------------------------------ per-layer immediate eviction (R10)
+def _layerwise_from(st):
+    return O.layerwise_prefill_state([[k.copy() for k in row] for row in st.K],
+                                     [[v.copy() for v in row] for row in st.V], st.budget)
+
+
+@pytest.mark.parametrize("r,sf", [(1, False), (3, False), (1, True)])
+def test_layerwise_with_one_layer_is_the_base_method(r, sf):
+    """One layer: the per-layer eviction after the layer's update is the step-end eviction,
+    and every live position is held by that layer -- identical to decode_step."""
+    rng = np.random.default_rng(11)
+    base = _rand_state(rng, layers=1, kv=2, L0=30, budget=9)
+    lw = _layerwise_from(base)
+    p = O.Params(alpha=0.8, refresh_period=r, score_free=sf)
+    q, kn, vn = _rand_inputs(rng, 8, layers=1)
+    for t in range(1, 9):
+        o_base = O.decode_step(base, t, q[t - 1], kn[t - 1], vn[t - 1], p)
+        o_lw, _ = O.decode_step_layerwise(lw, t, q[t - 1], kn[t - 1], vn[t - 1], p)
+        assert np.array_equal(o_base, o_lw)
+        assert np.array_equal(base.pos[0], lw.pos[0])
+        assert np.array_equal(base.m[0], lw.m[lw.pos[0]])
+
+
+def _worked_example(refresh_period):
+    """Two layers, one head, d = 1, q = 1 (so each logit is the key itself), budget 2,
+    alpha 1/2, prefill positions 0 and 1; tokens 2 and 3 arrive at steps 1 and 2.
+    Keys are logs of small integers, so every softmax is a ratio of integers:
+        layer 0: positions 0..3 -> ln 1, ln 2, ln 3, ln 1
+        layer 1: positions 0..3 -> ln 3, ln 2, ln 2, ln 6
+    Values: v = 10 * layer + position (one dimension)."""
+    lnk = [[math.log(1), math.log(2), math.log(3), math.log(1)], [math.log(3), math.log(2), math.log(2), math.log(6)]]
+    K = [[np.array([[lnk[l][0]], [lnk[l][1]]])] for l in range(2)]
+    V = [[np.array([[10.0 * l + 0], [10.0 * l + 1]])] for l in range(2)]
+    st = O.layerwise_prefill_state(K, V, budget=2)
+    p = O.Params(alpha=0.5, refresh_period=refresh_period)
+    steps = []
+    for t, newp in ((1, 2), (2, 3)):
+        q = np.ones((2, 1, 1))
+        kn = np.array([[[lnk[l][newp]]] for l in range(2)])
+        vn = np.array([[[10.0 * l + newp]] for l in range(2)])
+        out, tr = O.decode_step_layerwise(st, t, q, kn, vn, p)
+        steps.append((out, tr, [x.copy() for x in st.pos], st.m.copy()))
+    return steps
+
+
+def test_layerwise_worked_example_full_refresh():
+    """Hand-derived from Eq. 1, Eq. 4 and reading R10.
+    Step 1, layer 0 attends [0,1,2] with weights 1:2:3, so m = (1/12, 2/12, 3/12) and it keeps
+    {1, 2}.  Layer 1 attends [0,1,2] with 3:2:2 (the position layer 0 dropped is still live
+    through layer 1): m = m/2 + (3/14, 1/7, 1/7) = (43, 38, 45)/168; it keeps {0, 2}.
+    Step 2 appends 3 with m = 0.  Layer 0 attends [1,2,3] with 2:3:1; position 0 (held only by
+    layer 1) gets score 0 and decays: m = (43, 94, 129, 28)/336; layer 0 keeps {1, 2}.
+    Layer 1 attends [0,2,3] with 3:2:6 (position 1, held only by layer 0, decays):
+    m = (1481, 1034, 2091, 2324)/7392; layer 1 keeps {2, 3}."""
+    (o1, tr1, pos1, m1), (o2, tr2, pos2, m2) = _worked_example(1)
+    assert [list(x) for x in pos1] == [[1, 2], [0, 2]]
+    np.testing.assert_allclose(tr1[0].m, np.array([1, 2, 3]) / 12, rtol=1e-15)
+    np.testing.assert_allclose(m1, np.array([43, 38, 45]) / 168, rtol=1e-15)
+    assert [list(x) for x in pos2] == [[1, 2], [2, 3]]
+    np.testing.assert_allclose(tr2[0].m, np.array([94, 129, 28]) / 336, rtol=1e-15)
+    np.testing.assert_allclose(m2, np.array([1481, 1034, 2091, 2324]) / 7392, rtol=1e-15)
+    # outputs: softmax-weighted values of each layer's held tokens at attention time
+    np.testing.assert_allclose(o1[0, 0, 0], (1 * 0 + 2 * 1 + 3 * 2) / 6, rtol=1e-15)
+    np.testing.assert_allclose(o1[1, 0, 0], (3 * 10 + 2 * 11 + 2 * 12) / 7, rtol=1e-15)
+    np.testing.assert_allclose(o2[0, 0, 0], (2 * 1 + 3 * 2 + 1 * 3) / 6, rtol=1e-15)
+    np.testing.assert_allclose(o2[1, 0, 0], (3 * 10 + 2 * 12 + 6 * 13) / 11, rtol=1e-15)
+
+
+def test_layerwise_worked_example_lazy_mean_init():
+    """Refresh period 2: step 2 carries the state; the new token starts at the mean over the
+    live positions {0, 1, 2} (position 0 is held by layer 1 only): (43+38+45)/(3*168) = 42/168.
+    Layer 0 then keeps {2, 3} from (38, 45, 42)/168 and layer 1 keeps {0, 2} from (43, 45, 42)/168."""
+    (_, _, pos1, m1), (_, tr2, pos2, m2) = _worked_example(2)
+    assert [list(x) for x in pos1] == [[1, 2], [0, 2]]
+    np.testing.assert_allclose(m2, np.array([43, 38, 45, 42]) / 168, rtol=1e-15)
+    assert [list(x) for x in pos2] == [[2, 3], [0, 2]]
+    np.testing.assert_allclose(tr2[1].m, np.array([43, 45, 42]) / 168, rtol=1e-15)
+
+
+def test_layerwise_alpha_one_keeps_the_oldest_everywhere():
+    """alpha = 1: Eq. 4 never moves the state, refresh steps give new tokens 0, so every layer
+    ranks all-equal utilities and keeps its lowest slots (R4) -- the B oldest positions, in
+    every layer, as the base method does."""
+    rng = np.random.default_rng(5)
+    base = _rand_state(rng, layers=3, kv=2, L0=20, budget=7)
+    lw = _layerwise_from(base)
+    p = O.Params(alpha=1.0)
+    q, kn, vn = _rand_inputs(rng, 5, layers=3)
+    for t in range(1, 6):
+        O.decode_step(base, t, q[t - 1], kn[t - 1], vn[t - 1], p)
+        O.decode_step_layerwise(lw, t, q[t - 1], kn[t - 1], vn[t - 1], p)
+        for l in range(3):
+            assert list(lw.pos[l]) == list(range(7)) == list(base.pos[0])
+
+
+def test_layerwise_invariants():
+    """Every layer holds min(L, B) tokens in ascending position order, drawn from what it held
+    plus the new token; each layer's choice is the top B of its held tokens by the state it
+    saw (R4 ties); live positions are exactly the union of the layers' sets."""
+    rng = np.random.default_rng(8)
+    base = _rand_state(rng, layers=4, kv=2, L0=25, budget=8)
+    lw = _layerwise_from(base)
+    p = O.Params(alpha=0.7, refresh_period=2)
+    q, kn, vn = _rand_inputs(rng, 10, layers=4)
+    diverged = False
+    for t in range(1, 11):
+        before = [set(x.tolist()) | {lw.next_pos} for x in lw.pos]
+        _, tr = O.decode_step_layerwise(lw, t, q[t - 1], kn[t - 1], vn[t - 1], p)
+        for l in range(4):
+            held = lw.pos[l]
+            assert len(held) == 8 and np.all(np.diff(held) > 0)
+            assert set(held.tolist()) <= before[l]
+            order = sorted(range(len(tr[l].m)), key=lambda i: (-tr[l].m[i], i))[:8]
+            assert set(tr[l].pos[order].tolist()) == set(held.tolist())
+        assert set(lw.live().tolist()) == set().union(*[set(x.tolist()) for x in lw.pos])
+        diverged |= len({tuple(x) for x in lw.pos}) > 1
+    assert diverged  # the layers' sets do part ways on this input
