@@ -48,6 +48,10 @@
  *  (rows = batch * kv_heads, row index b * kv_heads + g), the score averages
  *  that KV head's query group, and the kept set applies to that KV head in
  *  every layer.  ema, pos and keep arrays are [rows][cap].
+ *  Per-layer eviction (ikv_params.evict_mode = IKV_EVICT_LAYER, IKV_GRAN_SEQ):
+ *  every layer keeps its own token set, so pos is [batch][layers][cap] (row
+ *  b * layers + l lists layer l's positions by slot) and the utility is one
+ *  state per token position: ema is [batch][pos_cap], indexed by position.
  */
 #ifndef IKV_H
 #define IKV_H
@@ -83,6 +87,10 @@ enum { IKV_AGG_EMA = 0, IKV_AGG_CUMULATIVE = 1, IKV_AGG_SINGLE_STEP = 2 };
  * its (layer, kv head)); entropy weighting (each layer's pooled score times the
  * normalized entropy H(s) / ln n of that score over the n live slots, 1 if n = 1). */
 enum { IKV_SCORE_ATTENTION = 0, IKV_SCORE_VNORM = 1, IKV_SCORE_ENTROPY = 2 };
+/* When tokens are evicted: once per step after the last layer, one kept set for every
+ * layer (default); or by every layer right after its own update of the state, from the
+ * tokens that layer holds (Appendix "Layer scoring" hooks; layers' sets then differ). */
+enum { IKV_EVICT_STEP = 0, IKV_EVICT_LAYER = 1 };
 
 typedef struct {
     int32_t batch, layers, q_heads, kv_heads, head_dim;
@@ -113,6 +121,9 @@ typedef struct {
                                     when set, ikv_append_token / ikv_step store the new row's norm and
                                     compaction moves the norms with their rows.  Fill it once for the
                                     prefill with ikv_value_norms. */
+    int32_t pos_cap;             /* per-layer eviction: token positions the position-indexed state
+                                    holds (ema is [batch][pos_cap]; every next_pos[b] must stay below
+                                    it); sizes the step workspace.  0 otherwise. */
 } ikv_cache;
 
 /* Optional per-kernel CUDA events recorded on the call's stream by ikv_step
@@ -151,6 +162,14 @@ typedef struct {
                                        IKV_AGG_SINGLE_STEP m = s (Eq. 2) */
     int32_t scorer;                 /* IKV_SCORE_ATTENTION (Eq. 1, default) | IKV_SCORE_VNORM (needs
                                        cache->vnorm) | IKV_SCORE_ENTROPY */
+    int32_t evict_mode;             /* IKV_EVICT_STEP (default) | IKV_EVICT_LAYER: each layer, after
+                                       folding its score into the position-indexed state, keeps the
+                                       budget[b] highest-utility tokens it holds and compacts its own
+                                       rows.  A live position a layer does not hold scores 0 there, so
+                                       its state decays by alpha (Eq. 1, Eq. 4); the mean initialisation
+                                       averages the positions some layer holds.  Needs IKV_GRAN_SEQ,
+                                       IKV_COMPACT_STABLE, max_holes 0, IKV_AGG_EMA, IKV_SCORE_ATTENTION,
+                                       cache->pos_cap > 0 and the layout described under "Utility rows". */
 } ikv_params;
 
 /* Message for the last error on this thread ("" if none). */
@@ -163,7 +182,9 @@ int64_t ikv_launch_count(void);
  * the device).  0 = no error.  Bit 0: a bounded wait inside the tensor-core
  * attention kernel ran out (the kernel abandoned its work and returned);
  * bit 1: a split longer than the kernel's TMEM budget reached the device;
- * bit 2: an append found no free slot (start + len = cap) and was dropped. */
+ * bit 2: an append found no free slot (start + len = cap) and was dropped;
+ * bit 3: per-layer eviction, a sequence's next_pos reached cache->pos_cap (the token
+ * was dropped). */
 ikv_status ikv_device_status(uint32_t *flags);
 
 /* Which decode-attention kernel ikv_decode_attend_score and ikv_step launch for

@@ -56,13 +56,15 @@ class DecodeCache:
     block_table: [batch][max_pages] int32 physical page of each logical page
     len:         [batch] int32 slots in use (dead slots included);  next_pos: [batch] int32
     pos, ema:    [rows][cap] int32 / fp32, rows = batch (per-sequence state) or batch * kv_heads;
-                 pos = -1 marks a dead slot (deferred compaction)
+                 pos = -1 marks a dead slot (deferred compaction).  With pos_cap > 0 (per-layer
+                 eviction): pos is [batch * layers][cap] and ema [batch][pos_cap], by position
     budget:      [batch] int32
     """
 
     def __init__(self, batch: int, layers: int, q_heads: int, kv_heads: int, head_dim: int, cap_tokens: int,
                  dtype: int = ikv.IKV_BF16, page_size: int = 64, granularity: int = ikv.IKV_GRAN_SEQ,
-                 device: str = "cuda", page_perm_seed: Optional[int] = None, value_norms: bool = False):
+                 device: str = "cuda", page_perm_seed: Optional[int] = None, value_norms: bool = False,
+                 pos_cap: int = 0):
         self.batch, self.layers, self.q_heads, self.kv_heads, self.head_dim = batch, layers, q_heads, kv_heads, head_dim
         self.dtype, self.granularity, self.page_size = dtype, granularity, page_size
         self.max_pages = (cap_tokens + page_size - 1) // page_size
@@ -81,8 +83,12 @@ class DecodeCache:
         self.rows = batch if granularity == ikv.IKV_GRAN_SEQ else batch * kv_heads
         self.len = torch.zeros(batch, dtype=torch.int32, device=device)
         self.next_pos = torch.zeros(batch, dtype=torch.int32, device=device)
-        self.pos = torch.zeros((self.rows, self.cap), dtype=torch.int32, device=device)
-        self.ema = torch.zeros((self.rows, self.cap), dtype=torch.float32, device=device)
+        # per-layer eviction (pos_cap > 0): a position row per (sequence, layer) and the
+        # utility state indexed by token position
+        self.pos_cap = pos_cap
+        pos_rows = batch * layers if pos_cap > 0 else self.rows
+        self.pos = torch.zeros((pos_rows, self.cap), dtype=torch.int32, device=device)
+        self.ema = torch.zeros((self.rows, pos_cap if pos_cap > 0 else self.cap), dtype=torch.float32, device=device)
         self.budget = torch.zeros(batch, dtype=torch.int32, device=device)
         self.start = torch.zeros(batch, dtype=torch.int32, device=device)
         # per-slot value-row norms, for the VNorm scorer
@@ -100,7 +106,7 @@ class DecodeCache:
         return ikv.ikv_cache(self.k.data_ptr(), self.v.data_ptr(), self.block_table.data_ptr(), self.num_pages,
                              self.page_size, self.max_pages, self.len.data_ptr(), self.pos.data_ptr(),
                              self.next_pos.data_ptr(), ml, self.start.data_ptr(), 1 if dead_slots else 0,
-                             self.vnorm.data_ptr() if self.vnorm is not None else None)
+                             self.vnorm.data_ptr() if self.vnorm is not None else None, self.pos_cap)
 
     @property
     def rows_per_seq(self) -> int:
@@ -114,7 +120,7 @@ class DecodeCache:
         self.next_pos.copy_(self.len)
         self.budget.copy_(torch.tensor(list(budgets), dtype=torch.int32, device=dev))
         ar = torch.arange(self.cap, dtype=torch.int32, device=dev)
-        self.pos.copy_(ar.expand(self.rows, self.cap))
+        self.pos.copy_(ar.expand(self.pos.shape[0], self.cap))
         self.ema.zero_()
         self.start.zero_()
         self.max_len = max(lengths)
@@ -143,7 +149,8 @@ class DecodeCache:
     def params(self, alpha: float, refresh_period: int = 1, score_free: bool = False,
                compact_mode: int = ikv.IKV_COMPACT_STABLE, refresh_init: int = ikv.IKV_INIT_ZERO,
                layer_eligible: Optional[Sequence[int]] = None, max_holes: int = 0,
-               agg_mode: int = ikv.IKV_AGG_EMA, scorer: int = ikv.IKV_SCORE_ATTENTION) -> ikv.ikv_params:
+               agg_mode: int = ikv.IKV_AGG_EMA, scorer: int = ikv.IKV_SCORE_ATTENTION,
+               evict_mode: int = ikv.IKV_EVICT_STEP) -> ikv.ikv_params:
         p = ikv.ikv_params()
         p.alpha = alpha
         p.refresh_period = refresh_period
@@ -157,6 +164,7 @@ class DecodeCache:
         p.max_holes = max_holes
         p.agg_mode = agg_mode
         p.scorer = scorer
+        p.evict_mode = evict_mode
         return p
 
 

@@ -131,10 +131,10 @@ AttendWs attend_ws(const ikv_shape *s, int32_t cap, int n_layers, bool logits) {
 
 struct StepWs {
     AttendWs at;
-    size_t keep, keep_len, done, cdone, moves, n_moves, sbuf, epart, vmean, slot, end;
+    size_t keep, keep_len, done, cdone, moves, n_moves, sbuf, epart, vmean, slot, lam, util, end;
 };
 
-StepWs step_ws(const ikv_shape *s, int32_t cap) {
+StepWs step_ws(const ikv_shape *s, int32_t cap, int32_t pos_cap) {
     StepWs w;
     w.at = attend_ws(s, cap, s->layers, true);
     size_t off = w.at.end;
@@ -160,6 +160,11 @@ StepWs step_ws(const ikv_shape *s, int32_t cap) {
     off = align256(off + (size_t)s->batch * s->layers * s->kv_heads * sizeof(float));
     w.slot = off;  // split step: each sequence's reserved slot
     off = align256(off + (size_t)s->batch * sizeof(int32_t));
+    // per-layer eviction: pending-update marks by position, one layer's utilities by slot
+    w.lam = off;
+    if (pos_cap > 0) off = align256(off + (size_t)s->batch * pos_cap * sizeof(int32_t));
+    w.util = off;
+    if (pos_cap > 0) off = align256(off + (size_t)s->batch * cap * sizeof(float));
     w.end = off;
     return w;
 }
@@ -451,7 +456,7 @@ ikv_status ikv_compact_workspace_size(const ikv_shape *shape, const ikv_cache *c
 
 static ikv_status compact_impl(const ikv_shape *shape, ikv_cache *cache, const int32_t *keep, const int32_t *keep_len,
                                float *ema, int32_t mode, int32_t *moves, int32_t *n_moves, int32_t *done,
-                               cudaStream_t stream, int32_t max_holes = 0) {
+                               cudaStream_t stream, int32_t max_holes = 0, int32_t layer = -1) {
     CompactArgs a{};
     a.k = cache->k;
     a.v = cache->v;
@@ -473,6 +478,15 @@ static ikv_status compact_impl(const ikv_shape *shape, ikv_cache *cache, const i
     a.n_moves = n_moves;
     a.max_holes = max_holes;
     a.vnorm = cache->vnorm;
+    a.pos_rows = a.rows_per_seq;
+    a.publish_len = 1;
+    if (layer >= 0) {  // per-layer eviction: that layer's rows and position row; len published later
+        a.layers = 1;
+        a.layer0 = layer;
+        a.pos_rows = shape->layers;
+        a.pos_row0 = layer;
+        a.publish_len = 0;
+    }
     IKV_TRY_CUDA(launch_compact(a, mode, stream), "compact launch");
     return IKV_OK;
 }
@@ -551,7 +565,7 @@ struct StepCtx {
     ikv_cache cv;
     StepWs w;
     int32_t cap, L1, init_mean;
-    bool scoring;
+    bool scoring, layerwise;
     int32_t elig[kMaxLayers];
     int n_elig;
     ScorerWs sw;
@@ -580,12 +594,23 @@ static ikv_status prepare_step(const ikv_shape *shape, const ikv_params *p, cons
     if (p->scorer != IKV_SCORE_ATTENTION && p->scorer != IKV_SCORE_VNORM && p->scorer != IKV_SCORE_ENTROPY)
         return fail(IKV_ERR_ARG, "unknown scorer %d", p->scorer);
     if (p->scorer == IKV_SCORE_VNORM && !cache->vnorm) return fail(IKV_ERR_ARG, "IKV_SCORE_VNORM needs cache->vnorm");
+    cx->layerwise = p->evict_mode == IKV_EVICT_LAYER;
+    if (p->evict_mode != IKV_EVICT_STEP && !cx->layerwise) return fail(IKV_ERR_ARG, "unknown evict_mode %d", p->evict_mode);
+    if (cx->layerwise) {
+        if (shape->granularity != IKV_GRAN_SEQ || p->compact_mode != IKV_COMPACT_STABLE || p->max_holes != 0 ||
+            p->agg_mode != IKV_AGG_EMA || p->scorer != IKV_SCORE_ATTENTION)
+            return fail(IKV_ERR_UNSUPPORTED,
+                        "IKV_EVICT_LAYER needs IKV_GRAN_SEQ, IKV_COMPACT_STABLE, max_holes 0, IKV_AGG_EMA and "
+                        "IKV_SCORE_ATTENTION");
+        if (cache->pos_cap <= 0) return fail(IKV_ERR_ARG, "IKV_EVICT_LAYER needs cache->pos_cap > 0");
+        if (cache->dead_slots) return fail(IKV_ERR_ARG, "IKV_EVICT_LAYER does not use dead slots");
+    }
     // with deferred compaction every kernel of the step treats pos < 0 as a dead slot
     cx->cv = *cache;
     if (p->max_holes > 0) cx->cv.dead_slots = 1;
     cx->cap = cap_of(cache);
     if (cache->max_len + 1 > cx->cap) return fail(IKV_ERR_SHAPE, "no free slot: max_len + 1 > cap");
-    cx->w = step_ws(shape, cx->cap);
+    cx->w = step_ws(shape, cx->cap, cache->pos_cap);
     if (!ws || ws_bytes < cx->w.end) return fail(IKV_ERR_WORKSPACE, "workspace needs %zu bytes", cx->w.end);
     const bool refresh = p->score_free ? (t == 1) : ((t - 1) % p->refresh_period == 0);
     cx->n_elig = 0;
@@ -616,13 +641,71 @@ static ikv_status evict_impl(const ikv_shape *shape, const ikv_params *p, ikv_ca
                         p->max_holes);
 }
 
+// Per-layer eviction: the arguments every layer-wise kernel of a step shares.
+static LayerArgs layer_args(const ikv_shape *shape, const ikv_params *p, const ikv_cache *cache, float *ema, void *ws,
+                            const StepCtx &cx) {
+    LayerArgs a{};
+    a.batch = shape->batch;
+    a.layers = shape->layers;
+    a.q_heads = shape->q_heads;
+    a.cap = cx.cap;
+    a.pos_cap = cache->pos_cap;
+    a.len = cache->len;
+    a.next_pos = cache->next_pos;
+    a.pos = cache->pos;
+    a.start = cache->start;
+    a.m = ema;
+    a.lam = at<int32_t>(ws, cx.w.lam);
+    a.util = at<float>(ws, cx.w.util);
+    a.logits = at<float>(ws, cx.w.at.logits);
+    a.lse2 = at<float>(ws, cx.w.at.lse2);
+    a.sc_layers = shape->layers;
+    a.lstride = logit_stride(cx.cap);
+    a.alpha = p->alpha;
+    a.init_mean = cx.init_mean;
+    a.slot = at<int32_t>(ws, cx.w.slot);
+    a.keep_len = at<int32_t>(ws, cx.w.keep_len);
+    return a;
+}
+
+// Per-layer eviction of one layer after its attention: its utilities (with its score
+// folded in on scoring layers), its top-budget selection and the compaction of its rows.
+static ikv_status evict_layer(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, void *ws,
+                              const StepCtx &cx, int32_t layer, cudaStream_t stream) {
+    LayerArgs la = layer_args(shape, p, cache, ema, ws, cx);
+    int k_done = 0;
+    bool eligible = false;
+    for (int k = 0; k < cx.n_elig; ++k) {
+        if (cx.elig[k] < layer) ++k_done;
+        eligible |= cx.elig[k] == layer;
+    }
+    la.layer = layer;
+    la.k_done = cx.scoring ? k_done : 0;
+    la.scoring = cx.scoring && eligible;
+    IKV_TRY_CUDA(launch_layer_util(la, cx.L1, stream), "layer utility launch");
+    IKV_TRY_CUDA(launch_select(shape->batch, cx.cap, la.util, cache->len, 1, p->budget, nullptr,
+                               at<int32_t>(ws, cx.w.keep), at<int32_t>(ws, cx.w.keep_len), DeferArgs{0, cx.cap, nullptr},
+                               stream),
+                 "select launch");
+    return compact_impl(shape, cache, at<int32_t>(ws, cx.w.keep), at<int32_t>(ws, cx.w.keep_len), nullptr,
+                        IKV_COMPACT_STABLE, nullptr, nullptr, at<int32_t>(ws, cx.w.cdone), stream, 0, layer);
+}
+
+static ikv_status layer_end(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, void *ws,
+                            const StepCtx &cx, cudaStream_t stream) {
+    LayerArgs la = layer_args(shape, p, cache, ema, ws, cx);
+    la.n_elig = cx.scoring ? cx.n_elig : 0;
+    IKV_TRY_CUDA(launch_layer_end(la, stream), "layer end launch");
+    return IKV_OK;
+}
+
 ikv_status ikv_step_workspace_size(const ikv_shape *shape, const ikv_cache *cache, size_t *bytes) {
     g_err[0] = 0;
     ikv_status e = check_shape(shape);
     if (e) return e;
     if ((e = check_cache(shape, cache, false))) return e;
     if (!bytes) return fail(IKV_ERR_ARG, "bytes is NULL");
-    *bytes = step_ws(shape, cap_of(cache)).end;
+    *bytes = step_ws(shape, cap_of(cache), cache->pos_cap).end;
     return IKV_OK;
 }
 
@@ -639,6 +722,35 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     cache = &cx.cv;
     const StepWs &w = cx.w;
     const ikv_timing *tm = p->timing;
+    if (cx.layerwise) {
+        // begin, every layer's new rows, one attention launch for all layers (each reads
+        // its own rows as they stood before this step's evictions), then layer by layer:
+        // utilities, selection, compaction; the pending decays at the end
+        IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.at.arrivals), 0, w.at.logits - w.at.arrivals, stream),
+                     "cudaMemsetAsync");
+        LayerArgs la = layer_args(shape, p, cache, ema, ws, cx);
+        IKV_TRY_CUDA(launch_layer_begin(la, stream), "layer begin launch");
+        PdlScope pdl;
+        AppendArgs ap{};
+        ap.k = cache->k;
+        ap.v = cache->v;
+        ap.pv = view_of(shape, cache);
+        ap.batch = shape->batch;
+        ap.layers = shape->layers;
+        ap.cap = cx.cap;
+        ap.elem_bytes = elem_bytes(shape);
+        ap.k_new = k_new;
+        ap.v_new = v_new;
+        ap.vnorm = cache->vnorm;
+        ap.slot = at<int32_t>(ws, w.slot);
+        IKV_TRY_CUDA(launch_append_rows(ap, stream), "append rows launch");
+        if ((e = run_attend(shape, cache, 0, shape->layers, cx.L1, q, out, ws, w.at, cx.scoring, nullptr, nullptr,
+                            stream, nullptr, true)))
+            return e;
+        for (int l = 0; l < shape->layers; ++l)
+            if ((e = evict_layer(shape, p, cache, ema, ws, cx, l, stream))) return e;
+        return layer_end(shape, p, cache, ema, ws, cx, stream);
+    }
 
     // control words (append and split-arrival counters) start at zero
     IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.at.arrivals), 0, w.at.logits - w.at.arrivals, stream),
@@ -677,6 +789,10 @@ ikv_status ikv_step_begin(const ikv_shape *shape, const ikv_params *p, ikv_cache
                  "cudaMemsetAsync");
     IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, cx.w.done), 0, 2 * sizeof(int32_t) * shape->batch, stream),
                  "cudaMemsetAsync");
+    if (cx.layerwise) {
+        IKV_TRY_CUDA(launch_layer_begin(layer_args(shape, p, &cx.cv, ema, ws, cx), stream), "layer begin launch");
+        return IKV_OK;
+    }
     return append_impl(shape, &cx.cv, nullptr, nullptr, ema, cx.init_mean, at<int32_t>(ws, cx.w.done), stream, true,
                        at<int32_t>(ws, cx.w.slot));
 }
@@ -713,8 +829,10 @@ ikv_status ikv_step_layer(const ikv_shape *shape, const ikv_params *p, ikv_cache
     // the new token's rows and one layer's attention; on refresh steps its logits and
     // log-sum-exp land where the whole step's attention would put them, for
     // ikv_step_end's score pass
-    return run_attend(shape, cache, layer, 1, cx.L1, q, out, ws, cx.w.at, cx.scoring && eligible, nullptr, nullptr,
-                      stream, nullptr, true, shape->layers, layer, &a);
+    if ((e = run_attend(shape, cache, layer, 1, cx.L1, q, out, ws, cx.w.at, cx.scoring && eligible, nullptr, nullptr,
+                        stream, nullptr, true, shape->layers, layer, &a)))
+        return e;
+    return cx.layerwise ? evict_layer(shape, p, cache, ema, ws, cx, layer, stream) : IKV_OK;
 }
 
 ikv_status ikv_step_end(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, int32_t t,
@@ -724,6 +842,7 @@ ikv_status ikv_step_end(const ikv_shape *shape, const ikv_params *p, ikv_cache *
     ikv_status e = prepare_step(shape, p, cache, ema, t, ws, ws_bytes, &cx);
     if (e) return e;
     PdlScope pdl;
+    if (cx.layerwise) return layer_end(shape, p, &cx.cv, ema, ws, cx, stream);
     if (cx.scoring && (e = run_score(shape, &cx.cv, shape->layers, cx.elig, cx.n_elig, cx.L1, ws, cx.w.at, p->alpha,
                                      ema, nullptr, stream, p->agg_mode, p->scorer, cx.sw)))
         return e;

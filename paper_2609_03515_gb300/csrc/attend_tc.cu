@@ -729,9 +729,10 @@ extern "C" ikv_status ikv_device_status(uint32_t *flags) {
     unsigned int v = 0, z = 0;
     cudaError_t e = cudaMemcpyFromSymbol(&v, ikv::g_tc_error, sizeof(v));
     if (e == cudaSuccess) e = cudaMemcpyToSymbol(ikv::g_tc_error, &z, sizeof(z));
-    unsigned int ap = 0;
+    unsigned int ap = 0, lw = 0;
     if (e == cudaSuccess) e = ikv::read_clear_append_error(&ap);
+    if (e == cudaSuccess) e = ikv::read_clear_layer_error(&lw);
     if (e != cudaSuccess) return ikv::report(IKV_ERR_CUDA, "ikv_device_status: %s", cudaGetErrorString(e));
-    *flags = v | (ap ? 4u : 0u);
+    *flags = v | (ap ? 4u : 0u) | lw;
     return IKV_OK;
 }

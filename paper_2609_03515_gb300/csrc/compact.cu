@@ -154,9 +154,9 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
         }
     }
     // whatever the mode, the next append must find a free slot: else move every row to slot 0
-    if (a.start && new_start + n0 + 1 > a.cap) new_start = 0;
+    if (a.start && a.publish_len && new_start + n0 + 1 > a.cap) new_start = 0;
     if (x < nkv) {
-        const int l = x / kvh, g = x % kvh;
+        const int l = a.layer0 + x / kvh, g = x % kvh;
         const int r = b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g);
         const int n = a.keep_len[r];
         const int32_t *kp = a.keep + (int64_t)r * a.cap;
@@ -225,7 +225,7 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
         const int r = b * a.rows_per_seq + rr;
         const int n = a.keep_len[r];
         const int32_t *kp = a.keep + (int64_t)r * a.cap;
-        int32_t *pos = a.pos + (int64_t)r * a.cap;
+        int32_t *pos = a.pos + ((int64_t)b * a.pos_rows + a.pos_row0 + rr) * a.cap;
         float *ema = a.ema ? a.ema + (int64_t)r * a.cap : nullptr;
         constexpr int PER = 16;
         for (int base = 0; base < n; base += kCompThreads * PER) {
@@ -254,6 +254,7 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
         }
     }
     // publish len / start once every CTA of b has read them
+    if (!a.publish_len) return;
     __syncthreads();
     if (tid == 0) {
         __threadfence();
@@ -458,17 +459,18 @@ __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a
     }
 }
 
-// Split step: the new token's rows of one layer into the slot ikv_step_begin reserved.
-// CTA (x, b) copies kv heads 8x .. 8x+7 of sequence b and stores their value-row norms.
+// Split step: the new token's rows of layers layer0 .. layer0 + layers - 1 into the
+// slot the begin call reserved.  CTA (x, b) copies (layer, kv head) rows 8x .. 8x+7 of
+// sequence b and stores their value-row norms.
 __global__ void __launch_bounds__(kCompThreads) append_rows_kernel(const AppendArgs a) {
     pdl_wait();
     const int tid = threadIdx.x;
     const int b = blockIdx.y;
     const int kvh = a.pv.kv_heads;
+    const int nkv = a.layers * kvh;
     const int j = a.slot[b];
     if (j < 0) return;  // no room: the begin call flagged the error and kept len
     const int S = a.pv.start_of(b);
-    const int l = a.layer0;
     const int rowB = a.pv.head_dim * a.elem_bytes;
     const int CPR = rowB >> 4;
     unsigned char *kb = reinterpret_cast<unsigned char *>(a.k);
@@ -476,18 +478,20 @@ __global__ void __launch_bounds__(kCompThreads) append_rows_kernel(const AppendA
     const unsigned char *kn = reinterpret_cast<const unsigned char *>(a.k_new);
     const unsigned char *vn = reinterpret_cast<const unsigned char *>(a.v_new);
     for (int idx = tid; idx < kAppendRows * CPR; idx += kCompThreads) {
-        const int g = blockIdx.x * kAppendRows + idx / CPR, c = idx % CPR;
-        if (g < kvh) {
-            const int64_t src = ((int64_t)b * kvh + g) * rowB + c * 16;
-            const int64_t dst = a.pv.row_phys(b, l, g, S + j) * rowB + c * 16;
+        const int x = blockIdx.x * kAppendRows + idx / CPR, c = idx % CPR;
+        if (x < nkv) {
+            const int li = x / kvh, g = x % kvh;
+            const int64_t src = (((int64_t)li * a.batch + b) * kvh + g) * rowB + c * 16;
+            const int64_t dst = a.pv.row_phys(b, a.layer0 + li, g, S + j) * rowB + c * 16;
             *reinterpret_cast<uint4 *>(kb + dst) = *reinterpret_cast<const uint4 *>(kn + src);
             *reinterpret_cast<uint4 *>(vb + dst) = *reinterpret_cast<const uint4 *>(vn + src);
         }
     }
     if (a.vnorm) {
-        const int g = blockIdx.x * kAppendRows + (tid >> 5), lane = tid & 31;
-        if ((tid >> 5) < kAppendRows && g < kvh) {
-            const int64_t e0 = ((int64_t)b * kvh + g) * a.pv.head_dim;
+        const int x = blockIdx.x * kAppendRows + (tid >> 5), lane = tid & 31;
+        if ((tid >> 5) < kAppendRows && x < nkv) {
+            const int li = x / kvh, g = x % kvh;
+            const int64_t e0 = (((int64_t)li * a.batch + b) * kvh + g) * a.pv.head_dim;
             float sq = 0.f;
             for (int e = lane; e < a.pv.head_dim; e += 32) {
                 const float xv = a.elem_bytes == 2
@@ -497,7 +501,7 @@ __global__ void __launch_bounds__(kCompThreads) append_rows_kernel(const AppendA
             }
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
-            if (lane == 0) a.vnorm[(((int64_t)l * a.batch + b) * kvh + g) * a.cap + j] = sqrtf(sq);
+            if (lane == 0) a.vnorm[(((int64_t)(a.layer0 + li) * a.batch + b) * kvh + g) * a.cap + j] = sqrtf(sq);
         }
     }
 }
@@ -543,7 +547,7 @@ cudaError_t launch_append(const AppendArgs &a, cudaStream_t st) {
 }
 
 cudaError_t launch_append_rows(const AppendArgs &a, cudaStream_t st) {
-    dim3 grid((a.pv.kv_heads + kAppendRows - 1) / kAppendRows, a.batch);
+    dim3 grid((a.layers * a.pv.kv_heads + kAppendRows - 1) / kAppendRows, a.batch);
     cudaError_t e = launch_k(append_rows_kernel, grid, dim3(kCompThreads), 0, st, a);
     note_launch();
     return e != cudaSuccess ? e : cudaGetLastError();

@@ -183,6 +183,9 @@ struct CompactArgs {
     int32_t max_holes;          // > 0: while a sequence's dead slots stay <= max_holes, mark
                                 // the evicted slots dead (pos = -1) instead of compacting
     float *vnorm;               // [layers][batch][kv_heads][cap] value-row norms moved with the rows, or null
+    int32_t layer0;             // the K/V rows compacted are those of layers layer0 .. layer0 + layers - 1
+    int32_t pos_rows, pos_row0; // utility row rr of sequence b uses pos row b * pos_rows + pos_row0 + rr
+    int32_t publish_len;        // 1: the last CTA of b writes len / start; 0: left to the caller
 };
 cudaError_t launch_compact(const CompactArgs &a, int mode, cudaStream_t st);
 
@@ -204,7 +207,36 @@ struct AppendArgs {
     int32_t *slot;
 };
 cudaError_t launch_append(const AppendArgs &a, cudaStream_t st);
+// rows of layers layer0 .. layer0 + layers - 1 (k_new: [layers][batch][kv_heads][D]) into slot[b]
 cudaError_t launch_append_rows(const AppendArgs &a, cudaStream_t st);
+
+// Per-layer eviction (IKV_EVICT_LAYER): a position-indexed state m [batch][pos_cap]
+// shared by all layers, layer l's positions in pos row b * layers + l.  A layer's
+// update decays every live position it does not hold; that decay is applied lazily:
+// lam[p] is the index, among this step's eligible layers, of the last one that
+// updated p (-1: none yet), and the stored m[p] is its value as of that update.
+struct LayerArgs {
+    int32_t batch, layers, q_heads, cap, pos_cap;
+    int32_t *len, *next_pos, *pos;
+    const int32_t *start;       // [batch] or null
+    float *m;                   // [batch][pos_cap]
+    int32_t *lam;               // [batch][pos_cap] workspace
+    float *util;                // [batch][cap] workspace: the layer's utilities by slot
+    const float *logits, *lse2; // [batch][sc_layers][H][lstride], [batch][sc_layers][H]
+    int32_t sc_layers, lstride;
+    float alpha;
+    int32_t layer;              // util: the layer
+    int32_t k_done;             // util: eligible layers folded earlier in this step
+    int32_t scoring;            // util: fold this layer's Eq. 1 score
+    int32_t init_mean;          // begin: new token's state = mean over live positions (else 0)
+    int32_t *slot;              // begin: each sequence's reserved slot, -1 if none
+    const int32_t *keep_len;    // end: the step's kept count per sequence
+    int32_t n_elig;             // end: eligible layers folded this step (0: no pending decay)
+};
+cudaError_t launch_layer_begin(const LayerArgs &a, cudaStream_t st);
+cudaError_t launch_layer_util(const LayerArgs &a, int32_t max_len, cudaStream_t st);
+cudaError_t launch_layer_end(const LayerArgs &a, cudaStream_t st);
+cudaError_t read_clear_layer_error(unsigned int *v);
 // reads and clears the append kernel's device error word (bit 0: no free slot)
 cudaError_t read_clear_append_error(unsigned int *v);
 

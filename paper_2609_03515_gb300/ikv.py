@@ -22,6 +22,7 @@ IKV_INIT_ZERO, IKV_INIT_MEAN = 0, 1
 IKV_PATH_CUDA_CORE, IKV_PATH_TENSOR_CORE = 0, 1
 IKV_AGG_EMA, IKV_AGG_CUMULATIVE, IKV_AGG_SINGLE_STEP = 0, 1, 2
 IKV_SCORE_ATTENTION, IKV_SCORE_VNORM, IKV_SCORE_ENTROPY = 0, 1, 2
+IKV_EVICT_STEP, IKV_EVICT_LAYER = 0, 1
 
 P = ctypes.c_void_p
 I32 = ctypes.c_int32
@@ -37,7 +38,7 @@ class ikv_shape(ctypes.Structure):
 class ikv_cache(ctypes.Structure):
     _fields_ = [("k", P), ("v", P), ("block_table", P), ("num_pages", I32), ("page_size", I32), ("max_pages", I32),
                 ("len", P), ("pos", P), ("next_pos", P), ("max_len", I32), ("start", P), ("dead_slots", I32),
-                ("vnorm", P)]
+                ("vnorm", P), ("pos_cap", I32)]
 
 
 class ikv_timing(ctypes.Structure):
@@ -49,7 +50,7 @@ class ikv_params(ctypes.Structure):
     _fields_ = [("alpha", F32), ("refresh_period", I32), ("score_free", I32), ("budget", P),
                 ("layer_eligible", P), ("compact_mode", I32), ("refresh_init", I32),
                 ("timing", ctypes.POINTER(ikv_timing)), ("max_holes", I32), ("agg_mode", I32),
-                ("scorer", I32)]
+                ("scorer", I32), ("evict_mode", I32)]
 
 
 class IKVError(RuntimeError):

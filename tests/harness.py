@@ -297,3 +297,76 @@ def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1)
         reports.append(rep)
     assert ikv.ikv_device_status() == 0
     return reports
+
+
+def run_lockstep_layerwise(w: gen.Workload, steps: Optional[int] = None, page_perm_seed: Optional[int] = 7,
+                           refresh_init: int = ikv.IKV_INIT_ZERO, layer_eligible=None, per_layer: bool = False):
+    """Per-layer immediate eviction (IKV_EVICT_LAYER) in lock-step with the oracle's
+    decode_step_layerwise.  Per step: every layer's attention output, every layer's kept
+    positions under the boundary rule against the oracle's utilities at that layer's
+    eviction (the oracle then adopts the GPU's set), the state at every live position
+    (1e-3), and each layer's K/V rows bit for bit."""
+    T = w.steps if steps is None else steps
+    u = w.u_table()
+    pos_cap = max(w.prefill) + T + 1
+    c = DecodeCache(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.cap,
+                    dtype=ikv.IKV_BF16 if w.dtype == gen.BF16 else ikv.IKV_F32, page_size=w.page_size,
+                    page_perm_seed=page_perm_seed, pos_cap=pos_cap)
+    c.set_prefill(w.prefill, w.budgets())
+    kv = fill_host(c, w, u)
+    budgets = w.budgets()
+    sts = []
+    for b in range(w.batch):
+        K = [[kv[b][l][0][g] for g in range(w.kv_heads)] for l in range(w.layers)]
+        V = [[kv[b][l][1][g] for g in range(w.kv_heads)] for l in range(w.layers)]
+        sts.append(O.layerwise_prefill_state(K, V, budgets[b]))
+    op = O.Params(alpha=w.alpha, refresh_period=w.refresh_period, score_free=w.score_free,
+                  layer_mask=None if layer_eligible is None else [bool(x) for x in layer_eligible],
+                  refresh_init="zero" if refresh_init == ikv.IKV_INIT_ZERO else "mean")
+    p = c.params(w.alpha, w.refresh_period, w.score_free, ikv.IKV_COMPACT_STABLE, refresh_init, layer_eligible,
+                 evict_mode=ikv.IKV_EVICT_LAYER)
+    ws = c.step_workspace()
+    qs = w.queries(1, T + 1, u)
+    out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
+    reports = []
+    lens = list(w.prefill)
+    for t in range(1, T + 1):
+        kn, vn = w.new_tokens(t, u)
+        decode_step(c, p, c.cache(max(lens)), t, to_device(qs[t - 1], w), to_device(kn, w), to_device(vn, w), out,
+                    ws, per_layer)
+        lens = [min(L + 1, B) for L, B in zip(lens, budgets)]
+        torch.cuda.synchronize()
+        out_h = out.float().cpu().numpy()
+        m_h = c.ema.cpu().numpy()
+        pos_h = c.pos.cpu().numpy()
+        len_h = c.len.cpu().numpy()
+        rep = StepReport(t=t, refresh=O.is_refresh(t, w.refresh_period, w.score_free))
+        q64 = as_f64(qs[t - 1], w)
+        for b, st in enumerate(sts):
+            assert len_h[b] == lens[b], (t, b, len_h[b], lens[b])
+            gpu_kept = [pos_h[b * w.layers + l, :lens[b]].astype(np.int64) for l in range(w.layers)]
+
+            def adopt(l, tr, b=b):
+                kept = gpu_kept[l]
+                assert np.all(np.diff(kept) > 0), (t, b, l)   # stable: ascending positions
+                mask = np.isin(tr.pos, kept)
+                assert mask.sum() == len(kept), (t, b, l)      # kept positions were held by the layer
+                ok, _ = boundary_ok(tr.m, mask, budgets[b])
+                rep.set_ok &= ok
+                rep.strict_set_equal &= set(tr.kept.tolist()) == set(kept.tolist())
+                return kept
+
+            o_out, _ = O.decode_step_layerwise(st, t, q64[:, b], kn[:, b], vn[:, b], op, keep_override=adopt)
+            rep.out_err = max(rep.out_err, float(np.max(np.abs(out_h[:, b] - o_out))))
+            live = st.live()
+            rep.m_err = max(rep.m_err, float(np.max(np.abs(m_h[b, live] - st.m[live]))))
+            for l in range(w.layers):
+                assert np.array_equal(gpu_kept[l], st.pos[l]), (t, b, l)
+                for g in range(w.kv_heads):
+                    gk = c.gather(c.k, b, l, g, lens[b]).float().cpu().numpy()
+                    gv = c.gather(c.v, b, l, g, lens[b]).float().cpu().numpy()
+                    rep.kv_err = max(rep.kv_err, float(np.max(np.abs(gk - st.K[l][g]))),
+                                     float(np.max(np.abs(gv - st.V[l][g]))))
+        reports.append(rep)
+    assert ikv.ikv_device_status() == 0
+    return reports

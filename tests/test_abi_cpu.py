@@ -124,6 +124,33 @@ def test_split_step_rejects_bad_arguments(lib):
     assert lib.raw_status("ikv_step_begin", S, P, ctypes.byref(full), 16, 1, 16, big, None) == lib.IKV_ERR_SHAPE
 
 
+def test_per_layer_eviction_arguments(lib):
+    """IKV_EVICT_LAYER supports one configuration of the other options; the rest are refused
+    on the host."""
+    shp = _shape(lib)
+    cch = _cache(lib, pos_cap=200)
+    p = lib.ikv_params()
+    p.alpha, p.refresh_period, p.budget, p.evict_mode = 0.9, 1, 16, lib.IKV_EVICT_LAYER
+    call = lambda s, c: lib.raw_status("ikv_step", ctypes.byref(s), ctypes.byref(p), ctypes.byref(c), 16, 1, 16, 16,
+                                       16, 16, 16, 1 << 40, None)
+    p.max_holes = 4
+    assert call(shp, cch) == lib.IKV_ERR_UNSUPPORTED
+    p.max_holes, p.compact_mode = 0, lib.IKV_COMPACT_HOLEFILL
+    assert call(shp, cch) == lib.IKV_ERR_UNSUPPORTED
+    p.compact_mode, p.scorer = lib.IKV_COMPACT_STABLE, lib.IKV_SCORE_ENTROPY
+    assert call(shp, cch) == lib.IKV_ERR_UNSUPPORTED
+    p.scorer = lib.IKV_SCORE_ATTENTION
+    assert call(_shape(lib, granularity=lib.IKV_GRAN_KVHEAD), cch) == lib.IKV_ERR_UNSUPPORTED
+    assert call(shp, _cache(lib)) == lib.IKV_ERR_ARG             # pos_cap 0
+    p.evict_mode = 7
+    assert call(shp, cch) == lib.IKV_ERR_ARG
+    # the workspace grows with the position capacity
+    n0, n1 = lib.SZ(0), lib.SZ(0)
+    lib.raw_status("ikv_step_workspace_size", ctypes.byref(shp), ctypes.byref(_cache(lib)), ctypes.byref(n0))
+    lib.raw_status("ikv_step_workspace_size", ctypes.byref(shp), ctypes.byref(cch), ctypes.byref(n1))
+    assert n1.value >= n0.value + 200 * 4
+
+
 def test_deferred_compaction_arguments(lib):
     shp, cch = _shape(lib), _cache(lib)
     p = lib.ikv_params()

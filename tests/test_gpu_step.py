@@ -202,3 +202,24 @@ def test_per_layer_split_equals_whole_step():
         assert torch.equal(outs[0], outs[1]), t
         max_len = int(a.len.max())
     assert ikv.ikv_device_status() == 0
+
+
+def test_per_layer_immediate_eviction_trajectories():
+    """IKV_EVICT_LAYER: each layer evicts right after folding its score into the
+    position-indexed state (reading R10), through ikv_step and through the begin /
+    per-layer / end split, in lock-step with the oracle's decode_step_layerwise."""
+    from harness import run_lockstep_layerwise
+
+    _assert(run_lockstep_layerwise(gen.config(0)), 1e-4, strict_fraction=1.0)
+    _assert(run_lockstep_layerwise(gen.config(0), per_layer=True), 1e-4, strict_fraction=1.0)
+    _assert(run_lockstep_layerwise(gen.config(0).with_(refresh_period=3), refresh_init=ikv.IKV_INIT_MEAN),
+            1e-4, strict_fraction=1.0)
+    _assert(run_lockstep_layerwise(small_llama(steps=8)), 2e-2)
+    _assert(run_lockstep_layerwise(small_llama(steps=8), per_layer=True), 2e-2)
+    _assert(run_lockstep_layerwise(small_llama(steps=9, refresh_period=4)), 2e-2)
+    _assert(run_lockstep_layerwise(small_llama(steps=6, score_free=True, page_size=16), per_layer=True), 2e-2)
+    _assert(run_lockstep_layerwise(small_llama(steps=6, layers=4), layer_eligible=[0, 1, 1, 0],
+                                   refresh_init=ikv.IKV_INIT_MEAN), 2e-2)
+    w = gen.Workload(name="qwen-small", batch=2, layers=2, q_heads=28, kv_heads=4, head_dim=128, prefill=[700, 260],
+                     steps=5, dtype=gen.BF16, alpha=0.9, seed=9, page_size=32)
+    _assert(run_lockstep_layerwise(w, per_layer=True), 2e-2)
