@@ -235,7 +235,7 @@ class ClockSampler:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
-def setup(w, device, compact_mode):
+def setup(w, device, compact_mode, steps: int = 0):
     import numpy as np
     import torch
 
@@ -244,7 +244,8 @@ def setup(w, device, compact_mode):
 
     c = DecodeCache(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.cap,
                     dtype=ikv.IKV_BF16 if w.dtype == gen.BF16 else ikv.IKV_F32, page_size=w.page_size,
-                    device=device, page_perm_seed=1, value_norms=True)
+                    device=device, page_perm_seed=1, value_norms=True,
+                    pos_cap=max(w.prefill) + steps + 2)  # position state for per-layer eviction
     return c
 
 
@@ -336,18 +337,19 @@ def split_step(c, p, cache, t, q, kn, vn, out, ws, stream, foreign=None):
     ikv_step_end."""
     from paper_2609_03515_gb300 import ikv
 
-    ikv.ikv_step_begin(c.shape(), p, cache, c.ema, t, ws, ws.numel(), stream)
+    m = c.utility(p.evict_mode)
+    ikv.ikv_step_begin(c.shape(), p, cache, m, t, ws, ws.numel(), stream)
     for l in range(c.layers):
         if foreign is None:
-            ikv.ikv_step_layer(c.shape(), p, cache, c.ema, t, l, q[l], kn[l], vn[l], out[l], ws, ws.numel(), stream)
+            ikv.ikv_step_layer(c.shape(), p, cache, m, t, l, q[l], kn[l], vn[l], out[l], ws, ws.numel(), stream)
         else:
             ql, kl, vl = foreign(l)
-            ikv.ikv_step_layer(c.shape(), p, cache, c.ema, t, l, ql, kl, vl, out[l], ws, ws.numel(), stream)
-    ikv.ikv_step_end(c.shape(), p, cache, c.ema, t, ws, ws.numel(), stream)
+            ikv.ikv_step_layer(c.shape(), p, cache, m, t, l, ql, kl, vl, out[l], ws, ws.numel(), stream)
+    ikv.ikv_step_end(c.shape(), p, cache, m, t, ws, ws.numel(), stream)
 
 
 def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, sample_clocks: bool,
-                   mh: int = 0, scorer: int = 0, per_layer: str = ""):
+                   mh: int = 0, scorer: int = 0, per_layer: str = "", evict: int = 0):
     """The same schedule with each steady-state step replayed from a captured CUDA graph.
 
     After the eager warm-up (decode step 1 evicts ~90% of the prefill, later steps hold
@@ -363,7 +365,9 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     from paper_2609_03515_gb300 import ikv, step_lengths
 
     reset(c, w, u_dev)
-    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh, scorer=scorer)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh, scorer=scorer,
+                 evict_mode=evict)
+    m_state = c.utility(evict)
     budgets = w.budgets()
     assert all(L0 >= B for L0, B in zip(w.prefill, budgets)), "graph replay assumes every sequence at its budget"
     lens, live = list(w.prefill), list(w.prefill)
@@ -377,7 +381,7 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     def one(cache, t):
         st = torch.cuda.current_stream()
         if not per_layer:
-            ikv.ikv_step(c.shape(), p, cache, c.ema, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws,
+            ikv.ikv_step(c.shape(), p, cache, m_state, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws,
                          ws.numel(), st)
             return
 
@@ -576,7 +580,7 @@ def run_ours(args):
     dev = torch.device("cuda", torch.cuda.current_device())
     u = w.u_table()
     u_dev = torch.from_numpy(u).to(dev)
-    c = setup(w, dev, compact_mode)
+    c = setup(w, dev, compact_mode, total_steps)
     ws = c.step_workspace()
     T = total_steps
     qs_h = w.queries(1, T + 1, u)
@@ -623,25 +627,32 @@ def run_ours(args):
         lazy_w = w.with_(refresh_period=4, score_free=False)
         sf_w = w.with_(refresh_period=1, score_free=True)
         att, vnm, ent = ikv.IKV_SCORE_ATTENTION, ikv.IKV_SCORE_VNORM, ikv.IKV_SCORE_ENTROPY
-        variants = (("full", full_w, compact_mode, mh, att),
-                    ("lazy4", lazy_w, compact_mode, mh, att),
-                    ("score_free", sf_w, compact_mode, mh, att),
-                    ("full_vnorm", full_w, compact_mode, mh, vnm),
-                    ("full_entropy", full_w, compact_mode, mh, ent),
-                    ("full_every_step", full_w, compact_mode, 0, att),
-                    ("lazy4_every_step", lazy_w, compact_mode, 0, att),
-                    ("score_free_every_step", sf_w, compact_mode, 0, att),
-                    ("full_stable_left", full_w, ikv.IKV_COMPACT_STABLE, 0, att),
-                    ("full_holefill", full_w, ikv.IKV_COMPACT_HOLEFILL, 0, att),
-                    ("lazy4_holefill", lazy_w, ikv.IKV_COMPACT_HOLEFILL, 0, att),
-                    ("score_free_holefill", sf_w, ikv.IKV_COMPACT_HOLEFILL, 0, att))
-        for name, ww, cm, vmh, sc in variants:
-            if name == head_sched and cm == compact_mode and vmh == mh and sc == att:
+        stable, layer = ikv.IKV_COMPACT_STABLE, ikv.IKV_EVICT_LAYER
+        variants = (("full", full_w, compact_mode, mh, att, 0),
+                    ("lazy4", lazy_w, compact_mode, mh, att, 0),
+                    ("score_free", sf_w, compact_mode, mh, att, 0),
+                    ("full_vnorm", full_w, compact_mode, mh, vnm, 0),
+                    ("full_entropy", full_w, compact_mode, mh, ent, 0),
+                    ("full_every_step", full_w, compact_mode, 0, att, 0),
+                    ("lazy4_every_step", lazy_w, compact_mode, 0, att, 0),
+                    ("score_free_every_step", sf_w, compact_mode, 0, att, 0),
+                    ("full_stable_left", full_w, stable, 0, att, 0),
+                    ("full_holefill", full_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, 0),
+                    ("lazy4_holefill", lazy_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, 0),
+                    ("score_free_holefill", sf_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, 0),
+                    ("full_layer_evict", full_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, layer),
+                    ("lazy4_layer_evict", lazy_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, layer),
+                    ("full_layer_evict_stable", full_w, stable, 0, att, layer))
+        for name, ww, cm, vmh, sc, ev in variants:
+            if name == head_sched and cm == compact_mode and vmh == mh and sc == att and ev == 0:
                 modes[name] = full           # the headline run is this mode
                 continue
-            modes[name] = run_mode_graph(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, dist, False, vmh, sc)
+            modes[name] = run_mode_graph(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, dist, False, vmh, sc,
+                                         evict=ev)
         if args.mode_kernels:
-            for name, ww, cm, vmh, sc in variants:
+            for name, ww, cm, vmh, sc, ev in variants:
+                if ev:
+                    continue  # per-kernel events time the step-end eviction path only
                 mode_kernels[name] = run_mode(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, True, dist,
                                               vmh, sc)["kernel_ms"]
     K = args.steps
@@ -719,7 +730,10 @@ def run_ours(args):
                               "VNorm and entropy-weighted scorers under full refresh; *_every_step: the same "
                               "compaction run on every eviction (max_holes 0); full_stable_left: stable "
                               "compaction that always shifts the suffix left, every step; *_holefill: hole-fill "
-                              "compaction every step (same kept sets, survivors not kept in order)")
+                              "compaction every step (same kept sets, survivors not kept in order); "
+                              "*_layer_evict: per-layer immediate eviction (each layer keeps its own top-B "
+                              "right after its update of a position-indexed state), hole-fill compaction of "
+                              "every layer; full_layer_evict_stable: the same with order-preserving compaction")
     print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()

@@ -164,12 +164,16 @@ typedef struct {
                                        cache->vnorm) | IKV_SCORE_ENTROPY */
     int32_t evict_mode;             /* IKV_EVICT_STEP (default) | IKV_EVICT_LAYER: each layer, after
                                        folding its score into the position-indexed state, keeps the
-                                       budget[b] highest-utility tokens it holds and compacts its own
-                                       rows.  A live position a layer does not hold scores 0 there, so
-                                       its state decays by alpha (Eq. 1, Eq. 4); the mean initialisation
-                                       averages the positions some layer holds.  Needs IKV_GRAN_SEQ,
-                                       IKV_COMPACT_STABLE, max_holes 0, IKV_AGG_EMA, IKV_SCORE_ATTENTION,
-                                       cache->pos_cap > 0 and the layout described under "Utility rows". */
+                                       budget[b] highest-utility tokens it holds (by the state as of its
+                                       own update) and compacts its own rows (compact_mode; the shorter-
+                                       side mode moves suffixes left).  A live position a layer does not
+                                       hold scores 0 there, so its state decays by alpha (Eq. 1, Eq. 4);
+                                       the mean initialisation averages the positions some layer holds.
+                                       No layer's eviction changes another's inputs within a step, so the
+                                       library applies them all after the step's attention (in ikv_step_end
+                                       for the split step).  Needs IKV_GRAN_SEQ, max_holes 0, IKV_AGG_EMA,
+                                       IKV_SCORE_ATTENTION, cache->pos_cap > 0 and the layout described
+                                       under "Utility rows". */
 } ikv_params;
 
 /* Message for the last error on this thread ("" if none). */
@@ -364,7 +368,8 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *params, ikv_cache 
  *    attention logits in ws.  Every layer is called once, in ascending order.
  *  - ikv_step_end: step 4 -- the kept scores of every eligible layer folded into ema
  *    in ascending layer order, which is the order Eq. 4 prescribes; nothing reads ema
- *    before the eviction -- and step 5 (selection, deferred or immediate compaction).
+ *    before the eviction -- and step 5 (selection, deferred or immediate compaction;
+ *    under IKV_EVICT_LAYER every layer's own eviction).
  *  All three take the same shape, params, cache (max_len: the bound on len[]
  *  before the append, as for ikv_step), ema, t and ws (ikv_step_workspace_size
  *  bytes, which carries the step's state from call to call).  Argument errors are

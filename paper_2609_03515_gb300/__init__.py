@@ -57,7 +57,8 @@ class DecodeCache:
     len:         [batch] int32 slots in use (dead slots included);  next_pos: [batch] int32
     pos, ema:    [rows][cap] int32 / fp32, rows = batch (per-sequence state) or batch * kv_heads;
                  pos = -1 marks a dead slot (deferred compaction).  With pos_cap > 0 (per-layer
-                 eviction): pos is [batch * layers][cap] and ema [batch][pos_cap], by position
+                 eviction): pos has batch * layers rows (row b * layers + l: layer l's positions)
+                 and pos_state [batch][pos_cap] is the utility by token position
     budget:      [batch] int32
     """
 
@@ -84,11 +85,14 @@ class DecodeCache:
         self.len = torch.zeros(batch, dtype=torch.int32, device=device)
         self.next_pos = torch.zeros(batch, dtype=torch.int32, device=device)
         # per-layer eviction (pos_cap > 0): a position row per (sequence, layer) and the
-        # utility state indexed by token position
+        # utility state indexed by token position (pos_state); the step-end mode reads
+        # the first `rows` position rows and ema
         self.pos_cap = pos_cap
-        pos_rows = batch * layers if pos_cap > 0 else self.rows
+        pos_rows = max(self.rows, batch * layers) if pos_cap > 0 else self.rows
         self.pos = torch.zeros((pos_rows, self.cap), dtype=torch.int32, device=device)
-        self.ema = torch.zeros((self.rows, pos_cap if pos_cap > 0 else self.cap), dtype=torch.float32, device=device)
+        self.ema = torch.zeros((self.rows, self.cap), dtype=torch.float32, device=device)
+        self.pos_state = (torch.zeros((batch, pos_cap), dtype=torch.float32, device=device) if pos_cap > 0
+                          else None)
         self.budget = torch.zeros(batch, dtype=torch.int32, device=device)
         self.start = torch.zeros(batch, dtype=torch.int32, device=device)
         # per-slot value-row norms, for the VNorm scorer
@@ -122,6 +126,8 @@ class DecodeCache:
         ar = torch.arange(self.cap, dtype=torch.int32, device=dev)
         self.pos.copy_(ar.expand(self.pos.shape[0], self.cap))
         self.ema.zero_()
+        if self.pos_state is not None:
+            self.pos_state.zero_()
         self.start.zero_()
         self.max_len = max(lengths)
 
@@ -141,6 +147,10 @@ class DecodeCache:
         slots = torch.arange(s0, s0 + n, device=pool.device)
         pages = self.block_table[b, (slots // self.page_size).long()].long()
         pool[layer, pages, g, slots % self.page_size] = rows.to(pool.dtype)
+
+    def utility(self, evict_mode: int = ikv.IKV_EVICT_STEP) -> torch.Tensor:
+        """The utility array a step of this eviction mode updates (ema or pos_state)."""
+        return self.pos_state if evict_mode == ikv.IKV_EVICT_LAYER else self.ema
 
     def step_workspace(self) -> torch.Tensor:
         n = ikv.ikv_step_workspace_size(self.shape(), self.cache(self.cap - 1))

@@ -131,25 +131,28 @@ AttendWs attend_ws(const ikv_shape *s, int32_t cap, int n_layers, bool logits) {
 
 struct StepWs {
     AttendWs at;
-    size_t keep, keep_len, done, cdone, moves, n_moves, sbuf, epart, vmean, slot, lam, util, end;
+    size_t keep, keep_len, done, cdone, moves, n_moves, sbuf, epart, vmean, slot, inv, util, live, end;
 };
 
 StepWs step_ws(const ikv_shape *s, int32_t cap, int32_t pos_cap) {
     StepWs w;
     w.at = attend_ws(s, cap, s->layers, true);
     size_t off = w.at.end;
+    // utility rows; selection rows: one per utility row, or per (sequence, layer) under
+    // per-layer eviction
     const size_t R = (size_t)s->batch * rows_per_seq(s);
+    const size_t Rs = pos_cap > 0 && s->layers > rows_per_seq(s) ? (size_t)s->batch * s->layers : R;
     w.keep = off;
-    off = align256(off + R * cap * sizeof(int32_t));
+    off = align256(off + Rs * cap * sizeof(int32_t));
     w.keep_len = off;
-    off = align256(off + R * sizeof(int32_t));
+    off = align256(off + Rs * sizeof(int32_t));
     w.done = off;  // append arrivals, then compaction arrivals: one control block
     w.cdone = off + (size_t)s->batch * sizeof(int32_t);
     off = align256(off + 2 * (size_t)s->batch * sizeof(int32_t));
     w.moves = off;
-    off = align256(off + R * cap * 2 * sizeof(int32_t));
+    off = align256(off + Rs * cap * 2 * sizeof(int32_t));
     w.n_moves = off;
-    off = align256(off + R * sizeof(int32_t));
+    off = align256(off + Rs * sizeof(int32_t));
     // scorer variants: entropy pass buffers and VNorm means
     const size_t blk_max = ((size_t)cap + 31) / 32;
     w.sbuf = off;
@@ -160,11 +163,13 @@ StepWs step_ws(const ikv_shape *s, int32_t cap, int32_t pos_cap) {
     off = align256(off + (size_t)s->batch * s->layers * s->kv_heads * sizeof(float));
     w.slot = off;  // split step: each sequence's reserved slot
     off = align256(off + (size_t)s->batch * sizeof(int32_t));
-    // per-layer eviction: pending-update marks by position, one layer's utilities by slot
-    w.lam = off;
-    if (pos_cap > 0) off = align256(off + (size_t)s->batch * pos_cap * sizeof(int32_t));
+    // per-layer eviction: every layer's position -> slot map, every layer's utilities by slot
+    w.inv = off;
+    if (pos_cap > 0) off = align256(off + (size_t)s->batch * s->layers * pos_cap * sizeof(int32_t));
     w.util = off;
-    if (pos_cap > 0) off = align256(off + (size_t)s->batch * cap * sizeof(float));
+    if (pos_cap > 0) off = align256(off + (size_t)s->batch * s->layers * cap * sizeof(float));
+    w.live = off;
+    if (pos_cap > 0) off = align256(off + (size_t)s->batch * ((pos_cap + 31) / 32) * sizeof(uint32_t));
     w.end = off;
     return w;
 }
@@ -295,7 +300,7 @@ struct ScorerWs {
 ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, const int32_t *elig, int n_elig,
                      int32_t max_len, void *ws, const AttendWs &w, float alpha, float *ema, float *score,
                      cudaStream_t st, int32_t agg = IKV_AGG_EMA, int32_t scorer = IKV_SCORE_ATTENTION,
-                     const ScorerWs &sw = ScorerWs{}, int32_t layer0 = 0) {
+                     const ScorerWs &sw = ScorerWs{}, int32_t layer0 = 0, bool store_only = false) {
     ScoreArgs base{};
     base.len = c->len;
     base.batch = s->batch;
@@ -319,10 +324,11 @@ ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, c
     base.sbuf = sw.sbuf;
     base.epart = sw.epart;
     base.n_elig_total = n_elig;
+    base.store_only = store_only ? 1 : 0;
     int V = 1;
     base.nblk = score_blocks(base, max_len, sm_count(), &V);
     base.blk_tok = 32 * V;
-    if (scorer == IKV_SCORE_VNORM) IKV_TRY_CUDA(launch_vnorm_mean(base, st), "vnorm mean launch");
+    if (scorer == IKV_SCORE_VNORM && !store_only) IKV_TRY_CUDA(launch_vnorm_mean(base, st), "vnorm mean launch");
     for (int k0 = 0; k0 < n_elig; k0 += kMaxLayersPerScorePass) {
         ScoreArgs sa = base;
         sa.n_elig = n_elig - k0 < kMaxLayersPerScorePass ? n_elig - k0 : kMaxLayersPerScorePass;
@@ -330,7 +336,8 @@ ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, c
         for (int k = 0; k < sa.n_elig; ++k) sa.elig[k] = elig[k0 + k];
         IKV_TRY_CUDA(launch_score_ema(sa, max_len, sm_count(), st), "score launch");
     }
-    if (scorer == IKV_SCORE_ENTROPY) IKV_TRY_CUDA(launch_entropy_fold(base, max_len, st), "entropy fold launch");
+    if (scorer == IKV_SCORE_ENTROPY && !store_only)
+        IKV_TRY_CUDA(launch_entropy_fold(base, max_len, st), "entropy fold launch");
     return IKV_OK;
 }
 
@@ -456,7 +463,7 @@ ikv_status ikv_compact_workspace_size(const ikv_shape *shape, const ikv_cache *c
 
 static ikv_status compact_impl(const ikv_shape *shape, ikv_cache *cache, const int32_t *keep, const int32_t *keep_len,
                                float *ema, int32_t mode, int32_t *moves, int32_t *n_moves, int32_t *done,
-                               cudaStream_t stream, int32_t max_holes = 0, int32_t layer = -1) {
+                               cudaStream_t stream, int32_t max_holes = 0, bool by_layer = false) {
     CompactArgs a{};
     a.k = cache->k;
     a.v = cache->v;
@@ -478,14 +485,9 @@ static ikv_status compact_impl(const ikv_shape *shape, ikv_cache *cache, const i
     a.n_moves = n_moves;
     a.max_holes = max_holes;
     a.vnorm = cache->vnorm;
-    a.pos_rows = a.rows_per_seq;
-    a.publish_len = 1;
-    if (layer >= 0) {  // per-layer eviction: that layer's rows and position row; len published later
-        a.layers = 1;
-        a.layer0 = layer;
-        a.pos_rows = shape->layers;
-        a.pos_row0 = layer;
-        a.publish_len = 0;
+    if (by_layer) {  // per-layer eviction: keep row (b, l) governs layer l's rows and pos row
+        a.rows_per_seq = shape->layers;
+        a.row_by_layer = 1;
     }
     IKV_TRY_CUDA(launch_compact(a, mode, stream), "compact launch");
     return IKV_OK;
@@ -597,11 +599,10 @@ static ikv_status prepare_step(const ikv_shape *shape, const ikv_params *p, cons
     cx->layerwise = p->evict_mode == IKV_EVICT_LAYER;
     if (p->evict_mode != IKV_EVICT_STEP && !cx->layerwise) return fail(IKV_ERR_ARG, "unknown evict_mode %d", p->evict_mode);
     if (cx->layerwise) {
-        if (shape->granularity != IKV_GRAN_SEQ || p->compact_mode != IKV_COMPACT_STABLE || p->max_holes != 0 ||
-            p->agg_mode != IKV_AGG_EMA || p->scorer != IKV_SCORE_ATTENTION)
+        if (shape->granularity != IKV_GRAN_SEQ || p->max_holes != 0 || p->agg_mode != IKV_AGG_EMA ||
+            p->scorer != IKV_SCORE_ATTENTION)
             return fail(IKV_ERR_UNSUPPORTED,
-                        "IKV_EVICT_LAYER needs IKV_GRAN_SEQ, IKV_COMPACT_STABLE, max_holes 0, IKV_AGG_EMA and "
-                        "IKV_SCORE_ATTENTION");
+                        "IKV_EVICT_LAYER needs IKV_GRAN_SEQ, max_holes 0, IKV_AGG_EMA and IKV_SCORE_ATTENTION");
         if (cache->pos_cap <= 0) return fail(IKV_ERR_ARG, "IKV_EVICT_LAYER needs cache->pos_cap > 0");
         if (cache->dead_slots) return fail(IKV_ERR_ARG, "IKV_EVICT_LAYER does not use dead slots");
     }
@@ -647,7 +648,6 @@ static LayerArgs layer_args(const ikv_shape *shape, const ikv_params *p, const i
     LayerArgs a{};
     a.batch = shape->batch;
     a.layers = shape->layers;
-    a.q_heads = shape->q_heads;
     a.cap = cx.cap;
     a.pos_cap = cache->pos_cap;
     a.len = cache->len;
@@ -655,48 +655,40 @@ static LayerArgs layer_args(const ikv_shape *shape, const ikv_params *p, const i
     a.pos = cache->pos;
     a.start = cache->start;
     a.m = ema;
-    a.lam = at<int32_t>(ws, cx.w.lam);
+    a.inv = at<int32_t>(ws, cx.w.inv);
     a.util = at<float>(ws, cx.w.util);
-    a.logits = at<float>(ws, cx.w.at.logits);
-    a.lse2 = at<float>(ws, cx.w.at.lse2);
-    a.sc_layers = shape->layers;
+    a.live = at<uint32_t>(ws, cx.w.live);
+    a.live_words = (cache->pos_cap + 31) / 32;
+    a.sbuf = cx.sw.sbuf;
     a.lstride = logit_stride(cx.cap);
+    a.n_elig = cx.n_elig;
     a.alpha = p->alpha;
+    a.scoring = cx.scoring ? 1 : 0;
+    for (int k = 0; k < cx.n_elig; ++k) a.elig_bits[cx.elig[k] >> 5] |= 1u << (cx.elig[k] & 31);
     a.init_mean = cx.init_mean;
     a.slot = at<int32_t>(ws, cx.w.slot);
-    a.keep_len = at<int32_t>(ws, cx.w.keep_len);
     return a;
 }
 
-// Per-layer eviction of one layer after its attention: its utilities (with its score
-// folded in on scoring layers), its top-budget selection and the compaction of its rows.
-static ikv_status evict_layer(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, void *ws,
-                              const StepCtx &cx, int32_t layer, cudaStream_t stream) {
-    LayerArgs la = layer_args(shape, p, cache, ema, ws, cx);
-    int k_done = 0;
-    bool eligible = false;
-    for (int k = 0; k < cx.n_elig; ++k) {
-        if (cx.elig[k] < layer) ++k_done;
-        eligible |= cx.elig[k] == layer;
-    }
-    la.layer = layer;
-    la.k_done = cx.scoring ? k_done : 0;
-    la.scoring = cx.scoring && eligible;
-    IKV_TRY_CUDA(launch_layer_util(la, cx.L1, stream), "layer utility launch");
-    IKV_TRY_CUDA(launch_select(shape->batch, cx.cap, la.util, cache->len, 1, p->budget, nullptr,
+// Per-layer eviction after every layer's attention: the eligible layers' pooled scores
+// (refresh steps), the per-position fold giving each layer's utilities and the new
+// state, then every (sequence, layer) row selected and every layer compacted at once.
+static ikv_status layer_evict(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, void *ws,
+                              const StepCtx &cx, cudaStream_t stream) {
+    ikv_status e;
+    if (cx.scoring && (e = run_score(shape, cache, shape->layers, cx.elig, cx.n_elig, cx.L1, ws, cx.w.at, p->alpha,
+                                     nullptr, nullptr, stream, IKV_AGG_EMA, IKV_SCORE_ATTENTION, cx.sw, 0, true)))
+        return e;
+    IKV_TRY_CUDA(launch_layer_fold(layer_args(shape, p, cache, ema, ws, cx), cx.L1, cache->pos_cap, stream),
+                 "layer fold launch");
+    const int32_t K = shape->layers;
+    IKV_TRY_CUDA(launch_select(shape->batch * K, cx.cap, at<float>(ws, cx.w.util), cache->len, K, p->budget, nullptr,
                                at<int32_t>(ws, cx.w.keep), at<int32_t>(ws, cx.w.keep_len), DeferArgs{0, cx.cap, nullptr},
                                stream),
                  "select launch");
     return compact_impl(shape, cache, at<int32_t>(ws, cx.w.keep), at<int32_t>(ws, cx.w.keep_len), nullptr,
-                        IKV_COMPACT_STABLE, nullptr, nullptr, at<int32_t>(ws, cx.w.cdone), stream, 0, layer);
-}
-
-static ikv_status layer_end(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, void *ws,
-                            const StepCtx &cx, cudaStream_t stream) {
-    LayerArgs la = layer_args(shape, p, cache, ema, ws, cx);
-    la.n_elig = cx.scoring ? cx.n_elig : 0;
-    IKV_TRY_CUDA(launch_layer_end(la, stream), "layer end launch");
-    return IKV_OK;
+                        p->compact_mode, at<int32_t>(ws, cx.w.moves), at<int32_t>(ws, cx.w.n_moves),
+                        at<int32_t>(ws, cx.w.cdone), stream, 0, true);
 }
 
 ikv_status ikv_step_workspace_size(const ikv_shape *shape, const ikv_cache *cache, size_t *bytes) {
@@ -724,12 +716,15 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     const ikv_timing *tm = p->timing;
     if (cx.layerwise) {
         // begin, every layer's new rows, one attention launch for all layers (each reads
-        // its own rows as they stood before this step's evictions), then layer by layer:
-        // utilities, selection, compaction; the pending decays at the end
+        // its own rows), then the per-layer evictions
         IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.at.arrivals), 0, w.at.logits - w.at.arrivals, stream),
                      "cudaMemsetAsync");
+        IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.done), 0, 2 * sizeof(int32_t) * shape->batch, stream),
+                     "cudaMemsetAsync");
         LayerArgs la = layer_args(shape, p, cache, ema, ws, cx);
-        IKV_TRY_CUDA(launch_layer_begin(la, stream), "layer begin launch");
+        IKV_TRY_CUDA(cudaMemsetAsync(la.live, 0, sizeof(uint32_t) * (size_t)shape->batch * la.live_words, stream),
+                     "cudaMemsetAsync");
+        IKV_TRY_CUDA(launch_layer_begin(la, cache->max_len, stream), "layer begin launch");
         PdlScope pdl;
         AppendArgs ap{};
         ap.k = cache->k;
@@ -747,9 +742,7 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
         if ((e = run_attend(shape, cache, 0, shape->layers, cx.L1, q, out, ws, w.at, cx.scoring, nullptr, nullptr,
                             stream, nullptr, true)))
             return e;
-        for (int l = 0; l < shape->layers; ++l)
-            if ((e = evict_layer(shape, p, cache, ema, ws, cx, l, stream))) return e;
-        return layer_end(shape, p, cache, ema, ws, cx, stream);
+        return layer_evict(shape, p, cache, ema, ws, cx, stream);
     }
 
     // control words (append and split-arrival counters) start at zero
@@ -790,7 +783,10 @@ ikv_status ikv_step_begin(const ikv_shape *shape, const ikv_params *p, ikv_cache
     IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, cx.w.done), 0, 2 * sizeof(int32_t) * shape->batch, stream),
                  "cudaMemsetAsync");
     if (cx.layerwise) {
-        IKV_TRY_CUDA(launch_layer_begin(layer_args(shape, p, &cx.cv, ema, ws, cx), stream), "layer begin launch");
+        LayerArgs la = layer_args(shape, p, &cx.cv, ema, ws, cx);
+        IKV_TRY_CUDA(cudaMemsetAsync(la.live, 0, sizeof(uint32_t) * (size_t)shape->batch * la.live_words, stream),
+                     "cudaMemsetAsync");
+        IKV_TRY_CUDA(launch_layer_begin(la, cache->max_len, stream), "layer begin launch");
         return IKV_OK;
     }
     return append_impl(shape, &cx.cv, nullptr, nullptr, ema, cx.init_mean, at<int32_t>(ws, cx.w.done), stream, true,
@@ -829,10 +825,8 @@ ikv_status ikv_step_layer(const ikv_shape *shape, const ikv_params *p, ikv_cache
     // the new token's rows and one layer's attention; on refresh steps its logits and
     // log-sum-exp land where the whole step's attention would put them, for
     // ikv_step_end's score pass
-    if ((e = run_attend(shape, cache, layer, 1, cx.L1, q, out, ws, cx.w.at, cx.scoring && eligible, nullptr, nullptr,
-                        stream, nullptr, true, shape->layers, layer, &a)))
-        return e;
-    return cx.layerwise ? evict_layer(shape, p, cache, ema, ws, cx, layer, stream) : IKV_OK;
+    return run_attend(shape, cache, layer, 1, cx.L1, q, out, ws, cx.w.at, cx.scoring && eligible, nullptr, nullptr,
+                      stream, nullptr, true, shape->layers, layer, &a);
 }
 
 ikv_status ikv_step_end(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, int32_t t,
@@ -842,7 +836,7 @@ ikv_status ikv_step_end(const ikv_shape *shape, const ikv_params *p, ikv_cache *
     ikv_status e = prepare_step(shape, p, cache, ema, t, ws, ws_bytes, &cx);
     if (e) return e;
     PdlScope pdl;
-    if (cx.layerwise) return layer_end(shape, p, &cx.cv, ema, ws, cx, stream);
+    if (cx.layerwise) return layer_evict(shape, p, &cx.cv, ema, ws, cx, stream);
     if (cx.scoring && (e = run_score(shape, &cx.cv, shape->layers, cx.elig, cx.n_elig, cx.L1, ws, cx.w.at, p->alpha,
                                      ema, nullptr, stream, p->agg_mode, p->scorer, cx.sw)))
         return e;

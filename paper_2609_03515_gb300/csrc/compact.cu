@@ -154,10 +154,10 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
         }
     }
     // whatever the mode, the next append must find a free slot: else move every row to slot 0
-    if (a.start && a.publish_len && new_start + n0 + 1 > a.cap) new_start = 0;
+    if (a.start && new_start + n0 + 1 > a.cap) new_start = 0;
     if (x < nkv) {
-        const int l = a.layer0 + x / kvh, g = x % kvh;
-        const int r = b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g);
+        const int l = x / kvh, g = x % kvh;
+        const int r = b * a.rows_per_seq + (a.row_by_layer ? l : a.rows_per_seq == 1 ? 0 : g);
         const int n = a.keep_len[r];
         const int32_t *kp = a.keep + (int64_t)r * a.cap;
         const int shift = new_start - S;
@@ -225,7 +225,7 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
         const int r = b * a.rows_per_seq + rr;
         const int n = a.keep_len[r];
         const int32_t *kp = a.keep + (int64_t)r * a.cap;
-        int32_t *pos = a.pos + ((int64_t)b * a.pos_rows + a.pos_row0 + rr) * a.cap;
+        int32_t *pos = a.pos + (int64_t)r * a.cap;
         float *ema = a.ema ? a.ema + (int64_t)r * a.cap : nullptr;
         constexpr int PER = 16;
         for (int base = 0; base < n; base += kCompThreads * PER) {
@@ -254,7 +254,6 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
         }
     }
     // publish len / start once every CTA of b has read them
-    if (!a.publish_len) return;
     __syncthreads();
     if (tid == 0) {
         __threadfence();
@@ -321,7 +320,7 @@ __global__ void __launch_bounds__(kCompThreads) holefill_move_kernel(const Compa
     if (a.keep_len[b * a.rows_per_seq] < 0) return;  // selection marked the victim dead: nothing to do
     if (x < nkv) {
         const int l = x / kvh, g = x % kvh;
-        const int r = b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g);
+        const int r = b * a.rows_per_seq + (a.row_by_layer ? l : a.rows_per_seq == 1 ? 0 : g);
         const int nm = a.n_moves[r];  // -1: deferred, nothing moves
         const int32_t *mv = a.moves + (int64_t)r * a.cap * 2;
         const int S = a.pv.start_of(b);

@@ -129,6 +129,7 @@ struct ScoreArgs {
     int32_t blk_tok;            // entropy: tokens per block of the score pass
     int32_t k0;                 // eligible-layer index of this pass's first layer
     int32_t n_elig_total;       // eligible layers over all passes
+    int32_t store_only;         // Eq. 1 scorer: only store each layer's pooled score in sbuf
 };
 
 // tensor-core attention (bf16, head_dim 128): attend_tc.cu
@@ -183,9 +184,8 @@ struct CompactArgs {
     int32_t max_holes;          // > 0: while a sequence's dead slots stay <= max_holes, mark
                                 // the evicted slots dead (pos = -1) instead of compacting
     float *vnorm;               // [layers][batch][kv_heads][cap] value-row norms moved with the rows, or null
-    int32_t layer0;             // the K/V rows compacted are those of layers layer0 .. layer0 + layers - 1
-    int32_t pos_rows, pos_row0; // utility row rr of sequence b uses pos row b * pos_rows + pos_row0 + rr
-    int32_t publish_len;        // 1: the last CTA of b writes len / start; 0: left to the caller
+    int32_t row_by_layer;       // per-layer eviction: keep row b * rows_per_seq + l governs layer l
+                                // (all kv heads) and pos row b * rows_per_seq + l
 };
 cudaError_t launch_compact(const CompactArgs &a, int mode, cudaStream_t st);
 
@@ -211,31 +211,34 @@ cudaError_t launch_append(const AppendArgs &a, cudaStream_t st);
 cudaError_t launch_append_rows(const AppendArgs &a, cudaStream_t st);
 
 // Per-layer eviction (IKV_EVICT_LAYER): a position-indexed state m [batch][pos_cap]
-// shared by all layers, layer l's positions in pos row b * layers + l.  A layer's
-// update decays every live position it does not hold; that decay is applied lazily:
-// lam[p] is the index, among this step's eligible layers, of the last one that
-// updated p (-1: none yet), and the stored m[p] is its value as of that update.
+// shared by all layers; layer l's positions in pos row b * layers + l.  Within a step no
+// layer's eviction feeds another layer's inputs (each attends its own rows, and a
+// layer's update only reads the tokens it held before the step's evictions), so every
+// layer's utilities are computed after all attention, by one pass over positions that
+// walks the layers in order, and all layers are selected and compacted together.
 struct LayerArgs {
-    int32_t batch, layers, q_heads, cap, pos_cap;
+    int32_t batch, layers, cap, pos_cap;
     int32_t *len, *next_pos, *pos;
     const int32_t *start;       // [batch] or null
-    float *m;                   // [batch][pos_cap]
-    int32_t *lam;               // [batch][pos_cap] workspace
-    float *util;                // [batch][cap] workspace: the layer's utilities by slot
-    const float *logits, *lse2; // [batch][sc_layers][H][lstride], [batch][sc_layers][H]
-    int32_t sc_layers, lstride;
+    float *m;                   // [batch][pos_cap] state
+    int32_t *inv;               // [batch][layers][pos_cap] workspace: slot of position p in layer l
+                                // (stale entries are rejected by checking pos[l][slot] == p)
+    uint32_t *live;             // [batch][live_words] workspace: bit p = some layer holds position p
+    int32_t live_words;         // ceil(pos_cap / 32)
+    float *util;                // [batch][layers][cap] workspace: utilities by slot
+    const float *sbuf;          // [batch][n_elig][lstride] pooled scores of the eligible layers
+    int32_t lstride, n_elig;
     float alpha;
-    int32_t layer;              // util: the layer
-    int32_t k_done;             // util: eligible layers folded earlier in this step
-    int32_t scoring;            // util: fold this layer's Eq. 1 score
+    int32_t scoring;            // refresh step: fold the eligible layers' scores
+    uint32_t elig_bits[kMaxLayers / 32];
     int32_t init_mean;          // begin: new token's state = mean over live positions (else 0)
     int32_t *slot;              // begin: each sequence's reserved slot, -1 if none
-    const int32_t *keep_len;    // end: the step's kept count per sequence
-    int32_t n_elig;             // end: eligible layers folded this step (0: no pending decay)
 };
-cudaError_t launch_layer_begin(const LayerArgs &a, cudaStream_t st);
-cudaError_t launch_layer_util(const LayerArgs &a, int32_t max_len, cudaStream_t st);
-cudaError_t launch_layer_end(const LayerArgs &a, cudaStream_t st);
+// live-position bits of the cache before the append (live must be zeroed first), then
+// the append bookkeeping; max_len bounds len before the append
+cudaError_t launch_layer_begin(const LayerArgs &a, int32_t max_len, cudaStream_t st);
+// inverse maps of every layer, then the per-position fold (utilities and final state)
+cudaError_t launch_layer_fold(const LayerArgs &a, int32_t max_len, int32_t max_pos, cudaStream_t st);
 cudaError_t read_clear_layer_error(unsigned int *v);
 // reads and clears the append kernel's device error word (bit 0: no free slot)
 cudaError_t read_clear_append_error(unsigned int *v);

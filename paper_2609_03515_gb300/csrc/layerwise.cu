@@ -2,10 +2,14 @@
 // into a state indexed by token position and shared by all layers, then keeps the
 // budget's highest-utility tokens among those it holds (Appendix "Layer scoring",
 // each layer's hook acting at once).  A live position that a layer does not hold gets
-// score 0 there, so Eq. 4 multiplies it by alpha; rather than touching every live
-// position at every layer, the decay is applied when the position is next read (its
-// pending count is the eligible layers since its last update) and, for the rest, once
-// at the end of the step.
+// score 0 there, so Eq. 4 multiplies it by alpha.
+//
+// No layer's eviction changes another layer's inputs within a step: a layer attends
+// its own rows, and its update reads only the tokens it held before the step's
+// evictions.  So after all attention (and the stored per-layer scores), one pass over
+// token positions walks the layers in order -- the state as each layer saw it is that
+// layer's utility for its slot of the position -- and every layer is then selected
+// and compacted at once by the step's usual kernels (rows = batch x layers).
 #include "ikv_internal.cuh"
 
 namespace ikv {
@@ -16,15 +20,21 @@ namespace {
 
 constexpr int kBeginThreads = 1024;
 
-// alpha^n by repeated multiplication, n >= 0 (at most the layer count)
-__device__ __forceinline__ float decay(float v, float alpha, int n) {
-    for (int i = 0; i < n; ++i) v *= alpha;
-    return v;
+// The live positions (held by some layer) as bits, set by one thread per (sequence,
+// layer, slot) into the cleared bitmap.  Nothing is evicted between here and the fold,
+// so with the new token's bit (set by the begin kernel) this is the fold's live set.
+constexpr int kMarkThreads = 256;
+__global__ void __launch_bounds__(kMarkThreads) layer_mark_kernel(const LayerArgs a) {
+    pdl_wait();
+    const int b = blockIdx.z, l = blockIdx.y;
+    const int j = blockIdx.x * kMarkThreads + threadIdx.x;
+    if (j >= a.len[b]) return;
+    const int p = a.pos[((int64_t)b * a.layers + l) * a.cap + j];
+    if (p >= 0 && p < a.pos_cap) atomicOr(a.live + (int64_t)b * a.live_words + (p >> 5), 1u << (p & 31));
 }
 
-// One CTA per sequence: the new token's state (0, or the mean over the positions some
-// layer holds, found by marking them in lam), its position in every layer's row, the
-// pending-update marks reset, then len and next_pos advanced.
+// One CTA per sequence: the new token's state (0, or the mean over the live positions),
+// its live bit and position in every layer's row, then len and next_pos advanced.
 __global__ void __launch_bounds__(kBeginThreads) layer_begin_kernel(const LayerArgs a) {
     pdl_wait();
     __shared__ float red[2][kBeginThreads / 32];
@@ -33,8 +43,8 @@ __global__ void __launch_bounds__(kBeginThreads) layer_begin_kernel(const LayerA
     const int L = a.len[b];
     const int S = a.start ? a.start[b] : 0;
     const int np = a.next_pos[b];
-    int32_t *lam = a.lam + (int64_t)b * a.pos_cap;
     float *m = a.m + (int64_t)b * a.pos_cap;
+    uint32_t *bits = a.live + (int64_t)b * a.live_words;
     if (S + L >= a.cap || np >= a.pos_cap) {
         if (tid == 0) {
             a.slot[b] = -1;
@@ -44,17 +54,9 @@ __global__ void __launch_bounds__(kBeginThreads) layer_begin_kernel(const LayerA
     }
     float init = 0.f;
     if (a.init_mean) {
-        for (int p = tid; p < np; p += kBeginThreads) lam[p] = 0;
-        __syncthreads();
-        for (int64_t i = tid; i < (int64_t)a.layers * L; i += kBeginThreads) {
-            const int l = (int)(i / L), j = (int)(i % L);
-            const int p = a.pos[((int64_t)b * a.layers + l) * a.cap + j];
-            if (p >= 0 && p < np) lam[p] = 1;
-        }
-        __syncthreads();
         float sum = 0.f, cnt = 0.f;
         for (int p = tid; p < np; p += kBeginThreads)
-            if (lam[p] == 1) {
+            if ((bits[p >> 5] >> (p & 31)) & 1u) {
                 sum += m[p];
                 cnt += 1.f;
             }
@@ -69,10 +71,10 @@ __global__ void __launch_bounds__(kBeginThreads) layer_begin_kernel(const LayerA
         for (int w = 0; w < kBeginThreads / 32; ++w) ts += red[0][w], tc += red[1][w];
         init = tc > 0.f ? ts / tc : 0.f;
     }
-    __syncthreads();  // every thread has read len / next_pos and the marks
-    for (int p = tid; p <= np; p += kBeginThreads) lam[p] = -1;
+    __syncthreads();  // every thread has read len / next_pos and the bits
     for (int l = tid; l < a.layers; l += kBeginThreads) a.pos[((int64_t)b * a.layers + l) * a.cap + L] = np;
     if (tid == 0) {
+        bits[np >> 5] |= 1u << (np & 31);  // the new token is live too
         m[np] = init;
         a.slot[b] = L;
         a.next_pos[b] = np + 1;
@@ -80,73 +82,68 @@ __global__ void __launch_bounds__(kBeginThreads) layer_begin_kernel(const LayerA
     }
 }
 
-// One thread per slot j of layer `layer`: the position's utility as of this layer
-// (pending decays applied), with this layer's Eq. 1 score folded in on scoring layers
-// (then stored back, marked as updated by this layer).  Writes util[b][j].
-constexpr int kUtilThreads = 256;
-__global__ void __launch_bounds__(kUtilThreads) layer_util_kernel(const LayerArgs a) {
+// inv[b][l][pos[b][l][j]] = j for every slot j < len[b] of every layer
+constexpr int kInvThreads = 256;
+__global__ void __launch_bounds__(kInvThreads) layer_inverse_kernel(const LayerArgs a) {
     pdl_wait();
-    const int b = blockIdx.y;
-    const int j = blockIdx.x * kUtilThreads + threadIdx.x;
-    const int L = a.len[b];
-    if (j >= L) return;
-    const int p = a.pos[((int64_t)b * a.layers + a.layer) * a.cap + j];
-    float *util = a.util + (int64_t)b * a.cap;
-    if (p < 0 || p >= a.pos_cap) {  // not a valid position: never kept
-        util[j] = -INFINITY;
-        return;
-    }
-    float *m = a.m + (int64_t)b * a.pos_cap;
-    int32_t *lam = a.lam + (int64_t)b * a.pos_cap;
-    float v = decay(m[p], a.alpha, (a.k_done - 1) - lam[p]);
-    if (a.scoring) {
-        const int H = a.q_heads;
-        const int64_t row = (int64_t)b * a.sc_layers + a.layer;
-        const float *z = a.logits + row * H * (int64_t)a.lstride + j;
-        const float *l2 = a.lse2 + row * H;
-        float s = 0.f;
-        for (int h = 0; h < H; ++h) s += exp2f(__ldg(z + (int64_t)h * a.lstride) - __ldg(l2 + h));
-        v = a.alpha * v + (1.f - a.alpha) * (s / (float)H);
-        m[p] = v;
-        lam[p] = a.k_done;
-    }
-    util[j] = v;
+    const int b = blockIdx.z, l = blockIdx.y;
+    const int j = blockIdx.x * kInvThreads + threadIdx.x;
+    if (j >= a.len[b]) return;
+    const int p = a.pos[((int64_t)b * a.layers + l) * a.cap + j];
+    if (p >= 0 && p < a.pos_cap) a.inv[((int64_t)b * a.layers + l) * a.pos_cap + p] = j;
 }
 
-// End of a step: the decays still pending (eligible layers after a position's last
-// update) are applied to every position below next_pos; len becomes the kept count.
-constexpr int kEndThreads = 256;
-__global__ void __launch_bounds__(kEndThreads) layer_end_kernel(const LayerArgs a) {
+// One thread per live token position p (held by some layer): walks the layers in
+// order; at every eligible layer of a refresh step m <- alpha m + (1 - alpha) s, s the
+// layer's pooled score of p if it holds p, else 0; each layer holding p gets m as its
+// utility of p's slot.  The final m is stored.  Dead positions are left as they are.
+constexpr int kFoldThreads = 256;
+__global__ void __launch_bounds__(kFoldThreads) layer_fold_kernel(const LayerArgs a) {
     pdl_wait();
     const int b = blockIdx.y;
-    const int p = blockIdx.x * kEndThreads + threadIdx.x;
-    if (a.n_elig > 0 && p < a.next_pos[b] && p < a.pos_cap) {
-        float *m = a.m + (int64_t)b * a.pos_cap;
-        const int32_t *lam = a.lam + (int64_t)b * a.pos_cap;
-        m[p] = decay(m[p], a.alpha, (a.n_elig - 1) - lam[p]);
+    const int p = blockIdx.x * kFoldThreads + threadIdx.x;
+    if (p >= a.next_pos[b] || p >= a.pos_cap) return;
+    if (!((a.live[(int64_t)b * a.live_words + (p >> 5)] >> (p & 31)) & 1u)) return;
+    const int L = a.len[b];
+    float *mp = a.m + (int64_t)b * a.pos_cap + p;
+    float m = *mp;
+    int k = 0;  // eligible layers folded so far
+    for (int l = 0; l < a.layers; ++l) {
+        const int64_t row = (int64_t)b * a.layers + l;
+        const int j = a.inv[row * a.pos_cap + p];
+        const bool held = j >= 0 && j < L && a.pos[row * a.cap + j] == p;
+        if (a.scoring && ((a.elig_bits[l >> 5] >> (l & 31)) & 1u)) {
+            const float s = held ? a.sbuf[((int64_t)b * a.n_elig + k) * a.lstride + j] : 0.f;
+            m = a.alpha * m + (1.f - a.alpha) * s;
+            ++k;
+        }
+        if (held) a.util[row * a.cap + j] = m;
     }
-    if (blockIdx.x == 0 && threadIdx.x == 0) a.len[b] = a.keep_len[b];
+    *mp = m;
 }
 
 }  // namespace
 
-cudaError_t launch_layer_begin(const LayerArgs &a, cudaStream_t st) {
+cudaError_t launch_layer_begin(const LayerArgs &a, int32_t max_len, cudaStream_t st) {
+    if (max_len > 0) {
+        cudaError_t e = launch_k(layer_mark_kernel, dim3((max_len + kMarkThreads - 1) / kMarkThreads, a.layers, a.batch),
+                                 dim3(kMarkThreads), 0, st, a);
+        note_launch();
+        if (e != cudaSuccess) return e;
+    }
     cudaError_t e = launch_k(layer_begin_kernel, dim3(a.batch), dim3(kBeginThreads), 0, st, a);
     note_launch();
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-cudaError_t launch_layer_util(const LayerArgs &a, int32_t max_len, cudaStream_t st) {
-    if (max_len <= 0) return cudaSuccess;
-    dim3 grid((max_len + kUtilThreads - 1) / kUtilThreads, a.batch);
-    cudaError_t e = launch_k(layer_util_kernel, grid, dim3(kUtilThreads), 0, st, a);
+cudaError_t launch_layer_fold(const LayerArgs &a, int32_t max_len, int32_t max_pos, cudaStream_t st) {
+    if (max_len <= 0 || max_pos <= 0) return cudaSuccess;
+    cudaError_t e = launch_k(layer_inverse_kernel, dim3((max_len + kInvThreads - 1) / kInvThreads, a.layers, a.batch),
+                             dim3(kInvThreads), 0, st, a);
     note_launch();
-    return e != cudaSuccess ? e : cudaGetLastError();
-}
-
-cudaError_t launch_layer_end(const LayerArgs &a, cudaStream_t st) {
-    dim3 grid((a.pos_cap + kEndThreads - 1) / kEndThreads, a.batch);
-    cudaError_t e = launch_k(layer_end_kernel, grid, dim3(kEndThreads), 0, st, a);
+    if (e != cudaSuccess) return e;
+    e = launch_k(layer_fold_kernel, dim3((max_pos + kFoldThreads - 1) / kFoldThreads, a.batch), dim3(kFoldThreads), 0,
+                 st, a);
     note_launch();
     return e != cudaSuccess ? e : cudaGetLastError();
 }

@@ -118,6 +118,12 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
         }
 #pragma unroll
         for (int v = 0; v < V; ++v) sl[warp][lane * V + v] = acc[v] * inv;
+        if (SCORER != IKV_SCORE_ENTROPY && a.store_only) {  // each layer's pooled score, unfolded
+            const int k = a.k0 + warp;
+#pragma unroll
+            for (int v = 0; v < V; ++v)
+                if (il + v < L) a.sbuf[((int64_t)r * a.n_elig_total + k) * a.lstride + il + v] = acc[v] * inv;
+        }
         if (SCORER == IKV_SCORE_ENTROPY) {
             // the layer's pooled scores, and this block's share of -sum s ln s over them
             const int k = a.k0 + warp;
@@ -148,6 +154,7 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
         }
         return;
     }
+    if (a.store_only) return;
     __syncthreads();
     if (folds) {
         float sc = 0.f;

@@ -123,13 +123,14 @@ def live_slots(pos_row: np.ndarray, n: int) -> np.ndarray:
 def decode_step(c: DecodeCache, p, cache, t: int, q, kn, vn, out, ws, per_layer: bool = False) -> None:
     """One decode step through the C ABI: ikv_step, or its begin / per-layer / end split
     (q, kn, vn, out: [layers][batch][...] device tensors)."""
+    m = c.utility(p.evict_mode)
     if not per_layer:
-        ikv.ikv_step(c.shape(), p, cache, c.ema, t, q, kn, vn, out, ws, ws.numel())
+        ikv.ikv_step(c.shape(), p, cache, m, t, q, kn, vn, out, ws, ws.numel())
         return
-    ikv.ikv_step_begin(c.shape(), p, cache, c.ema, t, ws, ws.numel())
+    ikv.ikv_step_begin(c.shape(), p, cache, m, t, ws, ws.numel())
     for l in range(c.layers):
-        ikv.ikv_step_layer(c.shape(), p, cache, c.ema, t, l, q[l], kn[l], vn[l], out[l], ws, ws.numel())
-    ikv.ikv_step_end(c.shape(), p, cache, c.ema, t, ws, ws.numel())
+        ikv.ikv_step_layer(c.shape(), p, cache, m, t, l, q[l], kn[l], vn[l], out[l], ws, ws.numel())
+    ikv.ikv_step_end(c.shape(), p, cache, m, t, ws, ws.numel())
 
 
 def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: int = ikv.IKV_COMPACT_STABLE,
@@ -300,7 +301,8 @@ def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1)
 
 
 def run_lockstep_layerwise(w: gen.Workload, steps: Optional[int] = None, page_perm_seed: Optional[int] = 7,
-                           refresh_init: int = ikv.IKV_INIT_ZERO, layer_eligible=None, per_layer: bool = False):
+                           refresh_init: int = ikv.IKV_INIT_ZERO, layer_eligible=None, per_layer: bool = False,
+                           compact_mode: int = ikv.IKV_COMPACT_STABLE):
     """Per-layer immediate eviction (IKV_EVICT_LAYER) in lock-step with the oracle's
     decode_step_layerwise.  Per step: every layer's attention output, every layer's kept
     positions under the boundary rule against the oracle's utilities at that layer's
@@ -323,7 +325,7 @@ def run_lockstep_layerwise(w: gen.Workload, steps: Optional[int] = None, page_pe
     op = O.Params(alpha=w.alpha, refresh_period=w.refresh_period, score_free=w.score_free,
                   layer_mask=None if layer_eligible is None else [bool(x) for x in layer_eligible],
                   refresh_init="zero" if refresh_init == ikv.IKV_INIT_ZERO else "mean")
-    p = c.params(w.alpha, w.refresh_period, w.score_free, ikv.IKV_COMPACT_STABLE, refresh_init, layer_eligible,
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, refresh_init, layer_eligible,
                  evict_mode=ikv.IKV_EVICT_LAYER)
     ws = c.step_workspace()
     qs = w.queries(1, T + 1, u)
@@ -337,18 +339,22 @@ def run_lockstep_layerwise(w: gen.Workload, steps: Optional[int] = None, page_pe
         lens = [min(L + 1, B) for L, B in zip(lens, budgets)]
         torch.cuda.synchronize()
         out_h = out.float().cpu().numpy()
-        m_h = c.ema.cpu().numpy()
+        m_h = c.pos_state.cpu().numpy()
         pos_h = c.pos.cpu().numpy()
         len_h = c.len.cpu().numpy()
         rep = StepReport(t=t, refresh=O.is_refresh(t, w.refresh_period, w.score_free))
         q64 = as_f64(qs[t - 1], w)
         for b, st in enumerate(sts):
             assert len_h[b] == lens[b], (t, b, len_h[b], lens[b])
-            gpu_kept = [pos_h[b * w.layers + l, :lens[b]].astype(np.int64) for l in range(w.layers)]
+            gpu_slots = [pos_h[b * w.layers + l, :lens[b]].astype(np.int64) for l in range(w.layers)]
+            if compact_mode in STABLE_MODES:                    # survivors keep their order (R5)
+                for l in range(w.layers):
+                    assert np.all(np.diff(gpu_slots[l]) > 0), (t, b, l)
+            gpu_kept = [np.sort(x) for x in gpu_slots]
 
             def adopt(l, tr, b=b):
                 kept = gpu_kept[l]
-                assert np.all(np.diff(kept) > 0), (t, b, l)   # stable: ascending positions
+                assert len(np.unique(kept)) == len(kept), (t, b, l)
                 mask = np.isin(tr.pos, kept)
                 assert mask.sum() == len(kept), (t, b, l)      # kept positions were held by the layer
                 ok, _ = boundary_ok(tr.m, mask, budgets[b])
@@ -362,11 +368,97 @@ def run_lockstep_layerwise(w: gen.Workload, steps: Optional[int] = None, page_pe
             rep.m_err = max(rep.m_err, float(np.max(np.abs(m_h[b, live] - st.m[live]))))
             for l in range(w.layers):
                 assert np.array_equal(gpu_kept[l], st.pos[l]), (t, b, l)
+                order = np.argsort(gpu_slots[l])  # GPU slot order -> ascending positions
                 for g in range(w.kv_heads):
-                    gk = c.gather(c.k, b, l, g, lens[b]).float().cpu().numpy()
-                    gv = c.gather(c.v, b, l, g, lens[b]).float().cpu().numpy()
+                    gk = c.gather(c.k, b, l, g, lens[b]).float().cpu().numpy()[order]
+                    gv = c.gather(c.v, b, l, g, lens[b]).float().cpu().numpy()[order]
                     rep.kv_err = max(rep.kv_err, float(np.max(np.abs(gk - st.K[l][g]))),
                                      float(np.max(np.abs(gv - st.V[l][g]))))
+        reports.append(rep)
+    assert ikv.ikv_device_status() == 0
+    return reports
+
+
+def run_fullsize_sampled_layerwise(w: gen.Workload, seqs, steps: int, check_layers=(0, -1),
+                                   page_perm_seed: Optional[int] = 7, per_layer: bool = False):
+    """Full-size lock-step of per-layer immediate eviction for a few sequences (GRAN_SEQ).
+
+    As run_fullsize_sampled, but the oracle side keeps, per sampled sequence, each layer's
+    held positions and the position-indexed state, and restates decode_step_layerwise with
+    the layers' K/V rows regenerated by position (reading R10)."""
+    T = steps
+    u = w.u_table()
+    u_dev = torch.from_numpy(u).cuda()
+    c = DecodeCache(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.cap,
+                    dtype=ikv.IKV_BF16 if w.dtype == gen.BF16 else ikv.IKV_F32, page_size=w.page_size,
+                    page_perm_seed=page_perm_seed, pos_cap=max(w.prefill) + T + 1)
+    c.set_prefill(w.prefill, w.budgets())
+    fill_device(c, w, u_dev)
+    op = O.Params(alpha=w.alpha, refresh_period=w.refresh_period, score_free=w.score_free)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, ikv.IKV_COMPACT_STABLE, evict_mode=ikv.IKV_EVICT_LAYER)
+    ws = c.step_workspace()
+    qs = w.queries(1, T + 1, u)
+    budgets = w.budgets()
+    lens = list(w.prefill)
+    out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
+    sp = w.spec()
+    L0_dev = torch.tensor(w.prefill, dtype=torch.int32, device="cuda")
+    kn = torch.empty((1, w.layers, w.batch, w.kv_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
+    vn = torch.empty_like(kn)
+    state = {b: {"pos": [np.arange(w.prefill[b], dtype=np.int64) for _ in range(w.layers)],
+                 "m": np.zeros(w.prefill[b] + T + 1), "next": w.prefill[b]} for b in seqs}
+    reports = []
+    for t in range(1, T + 1):
+        assert gen.cuda_lib().ikvgen_fill_tokens_cuda(ctypes.byref(sp), u_dev.data_ptr(), L0_dev.data_ptr(), t, t + 1,
+                                                      w.dtype, kn.data_ptr(), vn.data_ptr(),
+                                                      torch.cuda.current_stream().cuda_stream) == 0
+        decode_step(c, p, c.cache(max(lens)), t, to_device(qs[t - 1], w), kn[0], vn[0], out, ws, per_layer)
+        lens = [min(L + 1, B) for L, B in zip(lens, budgets)]
+        torch.cuda.synchronize()
+        refresh = O.is_refresh(t, w.refresh_period, w.score_free)
+        rep = StepReport(t=t, refresh=refresh)
+        q64 = as_f64(qs[t - 1], w)
+        len_h = c.len.cpu().numpy()
+        pos_h = c.pos.cpu().numpy()
+        m_h = c.pos_state.cpu().numpy()
+        for b in seqs:
+            st = state[b]
+            assert len_h[b] == lens[b]
+            m = st["m"]
+            live = np.unique(np.concatenate(st["pos"]))
+            m[st["next"]] = 0.0 if refresh else float(np.mean(m[live]))
+            st["pos"] = [np.append(x, st["next"]) for x in st["pos"]]
+            st["next"] += 1
+            out_b = out[:, b].float().cpu().numpy()
+            for l in range(w.layers):
+                held = st["pos"][l]
+                k, v = w.kv_rows(b, l, held, u)
+                a_, o_ = O.last_query_attention(q64[l, b], [x.astype(np.float64) for x in k],
+                                                [x.astype(np.float64) for x in v])
+                rep.out_err = max(rep.out_err, float(np.max(np.abs(out_b[l] - o_))))
+                if refresh:
+                    s_pos = np.zeros_like(m)
+                    s_pos[held] = O.pooled_score(a_, O.GRAN_SEQ, w.kv_heads)[0]
+                    live = np.unique(np.concatenate(st["pos"]))
+                    m[live] = O.ema_update(m[live], s_pos[live], op.alpha)
+                m_l = m[held]
+                kept = pos_h[b * w.layers + l, :lens[b]].astype(np.int64)
+                assert np.all(np.diff(kept) > 0)
+                mask = np.isin(held, kept)
+                assert mask.sum() == len(kept)
+                ok, _ = boundary_ok(m_l, mask, budgets[b])
+                rep.set_ok &= ok
+                rep.strict_set_equal &= set(held[O.select_keep(m_l, budgets[b])].tolist()) == set(kept.tolist())
+                st["pos"][l] = kept
+            live = np.unique(np.concatenate(st["pos"]))
+            rep.m_err = max(rep.m_err, float(np.max(np.abs(m_h[b, live] - m[live]))))
+            for l in check_layers:
+                ll = l % w.layers
+                lk, lv = w.kv_rows(b, ll, st["pos"][ll], u)
+                for g in range(w.kv_heads):
+                    gk = c.gather(c.k, b, ll, g, lens[b]).float().cpu().numpy()
+                    gv = c.gather(c.v, b, ll, g, lens[b]).float().cpu().numpy()
+                    rep.kv_err = max(rep.kv_err, float(np.max(np.abs(gk - lk[g]))), float(np.max(np.abs(gv - lv[g]))))
         reports.append(rep)
     assert ikv.ikv_device_status() == 0
     return reports

@@ -135,9 +135,7 @@ def test_per_layer_eviction_arguments(lib):
                                        16, 16, 16, 1 << 40, None)
     p.max_holes = 4
     assert call(shp, cch) == lib.IKV_ERR_UNSUPPORTED
-    p.max_holes, p.compact_mode = 0, lib.IKV_COMPACT_HOLEFILL
-    assert call(shp, cch) == lib.IKV_ERR_UNSUPPORTED
-    p.compact_mode, p.scorer = lib.IKV_COMPACT_STABLE, lib.IKV_SCORE_ENTROPY
+    p.max_holes, p.scorer = 0, lib.IKV_SCORE_ENTROPY
     assert call(shp, cch) == lib.IKV_ERR_UNSUPPORTED
     p.scorer = lib.IKV_SCORE_ATTENTION
     assert call(_shape(lib, granularity=lib.IKV_GRAN_KVHEAD), cch) == lib.IKV_ERR_UNSUPPORTED

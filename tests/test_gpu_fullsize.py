@@ -10,7 +10,7 @@ and evicts ~90% of it.  Per step: attention outputs of every layer and head
 import pytest
 
 import gen
-from harness import run_fullsize_sampled
+from harness import run_fullsize_sampled, run_fullsize_sampled_layerwise
 from paper_2609_03515_gb300 import ikv
 
 pytestmark = pytest.mark.gpu
@@ -82,3 +82,14 @@ def test_config2_per_layer_split():
 @pytest.mark.timeout(1200)
 def test_config1_per_layer_split():
     _check(run_fullsize_sampled(gen.config(1), seqs=[0], steps=3, compact_mode=SHORT, max_holes=3, per_layer=True))
+
+
+@pytest.mark.timeout(1200)
+def test_config1_per_layer_immediate_eviction():
+    # every layer evicts right after its own update (step 1 drops ~90% of each layer's prefill)
+    _check(run_fullsize_sampled_layerwise(gen.config(1), seqs=[0], steps=3))
+
+
+@pytest.mark.timeout(1200)
+def test_config2_per_layer_immediate_eviction_split_lazy4():
+    _check(run_fullsize_sampled_layerwise(gen.config(2), seqs=[5], steps=5, per_layer=True))

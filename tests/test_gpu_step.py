@@ -220,6 +220,10 @@ def test_per_layer_immediate_eviction_trajectories():
     _assert(run_lockstep_layerwise(small_llama(steps=6, score_free=True, page_size=16), per_layer=True), 2e-2)
     _assert(run_lockstep_layerwise(small_llama(steps=6, layers=4), layer_eligible=[0, 1, 1, 0],
                                    refresh_init=ikv.IKV_INIT_MEAN), 2e-2)
+    _assert(run_lockstep_layerwise(small_llama(steps=8), compact_mode=ikv.IKV_COMPACT_HOLEFILL), 2e-2)
+    _assert(run_lockstep_layerwise(small_llama(steps=6, refresh_period=2), compact_mode=ikv.IKV_COMPACT_STABLE_SHORT,
+                                   per_layer=True), 2e-2)
+    _assert(run_lockstep_layerwise(gen.config(0), compact_mode=ikv.IKV_COMPACT_HOLEFILL), 1e-4)
     w = gen.Workload(name="qwen-small", batch=2, layers=2, q_heads=28, kv_heads=4, head_dim=128, prefill=[700, 260],
                      steps=5, dtype=gen.BF16, alpha=0.9, seed=9, page_size=32)
     _assert(run_lockstep_layerwise(w, per_layer=True), 2e-2)
