@@ -51,6 +51,14 @@ Readings taken where the paper is silent (each also stated where it is used):
   attention there, so its score is 0 (Eq. 1) and Eq. 4 decays it.  The new
   token's mean initialisation on non-refresh steps averages over the live
   positions.  With one layer this is the base method exactly.
+* R11 (rank-trace diagnostics, Appendix "Mechanistic Diagnostics"): on every
+  refresh step the raw top-k set R_t is the k = B tokens with the highest
+  single-step score (Eq. 2: the last eligible layer's Eq. 1 score, i.e. the
+  utility alpha = 0 would give), ties to the lower slot (R4), taken over the
+  step's cache before eviction; the EMA top-k set E_t is the kept set.  Churn of
+  a set is 1 - |X_t & X_{t'}| / |X_t| against the previous traced step t';
+  raw/EMA Jaccard |R_t & E_t| / |R_t | E_t|; raw-top evicted 1 - |R_t & E_t| / |R_t|.
+  Sets are compared by token position.
 * R9 (scorer variants, Appendix "Per-step scoring"): VNorm divides each value
   row's l2 norm by the mean norm over the cached tokens of its (layer, KV head);
   entropy weighting uses the normalized entropy H(s) / ln n of the layer's
@@ -247,6 +255,7 @@ class SeqState:
     budget: int
     next_pos: int
     granularity: int = GRAN_SEQ
+    raw: Optional[np.ndarray] = None   # [R, L] last eligible layer's score of the step (R11)
 
     @property
     def length(self) -> int:
@@ -317,6 +326,7 @@ def attend_and_score(st: SeqState, q_t: np.ndarray, refresh: bool, p: Params) ->
             if p.scorer == "entropy":
                 s = s * np.array([[entropy_weight(row)] for row in s])
             st.m = aggregate(st.m, s, p)
+            st.raw = s
     return np.stack(outs)
 
 
@@ -346,6 +356,7 @@ def decode_step(st: SeqState, t: int, q_t: np.ndarray, k_new: np.ndarray, v_new:
     q_t: [layers][H][d]; k_new, v_new: [layers][H_kv][d].
     """
     refresh = is_refresh(t, p.refresh_period, p.score_free)
+    st.raw = None
     append_token(st, k_new, v_new, refresh, p)
     out = attend_and_score(st, q_t, refresh, p)
     evict(st)
@@ -446,3 +457,39 @@ def decode_step_layerwise(st: LayerwiseState, t: int, q_t: np.ndarray, k_new: np
             st.K[l][g] = st.K[l][g][keep]
             st.V[l][g] = st.V[l][g][keep]
     return np.stack(outs), traces
+
+
+# --------------------------------------------------------------------------
+# Rank-trace diagnostics (reading R11)
+# --------------------------------------------------------------------------
+def topk_positions(score_row: np.ndarray, pos_row: np.ndarray, k: int) -> np.ndarray:
+    """Positions of the k highest scores of one row (ties: lower slot), ascending."""
+    return np.sort(np.asarray(pos_row)[select_keep(score_row, k)])
+
+
+def churn(cur: np.ndarray, prev: np.ndarray) -> float:
+    """Fraction of a top-k set replaced since the previous traced step."""
+    cur = set(np.asarray(cur).tolist())
+    return 1.0 - len(cur & set(np.asarray(prev).tolist())) / len(cur) if cur else 0.0
+
+
+def jaccard(a: np.ndarray, b: np.ndarray) -> float:
+    a, b = set(np.asarray(a).tolist()), set(np.asarray(b).tolist())
+    return len(a & b) / len(a | b) if a | b else 1.0
+
+
+def raw_top_evicted(raw: np.ndarray, kept: np.ndarray) -> float:
+    """Fraction of the raw top-k tokens not in the kept set."""
+    raw = set(np.asarray(raw).tolist())
+    return 1.0 - len(raw & set(np.asarray(kept).tolist())) / len(raw) if raw else 0.0
+
+
+def decode_step_traced(st: SeqState, t: int, q_t, k_new, v_new, p: Params):
+    """decode_step plus the step's rank-trace sets per row (R11): (out, [(R_t or None, E_t)])."""
+    refresh = is_refresh(t, p.refresh_period, p.score_free)
+    st.raw = None
+    append_token(st, k_new, v_new, refresh, p)
+    out = attend_and_score(st, q_t, refresh, p)
+    R = [None if st.raw is None else topk_positions(st.raw[r], st.pos[r], st.budget) for r in range(st.m.shape[0])]
+    evict(st)
+    return out, [(R[r], np.sort(st.pos[r])) for r in range(st.m.shape[0])]

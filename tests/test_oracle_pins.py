@@ -664,3 +664,64 @@ def test_layerwise_invariants():
         assert set(lw.live().tolist()) == set().union(*[set(x.tolist()) for x in lw.pos])
         diverged |= len({tuple(x) for x in lw.pos}) > 1
     assert diverged  # the layers' sets do part ways on this input
+
+
+# ------------------------------------------------------- rank-trace diagnostics (R11)
+def test_rank_trace_set_measures_closed_forms():
+    assert O.churn(np.array([1, 2, 3, 4]), np.array([1, 2, 3, 4])) == 0.0
+    assert O.churn(np.array([1, 2, 3, 4]), np.array([5, 6, 7, 8])) == 1.0
+    assert O.churn(np.array([1, 2, 3, 4]), np.array([0, 2, 3, 9])) == 0.5
+    assert O.jaccard(np.array([1, 2, 3]), np.array([2, 3, 4])) == 0.5
+    assert O.raw_top_evicted(np.array([1, 2, 3, 4]), np.array([2, 4, 6, 8])) == 0.5
+    # ties go to the lower slot (R4), the result is in position order
+    assert list(O.topk_positions(np.array([0.5, 0.2, 0.5, 0.9]), np.array([40, 10, 30, 20]), 2)) == [20, 40]
+
+
+def test_rank_trace_alpha_zero_raw_equals_ema():
+    """alpha = 0: the state after a refresh step is the last eligible layer's score (Eq. 4),
+    i.e. the raw score itself, so the kept set is the raw top-k: Jaccard 1, nothing of the
+    raw top-k evicted, equal churns."""
+    rng = np.random.default_rng(21)
+    st = _rand_state(rng, layers=3, kv=2, L0=30, budget=9)
+    p = O.Params(alpha=0.0)
+    q, kn, vn = _rand_inputs(rng, 6, layers=3)
+    prev = None
+    for t in range(1, 7):
+        _, sets = O.decode_step_traced(st, t, q[t - 1], kn[t - 1], vn[t - 1], p)
+        R, E = sets[0]
+        assert O.jaccard(R, E) == 1.0 and O.raw_top_evicted(R, E) == 0.0
+        if prev is not None:
+            assert O.churn(R, prev[0]) == O.churn(E, prev[1])
+        prev = (R, E)
+
+
+def test_rank_trace_alpha_one_freezes_the_kept_set():
+    """alpha = 1: utilities never move and new tokens start at 0 on refresh steps, so every
+    step evicts the new token and the EMA top-k never changes (churn 0), while the raw
+    top-k follows the queries."""
+    rng = np.random.default_rng(22)
+    st = _rand_state(rng, layers=2, kv=2, L0=24, budget=8)
+    p = O.Params(alpha=1.0)
+    q, kn, vn = _rand_inputs(rng, 6, layers=2)
+    prev = None
+    raw_churns = []
+    for t in range(1, 7):
+        _, sets = O.decode_step_traced(st, t, q[t - 1], kn[t - 1], vn[t - 1], p)
+        R, E = sets[0]
+        if prev is not None:
+            assert O.churn(E, prev[1]) == 0.0
+            raw_churns.append(O.churn(R, prev[0]))
+        prev = (R, E)
+    assert max(raw_churns) > 0.0
+
+
+def test_rank_trace_raw_is_last_eligible_layer_score():
+    """The traced raw score is the last eligible layer's Eq. 1 score, which single-step
+    aggregation (Eq. 2) also leaves as the utility."""
+    rng = np.random.default_rng(23)
+    a = _rand_state(rng, layers=3, kv=2, L0=20, budget=30)   # no eviction: compare full rows
+    b = _clone(a)
+    q, kn, vn = _rand_inputs(rng, 1, layers=3)
+    O.decode_step(a, 1, q[0], kn[0], vn[0], O.Params(alpha=0.8, layer_mask=[True, True, False]))
+    O.decode_step(b, 1, q[0], kn[0], vn[0], O.Params(aggregation="single", layer_mask=[True, True, False]))
+    np.testing.assert_array_equal(a.raw, b.m)
