@@ -135,6 +135,25 @@ typedef struct {
     cudaEvent_t begin, append_end, attend_end, combine_end, score_end, select_end, end;
 } ikv_timing;
 
+/* Rank-trace diagnostics (Appendix "Mechanistic Diagnostics"), an optional output of a
+ * step, per utility row r:
+ *  - raw top-k R_t: on refresh steps, the budget[b] tokens with the highest single-step
+ *    score (the last eligible layer's score, the utility Eq. 2 would leave; ties to the
+ *    lower slot), taken over the step's cache before eviction;
+ *  - EMA top-k E_t: the tokens live after the step (the kept set).
+ * Sets are token positions, ascending.  On entry raw_top / ema_top hold the previous
+ * traced step's sets and n_top[r] = {|R_prev|, |E_prev|} (0, 0 before the first); on exit
+ * this step's (raw_top and n_top[r][0] unchanged on steps without a raw score).
+ * counts[r] = {|R_t & R_prev|, |E_t & E_prev|, |R_t & E_t|, |R_t|, |E_t|}, the R entries -1
+ * on steps without a raw score.  Churn, Jaccard and the raw-top evicted fraction follow
+ * from them.  A set larger than 16384 tokens is not traced: bit 4 of the device error
+ * word, counts -2. */
+typedef struct {
+    int32_t *raw_top, *ema_top;  /* [rows][cap] device */
+    int32_t *n_top;              /* [rows][2] device */
+    int32_t *counts;             /* [rows][5] device, written */
+} ikv_trace;
+
 typedef struct {
     float alpha;                    /* EMA coefficient of Eq. 4, in [0, 1] */
     int32_t refresh_period;         /* r of Eq. 6 (>= 1; 1 = full refresh) */
@@ -174,6 +193,8 @@ typedef struct {
                                        for the split step).  Needs IKV_GRAN_SEQ, max_holes 0, IKV_AGG_EMA,
                                        IKV_SCORE_ATTENTION, cache->pos_cap > 0 and the layout described
                                        under "Utility rows". */
+    const ikv_trace *trace;         /* nullable: rank-trace diagnostics of the step (IKV_EVICT_STEP,
+                                       scorer other than IKV_SCORE_ENTROPY) */
 } ikv_params;
 
 /* Message for the last error on this thread ("" if none). */
@@ -188,7 +209,7 @@ int64_t ikv_launch_count(void);
  * bit 1: a split longer than the kernel's TMEM budget reached the device;
  * bit 2: an append found no free slot (start + len = cap) and was dropped;
  * bit 3: per-layer eviction, a sequence's next_pos reached cache->pos_cap (the token
- * was dropped). */
+ * was dropped); bit 4: a rank-trace set exceeded 16384 tokens (not traced). */
 ikv_status ikv_device_status(uint32_t *flags);
 
 /* Which decode-attention kernel ikv_decode_attend_score and ikv_step launch for

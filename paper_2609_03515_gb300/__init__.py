@@ -14,7 +14,7 @@ import torch
 
 from . import ikv
 
-__all__ = ["ikv", "DecodeCache", "step_lengths", "auto_max_holes"]
+__all__ = ["ikv", "DecodeCache", "RankTrace", "step_lengths", "auto_max_holes"]
 
 
 def auto_max_holes(budgets: Sequence[int]) -> int:
@@ -160,7 +160,7 @@ class DecodeCache:
                compact_mode: int = ikv.IKV_COMPACT_STABLE, refresh_init: int = ikv.IKV_INIT_ZERO,
                layer_eligible: Optional[Sequence[int]] = None, max_holes: int = 0,
                agg_mode: int = ikv.IKV_AGG_EMA, scorer: int = ikv.IKV_SCORE_ATTENTION,
-               evict_mode: int = ikv.IKV_EVICT_STEP) -> ikv.ikv_params:
+               evict_mode: int = ikv.IKV_EVICT_STEP, trace: "Optional[RankTrace]" = None) -> ikv.ikv_params:
         p = ikv.ikv_params()
         p.alpha = alpha
         p.refresh_period = refresh_period
@@ -175,6 +175,9 @@ class DecodeCache:
         p.agg_mode = agg_mode
         p.scorer = scorer
         p.evict_mode = evict_mode
+        if trace is not None:
+            p.trace = _ct.pointer(trace.struct)
+            self._trace = trace
         return p
 
 
@@ -185,3 +188,34 @@ ctypes_u8 = _ct.c_uint8
 
 def ctypes_addr(x) -> int:
     return _ct.addressof(x)
+
+
+class RankTrace:
+    """Device buffers of the rank-trace diagnostics (ikv_trace) for one DecodeCache: each
+    utility row's previous raw / EMA top-k positions, their sizes and the last step's
+    overlap counts {|R & R_prev|, |E & E_prev|, |R & E|, |R|, |E|}."""
+
+    def __init__(self, c: DecodeCache):
+        dev = c.k.device
+        self.raw_top = torch.zeros((c.rows, c.cap), dtype=torch.int32, device=dev)
+        self.ema_top = torch.zeros((c.rows, c.cap), dtype=torch.int32, device=dev)
+        self.n_top = torch.zeros((c.rows, 2), dtype=torch.int32, device=dev)
+        self.counts = torch.zeros((c.rows, 5), dtype=torch.int32, device=dev)
+        self.struct = ikv.ikv_trace(self.raw_top.data_ptr(), self.ema_top.data_ptr(), self.n_top.data_ptr(),
+                                    self.counts.data_ptr())
+
+    def reset(self) -> None:
+        self.n_top.zero_()
+
+    def stats(self):
+        """Per row: raw churn, EMA churn, raw/EMA Jaccard, raw-top evicted (None where the
+        step had no raw score or nothing to compare with)."""
+        out = []
+        for rr, re_, rx, nr, ne in self.counts.cpu().tolist():
+            row = {"ema_churn": 1.0 - re_ / ne if ne > 0 else None}
+            if nr > 0:
+                row["raw_churn"] = 1.0 - rr / nr
+                row["jaccard"] = rx / (nr + ne - rx)
+                row["raw_top_evicted"] = 1.0 - rx / nr
+            out.append(row)
+        return out

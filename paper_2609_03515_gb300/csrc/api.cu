@@ -131,7 +131,8 @@ AttendWs attend_ws(const ikv_shape *s, int32_t cap, int n_layers, bool logits) {
 
 struct StepWs {
     AttendWs at;
-    size_t keep, keep_len, done, cdone, moves, n_moves, sbuf, epart, vmean, slot, inv, util, live, end;
+    size_t keep, keep_len, done, cdone, moves, n_moves, sbuf, epart, vmean, slot, inv, util, live, raw, keep_raw,
+        n_raw, raw_pos, end;
 };
 
 StepWs step_ws(const ikv_shape *s, int32_t cap, int32_t pos_cap) {
@@ -170,6 +171,15 @@ StepWs step_ws(const ikv_shape *s, int32_t cap, int32_t pos_cap) {
     if (pos_cap > 0) off = align256(off + (size_t)s->batch * s->layers * cap * sizeof(float));
     w.live = off;
     if (pos_cap > 0) off = align256(off + (size_t)s->batch * ((pos_cap + 31) / 32) * sizeof(uint32_t));
+    // rank trace: the single-step score, its top-k slots and their positions
+    w.raw = off;
+    off = align256(off + R * cap * sizeof(float));
+    w.keep_raw = off;
+    off = align256(off + R * cap * sizeof(int32_t));
+    w.n_raw = off;
+    off = align256(off + R * sizeof(int32_t));
+    w.raw_pos = off;
+    off = align256(off + R * cap * sizeof(int32_t));
     w.end = off;
     return w;
 }
@@ -597,6 +607,13 @@ static ikv_status prepare_step(const ikv_shape *shape, const ikv_params *p, cons
         return fail(IKV_ERR_ARG, "unknown scorer %d", p->scorer);
     if (p->scorer == IKV_SCORE_VNORM && !cache->vnorm) return fail(IKV_ERR_ARG, "IKV_SCORE_VNORM needs cache->vnorm");
     cx->layerwise = p->evict_mode == IKV_EVICT_LAYER;
+    if (p->trace) {
+        const ikv_trace *tr = p->trace;
+        if (!tr->raw_top || !tr->ema_top || !tr->n_top || !tr->counts)
+            return fail(IKV_ERR_ARG, "trace raw_top/ema_top/n_top/counts is NULL");
+        if (cx->layerwise || p->scorer == IKV_SCORE_ENTROPY)
+            return fail(IKV_ERR_UNSUPPORTED, "the rank trace needs IKV_EVICT_STEP and a scorer other than IKV_SCORE_ENTROPY");
+    }
     if (p->evict_mode != IKV_EVICT_STEP && !cx->layerwise) return fail(IKV_ERR_ARG, "unknown evict_mode %d", p->evict_mode);
     if (cx->layerwise) {
         if (shape->granularity != IKV_GRAN_SEQ || p->max_holes != 0 || p->agg_mode != IKV_AGG_EMA ||
@@ -640,6 +657,47 @@ static ikv_status evict_impl(const ikv_shape *shape, const ikv_params *p, ikv_ca
     return compact_impl(shape, cache, at<int32_t>(ws, w.keep), at<int32_t>(ws, w.keep_len), ema, p->compact_mode,
                         at<int32_t>(ws, w.moves), at<int32_t>(ws, w.n_moves), at<int32_t>(ws, w.cdone), stream,
                         p->max_holes);
+}
+
+// Rank trace: the arguments of its kernels.
+static TraceArgs trace_args(const ikv_shape *shape, const ikv_params *p, const ikv_cache *cache, void *ws,
+                            const StepCtx &cx) {
+    TraceArgs t{};
+    t.rows = shape->batch * rows_per_seq(shape);
+    t.rows_per_seq = rows_per_seq(shape);
+    t.cap = cx.cap;
+    t.len = cache->len;
+    t.pos = cache->pos;
+    t.keep_raw = at<int32_t>(ws, cx.w.keep_raw);
+    t.n_raw = at<int32_t>(ws, cx.w.n_raw);
+    t.raw_pos = at<int32_t>(ws, cx.w.raw_pos);
+    t.has_raw = cx.scoring ? 1 : 0;
+    t.raw_top = p->trace->raw_top;
+    t.ema_top = p->trace->ema_top;
+    t.n_top = p->trace->n_top;
+    t.counts = p->trace->counts;
+    return t;
+}
+
+// Rank trace, before the eviction: the raw top-k slots of the single-step score and
+// their positions (refresh steps).
+static ikv_status trace_before(const ikv_shape *shape, const ikv_params *p, const ikv_cache *cache, void *ws,
+                               const StepCtx &cx, cudaStream_t stream) {
+    if (!p->trace || !cx.scoring) return IKV_OK;
+    const int32_t R = shape->batch * rows_per_seq(shape);
+    IKV_TRY_CUDA(launch_select(R, cx.cap, at<float>(ws, cx.w.raw), cache->len, rows_per_seq(shape), p->budget,
+                               cache->dead_slots ? cache->pos : nullptr, at<int32_t>(ws, cx.w.keep_raw),
+                               at<int32_t>(ws, cx.w.n_raw), DeferArgs{0, cx.cap, nullptr}, stream),
+                 "trace select launch");
+    IKV_TRY_CUDA(launch_trace_gather(trace_args(shape, p, cache, ws, cx), cx.L1, stream), "trace gather launch");
+    return IKV_OK;
+}
+
+static ikv_status trace_after(const ikv_shape *shape, const ikv_params *p, const ikv_cache *cache, void *ws,
+                              const StepCtx &cx, cudaStream_t stream) {
+    if (!p->trace) return IKV_OK;
+    IKV_TRY_CUDA(launch_trace(trace_args(shape, p, cache, ws, cx), stream), "trace launch");
+    return IKV_OK;
 }
 
 // Per-layer eviction: the arguments every layer-wise kernel of a step shares.
@@ -762,13 +820,15 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
                         tm, true)))
         return e;
     if (tm && (e = record(tm->combine_end, stream))) return e;
+    float *raw = p->trace ? at<float>(ws, w.raw) : nullptr;
     if (cx.scoring && (e = run_score(shape, cache, shape->layers, cx.elig, cx.n_elig, cx.L1, ws, w.at, p->alpha, ema,
-                                     nullptr, stream, p->agg_mode, p->scorer, cx.sw)))
+                                     raw, stream, p->agg_mode, p->scorer, cx.sw)))
         return e;
     if (tm && (e = record(tm->score_end, stream))) return e;
+    if ((e = trace_before(shape, p, cache, ws, cx, stream))) return e;
     if ((e = evict_impl(shape, p, cache, ema, ws, w, stream, tm))) return e;
     if (tm && (e = record(tm->end, stream))) return e;
-    return IKV_OK;
+    return trace_after(shape, p, cache, ws, cx, stream);
 }
 
 ikv_status ikv_step_begin(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, int32_t t,
@@ -837,10 +897,13 @@ ikv_status ikv_step_end(const ikv_shape *shape, const ikv_params *p, ikv_cache *
     if (e) return e;
     PdlScope pdl;
     if (cx.layerwise) return layer_evict(shape, p, &cx.cv, ema, ws, cx, stream);
+    float *raw = p->trace ? at<float>(ws, cx.w.raw) : nullptr;
     if (cx.scoring && (e = run_score(shape, &cx.cv, shape->layers, cx.elig, cx.n_elig, cx.L1, ws, cx.w.at, p->alpha,
-                                     ema, nullptr, stream, p->agg_mode, p->scorer, cx.sw)))
+                                     ema, raw, stream, p->agg_mode, p->scorer, cx.sw)))
         return e;
-    return evict_impl(shape, p, &cx.cv, ema, ws, cx.w, stream, nullptr);
+    if ((e = trace_before(shape, p, &cx.cv, ws, cx, stream))) return e;
+    if ((e = evict_impl(shape, p, &cx.cv, ema, ws, cx.w, stream, nullptr))) return e;
+    return trace_after(shape, p, &cx.cv, ws, cx, stream);
 }
 
 }  // extern "C"

@@ -729,10 +729,11 @@ extern "C" ikv_status ikv_device_status(uint32_t *flags) {
     unsigned int v = 0, z = 0;
     cudaError_t e = cudaMemcpyFromSymbol(&v, ikv::g_tc_error, sizeof(v));
     if (e == cudaSuccess) e = cudaMemcpyToSymbol(ikv::g_tc_error, &z, sizeof(z));
-    unsigned int ap = 0, lw = 0;
+    unsigned int ap = 0, lw = 0, tr = 0;
     if (e == cudaSuccess) e = ikv::read_clear_append_error(&ap);
     if (e == cudaSuccess) e = ikv::read_clear_layer_error(&lw);
+    if (e == cudaSuccess) e = ikv::read_clear_trace_error(&tr);
     if (e != cudaSuccess) return ikv::report(IKV_ERR_CUDA, "ikv_device_status: %s", cudaGetErrorString(e));
-    *flags = v | (ap ? 4u : 0u) | lw;
+    *flags = v | (ap ? 4u : 0u) | lw | tr;
     return IKV_OK;
 }

@@ -240,6 +240,20 @@ cudaError_t launch_layer_begin(const LayerArgs &a, int32_t max_len, cudaStream_t
 // inverse maps of every layer, then the per-position fold (utilities and final state)
 cudaError_t launch_layer_fold(const LayerArgs &a, int32_t max_len, int32_t max_pos, cudaStream_t st);
 cudaError_t read_clear_layer_error(unsigned int *v);
+
+// Rank-trace diagnostics (trace.cu)
+struct TraceArgs {
+    int32_t rows, rows_per_seq, cap;
+    const int32_t *len, *pos;       // [batch], [rows][cap] (after the step's eviction)
+    const int32_t *keep_raw, *n_raw; // raw top-k slots (ascending) and counts, before eviction
+    int32_t *raw_pos;               // [rows][cap] workspace: positions of the raw top-k
+    int32_t has_raw;                // refresh step: R_t exists
+    int32_t *raw_top, *ema_top, *n_top, *counts;
+};
+// raw_pos[r][j] = pos[r][keep_raw[r][j]] (before the eviction moves pos)
+cudaError_t launch_trace_gather(const TraceArgs &a, int32_t max_len, cudaStream_t st);
+cudaError_t launch_trace(const TraceArgs &a, cudaStream_t st);
+cudaError_t read_clear_trace_error(unsigned int *v);
 // reads and clears the append kernel's device error word (bit 0: no free slot)
 cudaError_t read_clear_append_error(unsigned int *v);
 

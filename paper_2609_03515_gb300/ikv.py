@@ -46,11 +46,15 @@ class ikv_timing(ctypes.Structure):
                 ("select_end", P), ("end", P)]
 
 
+class ikv_trace(ctypes.Structure):
+    _fields_ = [("raw_top", P), ("ema_top", P), ("n_top", P), ("counts", P)]
+
+
 class ikv_params(ctypes.Structure):
     _fields_ = [("alpha", F32), ("refresh_period", I32), ("score_free", I32), ("budget", P),
                 ("layer_eligible", P), ("compact_mode", I32), ("refresh_init", I32),
                 ("timing", ctypes.POINTER(ikv_timing)), ("max_holes", I32), ("agg_mode", I32),
-                ("scorer", I32), ("evict_mode", I32)]
+                ("scorer", I32), ("evict_mode", I32), ("trace", ctypes.POINTER(ikv_trace))]
 
 
 class IKVError(RuntimeError):

@@ -137,7 +137,7 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
                  steps: Optional[int] = None, kv_check_layers=(0, -1), page_perm_seed: Optional[int] = 7,
                  refresh_init: int = ikv.IKV_INIT_ZERO, layer_eligible=None, max_holes: int = 0,
                  agg_mode: int = ikv.IKV_AGG_EMA, scorer: int = ikv.IKV_SCORE_ATTENTION,
-                 per_layer: bool = False) -> List[StepReport]:
+                 per_layer: bool = False, trace: bool = False) -> List[StepReport]:
     T = w.steps if steps is None else steps
     u = w.u_table()
     c = make_cache(w, gran, page_perm_seed, value_norms=scorer == ikv.IKV_SCORE_VNORM)
@@ -153,10 +153,14 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
                                ikv.IKV_AGG_SINGLE_STEP: "single"}[agg_mode],
                   scorer={ikv.IKV_SCORE_ATTENTION: "attention", ikv.IKV_SCORE_VNORM: "vnorm",
                           ikv.IKV_SCORE_ENTROPY: "entropy"}[scorer])
+    from paper_2609_03515_gb300 import RankTrace
+
+    tr = RankTrace(c) if trace else None
     p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, refresh_init, layer_eligible, max_holes,
-                 agg_mode, scorer)
+                 agg_mode, scorer, trace=tr)
     ws = c.step_workspace()
     qs = w.queries(1, T + 1, u)
+    prev_sets = [(np.zeros(0, np.int64), np.zeros(0, np.int64))] * (w.batch * c.rows_per_seq)
     budgets = w.budgets()
     lens, live = list(w.prefill), list(w.prefill)
     out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
@@ -174,9 +178,15 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
         pos_h = c.pos.cpu().numpy()
         len_h = c.len.cpu().numpy()
         refresh = O.is_refresh(t, w.refresh_period, w.score_free)
+        if tr is not None:
+            cnt_h = tr.counts.cpu().numpy()
+            ntop_h = tr.n_top.cpu().numpy()
+            rawtop_h = tr.raw_top.cpu().numpy()
+            ematop_h = tr.ema_top.cpu().numpy()
         rep = StepReport(t=t, refresh=refresh)
         q64 = as_f64(qs[t - 1], w)
         for b, st in enumerate(sts):
+            st.raw = None
             O.append_token(st, kn[:, b], vn[:, b], refresh, op)
             o_out = O.attend_and_score(st, q64[:, b], refresh, op)
             rep.out_err = max(rep.out_err, float(np.max(np.abs(out_h[:, b] - o_out))))
@@ -200,6 +210,25 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
                 rep.set_ok &= ok
                 own = set(O.select_keep(st.m[rr], budgets[b]).tolist())
                 rep.strict_set_equal &= own == set(oslots.tolist())
+                if tr is not None:  # rank trace of this row (reading R11)
+                    Et = np.sort(gpos.astype(np.int64))
+                    nR, nE = int(ntop_h[r, 0]), int(ntop_h[r, 1])
+                    assert nE == len(Et) and np.array_equal(ematop_h[r, :nE], Et), (t, b, rr)
+                    Rp, Ep = prev_sets[r]
+                    c5 = cnt_h[r]
+                    assert c5[1] == len(set(Et.tolist()) & set(Ep.tolist())) and c5[4] == len(Et), (t, b, rr, c5)
+                    if refresh:
+                        Rt = rawtop_h[r, :nR].astype(np.int64)
+                        assert np.all(np.diff(Rt) > 0) and nR == min(st.length, budgets[b])
+                        rmask = np.isin(st.pos[rr], Rt)  # the oracle's raw score decides validity
+                        ok_r, _ = boundary_ok(st.raw[rr], rmask, budgets[b])
+                        rep.set_ok &= ok_r
+                        assert c5[3] == nR and c5[0] == len(set(Rt.tolist()) & set(Rp.tolist())), (t, b, rr, c5)
+                        assert c5[2] == len(set(Rt.tolist()) & set(Et.tolist())), (t, b, rr, c5)
+                        prev_sets[r] = (Rt, Et)
+                    else:
+                        assert c5[0] == -1 and c5[2] == -1 and c5[3] == -1
+                        prev_sets[r] = (Rp, Et)
                 rep.m_err = max(rep.m_err, float(np.max(np.abs(gm - st.m[rr][oslots]))))
                 keeps.append(np.sort(oslots))
             O.evict(st, keep_override=keeps)

@@ -149,6 +149,23 @@ def test_per_layer_eviction_arguments(lib):
     assert n1.value >= n0.value + 200 * 4
 
 
+def test_rank_trace_arguments(lib):
+    shp, cch = _shape(lib), _cache(lib)
+    p = lib.ikv_params()
+    p.alpha, p.refresh_period, p.budget = 0.9, 1, 16
+    tr = lib.ikv_trace(16, 16, 16, None)
+    p.trace = ctypes.pointer(tr)
+    call = lambda: lib.raw_status("ikv_step", ctypes.byref(shp), ctypes.byref(p), ctypes.byref(cch), 16, 1, 16, 16,
+                                  16, 16, 16, 1 << 40, None)
+    assert call() == lib.IKV_ERR_ARG                 # counts is NULL
+    tr.counts = 16
+    p.scorer = lib.IKV_SCORE_ENTROPY
+    assert call() == lib.IKV_ERR_UNSUPPORTED
+    p.scorer, p.evict_mode = lib.IKV_SCORE_ATTENTION, lib.IKV_EVICT_LAYER
+    cch.pos_cap = 100
+    assert call() == lib.IKV_ERR_UNSUPPORTED
+
+
 def test_deferred_compaction_arguments(lib):
     shp, cch = _shape(lib), _cache(lib)
     p = lib.ikv_params()

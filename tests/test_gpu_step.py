@@ -227,3 +227,17 @@ def test_per_layer_immediate_eviction_trajectories():
     w = gen.Workload(name="qwen-small", batch=2, layers=2, q_heads=28, kv_heads=4, head_dim=128, prefill=[700, 260],
                      steps=5, dtype=gen.BF16, alpha=0.9, seed=9, page_size=32)
     _assert(run_lockstep_layerwise(w, per_layer=True), 2e-2)
+
+
+def test_rank_trace_diagnostics():
+    """The step's rank trace (reading R11): the EMA top-k equals the kept positions, the raw
+    top-k is a valid top-B of the oracle's single-step score under the boundary rule, and
+    the overlap counts equal the set intersections of this and the previous traced step;
+    across schedules, granularities, compaction modes, deferral and the split step."""
+    _assert(run_lockstep(gen.config(0), trace=True), 1e-4, strict_fraction=1.0)
+    _assert(run_lockstep(small_llama(steps=8), trace=True), 2e-2)
+    _assert(run_lockstep(small_llama(steps=9, refresh_period=3), trace=True, max_holes=3,
+                         compact_mode=ikv.IKV_COMPACT_STABLE_SHORT), 2e-2)
+    _assert(run_lockstep(small_llama(steps=6), gran=ikv.IKV_GRAN_KVHEAD, compact_mode=ikv.IKV_COMPACT_HOLEFILL,
+                         trace=True), 2e-2)
+    _assert(run_lockstep(small_llama(steps=6), scorer=ikv.IKV_SCORE_VNORM, trace=True, per_layer=True), 2e-2)
