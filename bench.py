@@ -57,6 +57,7 @@ def parse():
     ap.add_argument("--mode-kernels", action="store_true",
                     help="also run every mode eagerly and report its per-kernel times")
     ap.add_argument("--cpu-steps", type=int, default=0, help="oracle steps in the CPU sample (0 = auto)")
+    ap.add_argument("--no-trace", action="store_true", help="skip the rank-trace diagnostics")
     return ap.parse_args()
 
 
@@ -431,6 +432,35 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     return res
 
 
+def run_trace(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, mh: int = 0):
+    """Rank-trace diagnostics (raw / EMA top-k churn, raw/EMA Jaccard, raw-top evicted)
+    over the timed steps of one schedule, launched eagerly with ikv_params.trace set;
+    means over the steps that have them and over the utility rows.  Not timed."""
+    import torch
+
+    from paper_2609_03515_gb300 import RankTrace, ikv, step_lengths
+
+    reset(c, w, u_dev)
+    tr = RankTrace(c)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh, trace=tr)
+    budgets = w.budgets()
+    lens, live = list(w.prefill), list(w.prefill)
+    out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=c.torch_dtype, device=c.k.device)
+    acc = {"raw_churn": [], "ema_churn": [], "jaccard": [], "raw_top_evicted": []}
+    W, K = args.warmup, min(args.steps, 50)
+    for t in range(1, W + K + 1):
+        ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws,
+                     ws.numel(), torch.cuda.current_stream())
+        lens, live = step_lengths(lens, live, budgets, mh)
+        if t > W:  # churn compares with the previous traced step, so the first timed step has one
+            for row in tr.stats():
+                for k, v in row.items():
+                    if v is not None and k in acc:
+                        acc[k].append(v)
+    torch.cuda.synchronize()
+    return {k: (sum(v) / len(v) if v else None) for k, v in acc.items()}
+
+
 def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist, mh: int = 0, scorer: int = 0):
     """Same steps through the C ABI, inputs from pinned host memory and the output read back every step.
 
@@ -655,6 +685,11 @@ def run_ours(args):
                     continue  # per-kernel events time the step-end eviction path only
                 mode_kernels[name] = run_mode(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, True, dist,
                                               vmh, sc)["kernel_ms"]
+    trace = None
+    if not args.no_trace:
+        # the Appendix's rank-trace table on this workload: full refresh at three alphas
+        trace = {f"alpha_{a}": run_trace(args, w.with_(alpha=a, refresh_period=1, score_free=False), c, u_dev, qs_dev,
+                                         kn_dev, vn_dev, ws, compact_mode, mh) for a in (0.3, 0.8, 0.9)}
     K = args.steps
     value = job_throughput(w.batch * K, world, full["ms"])
     if rank != 0:
@@ -720,6 +755,10 @@ def run_ours(args):
         "clocks": full["clocks"],
         "modes": {k: w.batch * K * world / (v["ms"] / 1e3) for k, v in modes.items()},
     }
+    if trace is not None:
+        line["rank_trace"] = dict(trace, note="full refresh, the headline's inputs and compaction; means over the "
+                                              "timed steps and utility rows; raw = the last layer's single-step "
+                                              "score, k = the budget (Appendix \"Mechanistic Diagnostics\")")
     if modes:
         full_v = line["modes"]["full"]
         line["speedup_vs_full"] = {k: v / full_v for k, v in line["modes"].items() if k != "full"}
