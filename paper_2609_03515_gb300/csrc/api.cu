@@ -131,7 +131,7 @@ AttendWs attend_ws(const ikv_shape *s, int32_t cap, int n_layers, bool logits) {
 
 struct StepWs {
     AttendWs at;
-    size_t keep, keep_len, done, cdone, moves, n_moves, sbuf, epart, vmean, slot, inv, util, live, raw, keep_raw,
+    size_t keep, keep_len, done, cdone, sdone, moves, n_moves, sbuf, epart, vmean, slot, inv, util, live, raw, keep_raw,
         n_raw, raw_pos, end;
 };
 
@@ -147,9 +147,12 @@ StepWs step_ws(const ikv_shape *s, int32_t cap, int32_t pos_cap) {
     off = align256(off + Rs * cap * sizeof(int32_t));
     w.keep_len = off;
     off = align256(off + Rs * sizeof(int32_t));
-    w.done = off;  // append arrivals, then compaction arrivals: one control block
+    // one control block: append arrivals [batch], compaction arrivals [batch], fused-
+    // selection arrivals [rows]
+    w.done = off;
     w.cdone = off + (size_t)s->batch * sizeof(int32_t);
-    off = align256(off + 2 * (size_t)s->batch * sizeof(int32_t));
+    w.sdone = off + 2 * (size_t)s->batch * sizeof(int32_t);
+    off = align256(off + (2 * (size_t)s->batch + R) * sizeof(int32_t));
     w.moves = off;
     off = align256(off + Rs * cap * 2 * sizeof(int32_t));
     w.n_moves = off;
@@ -307,10 +310,20 @@ struct ScorerWs {
     float *sbuf = nullptr, *epart = nullptr, *vmean = nullptr;
 };
 
+// Selection run by the score pass's last CTA of each row (ikv_step, ikv_step_end).
+struct SelectFuse {
+    int32_t *row_done;
+    const int32_t *budget;
+    int32_t *pos;
+    int32_t *keep, *keep_len;
+    DeferArgs df;
+};
+
 ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, const int32_t *elig, int n_elig,
                      int32_t max_len, void *ws, const AttendWs &w, float alpha, float *ema, float *score,
                      cudaStream_t st, int32_t agg = IKV_AGG_EMA, int32_t scorer = IKV_SCORE_ATTENTION,
-                     const ScorerWs &sw = ScorerWs{}, int32_t layer0 = 0, bool store_only = false) {
+                     const ScorerWs &sw = ScorerWs{}, int32_t layer0 = 0, bool store_only = false,
+                     const SelectFuse *fuse = nullptr, bool *fused = nullptr) {
     ScoreArgs base{};
     base.len = c->len;
     base.batch = s->batch;
@@ -339,11 +352,23 @@ ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, c
     base.nblk = score_blocks(base, max_len, sm_count(), &V);
     base.blk_tok = 32 * V;
     if (scorer == IKV_SCORE_VNORM && !store_only) IKV_TRY_CUDA(launch_vnorm_mean(base, st), "vnorm mean launch");
+    if (fused) *fused = false;
     for (int k0 = 0; k0 < n_elig; k0 += kMaxLayersPerScorePass) {
         ScoreArgs sa = base;
         sa.n_elig = n_elig - k0 < kMaxLayersPerScorePass ? n_elig - k0 : kMaxLayersPerScorePass;
         sa.k0 = k0;
         for (int k = 0; k < sa.n_elig; ++k) sa.elig[k] = elig[k0 + k];
+        // the last pass of an Eq. 1 / VNorm fold also selects
+        if (fuse && ema && !store_only && scorer != IKV_SCORE_ENTROPY && k0 + sa.n_elig == n_elig) {
+            sa.fuse_select = 1;
+            sa.row_done = fuse->row_done;
+            sa.budget = fuse->budget;
+            sa.sel_pos = fuse->pos;
+            sa.keep = fuse->keep;
+            sa.keep_len = fuse->keep_len;
+            sa.df = fuse->df;
+            if (fused) *fused = true;
+        }
         IKV_TRY_CUDA(launch_score_ema(sa, max_len, sm_count(), st), "score launch");
     }
     if (scorer == IKV_SCORE_ENTROPY && !store_only)
@@ -645,18 +670,32 @@ static ikv_status prepare_step(const ikv_shape *shape, const ikv_params *p, cons
 
 // Step 5: selection, then deferred or immediate compaction.
 static ikv_status evict_impl(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, void *ws,
-                             const StepWs &w, cudaStream_t stream, const ikv_timing *tm) {
+                             const StepWs &w, cudaStream_t stream, const ikv_timing *tm, bool selected = false) {
     const int32_t cap = cap_of(cache);
     const int32_t R = shape->batch * rows_per_seq(shape);
-    IKV_TRY_CUDA(launch_select(R, cap, ema, cache->len, rows_per_seq(shape), p->budget,
-                               cache->dead_slots ? cache->pos : nullptr, at<int32_t>(ws, w.keep),
-                               at<int32_t>(ws, w.keep_len), DeferArgs{p->max_holes, cap, cache->start}, stream),
-                 "select launch");
+    if (!selected)
+        IKV_TRY_CUDA(launch_select(R, cap, ema, cache->len, rows_per_seq(shape), p->budget,
+                                   cache->dead_slots ? cache->pos : nullptr, at<int32_t>(ws, w.keep),
+                                   at<int32_t>(ws, w.keep_len), DeferArgs{p->max_holes, cap, cache->start}, stream),
+                     "select launch");
     ikv_status e;
     if (tm && (e = record(tm->select_end, stream))) return e;
     return compact_impl(shape, cache, at<int32_t>(ws, w.keep), at<int32_t>(ws, w.keep_len), ema, p->compact_mode,
                         at<int32_t>(ws, w.moves), at<int32_t>(ws, w.n_moves), at<int32_t>(ws, w.cdone), stream,
                         p->max_holes);
+}
+
+// The selection the score pass may run itself (not under the rank trace, whose raw
+// top-k must read the positions before the selection marks a victim dead).
+static SelectFuse select_fuse(const ikv_params *p, const ikv_cache *cache, void *ws, const StepCtx &cx) {
+    SelectFuse f;
+    f.row_done = at<int32_t>(ws, cx.w.sdone);
+    f.budget = p->budget;
+    f.pos = cache->dead_slots ? cache->pos : nullptr;
+    f.keep = at<int32_t>(ws, cx.w.keep);
+    f.keep_len = at<int32_t>(ws, cx.w.keep_len);
+    f.df = DeferArgs{p->max_holes, cx.cap, cache->start};
+    return f;
 }
 
 // Rank trace: the arguments of its kernels.
@@ -777,8 +816,7 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
         // its own rows), then the per-layer evictions
         IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.at.arrivals), 0, w.at.logits - w.at.arrivals, stream),
                      "cudaMemsetAsync");
-        IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.done), 0, 2 * sizeof(int32_t) * shape->batch, stream),
-                     "cudaMemsetAsync");
+        IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.done), 0, w.moves - w.done, stream), "cudaMemsetAsync");
         LayerArgs la = layer_args(shape, p, cache, ema, ws, cx);
         IKV_TRY_CUDA(cudaMemsetAsync(la.live, 0, sizeof(uint32_t) * (size_t)shape->batch * la.live_words, stream),
                      "cudaMemsetAsync");
@@ -803,11 +841,10 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
         return layer_evict(shape, p, cache, ema, ws, cx, stream);
     }
 
-    // control words (append and split-arrival counters) start at zero
+    // control words (append, split-arrival and selection counters) start at zero
     IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.at.arrivals), 0, w.at.logits - w.at.arrivals, stream),
                  "cudaMemsetAsync");
-    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.done), 0, 2 * sizeof(int32_t) * shape->batch, stream),
-                 "cudaMemsetAsync");
+    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.done), 0, w.moves - w.done, stream), "cudaMemsetAsync");
     if (tm && (e = record(tm->begin, stream))) return e;
     if ((e = append_impl(shape, cache, k_new, v_new, ema, cx.init_mean, at<int32_t>(ws, w.done), stream, true)))
         return e;
@@ -821,12 +858,15 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
         return e;
     if (tm && (e = record(tm->combine_end, stream))) return e;
     float *raw = p->trace ? at<float>(ws, w.raw) : nullptr;
+    const SelectFuse fs = select_fuse(p, cache, ws, cx);
+    bool selected = false;
     if (cx.scoring && (e = run_score(shape, cache, shape->layers, cx.elig, cx.n_elig, cx.L1, ws, w.at, p->alpha, ema,
-                                     raw, stream, p->agg_mode, p->scorer, cx.sw)))
+                                     raw, stream, p->agg_mode, p->scorer, cx.sw, 0, false,
+                                     p->trace ? nullptr : &fs, &selected)))
         return e;
     if (tm && (e = record(tm->score_end, stream))) return e;
     if ((e = trace_before(shape, p, cache, ws, cx, stream))) return e;
-    if ((e = evict_impl(shape, p, cache, ema, ws, w, stream, tm))) return e;
+    if ((e = evict_impl(shape, p, cache, ema, ws, w, stream, tm, selected))) return e;
     if (tm && (e = record(tm->end, stream))) return e;
     return trace_after(shape, p, cache, ws, cx, stream);
 }
@@ -840,8 +880,7 @@ ikv_status ikv_step_begin(const ikv_shape *shape, const ikv_params *p, ikv_cache
     // control words start at zero (the attention leaves its arrival counters zero)
     IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, cx.w.at.arrivals), 0, cx.w.at.logits - cx.w.at.arrivals, stream),
                  "cudaMemsetAsync");
-    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, cx.w.done), 0, 2 * sizeof(int32_t) * shape->batch, stream),
-                 "cudaMemsetAsync");
+    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, cx.w.done), 0, cx.w.moves - cx.w.done, stream), "cudaMemsetAsync");
     if (cx.layerwise) {
         LayerArgs la = layer_args(shape, p, &cx.cv, ema, ws, cx);
         IKV_TRY_CUDA(cudaMemsetAsync(la.live, 0, sizeof(uint32_t) * (size_t)shape->batch * la.live_words, stream),
@@ -898,11 +937,14 @@ ikv_status ikv_step_end(const ikv_shape *shape, const ikv_params *p, ikv_cache *
     PdlScope pdl;
     if (cx.layerwise) return layer_evict(shape, p, &cx.cv, ema, ws, cx, stream);
     float *raw = p->trace ? at<float>(ws, cx.w.raw) : nullptr;
+    const SelectFuse fs = select_fuse(p, &cx.cv, ws, cx);
+    bool selected = false;
     if (cx.scoring && (e = run_score(shape, &cx.cv, shape->layers, cx.elig, cx.n_elig, cx.L1, ws, cx.w.at, p->alpha,
-                                     ema, raw, stream, p->agg_mode, p->scorer, cx.sw)))
+                                     ema, raw, stream, p->agg_mode, p->scorer, cx.sw, 0, false,
+                                     p->trace ? nullptr : &fs, &selected)))
         return e;
     if ((e = trace_before(shape, p, &cx.cv, ws, cx, stream))) return e;
-    if ((e = evict_impl(shape, p, &cx.cv, ema, ws, cx.w, stream, nullptr))) return e;
+    if ((e = evict_impl(shape, p, &cx.cv, ema, ws, cx.w, stream, nullptr, selected))) return e;
     return trace_after(shape, p, &cx.cv, ws, cx, stream);
 }
 

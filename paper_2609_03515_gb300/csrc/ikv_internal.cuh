@@ -105,6 +105,16 @@ struct CombineArgs {
     int32_t sc_layers, sc_layer0;
 };
 
+// Deferred compaction inside selection: when a row has exactly one slot too many and
+// the sequence may defer (len - budget <= max_holes and start + len < cap), select
+// marks the victim dead itself and writes keep_len = -1 - budget, which tells the
+// compaction kernels that nothing moves.  max_holes = 0 disables it.
+struct DeferArgs {
+    int32_t max_holes;
+    int32_t cap;
+    const int32_t *start;       // [batch] or null
+};
+
 struct ScoreArgs {
     const int32_t *len;         // [batch]
     int32_t batch, q_heads, kv_heads, rows_per_seq, n_layers, cap;
@@ -130,6 +140,14 @@ struct ScoreArgs {
     int32_t k0;                 // eligible-layer index of this pass's first layer
     int32_t n_elig_total;       // eligible layers over all passes
     int32_t store_only;         // Eq. 1 scorer: only store each layer's pooled score in sbuf
+    // selection fused into the (last) pass: the last CTA of each row to finish its
+    // utilities runs the budgeted selection of that row (select_row)
+    int32_t fuse_select;
+    int32_t *row_done;          // [rows] arrival counters, zero on entry, left zero
+    const int32_t *budget;      // [batch]
+    int32_t *sel_pos;           // pos when dead slots are in use, else null
+    int32_t *keep, *keep_len;   // [rows][cap], [rows]
+    DeferArgs df;
 };
 
 // tensor-core attention (bf16, head_dim 128): attend_tc.cu
@@ -156,15 +174,6 @@ cudaError_t launch_value_norms(const void *v, const PagedView &pv, const int32_t
                                int32_t cap, int dtype, float *vnorm, cudaStream_t st);
 cudaError_t launch_ema_update(int32_t rows, int32_t cap, float *ema, const float *score, const int32_t *len,
                               int32_t rows_per_seq, float alpha, int32_t max_len, cudaStream_t st);
-// Deferred compaction inside selection: when a row has exactly one slot too many and
-// the sequence may defer (len - budget <= max_holes and start + len < cap), select
-// marks the victim dead itself and writes keep_len = -1 - budget, which tells the
-// compaction kernels that nothing moves.  max_holes = 0 disables it.
-struct DeferArgs {
-    int32_t max_holes;
-    int32_t cap;
-    const int32_t *start;       // [batch] or null
-};
 cudaError_t launch_select(int32_t rows, int32_t cap, const float *util, const int32_t *len, int32_t rows_per_seq,
                           const int32_t *budget, int32_t *pos, int32_t *keep, int32_t *keep_len, const DeferArgs &df,
                           cudaStream_t st);

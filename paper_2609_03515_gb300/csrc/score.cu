@@ -11,11 +11,13 @@
 // token of a layer before its weight is known, so its first pass only stores s_l and
 // per-block partial entropies, and entropy_fold_kernel applies the weights and folds.
 #include "ikv_internal.cuh"
+#include "select_row.cuh"
 
 namespace ikv {
 namespace {
 
 constexpr int kScoreWarps = 32;   // one warp per eligible layer of a pass
+static_assert(kScoreWarps * 32 == kSelThreads, "the fused selection needs a full selection CTA");
 
 template <int V> struct VecF;
 template <> struct VecF<1> { using T = float; };
@@ -164,6 +166,23 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
         }
         if (a.ema) a.ema[at] = m;
         if (a.score) a.score[at] = sc;
+    }
+    if (a.fuse_select) {
+        // the row's CTAs that hold tokens arrive once their utilities are stored; the
+        // last one selects the row (arrival counter only: no CTA waits for another)
+        __shared__ int last;
+        __threadfence();
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            const int blocks = (L + kTok - 1) / kTok;
+            last = atomicAdd(&a.row_done[r], 1) == blocks - 1;
+            if (last) a.row_done[r] = 0;
+        }
+        __syncthreads();
+        if (last) {
+            __threadfence();
+            select_row(r, a.cap, a.ema, a.len, a.rows_per_seq, a.budget, a.sel_pos, a.keep, a.keep_len, a.df);
+        }
     }
 }
 
