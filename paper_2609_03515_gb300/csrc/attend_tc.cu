@@ -636,11 +636,14 @@ cudaError_t launch_tc_g(const CUtensorMap &mk, const CUtensorMap &mv, const TcAr
 int tc_max_split_tokens() { return kMaxTiles * kTile; }
 
 #ifndef IKV_TC_WAVES
-#define IKV_TC_WAVES 2
+#define IKV_TC_WAVES 1
 #endif
 // Chunking of the flattened (unit, tile) work for lengths up to max_len: enough
 // chunks for about IKV_TC_WAVES waves of two CTAs per SM, each chunk 1..15 tiles,
-// at most kMaxSplits chunks per unit.
+// at most kMaxSplits chunks per unit.  Measured at 32 layers x 8 KV heads x 27 tiles:
+// one wave's worth (chunks capped at 15 tiles, 512 CTAs) 77.3 us, two waves (12 tiles,
+// 768 CTAs) 81.2 us, three 83.2 us, four 87.1 us -- fewer, longer CTAs spend less on
+// prologues and merges.
 void tc_plan(int32_t max_len, int64_t units, int sms, int32_t *item_tiles, int32_t *n_chunks) {
     const int64_t tiles = ((int64_t)max_len + kTile - 1) / kTile;
     const int64_t target = (int64_t)2 * sms * IKV_TC_WAVES;
