@@ -490,6 +490,28 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (ok) ok = mbar_wait(o_full, 0, abort_flag);
         ok = __all_sync(0xffffffffu, ok);
         fence_after_sync();
+        if (ns_active == 1) {
+            // the unit's only chunk: its output and log-sum-exp need no merge
+            if (ok) {
+                float o[NC];
+                tmem_ld<NC>(tO + lane_off, o);
+#pragma unroll
+                for (int h = 0; h < G; ++h)
+                    a.out[(((int64_t)li * a.batch + b) * H + (int64_t)g * G + h) * kD + tid] =
+                        __float2bfloat16_rn(sum[h] > 0.f ? o[h] / sum[h] : 0.f);
+                if (tid < G) {
+                    float mm = -INFINITY, ss = 0.f;
+#pragma unroll
+                    for (int h = 0; h < G; ++h)
+                        if (h == tid) {
+                            mm = mx[h];
+                            ss = sum[h];
+                        }
+                    a.lse2[((int64_t)b * a.sc_layers + a.sc_layer0 + li) * H + (int64_t)g * G + tid] =
+                        ss > 0.f ? mm + log2f(ss) : -INFINITY;
+                }
+            }
+        } else {
         if (ok) {
             float o[NC];
             tmem_ld<NC>(tO + lane_off, o);
@@ -585,6 +607,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                         any ? M + log2f(W) : -INFINITY;
             }
             if (tid == 0) a.arrivals[unit] = 0;
+        }
         }
     }
     fence_before_sync();
