@@ -661,6 +661,12 @@ int tc_max_split_tokens() { return kMaxTiles * kTile; }
 #ifndef IKV_TC_WAVES
 #define IKV_TC_WAVES 1
 #endif
+// shortest chunk of a single-wave launch (one layer of a small batch); at 8 units x 27
+// tiles the split step measured 368 / 356 / 372 / 440 us per 32-layer step for 1 / 2 / 3 /
+// 5 tiles
+#ifndef IKV_TC_MIN_TILES
+#define IKV_TC_MIN_TILES 2
+#endif
 // Chunking of the flattened (unit, tile) work for lengths up to max_len: enough
 // chunks for about IKV_TC_WAVES waves of two CTAs per SM, each chunk 1..15 tiles,
 // at most kMaxSplits chunks per unit.  Measured at 32 layers x 8 KV heads x 27 tiles:
@@ -675,7 +681,10 @@ void tc_plan(int32_t max_len, int64_t units, int sms, int32_t *item_tiles, int32
     // of resident CTAs takes the shortest chunks that still fit it: every CTA runs from
     // the start and no short tail wave follows.
     const int64_t per_unit = (int64_t)2 * sms / (units > 0 ? units : 1);
-    if (per_unit >= 1 && (tiles + per_unit - 1) / per_unit <= kMaxTiles) c = (tiles + per_unit - 1) / per_unit;
+    if (per_unit >= 1 && (tiles + per_unit - 1) / per_unit <= kMaxTiles) {
+        c = (tiles + per_unit - 1) / per_unit;
+        if (c < IKV_TC_MIN_TILES) c = IKV_TC_MIN_TILES;
+    }
     const int64_t cmin = (tiles + kMaxSplits - 1) / kMaxSplits;
     if (c < cmin) c = cmin;
     if (c < 1) c = 1;
