@@ -400,8 +400,9 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
         lens, live = step_lengths(lens, live, budgets, mh)
     torch.cuda.synchronize()
     # the graphs' max_len bounds every later step: the budget plus the dead slots
-    # deferred compaction may hold
+    # deferred compaction may hold; the warm-up left the workspace's counters zero
     steady = c.cache(min(c.cap - 1, max(max(lens), max(budgets) + mh)))
+    p.ws_zeroed = 1
     graphs = []
     n0 = ikv.ikv_launch_count()
     for i in range(K):
@@ -537,6 +538,7 @@ def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist, mh: int
     run(1, W)
     torch.cuda.synchronize()
     steady = c.cache(min(c.cap - 1, max(max(lens), max(budgets) + mh)))
+    p.ws_zeroed = 1  # the warm-up left the workspace's counters zero
     for t in range(W + 1, W + 1 + K):
         key = (refresh(t), t % 2)
         if key in graphs:
@@ -727,7 +729,8 @@ def run_ours(args):
                    "kv_heads": w.kv_heads, "head_dim": w.head_dim, "prefill": w.prefill[0] if w.batch == 1 else w.prefill,
                    "budget": w.budgets(), "alpha": w.alpha, "refresh": head_sched, "compaction": args.compact, "max_holes": mh,
                    "timed_steps": f"decode steps {args.warmup + 1}..{args.warmup + K} (steady state; step 1 in warm-up)",
-                   "launch": "one CUDA graph per timed step, captured on that step's resident inputs",
+                   "launch": "one CUDA graph per timed step, captured on that step's resident inputs; "
+                             "workspace counters kept zero across steps (ikv_params.ws_zeroed)",
                    "l2": l2_note,
                    "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,

@@ -16,7 +16,8 @@
  *    the duration of the call.  The library allocates and frees nothing;
  *    scratch memory comes from the caller's workspace (ws, ws_bytes), sized
  *    by the matching *_workspace_size function.  The workspace needs no
- *    initialisation and carries nothing between calls.
+ *    initialisation and carries nothing between calls (ikv_params.ws_zeroed lets
+ *    a caller that keeps one workspace for its steps skip the per-step zeroing).
  *  - Work is enqueued asynchronously on the caller's stream; arguments are
  *    checked on the host before anything is launched.  Errors raised by a
  *    kernel after launch surface as IKV_ERR_CUDA on a later call.
@@ -195,6 +196,11 @@ typedef struct {
                                        under "Utility rows". */
     const ikv_trace *trace;         /* nullable: rank-trace diagnostics of the step (IKV_EVICT_STEP,
                                        scorer other than IKV_SCORE_ENTROPY) */
+    int32_t ws_zeroed;              /* nonzero: the caller asserts that the workspace's control words
+                                       are zero -- the workspace was zero-filled before its first step
+                                       and every step since ran to completion with ikv_device_status()
+                                       0 -- so ikv_step / ikv_step_begin skip re-zeroing them (two
+                                       memset launches).  Every step leaves them zero. */
 } ikv_params;
 
 /* Message for the last error on this thread ("" if none). */

@@ -153,14 +153,16 @@ class DecodeCache:
         return self.pos_state if evict_mode == ikv.IKV_EVICT_LAYER else self.ema
 
     def step_workspace(self) -> torch.Tensor:
+        """Zero-filled, so steps may run with ikv_params.ws_zeroed from the first one."""
         n = ikv.ikv_step_workspace_size(self.shape(), self.cache(self.cap - 1))
-        return torch.empty(n, dtype=torch.uint8, device=self.k.device)
+        return torch.zeros(n, dtype=torch.uint8, device=self.k.device)
 
     def params(self, alpha: float, refresh_period: int = 1, score_free: bool = False,
                compact_mode: int = ikv.IKV_COMPACT_STABLE, refresh_init: int = ikv.IKV_INIT_ZERO,
                layer_eligible: Optional[Sequence[int]] = None, max_holes: int = 0,
                agg_mode: int = ikv.IKV_AGG_EMA, scorer: int = ikv.IKV_SCORE_ATTENTION,
-               evict_mode: int = ikv.IKV_EVICT_STEP, trace: "Optional[RankTrace]" = None) -> ikv.ikv_params:
+               evict_mode: int = ikv.IKV_EVICT_STEP, trace: "Optional[RankTrace]" = None,
+               ws_zeroed: bool = False) -> ikv.ikv_params:
         p = ikv.ikv_params()
         p.alpha = alpha
         p.refresh_period = refresh_period
@@ -175,6 +177,7 @@ class DecodeCache:
         p.agg_mode = agg_mode
         p.scorer = scorer
         p.evict_mode = evict_mode
+        p.ws_zeroed = 1 if ws_zeroed else 0
         if trace is not None:
             p.trace = _ct.pointer(trace.struct)
             self._trace = trace

@@ -668,6 +668,16 @@ static ikv_status prepare_step(const ikv_shape *shape, const ikv_params *p, cons
     return IKV_OK;
 }
 
+// The step's counters -- attention arrivals, append / compaction / fused-selection
+// arrivals -- zeroed, unless the caller vouches that they are (ikv_params.ws_zeroed).
+static ikv_status zero_control_words(const ikv_params *p, void *ws, const StepWs &w, cudaStream_t stream) {
+    if (p->ws_zeroed) return IKV_OK;
+    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.at.arrivals), 0, w.at.logits - w.at.arrivals, stream),
+                 "cudaMemsetAsync");
+    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.done), 0, w.moves - w.done, stream), "cudaMemsetAsync");
+    return IKV_OK;
+}
+
 // Step 5: selection, then deferred or immediate compaction.
 static ikv_status evict_impl(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, void *ws,
                              const StepWs &w, cudaStream_t stream, const ikv_timing *tm, bool selected = false) {
@@ -814,9 +824,7 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     if (cx.layerwise) {
         // begin, every layer's new rows, one attention launch for all layers (each reads
         // its own rows), then the per-layer evictions
-        IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.at.arrivals), 0, w.at.logits - w.at.arrivals, stream),
-                     "cudaMemsetAsync");
-        IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.done), 0, w.moves - w.done, stream), "cudaMemsetAsync");
+        if ((e = zero_control_words(p, ws, w, stream))) return e;
         LayerArgs la = layer_args(shape, p, cache, ema, ws, cx);
         IKV_TRY_CUDA(cudaMemsetAsync(la.live, 0, sizeof(uint32_t) * (size_t)shape->batch * la.live_words, stream),
                      "cudaMemsetAsync");
@@ -841,10 +849,9 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
         return layer_evict(shape, p, cache, ema, ws, cx, stream);
     }
 
-    // control words (append, split-arrival and selection counters) start at zero
-    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.at.arrivals), 0, w.at.logits - w.at.arrivals, stream),
-                 "cudaMemsetAsync");
-    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, w.done), 0, w.moves - w.done, stream), "cudaMemsetAsync");
+    // control words (append, split-arrival and selection counters) start at zero; every
+    // kernel that counts leaves its counters zero again
+    if ((e = zero_control_words(p, ws, w, stream))) return e;
     if (tm && (e = record(tm->begin, stream))) return e;
     if ((e = append_impl(shape, cache, k_new, v_new, ema, cx.init_mean, at<int32_t>(ws, w.done), stream, true)))
         return e;
@@ -877,10 +884,8 @@ ikv_status ikv_step_begin(const ikv_shape *shape, const ikv_params *p, ikv_cache
     StepCtx cx;
     ikv_status e = prepare_step(shape, p, cache, ema, t, ws, ws_bytes, &cx);
     if (e) return e;
-    // control words start at zero (the attention leaves its arrival counters zero)
-    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, cx.w.at.arrivals), 0, cx.w.at.logits - cx.w.at.arrivals, stream),
-                 "cudaMemsetAsync");
-    IKV_TRY_CUDA(cudaMemsetAsync(at<int32_t>(ws, cx.w.done), 0, cx.w.moves - cx.w.done, stream), "cudaMemsetAsync");
+    // control words start at zero (every kernel that counts leaves its counters zero)
+    if ((e = zero_control_words(p, ws, cx.w, stream))) return e;
     if (cx.layerwise) {
         LayerArgs la = layer_args(shape, p, &cx.cv, ema, ws, cx);
         IKV_TRY_CUDA(cudaMemsetAsync(la.live, 0, sizeof(uint32_t) * (size_t)shape->batch * la.live_words, stream),

@@ -54,7 +54,7 @@ class ikv_params(ctypes.Structure):
     _fields_ = [("alpha", F32), ("refresh_period", I32), ("score_free", I32), ("budget", P),
                 ("layer_eligible", P), ("compact_mode", I32), ("refresh_init", I32),
                 ("timing", ctypes.POINTER(ikv_timing)), ("max_holes", I32), ("agg_mode", I32),
-                ("scorer", I32), ("evict_mode", I32), ("trace", ctypes.POINTER(ikv_trace))]
+                ("scorer", I32), ("evict_mode", I32), ("trace", ctypes.POINTER(ikv_trace)), ("ws_zeroed", I32)]
 
 
 class IKVError(RuntimeError):

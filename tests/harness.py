@@ -137,7 +137,7 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
                  steps: Optional[int] = None, kv_check_layers=(0, -1), page_perm_seed: Optional[int] = 7,
                  refresh_init: int = ikv.IKV_INIT_ZERO, layer_eligible=None, max_holes: int = 0,
                  agg_mode: int = ikv.IKV_AGG_EMA, scorer: int = ikv.IKV_SCORE_ATTENTION,
-                 per_layer: bool = False, trace: bool = False) -> List[StepReport]:
+                 per_layer: bool = False, trace: bool = False, ws_zeroed: bool = False) -> List[StepReport]:
     T = w.steps if steps is None else steps
     u = w.u_table()
     c = make_cache(w, gran, page_perm_seed, value_norms=scorer == ikv.IKV_SCORE_VNORM)
@@ -157,7 +157,7 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
 
     tr = RankTrace(c) if trace else None
     p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, refresh_init, layer_eligible, max_holes,
-                 agg_mode, scorer, trace=tr)
+                 agg_mode, scorer, trace=tr, ws_zeroed=ws_zeroed)
     ws = c.step_workspace()
     qs = w.queries(1, T + 1, u)
     prev_sets = [(np.zeros(0, np.int64), np.zeros(0, np.int64))] * (w.batch * c.rows_per_seq)

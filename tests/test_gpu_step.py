@@ -241,3 +241,14 @@ def test_rank_trace_diagnostics():
     _assert(run_lockstep(small_llama(steps=6), gran=ikv.IKV_GRAN_KVHEAD, compact_mode=ikv.IKV_COMPACT_HOLEFILL,
                          trace=True), 2e-2)
     _assert(run_lockstep(small_llama(steps=6), scorer=ikv.IKV_SCORE_VNORM, trace=True, per_layer=True), 2e-2)
+
+
+def test_workspace_kept_zero_across_steps():
+    """ikv_params.ws_zeroed: with a zero-filled workspace every step leaves its counters zero,
+    so steps that skip re-zeroing them give the same trajectories (whole step with
+    multi-chunk attention units and the fused selection, deferral, the split step)."""
+    _assert(run_lockstep(gen.config(0), ws_zeroed=True), 1e-4, strict_fraction=1.0)
+    _assert(run_lockstep(small_llama(steps=8, prefill=[300, 2000, 1200]), ws_zeroed=True), 2e-2)
+    _assert(run_lockstep(small_llama(steps=9, refresh_period=3), max_holes=3, ws_zeroed=True,
+                         compact_mode=ikv.IKV_COMPACT_STABLE_SHORT), 2e-2)
+    _assert(run_lockstep(small_llama(steps=6), per_layer=True, ws_zeroed=True), 2e-2)
