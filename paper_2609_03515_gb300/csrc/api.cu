@@ -226,11 +226,20 @@ static bool use_tc(const ikv_shape *s, const ikv_cache *c, int32_t layers_touche
            (int64_t)max_len + 127 <= (int64_t)kMaxSplits * tc_max_split_tokens() && pool_rows < (1ull << 31);
 }
 
+// Whether an attention launch over n_layers layers at max_len writes normalised group sums
+// (run_attend with a gsum request): the tensor-core kernel with one chunk per unit.
+bool attend_gsum(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, int32_t max_len) {
+    if (!use_tc(s, c, s->layers, max_len)) return false;
+    int32_t it = 0, nc = 0;
+    tc_plan(max_len + 127, (int64_t)s->batch * n_layers * s->kv_heads, sm_count(), &it, &nc);
+    return nc == 1;
+}
+
 ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, int32_t n_layers, int32_t max_len,
                       const void *q, void *out, void *ws, const AttendWs &w, bool logits, int32_t *split_out,
                       int32_t *nsplit_out, cudaStream_t st, const ikv_timing *tm = nullptr,
                       bool counters_zeroed = false, int32_t sc_layers = 0, int32_t sc_layer0 = 0,
-                      const AppendArgs *append = nullptr) {
+                      const AppendArgs *append = nullptr, bool *gsum = nullptr) {
     AttendArgs a{};
     a.k = c->k;
     a.v = c->v;
@@ -249,10 +258,13 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
         tc_plan(max_len + 127, (int64_t)s->batch * n_layers * s->kv_heads, sm_count(), &it, &nc);
         a.split_tokens = it * 128;
         a.n_splits = nc;
+        // one chunk per unit: the kernel can hand the score pass normalised group sums
+        a.gsum = gsum && logits && nc == 1 && use_tc(s, c, s->layers, max_len) ? 1 : 0;
     } else
         choose_splits(s, n_layers, max_len, kTileTokens, 1 << 30, &a.split_tokens, &a.n_splits);
     a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)s->head_dim));
     a.logits = logits ? at<float>(ws, w.logits) : nullptr;
+    if (gsum) *gsum = false;
     a.cap = cap_of(c);
     a.lstride = logit_stride(a.cap);
     a.part_ml = at<float>(ws, w.part_ml);
@@ -301,6 +313,7 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
     }
     if (split_out) *split_out = a.split_tokens;
     if (nsplit_out) *nsplit_out = a.n_splits;
+    if (gsum) *gsum = a.gsum != 0;
     return IKV_OK;
 }
 
@@ -323,7 +336,7 @@ ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, c
                      int32_t max_len, void *ws, const AttendWs &w, float alpha, float *ema, float *score,
                      cudaStream_t st, int32_t agg = IKV_AGG_EMA, int32_t scorer = IKV_SCORE_ATTENTION,
                      const ScorerWs &sw = ScorerWs{}, int32_t layer0 = 0, bool store_only = false,
-                     const SelectFuse *fuse = nullptr, bool *fused = nullptr) {
+                     const SelectFuse *fuse = nullptr, bool *fused = nullptr, bool gsum = false) {
     ScoreArgs base{};
     base.len = c->len;
     base.batch = s->batch;
@@ -348,6 +361,7 @@ ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, c
     base.epart = sw.epart;
     base.n_elig_total = n_elig;
     base.store_only = store_only ? 1 : 0;
+    base.gsum = gsum ? 1 : 0;
     int V = 1;
     base.nblk = score_blocks(base, max_len, sm_count(), &V);
     base.blk_tok = 32 * V;
@@ -781,10 +795,11 @@ static LayerArgs layer_args(const ikv_shape *shape, const ikv_params *p, const i
 // (refresh steps), the per-position fold giving each layer's utilities and the new
 // state, then every (sequence, layer) row selected and every layer compacted at once.
 static ikv_status layer_evict(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, void *ws,
-                              const StepCtx &cx, cudaStream_t stream) {
+                              const StepCtx &cx, cudaStream_t stream, bool gsum = false) {
     ikv_status e;
     if (cx.scoring && (e = run_score(shape, cache, shape->layers, cx.elig, cx.n_elig, cx.L1, ws, cx.w.at, p->alpha,
-                                     nullptr, nullptr, stream, IKV_AGG_EMA, IKV_SCORE_ATTENTION, cx.sw, 0, true)))
+                                     nullptr, nullptr, stream, IKV_AGG_EMA, IKV_SCORE_ATTENTION, cx.sw, 0, true,
+                                     nullptr, nullptr, gsum)))
         return e;
     IKV_TRY_CUDA(launch_layer_fold(layer_args(shape, p, cache, ema, ws, cx), cx.L1, cache->pos_cap, stream),
                  "layer fold launch");
@@ -843,10 +858,11 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
         ap.vnorm = cache->vnorm;
         ap.slot = at<int32_t>(ws, w.slot);
         IKV_TRY_CUDA(launch_append_rows(ap, stream), "append rows launch");
+        bool gsum = false;
         if ((e = run_attend(shape, cache, 0, shape->layers, cx.L1, q, out, ws, w.at, cx.scoring, nullptr, nullptr,
-                            stream, nullptr, true)))
+                            stream, nullptr, true, 0, 0, nullptr, &gsum)))
             return e;
-        return layer_evict(shape, p, cache, ema, ws, cx, stream);
+        return layer_evict(shape, p, cache, ema, ws, cx, stream, gsum);
     }
 
     // control words (append, split-arrival and selection counters) start at zero; every
@@ -860,8 +876,9 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     // (not when per-kernel events are recorded: those time each kernel alone)
     std::optional<PdlScope> pdl;
     if (!tm) pdl.emplace();
+    bool gsum = false;  // the attention may hand over normalised group sums instead of logits
     if ((e = run_attend(shape, cache, 0, shape->layers, cx.L1, q, out, ws, w.at, cx.scoring, nullptr, nullptr, stream,
-                        tm, true)))
+                        tm, true, 0, 0, nullptr, &gsum)))
         return e;
     if (tm && (e = record(tm->combine_end, stream))) return e;
     float *raw = p->trace ? at<float>(ws, w.raw) : nullptr;
@@ -869,7 +886,7 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     bool selected = false;
     if (cx.scoring && (e = run_score(shape, cache, shape->layers, cx.elig, cx.n_elig, cx.L1, ws, w.at, p->alpha, ema,
                                      raw, stream, p->agg_mode, p->scorer, cx.sw, 0, false,
-                                     p->trace ? nullptr : &fs, &selected)))
+                                     p->trace ? nullptr : &fs, &selected, gsum)))
         return e;
     if (tm && (e = record(tm->score_end, stream))) return e;
     if ((e = trace_before(shape, p, cache, ws, cx, stream))) return e;
@@ -929,8 +946,9 @@ ikv_status ikv_step_layer(const ikv_shape *shape, const ikv_params *p, ikv_cache
     // the new token's rows and one layer's attention; on refresh steps its logits and
     // log-sum-exp land where the whole step's attention would put them, for
     // ikv_step_end's score pass
+    bool gsum = false;  // the same for every layer call of the step (attend_gsum)
     return run_attend(shape, cache, layer, 1, cx.L1, q, out, ws, cx.w.at, cx.scoring && eligible, nullptr, nullptr,
-                      stream, nullptr, true, shape->layers, layer, &a);
+                      stream, nullptr, true, shape->layers, layer, &a, &gsum);
 }
 
 ikv_status ikv_step_end(const ikv_shape *shape, const ikv_params *p, ikv_cache *cache, float *ema, int32_t t,
@@ -940,13 +958,15 @@ ikv_status ikv_step_end(const ikv_shape *shape, const ikv_params *p, ikv_cache *
     ikv_status e = prepare_step(shape, p, cache, ema, t, ws, ws_bytes, &cx);
     if (e) return e;
     PdlScope pdl;
-    if (cx.layerwise) return layer_evict(shape, p, &cx.cv, ema, ws, cx, stream);
+    // what the layer calls' attention handed over: group sums when each launch had one chunk per unit
+    const bool gsum = attend_gsum(shape, &cx.cv, 1, cx.L1);
+    if (cx.layerwise) return layer_evict(shape, p, &cx.cv, ema, ws, cx, stream, gsum);
     float *raw = p->trace ? at<float>(ws, cx.w.raw) : nullptr;
     const SelectFuse fs = select_fuse(p, &cx.cv, ws, cx);
     bool selected = false;
     if (cx.scoring && (e = run_score(shape, &cx.cv, shape->layers, cx.elig, cx.n_elig, cx.L1, ws, cx.w.at, p->alpha,
                                      ema, raw, stream, p->agg_mode, p->scorer, cx.sw, 0, false,
-                                     p->trace ? nullptr : &fs, &selected)))
+                                     p->trace ? nullptr : &fs, &selected, gsum)))
         return e;
     if ((e = trace_before(shape, p, &cx.cv, ws, cx, stream))) return e;
     if ((e = evict_impl(shape, p, &cx.cv, ema, ws, cx.w, stream, nullptr, selected))) return e;

@@ -79,6 +79,9 @@ struct TcArgs {
     const int32_t *slot;
     __nv_bfloat16 *k_pool, *v_pool;
     float *vnorm;
+    // every unit is a single chunk: instead of per-head logits, write per token the KV
+    // head's group sum of normalised probabilities, [batch][sc_layers][kv_heads][lstride]
+    int32_t gsum;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -465,7 +468,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             for (int h = 0; h < G; ++h) {
                 const float z = v[h] * a.scale_log2;
                 float p = 0.f;
-                if (valid && a.logits) a.logits[lbase + (int64_t)h * a.lstride + (tok - S0)] = live ? z : -INFINITY;
+                if (valid && a.logits && !a.gsum) a.logits[lbase + (int64_t)h * a.lstride + (tok - S0)] = live ? z : -INFINITY;
                 if (live) {  // mx[h] is finite here: it covers this row
                     p = exp2f(z - mx[h]);
                     sum[h] += p;
@@ -486,6 +489,33 @@ __global__ void __launch_bounds__(kThreads, 2)
         softmax_bar();
 #pragma unroll
         for (int h = 0; h < G; ++h) sum[h] = red[h] + red[kN + h] + red[2 * kN + h] + red[3 * kN + h];
+
+        // sweep 3 (single-chunk units): the chunk's max and sum are the unit's, so each row's
+        // normalised probabilities are final; their sum over the KV head's query group is
+        // stored per token.  The S tiles are still in TMEM (the PV products go to O).
+        if (a.gsum && a.logits && ok) {
+            if (ns_active == 1) {
+                float inv[G];
+#pragma unroll
+                for (int h = 0; h < G; ++h) inv[h] = sum[h] > 0.f ? 1.f / sum[h] : 0.f;
+                const int64_t gbase = (((int64_t)b * a.sc_layers + a.sc_layer0 + li) * a.kv_heads + g) * a.lstride;
+                for (int i = 0; i < n; ++i) {
+                    float v[NC];
+                    tmem_ld<NC>(tS + lane_off + kN * i, v);
+                    const int tok = t0 + i * kTile + tid;
+                    if (tok >= lo && tok < t1) {
+                        float acc = 0.f;
+                        if ((live_bits >> i) & 1u) {
+#pragma unroll
+                            for (int h = 0; h < G; ++h) acc += exp2f(v[h] * a.scale_log2 - mx[h]) * inv[h];
+                        }
+                        a.logits[gbase + (tok - S0)] = acc;
+                    }
+                }
+            } else if (tid == 0) {
+                atomicOr(&g_tc_error, 2u);  // the host only asks for group sums when every unit has one chunk
+            }
+        }
 
         if (ok) ok = mbar_wait(o_full, 0, abort_flag);
         ok = __all_sync(0xffffffffu, ok);
@@ -743,6 +773,7 @@ cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group,
     t.k_pool = reinterpret_cast<__nv_bfloat16 *>(const_cast<void *>(a.k));
     t.v_pool = reinterpret_cast<__nv_bfloat16 *>(const_cast<void *>(a.v));
     t.vnorm = a.vnorm;
+    t.gsum = a.gsum;
     dim3 grid(a.n_splits * a.pv.kv_heads * a.batch * a.n_layers);
     cudaError_t e;
     switch (group) {

@@ -94,6 +94,10 @@ struct AttendArgs {
     const void *k_new, *v_new;
     const int32_t *slot;
     float *vnorm;
+    // tensor-core kernel, every unit one chunk: logits holds, per token, each KV head's sum
+    // of its query group's normalised probabilities ([batch][sc_layers][kv_heads][lstride])
+    // instead of per-head logits
+    int32_t gsum;
 };
 
 struct CombineArgs {
@@ -140,6 +144,7 @@ struct ScoreArgs {
     int32_t k0;                 // eligible-layer index of this pass's first layer
     int32_t n_elig_total;       // eligible layers over all passes
     int32_t store_only;         // Eq. 1 scorer: only store each layer's pooled score in sbuf
+    int32_t gsum;               // logits holds KV-head group sums of probabilities (see AttendArgs)
     // selection fused into the (last) pass: the last CTA of each row to finish its
     // utilities runs the budgeted selection of that row (select_row)
     int32_t fuse_select;

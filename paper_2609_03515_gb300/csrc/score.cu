@@ -92,9 +92,14 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
         float acc[V];
 #pragma unroll
         for (int v = 0; v < V; ++v) acc[v] = 0.f;
-        for (int hb = 0; hb < nh; hb += kHB) {
-            const int nb = min(kHB, nh - hb);
-            const float lse_lane = lane < nb ? ll[hb + lane] : 0.f;
+        // rows: the heads' log2-domain logits (normalised here by their log-sum-exp), or with
+        // gsum one row per KV head of the utility row holding its query group's normalised
+        // probabilities already summed
+        const int nrows = a.gsum ? ng : nh;
+        if (a.gsum) zp = a.logits + (((int64_t)b * a.n_layers + li) * a.kv_heads + g0) * (int64_t)a.lstride + il;
+        for (int hb = 0; hb < nrows; hb += kHB) {
+            const int nb = min(kHB, nrows - hb);
+            const float lse_lane = !a.gsum && lane < nb ? ll[hb + lane] : 0.f;
             VT z[kHB];
 #pragma unroll
             for (int j = 0; j < kHB; ++j) {
@@ -109,12 +114,14 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
 #pragma unroll
                     for (int v = 0; v < V; ++v) w[v] = 1.f;
                     if (SCORER == IKV_SCORE_VNORM) {
-                        const float *wg = wv + ((h0 + hb + j) / G - g0) * kTok + lane * V;
+                        const int gr = a.gsum ? hb + j : (h0 + hb + j) / G - g0;  // the row's kv head
+                        const float *wg = wv + gr * kTok + lane * V;
 #pragma unroll
                         for (int v = 0; v < V; ++v) w[v] = wg[v];
                     }
 #pragma unroll
-                    for (int v = 0; v < V; ++v) acc[v] += exp2f(vget(z[j], v) - lj) * w[v];
+                    for (int v = 0; v < V; ++v)
+                        acc[v] += (a.gsum ? vget(z[j], v) : exp2f(vget(z[j], v) - lj)) * w[v];
                 }
             }
         }
