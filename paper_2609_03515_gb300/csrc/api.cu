@@ -132,7 +132,7 @@ AttendWs attend_ws(const ikv_shape *s, int32_t cap, int n_layers, bool logits) {
 struct StepWs {
     AttendWs at;
     size_t keep, keep_len, done, cdone, sdone, moves, n_moves, sbuf, epart, vmean, slot, inv, util, live, raw, keep_raw,
-        n_raw, raw_pos, end;
+        n_raw, raw_pos, sel_best, sel_cnt, end;
 };
 
 StepWs step_ws(const ikv_shape *s, int32_t cap, int32_t pos_cap) {
@@ -183,6 +183,11 @@ StepWs step_ws(const ikv_shape *s, int32_t cap, int32_t pos_cap) {
     off = align256(off + R * sizeof(int32_t));
     w.raw_pos = off;
     off = align256(off + R * cap * sizeof(int32_t));
+    // fused selection: per score block, the lowest (key, slot) and the live count
+    w.sel_best = off;
+    off = align256(off + R * blk_max * sizeof(unsigned long long));
+    w.sel_cnt = off;
+    off = align256(off + R * blk_max * sizeof(uint32_t));
     w.end = off;
     return w;
 }
@@ -325,6 +330,8 @@ struct ScorerWs {
 
 // Selection run by the score pass's last CTA of each row (ikv_step, ikv_step_end).
 struct SelectFuse {
+    unsigned long long *best;  // [rows][blk_max]
+    uint32_t *cnt;             // [rows][blk_max]
     int32_t *row_done;
     const int32_t *budget;
     int32_t *pos;
@@ -381,6 +388,8 @@ ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, c
             sa.keep = fuse->keep;
             sa.keep_len = fuse->keep_len;
             sa.df = fuse->df;
+            sa.sel_best = fuse->best;
+            sa.sel_cnt = fuse->cnt;
             if (fused) *fused = true;
         }
         IKV_TRY_CUDA(launch_score_ema(sa, max_len, sm_count(), st), "score launch");
@@ -713,6 +722,8 @@ static ikv_status evict_impl(const ikv_shape *shape, const ikv_params *p, ikv_ca
 // top-k must read the positions before the selection marks a victim dead).
 static SelectFuse select_fuse(const ikv_params *p, const ikv_cache *cache, void *ws, const StepCtx &cx) {
     SelectFuse f;
+    f.best = at<unsigned long long>(ws, cx.w.sel_best);
+    f.cnt = at<uint32_t>(ws, cx.w.sel_cnt);
     f.row_done = at<int32_t>(ws, cx.w.sdone);
     f.budget = p->budget;
     f.pos = cache->dead_slots ? cache->pos : nullptr;

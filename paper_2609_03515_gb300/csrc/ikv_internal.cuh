@@ -153,6 +153,8 @@ struct ScoreArgs {
     int32_t *sel_pos;           // pos when dead slots are in use, else null
     int32_t *keep, *keep_len;   // [rows][cap], [rows]
     DeferArgs df;
+    unsigned long long *sel_best;  // [rows][nblk] each block's lowest (key, ~slot) among live slots
+    uint32_t *sel_cnt;             // [rows][nblk] each block's live slots
 };
 
 // tensor-core attention (bf16, head_dim 128): attend_tc.cu

@@ -175,20 +175,90 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
         if (a.score) a.score[at] = sc;
     }
     if (a.fuse_select) {
+        // This block's share of the selection's first pass -- its live slots and their
+        // lowest (key, highest slot) -- so that the common case (one slot too many,
+        // eviction deferred) needs no rescan of the row.
+        __shared__ unsigned long long blk_best[kTok / 32];
+        __shared__ uint32_t blk_cnt[kTok / 32];
+        const int blocks = (L + kTok - 1) / kTok;
+        if (threadIdx.x < kTok) {
+            uint32_t c = 0u;
+            unsigned long long best = ~0ull;
+            if (folds && (!a.sel_pos || a.sel_pos[at] >= 0)) {
+                c = 1u;
+                best = ((unsigned long long)ord_key(m) << 32) | (uint32_t)(~(uint32_t)fi);
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                c += __shfl_xor_sync(0xffffffffu, c, o);
+                const unsigned long long y = __shfl_xor_sync(0xffffffffu, best, o);
+                best = y < best ? y : best;
+            }
+            if (lane == 0) {
+                blk_best[warp] = best;
+                blk_cnt[warp] = c;
+            }
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            unsigned long long best = ~0ull;
+            uint32_t c = 0u;
+            for (int w = 0; w < kTok / 32; ++w) {
+                best = blk_best[w] < best ? blk_best[w] : best;
+                c += blk_cnt[w];
+            }
+            a.sel_best[(int64_t)r * a.nblk + blockIdx.x] = best;
+            a.sel_cnt[(int64_t)r * a.nblk + blockIdx.x] = c;
+        }
         // the row's CTAs that hold tokens arrive once their utilities are stored; the
         // last one selects the row (arrival counter only: no CTA waits for another)
         __shared__ int last;
         __threadfence();
         __syncthreads();
         if (threadIdx.x == 0) {
-            const int blocks = (L + kTok - 1) / kTok;
             last = atomicAdd(&a.row_done[r], 1) == blocks - 1;
             if (last) a.row_done[r] = 0;
         }
         __syncthreads();
         if (last) {
             __threadfence();
-            select_row(r, a.cap, a.ema, a.len, a.rows_per_seq, a.budget, a.sel_pos, a.keep, a.keep_len, a.df);
+            // the blocks' partials give the live count and the victim candidate
+            __shared__ unsigned long long s_best;
+            __shared__ uint32_t s_cnt;
+            if (warp == 0) {
+                unsigned long long best = ~0ull;
+                uint32_t c = 0u;
+                for (int j = lane; j < blocks; j += 32) {
+                    const unsigned long long y = __ldcg(a.sel_best + (int64_t)r * a.nblk + j);
+                    best = y < best ? y : best;
+                    c += __ldcg(a.sel_cnt + (int64_t)r * a.nblk + j);
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    c += __shfl_xor_sync(0xffffffffu, c, o);
+                    const unsigned long long y = __shfl_xor_sync(0xffffffffu, best, o);
+                    best = y < best ? y : best;
+                }
+                if (lane == 0) {
+                    s_best = best;
+                    s_cnt = c;
+                }
+            }
+            __syncthreads();
+            const int B = max(a.budget[b], 0);
+            const int n_live = (int)s_cnt;
+            const int S = a.df.start ? a.df.start[b] : 0;
+            if (a.sel_pos && a.df.max_holes > 0 && B > 0 && n_live == B + 1 && L - B <= a.df.max_holes &&
+                S + L < a.df.cap) {
+                // one slot too many and the sequence may defer: mark the victim dead, as
+                // the selection itself would
+                if (threadIdx.x == 0) {
+                    a.sel_pos[(int64_t)r * a.cap + (int)(~(uint32_t)(s_best & 0xFFFFFFFFull))] = -1;
+                    a.keep_len[r] = -1 - B;
+                }
+            } else {
+                select_row(r, a.cap, a.ema, a.len, a.rows_per_seq, a.budget, a.sel_pos, a.keep, a.keep_len, a.df);
+            }
         }
     }
 }
