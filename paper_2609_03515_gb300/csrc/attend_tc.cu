@@ -1,12 +1,13 @@
 // Tensor-core split-K decode attention with logits, bf16, head_dim 128 (sm_103a).
 //
 // The cache of every (sequence, layer, kv head) unit is cut into chunks of up to
-// 15 tiles of 128 tokens; one CTA handles one chunk (the G query heads of its
-// kv head), writes that chunk's log2-domain logits and its (max, sum, O)
-// partial, and the unit's last chunk to finish merges the partials into the
-// output and the per-head log-sum-exp (arrival counter, no waiting).  The 1-D
-// grid is chunk-major, so every unit's short remainder chunk is dispatched last
-// and fills the final wave.  Two CTAs share an SM.  Built from Blackwell pieces:
+// 15 tiles of 128 tokens; one CTA handles one chunk, or several consecutive
+// chunks as passes (the G query heads of its kv head), writes their log2-domain
+// logits and its (max, sum, O) partial, and the unit's last CTA to finish merges
+// the partials into the output and the per-head log-sum-exp (arrival counter, no
+// waiting); a unit covered by one CTA writes them directly.  The 1-D grid is
+// chunk-major, so every unit's short remainder chunk is dispatched last and fills
+// the final wave.  Two CTAs share an SM.  Built from Blackwell pieces:
 //   * TMA (cp.async.bulk.tensor.2d, 128-byte swizzle) streams 128-token K and V
 //     tiles out of the paged pool (one box per page segment and 64-column half)
 //     into a 3-stage ring guarded by mbarriers;
@@ -16,7 +17,10 @@
 //     with K-major operands for QK and an MN-major (transposed) V for PV;
 //   * the softmax runs as two sweeps over the S tiles kept in TMEM: the chunk
 //     maximum per head, then logits write-out, exp2, row sums and the bf16 P
-//     operand (double-buffered in shared memory) that feeds the PV MMA.
+//     operand (double-buffered in shared memory) that feeds the PV MMA;
+//   * between passes the softmax frees the S tiles and O (s_free, o_free
+//     barriers) and folds the pass's (max, sum, O) into running registers, the
+//     online-softmax rescaling by exp2(m_old - m_new).
 // Warp roles (192 threads): warps 0-3 own TMEM lanes 0-127 (softmax, epilogue),
 // warp 4 issues TMA loads, warp 5 issues MMAs.  Every mbarrier wait is bounded;
 // on timeout the CTA records an error code, stops issuing work, waits for its
@@ -49,8 +53,8 @@ constexpr int kOffQ = kNst * kStage;
 constexpr int kOffP = kOffQ + kOpBytes;
 constexpr int kOffRed = kOffP + 2 * kOpBytes;
 constexpr int kOffBar = kOffRed + 4 * kN * 4;
-// barriers: full[kNst], empty[kNst], s_full, p_full[2], p_empty[2], o_full
-constexpr int kNumBar = 2 * kNst + 6;
+// barriers: full[kNst], empty[kNst], s_full, p_full[2], p_empty[2], o_full, s_free, o_free
+constexpr int kNumBar = 2 * kNst + 8;
 constexpr int kOffMisc = kOffBar + kNumBar * 8;
 constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // misc: tmem slot, abort flag, last-split flag   // + slack for 1024-byte alignment
 
@@ -82,6 +86,7 @@ struct TcArgs {
     // every unit is a single chunk: instead of per-head logits, write per token the KV
     // head's group sum of normalised probabilities, [batch][sc_layers][kv_heads][lstride]
     int32_t gsum;
+    int32_t passes;  // consecutive chunks per CTA (>= 1)
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -207,10 +212,12 @@ __global__ void __launch_bounds__(kThreads, 2)
     unsigned char *sm = smem_raw + (base - raw);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    // 1-D grid, chunk-major: CTA i handles chunk i / n_units of unit i % n_units, so every
-    // unit's short remainder chunk is dispatched last and fills the final wave
+    // 1-D grid, chunk-major: CTA i takes a.passes consecutive chunks of unit i % n_units,
+    // starting at chunk (i / n_units) * a.passes, so every unit's short remainder is
+    // dispatched last and fills the final wave.  The chunks of one CTA run as passes over
+    // the same TMEM columns; their (max, sum, output) are merged in registers.
     const int n_units = a.batch * a.n_layers * a.kv_heads;
-    const int s = blockIdx.x / n_units;
+    const int cta = blockIdx.x / n_units;  // CTA index within the unit
     const int unit_id = blockIdx.x % n_units;
     const int g = unit_id % a.kv_heads;
     const int b = (unit_id / a.kv_heads) % a.batch, li = (unit_id / a.kv_heads) / a.batch;
@@ -222,8 +229,10 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int ft = S0 / kTile;
     const int nt_unit = L > 0 ? (S0 + L + kTile - 1) / kTile - ft : 0;
     const int item = a.split_tokens / kTile;  // tiles per chunk
-    if (s * item >= nt_unit) {
-        if (s == 0) {  // empty sequence: zero output, log-sum-exp -inf
+    const int ns_active = (nt_unit + item - 1) / item;  // chunks of the unit
+    const int c0 = cta * a.passes;                      // this CTA's first chunk
+    if (c0 >= ns_active) {
+        if (cta == 0) {  // empty sequence: zero output, log-sum-exp -inf
             for (int i = threadIdx.x; i < G * kD; i += kThreads)
                 a.out[(((int64_t)li * a.batch + b) * a.q_heads + (int64_t)g * G) * kD + i] = __float2bfloat16_rn(0.f);
             if (threadIdx.x < G)
@@ -232,14 +241,15 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         return;
     }
-    const int n = min(item, nt_unit - s * item);           // tiles of this chunk
-    const int t0 = (ft + s * item) * kTile;                  // physical slot of its first row
-    const int lo = max(t0, S0), t1 = min(t0 + n * kTile, S0 + L);  // its valid rows [lo, t1)
-    const int ns_active = (nt_unit + item - 1) / item;
-    if (n > kMaxTiles) {  // the host sizes splits to fit TMEM; refuse rather than overrun
+    const int np = min(a.passes, ns_active - c0);             // passes of this CTA
+    const int nc_unit = (ns_active + a.passes - 1) / a.passes;  // CTAs that cover the unit
+    if (item > kMaxTiles) {  // the host sizes chunks to fit TMEM; refuse rather than overrun
         if (threadIdx.x == 0) atomicOr(&g_tc_error, 2u);
         return;
     }
+    // pass p: tiles and physical slot of the first row
+    auto chunk_n = [&](int p) { return min(item, nt_unit - (c0 + p) * item); };
+    auto chunk_t0 = [&](int p) { return (ft + (c0 + p) * item) * kTile; };
     const int H = a.q_heads;
 
     const uint32_t sQ = base + kOffQ, sP = base + kOffP;
@@ -251,39 +261,48 @@ __global__ void __launch_bounds__(kThreads, 2)
     auto p_full = [&](int i) { return bar0 + 8u * (2 * kNst + 1 + i); };
     auto p_empty = [&](int i) { return bar0 + 8u * (2 * kNst + 3 + i); };
     const uint32_t o_full = bar0 + 8u * (2 * kNst + 5);
+    const uint32_t s_free = bar0 + 8u * (2 * kNst + 6);  // the softmax is done with a pass's S tiles
+    const uint32_t o_free = bar0 + 8u * (2 * kNst + 7);  // the softmax has read a pass's O
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(sm + kOffMisc);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + kOffMisc + 4);
 
-    // pool row of box bx of load j (loads 0..n-1: K tiles, n..2n-1: V tiles)
+    // The load stream: per pass, its K tiles then its V tiles; load J of the stream goes
+    // to ring stage J % kNst.  pool row of box bx of load j of pass p:
     const int boxes = kTile / a.rows_per_box;
-    auto box_row = [&](int j, int bx) {
+    auto box_row = [&](int p, int j, int bx) {
+        const int n = chunk_n(p);
         const int tile = j < n ? j : j - n;
-        const int tok = t0 + tile * kTile + bx * a.rows_per_box;
+        const int tok = chunk_t0(p) + tile * kTile + bx * a.rows_per_box;
         int lp = tok / a.page_size;
         if (lp >= a.max_pages) lp = a.max_pages - 1;
         const int page = a.block_table[(int64_t)b * a.max_pages + lp];
         return ((l * a.num_pages + page) * a.kv_heads + g) * a.page_size + tok % a.page_size;
     };
-    auto issue = [&](int j) {
-        const int st = j % kNst;
+    int ld_J = 0, ld_p = 0, ld_j = 0;  // producer cursor: loads issued, pass and load of the next one
+    auto issue_next = [&]() {
+        const int st = ld_J % kNst;
         mbar_expect_tx(full(st), kStage);
-        const CUtensorMap *tm = j < n ? &tmK : &tmV;
+        const CUtensorMap *tm = ld_j < chunk_n(ld_p) ? &tmK : &tmV;
         const uint32_t dst = base + st * kStage;
         for (int bx = 0; bx < boxes; ++bx) {
-            const int row = box_row(j, bx);
+            const int row = box_row(ld_p, ld_j, bx);
             tma_load_2d(dst + bx * a.rows_per_box * 128, tm, 0, row, full(st));
             tma_load_2d(dst + kHalf + bx * a.rows_per_box * 128, tm, 64, row, full(st));
         }
+        ++ld_J;
+        if (++ld_j == 2 * chunk_n(ld_p)) {
+            ++ld_p;
+            ld_j = 0;
+        }
     };
-    const int n_first = min(2 * n, kNst);  // loads issued before the CTA-wide barrier
     if (warp == 4) {
-        // Split step: the CTA whose chunk holds the new token's slot stores the token's K
+        // Split step: the CTA whose chunks hold the new token's slot stores the token's K
         // and V rows into the cache (lanes 0-15: K, 16-31: V, 16 bytes each) before its
         // TMA loads read that tile; the proxy fence orders the stores before them.
         if (a.k_new) {
             const int j = a.slot[b];
             const int p = S0 + j;
-            if (j >= 0 && p >= t0 && p < t0 + n * kTile) {
+            if (j >= 0 && p >= chunk_t0(0) && p < chunk_t0(np - 1) + chunk_n(np - 1) * kTile) {
                 const int page = a.block_table[(int64_t)b * a.max_pages + p / a.page_size];
                 const int64_t row = ((int64_t)(l * a.num_pages + page) * a.kv_heads + g) * a.page_size + p % a.page_size;
                 const bool isv = lane >= 16;
@@ -320,9 +339,11 @@ __global__ void __launch_bounds__(kThreads, 2)
             mbar_init(p_empty(0), 1);
             mbar_init(p_empty(1), 1);
             mbar_init(o_full, 1);
+            mbar_init(s_free, 128);
+            mbar_init(o_free, 128);
             *abort_flag = 0;
             asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-            for (int j = 0; j < n_first; ++j) issue(j);
+            while (ld_J < kNst && ld_p < np) issue_next();
         }
         __syncwarp();
     }
@@ -353,15 +374,13 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (warp == 4) {
         // ---------------- TMA producer
         if (lane == 0) {
-            int issued = n_first;
-            for (int j = n_first; j < 2 * n; ++j) {
-                const int st = j % kNst;
-                if (!mbar_wait(empty(st), ((j / kNst) - 1) & 1, abort_flag)) break;
-                issue(j);
-                issued = j + 1;
+            while (ld_p < np) {
+                const int st = ld_J % kNst;  // ld_J >= kNst here: the first kNst loads went out above
+                if (!mbar_wait(empty(st), ((ld_J / kNst) - 1) & 1, abort_flag)) break;
+                issue_next();
             }
             // drain: the last phase issued on each stage must have landed before the CTA exits
-            for (int j = issued - 1; j >= 0 && j >= issued - kNst; --j) (void)mbar_wait(full(j % kNst), (j / kNst) & 1, abort_flag);
+            for (int j = ld_J - 1; j >= 0 && j >= ld_J - kNst; --j) (void)mbar_wait(full(j % kNst), (j / kNst) & 1, abort_flag);
         }
         __syncwarp();
     } else if (warp == 5) {
@@ -370,274 +389,321 @@ __global__ void __launch_bounds__(kThreads, 2)
             constexpr uint32_t id_qk = idesc_bf16(false, 128, kN);
             constexpr uint32_t id_pv = idesc_bf16(true, 128, kN);
             bool ok = true;
-            for (int i = 0; i < n && ok; ++i) {
-                const int st = i % kNst;
-                if (!(ok = mbar_wait(full(st), (i / kNst) & 1, abort_flag))) break;
+            int J = 0, Q = 0;  // loads and P tiles consumed so far
+            for (int p = 0; p < np && ok; ++p) {
+                const int n = chunk_n(p);
+                // the S tiles of the previous pass must have been read
+                if (p > 0 && !(ok = mbar_wait(s_free, (p - 1) & 1, abort_flag))) break;
                 fence_after_sync();
-                const uint32_t ka = base + st * kStage;
+                for (int i = 0; i < n; ++i) {
+                    const int st = (J + i) % kNst;
+                    if (!(ok = mbar_wait(full(st), ((J + i) / kNst) & 1, abort_flag))) break;
+                    fence_after_sync();
+                    const uint32_t ka = base + st * kStage;
 #pragma unroll
-                for (int kk = 0; kk < kD / 16; ++kk) {
-                    const uint64_t da = sdesc(ka + (kk >> 2) * kHalf + (kk & 3) * 32, 16, 1024);
-                    const uint64_t db = sdesc(sQ + (kk >> 2) * (kN * 128) + (kk & 3) * 32, 16, 1024);
-                    mma_bf16(tS + kN * i, da, db, id_qk, kk > 0 ? 1u : 0u);
+                    for (int kk = 0; kk < kD / 16; ++kk) {
+                        const uint64_t da = sdesc(ka + (kk >> 2) * kHalf + (kk & 3) * 32, 16, 1024);
+                        const uint64_t db = sdesc(sQ + (kk >> 2) * (kN * 128) + (kk & 3) * 32, 16, 1024);
+                        mma_bf16(tS + kN * i, da, db, id_qk, kk > 0 ? 1u : 0u);
+                    }
+                    mma_commit(empty(st));
                 }
-                mma_commit(empty(st));
-            }
-            mma_commit(s_full);
-            for (int i = 0; i < n && ok; ++i) {
-                const int j = n + i, st = j % kNst;
-                if (!(ok = mbar_wait(full(st), (j / kNst) & 1, abort_flag))) break;
-                if (!(ok = mbar_wait(p_full(i & 1), (i >> 1) & 1, abort_flag))) break;
-                fence_after_sync();
-                const uint32_t va = base + st * kStage;
-                const uint32_t pb = sP + (i & 1) * kOpBytes;
+                if (!ok) break;
+                J += n;
+                mma_commit(s_full);
+                // O of the previous pass must have been read before this pass overwrites it
+                if (p > 0 && !(ok = mbar_wait(o_free, (p - 1) & 1, abort_flag))) break;
+                for (int i = 0; i < n; ++i) {
+                    const int st = (J + i) % kNst, q = Q + i;
+                    if (!(ok = mbar_wait(full(st), ((J + i) / kNst) & 1, abort_flag))) break;
+                    if (!(ok = mbar_wait(p_full(q & 1), (q >> 1) & 1, abort_flag))) break;
+                    fence_after_sync();
+                    const uint32_t va = base + st * kStage;
+                    const uint32_t pb = sP + (q & 1) * kOpBytes;
 #pragma unroll
-                for (int kk = 0; kk < kTile / 16; ++kk) {
-                    // A = V^T (MN-major): 64-dim atoms 16 KB apart (LBO), 8-token groups 1 KB apart (SBO)
-                    const uint64_t da = sdesc(va + kk * 2048, kHalf, 1024);
-                    const uint64_t db = sdesc(pb + (kk >> 2) * (kN * 128) + (kk & 3) * 32, 16, 1024);
-                    mma_bf16(tO, da, db, id_pv, (i > 0 || kk > 0) ? 1u : 0u);
+                    for (int kk = 0; kk < kTile / 16; ++kk) {
+                        // A = V^T (MN-major): 64-dim atoms 16 KB apart (LBO), 8-token groups 1 KB apart (SBO)
+                        const uint64_t da = sdesc(va + kk * 2048, kHalf, 1024);
+                        const uint64_t db = sdesc(pb + (kk >> 2) * (kN * 128) + (kk & 3) * 32, 16, 1024);
+                        mma_bf16(tO, da, db, id_pv, (i > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    mma_commit(empty(st));
+                    mma_commit(p_empty(q & 1));
                 }
-                mma_commit(empty(st));
-                mma_commit(p_empty(i & 1));
+                if (!ok) break;
+                J += n;
+                Q += n;
+                mma_commit(o_full);
             }
-            mma_commit(o_full);
         }
         __syncwarp();
     } else {
         // ---------------- softmax / epilogue: thread tid owns TMEM lane tid
         const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
-        float mx[G], sum[G];
+        // running (max, sum) per head over the CTA's passes, and output dim tid of each head
+        float M[G], W[G], acc[G];
 #pragma unroll
         for (int h = 0; h < G; ++h) {
-            mx[h] = -INFINITY;
-            sum[h] = 0.f;
+            M[h] = -INFINITY;
+            W[h] = 0.f;
+            acc[h] = 0.f;
         }
-        // bit i: this thread's row of tile i is a valid, live slot.  The liveness of every
-        // tile is fetched before the wait for the QK products, so its latency is hidden.
-        uint32_t live_bits = 0u;
-        {
-            const int32_t *prow =
-                a.pos ? a.pos + ((int64_t)b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g)) * a.cap : nullptr;
+        const int32_t *prow =
+            a.pos ? a.pos + ((int64_t)b * a.rows_per_seq + (a.rows_per_seq == 1 ? 0 : g)) * a.cap : nullptr;
+        const int64_t lbase = (((int64_t)b * a.sc_layers + a.sc_layer0 + li) * H + (int64_t)g * G) * a.lstride;
+        bool ok = true;
+        int Q = 0;  // P tiles written so far
+        // Every bar.sync below runs once per pass in every softmax warp, whatever ok says.
+        for (int p = 0; p < np; ++p) {
+            const int n = chunk_n(p), t0 = chunk_t0(p);
+            const int lo = max(t0, S0), t1 = min(t0 + n * kTile, S0 + L);  // the chunk's valid rows
+            float mx[G], sum[G];
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                mx[h] = -INFINITY;
+                sum[h] = 0.f;
+            }
+            // bit i: this thread's row of tile i is a valid, live slot.  The liveness of every
+            // tile is fetched before the wait for the QK products, so its latency is hidden.
+            uint32_t live_bits = 0u;
             for (int i = 0; i < n; ++i) {
                 const int tok = t0 + i * kTile + tid;  // physical slot; logical slot tok - S0
                 if (tok >= lo && tok < t1 && (!prow || __ldg(prow + (tok - S0)) >= 0)) live_bits |= 1u << i;
             }
-        }
-        bool ok = __all_sync(0xffffffffu, mbar_wait(s_full, 0, abort_flag));
-        fence_after_sync();
-        // sweep 1: split maximum (-inf for a head when every row of the chunk is dead)
-        if (ok) {
-            for (int i = 0; i < n; ++i) {
-                float v[NC];
-                tmem_ld<NC>(tS + lane_off + kN * i, v);
-                if ((live_bits >> i) & 1u) {
-#pragma unroll
-                    for (int h = 0; h < G; ++h) mx[h] = fmaxf(mx[h], v[h] * a.scale_log2);
-                }
-            }
-        }
-        // split max per head over the 128 softmax threads
-#pragma unroll
-        for (int h = 0; h < G; ++h) {
-            float m = mx[h];
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-            if (lane == 0) red[warp * kN + h] = m;
-        }
-        __syncwarp();
-        softmax_bar();
-#pragma unroll
-        for (int h = 0; h < G; ++h) mx[h] = fmaxf(fmaxf(red[h], red[kN + h]), fmaxf(red[2 * kN + h], red[3 * kN + h]));
-        softmax_bar();
-
-        // sweep 2: logits write-out, exp2, row sums and the P operand of each tile.  The
-        // logits stores sit here, interleaved with the V stream; issued as a burst in
-        // sweep 1 they measured slower.
-        const int64_t lbase = (((int64_t)b * a.sc_layers + a.sc_layer0 + li) * H + (int64_t)g * G) * a.lstride;
-        for (int i = 0; i < n && ok; ++i) {
-            if (i >= 2 && !(ok = __all_sync(0xffffffffu, mbar_wait(p_empty(i & 1), ((i >> 1) - 1) & 1, abort_flag))))
-                break;
-            float v[NC];
-            tmem_ld<NC>(tS + lane_off + kN * i, v);
-            const int tok = t0 + i * kTile + tid;
-            const bool valid = tok >= lo && tok < t1;
-            const bool live = (live_bits >> i) & 1u;  // valid and not dead
-            unsigned char *pbuf = sm + kOffP + (i & 1) * kOpBytes + (tid >> 6) * (kN * 128);
-#pragma unroll
-            for (int h = 0; h < G; ++h) {
-                const float z = v[h] * a.scale_log2;
-                float p = 0.f;
-                if (valid && a.logits && !a.gsum) a.logits[lbase + (int64_t)h * a.lstride + (tok - S0)] = live ? z : -INFINITY;
-                if (live) {  // mx[h] is finite here: it covers this row
-                    p = exp2f(z - mx[h]);
-                    sum[h] += p;
-                }
-                *reinterpret_cast<__nv_bfloat16 *>(pbuf + sw128(h, tid & 63)) = __float2bfloat16_rn(p);
-            }
-            fence_async_smem();
-            mbar_arrive(p_full(i & 1));
-        }
-#pragma unroll
-        for (int h = 0; h < G; ++h) {
-            float t = sum[h];
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-            if (lane == 0) red[warp * kN + h] = t;
-        }
-        __syncwarp();
-        softmax_bar();
-#pragma unroll
-        for (int h = 0; h < G; ++h) sum[h] = red[h] + red[kN + h] + red[2 * kN + h] + red[3 * kN + h];
-
-        // sweep 3 (single-chunk units): the chunk's max and sum are the unit's, so each row's
-        // normalised probabilities are final; their sum over the KV head's query group is
-        // stored per token.  The S tiles are still in TMEM (the PV products go to O).
-        if (a.gsum && a.logits && ok) {
-            if (ns_active == 1) {
-                float inv[G];
-#pragma unroll
-                for (int h = 0; h < G; ++h) inv[h] = sum[h] > 0.f ? 1.f / sum[h] : 0.f;
-                const int64_t gbase = (((int64_t)b * a.sc_layers + a.sc_layer0 + li) * a.kv_heads + g) * a.lstride;
+            if (ok) ok = mbar_wait(s_full, p & 1, abort_flag);
+            ok = __all_sync(0xffffffffu, ok);
+            fence_after_sync();
+            // sweep 1: chunk maximum (-inf for a head when every row of the chunk is dead)
+            if (ok) {
                 for (int i = 0; i < n; ++i) {
                     float v[NC];
                     tmem_ld<NC>(tS + lane_off + kN * i, v);
-                    const int tok = t0 + i * kTile + tid;
-                    if (tok >= lo && tok < t1) {
-                        float acc = 0.f;
-                        if ((live_bits >> i) & 1u) {
+                    if ((live_bits >> i) & 1u) {
 #pragma unroll
-                            for (int h = 0; h < G; ++h) acc += exp2f(v[h] * a.scale_log2 - mx[h]) * inv[h];
-                        }
-                        a.logits[gbase + (tok - S0)] = acc;
+                        for (int h = 0; h < G; ++h) mx[h] = fmaxf(mx[h], v[h] * a.scale_log2);
                     }
                 }
-            } else if (tid == 0) {
-                atomicOr(&g_tc_error, 2u);  // the host only asks for group sums when every unit has one chunk
+            }
+            // chunk max per head over the 128 softmax threads
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                float m = mx[h];
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+                if (lane == 0) red[warp * kN + h] = m;
+            }
+            __syncwarp();
+            softmax_bar();
+#pragma unroll
+            for (int h = 0; h < G; ++h) mx[h] = fmaxf(fmaxf(red[h], red[kN + h]), fmaxf(red[2 * kN + h], red[3 * kN + h]));
+            softmax_bar();
+
+            // sweep 2: logits write-out, exp2, row sums and the P operand of each tile.  The
+            // logits stores sit here, interleaved with the V stream; issued as a burst in
+            // sweep 1 they measured slower.
+            for (int i = 0; i < n && ok; ++i) {
+                const int q = Q + i;
+                if (q >= 2 && !(ok = __all_sync(0xffffffffu, mbar_wait(p_empty(q & 1), ((q >> 1) - 1) & 1, abort_flag))))
+                    break;
+                float v[NC];
+                tmem_ld<NC>(tS + lane_off + kN * i, v);
+                const int tok = t0 + i * kTile + tid;
+                const bool valid = tok >= lo && tok < t1;
+                const bool live = (live_bits >> i) & 1u;  // valid and not dead
+                unsigned char *pbuf = sm + kOffP + (q & 1) * kOpBytes + (tid >> 6) * (kN * 128);
+#pragma unroll
+                for (int h = 0; h < G; ++h) {
+                    const float z = v[h] * a.scale_log2;
+                    float pr = 0.f;
+                    if (valid && a.logits && !a.gsum) a.logits[lbase + (int64_t)h * a.lstride + (tok - S0)] = live ? z : -INFINITY;
+                    if (live) {  // mx[h] is finite here: it covers this row
+                        pr = exp2f(z - mx[h]);
+                        sum[h] += pr;
+                    }
+                    *reinterpret_cast<__nv_bfloat16 *>(pbuf + sw128(h, tid & 63)) = __float2bfloat16_rn(pr);
+                }
+                fence_async_smem();
+                mbar_arrive(p_full(q & 1));
+            }
+            Q += n;
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                float t = sum[h];
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+                if (lane == 0) red[warp * kN + h] = t;
+            }
+            __syncwarp();
+            softmax_bar();
+#pragma unroll
+            for (int h = 0; h < G; ++h) sum[h] = red[h] + red[kN + h] + red[2 * kN + h] + red[3 * kN + h];
+            if (p + 1 < np) softmax_bar();  // red is rewritten by the next pass
+
+            // sweep 3 (single-chunk units): the chunk's max and sum are the unit's, so each row's
+            // normalised probabilities are final; their sum over the KV head's query group is
+            // stored per token.  The S tiles are still in TMEM (the PV products go to O).
+            if (a.gsum && a.logits && ok) {
+                if (ns_active == 1) {
+                    float inv[G];
+#pragma unroll
+                    for (int h = 0; h < G; ++h) inv[h] = sum[h] > 0.f ? 1.f / sum[h] : 0.f;
+                    const int64_t gbase = (((int64_t)b * a.sc_layers + a.sc_layer0 + li) * a.kv_heads + g) * a.lstride;
+                    for (int i = 0; i < n; ++i) {
+                        float v[NC];
+                        tmem_ld<NC>(tS + lane_off + kN * i, v);
+                        const int tok = t0 + i * kTile + tid;
+                        if (tok >= lo && tok < t1) {
+                            float gs = 0.f;
+                            if ((live_bits >> i) & 1u) {
+#pragma unroll
+                                for (int h = 0; h < G; ++h) gs += exp2f(v[h] * a.scale_log2 - mx[h]) * inv[h];
+                            }
+                            a.logits[gbase + (tok - S0)] = gs;
+                        }
+                    }
+                } else if (tid == 0) {
+                    atomicOr(&g_tc_error, 2u);  // the host only asks for group sums when every unit has one chunk
+                }
+            }
+            fence_before_sync();
+            mbar_arrive(s_free);
+
+            if (ok) ok = mbar_wait(o_full, p & 1, abort_flag);
+            ok = __all_sync(0xffffffffu, ok);
+            fence_after_sync();
+            float o[NC];
+#pragma unroll
+            for (int h = 0; h < NC; ++h) o[h] = 0.f;
+            if (ok) tmem_ld<NC>(tO + lane_off, o);
+            fence_before_sync();
+            mbar_arrive(o_free);
+            // fold the pass into the running (max, sum, output); a pass whose rows are all
+            // dead (mx = -inf, sum = 0, O = 0) leaves them unchanged
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                const float mn = fmaxf(M[h], mx[h]);
+                if (mn != -INFINITY) {
+                    const float a_old = exp2f(M[h] - mn), a_new = exp2f(mx[h] - mn);
+                    acc[h] = acc[h] * a_old + o[h] * a_new;
+                    W[h] = W[h] * a_old + sum[h] * a_new;
+                    M[h] = mn;
+                }
             }
         }
 
-        if (ok) ok = mbar_wait(o_full, 0, abort_flag);
-        ok = __all_sync(0xffffffffu, ok);
-        fence_after_sync();
-        if (ns_active == 1) {
-            // the unit's only chunk: its output and log-sum-exp need no merge
+        if (nc_unit == 1) {
+            // the unit's only CTA: its output and log-sum-exp need no merge
             if (ok) {
-                float o[NC];
-                tmem_ld<NC>(tO + lane_off, o);
 #pragma unroll
                 for (int h = 0; h < G; ++h)
                     a.out[(((int64_t)li * a.batch + b) * H + (int64_t)g * G + h) * kD + tid] =
-                        __float2bfloat16_rn(sum[h] > 0.f ? o[h] / sum[h] : 0.f);
+                        __float2bfloat16_rn(W[h] > 0.f ? acc[h] / W[h] : 0.f);
                 if (tid < G) {
                     float mm = -INFINITY, ss = 0.f;
 #pragma unroll
                     for (int h = 0; h < G; ++h)
                         if (h == tid) {
-                            mm = mx[h];
-                            ss = sum[h];
+                            mm = M[h];
+                            ss = W[h];
                         }
                     a.lse2[((int64_t)b * a.sc_layers + a.sc_layer0 + li) * H + (int64_t)g * G + tid] =
                         ss > 0.f ? mm + log2f(ss) : -INFINITY;
                 }
             }
         } else {
-        if (ok) {
-            float o[NC];
-            tmem_ld<NC>(tO + lane_off, o);
             const int64_t pbase = (((int64_t)b * a.n_layers + li) * H + (int64_t)g * G) * a.n_splits;
+            if (ok) {
 #pragma unroll
-            for (int h = 0; h < G; ++h) a.part_o[((pbase + (int64_t)h * a.n_splits) + s) * kD + tid] = o[h];
-            if (tid < G) {
-                float mm = -INFINITY, ss = 0.f;
+                for (int h = 0; h < G; ++h) a.part_o[((pbase + (int64_t)h * a.n_splits) + cta) * kD + tid] = acc[h];
+                if (tid < G) {
+                    float mm = -INFINITY, ss = 0.f;
 #pragma unroll
-                for (int h = 0; h < G; ++h)
-                    if (h == tid) {
-                        mm = mx[h];
-                        ss = sum[h];
-                    }
-                a.part_ml[((pbase + (int64_t)tid * a.n_splits) + s) * 2 + 0] = mm;
-                a.part_ml[((pbase + (int64_t)tid * a.n_splits) + s) * 2 + 1] = ss;
+                    for (int h = 0; h < G; ++h)
+                        if (h == tid) {
+                            mm = M[h];
+                            ss = W[h];
+                        }
+                    a.part_ml[((pbase + (int64_t)tid * a.n_splits) + cta) * 2 + 0] = mm;
+                    a.part_ml[((pbase + (int64_t)tid * a.n_splits) + cta) * 2 + 1] = ss;
+                }
             }
-        }
-        // The last split of (sequence, layer, kv head) to finish merges every
-        // split's partial into the output and the per-head log-sum-exp.  Arrival
-        // counter only: no CTA waits for another.
-        __threadfence();
-        __syncwarp();
-        softmax_bar();
-        int *last_flag = reinterpret_cast<int *>(sm + kOffMisc + 8);
-        const int64_t unit = ((int64_t)b * a.n_layers + li) * a.kv_heads + g;
-        if (tid == 0) *last_flag = (atomicAdd(&a.arrivals[unit], 1) == ns_active - 1) ? 1 : 0;
-        softmax_bar();
-        if (*last_flag && ok) {
+            // The last CTA of (sequence, layer, kv head) to finish merges every CTA's
+            // partial into the output and the per-head log-sum-exp.  Arrival counter
+            // only: no CTA waits for another.
             __threadfence();
-            const int64_t pbase = (((int64_t)b * a.n_layers + li) * H + (int64_t)g * G) * a.n_splits;
-            // split weights [G][n_splits] in the P buffers (every MMA has completed)
-            float *wq = reinterpret_cast<float *>(sm + kOffP);
-            // warp w merges heads w, w + 4: (1) the splits' (max, sum) pairs give the head's
-            // maximum M, each split's weight exp2(m - M) (0 for a split whose rows are all
-            // dead) and the total W; (2) lane i sums the weighted partial outputs of dims
-            // 4i .. 4i+3.  All loads of a phase are independent, so the merge costs a few
-            // L2 round trips whatever the number of splits.
-            for (int h = warp; h < G; h += 4) {
-                const float2 *ml = reinterpret_cast<const float2 *>(a.part_ml) + pbase + (int64_t)h * a.n_splits;
-                float mv[kMaxSplits / 32], lv[kMaxSplits / 32];
-                float M = -INFINITY;
+            __syncwarp();
+            softmax_bar();
+            int *last_flag = reinterpret_cast<int *>(sm + kOffMisc + 8);
+            const int64_t unit = ((int64_t)b * a.n_layers + li) * a.kv_heads + g;
+            if (tid == 0) *last_flag = (atomicAdd(&a.arrivals[unit], 1) == nc_unit - 1) ? 1 : 0;
+            softmax_bar();
+            if (*last_flag && ok) {
+                __threadfence();
+                // partial weights [G][n_splits] in the P buffers (every MMA has completed)
+                float *wq = reinterpret_cast<float *>(sm + kOffP);
+                // warp w merges heads w, w + 4: (1) the partials' (max, sum) pairs give the
+                // head's maximum M, each partial's weight exp2(m - M) (0 for one whose rows are
+                // all dead) and the total W; (2) lane i sums the weighted partial outputs of
+                // dims 4i .. 4i+3.  All loads of a phase are independent, so the merge costs a
+                // few L2 round trips whatever the number of partials.
+                for (int h = warp; h < G; h += 4) {
+                    const float2 *ml = reinterpret_cast<const float2 *>(a.part_ml) + pbase + (int64_t)h * a.n_splits;
+                    float mv[kMaxSplits / 32], lv[kMaxSplits / 32];
+                    float Mh = -INFINITY;
 #pragma unroll
-                for (int k = 0; k < kMaxSplits / 32; ++k) {
-                    const int q = lane + 32 * k;
-                    const float2 x = q < ns_active ? __ldcg(ml + q) : make_float2(-INFINITY, 0.f);
-                    mv[k] = x.x;
-                    lv[k] = x.y;
-                    M = fmaxf(M, x.x);
-                }
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-                const float mref = M == -INFINITY ? 0.f : M;
-                float W = 0.f;
-#pragma unroll
-                for (int k = 0; k < kMaxSplits / 32; ++k) {
-                    const int q = lane + 32 * k;
-                    const float wk = exp2f(mv[k] - mref);
-                    W += lv[k] * wk;
-                    if (q < ns_active) wq[h * a.n_splits + q] = wk;
-                }
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) W += __shfl_xor_sync(0xffffffffu, W, o);
-                __syncwarp();
-                const float4 *po =
-                    reinterpret_cast<const float4 *>(a.part_o + (pbase + (int64_t)h * a.n_splits) * kD) + lane;
-                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-                for (int q0 = 0; q0 < ns_active; q0 += 8) {
-                    float4 ov[8];
-#pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        ov[j] = q0 + j < ns_active ? __ldcg(po + (int64_t)(q0 + j) * (kD / 4))
-                                                   : make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        const float wj = q0 + j < ns_active ? wq[h * a.n_splits + q0 + j] : 0.f;
-                        acc.x += wj * ov[j].x;
-                        acc.y += wj * ov[j].y;
-                        acc.z += wj * ov[j].z;
-                        acc.w += wj * ov[j].w;
+                    for (int k = 0; k < kMaxSplits / 32; ++k) {
+                        const int q = lane + 32 * k;
+                        const float2 x = q < nc_unit ? __ldcg(ml + q) : make_float2(-INFINITY, 0.f);
+                        mv[k] = x.x;
+                        lv[k] = x.y;
+                        Mh = fmaxf(Mh, x.x);
                     }
+#pragma unroll
+                    for (int o = 16; o > 0; o >>= 1) Mh = fmaxf(Mh, __shfl_xor_sync(0xffffffffu, Mh, o));
+                    const float mref = Mh == -INFINITY ? 0.f : Mh;
+                    float Wh = 0.f;
+#pragma unroll
+                    for (int k = 0; k < kMaxSplits / 32; ++k) {
+                        const int q = lane + 32 * k;
+                        const float wk = exp2f(mv[k] - mref);
+                        Wh += lv[k] * wk;
+                        if (q < nc_unit) wq[h * a.n_splits + q] = wk;
+                    }
+#pragma unroll
+                    for (int o = 16; o > 0; o >>= 1) Wh += __shfl_xor_sync(0xffffffffu, Wh, o);
+                    __syncwarp();
+                    const float4 *po =
+                        reinterpret_cast<const float4 *>(a.part_o + (pbase + (int64_t)h * a.n_splits) * kD) + lane;
+                    float4 sacc = make_float4(0.f, 0.f, 0.f, 0.f);
+                    for (int q0 = 0; q0 < nc_unit; q0 += 8) {
+                        float4 ov[8];
+#pragma unroll
+                        for (int j = 0; j < 8; ++j)
+                            ov[j] = q0 + j < nc_unit ? __ldcg(po + (int64_t)(q0 + j) * (kD / 4))
+                                                     : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) {
+                            const float wj = q0 + j < nc_unit ? wq[h * a.n_splits + q0 + j] : 0.f;
+                            sacc.x += wj * ov[j].x;
+                            sacc.y += wj * ov[j].y;
+                            sacc.z += wj * ov[j].z;
+                            sacc.w += wj * ov[j].w;
+                        }
+                    }
+                    const bool any = Wh > 0.f;  // false only if every slot of the unit is dead
+                    __nv_bfloat162 r0 = __floats2bfloat162_rn(any ? sacc.x / Wh : 0.f, any ? sacc.y / Wh : 0.f);
+                    __nv_bfloat162 r1 = __floats2bfloat162_rn(any ? sacc.z / Wh : 0.f, any ? sacc.w / Wh : 0.f);
+                    uint2 packed;
+                    packed.x = *reinterpret_cast<uint32_t *>(&r0);
+                    packed.y = *reinterpret_cast<uint32_t *>(&r1);
+                    *reinterpret_cast<uint2 *>(a.out + (((int64_t)li * a.batch + b) * H + (int64_t)g * G + h) * kD +
+                                               4 * lane) = packed;
+                    if (lane == 0)
+                        a.lse2[((int64_t)b * a.sc_layers + a.sc_layer0 + li) * H + (int64_t)g * G + h] =
+                            any ? Mh + log2f(Wh) : -INFINITY;
                 }
-                const bool any = W > 0.f;  // false only if every slot of the unit is dead
-                __nv_bfloat162 r0 = __floats2bfloat162_rn(any ? acc.x / W : 0.f, any ? acc.y / W : 0.f);
-                __nv_bfloat162 r1 = __floats2bfloat162_rn(any ? acc.z / W : 0.f, any ? acc.w / W : 0.f);
-                uint2 packed;
-                packed.x = *reinterpret_cast<uint32_t *>(&r0);
-                packed.y = *reinterpret_cast<uint32_t *>(&r1);
-                *reinterpret_cast<uint2 *>(a.out + (((int64_t)li * a.batch + b) * H + (int64_t)g * G + h) * kD +
-                                           4 * lane) = packed;
-                if (lane == 0)
-                    a.lse2[((int64_t)b * a.sc_layers + a.sc_layer0 + li) * H + (int64_t)g * G + h] =
-                        any ? M + log2f(W) : -INFINITY;
+                if (tid == 0) a.arrivals[unit] = 0;
             }
-            if (tid == 0) a.arrivals[unit] = 0;
-        }
         }
     }
     fence_before_sync();
@@ -731,8 +797,20 @@ bool tc_supported(int dtype, int head_dim, int group, int page_size) {
     return page_size >= 8 && 128 % page_size == 0;
 }
 
+#ifndef IKV_TC_PASSES
+#define IKV_TC_PASSES 1
+#endif
+// Consecutive chunks per CTA.  When the launch's units nearly fill one wave of resident
+// CTAs on their own but their chunks do not (each chunk is at most 15 tiles), one CTA per
+// unit takes all of the unit's chunks as passes: no second wave and no cross-CTA merge.
+static int tc_passes(int64_t units, int n_chunks, int sms, bool gsum) {
+    if (!IKV_TC_PASSES || gsum || n_chunks <= 1 || units <= 0) return 1;
+    const int64_t slots = (int64_t)2 * sms;
+    if (units > slots || units * 4 < slots * 3) return 1;
+    return n_chunks;
+}
+
 cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group, int sms, cudaStream_t st) {
-    (void)sms;
     const int rpb = a.pv.page_size >= kTile ? kTile : a.pv.page_size;
     // rows of every layer the launch can touch: [layers][num_pages][kv_heads][page_size]
     const uint64_t rows = (uint64_t)(a.layer0 + a.n_layers) * a.pv.num_pages * a.pv.kv_heads * a.pv.page_size;
@@ -774,7 +852,9 @@ cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group,
     t.v_pool = reinterpret_cast<__nv_bfloat16 *>(const_cast<void *>(a.v));
     t.vnorm = a.vnorm;
     t.gsum = a.gsum;
-    dim3 grid(a.n_splits * a.pv.kv_heads * a.batch * a.n_layers);
+    const int64_t units = (int64_t)a.pv.kv_heads * a.batch * a.n_layers;
+    t.passes = tc_passes(units, a.n_splits, sms, a.gsum != 0);
+    dim3 grid((unsigned)(((a.n_splits + t.passes - 1) / t.passes) * units));
     cudaError_t e;
     switch (group) {
         case 1: e = launch_tc_g<1>(mk, mv, t, grid, st); break;

@@ -195,6 +195,57 @@ def test_decode_attend_score_skips_dead_slots(ps):
         assert np.array_equal(ema[b, :L].cpu().numpy()[dead], (np.float32(alpha) * e0[dead]).astype(np.float32))
 
 
+def test_attend_multi_pass_units():
+    """256 (sequence, kv head) units of up to 30 tiles: the units nearly fill one wave of
+    resident CTAs but their 15-tile chunks do not, so each CTA takes its unit's chunks as
+    consecutive passes.  Ragged lengths (one chunk, two, an empty sequence), a sequence
+    whose first chunk is all dead, one whose second chunk is all dead and one whose only
+    live slot sits in its second chunk."""
+    rng = np.random.default_rng(31)
+    lens = [int(x) for x in rng.integers(1, 3841, size=32)]
+    lens[:6] = [3840, 3840, 3000, 0, 1920, 1921]
+    w = gen.Workload("a", 32, 2, 32, 8, 128, lens, 1, dtype=gen.BF16, seed=27, page_size=64)
+    u = w.u_table()
+    c = make_cache(w, page_perm_seed=8)
+    fill_device(c, w, torch.from_numpy(u).cuda())
+    pos = c.pos.cpu().numpy()
+    pos[0, :1920] = -1          # first chunk dead
+    pos[1, 1920:3840] = -1      # second chunk dead
+    pos[2, :3000] = -1
+    pos[2, 2500] = 2500         # one live slot, in the second chunk
+    pos[6, :lens[6]][rng.random(lens[6]) < 0.3] = -1
+    c.pos.copy_(torch.from_numpy(pos).cuda())
+    layer = 1
+    q_h = w.queries(1, 2, u)[0, layer]
+    q = to_device(q_h, w)
+    out = torch.full((32, 32, 128), 7.0, dtype=q.dtype, device="cuda")
+    score = torch.full((c.rows, c.cap), -7.0, device="cuda")
+    ema0 = torch.from_numpy(rng.random((c.rows, c.cap)).astype(np.float32)).cuda()
+    ema = ema0.clone()
+    cch = c.cache(max(lens), dead_slots=True)
+    ws = torch.empty(ikv.ikv_attend_workspace_size(c.shape(), cch), dtype=torch.uint8, device="cuda")
+    alpha = 0.6
+    ikv.ikv_decode_attend_score(c.shape(), cch, layer, q, out, score, ema, alpha, ws, ws.numel())
+    torch.cuda.synchronize()
+    assert ikv.ikv_device_status() == 0
+    q64 = as_f64(q_h, w)
+    for b, L in enumerate(lens):
+        if L == 0:
+            assert torch.all(out[b] == 0)
+            continue
+        live = np.nonzero(pos[b, :L] >= 0)[0]
+        k, v = w.kv_rows(b, layer, live, u)
+        a_, o = O.last_query_attention(q64[b], [x.astype(np.float64) for x in k], [x.astype(np.float64) for x in v])
+        assert np.max(np.abs(out[b].float().cpu().numpy() - o)) < 2e-2, b
+        sc = O.pooled_score(a_, O.GRAN_SEQ, 8)[0]
+        got = score[b, :L].cpu().numpy()
+        assert np.max(np.abs(got[live] - sc)) < 2e-5, b
+        assert np.all(got[pos[b, :L] < 0] == 0.0), b
+        want = O.ema_update(ema0[b, :L].double().cpu().numpy(), np.where(pos[b, :L] >= 0, 0.0, 0.0), alpha)
+        want[live] = O.ema_update(ema0[b, :L].double().cpu().numpy()[live], sc, alpha)
+        assert np.max(np.abs(ema[b, :L].cpu().numpy() - want)) < 2e-5, b
+
+
 def _attend_case(w, c, layer, kv=None, u=None, alpha=0.5):
     """Run one attention layer through the ABI and compare it with the oracle (GRAN_SEQ)."""
     u = w.u_table() if u is None else u
