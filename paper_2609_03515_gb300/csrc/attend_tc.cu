@@ -201,7 +201,9 @@ __device__ __forceinline__ uint32_t sw128(uint32_t row, uint32_t col) {
     return row * 128u + ((((col >> 3) ^ row) & 7u) << 4) + ((col & 7u) << 1);
 }
 
-template <int G>
+// MP: the launch may give a CTA more than one pass (a.passes > 1); without it the pass
+// loop, the s_free / o_free handshakes and the register fold compile away.
+template <int G, bool MP>
 __global__ void __launch_bounds__(kThreads, 2)
     attend_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, const TcArgs a) {
     constexpr int NC = G <= 4 ? 4 : 8;  // TMEM columns read per S tile
@@ -241,15 +243,15 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         return;
     }
-    const int np = min(a.passes, ns_active - c0);             // passes of this CTA
-    const int nc_unit = (ns_active + a.passes - 1) / a.passes;  // CTAs that cover the unit
+    const int np = MP ? min(a.passes, ns_active - c0) : 1;             // passes of this CTA
+    const int nc_unit = MP ? (ns_active + a.passes - 1) / a.passes : ns_active;  // CTAs that cover the unit
     if (item > kMaxTiles) {  // the host sizes chunks to fit TMEM; refuse rather than overrun
         if (threadIdx.x == 0) atomicOr(&g_tc_error, 2u);
         return;
     }
     // pass p: tiles and physical slot of the first row
-    auto chunk_n = [&](int p) { return min(item, nt_unit - (c0 + p) * item); };
-    auto chunk_t0 = [&](int p) { return (ft + (c0 + p) * item) * kTile; };
+    auto chunk_n = [&](int p) { return min(item, nt_unit - (c0 + (MP ? p : 0)) * item); };
+    auto chunk_t0 = [&](int p) { return (ft + (c0 + (MP ? p : 0)) * item) * kTile; };
     const int H = a.q_heads;
 
     const uint32_t sQ = base + kOffQ, sP = base + kOffP;
@@ -565,8 +567,10 @@ __global__ void __launch_bounds__(kThreads, 2)
                     atomicOr(&g_tc_error, 2u);  // the host only asks for group sums when every unit has one chunk
                 }
             }
-            fence_before_sync();
-            mbar_arrive(s_free);
+            if (MP) {
+                fence_before_sync();
+                mbar_arrive(s_free);
+            }
 
             if (ok) ok = mbar_wait(o_full, p & 1, abort_flag);
             ok = __all_sync(0xffffffffu, ok);
@@ -575,18 +579,27 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
             for (int h = 0; h < NC; ++h) o[h] = 0.f;
             if (ok) tmem_ld<NC>(tO + lane_off, o);
-            fence_before_sync();
-            mbar_arrive(o_free);
-            // fold the pass into the running (max, sum, output); a pass whose rows are all
-            // dead (mx = -inf, sum = 0, O = 0) leaves them unchanged
+            if (MP) {
+                fence_before_sync();
+                mbar_arrive(o_free);
+                // fold the pass into the running (max, sum, output); a pass whose rows are
+                // all dead (mx = -inf, sum = 0, O = 0) leaves them unchanged
 #pragma unroll
-            for (int h = 0; h < G; ++h) {
-                const float mn = fmaxf(M[h], mx[h]);
-                if (mn != -INFINITY) {
-                    const float a_old = exp2f(M[h] - mn), a_new = exp2f(mx[h] - mn);
-                    acc[h] = acc[h] * a_old + o[h] * a_new;
-                    W[h] = W[h] * a_old + sum[h] * a_new;
-                    M[h] = mn;
+                for (int h = 0; h < G; ++h) {
+                    const float mn = fmaxf(M[h], mx[h]);
+                    if (mn != -INFINITY) {
+                        const float a_old = exp2f(M[h] - mn), a_new = exp2f(mx[h] - mn);
+                        acc[h] = acc[h] * a_old + o[h] * a_new;
+                        W[h] = W[h] * a_old + sum[h] * a_new;
+                        M[h] = mn;
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int h = 0; h < G; ++h) {
+                    M[h] = mx[h];
+                    W[h] = sum[h];
+                    acc[h] = o[h];
                 }
             }
         }
@@ -739,15 +752,19 @@ bool make_map(CUtensorMap *m, const void *pool, uint64_t rows, int rows_per_box)
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int G>
-cudaError_t launch_tc_g(const CUtensorMap &mk, const CUtensorMap &mv, const TcArgs &t, dim3 grid, cudaStream_t st) {
+template <int G, bool MP>
+cudaError_t launch_tc_gm(const CUtensorMap &mk, const CUtensorMap &mv, const TcArgs &t, dim3 grid, cudaStream_t st) {
     static bool attr = false;
     if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(attend_tc_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        cudaError_t e = cudaFuncSetAttribute(attend_tc_kernel<G, MP>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
         if (e != cudaSuccess) return e;
         attr = true;
     }
-    return launch_k(attend_tc_kernel<G>, grid, dim3(kThreads), kSmemBytes, st, mk, mv, t);
+    return launch_k(attend_tc_kernel<G, MP>, grid, dim3(kThreads), kSmemBytes, st, mk, mv, t);
+}
+template <int G>
+cudaError_t launch_tc_g(const CUtensorMap &mk, const CUtensorMap &mv, const TcArgs &t, dim3 grid, cudaStream_t st) {
+    return t.passes > 1 ? launch_tc_gm<G, true>(mk, mv, t, grid, st) : launch_tc_gm<G, false>(mk, mv, t, grid, st);
 }
 
 }  // namespace
