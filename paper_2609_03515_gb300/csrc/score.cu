@@ -106,22 +106,36 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
                 if (il < L && j < nb) z[j] = __ldg(reinterpret_cast<const VT *>(zp));
                 zp += a.lstride;
             }
+            // each row's probabilities times the VNorm weight (1 for the other scorers)
+            auto weight = [&](int j, float *w) {
 #pragma unroll
-            for (int j = 0; j < kHB; ++j) {
-                const float lj = __shfl_sync(0xffffffffu, lse_lane, j);
-                if (il < L && j < nb) {
-                    float w[V];
+                for (int v = 0; v < V; ++v) w[v] = 1.f;
+                if (SCORER == IKV_SCORE_VNORM) {
+                    const int gr = a.gsum ? hb + j : (h0 + hb + j) / G - g0;  // the row's kv head
+                    const float *wg = wv + gr * kTok + lane * V;
 #pragma unroll
-                    for (int v = 0; v < V; ++v) w[v] = 1.f;
-                    if (SCORER == IKV_SCORE_VNORM) {
-                        const int gr = a.gsum ? hb + j : (h0 + hb + j) / G - g0;  // the row's kv head
-                        const float *wg = wv + gr * kTok + lane * V;
+                    for (int v = 0; v < V; ++v) w[v] = wg[v];
+                }
+            };
+            if (a.gsum) {
 #pragma unroll
-                        for (int v = 0; v < V; ++v) w[v] = wg[v];
+                for (int j = 0; j < kHB; ++j)
+                    if (il < L && j < nb) {
+                        float w[V];
+                        weight(j, w);
+#pragma unroll
+                        for (int v = 0; v < V; ++v) acc[v] += vget(z[j], v) * w[v];
                     }
+            } else {
 #pragma unroll
-                    for (int v = 0; v < V; ++v)
-                        acc[v] += (a.gsum ? vget(z[j], v) : exp2f(vget(z[j], v) - lj)) * w[v];
+                for (int j = 0; j < kHB; ++j) {
+                    const float lj = __shfl_sync(0xffffffffu, lse_lane, j);
+                    if (il < L && j < nb) {
+                        float w[V];
+                        weight(j, w);
+#pragma unroll
+                        for (int v = 0; v < V; ++v) acc[v] += exp2f(vget(z[j], v) - lj) * w[v];
+                    }
                 }
             }
         }
@@ -213,9 +227,9 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
         // the row's CTAs that hold tokens arrive once their utilities are stored; the
         // last one selects the row (arrival counter only: no CTA waits for another)
         __shared__ int last;
-        __threadfence();
         __syncthreads();
         if (threadIdx.x == 0) {
+            __threadfence();  // after the barrier: releases every thread's stores of this block
             last = atomicAdd(&a.row_done[r], 1) == blocks - 1;
             if (last) a.row_done[r] = 0;
         }
