@@ -117,6 +117,20 @@ def test_deferred_compaction_trajectories():
     _assert(run_lockstep(small_llama(steps=8, refresh_period=2), refresh_init=ikv.IKV_INIT_MEAN, max_holes=64), 2e-2)
 
 
+def test_multi_pass_trajectories():
+    """256 (sequence, layer, kv head) units of 16-31 tiles: the units nearly fill one wave of
+    resident CTAs, so each CTA takes its unit's 15-tile chunks as passes, merged in registers.
+    A 90% budget keeps the units long on every step; ragged lengths, deferred compaction
+    (dead slots inside the passes), the KV-head granularity and the VNorm scorer."""
+    rng = np.random.default_rng(41)
+    prefill = [int(x) for x in rng.integers(1900, 3800, size=16)]
+    w = small_llama(batch=16, layers=2, prefill=prefill, steps=4, budget_frac=0.9)
+    _assert(run_lockstep(w), 2e-2)
+    _assert(run_lockstep(w, max_holes=64, compact_mode=ikv.IKV_COMPACT_STABLE_SHORT), 2e-2)
+    _assert(run_lockstep(w.with_(steps=3), gran=ikv.IKV_GRAN_KVHEAD), 2e-2)
+    _assert(run_lockstep(w.with_(steps=3), scorer=ikv.IKV_SCORE_VNORM), 2e-2)
+
+
 def test_cumulative_and_single_step_aggregation():
     """Eq. 3 (cumulative) and Eq. 2 (single-step) in place of the EMA, under full refresh,
     Lazy refresh and deferred compaction."""
