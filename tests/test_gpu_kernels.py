@@ -195,16 +195,17 @@ def test_decode_attend_score_skips_dead_slots(ps):
         assert np.array_equal(ema[b, :L].cpu().numpy()[dead], (np.float32(alpha) * e0[dead]).astype(np.float32))
 
 
-def test_attend_multi_pass_units():
-    """256 (sequence, kv head) units of up to 30 tiles: the units nearly fill one wave of
-    resident CTAs but their 15-tile chunks do not, so each CTA takes its unit's chunks as
-    consecutive passes.  Ragged lengths (one chunk, two, an empty sequence), a sequence
-    whose first chunk is all dead, one whose second chunk is all dead and one whose only
-    live slot sits in its second chunk."""
+@pytest.mark.parametrize("H,Hkv,batch", [(32, 8, 32), (28, 4, 64), (64, 8, 32), (16, 8, 32), (8, 8, 32)])
+def test_attend_multi_pass_units(H, Hkv, batch):
+    """256 (sequence, kv head) units of up to 30 tiles, G = 4, 7, 8, 2 and 1: the units nearly
+    fill one wave of resident CTAs but their 15-tile chunks do not, so each CTA takes its
+    unit's chunks as consecutive passes.  Ragged lengths (one chunk, two, an empty
+    sequence), a sequence whose first chunk is all dead, one whose second chunk is all dead
+    and one whose only live slot sits in its second chunk."""
     rng = np.random.default_rng(31)
-    lens = [int(x) for x in rng.integers(1, 3841, size=32)]
+    lens = [int(x) for x in rng.integers(1, 3841, size=batch)]
     lens[:6] = [3840, 3840, 3000, 0, 1920, 1921]
-    w = gen.Workload("a", 32, 2, 32, 8, 128, lens, 1, dtype=gen.BF16, seed=27, page_size=64)
+    w = gen.Workload("a", batch, 2, H, Hkv, 128, lens, 1, dtype=gen.BF16, seed=27, page_size=64)
     u = w.u_table()
     c = make_cache(w, page_perm_seed=8)
     fill_device(c, w, torch.from_numpy(u).cuda())
@@ -218,7 +219,7 @@ def test_attend_multi_pass_units():
     layer = 1
     q_h = w.queries(1, 2, u)[0, layer]
     q = to_device(q_h, w)
-    out = torch.full((32, 32, 128), 7.0, dtype=q.dtype, device="cuda")
+    out = torch.full((batch, H, 128), 7.0, dtype=q.dtype, device="cuda")
     score = torch.full((c.rows, c.cap), -7.0, device="cuda")
     ema0 = torch.from_numpy(rng.random((c.rows, c.cap)).astype(np.float32)).cuda()
     ema = ema0.clone()
@@ -237,7 +238,7 @@ def test_attend_multi_pass_units():
         k, v = w.kv_rows(b, layer, live, u)
         a_, o = O.last_query_attention(q64[b], [x.astype(np.float64) for x in k], [x.astype(np.float64) for x in v])
         assert np.max(np.abs(out[b].float().cpu().numpy() - o)) < 2e-2, b
-        sc = O.pooled_score(a_, O.GRAN_SEQ, 8)[0]
+        sc = O.pooled_score(a_, O.GRAN_SEQ, Hkv)[0]
         got = score[b, :L].cpu().numpy()
         assert np.max(np.abs(got[live] - sc)) < 2e-5, b
         assert np.all(got[pos[b, :L] < 0] == 0.0), b
