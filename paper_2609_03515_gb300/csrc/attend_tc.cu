@@ -24,7 +24,7 @@
 // Warp roles (192 threads): warps 0-3 own TMEM lanes 0-127 (softmax, epilogue),
 // warp 4 issues TMA loads, warp 5 issues MMAs.  Every mbarrier wait is bounded;
 // on timeout the CTA records an error code, stops issuing work, waits for its
-// in-flight copies, frees its TMEM and returns.
+// in-flight copies and MMAs, frees its TMEM and returns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -53,8 +53,8 @@ constexpr int kOffQ = kNst * kStage;
 constexpr int kOffP = kOffQ + kOpBytes;
 constexpr int kOffRed = kOffP + 2 * kOpBytes;
 constexpr int kOffBar = kOffRed + 4 * kN * 4;
-// barriers: full[kNst], empty[kNst], s_full, p_full[2], p_empty[2], o_full, s_free, o_free
-constexpr int kNumBar = 2 * kNst + 8;
+// barriers: full[kNst], empty[kNst], s_full, p_full[2], p_empty[2], o_full, s_free, o_free, mma_done
+constexpr int kNumBar = 2 * kNst + 9;
 constexpr int kOffMisc = kOffBar + kNumBar * 8;
 constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // misc: tmem slot, abort flag, last-split flag   // + slack for 1024-byte alignment
 
@@ -133,6 +133,19 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
     *abort = 1;
     atomicOr(&g_tc_error, kErrTimeout);
     return false;
+}
+
+// Wait for the MMAs this thread has issued, whatever the abort flag says (at most kWaitNs):
+// TMEM is freed only after every tcgen05 operation writing it has completed.
+__device__ __forceinline__ void mbar_drain(uint32_t bar, uint32_t parity) {
+    const uint64_t start = global_ns();
+    for (uint32_t i = 0; !mbar_test(bar, parity); ++i) {
+        if (i > 64) __nanosleep(32);
+        if ((i & 63u) == 63u && global_ns() - start > kWaitNs) {
+            atomicOr(&g_tc_error, kErrTimeout);
+            return;
+        }
+    }
 }
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uint32_t bar) {
@@ -265,6 +278,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     const uint32_t o_full = bar0 + 8u * (2 * kNst + 5);
     const uint32_t s_free = bar0 + 8u * (2 * kNst + 6);  // the softmax is done with a pass's S tiles
     const uint32_t o_free = bar0 + 8u * (2 * kNst + 7);  // the softmax has read a pass's O
+    const uint32_t mma_done = bar0 + 8u * (2 * kNst + 8);  // every MMA of the CTA has completed
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(sm + kOffMisc);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + kOffMisc + 4);
 
@@ -343,6 +357,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             mbar_init(o_full, 1);
             mbar_init(s_free, 128);
             mbar_init(o_free, 128);
+            mbar_init(mma_done, 1);
             *abort_flag = 0;
             asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
             while (ld_J < kNst && ld_p < np) issue_next();
@@ -437,6 +452,9 @@ __global__ void __launch_bounds__(kThreads, 2)
                 Q += n;
                 mma_commit(o_full);
             }
+            // also after an abort: no MMA may still write TMEM when it is freed
+            mma_commit(mma_done);
+            mbar_drain(mma_done, 0);
         }
         __syncwarp();
     } else {
