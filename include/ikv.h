@@ -229,6 +229,22 @@ ikv_status ikv_device_status(uint32_t *flags);
 enum { IKV_PATH_CUDA_CORE = 0, IKV_PATH_TENSOR_CORE = 1 };
 ikv_status ikv_attend_path(const ikv_shape *shape, const ikv_cache *cache, int32_t *path);
 
+/* How one attention launch over n_layers layers of every sequence (shape->layers: the
+ * launch ikv_step makes; 1: a layer call of the split step) at lengths up to
+ * cache->max_len is partitioned on a GPU with sms SMs (0: the current device's).  Each
+ * (sequence, layer, KV head) unit's slots are cut into *n_chunks chunks of *chunk_tokens
+ * slots (the tensor-core kernel sizes them for about one wave of two CTAs per SM, at
+ * most 15 tiles of 128 slots); a CTA takes *passes consecutive chunks of its unit in turn
+ * (more than 1 when the units alone nearly fill that wave but their chunks do not);
+ * *group_sums is 1 when every unit is one chunk, so the launch hands the score pass
+ * per-KV-head sums of normalised probabilities instead of per-head logits (Eq. 1 needs
+ * only those).  *path as ikv_attend_path.  Host only; launches nothing.  Any output
+ * pointer may be NULL; fails with IKV_ERR_ARG if n_layers is outside [1, layers] or
+ * sms < 0. */
+ikv_status ikv_attend_plan(const ikv_shape *shape, const ikv_cache *cache, int32_t n_layers, int32_t sms,
+                           int32_t *path, int32_t *chunk_tokens, int32_t *n_chunks, int32_t *passes,
+                           int32_t *group_sums);
+
 /* ---------------------------------------------------------------------------
  * ikv_decode_attend_score -- one layer of decode attention plus its score.
  *

@@ -201,9 +201,9 @@ T *at(void *ws, size_t off) {
 // (ctas_per_sm x SMs), splits a multiple of `granule` tokens and at most
 // `max_split` tokens long, at most kMaxSplits per (sequence, layer, kv head)
 void choose_splits(const ikv_shape *s, int n_layers, int32_t max_len, int granule, int max_split,
-                   int32_t *split_tokens, int32_t *n_splits) {
+                   int32_t *split_tokens, int32_t *n_splits, int sms) {
     const int64_t units = (int64_t)s->batch * n_layers * s->kv_heads;
-    const int64_t want = (int64_t)sm_count() * 4;
+    const int64_t want = (int64_t)sms * 4;
     int64_t splits = (want + units - 1) / units;
     const int64_t by_len = (max_len + kMinSplitTokens - 1) / kMinSplitTokens;
     if (splits > by_len) splits = by_len;
@@ -266,7 +266,7 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
         // one chunk per unit: the kernel can hand the score pass normalised group sums
         a.gsum = gsum && logits && nc == 1 && use_tc(s, c, s->layers, max_len) ? 1 : 0;
     } else
-        choose_splits(s, n_layers, max_len, kTileTokens, 1 << 30, &a.split_tokens, &a.n_splits);
+        choose_splits(s, n_layers, max_len, kTileTokens, 1 << 30, &a.split_tokens, &a.n_splits, sm_count());
     a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)s->head_dim));
     a.logits = logits ? at<float>(ws, w.logits) : nullptr;
     if (gsum) *gsum = false;
@@ -441,6 +441,39 @@ ikv_status ikv_attend_path(const ikv_shape *shape, const ikv_cache *cache, int32
     if ((e = check_cache(shape, cache, false))) return e;
     if (!path) return fail(IKV_ERR_ARG, "path is NULL");
     *path = use_tc(shape, cache, shape->layers, cache->max_len) ? IKV_PATH_TENSOR_CORE : IKV_PATH_CUDA_CORE;
+    return IKV_OK;
+}
+
+ikv_status ikv_attend_plan(const ikv_shape *shape, const ikv_cache *cache, int32_t n_layers, int32_t sms,
+                           int32_t *path, int32_t *chunk_tokens, int32_t *n_chunks, int32_t *passes,
+                           int32_t *group_sums) {
+    g_err[0] = 0;
+    ikv_status e = check_shape(shape);
+    if (e) return e;
+    if ((e = check_cache(shape, cache, false))) return e;
+    if (n_layers < 1 || n_layers > shape->layers)
+        return fail(IKV_ERR_ARG, "n_layers %d outside [1, %d]", n_layers, shape->layers);
+    if (sms < 0) return fail(IKV_ERR_ARG, "sms must be >= 0");
+    if (sms == 0) sms = sm_count();
+    // the decisions run_attend and launch_attend_tc take for a launch from layer 0
+    const int32_t max_len = cache->max_len;
+    const int64_t units = (int64_t)shape->batch * n_layers * shape->kv_heads;
+    const bool tc = use_tc(shape, cache, n_layers, max_len);
+    int32_t ct = 0, nc = 0, np = 1, gs = 0;
+    if (tc) {
+        int32_t it = 0;
+        tc_plan(max_len + 127, units, sms, &it, &nc);
+        ct = it * 128;
+        gs = nc == 1 && use_tc(shape, cache, shape->layers, max_len) ? 1 : 0;
+        np = tc_passes(units, nc, sms, gs != 0);
+    } else {
+        choose_splits(shape, n_layers, max_len, kTileTokens, 1 << 30, &ct, &nc, sms);
+    }
+    if (path) *path = tc ? IKV_PATH_TENSOR_CORE : IKV_PATH_CUDA_CORE;
+    if (chunk_tokens) *chunk_tokens = ct;
+    if (n_chunks) *n_chunks = nc;
+    if (passes) *passes = np;
+    if (group_sums) *group_sums = gs;
     return IKV_OK;
 }
 

@@ -838,7 +838,7 @@ bool tc_supported(int dtype, int head_dim, int group, int page_size) {
 // Consecutive chunks per CTA.  When the launch's units nearly fill one wave of resident
 // CTAs on their own but their chunks do not (each chunk is at most 15 tiles), one CTA per
 // unit takes all of the unit's chunks as passes: no second wave and no cross-CTA merge.
-static int tc_passes(int64_t units, int n_chunks, int sms, bool gsum) {
+int tc_passes(int64_t units, int n_chunks, int sms, bool gsum) {
     if (!IKV_TC_PASSES || gsum || n_chunks <= 1 || units <= 0) return 1;
     const int64_t slots = (int64_t)2 * sms;
     if (units > slots || units * 4 < slots * 3) return 1;

@@ -167,6 +167,8 @@ struct TcOutputs {
     int32_t *arrivals;          // [batch][n_layers][kv_heads] zeroed before the launch
 };
 void tc_plan(int32_t max_len, int64_t units, int sms, int32_t *item_tiles, int32_t *n_chunks);
+// consecutive chunks one CTA of the tensor-core kernel takes, for that chunk plan
+int tc_passes(int64_t units, int n_chunks, int sms, bool gsum);
 cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group, int sms, cudaStream_t st);
 
 // launchers (return cudaError_t of the launch)

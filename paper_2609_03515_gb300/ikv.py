@@ -73,6 +73,7 @@ def _load():
         "ikv_launch_count": ([], ctypes.c_int64),
         "ikv_device_status": ([ctypes.POINTER(ctypes.c_uint32)], I32),
         "ikv_attend_path": ([SP, CP, ctypes.POINTER(I32)], I32),
+        "ikv_attend_plan": ([SP, CP, I32, I32] + [ctypes.POINTER(I32)] * 5, I32),
         "ikv_attend_workspace_size": ([SP, CP, ctypes.POINTER(SZ)], I32),
         "ikv_decode_attend_score": ([SP, CP, I32, P, P, P, P, F32, P, SZ, P], I32),
         "ikv_static_scratch_bytes": ([], SZ),
@@ -138,6 +139,15 @@ def ikv_attend_path(shape: ikv_shape, cache: ikv_cache) -> int:
     v = I32(0)
     _check(_lib.ikv_attend_path(ctypes.byref(shape), ctypes.byref(cache), ctypes.byref(v)), "ikv_attend_path")
     return int(v.value)
+
+
+def ikv_attend_plan(shape: ikv_shape, cache: ikv_cache, n_layers: int, sms: int = 0) -> dict:
+    """The partition of one attention launch over n_layers layers (see include/ikv.h)."""
+    v = [I32(0) for _ in range(5)]
+    _check(_lib.ikv_attend_plan(ctypes.byref(shape), ctypes.byref(cache), n_layers, sms,
+                                *[ctypes.byref(x) for x in v]), "ikv_attend_plan")
+    keys = ("path", "chunk_tokens", "n_chunks", "passes", "group_sums")
+    return {k: int(x.value) for k, x in zip(keys, v)}
 
 
 def ikv_attend_workspace_size(shape: ikv_shape, cache: ikv_cache) -> int:

@@ -252,6 +252,38 @@ def test_attend_path_query(lib):
         path(dict(bf, q_heads=5, kv_heads=2), {})
 
 
+def test_attend_plan_query(lib):
+    """How each workload's attention launch is partitioned is decided on the host (152 SMs):
+    chunk size and count per (sequence, layer, KV head) unit, the passes one CTA takes, and
+    whether the launch hands the score pass group sums."""
+    def plan(batch, layers, H, Hkv, max_len, n_layers, dtype=lib.IKV_BF16, d=128, sms=152):
+        pages = (max_len + 1 + 63) // 64 + 1
+        shp = _shape(lib, batch=batch, layers=layers, q_heads=H, kv_heads=Hkv, head_dim=d, dtype=dtype)
+        cch = _cache(lib, num_pages=batch * pages, max_pages=pages, max_len=max_len)
+        return lib.ikv_attend_plan(shp, cch, n_layers, sms)
+    tc, cc = lib.IKV_PATH_TENSOR_CORE, lib.IKV_PATH_CUDA_CORE
+    # Llama b = 1, 3278 slots (+ one decode token): 256 units of 27 tiles fill 256 of 304
+    # slots, so each CTA takes its unit's two 15-tile chunks in turn
+    assert plan(1, 32, 32, 8, 3279, 32) == dict(path=tc, chunk_tokens=1920, n_chunks=2, passes=2, group_sums=0)
+    # ... and one layer of it (split step): 8 units, the shortest chunks that fill one wave
+    assert plan(1, 32, 32, 8, 3279, 1) == dict(path=tc, chunk_tokens=256, n_chunks=14, passes=1, group_sums=0)
+    # Llama b = 8, 6554 slots: 2048 units, one wave's worth of 15-tile chunks, merged
+    assert plan(8, 32, 32, 8, 6555, 32) == dict(path=tc, chunk_tokens=1920, n_chunks=4, passes=1, group_sums=0)
+    # Llama b = 16 at ~800 slots and Qwen b = 32 at 1638: every unit one chunk -> group sums
+    assert plan(16, 32, 32, 8, 820, 32) == dict(path=tc, chunk_tokens=1920, n_chunks=1, passes=1, group_sums=1)
+    assert plan(32, 28, 28, 4, 1639, 28) == dict(path=tc, chunk_tokens=1920, n_chunks=1, passes=1, group_sums=1)
+    # units that overfill the wave take no passes
+    assert plan(2, 32, 32, 8, 3279, 32)["passes"] == 1
+    # the CUDA-core kernel (fp32, d = 64): split-K, no passes, logits
+    r = plan(1, 2, 4, 2, 100, 2, dtype=lib.IKV_F32, d=64)
+    assert r["path"] == cc and r["passes"] == 1 and r["group_sums"] == 0 and r["n_chunks"] * r["chunk_tokens"] >= 100
+    for bad in (0, 33):
+        with pytest.raises(lib.IKVError):
+            plan(1, 32, 32, 8, 3279, bad)
+    with pytest.raises(lib.IKVError):
+        plan(1, 32, 32, 8, 3279, 32, sms=-1)
+
+
 def test_product_package_does_not_reference_the_oracle():
     """The CUDA path and its binding never import or link the CPU oracle."""
     pkg = os.path.join(ROOT, "paper_2609_03515_gb300")
