@@ -350,7 +350,7 @@ def split_step(c, p, cache, t, q, kn, vn, out, ws, stream, foreign=None):
 
 
 def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, sample_clocks: bool,
-                   mh: int = 0, scorer: int = 0, per_layer: str = "", evict: int = 0):
+                   mh: int = 0, scorer: int = 0, per_layer: str = "", evict: int = 0, agg: int = 0):
     """The same schedule with each steady-state step replayed from a captured CUDA graph.
 
     After the eager warm-up (decode step 1 evicts ~90% of the prefill, later steps hold
@@ -367,7 +367,7 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
 
     reset(c, w, u_dev)
     p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh, scorer=scorer,
-                 evict_mode=evict)
+                 evict_mode=evict, agg_mode=agg)
     m_state = c.utility(evict)
     budgets = w.budgets()
     assert all(L0 >= B for L0, B in zip(w.prefill, budgets)), "graph replay assumes every sequence at its budget"
@@ -660,31 +660,34 @@ def run_ours(args):
         sf_w = w.with_(refresh_period=1, score_free=True)
         att, vnm, ent = ikv.IKV_SCORE_ATTENTION, ikv.IKV_SCORE_VNORM, ikv.IKV_SCORE_ENTROPY
         stable, layer = ikv.IKV_COMPACT_STABLE, ikv.IKV_EVICT_LAYER
-        variants = (("full", full_w, compact_mode, mh, att, 0),
-                    ("lazy4", lazy_w, compact_mode, mh, att, 0),
-                    ("score_free", sf_w, compact_mode, mh, att, 0),
-                    ("full_vnorm", full_w, compact_mode, mh, vnm, 0),
-                    ("full_entropy", full_w, compact_mode, mh, ent, 0),
-                    ("full_every_step", full_w, compact_mode, 0, att, 0),
-                    ("lazy4_every_step", lazy_w, compact_mode, 0, att, 0),
-                    ("score_free_every_step", sf_w, compact_mode, 0, att, 0),
-                    ("full_stable_left", full_w, stable, 0, att, 0),
-                    ("full_holefill", full_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, 0),
-                    ("lazy4_holefill", lazy_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, 0),
-                    ("score_free_holefill", sf_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, 0),
-                    ("full_layer_evict", full_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, layer),
-                    ("lazy4_layer_evict", lazy_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, layer),
-                    ("full_layer_evict_stable", full_w, stable, 0, att, layer))
-        for name, ww, cm, vmh, sc, ev in variants:
-            if name == head_sched and cm == compact_mode and vmh == mh and sc == att and ev == 0:
+        ema, cum, single = ikv.IKV_AGG_EMA, ikv.IKV_AGG_CUMULATIVE, ikv.IKV_AGG_SINGLE_STEP
+        variants = (("full", full_w, compact_mode, mh, att, 0, ema),
+                    ("lazy4", lazy_w, compact_mode, mh, att, 0, ema),
+                    ("score_free", sf_w, compact_mode, mh, att, 0, ema),
+                    ("full_vnorm", full_w, compact_mode, mh, vnm, 0, ema),
+                    ("full_entropy", full_w, compact_mode, mh, ent, 0, ema),
+                    ("full_cumulative", full_w, compact_mode, mh, att, 0, cum),
+                    ("full_single_step", full_w, compact_mode, mh, att, 0, single),
+                    ("full_every_step", full_w, compact_mode, 0, att, 0, ema),
+                    ("lazy4_every_step", lazy_w, compact_mode, 0, att, 0, ema),
+                    ("score_free_every_step", sf_w, compact_mode, 0, att, 0, ema),
+                    ("full_stable_left", full_w, stable, 0, att, 0, ema),
+                    ("full_holefill", full_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, 0, ema),
+                    ("lazy4_holefill", lazy_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, 0, ema),
+                    ("score_free_holefill", sf_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, 0, ema),
+                    ("full_layer_evict", full_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, layer, ema),
+                    ("lazy4_layer_evict", lazy_w, ikv.IKV_COMPACT_HOLEFILL, 0, att, layer, ema),
+                    ("full_layer_evict_stable", full_w, stable, 0, att, layer, ema))
+        for name, ww, cm, vmh, sc, ev, ag in variants:
+            if name == head_sched and cm == compact_mode and vmh == mh and sc == att and ev == 0 and ag == ema:
                 modes[name] = full           # the headline run is this mode
                 continue
             modes[name] = run_mode_graph(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, dist, False, vmh, sc,
-                                         evict=ev)
+                                         evict=ev, agg=ag)
         if args.mode_kernels:
-            for name, ww, cm, vmh, sc, ev in variants:
-                if ev:
-                    continue  # per-kernel events time the step-end eviction path only
+            for name, ww, cm, vmh, sc, ev, ag in variants:
+                if ev or ag != ema:
+                    continue  # per-kernel events time the step-end EMA eviction path only
                 mode_kernels[name] = run_mode(args, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, cm, True, dist,
                                               vmh, sc)["kernel_ms"]
     trace = None
@@ -769,7 +772,9 @@ def run_ours(args):
             line["mode_kernel_ms_per_step"] = mode_kernels
         line["modes_note"] = ("full / lazy4 / score_free: refresh every step / every 4th step (Eq. 6) / step 1 "
                               "only, same inputs and compaction as the headline; full_vnorm / full_entropy: the "
-                              "VNorm and entropy-weighted scorers under full refresh; *_every_step: the same "
+                              "VNorm and entropy-weighted scorers under full refresh; full_cumulative / "
+                              "full_single_step: the Eq. 3 and Eq. 2 aggregation rules in place of the EMA, full "
+                              "refresh; *_every_step: the same "
                               "compaction run on every eviction (max_holes 0); full_stable_left: stable "
                               "compaction that always shifts the suffix left, every step; *_holefill: hole-fill "
                               "compaction every step (same kept sets, survivors not kept in order); "
