@@ -284,6 +284,42 @@ def test_attend_plan_query(lib):
         plan(1, 32, 32, 8, 3279, 32, sms=-1)
 
 
+def test_attend_plan_properties(lib):
+    """For random shapes and lengths the plan covers every slot (plus a start offset's
+    slack on the tensor-core kernel), keeps chunks within TMEM and the partial buffers,
+    gives a CTA either one chunk or all of its unit's, and hands over group sums only
+    when every unit is one chunk."""
+    import random
+
+    rng = random.Random(7)
+    for _ in range(400):
+        G = rng.choice([1, 2, 4, 7, 8])
+        Hkv = rng.choice([1, 2, 4, 8])
+        layers = rng.randint(1, 80)
+        batch = rng.randint(1, 64)
+        max_len = rng.randint(1, 200000)
+        ps = rng.choice([16, 64, 128, 256])
+        sms = rng.choice([1, 8, 148, 152, 160])
+        n_layers = rng.choice([1, layers])
+        pages = (max_len + ps) // ps + 1
+        shp = _shape(lib, batch=batch, layers=layers, q_heads=G * Hkv, kv_heads=Hkv, head_dim=128, dtype=lib.IKV_BF16)
+        cch = _cache(lib, num_pages=min(batch * pages, 1 << 20), page_size=ps, max_pages=pages, max_len=max_len)
+        r = lib.ikv_attend_plan(shp, cch, n_layers, sms)
+        slack = 127 if r["path"] == lib.IKV_PATH_TENSOR_CORE else 0
+        assert r["n_chunks"] * r["chunk_tokens"] >= max_len + slack, r
+        assert 1 <= r["n_chunks"] <= 128, r
+        assert r["passes"] in (1, r["n_chunks"]), r
+        if r["path"] == lib.IKV_PATH_TENSOR_CORE:
+            assert r["chunk_tokens"] % 128 == 0 and r["chunk_tokens"] <= 15 * 128, r
+            units = batch * n_layers * Hkv
+            if r["passes"] > 1:                      # one CTA per unit, one wave of two per SM
+                assert 4 * units >= 3 * 2 * sms and units <= 2 * sms, (r, units)
+        else:
+            assert r["passes"] == 1 and r["group_sums"] == 0, r
+        if r["group_sums"]:
+            assert r["n_chunks"] == 1, r
+
+
 def test_product_package_does_not_reference_the_oracle():
     """The CUDA path and its binding never import or link the CPU oracle."""
     pkg = os.path.join(ROOT, "paper_2609_03515_gb300")
