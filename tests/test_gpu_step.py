@@ -121,7 +121,8 @@ def test_multi_pass_trajectories():
     """256 (sequence, layer, kv head) units of 16-31 tiles: the units nearly fill one wave of
     resident CTAs, so each CTA takes its unit's 15-tile chunks as passes, merged in registers.
     A 90% budget keeps the units long on every step; ragged lengths, deferred compaction
-    (dead slots inside the passes), the KV-head granularity and the VNorm scorer."""
+    (dead slots inside the passes), the KV-head granularity and the VNorm scorer; and the
+    split step, whose per-layer launches are multi-pass and store the new rows themselves."""
     rng = np.random.default_rng(41)
     prefill = [int(x) for x in rng.integers(1900, 3800, size=16)]
     w = small_llama(batch=16, layers=2, prefill=prefill, steps=4, budget_frac=0.9)
@@ -129,6 +130,13 @@ def test_multi_pass_trajectories():
     _assert(run_lockstep(w, max_holes=64, compact_mode=ikv.IKV_COMPACT_STABLE_SHORT), 2e-2)
     _assert(run_lockstep(w.with_(steps=3), gran=ikv.IKV_GRAN_KVHEAD), 2e-2)
     _assert(run_lockstep(w.with_(steps=3), scorer=ikv.IKV_SCORE_VNORM), 2e-2)
+    # the split step: each layer call is itself a multi-pass launch (32 sequences x 8 KV
+    # heads = 256 units of 16-31 tiles) whose CTAs also store the layer's new rows
+    w32 = small_llama(batch=32, layers=2, prefill=[int(x) for x in rng.integers(1900, 3800, size=32)], steps=3,
+                      budget_frac=0.9)
+    _assert(run_lockstep(w32, per_layer=True), 2e-2)
+    _assert(run_lockstep(w32, per_layer=True, max_holes=64, compact_mode=ikv.IKV_COMPACT_STABLE_SHORT,
+                         scorer=ikv.IKV_SCORE_VNORM), 2e-2)
 
 
 def test_cumulative_and_single_step_aggregation():
