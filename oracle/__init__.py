@@ -364,6 +364,108 @@ def decode_step(st: SeqState, t: int, q_t: np.ndarray, k_new: np.ndarray, v_new:
 
 
 # --------------------------------------------------------------------------
+# The same step for a sequence whose K/V rows are not held (workload sizes)
+# --------------------------------------------------------------------------
+@dataclass
+class StreamState:
+    """One sequence's eviction state without its cache: for every utility row r, the
+    original token positions held, in slot order (``pos[r]``), and their utilities
+    (``m[r]``).  A token's K/V rows never change (Sec. 3: eviction only removes tokens),
+    so a step fetches the rows it needs by position instead of keeping them."""
+
+    pos: np.ndarray
+    m: np.ndarray
+    budget: int
+    next_pos: int
+    layers: int
+    kv_heads: int
+    granularity: int = GRAN_SEQ
+    raw: Optional[np.ndarray] = None
+
+    @property
+    def length(self) -> int:
+        return self.m.shape[1]
+
+
+def stream_prefill_state(L0: int, budget: int, layers: int, kv_heads: int,
+                         granularity: int = GRAN_SEQ) -> StreamState:
+    """State after prefill: positions 0..L0-1 in order, m_0 = 0 (Appendix "Momentum initialization")."""
+    R = 1 if granularity == GRAN_SEQ else kv_heads
+    return StreamState(pos=np.tile(np.arange(L0, dtype=np.int64), (R, 1)), m=np.zeros((R, L0)), budget=budget,
+                       next_pos=L0, layers=layers, kv_heads=kv_heads, granularity=granularity)
+
+
+def decode_step_streaming(st: StreamState, t: int, q_t: np.ndarray, kv_rows, p: Params,
+                          keep_override=None) -> np.ndarray:
+    """One decode step t (1-based) of one sequence, as ``decode_step``, with the cached
+    rows fetched by position: ``kv_rows(l, g, positions)`` returns (K, V), each
+    [len(positions), d], the rows of layer l / KV head g at those original positions
+    (the appended token's position included).
+
+    Steps in the paper's order: (1) append the new token at the end of every row, state 0
+    on refresh steps (reading R3) or the mean of the row's existing states (Appendix "New
+    token insertion"); (2) every layer's last-query attention over the row's tokens and, on
+    refresh steps of an eligible layer, its Eq. 1 score (or the VNorm / entropy-weighted
+    score) folded into the state in ascending layer order (Eq. 2-4, Appendix "Layer
+    scoring"); (3) if the row holds more than B tokens, keep the B highest utilities (ties
+    to the lower slot) in slot order (Sec. 3, R4, R5).
+
+    keep_override(r, m_row, pos_row) may return the kept slots of row r (ascending)
+    instead of the row's own top-B choice; it is called for every row after step (2),
+    with the row's state as the selection sees it (lock-step tests).  Returns the
+    attention outputs [layers][H][d]."""
+    refresh = is_refresh(t, p.refresh_period, p.score_free)
+    st.raw = None
+    R = st.m.shape[0]
+    # (1) append
+    init = np.array([new_token_state(st.m[r], refresh, p.refresh_init) for r in range(R)])
+    st.m = np.concatenate([st.m, init[:, None]], axis=1)
+    st.pos = np.concatenate([st.pos, np.full((R, 1), st.next_pos, np.int64)], axis=1)
+    st.next_pos += 1
+    # (2) attention of every layer; the score and the layer-sequential update on refresh steps
+    outs = []
+    for l in range(st.layers):
+        H = q_t[l].shape[0]
+        group = H // st.kv_heads
+        if st.granularity == GRAN_SEQ:
+            rows = [kv_rows(l, g, st.pos[0]) for g in range(st.kv_heads)]
+            K_l = [np.asarray(k, np.float64) for k, _ in rows]
+            V_l = [np.asarray(v, np.float64) for _, v in rows]
+            a, o = last_query_attention(q_t[l], K_l, V_l)
+        else:
+            # reading R1: KV head g holds its own tokens; its query group reads them
+            a_parts, o_parts, V_l = [], [], []
+            for g in range(st.kv_heads):
+                k, v = kv_rows(l, g, st.pos[g])
+                V_l.append(np.asarray(v, np.float64))
+                ag, og = last_query_attention(q_t[l][g * group:(g + 1) * group], [np.asarray(k, np.float64)],
+                                              [V_l[g]])
+                a_parts.append(ag)
+                o_parts.append(og)
+            a, o = np.vstack(a_parts), np.vstack(o_parts)
+        outs.append(o)
+        eligible = p.layer_mask is None or p.layer_mask[l]
+        if refresh and eligible:
+            if p.scorer == "vnorm":
+                s = vnorm_score(a, V_l, st.granularity, st.kv_heads)
+            else:
+                s = pooled_score(a, st.granularity, st.kv_heads)
+            if p.scorer == "entropy":
+                s = s * np.array([[entropy_weight(row)] for row in s])
+            st.m = aggregate(st.m, s, p)
+            st.raw = s
+    # (3) eviction down to the budget, survivors in slot order
+    keeps = []
+    for r in range(R):
+        keep = None if keep_override is None else keep_override(r, st.m[r].copy(), st.pos[r].copy())
+        keeps.append(select_keep(st.m[r], st.budget) if keep is None else np.asarray(keep, np.int64))
+    if st.length > st.budget or keep_override is not None:
+        st.m = np.stack([st.m[r][keeps[r]] for r in range(R)])
+        st.pos = np.stack([st.pos[r][keeps[r]] for r in range(R)])
+    return np.stack(outs)
+
+
+# --------------------------------------------------------------------------
 # Per-layer immediate eviction (reading R10)
 # --------------------------------------------------------------------------
 @dataclass
@@ -456,6 +558,78 @@ def decode_step_layerwise(st: LayerwiseState, t: int, q_t: np.ndarray, k_new: np
         for g in range(st.kv_heads):
             st.K[l][g] = st.K[l][g][keep]
             st.V[l][g] = st.V[l][g][keep]
+    return np.stack(outs), traces
+
+
+@dataclass
+class LayerwiseStreamState:
+    """Per-layer eviction state of one sequence without its cache: the positions layer l
+    holds, in slot order (``pos[l]``), and the state of every position appended so far
+    (``m[p]``).  Rows are fetched by position when a step needs them."""
+
+    pos: List[np.ndarray]
+    m: np.ndarray
+    budget: int
+    next_pos: int
+    kv_heads: int
+
+    @property
+    def layers(self) -> int:
+        return len(self.pos)
+
+    def live(self) -> np.ndarray:
+        return np.unique(np.concatenate(self.pos))
+
+
+def layerwise_stream_prefill_state(L0: int, budget: int, layers: int, kv_heads: int) -> LayerwiseStreamState:
+    return LayerwiseStreamState(pos=[np.arange(L0, dtype=np.int64) for _ in range(layers)], m=np.zeros(L0),
+                                budget=budget, next_pos=L0, kv_heads=kv_heads)
+
+
+def decode_step_layerwise_streaming(st: LayerwiseStreamState, t: int, q_t: np.ndarray, kv_rows, p: Params,
+                                    keep_override=None):
+    """``decode_step_layerwise`` (reading R10) with every layer's rows fetched by position:
+    ``kv_rows(l, g, positions)`` -> (K, V), each [len(positions), d].
+
+    (1) every layer appends the new token; its state is 0 on refresh steps (R3), else the
+    mean over the live positions; (2) layer by layer: attention over the layer's own
+    tokens; on refresh steps of an eligible layer the Eq. 1 score (0 at live positions the
+    layer does not hold) updates every live position by Eq. 4; then the layer keeps the B
+    highest states among its tokens (ties to the lower slot), in slot order.
+    keep_override(l, LayerTrace) as in ``decode_step_layerwise``.
+    Returns (attention outputs [layers][H][d], [LayerTrace per layer])."""
+    refresh = is_refresh(t, p.refresh_period, p.score_free)
+    live = st.live()
+    if refresh and p.refresh_init == "zero":
+        init = 0.0
+    else:
+        init = float(np.mean(st.m[live])) if live.size else 0.0
+    st.m = np.append(st.m, init)
+    for l in range(st.layers):
+        st.pos[l] = np.append(st.pos[l], st.next_pos)
+    st.next_pos += 1
+    outs, traces = [], []
+    for l in range(st.layers):
+        rows = [kv_rows(l, g, st.pos[l]) for g in range(st.kv_heads)]
+        a, o = last_query_attention(q_t[l], [np.asarray(k, np.float64) for k, _ in rows],
+                                    [np.asarray(v, np.float64) for _, v in rows])
+        outs.append(o)
+        eligible = p.layer_mask is None or p.layer_mask[l]
+        if refresh and eligible:
+            s_pos = np.zeros_like(st.m)
+            s_pos[st.pos[l]] = pooled_score(a, GRAN_SEQ, st.kv_heads)[0]
+            live = st.live()
+            st.m[live] = ema_update(st.m[live], s_pos[live], p.alpha)
+        m_l = st.m[st.pos[l]]
+        keep = select_keep(m_l, st.budget)
+        tr = LayerTrace(pos=st.pos[l].copy(), m=m_l.copy(), kept=st.pos[l][keep])
+        if keep_override is not None:
+            kp = keep_override(l, tr)
+            if kp is not None:
+                keep = np.searchsorted(st.pos[l], np.sort(np.asarray(kp, np.int64)))
+                tr.kept = st.pos[l][keep]
+        traces.append(tr)
+        st.pos[l] = st.pos[l][keep]
     return np.stack(outs), traces
 
 

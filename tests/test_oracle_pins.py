@@ -725,3 +725,153 @@ def test_rank_trace_raw_is_last_eligible_layer_score():
     O.decode_step(a, 1, q[0], kn[0], vn[0], O.Params(alpha=0.8, layer_mask=[True, True, False]))
     O.decode_step(b, 1, q[0], kn[0], vn[0], O.Params(aggregation="single", layer_mask=[True, True, False]))
     np.testing.assert_array_equal(a.raw, b.m)
+
+
+# ------------------------------------- the step with rows fetched by position
+def _position_table(rng, layers, kv, n_pos, d, heavy=True):
+    """K/V rows of every (layer, KV head, original position): the cache a sequence would
+    hold, addressed by position."""
+    K = rng.standard_normal((layers, kv, n_pos, d))
+    V = rng.standard_normal((layers, kv, n_pos, d))
+    if heavy:
+        K[:, :, ::7] *= 3.0
+    return K, V
+
+
+_STREAM_CASES = [
+    dict(),                                                     # full refresh, Eq. 4
+    dict(refresh_period=3),                                     # Lazy-3 (Eq. 6)
+    dict(score_free=True),                                      # Score-Free
+    dict(refresh_init="mean", layer_mask=[True, False, True]),  # mean init, sparse layer mask
+    dict(gran=O.GRAN_KVHEAD, refresh_period=2),                 # one row per KV head
+    dict(scorer="vnorm"),
+    dict(scorer="entropy", refresh_period=2),
+    dict(aggregation="cumulative"),
+    dict(aggregation="single"),
+]
+
+
+@pytest.mark.parametrize("case", _STREAM_CASES, ids=[str(i) for i in range(len(_STREAM_CASES))])
+def test_streaming_step_equals_cache_holding_step(case):
+    """decode_step_streaming keeps only (positions, utilities) and fetches rows by position;
+    on the same sequence it gives decode_step's outputs, utilities and kept positions bit
+    for bit over a run that evicts every step (positions are the rows' identity, so the
+    position bookkeeping is what this pins)."""
+    case = dict(case)
+    gran = case.pop("gran", O.GRAN_SEQ)
+    rng = np.random.default_rng(31)
+    layers, kv, H, d, L0, B, T = 3, 2, 4, 8, 30, 10, 9
+    Kt, Vt = _position_table(rng, layers, kv, L0 + T, d)
+    held = O.prefill_state([[Kt[l, g, :L0] for g in range(kv)] for l in range(layers)],
+                           [[Vt[l, g, :L0] for g in range(kv)] for l in range(layers)], B, gran)
+    st = O.stream_prefill_state(L0, B, layers, kv, gran)
+    p = O.Params(alpha=0.8, **case)
+    q = rng.standard_normal((T, layers, H, d))
+    fetched = []
+
+    def rows(l, g, positions):
+        fetched.append(len(positions))
+        return Kt[l, g, positions], Vt[l, g, positions]
+
+    for t in range(1, T + 1):
+        newp = L0 + t - 1
+        o_held = O.decode_step(held, t, q[t - 1], Kt[:, :, newp], Vt[:, :, newp], p)
+        o_st = O.decode_step_streaming(st, t, q[t - 1], rows, p)
+        assert np.array_equal(o_held, o_st), t
+        assert np.array_equal(held.m, st.m), t
+        assert np.array_equal(held.pos, st.pos), t
+        assert st.length == min(L0 + t, B)
+    assert min(fetched) == B + 1  # steady state: the budget plus the new token
+
+
+def test_streaming_step_adopts_an_override_like_evict():
+    """keep_override replaces the row's own choice exactly as evict(keep_override=...) does."""
+    rng = np.random.default_rng(32)
+    layers, kv, H, d, L0, B, T = 2, 2, 4, 8, 20, 6, 4
+    Kt, Vt = _position_table(rng, layers, kv, L0 + T, d)
+    held = O.prefill_state([[Kt[l, g, :L0] for g in range(kv)] for l in range(layers)],
+                           [[Vt[l, g, :L0] for g in range(kv)] for l in range(layers)], B)
+    st = O.stream_prefill_state(L0, B, layers, kv)
+    p = O.Params(alpha=0.5)
+    q = rng.standard_normal((T, layers, H, d))
+    seen = []
+
+    def pick(r, m_row, pos_row):  # any B slots: here the oldest ones
+        seen.append((m_row.copy(), pos_row.copy()))
+        return np.arange(min(B, len(m_row)))
+
+    for t in range(1, T + 1):
+        newp = L0 + t - 1
+        O.append_token(held, Kt[:, :, newp], Vt[:, :, newp], O.is_refresh(t, 1, False), p)
+        o_held = O.attend_and_score(held, q[t - 1], True, p)
+        m_before = held.m[0].copy()
+        O.evict(held, keep_override=[np.arange(min(B, held.length))])
+        o_st = O.decode_step_streaming(st, t, q[t - 1], lambda l, g, ps: (Kt[l, g, ps], Vt[l, g, ps]), p,
+                                       keep_override=pick)
+        assert np.array_equal(o_held, o_st)
+        assert np.array_equal(seen[-1][0], m_before)       # the override sees the state the selection sees
+        assert np.array_equal(held.pos, st.pos) and np.array_equal(held.m, st.m)
+    assert st.pos[0].tolist() == list(range(B))
+
+
+def test_streaming_step_with_generator_rows_by_position():
+    """The workload generator's rows at arbitrary positions are the rows of its prefill
+    block and of its appended tokens, so the streaming oracle driven by kv_rows follows the
+    cache-holding oracle on a generated (bf16) workload."""
+    import gen
+
+    w = gen.Workload("pin", 2, 2, 8, 2, 64, [90, 70], 5, dtype=gen.BF16, seed=12, page_size=16)
+    u = w.u_table()
+    qs = w.queries(1, w.steps + 1, u)
+    q64 = gen.bf16_to_f32(qs).astype(np.float64)
+    p = O.Params(alpha=0.9, refresh_period=2)
+    B = w.budgets()
+    for b in range(w.batch):
+        K, V = [], []
+        for l in range(w.layers):
+            k, v = w.kv_block(b, l, 0, w.prefill[b], u)
+            K.append([k[g].astype(np.float64) for g in range(w.kv_heads)])
+            V.append([v[g].astype(np.float64) for g in range(w.kv_heads)])
+        held = O.prefill_state(K, V, B[b])
+        st = O.stream_prefill_state(w.prefill[b], B[b], w.layers, w.kv_heads)
+
+        def rows(l, g, positions, b=b):
+            k, v = w.kv_rows(b, l, positions, u)
+            return k[g], v[g]
+
+        for t in range(1, w.steps + 1):
+            kn, vn = w.new_tokens(t, u)
+            o_held = O.decode_step(held, t, q64[t - 1][:, b], kn[:, b], vn[:, b], p)
+            o_st = O.decode_step_streaming(st, t, q64[t - 1][:, b], rows, p)
+            assert np.array_equal(o_held, o_st), (b, t)
+            assert np.array_equal(held.m, st.m) and np.array_equal(held.pos, st.pos), (b, t)
+
+
+@pytest.mark.parametrize("case", [dict(), dict(refresh_period=3), dict(score_free=True),
+                                  dict(refresh_init="mean", layer_mask=[False, True, True, False])],
+                         ids=["full", "lazy3", "score_free", "mean_sparse"])
+def test_layerwise_streaming_equals_cache_holding_step(case):
+    """decode_step_layerwise_streaming (reading R10 with rows fetched by position) gives
+    decode_step_layerwise's outputs, per-layer kept positions, states and traces bit for bit."""
+    rng = np.random.default_rng(33)
+    layers, kv, H, d, L0, B, T = 4, 2, 4, 8, 26, 8, 8
+    Kt, Vt = _position_table(rng, layers, kv, L0 + T, d)
+    held = O.layerwise_prefill_state([[Kt[l, g, :L0] for g in range(kv)] for l in range(layers)],
+                                     [[Vt[l, g, :L0] for g in range(kv)] for l in range(layers)], B)
+    st = O.layerwise_stream_prefill_state(L0, B, layers, kv)
+    p = O.Params(alpha=0.7, **case)
+    q = rng.standard_normal((T, layers, H, d))
+    diverged = False
+    for t in range(1, T + 1):
+        newp = L0 + t - 1
+        o_held, tr_h = O.decode_step_layerwise(held, t, q[t - 1], Kt[:, :, newp], Vt[:, :, newp], p)
+        o_st, tr_s = O.decode_step_layerwise_streaming(st, t, q[t - 1],
+                                                       lambda l, g, ps: (Kt[l, g, ps], Vt[l, g, ps]), p)
+        assert np.array_equal(o_held, o_st), t
+        assert np.array_equal(held.m, st.m), t
+        for l in range(layers):
+            assert np.array_equal(held.pos[l], st.pos[l]), (t, l)
+            assert np.array_equal(tr_h[l].m, tr_s[l].m) and np.array_equal(tr_h[l].kept, tr_s[l].kept)
+        diverged |= any(not np.array_equal(st.pos[0], st.pos[l]) for l in range(1, layers))
+    if not case:
+        assert diverged  # the layers' sets do differ, so every layer's bookkeeping is exercised
