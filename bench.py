@@ -236,6 +236,34 @@ class ClockSampler:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
+def device_inputs(w, u, u_dev, T: int, dev):
+    """Every decode step's inputs, resident on the device: q [T][layers][batch][q_heads][d]
+    from the host generator, k_new / v_new [T][layers][batch][kv_heads][d] from the device
+    generator (bit-identical to the host's)."""
+    import numpy as np
+    import torch
+
+    import gen
+
+    qs_h = w.queries(1, T + 1, u)
+    tdt = torch.bfloat16 if w.dtype == gen.BF16 else torch.float32
+    if w.dtype == gen.BF16:
+        qs_t = torch.from_numpy(qs_h.view(np.int16)).view(torch.bfloat16)
+    else:
+        qs_t = torch.from_numpy(qs_h)
+    qs_dev = qs_t.to(dev)
+    kn_dev = torch.empty((T, w.layers, w.batch, w.kv_heads, w.head_dim), dtype=tdt, device=dev)
+    vn_dev = torch.empty_like(kn_dev)
+    sp = w.spec()
+    L0 = torch.tensor(w.prefill, dtype=torch.int32, device=dev)
+    rc = gen.cuda_lib().ikvgen_fill_tokens_cuda(ctypes.byref(sp), u_dev.data_ptr(), L0.data_ptr(), 1, T + 1, w.dtype,
+                                                kn_dev.data_ptr(), vn_dev.data_ptr(),
+                                                torch.cuda.current_stream().cuda_stream)
+    assert rc == 0
+    torch.cuda.synchronize()
+    return qs_dev, kn_dev, vn_dev
+
+
 def setup(w, device, compact_mode, steps: int = 0):
     import numpy as np
     import torch
@@ -350,7 +378,8 @@ def split_step(c, p, cache, t, q, kn, vn, out, ws, stream, foreign=None):
 
 
 def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, sample_clocks: bool,
-                   mh: int = 0, scorer: int = 0, per_layer: str = "", evict: int = 0, agg: int = 0):
+                   mh: int = 0, scorer: int = 0, per_layer: str = "", evict: int = 0, agg: int = 0,
+                   after_step=None):
     """The same schedule with each steady-state step replayed from a captured CUDA graph.
 
     After the eager warm-up (decode step 1 evicts ~90% of the prefill, later steps hold
@@ -360,7 +389,9 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     per_layer "split": the step as ikv_step_begin / one ikv_step_layer per layer /
     ikv_step_end; "foreign": the same, with the layer's q, k_new and v_new first copied
     by PyTorch kernels into per-layer buffers (standing in for the projection that a
-    model runs before each layer's attention)."""
+    model runs before each layer's attention).
+    after_step(t, out): called after each warm-up step and each replayed step, once the
+    device is idle (parity tests of this exact path); None in a timed run."""
     import torch
 
     from paper_2609_03515_gb300 import ikv, step_lengths
@@ -398,6 +429,9 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     for t in range(1, W + 1):
         one(c.cache(max(lens)), t)
         lens, live = step_lengths(lens, live, budgets, mh)
+        if after_step is not None:
+            torch.cuda.synchronize()
+            after_step(t, out)
     torch.cuda.synchronize()
     # the graphs' max_len bounds every later step: the budget plus the dead slots
     # deferred compaction may hold; the warm-up left the workspace's counters zero
@@ -421,9 +455,12 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     clocks = ClockSampler(torch.cuda.current_device()) if sample_clocks else None
     launches = 0
     start.record(stream)
-    for g, nl in graphs:
+    for i, (g, nl) in enumerate(graphs):
         g.replay()
         launches += nl
+        if after_step is not None:
+            torch.cuda.synchronize()
+            after_step(W + 1 + i, out)
     stop.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(start.elapsed_time(stop), dist, dev)
@@ -614,23 +651,8 @@ def run_ours(args):
     u_dev = torch.from_numpy(u).to(dev)
     c = setup(w, dev, compact_mode, total_steps)
     ws = c.step_workspace()
-    T = total_steps
-    qs_h = w.queries(1, T + 1, u)
-    tdt = c.torch_dtype
-    if w.dtype == gen.BF16:
-        qs_t = torch.from_numpy(qs_h.view(np.int16)).view(torch.bfloat16)
-    else:
-        qs_t = torch.from_numpy(qs_h)
-    qs_dev = qs_t.to(dev)
-    kn_dev = torch.empty((T, w.layers, w.batch, w.kv_heads, w.head_dim), dtype=tdt, device=dev)
-    vn_dev = torch.empty_like(kn_dev)
-    sp = w.spec()
-    L0 = torch.tensor(w.prefill, dtype=torch.int32, device=dev)
-    rc = gen.cuda_lib().ikvgen_fill_tokens_cuda(ctypes.byref(sp), u_dev.data_ptr(), L0.data_ptr(), 1, T + 1, w.dtype,
-                                                kn_dev.data_ptr(), vn_dev.data_ptr(),
-                                                torch.cuda.current_stream().cuda_stream)
-    assert rc == 0
-    torch.cuda.synchronize()
+    qs_dev, kn_dev, vn_dev = device_inputs(w, u, u_dev, total_steps, dev)
+    qs_t = qs_dev.cpu()
 
     from paper_2609_03515_gb300 import auto_max_holes
 

@@ -282,7 +282,9 @@ ikv_status ikv_decode_attend_score(const ikv_shape *shape, const ikv_cache *cach
  *  - Shapes whose scratch (ikv_attend_workspace_size) exceeds the array are
  *    rejected with IKV_ERR_WORKSPACE and a message; nothing is launched.
  *  - The first call on a device looks up the array's device address (with
- *    that device current); make that first call before any stream capture.
+ *    that device current) and keeps it for the life of the process; make that
+ *    first call before any stream capture.  After cudaDeviceReset the kept
+ *    address is stale: do not call this entry point again in that process.
  *  - All calls share the one array, which keeps the last call's contents
  *    (nothing in it needs clearing).  Calls whose GPU work overlaps -- other
  *    streams or other host threads on the same device -- race on it; the

@@ -11,7 +11,9 @@
 // The array lives for as long as the library is loaded on a device (every GPU
 // that loads the library holds kStaticScratchBytes of it until the process
 // exits).  Its device address is looked up once per device, with that device
-// current, on the first call made on it.  All calls share the array and it
+// current, on the first call made on it, and kept for the life of the process
+// (a cudaDeviceReset would leave the kept address stale, so the entry point is
+// not for use after one).  All calls share the array and it
 // keeps the last call's contents; the attention path fully writes every
 // scratch word before reading it, so nothing needs clearing between calls.
 // Two calls whose work overlaps on the GPU (different streams, or different

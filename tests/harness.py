@@ -40,19 +40,36 @@ def make_cache(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, page_perm_seed: Op
     return c
 
 
-def fill_host(c: DecodeCache, w: gen.Workload, u: np.ndarray):
-    """Upload host-generated prefill K/V; returns them as [b][l] -> (K[g], V[g]) float64 lists."""
+def fill_prefill(c: DecodeCache, w: gen.Workload, u: np.ndarray):
+    """Write the prefill K/V into the device pools with the device generator and return the
+    host generator's draws of the same rows for the oracle, [b][l] -> (K[g], V[g]) float64
+    (the two halves agree bit for bit: test_generator_bits_host_equals_device)."""
+    fill_device(c, w, torch.from_numpy(u).cuda())
     kv = []
     for b in range(w.batch):
         per_l = []
         for l in range(w.layers):
             k, v = w.kv_block(b, l, 0, w.prefill[b], u)
-            for g in range(w.kv_heads):
-                c.scatter(c.k, b, l, g, torch.from_numpy(k[g]).cuda())
-                c.scatter(c.v, b, l, g, torch.from_numpy(v[g]).cuda())
             per_l.append((k.astype(np.float64), v.astype(np.float64)))
         kv.append(per_l)
     return kv
+
+
+class HostPools:
+    """The K/V pools and the slot map copied to the host once, gathered there (the small
+    lock-step checks launch no indexing kernels this way)."""
+
+    def __init__(self, c: DecodeCache):
+        self.c = c
+        self.k = c.k.cpu().float().numpy()
+        self.v = c.v.cpu().float().numpy()
+        self.bt = c.block_table.cpu().numpy()
+        self.start = c.start.cpu().numpy()
+
+    def rows(self, pool: np.ndarray, b: int, l: int, g: int, n: int) -> np.ndarray:
+        slots = np.arange(n) + int(self.start[b])
+        pages = self.bt[b, slots // self.c.page_size]
+        return pool[l, pages, g, slots % self.c.page_size]
 
 
 def fill_device(c: DecodeCache, w: gen.Workload, u_dev: torch.Tensor) -> None:
@@ -89,12 +106,17 @@ def to_device(x: np.ndarray, w: gen.Workload) -> torch.Tensor:
     return torch.from_numpy(np.ascontiguousarray(x, np.float32)).cuda()
 
 
-def boundary_ok(m_o: np.ndarray, kept_mask: np.ndarray, budget: int, gap: float = GAP):
-    """Retained-set rule against the oracle's utilities m_o (one row)."""
+def boundary_ok(m_o: np.ndarray, kept_mask: np.ndarray, budget: int, gap: float = GAP, relative: bool = False):
+    """Retained-set rule against the oracle's utilities m_o (one row): with theta the
+    oracle's B-th largest utility, every token above theta + gap is kept and every token
+    below theta - gap evicted.  relative: the gap is gap * theta (the stricter rule for
+    utilities far below 1)."""
     L = m_o.shape[0]
     if L <= budget:
         return bool(kept_mask.all()), 0.0
     theta = np.sort(m_o)[::-1][budget - 1]
+    if relative:
+        gap = gap * abs(theta)
     must_keep = m_o > theta + gap
     must_drop = m_o < theta - gap
     ok = bool(np.all(kept_mask[must_keep]) and not np.any(kept_mask[must_drop]) and kept_mask.sum() == budget)
@@ -105,9 +127,11 @@ def boundary_ok(m_o: np.ndarray, kept_mask: np.ndarray, budget: int, gap: float 
 class StepReport:
     t: int
     out_err: float = 0.0
-    m_err: float = 0.0
+    m_err: float = 0.0           # kept utilities, absolute error against the oracle
+    m_rel_err: float = 0.0       # the same, relative (full-size runs)
     kv_err: float = 0.0
-    set_ok: bool = True
+    set_ok: bool = True          # boundary rule, absolute gap
+    rel_set_ok: bool = True      # boundary rule, relative gap (full-size runs)
     strict_set_equal: bool = True
     refresh: bool = True
 
@@ -141,7 +165,7 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
     T = w.steps if steps is None else steps
     u = w.u_table()
     c = make_cache(w, gran, page_perm_seed, value_norms=scorer == ikv.IKV_SCORE_VNORM)
-    kv = fill_host(c, w, u)
+    kv = fill_prefill(c, w, u)
     if c.vnorm is not None:
         ikv.ikv_value_norms(c.shape(), c.cache(max(w.prefill)))
     sts = oracle_states(w, kv, gran)
@@ -173,7 +197,7 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
                     ws, per_layer)
         lens, live = step_lengths(lens, live, budgets, max_holes)
         torch.cuda.synchronize()
-        out_h = out.float().cpu().numpy()
+        out_h = out.cpu().float().numpy()
         ema_h = c.ema.cpu().numpy()
         pos_h = c.pos.cpu().numpy()
         len_h = c.len.cpu().numpy()
@@ -185,6 +209,7 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
             ematop_h = tr.ema_top.cpu().numpy()
         rep = StepReport(t=t, refresh=refresh)
         q64 = as_f64(qs[t - 1], w)
+        hp = HostPools(c) if kv_check_layers else None
         for b, st in enumerate(sts):
             st.raw = None
             O.append_token(st, kn[:, b], vn[:, b], refresh, op)
@@ -237,8 +262,8 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
                 for g in range(w.kv_heads):
                     rr = 0 if R == 1 else g
                     ls = live_slots(pos_h[b * R + rr], int(len_h[b]))
-                    gk = c.gather(c.k, b, l % w.layers, g, int(len_h[b])).float().cpu().numpy()[ls]
-                    gv = c.gather(c.v, b, l % w.layers, g, int(len_h[b])).float().cpu().numpy()[ls]
+                    gk = hp.rows(hp.k, b, l % w.layers, g, int(len_h[b]))[ls]
+                    gv = hp.rows(hp.v, b, l % w.layers, g, int(len_h[b]))[ls]
                     order = np.argsort(np.argsort(pos_h[b * R + rr, ls]))  # gpu live slot -> rank by position
                     ok_rows = st.K[l][g][order]
                     ov_rows = st.V[l][g][order]
@@ -248,85 +273,168 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
     return reports
 
 
-def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1), page_perm_seed: Optional[int] = 7,
-                         compact_mode: int = ikv.IKV_COMPACT_STABLE, max_holes: int = 0, per_layer: bool = False):
-    """Full-size lock-step for a few sequences of a workload (GRAN_SEQ).
+class KVRowsByPosition:
+    """kv_rows(l, g, positions) for the streaming oracle of sequence b: the workload
+    generator's K/V rows at those original positions (exactly the values the device
+    generator wrote into the cache).  Each layer's last answer is memoised, so a step that
+    keeps most positions regenerates only the new ones."""
 
-    The GPU decodes the whole batch at its real size (device-generated prefill, the
-    same launch configuration as the benchmark).  For each sampled sequence the
-    oracle keeps only (original positions, utilities) and, layer by layer,
-    regenerates the cached K/V rows from the seeded generator by position -- so a
-    32k x 32-layer fp64 cache never has to exist at once.  Sequences are independent,
-    so sampling them checks the full-batch run."""
-    T = steps
+    def __init__(self, w: gen.Workload, b: int, u: np.ndarray):
+        self.w, self.b, self.u = w, b, u
+        self.memo = {}
+
+    def __call__(self, l: int, g: int, positions):
+        P = np.asarray(positions, dtype=np.int64)
+        ent = self.memo.get(l)
+        if ent is None or ent[0].shape != P.shape or not np.array_equal(ent[0], P):
+            ent = self._fetch(l, P, ent)
+            self.memo[l] = ent
+        return ent[1][g], ent[2][g]
+
+    def _fetch(self, l, P, old):
+        w = self.w
+        K = np.empty((w.kv_heads, P.shape[0], w.head_dim), np.float32)
+        V = np.empty_like(K)
+        miss = np.ones(P.shape[0], bool)
+        if old is not None and old[0].size:
+            order = np.argsort(old[0], kind="stable")
+            sp = old[0][order]
+            i = np.minimum(np.searchsorted(sp, P), sp.shape[0] - 1)
+            found = sp[i] == P
+            src = order[i[found]]
+            K[:, found] = old[1][:, src]
+            V[:, found] = old[2][:, src]
+            miss = ~found
+        if miss.any():
+            k, v = w.kv_rows(self.b, l, P[miss], self.u)
+            K[:, miss] = k
+            V[:, miss] = v
+        return P.copy(), K, V
+
+
+def rel_err(g: np.ndarray, o: np.ndarray) -> float:
+    """Largest relative error of g against the oracle's o (entries where o is 0 compare absolutely)."""
+    if g.size == 0:
+        return 0.0
+    den = np.where(o != 0, np.abs(o), 1.0)
+    return float(np.max(np.abs(g - o) / den))
+
+
+class SampledOracle:
+    """The streaming oracle (oracle.decode_step_streaming) following a few sequences of a
+    full-size GPU run in lock-step (GRAN_SEQ).  Each sampled sequence keeps only its
+    positions and utilities; its K/V rows are regenerated by position.  Sequences are
+    independent, so sampling them checks the whole batch.  check(t, out) runs after the
+    GPU finished step t and compares, per sampled sequence:
+      - every layer's and head's attention output;
+      - the kept set under the 1e-4 boundary rule and under the relative one (1e-4 theta);
+        whether it equals the oracle's own top-B (strict); the oracle then adopts it;
+      - the kept utilities, absolute and relative error;
+      - the K/V rows of check_layers at the live slots, bit for bit."""
+
+    def __init__(self, w: gen.Workload, c: DecodeCache, seqs, u: np.ndarray, compact_mode: int,
+                 check_layers=(0, -1), refresh_init: int = ikv.IKV_INIT_ZERO):
+        self.w, self.c, self.seqs, self.u = w, c, list(seqs), u
+        self.compact_mode, self.check_layers = compact_mode, check_layers
+        self.op = O.Params(alpha=w.alpha, refresh_period=w.refresh_period, score_free=w.score_free,
+                           refresh_init="zero" if refresh_init == ikv.IKV_INIT_ZERO else "mean")
+        B = w.budgets()
+        self.states = {b: O.stream_prefill_state(w.prefill[b], B[b], w.layers, w.kv_heads) for b in self.seqs}
+        self.rows = {b: KVRowsByPosition(w, b, u) for b in self.seqs}
+        self.reports: List[StepReport] = []
+
+    def check(self, t: int, out: torch.Tensor) -> StepReport:
+        w, c = self.w, self.c
+        torch.cuda.synchronize()
+        rep = StepReport(t=t, refresh=O.is_refresh(t, w.refresh_period, w.score_free))
+        q64 = as_f64(w.queries(t, t + 1, self.u)[0], w)
+        len_h = c.len.cpu().numpy()
+        for b in self.seqs:
+            n_b = int(len_h[b])
+            pos_b = c.pos[b, :n_b].cpu().numpy().astype(np.int64)
+            ema_b = c.ema[b, :n_b].cpu().numpy()
+            ls = live_slots(pos_b, n_b)
+            gpos, gm = pos_b[ls], ema_b[ls]
+            if self.compact_mode in STABLE_MODES:  # survivors keep their order (R5)
+                assert np.all(np.diff(gpos) > 0), (t, b)
+            assert len(set(gpos.tolist())) == len(gpos), (t, b)
+            B = self.states[b].budget
+
+            def adopt(r, m_row, pos_row, rep=rep, gpos=gpos, gm=gm, B=B, b=b):
+                slot_of = {int(pp): i for i, pp in enumerate(pos_row)}
+                assert len(gpos) == min(len(pos_row), B), (t, b, len(gpos), len(pos_row))
+                oslots = np.array([slot_of[int(pp)] for pp in gpos], dtype=np.int64)
+                kept = np.zeros(len(pos_row), bool)
+                kept[oslots] = True
+                ok, _ = boundary_ok(m_row, kept, B)
+                rok, _ = boundary_ok(m_row, kept, B, relative=True)
+                rep.set_ok &= ok
+                rep.rel_set_ok &= rok
+                rep.strict_set_equal &= set(O.select_keep(m_row, B).tolist()) == set(oslots.tolist())
+                rep.m_err = max(rep.m_err, float(np.max(np.abs(gm - m_row[oslots]))) if len(gm) else 0.0)
+                rep.m_rel_err = max(rep.m_rel_err, rel_err(gm, m_row[oslots]))
+                return np.sort(oslots)
+
+            o_out = O.decode_step_streaming(self.states[b], t, q64[:, b], self.rows[b], self.op, keep_override=adopt)
+            out_b = out[:, b].float().cpu().numpy()
+            rep.out_err = max(rep.out_err, float(np.max(np.abs(out_b - o_out))))
+            for l in self.check_layers:
+                lk, lv = w.kv_rows(b, l % w.layers, gpos, self.u)
+                for g in range(w.kv_heads):
+                    gk = c.gather(c.k, b, l % w.layers, g, n_b).float().cpu().numpy()[ls]
+                    gv = c.gather(c.v, b, l % w.layers, g, n_b).float().cpu().numpy()[ls]
+                    rep.kv_err = max(rep.kv_err, float(np.max(np.abs(gk - lk[g]))), float(np.max(np.abs(gv - lv[g]))))
+        self.reports.append(rep)
+        return rep
+
+
+def fullsize_cache(w: gen.Workload, page_perm_seed: Optional[int] = 7, pos_cap: int = 0):
+    """The workload's device cache with its prefill written by the device generator."""
     u = w.u_table()
-    u_dev = torch.from_numpy(u).cuda()
-    c = make_cache(w, ikv.IKV_GRAN_SEQ, page_perm_seed)
-    fill_device(c, w, u_dev)
-    op = O.Params(alpha=w.alpha, refresh_period=w.refresh_period, score_free=w.score_free)
-    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=max_holes)
-    ws = c.step_workspace()
-    qs = w.queries(1, T + 1, u)
-    budgets = w.budgets()
-    lens, live = list(w.prefill), list(w.prefill)
-    out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
+    c = DecodeCache(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.cap,
+                    dtype=ikv.IKV_BF16 if w.dtype == gen.BF16 else ikv.IKV_F32, page_size=w.page_size,
+                    page_perm_seed=page_perm_seed, pos_cap=pos_cap)
+    c.set_prefill(w.prefill, w.budgets())
+    fill_device(c, w, torch.from_numpy(u).cuda())
+    return c, u
+
+
+def device_new_tokens(w: gen.Workload, u: np.ndarray, t: int):
+    """k_new, v_new of decode step t ([layers][batch][kv_heads][d]) from the device generator."""
     sp = w.spec()
+    u_dev = torch.from_numpy(u).cuda()
     L0_dev = torch.tensor(w.prefill, dtype=torch.int32, device="cuda")
     kn = torch.empty((1, w.layers, w.batch, w.kv_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
     vn = torch.empty_like(kn)
-    state = {b: {"pos": np.arange(w.prefill[b], dtype=np.int64), "m": np.zeros(w.prefill[b])} for b in seqs}
-    reports = []
-    for t in range(1, T + 1):
-        assert gen.cuda_lib().ikvgen_fill_tokens_cuda(ctypes.byref(sp), u_dev.data_ptr(), L0_dev.data_ptr(), t, t + 1,
-                                                      w.dtype, kn.data_ptr(), vn.data_ptr(),
-                                                      torch.cuda.current_stream().cuda_stream) == 0
-        decode_step(c, p, c.cache(max(lens)), t, to_device(qs[t - 1], w), kn[0], vn[0], out, ws, per_layer)
+    assert gen.cuda_lib().ikvgen_fill_tokens_cuda(ctypes.byref(sp), u_dev.data_ptr(), L0_dev.data_ptr(), t, t + 1,
+                                                  w.dtype, kn.data_ptr(), vn.data_ptr(),
+                                                  torch.cuda.current_stream().cuda_stream) == 0
+    return kn[0], vn[0]
+
+
+def run_fullsize_sampled(w: gen.Workload, seqs, steps: int, check_layers=(0, -1), page_perm_seed: Optional[int] = 7,
+                         compact_mode: int = ikv.IKV_COMPACT_STABLE, max_holes: int = 0, per_layer: bool = False):
+    """Full-size lock-step for a few sequences of a workload (GRAN_SEQ), eager calls.
+
+    The GPU decodes the whole batch at its real size (device-generated prefill, the same
+    launch configuration as the benchmark); SampledOracle follows the sampled sequences."""
+    c, u = fullsize_cache(w, page_perm_seed)
+    chk = SampledOracle(w, c, seqs, u, compact_mode, check_layers)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=max_holes)
+    ws = c.step_workspace()
+    qs = w.queries(1, steps + 1, u)
+    budgets = w.budgets()
+    lens, live = list(w.prefill), list(w.prefill)
+    out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
+    for t in range(1, steps + 1):
+        kn, vn = device_new_tokens(w, u, t)
+        decode_step(c, p, c.cache(max(lens)), t, to_device(qs[t - 1], w), kn, vn, out, ws, per_layer)
         lens, live = step_lengths(lens, live, budgets, max_holes)
         torch.cuda.synchronize()
-        refresh = O.is_refresh(t, w.refresh_period, w.score_free)
-        rep = StepReport(t=t, refresh=refresh)
-        q64 = as_f64(qs[t - 1], w)
-        len_h = c.len.cpu().numpy()
-        for b in seqs:
-            st = state[b]
-            # append (Appendix "New token insertion"; 0 on refresh steps)
-            st["m"] = np.append(st["m"], O.new_token_state(st["m"], refresh, op.refresh_init))
-            st["pos"] = np.append(st["pos"], w.prefill[b] + t - 1)
-            out_b = out[:, b].float().cpu().numpy()
-            for l in range(w.layers):
-                k, v = w.kv_rows(b, l, st["pos"], u)
-                a_, o_ = O.last_query_attention(q64[l, b], [x.astype(np.float64) for x in k],
-                                                [x.astype(np.float64) for x in v])
-                rep.out_err = max(rep.out_err, float(np.max(np.abs(out_b[l] - o_))))
-                if refresh:
-                    st["m"] = O.ema_update(st["m"], O.pooled_score(a_, O.GRAN_SEQ, w.kv_heads)[0], op.alpha)
-            assert len_h[b] == lens[b]
-            ls = live_slots(c.pos[b, :int(len_h[b])].cpu().numpy(), int(len_h[b]))
-            n = len(ls)
-            assert n == min(st["pos"].shape[0], budgets[b])
-            gpos = c.pos[b, :int(len_h[b])].cpu().numpy().astype(np.int64)[ls]
-            gm = c.ema[b, :int(len_h[b])].cpu().numpy()[ls]
-            if compact_mode in STABLE_MODES:
-                assert np.all(np.diff(gpos) > 0)
-            slot_of = {int(pp): i for i, pp in enumerate(st["pos"])}
-            oslots = np.array([slot_of[int(pp)] for pp in gpos])
-            kept = np.zeros(st["pos"].shape[0], bool)
-            kept[oslots] = True
-            ok, _ = boundary_ok(st["m"], kept, budgets[b])
-            rep.set_ok &= ok
-            rep.strict_set_equal &= set(O.select_keep(st["m"], budgets[b]).tolist()) == set(oslots.tolist())
-            rep.m_err = max(rep.m_err, float(np.max(np.abs(gm - st["m"][oslots]))))
-            keep = np.sort(oslots)
-            st["m"], st["pos"] = st["m"][keep], st["pos"][keep]
-            for l in check_layers:
-                lk, lv = w.kv_rows(b, l % w.layers, gpos, u)
-                for g in range(w.kv_heads):
-                    gk = c.gather(c.k, b, l % w.layers, g, int(len_h[b])).float().cpu().numpy()[ls]
-                    gv = c.gather(c.v, b, l % w.layers, g, int(len_h[b])).float().cpu().numpy()[ls]
-                    rep.kv_err = max(rep.kv_err, float(np.max(np.abs(gk - lk[g]))), float(np.max(np.abs(gv - lv[g]))))
-        reports.append(rep)
+        assert list(c.len.cpu().numpy()) == lens, t
+        chk.check(t, out)
     assert ikv.ikv_device_status() == 0
-    return reports
+    return chk.reports
 
 
 def run_lockstep_layerwise(w: gen.Workload, steps: Optional[int] = None, page_perm_seed: Optional[int] = 7,
@@ -344,7 +452,7 @@ def run_lockstep_layerwise(w: gen.Workload, steps: Optional[int] = None, page_pe
                     dtype=ikv.IKV_BF16 if w.dtype == gen.BF16 else ikv.IKV_F32, page_size=w.page_size,
                     page_perm_seed=page_perm_seed, pos_cap=pos_cap)
     c.set_prefill(w.prefill, w.budgets())
-    kv = fill_host(c, w, u)
+    kv = fill_prefill(c, w, u)
     budgets = w.budgets()
     sts = []
     for b in range(w.batch):
@@ -410,19 +518,11 @@ def run_lockstep_layerwise(w: gen.Workload, steps: Optional[int] = None, page_pe
 
 def run_fullsize_sampled_layerwise(w: gen.Workload, seqs, steps: int, check_layers=(0, -1),
                                    page_perm_seed: Optional[int] = 7, per_layer: bool = False):
-    """Full-size lock-step of per-layer immediate eviction for a few sequences (GRAN_SEQ).
-
-    As run_fullsize_sampled, but the oracle side keeps, per sampled sequence, each layer's
-    held positions and the position-indexed state, and restates decode_step_layerwise with
-    the layers' K/V rows regenerated by position (reading R10)."""
+    """Full-size lock-step of per-layer immediate eviction for a few sequences (GRAN_SEQ),
+    against oracle.decode_step_layerwise_streaming (reading R10 with every layer's K/V rows
+    regenerated by position)."""
     T = steps
-    u = w.u_table()
-    u_dev = torch.from_numpy(u).cuda()
-    c = DecodeCache(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.cap,
-                    dtype=ikv.IKV_BF16 if w.dtype == gen.BF16 else ikv.IKV_F32, page_size=w.page_size,
-                    page_perm_seed=page_perm_seed, pos_cap=max(w.prefill) + T + 1)
-    c.set_prefill(w.prefill, w.budgets())
-    fill_device(c, w, u_dev)
+    c, u = fullsize_cache(w, page_perm_seed, pos_cap=max(w.prefill) + T + 1)
     op = O.Params(alpha=w.alpha, refresh_period=w.refresh_period, score_free=w.score_free)
     p = c.params(w.alpha, w.refresh_period, w.score_free, ikv.IKV_COMPACT_STABLE, evict_mode=ikv.IKV_EVICT_LAYER)
     ws = c.step_workspace()
@@ -430,60 +530,50 @@ def run_fullsize_sampled_layerwise(w: gen.Workload, seqs, steps: int, check_laye
     budgets = w.budgets()
     lens = list(w.prefill)
     out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
-    sp = w.spec()
-    L0_dev = torch.tensor(w.prefill, dtype=torch.int32, device="cuda")
-    kn = torch.empty((1, w.layers, w.batch, w.kv_heads, w.head_dim), dtype=torch_dtype(w), device="cuda")
-    vn = torch.empty_like(kn)
-    state = {b: {"pos": [np.arange(w.prefill[b], dtype=np.int64) for _ in range(w.layers)],
-                 "m": np.zeros(w.prefill[b] + T + 1), "next": w.prefill[b]} for b in seqs}
+    states = {b: O.layerwise_stream_prefill_state(w.prefill[b], budgets[b], w.layers, w.kv_heads) for b in seqs}
+    rows = {b: {l: KVRowsByPosition(w, b, u) for l in range(w.layers)} for b in seqs}
     reports = []
     for t in range(1, T + 1):
-        assert gen.cuda_lib().ikvgen_fill_tokens_cuda(ctypes.byref(sp), u_dev.data_ptr(), L0_dev.data_ptr(), t, t + 1,
-                                                      w.dtype, kn.data_ptr(), vn.data_ptr(),
-                                                      torch.cuda.current_stream().cuda_stream) == 0
-        decode_step(c, p, c.cache(max(lens)), t, to_device(qs[t - 1], w), kn[0], vn[0], out, ws, per_layer)
+        kn, vn = device_new_tokens(w, u, t)
+        decode_step(c, p, c.cache(max(lens)), t, to_device(qs[t - 1], w), kn, vn, out, ws, per_layer)
         lens = [min(L + 1, B) for L, B in zip(lens, budgets)]
         torch.cuda.synchronize()
-        refresh = O.is_refresh(t, w.refresh_period, w.score_free)
-        rep = StepReport(t=t, refresh=refresh)
+        rep = StepReport(t=t, refresh=O.is_refresh(t, w.refresh_period, w.score_free))
         q64 = as_f64(qs[t - 1], w)
         len_h = c.len.cpu().numpy()
         pos_h = c.pos.cpu().numpy()
         m_h = c.pos_state.cpu().numpy()
         for b in seqs:
-            st = state[b]
             assert len_h[b] == lens[b]
-            m = st["m"]
-            live = np.unique(np.concatenate(st["pos"]))
-            m[st["next"]] = 0.0 if refresh else float(np.mean(m[live]))
-            st["pos"] = [np.append(x, st["next"]) for x in st["pos"]]
-            st["next"] += 1
-            out_b = out[:, b].float().cpu().numpy()
+            gpu_kept = [np.sort(pos_h[b * w.layers + l, :lens[b]].astype(np.int64)) for l in range(w.layers)]
             for l in range(w.layers):
-                held = st["pos"][l]
-                k, v = w.kv_rows(b, l, held, u)
-                a_, o_ = O.last_query_attention(q64[l, b], [x.astype(np.float64) for x in k],
-                                                [x.astype(np.float64) for x in v])
-                rep.out_err = max(rep.out_err, float(np.max(np.abs(out_b[l] - o_))))
-                if refresh:
-                    s_pos = np.zeros_like(m)
-                    s_pos[held] = O.pooled_score(a_, O.GRAN_SEQ, w.kv_heads)[0]
-                    live = np.unique(np.concatenate(st["pos"]))
-                    m[live] = O.ema_update(m[live], s_pos[live], op.alpha)
-                m_l = m[held]
-                kept = pos_h[b * w.layers + l, :lens[b]].astype(np.int64)
-                assert np.all(np.diff(kept) > 0)
-                mask = np.isin(held, kept)
-                assert mask.sum() == len(kept)
-                ok, _ = boundary_ok(m_l, mask, budgets[b])
+                assert np.all(np.diff(pos_h[b * w.layers + l, :lens[b]]) > 0), (t, b, l)
+
+            def adopt(l, tr, b=b, rep=rep):
+                kept = gpu_kept[l]
+                mask = np.isin(tr.pos, kept)
+                assert mask.sum() == len(kept), (t, b, l)      # kept positions were held by the layer
+                ok, _ = boundary_ok(tr.m, mask, budgets[b])
+                rok, _ = boundary_ok(tr.m, mask, budgets[b], relative=True)
                 rep.set_ok &= ok
-                rep.strict_set_equal &= set(held[O.select_keep(m_l, budgets[b])].tolist()) == set(kept.tolist())
-                st["pos"][l] = kept
-            live = np.unique(np.concatenate(st["pos"]))
-            rep.m_err = max(rep.m_err, float(np.max(np.abs(m_h[b, live] - m[live]))))
+                rep.rel_set_ok &= rok
+                rep.strict_set_equal &= set(tr.kept.tolist()) == set(kept.tolist())
+                return kept
+
+            st = states[b]
+            # every layer's rows by position (the layers hold different sets: one memo per layer)
+            o_out, _ = O.decode_step_layerwise_streaming(st, t, q64[:, b],
+                                                         lambda l, g, ps, b=b: rows[b][l](l, g, ps), op,
+                                                         keep_override=adopt)
+            out_b = out[:, b].float().cpu().numpy()
+            rep.out_err = max(rep.out_err, float(np.max(np.abs(out_b - o_out))))
+            live = st.live()
+            rep.m_err = max(rep.m_err, float(np.max(np.abs(m_h[b, live] - st.m[live]))))
+            rep.m_rel_err = max(rep.m_rel_err, rel_err(m_h[b, live], st.m[live]))
             for l in check_layers:
                 ll = l % w.layers
-                lk, lv = w.kv_rows(b, ll, st["pos"][ll], u)
+                assert np.array_equal(gpu_kept[ll], st.pos[ll])
+                lk, lv = w.kv_rows(b, ll, st.pos[ll], u)
                 for g in range(w.kv_heads):
                     gk = c.gather(c.k, b, ll, g, lens[b]).float().cpu().numpy()
                     gv = c.gather(c.v, b, ll, g, lens[b]).float().cpu().numpy()

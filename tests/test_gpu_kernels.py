@@ -224,6 +224,8 @@ def test_attend_multi_pass_units(H, Hkv, batch):
     ema0 = torch.from_numpy(rng.random((c.rows, c.cap)).astype(np.float32)).cuda()
     ema = ema0.clone()
     cch = c.cache(max(lens), dead_slots=True)
+    # the plan this device runs really is multi-pass (one layer per call)
+    assert ikv.ikv_attend_plan(c.shape(), cch, 1, 0)["passes"] > 1
     ws = torch.empty(ikv.ikv_attend_workspace_size(c.shape(), cch), dtype=torch.uint8, device="cuda")
     alpha = 0.6
     ikv.ikv_decode_attend_score(c.shape(), cch, layer, q, out, score, ema, alpha, ws, ws.numel())

@@ -12,7 +12,7 @@ import pytest
 import torch
 
 import gen
-from harness import decode_step, make_cache, fill_host, run_lockstep, to_device
+from harness import decode_step, make_cache, fill_prefill, run_lockstep, to_device
 from paper_2609_03515_gb300 import ikv
 
 pytestmark = pytest.mark.gpu
@@ -126,6 +126,10 @@ def test_multi_pass_trajectories():
     rng = np.random.default_rng(41)
     prefill = [int(x) for x in rng.integers(1900, 3800, size=16)]
     w = small_llama(batch=16, layers=2, prefill=prefill, steps=4, budget_frac=0.9)
+    # the whole step's launch (2 layers x 16 sequences x 8 KV heads) is multi-pass on this device
+    c0 = make_cache(w)
+    assert ikv.ikv_attend_plan(c0.shape(), c0.cache(max(prefill) + 1), w.layers, 0)["passes"] > 1
+    del c0
     _assert(run_lockstep(w), 2e-2)
     _assert(run_lockstep(w, max_holes=64, compact_mode=ikv.IKV_COMPACT_STABLE_SHORT), 2e-2)
     _assert(run_lockstep(w.with_(steps=3), gran=ikv.IKV_GRAN_KVHEAD), 2e-2)
@@ -134,6 +138,9 @@ def test_multi_pass_trajectories():
     # heads = 256 units of 16-31 tiles) whose CTAs also store the layer's new rows
     w32 = small_llama(batch=32, layers=2, prefill=[int(x) for x in rng.integers(1900, 3800, size=32)], steps=3,
                       budget_frac=0.9)
+    c0 = make_cache(w32)
+    assert ikv.ikv_attend_plan(c0.shape(), c0.cache(max(w32.prefill) + 1), 1, 0)["passes"] > 1
+    del c0
     _assert(run_lockstep(w32, per_layer=True), 2e-2)
     _assert(run_lockstep(w32, per_layer=True, max_holes=64, compact_mode=ikv.IKV_COMPACT_STABLE_SHORT,
                          scorer=ikv.IKV_SCORE_VNORM), 2e-2)
@@ -202,7 +209,7 @@ def test_per_layer_split_equals_whole_step():
     caches = []
     for per_layer in (False, True):
         c = make_cache(w)
-        fill_host(c, w, u)
+        fill_prefill(c, w, u)
         caches.append(c)
     p = [c.params(w.alpha, w.refresh_period, False, ikv.IKV_COMPACT_STABLE_SHORT, max_holes=3) for c in caches]
     ws = [c.step_workspace() for c in caches]
