@@ -149,6 +149,7 @@ StepWs step_ws(const ikv_shape *s, int32_t cap, int32_t pos_cap) {
     off = align256(off + Rs * sizeof(int32_t));
     // one control block: append arrivals [batch], compaction arrivals [batch], fused-
     // selection arrivals [rows]
+    const size_t blk_max = ((size_t)cap + 31) / 32;
     w.done = off;
     w.cdone = off + (size_t)s->batch * sizeof(int32_t);
     w.sdone = off + 2 * (size_t)s->batch * sizeof(int32_t);
@@ -158,7 +159,6 @@ StepWs step_ws(const ikv_shape *s, int32_t cap, int32_t pos_cap) {
     w.n_moves = off;
     off = align256(off + Rs * sizeof(int32_t));
     // scorer variants: entropy pass buffers and VNorm means
-    const size_t blk_max = ((size_t)cap + 31) / 32;
     w.sbuf = off;
     off = align256(off + R * s->layers * (size_t)logit_stride(cap) * sizeof(float));
     w.epart = off;
@@ -285,6 +285,11 @@ ikv_status run_attend(const ikv_shape *s, const ikv_cache *c, int32_t layer0, in
         a.v_new = append->v_new;
         a.slot = append->slot;
         a.vnorm = append->vnorm;
+        // a later layer call reads nothing before its dependency wait that the kernels
+        // still draining ahead of it (the previous layer calls, or the caller's work
+        // between them) write: the step's bookkeeping ran in ikv_step_begin, and this
+        // layer's cached rows change only through the launch itself
+        a.early = layer0 > 0 ? 1 : 0;
     } else if (append) {
         IKV_TRY_CUDA(launch_append_rows(*append, st), "append rows launch");
     }

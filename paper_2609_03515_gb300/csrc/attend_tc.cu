@@ -87,6 +87,12 @@ struct TcArgs {
     // head's group sum of normalised probabilities, [batch][sc_layers][kv_heads][lstride]
     int32_t gsum;
     int32_t passes;  // consecutive chunks per CTA (>= 1)
+    // nonzero: nothing the preceding kernels in the stream still write is read before the
+    // programmatic-dependency wait except through this launch's own new-token rows, so the
+    // CTA initialises and starts streaming its K/V tiles first (a later layer call of the
+    // split step: len, start, slot, pos, the block table and this layer's cached rows are
+    // fixed since the step's first call)
+    int32_t early;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -148,11 +154,19 @@ __device__ __forceinline__ void mbar_drain(uint32_t bar, uint32_t parity) {
     }
 }
 
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uint32_t bar) {
+// L2 policy for data read once and never again in the step (the K/V stream): its lines are
+// the first to go, so the logits this kernel writes for the score pass stay in L2
+__device__ __forceinline__ uint64_t l2_evict_first() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uint32_t bar,
+                                            uint64_t pol) {
     asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
-            dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1, {%2, "
+        "%3}], [%4], %5;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(pol)
         : "memory");
 }
 
@@ -220,7 +234,8 @@ template <int G, bool MP>
 __global__ void __launch_bounds__(kThreads, 2)
     attend_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, const TcArgs a) {
     constexpr int NC = G <= 4 ? 4 : 8;  // TMEM columns read per S tile
-    pdl_wait();
+    const bool early = a.early != 0;
+    if (!early) pdl_wait();
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -239,14 +254,16 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int l = a.layer0 + li;
     // The unit's valid rows are physical slots [S0, S0 + L).  Chunks cut the 128-aligned
     // physical tiles covering them (TMA boxes stay page aligned); rows outside are masked.
-    const int L = a.len[b];
-    const int S0 = a.start ? a.start[b] : 0;
+    // (L2 loads: an early CTA reads these before the dependency wait)
+    const int L = __ldcg(a.len + b);
+    const int S0 = a.start ? __ldcg(a.start + b) : 0;
     const int ft = S0 / kTile;
     const int nt_unit = L > 0 ? (S0 + L + kTile - 1) / kTile - ft : 0;
     const int item = a.split_tokens / kTile;  // tiles per chunk
     const int ns_active = (nt_unit + item - 1) / item;  // chunks of the unit
     const int c0 = cta * a.passes;                      // this CTA's first chunk
     if (c0 >= ns_active) {
+        if (early) pdl_wait();
         if (cta == 0) {  // empty sequence: zero output, log-sum-exp -inf
             for (int i = threadIdx.x; i < G * kD; i += kThreads)
                 a.out[(((int64_t)li * a.batch + b) * a.q_heads + (int64_t)g * G) * kD + i] = __float2bfloat16_rn(0.f);
@@ -295,6 +312,20 @@ __global__ void __launch_bounds__(kThreads, 2)
         return ((l * a.num_pages + page) * a.kv_heads + g) * a.page_size + tok % a.page_size;
     };
     int ld_J = 0, ld_p = 0, ld_j = 0;  // producer cursor: loads issued, pass and load of the next one
+    const uint64_t kv_pol = l2_evict_first();
+    // split step: the physical slot that receives the new token's rows (-1: none here); a
+    // load of the tile holding it waits until this CTA has stored them
+    int p_new = -1;
+    if (a.k_new) {
+        const int j = __ldcg(a.slot + b);
+        if (j >= 0) p_new = S0 + j;
+    }
+    auto blocked = [&](int p, int j) {
+        if (p_new < 0) return false;
+        const int n = chunk_n(p);
+        const int t0 = chunk_t0(p) + (j < n ? j : j - n) * kTile;
+        return p_new >= t0 && p_new < t0 + kTile;
+    };
     auto issue_next = [&]() {
         const int st = ld_J % kNst;
         mbar_expect_tx(full(st), kStage);
@@ -302,8 +333,8 @@ __global__ void __launch_bounds__(kThreads, 2)
         const uint32_t dst = base + st * kStage;
         for (int bx = 0; bx < boxes; ++bx) {
             const int row = box_row(ld_p, ld_j, bx);
-            tma_load_2d(dst + bx * a.rows_per_box * 128, tm, 0, row, full(st));
-            tma_load_2d(dst + kHalf + bx * a.rows_per_box * 128, tm, 64, row, full(st));
+            tma_load_2d(dst + bx * a.rows_per_box * 128, tm, 0, row, full(st), kv_pol);
+            tma_load_2d(dst + kHalf + bx * a.rows_per_box * 128, tm, 64, row, full(st), kv_pol);
         }
         ++ld_J;
         if (++ld_j == 2 * chunk_n(ld_p)) {
@@ -311,14 +342,46 @@ __global__ void __launch_bounds__(kThreads, 2)
             ld_j = 0;
         }
     };
+    // Prologue.  The producer lane initialises the barriers and starts the K/V stream at
+    // once (every load up to the ring's depth that does not read the new token's tile);
+    // the TMEM allocation and P zeroing below overlap the loads' latency.  An early CTA
+    // does all of this before the dependency wait, so it overlaps the previous kernel's tail.
+    if (warp == 4 && lane == 0) {
+        for (int i = 0; i < kNst; ++i) {
+            mbar_init(full(i), 1);
+            mbar_init(empty(i), 1);
+        }
+        mbar_init(s_full, 1);
+        mbar_init(p_full(0), 128);
+        mbar_init(p_full(1), 128);
+        mbar_init(p_empty(0), 1);
+        mbar_init(p_empty(1), 1);
+        mbar_init(o_full, 1);
+        mbar_init(s_free, 128);
+        mbar_init(o_free, 128);
+        mbar_init(mma_done, 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        while (ld_J < kNst && ld_p < np && !blocked(ld_p, ld_j)) issue_next();
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    // both P buffers zeroed (rows >= G stay zero)
+    for (int i = tid; i < 2 * kOpBytes / 16; i += kThreads)
+        reinterpret_cast<uint4 *>(sm + kOffP)[i] = make_uint4(0, 0, 0, 0);
+    if (early) pdl_wait();
     if (warp == 4) {
         // Split step: the CTA whose chunks hold the new token's slot stores the token's K
         // and V rows into the cache (lanes 0-15: K, 16-31: V, 16 bytes each) before its
         // TMA loads read that tile; the proxy fence orders the stores before them.
         if (a.k_new) {
-            const int j = a.slot[b];
-            const int p = S0 + j;
-            if (j >= 0 && p >= chunk_t0(0) && p < chunk_t0(np - 1) + chunk_n(np - 1) * kTile) {
+            const int j = p_new - S0;
+            const int p = p_new;
+            if (p_new >= 0 && p >= chunk_t0(0) && p < chunk_t0(np - 1) + chunk_n(np - 1) * kTile) {
                 const int page = a.block_table[(int64_t)b * a.max_pages + p / a.page_size];
                 const int64_t row = ((int64_t)(l * a.num_pages + page) * a.kv_heads + g) * a.page_size + p % a.page_size;
                 const bool isv = lane >= 16;
@@ -342,35 +405,12 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
             __syncwarp();
         }
-        // the producer initialises the barriers and starts the K/V stream at once; the
-        // Q staging and TMEM allocation below overlap the loads' latency
-        if (lane == 0) {
-            for (int i = 0; i < kNst; ++i) {
-                mbar_init(full(i), 1);
-                mbar_init(empty(i), 1);
-            }
-            mbar_init(s_full, 1);
-            mbar_init(p_full(0), 128);
-            mbar_init(p_full(1), 128);
-            mbar_init(p_empty(0), 1);
-            mbar_init(p_empty(1), 1);
-            mbar_init(o_full, 1);
-            mbar_init(s_free, 128);
-            mbar_init(o_free, 128);
-            mbar_init(mma_done, 1);
-            *abort_flag = 0;
-            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        // the rest of the ring's first fill (the loads the new token's rows held back)
+        if (lane == 0)
             while (ld_J < kNst && ld_p < np) issue_next();
-        }
         __syncwarp();
     }
-    if (warp == 0) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                     "r"(kTmemCols)
-                     : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-    }
-    // Q operand [16 heads][128 dims], heads >= G zero; both P buffers zeroed (rows >= G stay zero)
+    // Q operand [16 heads][128 dims], heads >= G zero
     {
         const __nv_bfloat16 *qg = a.q + (((int64_t)li * a.batch + b) * H + (int64_t)g * G) * kD;
         for (int i = tid; i < kN * kD; i += kThreads) {
@@ -378,8 +418,6 @@ __global__ void __launch_bounds__(kThreads, 2)
             const __nv_bfloat16 v = h < G ? qg[h * kD + c] : __float2bfloat16_rn(0.f);
             *reinterpret_cast<__nv_bfloat16 *>(sm + kOffQ + (c >> 6) * (kN * 128) + sw128(h, c & 63)) = v;
         }
-        for (int i = tid; i < 2 * kOpBytes / 16; i += kThreads)
-            reinterpret_cast<uint4 *>(sm + kOffP)[i] = make_uint4(0, 0, 0, 0);
     }
     fence_async_smem();
     fence_before_sync();
@@ -887,6 +925,7 @@ cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group,
     t.v_pool = reinterpret_cast<__nv_bfloat16 *>(const_cast<void *>(a.v));
     t.vnorm = a.vnorm;
     t.gsum = a.gsum;
+    t.early = a.early;
     const int64_t units = (int64_t)a.pv.kv_heads * a.batch * a.n_layers;
     t.passes = tc_passes(units, a.n_splits, sms, a.gsum != 0);
     dim3 grid((unsigned)(((a.n_splits + t.passes - 1) / t.passes) * units));

@@ -14,6 +14,7 @@ constexpr int kAttendThreads = 128;
 constexpr int kMaxSplits = 128;    // split-K partitions per (seq, layer, kv head)
 constexpr int kMinSplitTokens = 256;
 constexpr int kMaxLayersPerScorePass = 32;
+constexpr int kScoreLayersPerGroup = 8;   // eligible layers one score CTA folds (one warp each)
 constexpr int kMaxLayers = 512;
 
 // Launch-count bookkeeping (host).
@@ -98,6 +99,9 @@ struct AttendArgs {
     // of its query group's normalised probabilities ([batch][sc_layers][kv_heads][lstride])
     // instead of per-head logits
     int32_t gsum;
+    // tensor-core kernel: the launch may set up and start its K/V stream before the
+    // programmatic-dependency wait (see TcArgs::early)
+    int32_t early;
 };
 
 struct CombineArgs {
@@ -177,6 +181,8 @@ cudaError_t launch_combine(const CombineArgs &a, int dtype, cudaStream_t st);
 cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, int sms, cudaStream_t st);
 // token blocks (and tokens per lane V) the score pass uses for max_len
 int score_blocks(const ScoreArgs &a, int32_t max_len, int sms, int *V);
+// layer groups (grid z) of a score pass over n_elig eligible layers
+int score_layer_groups(int n_elig);
 cudaError_t launch_entropy_fold(const ScoreArgs &a, int32_t max_len, cudaStream_t st);
 cudaError_t launch_vnorm_mean(const ScoreArgs &a, cudaStream_t st);
 cudaError_t launch_value_norms(const void *v, const PagedView &pv, const int32_t *len, int32_t batch, int32_t layers,

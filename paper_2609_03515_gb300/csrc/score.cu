@@ -2,22 +2,28 @@
 // scoring"), fused with the softmax normalisation; the VNorm and entropy-weighted
 // scorers of the Appendix "Per-step scoring"; value-row norms for VNorm.
 //
-// score_kernel: one CTA per (32 V tokens, utility row), one warp per eligible layer
-// (up to 32 per pass, passes launched in layer order), V consecutive tokens per lane.
-// Warp l computes s_l(i) = mean over the row's heads of p_h(i) = exp2(z_h(i) - lse2_h)
-// from the attention kernel's log2-domain logits and log-sum-exp (VNorm: each head's
-// p_h(i) times its KV head's value-norm weight); the CTA's first 32 V threads then fold
-// the layers into the utility in ascending order.  The entropy scorer needs every
-// token of a layer before its weight is known, so its first pass only stores s_l and
-// per-block partial entropies, and entropy_fold_kernel applies the weights and folds.
+// score_kernel: one 256-thread CTA per (32 V tokens, utility row, layer group): each
+// group holds up to 8 consecutive eligible layers, one warp per layer, V consecutive
+// tokens per lane.  Warp l computes s_l(i) = mean over the row's heads of p_h(i) =
+// exp2(z_h(i) - lse2_h) from the attention kernel's log2-domain logits and log-sum-exp
+// (VNorm: each head's p_h(i) times its KV head's value-norm weight).  Each update of
+// Eq. 2-4 is an affine map of the utility, m -> a m + c, so a group folds its layers, in
+// ascending order, into one such map per token; the last CTA of the row to finish
+// applies the groups' maps to every utility in layer order (with one group each CTA runs
+// the plain layer-by-layer fold itself) and, in a step, selects the row.  Splitting the
+// layers over CTAs spreads a short cache over every SM, and one arrival per CTA keeps
+// the chain of dependent steps after the loads short.  The entropy scorer needs every
+// token of a layer before its weight is known,
+// so its first pass only stores s_l and per-block partial entropies, and
+// entropy_fold_kernel applies the weights and folds.
 #include "ikv_internal.cuh"
 #include "select_row.cuh"
 
 namespace ikv {
 namespace {
 
-constexpr int kScoreWarps = 32;   // one warp per eligible layer of a pass
-static_assert(kScoreWarps * 32 == kSelThreads, "the fused selection needs a full selection CTA");
+constexpr int kScoreWarps = kScoreLayersPerGroup;  // one warp per eligible layer of a layer group
+constexpr int kScoreThreads = kScoreWarps * 32;    // also the fused selection's CTA size
 
 template <int V> struct VecF;
 template <> struct VecF<1> { using T = float; };
@@ -32,6 +38,28 @@ __device__ __forceinline__ float aggregate(float m, float s, int agg, float alph
     if (agg == IKV_AGG_CUMULATIVE) return m + s;                    // Eq. 3
     return s;                                                       // Eq. 2
 }
+// the factor a of the affine map m -> a m + c that n consecutive updates compose to
+__device__ __forceinline__ float agg_factor(int n, int agg, float alpha) {
+    if (agg == IKV_AGG_CUMULATIVE) return 1.f;
+    if (agg != IKV_AGG_EMA) return n > 0 ? 0.f : 1.f;
+    float f = 1.f;
+    for (int k = 0; k < n; ++k) f *= alpha;
+    return f;
+}
+
+// thread-block cluster: barrier over every thread of the cluster (release / acquire), and a
+// load from the shared memory of the cluster's CTA `rank` at the address of `p` in this one
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ float ld_cluster_f32(const float *p, int rank) {
+    const uint32_t a = static_cast<uint32_t>(__cvta_generic_to_shared(p));
+    uint32_t ra;
+    float v;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(a), "r"(rank));
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(ra) : "memory");
+    return v;
+}
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
@@ -44,15 +72,16 @@ __device__ __forceinline__ float warp_sum(float v) {
 // before the loads.  V > 1 reads each head row in 256- or 512-byte runs, which DRAM
 // serves far better than scattered 128-byte pieces.
 template <int V, int SCORER>
-__global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreArgs a) {
+__global__ void __launch_bounds__(kScoreThreads, 4) score_kernel(const ScoreArgs a) {
     using VT = typename VecF<V>::T;
     pdl_wait();
     constexpr int kTok = 32 * V;   // tokens per CTA
     constexpr int kHB = 32 / V;    // heads per load batch (32 registers of loads)
-    __shared__ __align__(16) float sl[kMaxLayersPerScorePass][kTok];
+    __shared__ __align__(16) float sl[kScoreWarps][kTok];
     extern __shared__ float wsm[];  // VNorm: per warp, [row's kv heads][kTok] value-norm weights
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int r = blockIdx.y;
+    const int lg = blockIdx.z, n_lg = gridDim.z;  // this CTA's layer group, and how many there are
     const int b = r / a.rows_per_seq;
     const int L = a.len[b];
     const int i0 = blockIdx.x * kTok;
@@ -68,10 +97,12 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
     const int fi = i0 + (int)threadIdx.x;  // token folded by this thread (threads < kTok)
     const bool folds = threadIdx.x < kTok && fi < L;
     const int64_t at = (int64_t)r * a.cap + fi;
+    const int kw0 = lg * kScoreWarps;                        // the group's first eligible layer (pass index)
+    const int n_here = min(kScoreWarps, a.n_elig - kw0);     // layers of this group
     float m = 0.f;
     if (SCORER != IKV_SCORE_ENTROPY && folds && a.ema) m = a.ema[at];
-    if (warp < a.n_elig) {
-        const int li = a.elig[warp];
+    if (warp < n_here) {
+        const int li = a.elig[kw0 + warp];
         // row padding keeps i0 + kTok <= lstride, so the vector loads stay inside the row
         const float *zp = a.logits + (((int64_t)b * a.n_layers + li) * H + h0) * (int64_t)a.lstride + il;
         const float *ll = a.lse2 + ((int64_t)b * a.n_layers + li) * H + h0;
@@ -142,14 +173,14 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
 #pragma unroll
         for (int v = 0; v < V; ++v) sl[warp][lane * V + v] = acc[v] * inv;
         if (SCORER != IKV_SCORE_ENTROPY && a.store_only) {  // each layer's pooled score, unfolded
-            const int k = a.k0 + warp;
+            const int k = a.k0 + kw0 + warp;
 #pragma unroll
             for (int v = 0; v < V; ++v)
                 if (il + v < L) a.sbuf[((int64_t)r * a.n_elig_total + k) * a.lstride + il + v] = acc[v] * inv;
         }
         if (SCORER == IKV_SCORE_ENTROPY) {
             // the layer's pooled scores, and this block's share of -sum s ln s over them
-            const int k = a.k0 + warp;
+            const int k = a.k0 + kw0 + warp;
             float e = 0.f;
 #pragma unroll
             for (int v = 0; v < V; ++v) {
@@ -165,7 +196,7 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
         }
     }
     if (SCORER == IKV_SCORE_ENTROPY) {
-        if (warp == 0) {  // live slots of this block (the entropy normalisation is ln of their count)
+        if (warp == 0 && lg == 0) {  // live slots of this block (the entropy normalisation is ln of their count)
             float c = 0.f;
 #pragma unroll
             for (int v = 0; v < V; ++v) {
@@ -179,101 +210,111 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(const ScoreA
     }
     if (a.store_only) return;
     __syncthreads();
+    // Fold this CTA's layers for its tokens.  One group: the plain layer-by-layer fold onto
+    // the utility.  Several: the group's layers as one affine map m -> f m + c (c: the fold
+    // from zero); the token block's groups form one cluster, and its first CTA applies the
+    // groups' maps in layer order, reading the others' c from their shared memory.
+    __shared__ float cpart[kTok];
+    float sc = 0.f;  // the last eligible layer's score (with one layer: the step's score)
+    float c = n_lg == 1 ? m : 0.f;
     if (folds) {
-        float sc = 0.f;
-        for (int k = 0; k < a.n_elig; ++k) {
+        for (int k = 0; k < n_here; ++k) {
             sc = sl[k][threadIdx.x];
-            m = aggregate(m, sc, a.agg, a.alpha);
+            c = aggregate(c, sc, a.agg, a.alpha);
         }
-        if (a.ema) a.ema[at] = m;
-        if (a.score) a.score[at] = sc;
+        if (a.score && lg == n_lg - 1) a.score[at] = sc;
     }
-    if (a.fuse_select) {
-        // This block's share of the selection's first pass -- its live slots and their
-        // lowest (key, highest slot) -- so that the common case (one slot too many,
-        // eviction deferred) needs no rescan of the row.
-        __shared__ unsigned long long blk_best[kTok / 32];
-        __shared__ uint32_t blk_cnt[kTok / 32];
-        const int blocks = (L + kTok - 1) / kTok;
-        if (threadIdx.x < kTok) {
-            uint32_t c = 0u;
-            unsigned long long best = ~0ull;
-            if (folds && (!a.sel_pos || a.sel_pos[at] >= 0)) {
-                c = 1u;
-                best = ((unsigned long long)ord_key(m) << 32) | (uint32_t)(~(uint32_t)fi);
+    if (n_lg > 1) {
+        if (threadIdx.x < kTok) cpart[threadIdx.x] = c;
+        cluster_sync();  // every group's c is in its shared memory
+        if (lg == 0 && folds) {
+            for (int q = 0; q < n_lg; ++q) {
+                const float cq = q == 0 ? c : ld_cluster_f32(&cpart[threadIdx.x], q);
+                m = agg_factor(min(kScoreWarps, a.n_elig - q * kScoreWarps), a.agg, a.alpha) * m + cq;
             }
+        }
+        cluster_sync();  // the first CTA has read them: the others may exit
+        if (lg != 0) return;
+    } else {
+        m = c;
+    }
+    if (folds && a.ema) a.ema[at] = m;
+    if (!a.fuse_select) return;
+    // The selection's first pass for this block: its live slots and their lowest (key,
+    // highest slot), left for the row's last block to arrive
+    __shared__ unsigned long long red_best[kScoreWarps];
+    __shared__ uint32_t red_cnt[kScoreWarps];
+    auto block_reduce = [&](uint32_t cn, unsigned long long best) {
 #pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                c += __shfl_xor_sync(0xffffffffu, c, o);
-                const unsigned long long y = __shfl_xor_sync(0xffffffffu, best, o);
-                best = y < best ? y : best;
-            }
-            if (lane == 0) {
-                blk_best[warp] = best;
-                blk_cnt[warp] = c;
-            }
+        for (int o = 16; o > 0; o >>= 1) {
+            cn += __shfl_xor_sync(0xffffffffu, cn, o);
+            const unsigned long long y = __shfl_xor_sync(0xffffffffu, best, o);
+            best = y < best ? y : best;
+        }
+        if (lane == 0) {
+            red_best[warp] = best;
+            red_cnt[warp] = cn;
         }
         __syncthreads();
         if (threadIdx.x == 0) {
-            unsigned long long best = ~0ull;
-            uint32_t c = 0u;
-            for (int w = 0; w < kTok / 32; ++w) {
-                best = blk_best[w] < best ? blk_best[w] : best;
-                c += blk_cnt[w];
+            for (int w = 1; w < kScoreWarps; ++w) {
+                best = red_best[w] < best ? red_best[w] : best;
+                cn += red_cnt[w];
             }
-            a.sel_best[(int64_t)r * a.nblk + blockIdx.x] = best;
-            a.sel_cnt[(int64_t)r * a.nblk + blockIdx.x] = c;
+            red_best[0] = best;
+            red_cnt[0] = cn;
         }
-        // the row's CTAs that hold tokens arrive once their utilities are stored; the
-        // last one selects the row (arrival counter only: no CTA waits for another)
-        __shared__ int last;
         __syncthreads();
+    };
+    const int blocks = (L + kTok - 1) / kTok;
+    {
+        uint32_t cn = 0u;
+        unsigned long long best = ~0ull;
+        if (folds && (!a.sel_pos || a.sel_pos[at] >= 0)) {
+            cn = 1u;
+            best = ((unsigned long long)ord_key(m) << 32) | (uint32_t)(~(uint32_t)fi);
+        }
+        block_reduce(cn, best);
         if (threadIdx.x == 0) {
-            __threadfence();  // after the barrier: releases every thread's stores of this block
-            last = atomicAdd(&a.row_done[r], 1) == blocks - 1;
-            if (last) a.row_done[r] = 0;
+            a.sel_best[(int64_t)r * a.nblk + blockIdx.x] = red_best[0];
+            a.sel_cnt[(int64_t)r * a.nblk + blockIdx.x] = red_cnt[0];
         }
-        __syncthreads();
-        if (last) {
-            __threadfence();
-            // the blocks' partials give the live count and the victim candidate
-            __shared__ unsigned long long s_best;
-            __shared__ uint32_t s_cnt;
-            if (warp == 0) {
-                unsigned long long best = ~0ull;
-                uint32_t c = 0u;
-                for (int j = lane; j < blocks; j += 32) {
-                    const unsigned long long y = __ldcg(a.sel_best + (int64_t)r * a.nblk + j);
-                    best = y < best ? y : best;
-                    c += __ldcg(a.sel_cnt + (int64_t)r * a.nblk + j);
-                }
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) {
-                    c += __shfl_xor_sync(0xffffffffu, c, o);
-                    const unsigned long long y = __shfl_xor_sync(0xffffffffu, best, o);
-                    best = y < best ? y : best;
-                }
-                if (lane == 0) {
-                    s_best = best;
-                    s_cnt = c;
-                }
-            }
-            __syncthreads();
-            const int B = max(a.budget[b], 0);
-            const int n_live = (int)s_cnt;
-            const int S = a.df.start ? a.df.start[b] : 0;
-            if (a.sel_pos && a.df.max_holes > 0 && B > 0 && n_live == B + 1 && L - B <= a.df.max_holes &&
-                S + L < a.df.cap) {
-                // one slot too many and the sequence may defer: mark the victim dead, as
-                // the selection itself would
-                if (threadIdx.x == 0) {
-                    a.sel_pos[(int64_t)r * a.cap + (int)(~(uint32_t)(s_best & 0xFFFFFFFFull))] = -1;
-                    a.keep_len[r] = -1 - B;
-                }
-            } else {
-                select_row(r, a.cap, a.ema, a.len, a.rows_per_seq, a.budget, a.sel_pos, a.keep, a.keep_len, a.df);
-            }
+    }
+    // every token block of the row arrives once its stores are out; the last one selects the
+    // row (arrival counter only: no CTA waits for another)
+    __shared__ int last;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();  // after the barrier: releases every thread's stores of this block
+        last = atomicAdd(a.row_done + r, 1) == blocks - 1;
+        if (last) a.row_done[r] = 0;
+    }
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    // the blocks' partials give the live count and the victim candidate
+    uint32_t cn = 0u;
+    unsigned long long best = ~0ull;
+    for (int jb = threadIdx.x; jb < blocks; jb += kScoreThreads) {
+        const unsigned long long y = __ldcg(a.sel_best + (int64_t)r * a.nblk + jb);
+        best = y < best ? y : best;
+        cn += __ldcg(a.sel_cnt + (int64_t)r * a.nblk + jb);
+    }
+    block_reduce(cn, best);
+    const unsigned long long s_best = red_best[0];
+    const int n_live = (int)red_cnt[0];
+    const int B = max(a.budget[b], 0);
+    const int S = a.df.start ? a.df.start[b] : 0;
+    if (a.sel_pos && a.df.max_holes > 0 && B > 0 && n_live == B + 1 && L - B <= a.df.max_holes && S + L < a.df.cap) {
+        // one slot too many and the sequence may defer: mark the victim dead, as the
+        // selection itself would
+        if (threadIdx.x == 0) {
+            a.sel_pos[(int64_t)r * a.cap + (int)(~(uint32_t)(s_best & 0xFFFFFFFFull))] = -1;
+            a.keep_len[r] = -1 - B;
         }
+    } else {
+        select_row<kScoreThreads>(r, a.cap, a.ema, a.len, a.rows_per_seq, a.budget, a.sel_pos, a.keep, a.keep_len,
+                                  a.df);
     }
 }
 
@@ -391,9 +432,14 @@ static size_t vnorm_smem(const ScoreArgs &a, int V) {
 }
 constexpr size_t kVnormSmemMax = 160 * 1024;
 
+int score_layer_groups(int n_elig) {
+    const int n = n_elig < kMaxLayersPerScorePass ? n_elig : kMaxLayersPerScorePass;
+    return n <= 0 ? 1 : (n + kScoreWarps - 1) / kScoreWarps;
+}
+
 int score_blocks(const ScoreArgs &a, int32_t max_len, int sms, int *V) {
-    // widest token vector that still gives every SM two CTAs
-    const int64_t rows = (int64_t)a.batch * a.rows_per_seq;
+    // widest token vector that still gives every SM two CTAs (over all layer groups)
+    const int64_t rows = (int64_t)a.batch * a.rows_per_seq * score_layer_groups(a.n_elig_total);
     auto ctas = [&](int tok) { return rows * ((max_len + tok - 1) / tok); };
     int v = ctas(128) >= 2 * sms ? 4 : ctas(64) >= 2 * sms ? 2 : 1;
     if (a.scorer == IKV_SCORE_VNORM)  // the weight staging must fit in shared memory
@@ -402,6 +448,7 @@ int score_blocks(const ScoreArgs &a, int32_t max_len, int sms, int *V) {
     return (max_len + 32 * v - 1) / (32 * v);
 }
 
+// The layer groups of a token block (grid z) run as one cluster.
 template <int V, int SCORER>
 static cudaError_t launch_score_v(const ScoreArgs &a, dim3 grid, cudaStream_t st) {
     const size_t smem = SCORER == IKV_SCORE_VNORM ? vnorm_smem(a, V) : 0;
@@ -410,7 +457,22 @@ static cudaError_t launch_score_v(const ScoreArgs &a, dim3 grid, cudaStream_t st
                                              (int)smem);
         if (e != cudaSuccess) return e;
     }
-    return launch_k(score_kernel<V, SCORER>, grid, dim3(kScoreWarps * 32), smem, st, a);
+    if (grid.z == 1) return launch_k(score_kernel<V, SCORER>, grid, dim3(kScoreThreads), smem, st, a);
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(kScoreThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = grid.z;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl_enabled() ? 2 : 1;
+    return cudaLaunchKernelEx(&cfg, score_kernel<V, SCORER>, a);
 }
 
 template <int SCORER>
@@ -424,7 +486,8 @@ cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, int sms, cudaS
     if (max_len <= 0 || a.n_elig <= 0) return cudaSuccess;
     int V = 1;
     const int nblk = score_blocks(a, max_len, sms, &V);
-    dim3 grid(nblk, (unsigned)(a.batch * a.rows_per_seq));
+    const int n_lg = score_layer_groups(a.n_elig);
+    dim3 grid(nblk, (unsigned)(a.batch * a.rows_per_seq), (unsigned)n_lg);
     cudaError_t e;
     if (a.scorer == IKV_SCORE_VNORM)
         e = launch_score_t<IKV_SCORE_VNORM>(a, grid, V, st);

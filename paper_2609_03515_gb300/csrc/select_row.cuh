@@ -17,8 +17,10 @@ __device__ __forceinline__ uint32_t ord_key(float f) {
 }
 constexpr uint32_t kDeadKey = 0u;  // dead slots: below every live key, never kept
 
-// exclusive scan of one value per thread across the block; returns (exclusive, total)
+// exclusive scan of one value per thread across a block of NT threads; returns (exclusive, total)
+template <int NT>
 __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t *warp_tot, uint32_t &total) {
+    constexpr int NW = NT / 32;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     uint32_t x = v;
 #pragma unroll
@@ -29,27 +31,30 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t *warp_t
     if (lane == 31) warp_tot[warp] = x;
     __syncthreads();
     if (warp == 0) {
-        uint32_t t = warp_tot[lane];
+        uint32_t t = lane < NW ? warp_tot[lane] : 0u;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const uint32_t y = __shfl_up_sync(0xffffffffu, t, o);
             if (lane >= o) t += y;
         }
-        warp_tot[lane] = t;  // inclusive over warps
+        if (lane < NW) warp_tot[lane] = t;  // inclusive over warps
     }
     __syncthreads();
     const uint32_t before = warp == 0 ? 0u : warp_tot[warp - 1];
-    total = warp_tot[31];
+    total = warp_tot[NW - 1];
     __syncthreads();
     return before + x - v;
 }
 
-// The selection of utility row r by the calling CTA, which must have kSelThreads threads
-// and be entered by all of them.
+// The selection of utility row r by the calling CTA, which must have NT threads (256 or
+// 1024) and be entered by all of them.
+template <int NT = kSelThreads>
 __device__ __forceinline__ void select_row(int r, int32_t cap, const float *__restrict__ util,
                                            const int32_t *__restrict__ len, int32_t rps,
                                            const int32_t *__restrict__ budget, int32_t *pos, int32_t *keep,
                                            int32_t *keep_len, DeferArgs df) {
+    static_assert(NT == 256 || NT == 1024, "the digit scan needs 256 threads at least, whole warps");
+    constexpr int NW = NT / 32;
     __shared__ uint32_t hist[256];
     __shared__ uint32_t warp_tot[32];
     __shared__ unsigned long long s_min[32];
@@ -67,11 +72,11 @@ __device__ __forceinline__ void select_row(int r, int32_t cap, const float *__re
     // every slot i < L for which keep_if(i) holds, in ascending order (block scans)
     auto write_kept = [&](auto keep_if) {
         uint32_t run = 0u;
-        for (int base = 0; base < L; base += kSelThreads) {
+        for (int base = 0; base < L; base += NT) {
             const int i = base + tid;
             const uint32_t kf = (i < L && keep_if(i)) ? 1u : 0u;
             uint32_t tot;
-            const uint32_t at = block_excl_scan(kf, warp_tot, tot);
+            const uint32_t at = block_excl_scan<NT>(kf, warp_tot, tot);
             if (kf) kp[run + at] = i;
             run += tot;
         }
@@ -83,7 +88,7 @@ __device__ __forceinline__ void select_row(int r, int32_t cap, const float *__re
     __syncthreads();
     uint32_t c = 0u;
     unsigned long long best = ~0ull;
-    for (int i = tid; i < L; i += kSelThreads) {
+    for (int i = tid; i < L; i += NT) {
         if (!live(i)) continue;
         ++c;
         const unsigned long long v = ((unsigned long long)ord_key(u[i]) << 32) | (uint32_t)(~(uint32_t)i);
@@ -98,7 +103,7 @@ __device__ __forceinline__ void select_row(int r, int32_t cap, const float *__re
     if (lane == 0) s_min[warp] = best;
     __syncthreads();
     if (warp == 0) {
-        best = s_min[lane];
+        best = lane < NW ? s_min[lane] : ~0ull;
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
             const unsigned long long y = __shfl_xor_sync(0xffffffffu, best, o);
@@ -111,7 +116,7 @@ __device__ __forceinline__ void select_row(int r, int32_t cap, const float *__re
 
     if (n_live <= B) {
         if (n_live == L) {
-            for (int j = tid; j < L; j += kSelThreads) kp[j] = j;
+            for (int j = tid; j < L; j += NT) kp[j] = j;
         } else {
             write_kept([&](int i) { return live(i); });
         }
@@ -136,7 +141,7 @@ __device__ __forceinline__ void select_row(int r, int32_t cap, const float *__re
             return;
         }
         if (n_live == L) {
-            for (int j = tid; j < B; j += kSelThreads) kp[j] = j < ev ? j : j + 1;
+            for (int j = tid; j < B; j += NT) kp[j] = j < ev ? j : j + 1;
         } else {
             write_kept([&](int i) { return i != ev && live(i); });
         }
@@ -150,9 +155,9 @@ __device__ __forceinline__ void select_row(int r, int32_t cap, const float *__re
     uint32_t prefix = 0u, mask = 0u, k = (uint32_t)B;
     for (int pass = 0; pass < 4; ++pass) {
         const int shift = 24 - 8 * pass;
-        for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0u;
+        for (int i = tid; i < 256; i += NT) hist[i] = 0u;
         __syncthreads();
-        for (int base = 0; base < L; base += kSelThreads) {
+        for (int base = 0; base < L; base += NT) {
             const int i = base + tid;
             uint32_t digit = 0xFFFFu;
             if (i < L) {
@@ -197,7 +202,7 @@ __device__ __forceinline__ void select_row(int r, int32_t cap, const float *__re
     const uint32_t need_eq = k;  // theta-valued slots that survive (lowest slots first)
 
     uint32_t run_eq = 0u, run_keep = 0u;
-    for (int base = 0; base < L; base += kSelThreads) {
+    for (int base = 0; base < L; base += NT) {
         const int i = base + tid;
         uint32_t key = 0u;
         bool in = i < L;
@@ -205,9 +210,9 @@ __device__ __forceinline__ void select_row(int r, int32_t cap, const float *__re
         const uint32_t gt = (in && key > theta) ? 1u : 0u;
         const uint32_t eq = (in && key == theta) ? 1u : 0u;
         uint32_t eq_tot, kp_tot;
-        const uint32_t eq_rank = block_excl_scan(eq, warp_tot, eq_tot);
+        const uint32_t eq_rank = block_excl_scan<NT>(eq, warp_tot, eq_tot);
         const uint32_t kf = (gt || (eq && run_eq + eq_rank < need_eq)) ? 1u : 0u;
-        const uint32_t at = block_excl_scan(kf, warp_tot, kp_tot);
+        const uint32_t at = block_excl_scan<NT>(kf, warp_tot, kp_tot);
         if (kf) kp[run_keep + at] = i;
         run_eq += eq_tot;
         run_keep += kp_tot;
