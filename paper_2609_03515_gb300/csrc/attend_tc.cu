@@ -170,6 +170,12 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
         : "memory");
 }
 
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap *map, int x, int y) {
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(map)),
+                 "r"(x), "r"(y)
+                 : "memory");
+}
+
 // smem matrix descriptor, 128-byte swizzle (sm_100 family, version 1)
 __device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
     uint64_t d = (uint64_t)((saddr >> 4) & 0x3FFFu);
@@ -363,6 +369,25 @@ __global__ void __launch_bounds__(kThreads, 2)
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         while (ld_J < kNst && ld_p < np && !blocked(ld_p, ld_j)) issue_next();
+        // an early CTA also pulls the rest of its tiles into L2 while it waits, so the loads
+        // it can only issue once the ring turns over find them there (the new token's tile is
+        // left out: its rows change before it is read)
+        if (early) {
+            for (int p = ld_p, j = ld_j; p < np;) {
+                if (!blocked(p, j)) {
+                    const CUtensorMap *tm = j < chunk_n(p) ? &tmK : &tmV;
+                    for (int bx = 0; bx < boxes; ++bx) {
+                        const int row = box_row(p, j, bx);
+                        tma_prefetch_2d(tm, 0, row);
+                        tma_prefetch_2d(tm, 64, row);
+                    }
+                }
+                if (++j == 2 * chunk_n(p)) {
+                    ++p;
+                    j = 0;
+                }
+            }
+        }
     }
     if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
@@ -410,13 +435,14 @@ __global__ void __launch_bounds__(kThreads, 2)
             while (ld_J < kNst && ld_p < np) issue_next();
         __syncwarp();
     }
-    // Q operand [16 heads][128 dims], heads >= G zero
+    // Q operand [16 heads][128 dims], heads >= G zero: one 16-byte load per thread (8 dims
+    // of one head, which stay together as one 16-byte chunk of the swizzled layout)
     {
         const __nv_bfloat16 *qg = a.q + (((int64_t)li * a.batch + b) * H + (int64_t)g * G) * kD;
-        for (int i = tid; i < kN * kD; i += kThreads) {
-            const int h = i / kD, c = i % kD;
-            const __nv_bfloat16 v = h < G ? qg[h * kD + c] : __float2bfloat16_rn(0.f);
-            *reinterpret_cast<__nv_bfloat16 *>(sm + kOffQ + (c >> 6) * (kN * 128) + sw128(h, c & 63)) = v;
+        for (int i = tid; i < kN * (kD / 8); i += kThreads) {
+            const int h = i / (kD / 8), c = (i % (kD / 8)) * 8;
+            const uint4 v = h < G ? *reinterpret_cast<const uint4 *>(qg + h * kD + c) : make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4 *>(sm + kOffQ + (c >> 6) * (kN * 128) + sw128(h, c & 63)) = v;
         }
     }
     fence_async_smem();
