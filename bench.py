@@ -58,6 +58,8 @@ def parse():
                     help="also run every mode eagerly and report its per-kernel times")
     ap.add_argument("--cpu-steps", type=int, default=0, help="oracle steps in the CPU sample (0 = auto)")
     ap.add_argument("--no-trace", action="store_true", help="skip the rank-trace diagnostics")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the other workloads (per-configuration block and the Qwen-shaped sweep)")
     return ap.parse_args()
 
 
@@ -84,7 +86,7 @@ def rank_seed(base_seed: int, rank: int) -> int:
 
 
 # revision of each attention kernel; a committed ncu summary counts only for its own revision
-ATTEND_KERNEL_REV = {"attend_tc_kernel": "attend_tc_v10", "attend_split_kernel": "attend_split_v2"}
+ATTEND_KERNEL_REV = {"attend_tc_kernel": "attend_tc_v11", "attend_split_kernel": "attend_split_v2"}
 
 
 def schedule_name(w) -> str:
@@ -169,6 +171,52 @@ class OracleSample:
                 f"fp64 numpy, 1 BLAS thread; tokens/s = steps / summed step time")
 
 
+def _oracle_worker(w, n_warm: int, n_steps: int, barrier, queue):
+    """One host core's share of the all-cores oracle run (a spawned process): one
+    sequence's sample, its warm-up steps, then n_steps timed after every worker is ready."""
+    s = OracleSample(w, n_warm + n_steps)
+    for _ in range(n_warm):
+        s.step()
+    barrier.wait()
+    t0 = time.monotonic()
+    for _ in range(n_steps):
+        s.step()
+    queue.put((t0, time.monotonic()))
+
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def oracle_all_cores(w, n_warm: int, n_steps: int, cores: int = 0) -> dict:
+    """The oracle on every host core: one process per core (spawned, BLAS on 1 thread
+    each), each decoding its own sequence of the workload (a different seed) for n_steps
+    steps after n_warm untimed ones; tokens/s = all decoded tokens / the wall time from the
+    first worker's start to the last one's end."""
+    import multiprocessing as mp
+
+    n = cores or host_cores()
+    ctx = mp.get_context("spawn")
+    barrier = ctx.Barrier(n)
+    queue = ctx.Queue()
+    procs = [ctx.Process(target=_oracle_worker, args=(w.with_(seed=w.seed + 7919 * (i + 1)), n_warm, n_steps,
+                                                      barrier, queue)) for i in range(n)]
+    for p in procs:
+        p.start()
+    spans = [queue.get(timeout=1800) for _ in range(n)]
+    for p in procs:
+        p.join()
+    wall = max(b for _, b in spans) - min(a for a, _ in spans)
+    return {"value": n * n_steps / wall, "unit": "tokens/s", "cores": n, "kind": "oracle",
+            "sample": f"{n} processes, one per host core, each {n_steps} oracle decode steps (after {n_warm} "
+                      f"untimed) of its own sequence with a {w.budgets()[0]}-token cache, {w.layers} layers x "
+                      f"{w.q_heads} q heads / {w.kv_heads} kv heads x d {w.head_dim}, fp64 numpy, 1 BLAS thread "
+                      f"each; tokens/s = all steps / wall time", "wall_s": wall}
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -178,18 +226,15 @@ def run_reference(args):
     w = gen.config(args.config)
     if args.layers:
         w = w.with_(layers=args.layers, name=f"{w.name}-{args.layers}layers")
-    s = OracleSample(w, args.warmup + args.steps)
-    for _ in range(args.warmup):
-        s.step()
-    sec = sum(s.step() for _ in range(args.steps))
-    value = w.batch * args.steps / sec
+    # every host core runs the oracle on a sequence of its own (the workload's shape)
+    cb = oracle_all_cores(w, args.warmup, args.steps)
+    value = cb["value"]
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * sec / args.steps,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * cb["wall_s"] / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "config": {"workload": w.name, "prefill": w.prefill[0], "budget": w.budgets()[0],
                                             "alpha": w.alpha, "refresh_period": w.refresh_period},
-            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
-                             "sample": s.describe(args.steps)},
+            "cpu_baseline": cb,
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -470,6 +515,151 @@ def run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, 
     return res
 
 
+def run_trajectory(w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, mh: int, dist=None):
+    """The configuration's whole decode run: decode steps 1 .. w.steps from the prefill,
+    step 1 (which scores the whole prefill and evicts most of it) and every deferred
+    compaction included, each step replayed from a CUDA graph captured for it (step 1 with
+    the prefill's length bound, the others with the steady bound).  Returns the time of
+    all steps."""
+    import torch
+
+    from paper_2609_03515_gb300 import ikv, step_lengths
+
+    reset(c, w, u_dev)
+    p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, max_holes=mh)
+    p.ws_zeroed = 1  # the workspace is zero-filled at creation and every step leaves its counters zero
+    budgets = w.budgets()
+    dev = c.k.device
+    out = torch.empty((w.layers, w.batch, w.q_heads, w.head_dim), dtype=c.torch_dtype, device=dev)
+    lens, live = list(w.prefill), list(w.prefill)
+    bounds = []
+    for t in range(1, w.steps + 1):
+        bounds.append(max(lens))
+        lens, live = step_lengths(lens, live, budgets, mh)
+    steady = c.cache(min(c.cap - 1, max(bounds[1:] + [max(budgets) + mh])))
+    graphs = []
+    for t in range(1, w.steps + 1):
+        cache = c.cache(bounds[0]) if t == 1 else steady
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="thread_local"):
+            ikv.ikv_step(c.shape(), p, cache, c.ema, t, qs_dev[t - 1], kn_dev[t - 1], vn_dev[t - 1], out, ws,
+                         ws.numel(), torch.cuda.current_stream())
+        graphs.append(g)
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    start.record(stream)
+    for g in graphs:
+        g.replay()
+    stop.record(stream)
+    torch.cuda.synchronize()
+    assert ikv.ikv_device_status() == 0
+    return max_over_ranks(start.elapsed_time(stop), dist, dev)
+
+
+def sig(x, n: int = 4):
+    """x rounded to n significant digits (keeps the JSON line short)."""
+    if x is None or x == 0:
+        return x
+    from math import floor, log10
+
+    return round(x, -int(floor(log10(abs(x)))) + n - 1)
+
+
+def attention_bytes(w, esz: int) -> int:
+    """Algorithmic bytes of one steady-state attention launch over every layer: the K and
+    V rows of each sequence's B + 1 cached tokens, plus q."""
+    L = [min(x + 1, B + 1) for x, B in zip(w.prefill, w.budgets())]
+    return sum(L) * w.layers * w.kv_heads * w.head_dim * 2 * esz + w.layers * w.batch * w.q_heads * w.head_dim * esz
+
+
+def step_bytes(w, esz: int) -> int:
+    """Algorithmic bytes of one steady-state step (refresh): the attention's K/V and q reads,
+    the output write, the utilities read and written once, and the new token's K/V rows."""
+    L = [min(x + 1, B + 1) for x, B in zip(w.prefill, w.budgets())]
+    out = w.layers * w.batch * w.q_heads * w.head_dim * esz
+    util = 8 * sum(L)
+    append = w.layers * w.batch * w.kv_heads * w.head_dim * 2 * esz
+    return attention_bytes(w, esz) + out + util + append
+
+
+def run_other_config(args, cfg: int, dev, dist, rank: int, compact_mode, mh_arg: int, peak: float, sweep: bool):
+    """One more workload, for the per-configuration block: its headline schedule, the same
+    inputs under full refresh, the attention and attention + score + EMA roofline from
+    eager per-kernel events, and its whole trajectory; with sweep (the Qwen-shaped
+    workload) the budget x refresh-period x alpha grid as well.  Fewer timed steps than the
+    headline (at most 20 after 3 warm-up steps); everything is freed afterwards."""
+    import argparse
+
+    import torch
+
+    import gen
+    from paper_2609_03515_gb300 import auto_max_holes
+
+    w = gen.config(cfg)
+    w = w.with_(seed=rank_seed(w.seed, rank))
+    sub = argparse.Namespace(warmup=3, steps=min(args.steps, 20))
+    total = max(w.steps, sub.warmup + sub.steps)
+    w = w.with_(steps=total)
+    mh = mh_arg if mh_arg >= 0 else auto_max_holes(w.budgets())
+    u = w.u_table()
+    u_dev = torch.from_numpy(u).to(dev)
+    c = setup(w, dev, compact_mode, total)
+    ws = c.step_workspace()
+    qs_dev, kn_dev, vn_dev = device_inputs(w, u, u_dev, total, dev)
+    esz = 2 if w.dtype == gen.BF16 else 4
+    K = sub.steps
+    eager = run_mode(sub, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, True, dist, mh)
+    head = run_mode_graph(sub, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, False, mh)
+    full_w = w.with_(refresh_period=1, score_free=False)
+    sched = schedule_name(w)
+    full = head if sched == "full" else run_mode_graph(sub, full_w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode,
+                                                        dist, False, mh)
+    km = eager["kernel_ms"]
+    # the attention + score + EMA time of a refresh step: this schedule's eager score time
+    # is an average over its steps, so the full-refresh run's events give it
+    kf = km if sched == "full" else run_mode(sub, full_w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, True,
+                                             dist, mh)["kernel_ms"]
+    ab = attention_bytes(w, esz)
+    traj_w = w.with_(steps=gen.config(cfg).steps)
+    traj_ms = run_trajectory(traj_w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, mh, dist)
+    world = dist.get_world_size() if dist else 1
+    res = {"workload": w.name, "schedule": sched,
+           "value": sig(job_throughput(w.batch * K, world, head["ms"])),
+           "us_per_step": sig(1e3 * head["ms"] / K),
+           "attend_frac": sig(ab / (km["attend"] / 1e3) / 1e9 / peak),
+           "attend_score_ema_frac": sig((ab + 8 * sum(min(x + 1, B + 1) for x, B in zip(w.prefill, w.budgets())))
+                                        / ((kf["attend"] + kf["score_ema"]) / 1e3) / 1e9 / peak),
+           "full_value": sig(job_throughput(w.batch * K, world, full["ms"])),
+           "speedup_vs_full": sig(full["ms"] / head["ms"]),
+           "trajectory": {"steps": traj_w.steps, "value": sig(job_throughput(w.batch * traj_w.steps, world, traj_ms)),
+                          "ms": sig(traj_ms)}}
+    if sweep:
+        grid = {}
+        base = None
+        for bf in (0.5, 0.25, 0.1):
+            for r in (1, 2, 4, 8):
+                ww = w.with_(budget_frac=bf, refresh_period=r, score_free=False)
+                m = run_mode_graph(sub, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, False,
+                                   mh_arg if mh_arg >= 0 else auto_max_holes(ww.budgets()))
+                grid[f"b{int(bf * 100)}_r{r}"] = job_throughput(w.batch * K, world, m["ms"])
+        alphas = {}
+        for al in (0.5, 0.9, 0.99):
+            ww = w.with_(budget_frac=0.1, refresh_period=1, score_free=False, alpha=al)
+            m = run_mode_graph(sub, ww, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, False, mh)
+            alphas[f"a{al}"] = sig(job_throughput(w.batch * K, world, m["ms"]))
+        res["sweep"] = {"tok_s": {k: sig(v) for k, v in grid.items()},
+                        "lazy_speedup": {k: sig(v / grid[k.split("_")[0] + "_r1"]) for k, v in grid.items()
+                                         if not k.endswith("_r1")},
+                        "alpha_b10_r1": alphas}
+    del c, ws, qs_dev, kn_dev, vn_dev, u_dev
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_trace(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, mh: int = 0):
     """Rank-trace diagnostics (raw / EMA top-k churn, raw/EMA Jaccard, raw-top evicted)
     over the timed steps of one schedule, launched eagerly with ikv_params.trace set;
@@ -639,20 +829,27 @@ def run_ours(args):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
+        # the oracle on one host thread, then on every host core (one sequence per core)
         n = args.cpu_steps or 8
         smp = OracleSample(w, n + 1)
         smp.step()  # first step outside the sample (allocator warm-up)
         sec = sum(smp.step() for _ in range(n))
-        cpu = {"value": n / sec, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": smp.describe(n)}
+        single = {"value": n / sec, "unit": "tokens/s", "cores": 1, "sample": smp.describe(n)}
         del smp
+        cpu = oracle_all_cores(w, 1, n)
+        cpu["single_thread"] = single
 
     dev = torch.device("cuda", torch.cuda.current_device())
     u = w.u_table()
     u_dev = torch.from_numpy(u).to(dev)
+    # enough resident inputs for the timed steps and for the whole trajectory
+    total_steps = max(total_steps, gen.config(args.config).steps)
+    w = w.with_(steps=total_steps)
     c = setup(w, dev, compact_mode, total_steps)
     ws = c.step_workspace()
     qs_dev, kn_dev, vn_dev = device_inputs(w, u, u_dev, total_steps, dev)
-    qs_t = qs_dev.cpu()
+    T_io = args.warmup + args.steps
+    qs_t = qs_dev[:T_io].cpu()
 
     from paper_2609_03515_gb300 import auto_max_holes
 
@@ -661,8 +858,8 @@ def run_ours(args):
     full = run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, True, mh)
     # end to end right after the headline, before the mode comparisons
     qs_pin = qs_t.pin_memory()
-    kn_pin = kn_dev.cpu().pin_memory()
-    vn_pin = vn_dev.cpu().pin_memory()
+    kn_pin = kn_dev[:T_io].cpu().pin_memory()
+    vn_pin = vn_dev[:T_io].cpu().pin_memory()
     # five complete end-to-end runs, median reported: host-link bandwidth on the shared
     # machine varies from run to run
     e2e_runs = [run_e2e(args, w, c, u_dev, ws, compact_mode, qs_pin, kn_pin, vn_pin, dist, mh) for _ in range(5)]
@@ -672,6 +869,12 @@ def run_ours(args):
     # the model-integration form: the same headline steps split per layer
     per_layer = {k: run_mode_graph(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, dist, False, mh,
                                    per_layer=k) for k in ("split", "foreign")}
+    # the whole decode run of the headline configuration, step 1 and every compaction included
+    traj_w = w.with_(steps=gen.config(args.config).steps)
+    traj_ms = run_trajectory(traj_w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, mh, dist)
+    L = [min(x + 1, B + 1) for x, B in zip(w.prefill, w.budgets())]  # length seen by the timed steps
+    att_kernel = ("attend_tc_kernel" if ikv.ikv_attend_path(c.shape(), c.cache(max(L))) == ikv.IKV_PATH_TENSOR_CORE
+                  else "attend_split_kernel")
 
     head_sched = schedule_name(w)
     modes = {}
@@ -682,14 +885,14 @@ def run_ours(args):
         sf_w = w.with_(refresh_period=1, score_free=True)
         att, vnm, ent = ikv.IKV_SCORE_ATTENTION, ikv.IKV_SCORE_VNORM, ikv.IKV_SCORE_ENTROPY
         stable, layer = ikv.IKV_COMPACT_STABLE, ikv.IKV_EVICT_LAYER
-        ema, cum, single = ikv.IKV_AGG_EMA, ikv.IKV_AGG_CUMULATIVE, ikv.IKV_AGG_SINGLE_STEP
+        ema, cum, single_step = ikv.IKV_AGG_EMA, ikv.IKV_AGG_CUMULATIVE, ikv.IKV_AGG_SINGLE_STEP
         variants = (("full", full_w, compact_mode, mh, att, 0, ema),
                     ("lazy4", lazy_w, compact_mode, mh, att, 0, ema),
                     ("score_free", sf_w, compact_mode, mh, att, 0, ema),
                     ("full_vnorm", full_w, compact_mode, mh, vnm, 0, ema),
                     ("full_entropy", full_w, compact_mode, mh, ent, 0, ema),
                     ("full_cumulative", full_w, compact_mode, mh, att, 0, cum),
-                    ("full_single_step", full_w, compact_mode, mh, att, 0, single),
+                    ("full_single_step", full_w, compact_mode, mh, att, 0, single_step),
                     ("full_every_step", full_w, compact_mode, 0, att, 0, ema),
                     ("lazy4_every_step", lazy_w, compact_mode, 0, att, 0, ema),
                     ("score_free_every_step", sf_w, compact_mode, 0, att, 0, ema),
@@ -719,22 +922,35 @@ def run_ours(args):
                                          kn_dev, vn_dev, ws, compact_mode, mh) for a in (0.3, 0.8, 0.9)}
     K = args.steps
     value = job_throughput(w.batch * K, world, full["ms"])
+    peak, peak_kind = load_peaks()
+    # the other workloads: Lazy4 (ragged batch), Score-Free (64k), and the Qwen-shaped one
+    # with its budget x refresh-period x alpha sweep; freed before the next one
+    others = {}
+    if args.config == 1 and not args.no_configs:
+        del c, ws, qs_dev, kn_dev, vn_dev
+        torch.cuda.empty_cache()
+        for cfg in (2, 3, 4):
+            others[str(cfg)] = run_other_config(args, cfg, dev, dist, rank, compact_mode, args.max_holes, peak,
+                                                sweep=cfg == 4)
     if rank != 0:
         if dist:
             dist.destroy_process_group()
         return
 
-    peak, peak_kind = load_peaks()
-    # attention kernel roofline: algorithmic bytes of one launch at the steady-state length
-    L = [min(x + 1, B + 1) for x, B in zip(w.prefill, w.budgets())]  # length seen by the timed steps
     esz = 2 if w.dtype == gen.BF16 else 4
-    kv_bytes = sum(L) * w.layers * w.kv_heads * w.head_dim * 2 * esz
-    q_bytes = w.layers * w.batch * w.q_heads * w.head_dim * esz
+    # attention kernel roofline: algorithmic bytes of one launch at the steady-state length
+    ab = attention_bytes(w, esz)
+    kv_bytes = ab - w.layers * w.batch * w.q_heads * w.head_dim * esz
     att_ms = eager["kernel_ms"]["attend"]
-    achieved = (kv_bytes + q_bytes) / (att_ms / 1e3) / 1e9
-    att_path = ikv.ikv_attend_path(c.shape(), c.cache(max(L)))
-    att_kernel = "attend_tc_kernel" if att_path == ikv.IKV_PATH_TENSOR_CORE else "attend_split_kernel"
+    achieved = ab / (att_ms / 1e3) / 1e9
     traffic = profiled_traffic(att_kernel, w.name)
+    # the unit the method's cost is stated in: attention + score + EMA (one launch each per
+    # step; eager per-kernel events, so each includes a launch gap), and the whole graphed step
+    ase_bytes = ab + 8 * sum(L)
+    ase_ms = eager["kernel_ms"]["attend"] + eager["kernel_ms"]["score_ema"]
+    st_bytes = step_bytes(w, esz)
+    st_ms = full["ms"] / K
+    nominal = 8000.0
     l2_note = ("inputs exceed L2 (K/V working set %.0f MB > 129 MB), no flush" % (kv_bytes / 1e6) if kv_bytes > 129e6
                else "K/V working set %.2f MB stays in L2 (launch-bound case), no flush" % (kv_bytes / 1e6))
     line = {
@@ -760,7 +976,15 @@ def run_ours(args):
                    "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                      "traffic": traffic, "kernel": att_kernel, "peak_kind": peak_kind,
-                     "bytes_per_launch": kv_bytes + q_bytes, "ms_per_launch": att_ms},
+                     "bytes_per_launch": ab, "ms_per_launch": att_ms,
+                     "attend_score_ema": {"bytes": ase_bytes, "ms": ase_ms,
+                                          "frac": ase_bytes / (ase_ms / 1e3) / 1e9 / peak,
+                                          "frac_of_nominal_8tbs": ase_bytes / (ase_ms / 1e3) / 1e9 / nominal,
+                                          "note": "K/V + q reads and the utilities' read + write over the eager "
+                                                  "events of the attention and score kernels (each with its launch gap)"},
+                     "step": {"bytes": st_bytes, "ms": st_ms, "frac": st_bytes / (st_ms / 1e3) / 1e9 / peak,
+                              "frac_of_nominal_8tbs": st_bytes / (st_ms / 1e3) / 1e9 / nominal,
+                              "note": "the whole graphed step: attention, output, utilities, new rows"}},
         "kernel_ms_per_step": eager["kernel_ms"],
         "eager": {"value": job_throughput(w.batch * K, world, eager["ms"]), "ms_per_step": eager["ms"] / K,
                   "note": "same steps launched one by one (per-kernel events above come from this run)"},
@@ -770,26 +994,12 @@ def run_ours(args):
                 "note": "median of five runs; inputs uploaded from pinned host memory and outputs read back "
                         "every step, overlapped with the previous / next step's compute"},
         "gpu_launches": full["launches"],
-        "per_layer": {
-            "value": job_throughput(w.batch * K, world, per_layer["split"]["ms"]),
-            "ms_per_step": per_layer["split"]["ms"] / K,
-            "vs_whole_step": full["ms"] / per_layer["split"]["ms"],
-            "gpu_launches": per_layer["split"]["launches"],
-            "with_foreign_copies": {"value": job_throughput(w.batch * K, world, per_layer["foreign"]["ms"]),
-                                    "ms_per_step": per_layer["foreign"]["ms"] / K},
-            "note": "the headline steps as ikv_step_begin / one ikv_step_layer per layer / ikv_step_end, one CUDA "
-                    "graph per step (PDL between the library's kernels); with_foreign_copies: each layer's q, "
-                    "k_new, v_new first copied by PyTorch kernels (3 per layer, not counted in gpu_launches)"},
         "clocks": full["clocks"],
-        "modes": {k: w.batch * K * world / (v["ms"] / 1e3) for k, v in modes.items()},
+        "modes": {k: sig(w.batch * K * world / (v["ms"] / 1e3)) for k, v in modes.items()},
     }
-    if trace is not None:
-        line["rank_trace"] = dict(trace, note="full refresh, the headline's inputs and compaction; means over the "
-                                              "timed steps and utility rows; raw = the last layer's single-step "
-                                              "score, k = the budget (Appendix \"Mechanistic Diagnostics\")")
     if modes:
         full_v = line["modes"]["full"]
-        line["speedup_vs_full"] = {k: v / full_v for k, v in line["modes"].items() if k != "full"}
+        line["speedup_vs_full"] = {k: sig(v / full_v) for k, v in line["modes"].items() if k != "full"}
         if mode_kernels:
             line["mode_kernel_ms_per_step"] = mode_kernels
         line["modes_note"] = ("full / lazy4 / score_free: refresh every step / every 4th step (Eq. 6) / step 1 "
@@ -803,6 +1013,32 @@ def run_ours(args):
                               "*_layer_evict: per-layer immediate eviction (each layer keeps its own top-B "
                               "right after its update of a position-indexed state), hole-fill compaction of "
                               "every layer; full_layer_evict_stable: the same with order-preserving compaction")
+    if trace is not None:
+        line["rank_trace"] = dict({k: {kk: sig(vv) for kk, vv in v.items()} for k, v in trace.items()},
+                                  note="full refresh, the headline's inputs and compaction; means over the timed "
+                                       "steps and utility rows; raw = the last layer's single-step score, k = the "
+                                       "budget (Appendix \"Mechanistic Diagnostics\")")
+    line["notes"] = ("per_layer: the headline steps as ikv_step_begin / one ikv_step_layer per layer / ikv_step_end, "
+                     "one CUDA graph per step; with_foreign: each layer's q, k_new, v_new first copied by 3 PyTorch "
+                     "kernels (not counted in gpu_launches).  trajectory: every decode step of the configuration "
+                     "from step 1 (which evicts ~90% of the prefill), deferred compactions included, one graph per "
+                     "step.  per_config: the other workloads with their headline schedules, at most 20 timed steps "
+                     "after 3 warm-up steps; attend_frac / attend_score_ema_frac of the measured copy peak from "
+                     "eager events; speedup_vs_full on the same inputs.  sweep (Qwen-shaped, b=32, 16k): tok/s per "
+                     "budget (%) x refresh period r, Lazy speedup over r = 1, alpha at 10% / r = 1.")
+    # the last keys: the driver keeps the tail of the line
+    line["per_layer"] = {"value": sig(job_throughput(w.batch * K, world, per_layer["split"]["ms"])),
+                         "us_per_step": sig(1e3 * per_layer["split"]["ms"] / K),
+                         "vs_whole_step": sig(full["ms"] / per_layer["split"]["ms"]),
+                         "gpu_launches": per_layer["split"]["launches"],
+                         "with_foreign_value": sig(job_throughput(w.batch * K, world, per_layer["foreign"]["ms"]))}
+    line["trajectory"] = {"steps": traj_w.steps, "value": sig(job_throughput(w.batch * traj_w.steps, world, traj_ms)),
+                          "ms": sig(traj_ms)}
+    if others:
+        sweep = others["4"].pop("sweep", None)
+        line["per_config"] = others
+        if sweep:
+            line["sweep"] = sweep
     print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()
