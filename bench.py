@@ -660,6 +660,21 @@ def run_other_config(args, cfg: int, dev, dist, rank: int, compact_mode, mh_arg:
     return res
 
 
+def trace_ratios(counts):
+    """The Appendix's rank-trace measures from one step's overlap counts per utility row,
+    {|R & R_prev|, |E & E_prev|, |R & E|, |R|, |E|} (ikv_trace.counts): EMA churn, and on
+    steps with a raw top-k its churn, the raw/EMA Jaccard and the raw-top evicted fraction."""
+    out = []
+    for rr, re_, rx, nr, ne in counts:
+        row = {"ema_churn": 1.0 - re_ / ne if ne > 0 else None}
+        if nr > 0:
+            row["raw_churn"] = 1.0 - rr / nr
+            row["jaccard"] = rx / (nr + ne - rx)
+            row["raw_top_evicted"] = 1.0 - rx / nr
+        out.append(row)
+    return out
+
+
 def run_trace(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, mh: int = 0):
     """Rank-trace diagnostics (raw / EMA top-k churn, raw/EMA Jaccard, raw-top evicted)
     over the timed steps of one schedule, launched eagerly with ikv_params.trace set;
@@ -681,7 +696,7 @@ def run_trace(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, mh: i
                      ws.numel(), torch.cuda.current_stream())
         lens, live = step_lengths(lens, live, budgets, mh)
         if t > W:  # churn compares with the previous traced step, so the first timed step has one
-            for row in tr.stats():
+            for row in trace_ratios(tr.counts.cpu().tolist()):
                 for k, v in row.items():
                     if v is not None and k in acc:
                         acc[k].append(v)

@@ -218,6 +218,14 @@ int64_t ikv_launch_count(void);
  * was dropped); bit 4: a rank-trace set exceeded 16384 tokens (not traced). */
 ikv_status ikv_device_status(uint32_t *flags);
 
+/* Test of the bounded waits (no counterpart in the paper): the next tensor-core attention
+ * launch of this process starts with a wait, limited to 10 us, on a barrier that nothing
+ * arrives at.  The wait runs out, so every CTA of that launch takes the timeout path --
+ * abort flag, bit 0 of the device error word, its in-flight copies drained, TMEM freed --
+ * and its outputs are undefined; later launches run normally.  Nothing faults or hangs.
+ * Host only; launches nothing. */
+ikv_status ikv_test_stall_next_attention(void);
+
 /* Which decode-attention kernel ikv_decode_attend_score and ikv_step launch for
  * this shape and cache (all layers, cache->max_len):
  * IKV_PATH_TENSOR_CORE -- TMA-staged K/V tiles, tcgen05 QK^T and PV with TMEM

@@ -209,16 +209,3 @@ class RankTrace:
 
     def reset(self) -> None:
         self.n_top.zero_()
-
-    def stats(self):
-        """Per row: raw churn, EMA churn, raw/EMA Jaccard, raw-top evicted (None where the
-        step had no raw score or nothing to compare with)."""
-        out = []
-        for rr, re_, rx, nr, ne in self.counts.cpu().tolist():
-            row = {"ema_churn": 1.0 - re_ / ne if ne > 0 else None}
-            if nr > 0:
-                row["raw_churn"] = 1.0 - rr / nr
-                row["jaccard"] = rx / (nr + ne - rx)
-                row["raw_top_evicted"] = 1.0 - rx / nr
-            out.append(row)
-        return out

@@ -25,6 +25,8 @@
 // warp 4 issues TMA loads, warp 5 issues MMAs.  Every mbarrier wait is bounded;
 // on timeout the CTA records an error code, stops issuing work, waits for its
 // in-flight copies and MMAs, frees its TMEM and returns.
+#include <atomic>
+
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -53,8 +55,10 @@ constexpr int kOffQ = kNst * kStage;
 constexpr int kOffP = kOffQ + kOpBytes;
 constexpr int kOffRed = kOffP + 2 * kOpBytes;
 constexpr int kOffBar = kOffRed + 4 * kN * 4;
-// barriers: full[kNst], empty[kNst], s_full, p_full[2], p_empty[2], o_full, s_free, o_free, mma_done
-constexpr int kNumBar = 2 * kNst + 9;
+// barriers: full[kNst], empty[kNst], s_full, p_full[2], p_empty[2], o_full, s_free, o_free, mma_done,
+// stall (the bounded-wait test's barrier, which nothing arrives at)
+constexpr int kNumBar = 2 * kNst + 10;
+constexpr uint64_t kStallNs = 10000ull;       // the bounded-wait test's limit: 10 us
 constexpr int kOffMisc = kOffBar + kNumBar * 8;
 constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // misc: tmem slot, abort flag, last-split flag   // + slack for 1024-byte alignment
 
@@ -93,6 +97,9 @@ struct TcArgs {
     // split step: len, start, slot, pos, the block table and this layer's cached rows are
     // fixed since the step's first call)
     int32_t early;
+    // nonzero (tests of the bounded waits): the MMA issuer first waits, at most kStallNs, on a
+    // barrier that nothing arrives at, so the wait runs out and the CTA takes its abort path
+    int32_t stall;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -125,7 +132,8 @@ __device__ __forceinline__ uint64_t global_ns() {
 // time).  Returns false -- raising the CTA's abort flag and the global error
 // word -- if the phase does not complete in time, or returns false at once if
 // another role of the CTA has already aborted.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort) {
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort,
+                                          uint64_t limit_ns = kWaitNs) {
     if (mbar_test(bar, parity)) return true;
     const uint64_t start = global_ns();
     for (uint32_t i = 1;; ++i) {
@@ -133,7 +141,7 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
         if (i > 64) __nanosleep(32);
         if ((i & 63u) == 0) {
             if (*abort) return false;
-            if (global_ns() - start > kWaitNs) break;
+            if (global_ns() - start > limit_ns) break;
         }
     }
     *abort = 1;
@@ -302,6 +310,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     const uint32_t s_free = bar0 + 8u * (2 * kNst + 6);  // the softmax is done with a pass's S tiles
     const uint32_t o_free = bar0 + 8u * (2 * kNst + 7);  // the softmax has read a pass's O
     const uint32_t mma_done = bar0 + 8u * (2 * kNst + 8);  // every MMA of the CTA has completed
+    const uint32_t stall_bar = bar0 + 8u * (2 * kNst + 9);  // nothing arrives here (a.stall)
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(sm + kOffMisc);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + kOffMisc + 4);
 
@@ -366,6 +375,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         mbar_init(s_free, 128);
         mbar_init(o_free, 128);
         mbar_init(mma_done, 1);
+        mbar_init(stall_bar, 1);
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         while (ld_J < kNst && ld_p < np && !blocked(ld_p, ld_j)) issue_next();
@@ -460,8 +470,9 @@ __global__ void __launch_bounds__(kThreads, 2)
                 if (!mbar_wait(empty(st), ((ld_J / kNst) - 1) & 1, abort_flag)) break;
                 issue_next();
             }
-            // drain: the last phase issued on each stage must have landed before the CTA exits
-            for (int j = ld_J - 1; j >= 0 && j >= ld_J - kNst; --j) (void)mbar_wait(full(j % kNst), (j / kNst) & 1, abort_flag);
+            // drain: the last phase issued on each stage must have landed before the CTA exits,
+            // also after an abort (mbar_drain does not give up when the abort flag is set)
+            for (int j = ld_J - 1; j >= 0 && j >= ld_J - kNst; --j) mbar_drain(full(j % kNst), (j / kNst) & 1);
         }
         __syncwarp();
     } else if (warp == 5) {
@@ -471,6 +482,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             constexpr uint32_t id_pv = idesc_bf16(true, 128, kN);
             bool ok = true;
             int J = 0, Q = 0;  // loads and P tiles consumed so far
+            if (a.stall) ok = mbar_wait(stall_bar, 0, abort_flag, kStallNs);  // runs out: abort
             for (int p = 0; p < np && ok; ++p) {
                 const int n = chunk_n(p);
                 // the S tiles of the previous pass must have been read
@@ -909,6 +921,8 @@ int tc_passes(int64_t units, int n_chunks, int sms, bool gsum) {
     return n_chunks;
 }
 
+std::atomic<int> g_stall_next{0};
+
 cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group, int sms, cudaStream_t st) {
     const int rpb = a.pv.page_size >= kTile ? kTile : a.pv.page_size;
     // rows of every layer the launch can touch: [layers][num_pages][kv_heads][page_size]
@@ -952,6 +966,7 @@ cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group,
     t.vnorm = a.vnorm;
     t.gsum = a.gsum;
     t.early = a.early;
+    t.stall = g_stall_next.exchange(0);
     const int64_t units = (int64_t)a.pv.kv_heads * a.batch * a.n_layers;
     t.passes = tc_passes(units, a.n_splits, sms, a.gsum != 0);
     dim3 grid((unsigned)(((a.n_splits + t.passes - 1) / t.passes) * units));
@@ -969,6 +984,11 @@ cudaError_t launch_attend_tc(const AttendArgs &a, const TcOutputs &o, int group,
 }
 
 }  // namespace ikv
+
+extern "C" ikv_status ikv_test_stall_next_attention(void) {
+    ikv::g_stall_next.store(1);
+    return IKV_OK;
+}
 
 extern "C" ikv_status ikv_device_status(uint32_t *flags) {
     if (!flags) return ikv::report(IKV_ERR_ARG, "flags is NULL");

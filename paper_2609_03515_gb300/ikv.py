@@ -72,6 +72,7 @@ def _load():
         "ikv_last_error": ([], ctypes.c_char_p),
         "ikv_launch_count": ([], ctypes.c_int64),
         "ikv_device_status": ([ctypes.POINTER(ctypes.c_uint32)], I32),
+        "ikv_test_stall_next_attention": ([], I32),
         "ikv_attend_path": ([SP, CP, ctypes.POINTER(I32)], I32),
         "ikv_attend_plan": ([SP, CP, I32, I32] + [ctypes.POINTER(I32)] * 5, I32),
         "ikv_attend_workspace_size": ([SP, CP, ctypes.POINTER(SZ)], I32),
@@ -133,6 +134,10 @@ def ikv_device_status() -> int:
     v = ctypes.c_uint32(0)
     _check(_lib.ikv_device_status(ctypes.byref(v)), "ikv_device_status")
     return int(v.value)
+
+
+def ikv_test_stall_next_attention() -> None:
+    _check(_lib.ikv_test_stall_next_attention(), "ikv_test_stall_next_attention")
 
 
 def ikv_attend_path(shape: ikv_shape, cache: ikv_cache) -> int:

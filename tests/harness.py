@@ -123,6 +123,64 @@ def boundary_ok(m_o: np.ndarray, kept_mask: np.ndarray, budget: int, gap: float 
     return ok, float(theta)
 
 
+class Canaries:
+    """Guard regions around every buffer a step writes, each holding a fixed bit pattern
+    that no call may change (the substitute for a memory checker on this GPU pool):
+      - spare pages in the K/V pools, interleaved at random with the used pages and never
+        named by the block table;
+      - tails after pos, ema and (with VNorm) vnorm;
+      - a tail after the workspace.
+    Install on a fresh DecodeCache before its prefill is written; check() after each call."""
+
+    TAIL = 1024  # elements (bytes for the workspace)
+
+    def __init__(self, c: DecodeCache, ws_bytes: int, seed: int = 11):
+        self.c = c
+        dev = c.k.device
+        P = c.num_pages
+        S = max(2, P // 3)
+        rng = np.random.default_rng(seed)
+        perm = rng.permutation(P + S)
+        self.spare = torch.from_numpy(np.sort(perm[P:]).astype(np.int64)).to(dev)
+        bt = perm[:P][c.block_table.cpu().numpy()]
+        shp = list(c.k.shape)
+        shp[1] = P + S
+        self.ik = torch.int16 if c.k.dtype == torch.bfloat16 else torch.int32
+        self.kpat = 0x7F7F if self.ik == torch.int16 else 0x7F7F7F7F  # finite values, never read
+        for name in ("k", "v"):
+            pool = torch.empty(shp, dtype=c.k.dtype, device=dev)
+            pool.view(self.ik).fill_(self.kpat)
+            used = torch.from_numpy(perm[:P].astype(np.int64)).to(dev)
+            pool[:, used] = getattr(c, name)
+            setattr(c, name, pool)
+        c.block_table = torch.from_numpy(bt.astype(np.int32)).to(dev)
+        c.num_pages = P + S
+        self.tails = {}
+        for name in ("pos", "ema", "vnorm"):
+            t = getattr(c, name)
+            if t is None:
+                continue
+            n = t.numel()
+            big = torch.empty(n + self.TAIL, dtype=t.dtype, device=dev)
+            big.view(torch.int32).fill_(0x5A5AA5A5)
+            big[:n].copy_(t.reshape(-1))
+            setattr(c, name, big[:n].view(t.shape))
+            self.tails[name] = big[n:]
+        self.ws_big = torch.zeros(ws_bytes + self.TAIL, dtype=torch.uint8, device=dev)
+        self.ws_big[ws_bytes:].fill_(0xA5)
+        self.ws = self.ws_big[:ws_bytes]
+        self.ws_bytes = ws_bytes
+
+    def check(self, where=""):
+        c = self.c
+        for name in ("k", "v"):
+            pages = getattr(c, name)[:, self.spare].contiguous().view(self.ik)
+            assert bool((pages == self.kpat).all()), f"{where}: a spare {name} page was written"
+        for name, t in self.tails.items():
+            assert bool((t.view(torch.int32) == 0x5A5AA5A5).all()), f"{where}: the tail after {name} was written"
+        assert bool((self.ws_big[self.ws_bytes:] == 0xA5).all()), f"{where}: the tail after the workspace was written"
+
+
 @dataclass
 class StepReport:
     t: int
@@ -161,10 +219,12 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
                  steps: Optional[int] = None, kv_check_layers=(0, -1), page_perm_seed: Optional[int] = 7,
                  refresh_init: int = ikv.IKV_INIT_ZERO, layer_eligible=None, max_holes: int = 0,
                  agg_mode: int = ikv.IKV_AGG_EMA, scorer: int = ikv.IKV_SCORE_ATTENTION,
-                 per_layer: bool = False, trace: bool = False, ws_zeroed: bool = False) -> List[StepReport]:
+                 per_layer: bool = False, trace: bool = False, ws_zeroed: bool = False,
+                 canaries: bool = False) -> List[StepReport]:
     T = w.steps if steps is None else steps
     u = w.u_table()
     c = make_cache(w, gran, page_perm_seed, value_norms=scorer == ikv.IKV_SCORE_VNORM)
+    guard = Canaries(c, c.step_workspace().numel()) if canaries else None
     kv = fill_prefill(c, w, u)
     if c.vnorm is not None:
         ikv.ikv_value_norms(c.shape(), c.cache(max(w.prefill)))
@@ -182,7 +242,7 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
     tr = RankTrace(c) if trace else None
     p = c.params(w.alpha, w.refresh_period, w.score_free, compact_mode, refresh_init, layer_eligible, max_holes,
                  agg_mode, scorer, trace=tr, ws_zeroed=ws_zeroed)
-    ws = c.step_workspace()
+    ws = c.step_workspace() if guard is None else guard.ws
     qs = w.queries(1, T + 1, u)
     prev_sets = [(np.zeros(0, np.int64), np.zeros(0, np.int64))] * (w.batch * c.rows_per_seq)
     budgets = w.budgets()
@@ -197,6 +257,8 @@ def run_lockstep(w: gen.Workload, gran: int = ikv.IKV_GRAN_SEQ, compact_mode: in
                     ws, per_layer)
         lens, live = step_lengths(lens, live, budgets, max_holes)
         torch.cuda.synchronize()
+        if guard is not None:
+            guard.check(f"step {t}")
         out_h = out.cpu().float().numpy()
         ema_h = c.ema.cpu().numpy()
         pos_h = c.pos.cpu().numpy()

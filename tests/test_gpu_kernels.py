@@ -637,3 +637,37 @@ def test_compact_short_side_relocates_and_skips_in_place():
             for g in range(2):
                 assert np.array_equal(c.gather(c.k, b, l, g, n).float().cpu().numpy(), k[g])
                 assert np.array_equal(c.gather(c.v, b, l, g, n).float().cpu().numpy(), v[g])
+
+
+def test_bounded_wait_runs_out_and_the_next_launch_is_correct():
+    """The tensor-core kernel's waits are bounded.  ikv_test_stall_next_attention makes the
+    next launch start with a wait (10 us) on a barrier nothing arrives at: every CTA takes its
+    timeout path (abort flag, in-flight copies drained, TMEM freed, no fault), the device
+    error word reports bit 0, and the following launch on the same inputs is correct."""
+    w = gen.Workload("stall", 2, 2, 32, 8, 128, [700, 200], 1, dtype=gen.BF16, seed=29, page_size=64)
+    u = w.u_table()
+    c = make_cache(w, page_perm_seed=3)
+    fill_device(c, w, torch.from_numpy(u).cuda())
+    cch = c.cache(max(w.prefill))
+    assert ikv.ikv_attend_path(c.shape(), cch) == ikv.IKV_PATH_TENSOR_CORE
+    layer = 1
+    q_h = w.queries(1, 2, u)[0, layer]
+    q = to_device(q_h, w)
+    ws = torch.empty(ikv.ikv_attend_workspace_size(c.shape(), cch), dtype=torch.uint8, device="cuda")
+    out = torch.empty((w.batch, w.q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+    score = torch.zeros((c.rows, c.cap), device="cuda")
+    assert ikv.ikv_device_status() == 0
+    ikv.ikv_test_stall_next_attention()
+    ikv.ikv_decode_attend_score(c.shape(), cch, layer, q, out, score, None, 0.0, ws, ws.numel())
+    torch.cuda.synchronize()
+    assert ikv.ikv_device_status() & 1          # the wait ran out; the context is intact
+    assert ikv.ikv_device_status() == 0         # and the word was cleared
+    ikv.ikv_decode_attend_score(c.shape(), cch, layer, q, out, score, None, 0.0, ws, ws.numel())
+    torch.cuda.synchronize()
+    assert ikv.ikv_device_status() == 0
+    q64 = as_f64(q_h, w)
+    for b, L in enumerate(w.prefill):
+        k, v = w.kv_block(b, layer, 0, L, u)
+        a, o = O.last_query_attention(q64[b], [x.astype(np.float64) for x in k], [x.astype(np.float64) for x in v])
+        assert np.max(np.abs(out[b].cpu().float().numpy() - o)) < 2e-2
+        assert np.max(np.abs(score[b, :L].cpu().numpy() - O.pooled_score(a, O.GRAN_SEQ, w.kv_heads)[0])) < 2e-5

@@ -281,3 +281,26 @@ def test_workspace_kept_zero_across_steps():
     _assert(run_lockstep(small_llama(steps=9, refresh_period=3), max_holes=3, ws_zeroed=True,
                          compact_mode=ikv.IKV_COMPACT_STABLE_SHORT), 2e-2)
     _assert(run_lockstep(small_llama(steps=6), per_layer=True, ws_zeroed=True), 2e-2)
+
+
+@pytest.mark.parametrize("case", [
+    dict(compact_mode=ikv.IKV_COMPACT_STABLE_SHORT, max_holes=2),     # prefix moves right, start advances
+    dict(compact_mode=ikv.IKV_COMPACT_STABLE_SHORT, tight=True),      # append at cap - 1, relocation to slot 0
+    dict(compact_mode=ikv.IKV_COMPACT_HOLEFILL, scorer=ikv.IKV_SCORE_VNORM),
+    dict(compact_mode=ikv.IKV_COMPACT_STABLE, gran=ikv.IKV_GRAN_KVHEAD),
+    dict(compact_mode=ikv.IKV_COMPACT_STABLE_SHORT, max_holes=3, per_layer=True),
+], ids=["short_deferred", "short_tight_cap", "holefill_vnorm", "stable_kvhead", "split_step"])
+def test_nothing_written_outside_the_buffers(case):
+    """Canaries around every buffer (spare pool pages among the used ones, tails after pos,
+    ema, vnorm and the workspace) stay intact through lock-step runs that exercise the
+    shorter-side moves (right moves, relocation to slot 0), an append into the last slot of
+    the slot space, hole-fill with value norms, KV-head rows and the split step."""
+    case = dict(case)
+    tight = case.pop("tight", False)
+    if tight:
+        # cap = 320 slots: sequence 0's first append lands in slot 319, and the shorter-side
+        # compaction runs out of room on the right
+        w = small_llama(prefill=[319, 200], batch=2, steps=8, budget_frac=0.5)
+    else:
+        w = small_llama(steps=6)
+    _assert(run_lockstep(w, canaries=True, **case), 2e-2)
