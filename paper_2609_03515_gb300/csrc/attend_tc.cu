@@ -48,13 +48,15 @@ constexpr int kOpBytes = kN * kD * 2;           // 4 KB: Q or one P operand
 constexpr int kTmemCols = 256;
 constexpr int kOcol = kTmemCols - kN;           // O accumulator columns [240, 256)
 constexpr int kMaxTiles = kOcol / kN;           // 15 S tiles
+constexpr int kEarlyChunks = 16;                // merge: partial outputs loaded with the (max, sum) pairs
 constexpr int kThreads = 192;
 constexpr uint64_t kWaitNs = 1000000000ull;   // 1 s: orders of magnitude above any legitimate wait
 
 constexpr int kOffQ = kNst * kStage;
 constexpr int kOffP = kOffQ + kOpBytes;
 constexpr int kOffRed = kOffP + 2 * kOpBytes;
-constexpr int kOffBar = kOffRed + 4 * kN * 4;
+constexpr int kOffNew = kOffRed + 4 * kN * 4;   // split step: the new token's K and V rows (2 x 256 B)
+constexpr int kOffBar = kOffNew + 2 * kD * 2;
 // barriers: full[kNst], empty[kNst], s_full, p_full[2], p_empty[2], o_full, s_free, o_free, mma_done,
 // stall (the bounded-wait test's barrier, which nothing arrives at)
 constexpr int kNumBar = 2 * kNst + 10;
@@ -178,6 +180,9 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
         : "memory");
 }
 
+__device__ __forceinline__ void bulk_prefetch_l2(const void *p, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
 __device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap *map, int x, int y) {
     asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(map)),
                  "r"(x), "r"(y)
@@ -328,19 +333,15 @@ __global__ void __launch_bounds__(kThreads, 2)
     };
     int ld_J = 0, ld_p = 0, ld_j = 0;  // producer cursor: loads issued, pass and load of the next one
     const uint64_t kv_pol = l2_evict_first();
-    // split step: the physical slot that receives the new token's rows (-1: none here); a
-    // load of the tile holding it waits until this CTA has stored them
+    // split step: the physical slot that receives the new token's rows (-1: none, or not in
+    // this CTA's chunks).  The tiles holding it are loaded like any other; the MMA thread
+    // writes the new rows into the loaded K and V tiles before their products read them.
     int p_new = -1;
     if (a.k_new) {
         const int j = __ldcg(a.slot + b);
-        if (j >= 0) p_new = S0 + j;
+        const int pn = S0 + j;
+        if (j >= 0 && pn >= chunk_t0(0) && pn < chunk_t0(np - 1) + chunk_n(np - 1) * kTile) p_new = pn;
     }
-    auto blocked = [&](int p, int j) {
-        if (p_new < 0) return false;
-        const int n = chunk_n(p);
-        const int t0 = chunk_t0(p) + (j < n ? j : j - n) * kTile;
-        return p_new >= t0 && p_new < t0 + kTile;
-    };
     auto issue_next = [&]() {
         const int st = ld_J % kNst;
         mbar_expect_tx(full(st), kStage);
@@ -358,9 +359,9 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
     };
     // Prologue.  The producer lane initialises the barriers and starts the K/V stream at
-    // once (every load up to the ring's depth that does not read the new token's tile);
-    // the TMEM allocation and P zeroing below overlap the loads' latency.  An early CTA
-    // does all of this before the dependency wait, so it overlaps the previous kernel's tail.
+    // once (every load up to the ring's depth); the TMEM allocation and P zeroing below
+    // overlap the loads' latency.  An early CTA does all of this before the dependency
+    // wait, so it overlaps the previous kernel's tail.
     if (warp == 4 && lane == 0) {
         for (int i = 0; i < kNst; ++i) {
             mbar_init(full(i), 1);
@@ -378,25 +379,24 @@ __global__ void __launch_bounds__(kThreads, 2)
         mbar_init(stall_bar, 1);
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        while (ld_J < kNst && ld_p < np && !blocked(ld_p, ld_j)) issue_next();
-        // an early CTA also pulls the rest of its tiles into L2 while it waits, so the loads
-        // it can only issue once the ring turns over find them there (the new token's tile is
-        // left out: its rows change before it is read)
+        while (ld_J < kNst && ld_p < np) issue_next();
+        // an early CTA also pulls the rest of its tiles, and its q rows, into L2 while it
+        // waits, so the loads it can only issue later find them there (a prefetch cannot
+        // return stale data: L2 is where writes land)
         if (early) {
             for (int p = ld_p, j = ld_j; p < np;) {
-                if (!blocked(p, j)) {
-                    const CUtensorMap *tm = j < chunk_n(p) ? &tmK : &tmV;
-                    for (int bx = 0; bx < boxes; ++bx) {
-                        const int row = box_row(p, j, bx);
-                        tma_prefetch_2d(tm, 0, row);
-                        tma_prefetch_2d(tm, 64, row);
-                    }
+                const CUtensorMap *tm = j < chunk_n(p) ? &tmK : &tmV;
+                for (int bx = 0; bx < boxes; ++bx) {
+                    const int row = box_row(p, j, bx);
+                    tma_prefetch_2d(tm, 0, row);
+                    tma_prefetch_2d(tm, 64, row);
                 }
                 if (++j == 2 * chunk_n(p)) {
                     ++p;
                     j = 0;
                 }
             }
+            bulk_prefetch_l2(a.q + (((int64_t)li * a.batch + b) * a.q_heads + (int64_t)g * G) * kD, G * kD * 2);
         }
     }
     if (warp == 0) {
@@ -411,18 +411,20 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (early) pdl_wait();
     if (warp == 4) {
         // Split step: the CTA whose chunks hold the new token's slot stores the token's K
-        // and V rows into the cache (lanes 0-15: K, 16-31: V, 16 bytes each) before its
-        // TMA loads read that tile; the proxy fence orders the stores before them.
+        // and V rows into the cache (lanes 0-15: K, 16-31: V, 16 bytes each) for later steps,
+        // and stages them in shared memory for its own MMAs (the tiles it loads may hold the
+        // slot's old contents: the MMA thread overwrites that row before using them)
         if (a.k_new) {
             const int j = p_new - S0;
             const int p = p_new;
-            if (p_new >= 0 && p >= chunk_t0(0) && p < chunk_t0(np - 1) + chunk_n(np - 1) * kTile) {
+            if (p_new >= 0) {
                 const int page = a.block_table[(int64_t)b * a.max_pages + p / a.page_size];
                 const int64_t row = ((int64_t)(l * a.num_pages + page) * a.kv_heads + g) * a.page_size + p % a.page_size;
                 const bool isv = lane >= 16;
                 const int c = lane & 15;
                 const uint4 x = reinterpret_cast<const uint4 *>(isv ? a.v_new : a.k_new)[((int64_t)b * a.kv_heads + g) * 16 + c];
                 reinterpret_cast<uint4 *>(isv ? a.v_pool : a.k_pool)[row * 16 + c] = x;
+                reinterpret_cast<uint4 *>(sm + kOffNew)[lane] = x;
                 float sq = 0.f;
                 if (isv) {
                     const uint32_t w4[4] = {x.x, x.y, x.z, x.w};
@@ -436,14 +438,9 @@ __global__ void __launch_bounds__(kThreads, 2)
                 for (int o = 8; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
                 if (a.vnorm && lane == 16)
                     a.vnorm[(((int64_t)l * a.batch + b) * a.kv_heads + g) * a.cap + j] = sqrtf(sq);
-                asm volatile("fence.proxy.async.global;" ::: "memory");
             }
             __syncwarp();
         }
-        // the rest of the ring's first fill (the loads the new token's rows held back)
-        if (lane == 0)
-            while (ld_J < kNst && ld_p < np) issue_next();
-        __syncwarp();
     }
     // Q operand [16 heads][128 dims], heads >= G zero: one 16-byte load per thread (8 dims
     // of one head, which stay together as one 16-byte chunk of the swizzled layout)
@@ -480,6 +477,17 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (lane == 0) {
             constexpr uint32_t id_qk = idesc_bf16(false, 128, kN);
             constexpr uint32_t id_pv = idesc_bf16(true, 128, kN);
+            // the new token's K (which = 0) or V (1) row over tile row r of ring stage st, in
+            // the 128-byte swizzle the TMA wrote; the proxy fence orders the stores before the
+            // MMAs that read the stage
+            auto patch_new_row = [&](int st, int r, int which) {
+                const uint4 *src = reinterpret_cast<const uint4 *>(sm + kOffNew) + which * 16;
+                unsigned char *tile = sm + st * kStage;
+#pragma unroll
+                for (int c = 0; c < 16; ++c)
+                    *reinterpret_cast<uint4 *>(tile + (c >> 3) * kHalf + r * 128 + ((((c & 7) ^ r) & 7) << 4)) = src[c];
+                fence_async_smem();
+            };
             bool ok = true;
             int J = 0, Q = 0;  // loads and P tiles consumed so far
             if (a.stall) ok = mbar_wait(stall_bar, 0, abort_flag, kStallNs);  // runs out: abort
@@ -492,6 +500,8 @@ __global__ void __launch_bounds__(kThreads, 2)
                     const int st = (J + i) % kNst;
                     if (!(ok = mbar_wait(full(st), ((J + i) / kNst) & 1, abort_flag))) break;
                     fence_after_sync();
+                    const int rn = p_new - (chunk_t0(p) + i * kTile);
+                    if (p_new >= 0 && rn >= 0 && rn < kTile) patch_new_row(st, rn, 0);
                     const uint32_t ka = base + st * kStage;
 #pragma unroll
                     for (int kk = 0; kk < kD / 16; ++kk) {
@@ -511,6 +521,8 @@ __global__ void __launch_bounds__(kThreads, 2)
                     if (!(ok = mbar_wait(full(st), ((J + i) / kNst) & 1, abort_flag))) break;
                     if (!(ok = mbar_wait(p_full(q & 1), (q >> 1) & 1, abort_flag))) break;
                     fence_after_sync();
+                    const int rn = p_new - (chunk_t0(p) + i * kTile);
+                    if (p_new >= 0 && rn >= 0 && rn < kTile) patch_new_row(st, rn, 1);
                     const uint32_t va = base + st * kStage;
                     const uint32_t pb = sP + (q & 1) * kOpBytes;
 #pragma unroll
@@ -755,6 +767,14 @@ __global__ void __launch_bounds__(kThreads, 2)
                 // few L2 round trips whatever the number of partials.
                 for (int h = warp; h < G; h += 4) {
                     const float2 *ml = reinterpret_cast<const float2 *>(a.part_ml) + pbase + (int64_t)h * a.n_splits;
+                    // the first kEarlyChunks partial outputs are loaded together with the
+                    // (max, sum) pairs: their addresses do not depend on the weights
+                    const float4 *po =
+                        reinterpret_cast<const float4 *>(a.part_o + (pbase + (int64_t)h * a.n_splits) * kD) + lane;
+                    float4 ov0[kEarlyChunks];
+#pragma unroll
+                    for (int j = 0; j < kEarlyChunks; ++j)
+                        ov0[j] = j < nc_unit ? __ldcg(po + (int64_t)j * (kD / 4)) : make_float4(0.f, 0.f, 0.f, 0.f);
                     float mv[kMaxSplits / 32], lv[kMaxSplits / 32];
                     float Mh = -INFINITY;
 #pragma unroll
@@ -779,10 +799,16 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
                     for (int o = 16; o > 0; o >>= 1) Wh += __shfl_xor_sync(0xffffffffu, Wh, o);
                     __syncwarp();
-                    const float4 *po =
-                        reinterpret_cast<const float4 *>(a.part_o + (pbase + (int64_t)h * a.n_splits) * kD) + lane;
                     float4 sacc = make_float4(0.f, 0.f, 0.f, 0.f);
-                    for (int q0 = 0; q0 < nc_unit; q0 += 8) {
+#pragma unroll
+                    for (int j = 0; j < kEarlyChunks; ++j) {
+                        const float wj = j < nc_unit ? wq[h * a.n_splits + j] : 0.f;
+                        sacc.x += wj * ov0[j].x;
+                        sacc.y += wj * ov0[j].y;
+                        sacc.z += wj * ov0[j].z;
+                        sacc.w += wj * ov0[j].w;
+                    }
+                    for (int q0 = kEarlyChunks; q0 < nc_unit; q0 += 8) {
                         float4 ov[8];
 #pragma unroll
                         for (int j = 0; j < 8; ++j)
