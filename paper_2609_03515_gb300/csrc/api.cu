@@ -918,16 +918,28 @@ ikv_status ikv_step(const ikv_shape *shape, const ikv_params *p, ikv_cache *cach
     // kernel that counts leaves its counters zero again
     if ((e = zero_control_words(p, ws, w, stream))) return e;
     if (tm && (e = record(tm->begin, stream))) return e;
-    if ((e = append_impl(shape, cache, k_new, v_new, ema, cx.init_mean, at<int32_t>(ws, w.done), stream, true)))
+    // With the tensor-core attention the append is bookkeeping only (the new token's slot,
+    // position and utility; len += 1, one CTA per sequence): the attention CTA whose chunk
+    // holds the new slot stores that layer and KV head's rows itself and uses them in place
+    // of the slot's old contents.  The CUDA-core path appends the rows first.
+    const bool tc_rows = use_tc(shape, cache, shape->layers, cx.L1);
+    int32_t *slot = at<int32_t>(ws, w.slot);
+    if ((e = append_impl(shape, cache, tc_rows ? nullptr : k_new, tc_rows ? nullptr : v_new, ema, cx.init_mean,
+                         at<int32_t>(ws, w.done), stream, true, tc_rows ? slot : nullptr)))
         return e;
     if (tm && (e = record(tm->append_end, stream))) return e;
     // the rest of the chain may overlap each kernel's ramp-up with its predecessor's tail
     // (not when per-kernel events are recorded: those time each kernel alone)
     std::optional<PdlScope> pdl;
     if (!tm) pdl.emplace();
+    AppendArgs rows{};
+    rows.k_new = k_new;
+    rows.v_new = v_new;
+    rows.slot = slot;
+    rows.vnorm = cache->vnorm;
     bool gsum = false;  // the attention may hand over normalised group sums instead of logits
     if ((e = run_attend(shape, cache, 0, shape->layers, cx.L1, q, out, ws, w.at, cx.scoring, nullptr, nullptr, stream,
-                        tm, true, 0, 0, nullptr, &gsum)))
+                        tm, true, 0, 0, tc_rows ? &rows : nullptr, &gsum)))
         return e;
     if (tm && (e = record(tm->combine_end, stream))) return e;
     float *raw = p->trace ? at<float>(ws, w.raw) : nullptr;

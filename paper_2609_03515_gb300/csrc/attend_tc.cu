@@ -83,8 +83,9 @@ struct TcArgs {
     const int32_t *pos;         // [rows][cap], -1 at dead slots; null: every slot below len is live
     int32_t rows_per_seq;
     int32_t sc_layers, sc_layer0;  // local layer li is layer sc_layer0 + li of logits / lse2
-    // split step: the new token's K/V rows ([batch][kv_heads][128]) go to logical slot
-    // slot[b] (-1: none) before the attention reads it; vnorm (or null) gets its V norm
+    // the new token's K/V rows ([n_layers][batch][kv_heads][128]) go to logical slot slot[b]
+    // (-1: none), written by the CTA whose chunk holds it, which also uses them in place of
+    // the slot's old contents; vnorm (or null) gets their V norms
     const __nv_bfloat16 *k_new, *v_new;
     const int32_t *slot;
     __nv_bfloat16 *k_pool, *v_pool;
@@ -422,7 +423,8 @@ __global__ void __launch_bounds__(kThreads, 2)
                 const int64_t row = ((int64_t)(l * a.num_pages + page) * a.kv_heads + g) * a.page_size + p % a.page_size;
                 const bool isv = lane >= 16;
                 const int c = lane & 15;
-                const uint4 x = reinterpret_cast<const uint4 *>(isv ? a.v_new : a.k_new)[((int64_t)b * a.kv_heads + g) * 16 + c];
+                const uint4 x = reinterpret_cast<const uint4 *>(
+                    isv ? a.v_new : a.k_new)[(((int64_t)li * a.batch + b) * a.kv_heads + g) * 16 + c];
                 reinterpret_cast<uint4 *>(isv ? a.v_pool : a.k_pool)[row * 16 + c] = x;
                 reinterpret_cast<uint4 *>(sm + kOffNew)[lane] = x;
                 float sq = 0.f;

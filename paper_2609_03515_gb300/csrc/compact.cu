@@ -442,6 +442,18 @@ __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a
         }
     }
     __syncthreads();
+    if (gridDim.x == 1) {
+        // bookkeeping only (one CTA per sequence, which has read len[b] above): no arrival
+        if (tid == 0) {
+            if (S + L < a.cap) {
+                a.len[b] = L + 1;
+                a.next_pos[b] = a.next_pos[b] + 1;
+            } else {
+                atomicOr(&g_append_error, 1u);  // the token was not stored; ikv_device_status reports it
+            }
+        }
+        return;
+    }
     if (tid == 0) {
         __threadfence();
         const int prev = atomicAdd(&a.done[b], 1);
