@@ -712,8 +712,9 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
         }
 
-        if (nc_unit == 1) {
-            // the unit's only CTA: its output and log-sum-exp need no merge
+        if (MP || nc_unit == 1) {
+            // the unit's only CTA (always so in a multi-pass launch, whose CTAs take all of
+            // their unit's chunks): its output and log-sum-exp need no merge
             if (ok) {
 #pragma unroll
                 for (int h = 0; h < G; ++h)
