@@ -752,15 +752,12 @@ __global__ void __launch_bounds__(kThreads, 2)
             // The last CTA of (sequence, layer, kv head) to finish merges every CTA's
             // partial into the output and the per-head log-sum-exp.  Arrival counter
             // only: no CTA waits for another.
-            __threadfence();
-            __syncwarp();
             softmax_bar();
             int *last_flag = reinterpret_cast<int *>(sm + kOffMisc + 8);
             const int64_t unit = ((int64_t)b * a.n_layers + li) * a.kv_heads + g;
-            if (tid == 0) *last_flag = (atomicAdd(&a.arrivals[unit], 1) == nc_unit - 1) ? 1 : 0;
+            if (tid == 0) *last_flag = arrive_acq_rel(a.arrivals + unit) == nc_unit - 1 ? 1 : 0;
             softmax_bar();
             if (*last_flag && ok) {
-                __threadfence();
                 // partial weights [G][n_splits] in the P buffers (every MMA has completed)
                 float *wq = reinterpret_cast<float *>(sm + kOffP);
                 // warp w merges heads w, w + 4: (1) the partials' (max, sum) pairs give the

@@ -256,9 +256,7 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
     // publish len / start once every CTA of b has read them
     __syncthreads();
     if (tid == 0) {
-        __threadfence();
-        if (atomicAdd(&a.done[b], 1) == (int)gridDim.x - 1) {
-            __threadfence();
+        if (arrive_acq_rel(&a.done[b]) == (int)gridDim.x - 1) {
             a.len[b] = n0;
             if (a.start) a.start[b] = new_start;
             a.done[b] = 0;
@@ -455,10 +453,7 @@ __global__ void __launch_bounds__(kCompThreads) append_kernel(const AppendArgs a
         return;
     }
     if (tid == 0) {
-        __threadfence();
-        const int prev = atomicAdd(&a.done[b], 1);
-        if (prev == (int)gridDim.x - 1) {
-            __threadfence();
+        if (arrive_acq_rel(&a.done[b]) == (int)gridDim.x - 1) {
             if (S + L < a.cap) {
                 a.len[b] = L + 1;
                 a.next_pos[b] = a.next_pos[b] + 1;

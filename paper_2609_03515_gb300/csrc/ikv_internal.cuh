@@ -38,6 +38,17 @@ __device__ __forceinline__ void pdl_wait() {
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
+// A CTA's arrival on a counter shared by a group of CTAs, by one thread after a CTA
+// barrier: an acquire-release add, so it releases the CTA's stores (the barrier orders
+// the other threads' stores before it, and release is cumulative) and, for the last CTA
+// to arrive, acquires every other CTA's before the barrier that follows.  Returns the
+// count before the add.  (Measured: a gpu-scope fence on either side of a relaxed add
+// cost ~0.4 us more per arrival chain.)
+__device__ __forceinline__ int arrive_acq_rel(int *counter) {
+    int before;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;" : "=r"(before) : "l"(counter) : "memory");
+    return before;
+}
 template <typename... KArgs, typename... Args>
 cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args... args) {
     if (!pdl_enabled()) {

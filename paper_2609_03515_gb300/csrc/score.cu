@@ -285,13 +285,11 @@ __global__ void __launch_bounds__(kScoreThreads, 4) score_kernel(const ScoreArgs
     __shared__ int last;
     __syncthreads();
     if (threadIdx.x == 0) {
-        __threadfence();  // after the barrier: releases every thread's stores of this block
-        last = atomicAdd(a.row_done + r, 1) == blocks - 1;
+        last = arrive_acq_rel(a.row_done + r) == blocks - 1;
         if (last) a.row_done[r] = 0;
     }
     __syncthreads();
     if (!last) return;
-    __threadfence();
     // the blocks' partials give the live count and the victim candidate
     uint32_t cn = 0u;
     unsigned long long best = ~0ull;
