@@ -83,9 +83,11 @@ __global__ void __launch_bounds__(kScoreThreads, 4) score_kernel(const ScoreArgs
     const int r = blockIdx.y;
     const int lg = blockIdx.z, n_lg = gridDim.z;  // this CTA's layer group, and how many there are
     const int b = r / a.rows_per_seq;
+    // The row's length decides which tokens count, not which addresses are read (rows of
+    // the logits and the utility are padded past every block), so the loads below do not
+    // wait for it; a block past the length leaves once they are issued.
     const int L = a.len[b];
     const int i0 = blockIdx.x * kTok;
-    if (i0 >= L) return;
     const int il = i0 + lane * V;  // first token of this lane
     int h0 = 0, nh = a.q_heads;
     if (a.rows_per_seq > 1) {
@@ -100,7 +102,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) score_kernel(const ScoreArgs
     const int kw0 = lg * kScoreWarps;                        // the group's first eligible layer (pass index)
     const int n_here = min(kScoreWarps, a.n_elig - kw0);     // layers of this group
     float m = 0.f;
-    if (SCORER != IKV_SCORE_ENTROPY && folds && a.ema) m = a.ema[at];
+    if (SCORER != IKV_SCORE_ENTROPY && threadIdx.x < kTok && fi < a.cap && a.ema) m = a.ema[at];
     if (warp < n_here) {
         const int li = a.elig[kw0 + warp];
         // row padding keeps i0 + kTok <= lstride, so the vector loads stay inside the row
@@ -134,7 +136,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) score_kernel(const ScoreArgs
             VT z[kHB];
 #pragma unroll
             for (int j = 0; j < kHB; ++j) {
-                if (il < L && j < nb) z[j] = __ldg(reinterpret_cast<const VT *>(zp));
+                if (j < nb) z[j] = __ldg(reinterpret_cast<const VT *>(zp));
                 zp += a.lstride;
             }
             // each row's probabilities times the VNorm weight (1 for the other scorers)
@@ -195,6 +197,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) score_kernel(const ScoreArgs
             if (lane == 0) a.epart[((int64_t)r * (a.n_elig_total + 1) + k) * a.nblk + blockIdx.x] = e;
         }
     }
+    if (i0 >= L) return;  // every CTA of a cluster (one token block) leaves together
     if (SCORER == IKV_SCORE_ENTROPY) {
         if (warp == 0 && lg == 0) {  // live slots of this block (the entropy normalisation is ln of their count)
             float c = 0.f;
