@@ -449,14 +449,31 @@ int score_blocks(const ScoreArgs &a, int32_t max_len, int sms, int *V) {
     return (max_len + 32 * v - 1) / (32 * v);
 }
 
+// Shared memory a score CTA reserves so that no more than k CTAs share an SM, when the
+// whole grid fits at k per SM for some k < 4 (four fit by registers).  Left to itself the
+// block scheduler puts four CTAs on some SMs and one on others, and the most loaded SM
+// sets the pass's pace (config 1: 412 CTAs; with at most three per SM the graphed step
+// measured 81.7 -> 80.3 us).  Each size admits exactly k CTAs of this kernel (its static
+// shared memory and the 1 KB reserved per CTA included) in an SM's 228 KB.
+static size_t spread_smem(int64_t ctas, int sms) {
+    const int64_t k = sms > 0 ? (ctas + sms - 1) / sms : 4;
+    if (k >= 4 || k < 1) return 0;
+    return k == 3 ? 60 * 1024 : k == 2 ? 100 * 1024 : 150 * 1024;
+}
+constexpr size_t kScoreSmemAttr = 180 * 1024;  // dynamic shared-memory limit set once per instantiation
+static_assert(kVnormSmemMax <= kScoreSmemAttr, "VNorm staging within the limit");
+
 // The layer groups of a token block (grid z) run as one cluster.
 template <int V, int SCORER>
-static cudaError_t launch_score_v(const ScoreArgs &a, dim3 grid, cudaStream_t st) {
-    const size_t smem = SCORER == IKV_SCORE_VNORM ? vnorm_smem(a, V) : 0;
-    if (smem > 48 * 1024) {
+static cudaError_t launch_score_v(const ScoreArgs &a, dim3 grid, size_t reserve, cudaStream_t st) {
+    size_t smem = SCORER == IKV_SCORE_VNORM ? vnorm_smem(a, V) : 0;
+    if (smem < reserve) smem = reserve;
+    static bool limit_set = false;
+    if (!limit_set) {
         cudaError_t e = cudaFuncSetAttribute(score_kernel<V, SCORER>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)smem);
+                                             (int)kScoreSmemAttr);
         if (e != cudaSuccess) return e;
+        limit_set = true;
     }
     if (grid.z == 1) return launch_k(score_kernel<V, SCORER>, grid, dim3(kScoreThreads), smem, st, a);
     cudaLaunchConfig_t cfg{};
@@ -477,10 +494,10 @@ static cudaError_t launch_score_v(const ScoreArgs &a, dim3 grid, cudaStream_t st
 }
 
 template <int SCORER>
-static cudaError_t launch_score_t(const ScoreArgs &a, dim3 grid, int V, cudaStream_t st) {
-    if (V == 4) return launch_score_v<4, SCORER>(a, grid, st);
-    if (V == 2) return launch_score_v<2, SCORER>(a, grid, st);
-    return launch_score_v<1, SCORER>(a, grid, st);
+static cudaError_t launch_score_t(const ScoreArgs &a, dim3 grid, int V, size_t reserve, cudaStream_t st) {
+    if (V == 4) return launch_score_v<4, SCORER>(a, grid, reserve, st);
+    if (V == 2) return launch_score_v<2, SCORER>(a, grid, reserve, st);
+    return launch_score_v<1, SCORER>(a, grid, reserve, st);
 }
 
 cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, int sms, cudaStream_t st) {
@@ -489,13 +506,14 @@ cudaError_t launch_score_ema(const ScoreArgs &a, int32_t max_len, int sms, cudaS
     const int nblk = score_blocks(a, max_len, sms, &V);
     const int n_lg = score_layer_groups(a.n_elig);
     dim3 grid(nblk, (unsigned)(a.batch * a.rows_per_seq), (unsigned)n_lg);
+    const size_t reserve = spread_smem((int64_t)grid.x * grid.y * grid.z, sms);
     cudaError_t e;
     if (a.scorer == IKV_SCORE_VNORM)
-        e = launch_score_t<IKV_SCORE_VNORM>(a, grid, V, st);
+        e = launch_score_t<IKV_SCORE_VNORM>(a, grid, V, reserve, st);
     else if (a.scorer == IKV_SCORE_ENTROPY)
-        e = launch_score_t<IKV_SCORE_ENTROPY>(a, grid, V, st);
+        e = launch_score_t<IKV_SCORE_ENTROPY>(a, grid, V, reserve, st);
     else
-        e = launch_score_t<IKV_SCORE_ATTENTION>(a, grid, V, st);
+        e = launch_score_t<IKV_SCORE_ATTENTION>(a, grid, V, reserve, st);
     if (e != cudaSuccess) return e;
     note_launch();
     return cudaGetLastError();
