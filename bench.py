@@ -86,7 +86,7 @@ def rank_seed(base_seed: int, rank: int) -> int:
 
 
 # revision of each attention kernel; a committed ncu summary counts only for its own revision
-ATTEND_KERNEL_REV = {"attend_tc_kernel": "attend_tc_v12", "attend_split_kernel": "attend_split_v2"}
+ATTEND_KERNEL_REV = {"attend_tc_kernel": "attend_tc_v13", "attend_split_kernel": "attend_split_v2"}
 
 
 def schedule_name(w) -> str:
