@@ -709,12 +709,12 @@ def run_trace(args, w, c, u_dev, qs_dev, kn_dev, vn_dev, ws, compact_mode, mh: i
 def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist, mh: int = 0, scorer: int = 0):
     """Same steps through the C ABI, inputs from pinned host memory and the output read back every step.
 
-    Two buffer sets and one copy stream per direction: the upload of step t+1's inputs
-    and the read-back of step t-1's output run while step t computes.  Every step's copies lie inside the
-    timed region (the compute stream waits for the copy stream before the stop event).
-    After the eager warm-up, each timed step replays ikv_step from a CUDA graph captured
-    for its kind (refresh / carry-over) and buffer set, so a stall of the host thread does
-    not leave the GPU idle."""
+    Two device buffer sets: the upload of step t+1's inputs and the read-back of step t-1's
+    output run while step t computes.  The warm-up launches the steps eagerly with one copy
+    stream per direction.  Each timed step then replays a CUDA graph captured for it that
+    holds ikv_step(t) and, on a forked branch joined at its end, those two copies (from and
+    to fixed pinned host buffers); the first step's upload and the last step's read-back
+    are issued around the graphs.  Every step's copies lie inside the timed region."""
     import torch
 
     from paper_2609_03515_gb300 import ikv, step_lengths
@@ -746,7 +746,7 @@ def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist, mh: int
             in_ready[i].record(up)
 
     def run(t0, n):
-        """Steps t0 .. t0+n-1; the upload of t0 is issued here, the last read-back is waited for."""
+        """Eager steps t0 .. t0+n-1; the upload of t0 is issued here, the last read-back is waited for."""
         nonlocal lens, live
         up.wait_stream(comp)
         down.wait_stream(comp)
@@ -760,11 +760,8 @@ def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist, mh: int
             comp.wait_event(in_ready[i])
             if t >= t0 + 2:
                 comp.wait_event(read[i])             # step t-2's output has been read back
-            if graphs:
-                graphs[(refresh(t), i)].replay()
-            else:
-                ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, q_d[i], kn_d[i], vn_d[i], out_d[i], ws,
-                             ws.numel(), comp)
+            ikv.ikv_step(c.shape(), p, c.cache(max(lens)), c.ema, t, q_d[i], kn_d[i], vn_d[i], out_d[i], ws,
+                         ws.numel(), comp)
             done[i].record(comp)
             with torch.cuda.stream(down):
                 down.wait_event(done[i])
@@ -774,31 +771,42 @@ def run_e2e(args, w, c, u_dev, ws, compact_mode, qs_h, kn_h, vn_h, dist, mh: int
         comp.wait_stream(up)
         comp.wait_stream(down)
 
-    def refresh(t):
-        return t == 1 if w.score_free else (t - 1) % w.refresh_period == 0
-
-    graphs = {}
     W, K = args.warmup, args.steps
     run(1, W)
     torch.cuda.synchronize()
     steady = c.cache(min(c.cap - 1, max(max(lens), max(budgets) + mh)))
     p.ws_zeroed = 1  # the warm-up left the workspace's counters zero
-    for t in range(W + 1, W + 1 + K):
-        key = (refresh(t), t % 2)
-        if key in graphs:
-            continue
+    T0 = W + 1
+    side = torch.cuda.Stream(device=dev)
+    step_graphs = []
+    for t in range(T0, T0 + K):
+        i = t % 2
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, capture_error_mode="thread_local"):
-            i = t % 2
-            ikv.ikv_step(c.shape(), p, steady, c.ema, t, q_d[i], kn_d[i], vn_d[i], out_d[i], ws, ws.numel(),
-                         torch.cuda.current_stream())
-        graphs[key] = g
+            cs = torch.cuda.current_stream()
+            side.wait_stream(cs)
+            with torch.cuda.stream(side):
+                if t + 1 < T0 + K:  # step t+1's inputs into the other buffer set
+                    q_d[1 - i].copy_(qs_h[t], non_blocking=True)
+                    kn_d[1 - i].copy_(kn_h[t], non_blocking=True)
+                    vn_d[1 - i].copy_(vn_h[t], non_blocking=True)
+                if t > T0:  # step t-1's output
+                    out_h[1 - i].copy_(out_d[1 - i], non_blocking=True)
+            ikv.ikv_step(c.shape(), p, steady, c.ema, t, q_d[i], kn_d[i], vn_d[i], out_d[i], ws, ws.numel(), cs)
+            cs.wait_stream(side)
+        step_graphs.append(g)
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     start.record(comp)
-    run(W + 1, K)
+    i0, il = T0 % 2, (T0 + K - 1) % 2
+    q_d[i0].copy_(qs_h[T0 - 1], non_blocking=True)
+    kn_d[i0].copy_(kn_h[T0 - 1], non_blocking=True)
+    vn_d[i0].copy_(vn_h[T0 - 1], non_blocking=True)
+    for g in step_graphs:
+        g.replay()
+    out_h[il].copy_(out_d[il], non_blocking=True)
     stop.record(comp)
     torch.cuda.synchronize()
     ms = max_over_ranks(start.elapsed_time(stop), dist, dev)
@@ -1009,7 +1017,8 @@ def run_ours(args):
         "e2e": {"value": w.batch * K * world / (e2e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "runs": [w.batch * K * world / (m / 1e3) for m in e2e_all],
                 "note": "median of five runs; inputs uploaded from pinned host memory and outputs read back "
-                        "every step, overlapped with the previous / next step's compute"},
+                        "every step: each step's CUDA graph holds ikv_step and, on a forked branch, the upload of "
+                        "the next step's inputs and the read-back of the previous step's output"},
         "gpu_launches": full["launches"],
         "clocks": full["clocks"],
         "modes": {k: sig(w.batch * K * world / (v["ms"] / 1e3)) for k, v in modes.items()},
