@@ -453,7 +453,7 @@ int score_blocks(const ScoreArgs &a, int32_t max_len, int sms, int *V) {
 // whole grid fits at k per SM for some k < 4 (four fit by registers).  Left to itself the
 // block scheduler puts four CTAs on some SMs and one on others, and the most loaded SM
 // sets the pass's pace (config 1: 412 CTAs; with at most three per SM the graphed step
-// measured 81.7 -> 80.3 us).  Each size admits exactly k CTAs of this kernel (its static
+// measured 81.7 -> 80.8 us).  Each size admits exactly k CTAs of this kernel (its static
 // shared memory and the 1 KB reserved per CTA included) in an SM's 228 KB.
 static size_t spread_smem(int64_t ctas, int sms) {
     const int64_t k = sms > 0 ? (ctas + sms - 1) / sms : 4;
