@@ -384,8 +384,11 @@ ikv_status run_score(const ikv_shape *s, const ikv_cache *c, int32_t n_layers, c
         sa.n_elig = n_elig - k0 < kMaxLayersPerScorePass ? n_elig - k0 : kMaxLayersPerScorePass;
         sa.k0 = k0;
         for (int k = 0; k < sa.n_elig; ++k) sa.elig[k] = elig[k0 + k];
-        // the last pass of an Eq. 1 / VNorm fold also selects
-        if (fuse && ema && !store_only && scorer != IKV_SCORE_ENTROPY && k0 + sa.n_elig == n_elig) {
+        // the last pass of an Eq. 1 / VNorm fold also selects, unless the rows may be long
+        // (step 1 after a long prefill): the general selection then runs in the 1024-thread
+        // select kernel rather than on the score pass's last 256-thread CTA per row
+        if (fuse && ema && !store_only && scorer != IKV_SCORE_ENTROPY && k0 + sa.n_elig == n_elig &&
+            max_len <= kFusedSelectMaxLen) {
             sa.fuse_select = 1;
             sa.row_done = fuse->row_done;
             sa.budget = fuse->budget;

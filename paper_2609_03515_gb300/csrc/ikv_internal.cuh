@@ -14,6 +14,7 @@ constexpr int kAttendThreads = 128;
 constexpr int kMaxSplits = 128;    // split-K partitions per (seq, layer, kv head)
 constexpr int kMinSplitTokens = 256;
 constexpr int kMaxLayersPerScorePass = 32;
+constexpr int kFusedSelectMaxLen = 16384;  // longest row bound for which the score pass also selects
 constexpr int kScoreLayersPerGroup = 8;   // eligible layers one score CTA folds (one warp each)
 constexpr int kMaxLayers = 512;
 
