@@ -588,7 +588,7 @@ static ikv_status compact_impl(const ikv_shape *shape, ikv_cache *cache, const i
         a.rows_per_seq = shape->layers;
         a.row_by_layer = 1;
     }
-    IKV_TRY_CUDA(launch_compact(a, mode, stream), "compact launch");
+    IKV_TRY_CUDA(launch_compact(a, mode, sm_count(), stream), "compact launch");
     return IKV_OK;
 }
 

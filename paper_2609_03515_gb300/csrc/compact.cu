@@ -109,15 +109,13 @@ __device__ __forceinline__ void mark_dead_row(const CompactArgs &a, int r, int L
     }
 }
 
-// Stable compaction of one sequence's rows (see the file comment).  Every CTA of
-// sequence b reads len[b] and start[b] first; the last CTA of b to arrive writes
-// the new values, so no CTA sees them early.
-__global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const CompactArgs a) {
-    pdl_wait();
-    extern __shared__ __align__(16) unsigned char cbuf[];
-    __shared__ int scratch[32];
+// Stable compaction of one item of sequence b (see the file comment): item x < nkv moves
+// the K/V rows of (layer, KV head) x, item nkv + rr gathers utility / position row rr.
+// Every item of b reads len[b] and start[b] first; the last of b's items to arrive
+// writes the new values, so no item sees them early.  Entered by every thread of the CTA.
+__device__ __forceinline__ void compact_stable_item(const CompactArgs &a, const int x, const int b,
+                                                    unsigned char *cbuf, int *scratch) {
     const int tid = threadIdx.x;
-    const int b = blockIdx.y, x = blockIdx.x;
     const int kvh = a.pv.kv_heads;
     const int nkv = a.layers * kvh;
     if (a.keep_len[b * a.rows_per_seq] < 0) return;  // selection marked the victim dead: nothing to do
@@ -253,14 +251,54 @@ __global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const Comp
             __syncthreads();
         }
     }
-    // publish len / start once every CTA of b has read them
+    // publish len / start once every item of b has read them
     __syncthreads();
     if (tid == 0) {
-        if (arrive_acq_rel(&a.done[b]) == (int)gridDim.x - 1) {
+        if (arrive_acq_rel(&a.done[b]) == nkv + a.rows_per_seq - 1) {
             a.len[b] = n0;
             if (a.start) a.start[b] = new_start;
             a.done[b] = 0;
         }
+    }
+}
+
+// The stable compaction, one CTA per item: grid (items per sequence, sequences).
+__global__ void __launch_bounds__(kCompThreads) compact_stable_kernel(const CompactArgs a) {
+    pdl_wait();
+    extern __shared__ __align__(16) unsigned char cbuf[];
+    __shared__ int scratch[32];
+    compact_stable_item(a, blockIdx.x, blockIdx.y, cbuf, scratch);
+}
+
+// The same over a fixed grid of one wave of CTAs, for launches with more items than fit
+// at once: CTA i takes items i, i + gridDim.x, ... of the (sequence, item) list.  Items of
+// a sequence whose row the selection flagged (keep_len < 0: the victim is marked dead,
+// nothing moves) are skipped; their flags are read for 32 of the CTA's items at once, so a
+// step in which nothing moves costs one round of loads per CTA.  (One CTA per item: 16
+// sequences x 257 items of 64 KB shared memory took ~9 launch waves just to exit.)
+__global__ void __launch_bounds__(kCompThreads) compact_stable_strided_kernel(const CompactArgs a) {
+    pdl_wait();
+    extern __shared__ __align__(16) unsigned char cbuf[];
+    __shared__ int scratch[32];
+    __shared__ int flagged[32];
+    const int nx = a.layers * a.pv.kv_heads + a.rows_per_seq;
+    const int n_items = nx * a.batch;
+#pragma unroll 1
+    for (int k0 = 0; blockIdx.x + (int64_t)k0 * gridDim.x < n_items; k0 += 32) {
+        if (threadIdx.x < 32) {
+            const int64_t item = blockIdx.x + (int64_t)(k0 + threadIdx.x) * gridDim.x;
+            flagged[threadIdx.x] = item < n_items ? a.keep_len[(int)(item / nx) * a.rows_per_seq] < 0 : 1;
+        }
+        __syncthreads();
+#pragma unroll 1
+        for (int k = 0; k < 32; ++k) {
+            const int64_t item = blockIdx.x + (int64_t)(k0 + k) * gridDim.x;
+            if (item >= n_items) break;
+            if (flagged[k]) continue;
+            compact_stable_item(a, (int)(item % nx), (int)(item / nx), cbuf, scratch);
+            __syncthreads();  // the next item reuses the shared buffers
+        }
+        __syncthreads();  // flagged is rewritten
     }
 }
 
@@ -514,18 +552,31 @@ __global__ void __launch_bounds__(kCompThreads) append_rows_kernel(const AppendA
 
 }  // namespace
 
-cudaError_t launch_compact(const CompactArgs &a, int mode, cudaStream_t st) {
+cudaError_t launch_compact(const CompactArgs &a, int mode, int sms, cudaStream_t st) {
     dim3 grid(a.layers * a.pv.kv_heads + a.rows_per_seq, a.batch);
     if (mode == IKV_COMPACT_STABLE || mode == IKV_COMPACT_STABLE_SHORT) {
         const int smem = kCompStages * 2 * kCompRows * a.pv.head_dim * a.elem_bytes;
-        static int attr_smem = 0;  // raise the dynamic shared-memory limit once per size
-        if (smem > attr_smem) {
+        static int attr_smem = 0;  // raise the dynamic shared-memory limits once per size
+        static int per_sm = 0;     // resident CTAs per SM of the strided kernel at attr_smem
+        if (smem > attr_smem || per_sm == 0) {
             cudaError_t e =
                 cudaFuncSetAttribute(compact_stable_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+            if (e == cudaSuccess)
+                e = cudaFuncSetAttribute(compact_stable_strided_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         smem);
+            if (e == cudaSuccess)
+                e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, compact_stable_strided_kernel,
+                                                                  kCompThreads, smem);
             if (e != cudaSuccess) return e;
+            if (per_sm < 1) per_sm = 1;
             attr_smem = smem;
         }
-        cudaError_t e = launch_k(compact_stable_kernel, grid, dim3(kCompThreads), smem, st, a);
+        const int64_t items = (int64_t)grid.x * grid.y;
+        const int64_t wave = (int64_t)per_sm * (sms > 0 ? sms : 1);
+        cudaError_t e = items <= wave
+                            ? launch_k(compact_stable_kernel, grid, dim3(kCompThreads), smem, st, a)
+                            : launch_k(compact_stable_strided_kernel, dim3((unsigned)wave), dim3(kCompThreads), smem,
+                                       st, a);
         note_launch();
         return e != cudaSuccess ? e : cudaGetLastError();
     }

@@ -223,7 +223,7 @@ struct CompactArgs {
     int32_t row_by_layer;       // per-layer eviction: keep row b * rows_per_seq + l governs layer l
                                 // (all kv heads) and pos row b * rows_per_seq + l
 };
-cudaError_t launch_compact(const CompactArgs &a, int mode, cudaStream_t st);
+cudaError_t launch_compact(const CompactArgs &a, int mode, int sms, cudaStream_t st);
 
 struct AppendArgs {
     void *k, *v;
