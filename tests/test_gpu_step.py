@@ -289,15 +289,21 @@ def test_workspace_kept_zero_across_steps():
     dict(compact_mode=ikv.IKV_COMPACT_HOLEFILL, scorer=ikv.IKV_SCORE_VNORM),
     dict(compact_mode=ikv.IKV_COMPACT_STABLE, gran=ikv.IKV_GRAN_KVHEAD),
     dict(compact_mode=ikv.IKV_COMPACT_STABLE_SHORT, max_holes=3, per_layer=True),
-], ids=["short_deferred", "short_tight_cap", "holefill_vnorm", "stable_kvhead", "split_step"])
+    dict(compact_mode=ikv.IKV_COMPACT_STABLE_SHORT, max_holes=2, strided=True),
+], ids=["short_deferred", "short_tight_cap", "holefill_vnorm", "stable_kvhead", "split_step", "short_strided"])
 def test_nothing_written_outside_the_buffers(case):
     """Canaries around every buffer (spare pool pages among the used ones, tails after pos,
     ema, vnorm and the workspace) stay intact through lock-step runs that exercise the
     shorter-side moves (right moves, relocation to slot 0), an append into the last slot of
-    the slot space, hole-fill with value norms, KV-head rows and the split step."""
+    the slot space, hole-fill with value norms, KV-head rows, the split step, and the
+    compaction's grid-stride form (16 sequences x 33 items: more than one wave of its CTAs)."""
     case = dict(case)
     tight = case.pop("tight", False)
-    if tight:
+    strided = case.pop("strided", False)
+    if strided:
+        w = small_llama(batch=16, layers=4, steps=6,
+                        prefill=[150 + 29 * i for i in range(16)])
+    elif tight:
         # cap = 320 slots: sequence 0's first append lands in slot 319, and the shorter-side
         # compaction runs out of room on the right
         w = small_llama(prefill=[319, 200], batch=2, steps=8, budget_frac=0.5)
