@@ -231,10 +231,15 @@ __global__ void __launch_bounds__(kScoreThreads, 4) score_kernel(const ScoreArgs
         if (threadIdx.x < kTok) cpart[threadIdx.x] = c;
         cluster_sync();  // every group's c is in its shared memory
         if (lg == 0 && folds) {
-            for (int q = 0; q < n_lg; ++q) {
-                const float cq = q == 0 ? c : ld_cluster_f32(&cpart[threadIdx.x], q);
-                m = agg_factor(min(kScoreWarps, a.n_elig - q * kScoreWarps), a.agg, a.alpha) * m + cq;
-            }
+            // every group's c is loaded before any is used, so the remote loads overlap
+            constexpr int kMaxGroups = (kMaxLayersPerScorePass + kScoreWarps - 1) / kScoreWarps;
+            float cq[kMaxGroups];
+#pragma unroll
+            for (int q = 1; q < kMaxGroups; ++q) cq[q] = q < n_lg ? ld_cluster_f32(&cpart[threadIdx.x], q) : 0.f;
+            cq[0] = c;
+#pragma unroll
+            for (int q = 0; q < kMaxGroups; ++q)
+                if (q < n_lg) m = agg_factor(min(kScoreWarps, a.n_elig - q * kScoreWarps), a.agg, a.alpha) * m + cq[q];
         }
         cluster_sync();  // the first CTA has read them: the others may exit
         if (lg != 0) return;
